@@ -1,0 +1,432 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: a
+hand-worked fixture in tests/golden/, a closed form, brute force on tiny
+inputs, or an identity of App. A. A plausible slip in the oracle (a dropped
+term, a wrong sign, a swapped index or operand, a wrong rounding mode) fails
+at least one of them.
+"""
+
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import sgat, tac
+from tests.conftest import GOLDEN
+
+F32 = np.float32
+U32 = 2.0 ** -24
+
+
+def golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+# ---------------------------------------------------------------------------
+# Basis and fast transform (Eq. 8, Hadamard reading)
+# ---------------------------------------------------------------------------
+
+def test_hadamard_golden_h4():
+    g = golden("hadamard_h4.json")
+    H = sgat.hadamard_sylvester(4)
+    assert H.tolist() == g["H4"]
+    x = np.array(g["x"], dtype=F32)
+    assert sgat.fwht_f32(x[None], 4)[0].tolist() == g["xH"]
+
+
+@pytest.mark.parametrize("n", [1, 2, 8, 64, 512])
+def test_hadamard_orthogonal_symmetric(n):
+    H = sgat.hadamard_sylvester(n)
+    assert np.array_equal(H, H.T)
+    assert np.array_equal(H @ H.T, n * np.eye(n, dtype=np.int64))
+    assert set(np.unique(H).tolist()) <= {-1, 1}
+
+
+def brute_hadamard_entry(i, j):
+    """Sylvester H_ij = (-1)^popcount(i & j), written independently."""
+    return -1 if bin(i & j).count("1") % 2 else 1
+
+
+@pytest.mark.parametrize("hb,K", [(2, 2), (8, 8), (16, 48), (256, 256), (512, 1536)])
+def test_fwht_equals_dense_on_integers(hb, K):
+    """On small integers every float32 butterfly is exact, so the fast
+    transform must equal x @ blockdiag(H_hb) exactly."""
+    rng = np.random.default_rng(hb + K)
+    x = rng.integers(-8, 9, (5, K)).astype(F32)
+    Hd = np.array([[brute_hadamard_entry(i, j) for j in range(hb)] for i in range(hb)], dtype=np.int64)
+    BD = np.kron(np.eye(K // hb, dtype=np.int64), Hd)
+    ref = x.astype(np.int64) @ BD
+    out = sgat.fwht_f32(x, hb)
+    assert np.array_equal(out.astype(np.int64), ref)
+
+
+@pytest.mark.parametrize("hb", [64, 4096])
+def test_fwht_float32_error_bound(hb):
+    """Random normal input: each output is a sum of hb terms through log2(hb)
+    float32 roundings, so |err| <= log2(hb) * u * sum|x| (u = 2^-24) plus
+    second-order terms."""
+    rng = np.random.default_rng(7)
+    x = rng.standard_normal((3, hb)).astype(F32)
+    ref = x.astype(np.float64) @ sgat.hadamard_sylvester(hb).astype(np.float64)
+    out = sgat.fwht_f32(x, hb).astype(np.float64)
+    bound = math.log2(hb) * U32 * np.abs(x).astype(np.float64).sum(axis=1, keepdims=True) * 1.01
+    assert np.all(np.abs(out - ref) <= bound)
+
+
+def test_fwht_involution():
+    rng = np.random.default_rng(3)
+    x = rng.integers(-100, 101, (4, 1024)).astype(F32)
+    y = sgat.fwht_f32(sgat.fwht_f32(x, 1024), 1024)
+    assert np.array_equal(y, 1024 * x)
+
+
+# ---------------------------------------------------------------------------
+# Gates (Eq. 9)
+# ---------------------------------------------------------------------------
+
+def test_gates_golden():
+    g = golden("gates_k8.json")
+    g_m, g_u = sgat.state_gates(g["K"], g["d_sh"], g["d_m"], g["d_u"])
+    assert g_m.tolist() == g["g_m"]
+    assert g_u.tolist() == g["g_u"]
+
+
+def test_gates_partition():
+    K, d_sh, d_m, d_u = 4096, 3840, 128, 128
+    g_m, g_u = sgat.state_gates(K, d_sh, d_m, d_u)
+    shared = g_m * g_u
+    assert shared.sum() == d_sh and g_m.sum() == d_sh + d_m and g_u.sum() == d_sh + d_u
+    assert np.all(g_m + g_u - shared == 1)   # the three subspaces cover d
+
+
+# ---------------------------------------------------------------------------
+# Quantiser (Eq. 2-3, symmetric reading)
+# ---------------------------------------------------------------------------
+
+def test_quant_golden():
+    for c in golden("quant_examples.json")["cases"]:
+        q, s = sgat.quantize_rows_sym(np.array([c["v"]], dtype=F32), c["bits"])
+        assert q[0].tolist() == c["q"], c["name"]
+        assert float(s[0]) == c["s"], c["name"]
+
+
+def brute_quant_row(v, bits):
+    """Independent restatement: pick q in [-qmax, qmax] nearest to the float32
+    product p = fl32(v * r), ties to the even integer; distances exact in
+    float64."""
+    qmax = (1 << (bits - 1)) - 1
+    amax = max(abs(float(t)) for t in v)
+    if amax == 0:
+        return [0] * len(v), 0.0
+    r = np.float32(np.float32(qmax) / np.float32(amax))
+    s = float(np.float32(np.float32(amax) / np.float32(qmax)))
+    out = []
+    for t in v:
+        p = float(np.float32(np.float32(t) * r))
+        best = None
+        for q in range(-qmax, qmax + 1):
+            dist = abs(p - q)
+            key = (dist, q % 2)          # ties -> even
+            if best is None or key < best[0]:
+                best = (key, q)
+        out.append(best[1])
+    return out, s
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+def test_quant_brute_force(bits):
+    rng = np.random.default_rng(bits)
+    for trial in range(300):
+        n = int(rng.integers(1, 9))
+        kind = trial % 3
+        if kind == 0:
+            v = rng.standard_normal(n)
+        elif kind == 1:      # constructed near-ties: multiples of half a step
+            v = rng.integers(-2 * ((1 << (bits - 1)) - 1), 2 * ((1 << (bits - 1)) - 1) + 1, n) * 0.5
+        else:
+            v = rng.standard_normal(n) * 10.0 ** rng.integers(-3, 4)
+        v = v.astype(F32)
+        q, s = sgat.quantize_rows_sym(v[None], bits)
+        qb, sb = brute_quant_row(v, bits)
+        assert q[0].tolist() == qb, (v, bits)
+        assert float(s[0]) == sb
+
+
+def test_quant_error_bound_and_extremes():
+    rng = np.random.default_rng(11)
+    v = (rng.standard_normal((64, 512)) * rng.lognormal(0, 2, (64, 1))).astype(F32)
+    q, s = sgat.quantize_rows_sym(v, 4)
+    assert np.all(np.abs(q) <= 7)
+    err = np.abs(v.astype(np.float64) - q * s[:, None].astype(np.float64))
+    assert np.all(err <= 0.5 * s[:, None] * (1 + 1e-5) + 1e-30)
+    # the element of largest magnitude lands on +-qmax
+    arg = np.argmax(np.abs(v), axis=1)
+    assert np.all(np.abs(q[np.arange(64), arg]) == 7)
+
+
+def test_pack_golden_and_roundtrip():
+    g = golden("int4_packing.json")
+    p = sgat.pack_int4(np.array([g["codes"]]))
+    assert p[0].tolist() == g["bytes"]
+    rng = np.random.default_rng(5)
+    q = rng.integers(-8, 8, (7, 64))
+    assert np.array_equal(sgat.unpack_int4(sgat.pack_int4(q)), q)
+
+
+# ---------------------------------------------------------------------------
+# Integer GEMM (Eq. 5 / Eq. 13)
+# ---------------------------------------------------------------------------
+
+def test_int_gemm_triple_loop():
+    rng = np.random.default_rng(2)
+    qa = rng.integers(-7, 8, (5, 96))
+    qw = rng.integers(-7, 8, (6, 96))
+    acc = sgat.int_gemm(qa, qw)
+    for i, n in itertools.product(range(5), range(6)):
+        s = 0
+        for k in range(96):
+            s += int(qa[i, k]) * int(qw[n, k])
+        assert acc[i, n] == s
+
+
+def test_int_gemm_extreme_accumulators():
+    K = 18944
+    qa = np.full((2, K), 7)
+    qw = np.stack([np.full(K, 7), np.full(K, -7)])
+    acc = sgat.int_gemm(qa, qw)
+    assert acc[0, 0] == 49 * K and acc[0, 1] == -49 * K
+
+
+# ---------------------------------------------------------------------------
+# Quantised linear and the SGAT identities (Eq. 5, 6, 25-28)
+# ---------------------------------------------------------------------------
+
+def _case(L=24, K=256, N=40, seed=0):
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((L, K)).astype(F32)
+    X[:, 5] *= 12
+    W = (rng.standard_normal((N, K)) * 0.05).astype(F32)
+    mask = (rng.random(L) < 0.5).astype(np.uint8)
+    return X, W, mask
+
+
+def test_identity_transform_16bit_reproduces_fp_matmul():
+    """P = I, all gates on, b = 16: Y_hat = Q_a(X) Q_w(W^T) must equal X W^T up
+    to the quantisation error bound |x - x_hat| <= s_a/2, |w - w_hat| <= s_w/2
+    (Eq. 5)."""
+    X, W, mask = _case()
+    K = X.shape[1]
+    qw, s_w = sgat.prepare_weight(W, None, 1, 16)
+    Y, codes, s_a, acc = sgat.sgat_linear(X, mask, None, None, 1, K, 0, 0, qw, s_w, bits=16)
+    ref = X.astype(np.float64) @ W.astype(np.float64).T
+    ea = 0.5 * s_a.astype(np.float64)[:, None]
+    ew = 0.5 * s_w.astype(np.float64)[None, :]
+    bound = (ea * np.abs(W).astype(np.float64).sum(1)[None, :]
+             + ew * np.abs(X).astype(np.float64).sum(1)[:, None] + K * ea * ew)
+    assert np.all(np.abs(Y - ref) <= bound * 1.0001 + 1e-12)
+    assert np.linalg.norm(Y - ref) / np.linalg.norm(ref) < 2e-4
+
+
+def test_transform_cancellation_full_precision():
+    """Eq. 6 / Eq. 27 with G = I and a shared diagonal: (X P)(P^-1 W^T) = X W^T
+    to float32 round-off, for both states."""
+    X, W, mask = _case(K=512)
+    K = X.shape[1]
+    rng = np.random.default_rng(9)
+    a = np.exp(rng.normal(0, 0.5, K)).astype(F32)
+    V = sgat.sgat_transform(X, mask, a, a, 512, K, 0, 0).astype(np.float64)
+    Wt = sgat.transform_weight_f32(W, (1.0 / a.astype(np.float64)).astype(F32), 512).astype(np.float64)
+    Y = V @ Wt.T
+    ref = X.astype(np.float64) @ W.astype(np.float64).T
+    scale = np.abs(X).astype(np.float64) @ np.abs(W).astype(np.float64).T
+    assert np.all(np.abs(Y - ref) <= 64 * 12 * U32 * scale + 1e-12)
+
+
+def test_inactive_zero_condition_and_leakage():
+    """App. A: if X^s P G_s^perp = 0 (Eq. 25) the gated transform reproduces
+    X^s W^T; in general the difference equals Delta_s = X^s P G_s^perp P^T W^T
+    (Eq. 28)."""
+    L, K, N, hb = 16, 256, 24, 256
+    rng = np.random.default_rng(4)
+    d_m = d_u = K // 32
+    d_sh = K - d_m - d_u
+    g_m, g_u = sgat.state_gates(K, d_sh, d_m, d_u)
+    a = np.exp(rng.normal(0, 0.3, K)).astype(F32)
+    inv_a = (1.0 / a.astype(np.float64)).astype(F32)
+    W = (rng.standard_normal((N, K)) * 0.05).astype(F32)
+    H = sgat.hadamard_sylvester(hb).astype(np.float64)
+    Wt = sgat.transform_weight_f32(W, inv_a, hb).astype(np.float64)
+    for state, g in ((1, g_m), (0, g_u)):
+        mask = np.full(L, state, np.uint8)
+        # X^s built inside the active subspace: (X^s * a) H = U * g_s
+        U = rng.standard_normal((L, K))
+        Xs = (((U * g[None, :]) @ H / hb) / a.astype(np.float64)[None, :]).astype(F32)
+        V = sgat.sgat_transform(Xs, mask, a, a, hb, d_sh, d_m, d_u).astype(np.float64)
+        ref = Xs.astype(np.float64) @ W.astype(np.float64).T
+        scale = np.abs(Xs).astype(np.float64) @ np.abs(W).astype(np.float64).T
+        assert np.all(np.abs(V @ Wt.T - ref) <= 1e-5 * scale.max())
+        # general X^s: the deviation is the leakage term of Eq. 28
+        Xg = rng.standard_normal((L, K)).astype(F32)
+        Vg = sgat.sgat_transform(Xg, mask, a, a, hb, d_sh, d_m, d_u).astype(np.float64)
+        XP = (Xg.astype(np.float64) * a.astype(np.float64)) @ H
+        delta = (XP * (1 - g[None, :])) @ (H / hb) @ (W.astype(np.float64) * inv_a.astype(np.float64)).T
+        dev = Xg.astype(np.float64) @ W.astype(np.float64).T - Vg @ Wt.T
+        scale = np.abs(Xg).astype(np.float64) @ np.abs(W).astype(np.float64).T
+        assert np.all(np.abs(dev - delta) <= 1e-5 * scale.max())
+        assert np.abs(delta).max() > 1e-3 * scale.max()   # the leakage is really there
+
+
+def test_state_split_scatter():
+    """Eq. 7 and the scatter after Eq. 13: each token is transformed with its
+    own state's gate and smoothing, independent of the other tokens, and
+    returns to its own position."""
+    X, W, mask = _case(L=33, K=128, N=16, seed=3)
+    K = X.shape[1]
+    rng = np.random.default_rng(1)
+    a_m = np.exp(rng.normal(0, 0.5, K)).astype(F32)
+    a_u = np.exp(rng.normal(0, 0.5, K)).astype(F32)
+    args = (a_m, a_u, 128, K - 8, 4, 4)
+    codes, s_a = sgat.sgat_quantize_act(X, mask, *args, 4)
+    # all-masked and all-unmasked runs give the per-state rows
+    cm, sm = sgat.sgat_quantize_act(X, np.ones_like(mask), *args, 4)
+    cu, su = sgat.sgat_quantize_act(X, np.zeros_like(mask), *args, 4)
+    sel = mask[:, None] == 1
+    assert np.array_equal(codes, np.where(sel, cm, cu))
+    assert np.array_equal(s_a, np.where(mask == 1, sm, su))
+    assert not np.array_equal(cm, cu)
+    # permuting tokens permutes the result
+    perm = rng.permutation(len(mask))
+    cp, sp = sgat.sgat_quantize_act(X[perm], mask[perm], *args, 4)
+    assert np.array_equal(cp, codes[perm]) and np.array_equal(sp, s_a[perm])
+
+
+def test_weight_fold_scale_invariance():
+    """Folding the exact 1/hb into the weight (Eq. 12) scales s_w by 1/hb and
+    leaves every code unchanged."""
+    _, W, _ = _case(N=32, K=512)
+    q1, s1 = sgat.prepare_weight(W, None, 512, 4)
+    q2, s2 = sgat.quantize_rows_sym(sgat.fwht_f32(W, 512), 4)
+    assert np.array_equal(q1, q2)
+    assert np.array_equal(s1, (s2 / F32(512)).astype(F32))
+
+
+# ---------------------------------------------------------------------------
+# TAC (Eq. 17, App. C)
+# ---------------------------------------------------------------------------
+
+def test_tac_golden():
+    g = golden("tac_example.json")
+    out = tac.tac_apply(np.array(g["z"]), np.array(g["M"]), np.array(g["d"]), g["g"])
+    assert np.allclose(out, np.array(g["out"]), rtol=0, atol=1e-12)
+
+
+def test_tac_identity_and_column_form():
+    rng = np.random.default_rng(8)
+    N, C, g = 5, 48, 16
+    Z = rng.standard_normal((N, C))
+    B = C // g
+    eye = np.broadcast_to(np.eye(g), (B, g, g))
+    assert np.array_equal(tac.tac_apply(Z, eye, np.zeros((B, g)), g), Z)
+    M = rng.standard_normal((B, g, g))
+    d = rng.standard_normal((B, g))
+    out = tac.tac_apply(Z, M, d, g)
+    # column-vector form z_b <- M_b z_b + d_b, written as explicit loops
+    for i in range(N):
+        for b in range(B):
+            for r in range(g):
+                s = d[b, r]
+                for j in range(g):
+                    s += M[b, r, j] * Z[i, b * g + j]
+                assert abs(out[i, b * g + r] - s) <= 1e-12 * (1 + abs(s))
+
+
+def test_tac_hyperparameters_and_block_rule():
+    g = golden("hyperparameters.json")
+    for k, v in g["tac"].items():
+        assert tac.TAC_DEFAULTS[k] == v
+    for C, expect in g["block_size_rule"]:
+        assert tac.default_block_size(C) == expect
+
+
+def test_tac_scalar_calibration_golden():
+    g = golden("tac_scalar_calibration.json")
+    M, d = tac.tac_calibrate(np.array(g["Z_fp"])[:, None], np.array(g["Z_q"])[:, None], 1,
+                             rho=g["rho"], eps=g["eps"], eta=g["eta"], alpha=g["alpha"])
+    assert abs(M[0, 0, 0] - g["M_final"]) < 1e-12
+    assert abs(d[0, 0] - g["d"]) < 1e-12
+
+
+def test_tac_calibration_invariants():
+    rng = np.random.default_rng(12)
+    N, C, g = 4096, 32, 16
+    A = rng.standard_normal((C, C)) * 0.3 + np.eye(C)
+    Z_fp = rng.standard_normal((N, C)) @ A.T + rng.normal(0, 1, C)
+    Z_q = Z_fp * 0.9 + rng.standard_normal((N, C)) * 0.2 + 0.05
+    # compensated mean equals the full-precision mean (bias estimation, App. C)
+    M, d = tac.tac_calibrate(Z_fp, Z_q, g)
+    out = tac.tac_apply(Z_q, M, d, g)
+    assert np.allclose(out.mean(0), Z_fp.mean(0), atol=1e-10)
+    # alpha = 1: the matrix degenerates to identity, only the mean is corrected
+    M1, d1 = tac.tac_calibrate(Z_fp, Z_q, g, alpha=1.0)
+    assert np.allclose(M1, np.eye(g)[None], atol=1e-12)
+    assert np.allclose(d1.reshape(-1), Z_fp.mean(0) - Z_q.mean(0), atol=1e-12)
+    # rho = eta = alpha = 0: covariance matching, M Sigma_Q M^T = Sigma_FP (Eq. 18)
+    M0, _ = tac.tac_calibrate(Z_fp, Z_q, g, rho=0.0, eta=0.0, alpha=0.0)
+    _, S_fp = tac.block_stats(Z_fp, g)
+    _, S_q = tac.block_stats(Z_q, g)
+    for b in range(C // g):
+        assert np.allclose(M0[b] @ S_q[b] @ M0[b].T, S_fp[b], rtol=1e-8, atol=1e-9)
+    # eta = 1: all singular values equal their mean before shrinkage
+    Me, _ = tac.tac_calibrate(Z_fp, Z_q, g, eta=1.0, alpha=0.0)
+    sv = np.linalg.svd(Me[0], compute_uv=False)
+    assert np.allclose(sv, sv.mean(), rtol=1e-10)
+
+
+def test_sym_power_closed_form():
+    A = np.diag([4.0, 9.0, 0.0])
+    R = np.array([[0.6, -0.8, 0], [0.8, 0.6, 0], [0, 0, 1.0]])
+    B = R @ A @ R.T
+    assert np.allclose(tac.sym_power(B, 0.5), R @ np.diag([2.0, 3.0, 1e-6]) @ R.T, atol=1e-12)
+    assert np.allclose(tac.sym_power(B, -0.5), R @ np.diag([0.5, 1 / 3.0, 1e6]) @ R.T, rtol=1e-9)
+
+
+def test_phi_state_dense_reference():
+    """Phi_s(x) = ((x * a_s) H) G_s (Eq. 11) against a dense float64 product,
+    with distinct smoothing per state and both states present."""
+    L, K, hb = 20, 256, 128
+    rng = np.random.default_rng(21)
+    X = rng.standard_normal((L, K)).astype(F32)
+    mask = (np.arange(L) % 3 == 0).astype(np.uint8)
+    a_m = np.exp(rng.normal(0, 0.5, K)).astype(F32)
+    a_u = np.exp(rng.normal(0, 0.5, K)).astype(F32)
+    d_m = d_u = 8
+    d_sh = K - 16
+    g_m, g_u = sgat.state_gates(K, d_sh, d_m, d_u)
+    BD = np.kron(np.eye(K // hb), sgat.hadamard_sylvester(hb).astype(np.float64))
+    V = sgat.sgat_transform(X, mask, a_m, a_u, hb, d_sh, d_m, d_u).astype(np.float64)
+    for i in range(L):
+        a, g = (a_m, g_m) if mask[i] else (a_u, g_u)
+        ref = ((X[i].astype(np.float64) * a.astype(np.float64)) @ BD) * g
+        bound = 10 * U32 * (np.abs(X[i].astype(np.float64) * a) @ np.abs(BD)) + 1e-30
+        assert np.all(np.abs(V[i] - ref) <= bound), i
+
+
+def test_tac_singular_value_smoothing_formula():
+    """App. C: M_sv keeps the singular vectors of M and maps every singular
+    value to (1 - eta) sigma + eta mean(sigma)."""
+    rng = np.random.default_rng(13)
+    N, C, g = 2048, 16, 16
+    A = rng.standard_normal((C, C)) * 0.5 + np.eye(C)
+    Z_fp = rng.standard_normal((N, C)) @ A.T
+    Z_q = Z_fp + rng.standard_normal((N, C)) * 0.3
+    M0, _ = tac.tac_calibrate(Z_fp, Z_q, g, eta=0.0, alpha=0.0)
+    for eta in (0.15, 1.0):
+        Me, _ = tac.tac_calibrate(Z_fp, Z_q, g, eta=eta, alpha=0.0)
+        s0 = np.linalg.svd(M0[0], compute_uv=False)
+        se = np.linalg.svd(Me[0], compute_uv=False)
+        assert np.allclose(se, (1 - eta) * s0 + eta * s0.mean(), rtol=1e-10)
