@@ -1,0 +1,431 @@
+#!/usr/bin/env python
+"""Benchmark of the SGAT W4A4 hot path on GB300.
+
+Workload (one step): the LLaDA-8B attention projections at one denoising
+step -- 1024 tokens (prompt 512 unmasked, 512 generated with a 75% masked
+suffix), hidden 4096, fused QKV 4096 -> 12288 and O 4096 -> 4096, TAC with
+128 x 128 per-head blocks on the attention output, FP16 activations with
+0.5% Student-t(3) channels, random N(0, 0.02) weights prepared once
+(untimed) into folded int4 codes. A step is five kernels: quantise X, QKV
+GEMM, TAC on Z, quantise, O GEMM.
+
+Prints one JSON line (rank 0). Value = SGAT W4A4 linear throughput in TOPS
+(2 L N K integer ops of both GEMMs per step / step time), summed over ranks
+(weak scaling: every rank runs its own token batch, no collective on the
+data path). `--impl reference` times the CPU oracle on the same workload.
+"""
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "SGAT W4A4 linear TOPS & % INT8 tensor peak; denoise-step tokens/s at 8B shape"
+UNIT = "TOPS"
+L2_FLUSH_BYTES = 256 << 20
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FP8_PER_BF16 = 2.0   # nominal dense fp8 / bf16 tensor ratio (4.5 / 2.25 PFLOP/s)
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--no-graph", action="store_true")
+    p.add_argument("--cpu-sample-tokens", type=int, default=1024)
+    p.add_argument("--ref-sample-tokens", type=int, default=128)
+    p.add_argument("--skip-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def config_dict(graph):
+    return {"workload": "llada8b_attention_projections_step", "tokens": 1024, "hidden": 4096,
+            "qkv": "4096->12288", "o": "4096->4096", "tac_block": 128, "hadamard_block": 4096,
+            "gates": "d_m = d_u = 128", "mask": "0..639 unmasked, 640..1023 masked",
+            "l2": "flushed between timed steps (256 MiB write)", "cuda_graph": bool(graph)}
+
+
+# ---------------------------------------------------------------------------
+# Clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def kernel_source_hash():
+    p = os.path.join(ROOT, "paper_2606_04945_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in ("w4a4_gemm.cu", "common.cuh"):
+        with open(os.path.join(p, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic():
+    """DRAM bytes per launch of the GEMM from the committed ncu summary, if it
+    was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "w4a4_gemm_llada_qkv_traffic.txt")
+    try:
+        kv = {}
+        with open(path) as f:
+            for line in f:
+                if ":" in line:
+                    k, v = line.split(":", 1)
+                    kv[k.strip()] = v.strip()
+        if kv.get("kernel_source_sha256_16") != kernel_source_hash():
+            return None
+        return float(kv["dram_bytes_per_launch_avg"])
+    except Exception:
+        return None
+
+
+def time_kernel(fn, flush, reps, torch):
+    s = torch.cuda.current_stream()
+    ts = []
+    for _ in range(reps):
+        flush()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        fn()
+        e1.record(s)
+        e1.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    return statistics.mean(ts)
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi, inputs
+    from paper_2606_04945_gb300.pipeline import AttentionProjections
+
+    qkv_case, o_case = inputs.llada_attention(seed=rank)
+    step = AttentionProjections(qkv_case, o_case)
+    L, K = step.L, step.qkv.K
+    flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    flush = lambda: flush_buf.zero_()
+
+    # warm-up, then capture the step in a CUDA graph
+    for _ in range(max(args.warmup, 3)):
+        step.step()
+    abi.check_status()
+    graph = not args.no_graph
+    if graph:
+        step.capture()
+        run = step.replay
+    else:
+        run = step.step
+    for _ in range(max(args.warmup, 3)):
+        run()
+    abi.check_status()
+
+    # per-kernel durations (each kernel alone, L2 flushed before every launch)
+    Xq = torch.empty(L, K // 2, dtype=torch.uint8, device="cuda")
+    s_a = torch.empty(L, dtype=torch.float32, device="cuda")
+    zt = torch.empty(L, K, dtype=torch.float32, device="cuda")
+    q, o = step.qkv, step.o
+    reps = 20
+    t_quant_x = time_kernel(lambda: abi.sgat_quantize_act(step.X, step.mask, q.a_m, q.a_u, q.hb, q.d_sh, q.d_m,
+                                                          q.d_u, Xq, s_a), flush, reps, torch)
+    t_gemm_qkv = time_kernel(lambda: abi.w4a4_gemm(Xq, s_a, q.Wq, q.s_w, step.Y_qkv), flush, reps, torch)
+    t_tac = time_kernel(lambda: abi.tac_apply(step.Z, o.tac_M, o.tac_d, o.tac_g, zt), flush, reps, torch)
+    t_quant_z = time_kernel(lambda: abi.sgat_quantize_act(zt, step.mask, o.a_m, o.a_u, o.hb, o.d_sh, o.d_m,
+                                                          o.d_u, Xq, s_a), flush, reps, torch)
+    t_gemm_o = time_kernel(lambda: abi.w4a4_gemm(Xq, s_a, o.Wq, o.s_w, step.Y_o), flush, reps, torch)
+    abi.check_status()
+
+    # timed region: exactly `steps` steps, device-timed per step
+    clocks = ClockSampler(local)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    s = torch.cuda.current_stream()
+    evs = []
+    for _ in range(args.steps):
+        flush()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        run()
+        e1.record(s)
+        evs.append((e0, e1))
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    abi.check_status()
+    ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+
+    # end to end through the public API: pinned host inputs in, outputs out
+    X_h = step.X.cpu().pin_memory()
+    Z_h = step.Z.cpu().pin_memory()
+    m_h = step.mask.cpu().pin_memory()
+    Yq_h = torch.empty(step.Y_qkv.shape, dtype=step.Y_qkv.dtype).pin_memory()
+    Yo_h = torch.empty(step.Y_o.shape, dtype=step.Y_o.dtype).pin_memory()
+    h2d = X_h.numel() * X_h.element_size() + Z_h.numel() * Z_h.element_size() + m_h.numel()
+    d2h = Yq_h.numel() * Yq_h.element_size() + Yo_h.numel() * Yo_h.element_size()
+
+    def e2e_step():
+        step.X.copy_(X_h, non_blocking=True)
+        step.Z.copy_(Z_h, non_blocking=True)
+        step.mask.copy_(m_h, non_blocking=True)
+        run()
+        Yq_h.copy_(step.Y_qkv, non_blocking=True)
+        Yo_h.copy_(step.Y_o, non_blocking=True)
+
+    for _ in range(3):
+        e2e_step()
+    torch.cuda.synchronize()
+    ets = []
+    for _ in range(args.steps):
+        flush()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        e2e_step()
+        e1.record(s)
+        e1.synchronize()
+        ets.append(e0.elapsed_time(e1))
+    ms_e2e = statistics.mean(ets)
+
+    if world > 1:
+        t = torch.tensor([ms, ms_e2e], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, ms_e2e = float(t[0]), float(t[1])
+
+    ops = step.int_ops()
+    value = world * ops / (ms * 1e-3) / 1e12
+    tokens_s = world * L / (ms * 1e-3)
+    peaks, peak_src = load_peaks()
+    gemm_ops = q.int_ops() + o.int_ops()
+    gemm_ms = t_gemm_qkv + t_gemm_o
+    achieved = gemm_ops / (gemm_ms * 1e-3) / 1e12
+    peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]) * FP8_PER_BF16
+    hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    quant_x_bytes = L * K * 2 + L * K // 2 + 4 * L
+    quant_z_bytes = L * K * 4 + L * K // 2 + 4 * L
+    tac_bytes = L * K * 2 + L * K * 4 + K * o.tac_g * 4 + K * 4
+    traffic = profiled_traffic()
+    gemm_bytes = [L * K // 2 + q.N * K // 2 + 2 * L * q.N + 4 * (L + q.N),
+                  L * K // 2 + o.N * K // 2 + 2 * L * o.N + 4 * (L + o.N)]
+
+    if rank != 0:
+        return None
+    cpu = None
+    if world == 1 and not args.skip_cpu_baseline:
+        cpu = cpu_baseline(qkv_case, o_case, args.cpu_sample_tokens)
+    out = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "int4 (W4A4 codes, exact integer accumulation; fp32 transform and dequant; fp16 I/O)",
+        "data": "synthetic (seeded; LLaDA-8B-shaped activations and random-init weights)",
+        "config": config_dict(graph),
+        "tokens_per_s": round(tokens_s, 1),
+        "roofline": {
+            "bound": "tensor", "kernel": "w4a4_gemm_kernel (QKV + O launches)",
+            "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
+            "frac": round(achieved / peak, 4), "traffic": traffic,
+            "peak_source": f"{peak_src} bf16 dense burst x {FP8_PER_BF16} (fp8 kind::f8f6f4 path; "
+                           f"sm_103a has no integer tcgen05 MMA)",
+            "algorithmic": f"{gemm_ops} int ops per step over 2 launches; "
+                           f"{sum(gemm_bytes)} algorithmic bytes per step",
+            "launch_ms": {"qkv": round(t_gemm_qkv, 5), "o": round(t_gemm_o, 5)},
+        },
+        "roofline_hbm_kernels": {
+            "peak_gbs": hbm, "peak_source": peak_src,
+            "sgat_quantize_act_f16": {"ms": round(t_quant_x, 5), "bytes": quant_x_bytes,
+                                      "gbs": round(quant_x_bytes / t_quant_x / 1e6, 1),
+                                      "frac": round(quant_x_bytes / t_quant_x / 1e6 / hbm, 4)},
+            "tac_apply_g128": {"ms": round(t_tac, 5), "bytes": tac_bytes,
+                               "gbs": round(tac_bytes / t_tac / 1e6, 1),
+                               "frac": round(tac_bytes / t_tac / 1e6 / hbm, 4)},
+            "sgat_quantize_act_f32": {"ms": round(t_quant_z, 5), "bytes": quant_z_bytes,
+                                      "gbs": round(quant_z_bytes / t_quant_z / 1e6, 1),
+                                      "frac": round(quant_z_bytes / t_quant_z / 1e6 / hbm, 4)},
+        },
+        "e2e": {"value": round(world * ops / (ms_e2e * 1e-3) / 1e12, 3), "unit": UNIT,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms_e2e, 5)},
+        "gpu_launches": args.steps * step.KERNELS_PER_STEP,
+        "clocks": clk,
+        "cpu_baseline": cpu,
+    }
+    return out
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle legs
+# ---------------------------------------------------------------------------
+def oracle_prepare(qkv_case, o_case):
+    from oracle import sgat as osg
+    qw1, sw1 = osg.prepare_weight(qkv_case.W, qkv_case.xf.inv_a_w, qkv_case.xf.hb, 4)
+    qw2, sw2 = osg.prepare_weight(o_case.W, o_case.xf.inv_a_w, o_case.xf.hb, 4)
+    return (qw1, sw1), (qw2, sw2)
+
+
+def oracle_step(qkv_case, o_case, w, rows):
+    """One step of the oracle on the token rows `rows`: SGAT linear of X for
+    QKV, then TAC + SGAT linear of Z for O."""
+    from oracle import sgat as osg
+    from oracle import tac as otac
+    (qw1, sw1), (qw2, sw2) = w
+    xf = qkv_case.xf
+    osg.sgat_linear(qkv_case.X[rows], qkv_case.mask[rows], xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u,
+                    qw1, sw1, None, 4)
+    xf = o_case.xf
+    z = otac.tac_apply(o_case.X[rows], o_case.tac.M, o_case.tac.d, o_case.tac.g).astype("float32")
+    osg.sgat_linear(z, o_case.mask[rows], xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, qw2, sw2, None, 4)
+
+
+def cpu_cores():
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(var):
+            return int(os.environ[var])
+    return os.cpu_count() or 1
+
+
+def cpu_baseline(qkv_case, o_case, tokens):
+    import numpy as np
+    w = oracle_prepare(qkv_case, o_case)
+    rows = np.arange(min(tokens, qkv_case.L))
+    t0 = time.perf_counter()
+    oracle_step(qkv_case, o_case, w, rows)
+    dt = time.perf_counter() - t0
+    ops = 2 * len(rows) * (qkv_case.N + o_case.N) * qkv_case.K
+    return {"value": round(ops / dt / 1e12, 6), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"one full oracle step on {len(rows)} of {qkv_case.L} tokens "
+                      f"(TAC + SGAT quantise + exact int GEMM + dequant, both projections; "
+                      f"weight folding untimed); {dt:.2f} s",
+            "seconds": round(dt, 3)}
+
+
+def run_reference(args):
+    import numpy as np
+    from paper_2606_04945_gb300 import inputs
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return None
+    qkv_case, o_case = inputs.llada_attention(seed=0)
+    w = oracle_prepare(qkv_case, o_case)
+    S = min(args.ref_sample_tokens, qkv_case.L)
+    rng = np.random.default_rng(0)
+    for _ in range(args.warmup):
+        oracle_step(qkv_case, o_case, w, np.sort(rng.choice(qkv_case.L, S, replace=False)))
+    ts = []
+    for _ in range(args.steps):
+        rows = np.sort(rng.choice(qkv_case.L, S, replace=False))
+        t0 = time.perf_counter()
+        oracle_step(qkv_case, o_case, w, rows)
+        ts.append(time.perf_counter() - t0)
+    sec = statistics.mean(ts)
+    ops = 2 * S * (qkv_case.N + o_case.N) * qkv_case.K
+    value = ops / sec / 1e12
+    return {
+        "metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(sec * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int4 codes, int64-exact GEMM, fp32 transform, fp64 dequant",
+        "data": "synthetic (seeded; LLaDA-8B-shaped)", "config": config_dict(False), "impl": "reference",
+        "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "kind": "oracle", "cores": cpu_cores(),
+                         "sample": f"each step: {S} random tokens of the 1024-token workload"},
+        "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse()
+    out = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+    if args.impl == "ours" and int(os.environ.get("WORLD_SIZE", "1")) > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,170 @@
+/*
+ * starq.h -- C ABI of libstarq.so, the GB300 (sm_103a) hot path of the
+ * STaR-Quant quantised denoising step: the SGAT-transformed W4A4 linear and
+ * Temporal Attention Compensation (TAC).
+ *
+ * Conventions for every entry point:
+ *   - All array arguments are DEVICE pointers owned by the caller. The library
+ *     never allocates, frees or keeps a pointer past the call.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t passed as
+ *     void*; NULL = the legacy default stream). Arguments are validated on
+ *     the host before anything is launched; a call that returns an error
+ *     launched nothing.
+ *   - Return value: STARQ_OK (0) or a negative STARQ_ERR_* code; the
+ *     message of the last error on the calling thread is returned by
+ *     starq_last_error().
+ *   - Matrices are row-major and dense (row stride = number of columns).
+ *   - Packed int4: a [rows][K] code matrix is stored as uint8 [rows][K/2];
+ *     code k lives in byte k/2, even k in the low nibble, odd k in the high
+ *     nibble, each nibble in two's complement. Codes lie in [-7, 7].
+ *   - Mask: uint8 per token, 1 = masked (state m), 0 = unmasked (state u).
+ */
+#ifndef STARQ_H
+#define STARQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Element types of activations, weights and outputs. */
+enum starq_dtype { STARQ_F16 = 0, STARQ_BF16 = 1, STARQ_F32 = 2 };
+
+/* Return codes. */
+enum starq_status {
+    STARQ_OK = 0,
+    STARQ_ERR_ARG = -1,      /* null pointer or unknown enum value            */
+    STARQ_ERR_SHAPE = -2,    /* size outside the supported set (see each call) */
+    STARQ_ERR_ALIGN = -3,    /* pointer not aligned as the call requires       */
+    STARQ_ERR_BITS = -4,     /* bit-width other than 4 on the GPU path         */
+    STARQ_ERR_CUDA = -5,     /* a CUDA runtime call or launch failed           */
+    STARQ_ERR_TIMEOUT = -6   /* a kernel gave up a bounded wait (see status)   */
+};
+
+/* Library version (major * 10000 + minor * 100 + patch). */
+int starq_version(void);
+
+/* Message of the last error returned on the calling thread ("" if none). */
+const char* starq_last_error(void);
+
+/*
+ * Synchronise `stream`, then read and clear the device status word that the
+ * kernels set when a bounded wait inside them runs out. Returns STARQ_OK,
+ * STARQ_ERR_TIMEOUT (the kernel returned early; its outputs are undefined)
+ * or STARQ_ERR_CUDA.
+ */
+int starq_check_status(void* stream);
+
+/*
+ * sgat_quantize_act -- state-guided activation transform + per-token A4
+ * quantisation (Sec. 3.2 Eq. 7-11 and Eq. 13's Q_a; Sec. 3.1 Eq. 2-3).
+ *
+ * For every token i with state s = mask[i]:
+ *   v = ((X[i] * a_s) H_hb) G_s        (Phi_s of Eq. 11; H_hb is the
+ *                                        unnormalised block-diagonal Sylvester
+ *                                        Hadamard, fast transform in float32)
+ *   s_a[i] = amax / 7,  r = 7 / amax,  q = clamp(rne(v * r), -7, 7)
+ * Tokens are processed in place of the paper's split + scatter: each row
+ * picks its own transform, which gives the same rows in token order.
+ *
+ *   X       [L][K] activations, element type x_dtype (F16, BF16 or F32),
+ *           16-byte aligned.
+ *   mask    [L] uint8 or NULL (NULL = every token unmasked).
+ *   a_m,a_u [K] float32 per-state diagonal smoothing, 16-byte aligned, or
+ *           NULL (= ones).
+ *   hb      Hadamard block: power of two, 1 <= hb <= 4096, K % hb == 0
+ *           (hb = 1 is the identity).
+ *   d_sh,d_m,d_u  gate layout over transformed coordinates (Eq. 8-9):
+ *           [0, d_sh) shared, [d_sh, d_sh + d_m) masked-only, the rest
+ *           unmasked-only; each >= 0 and d_sh + d_m + d_u == K.
+ *   bits    must be 4.
+ *   Xq      [L][K/2] packed int4 codes out, 8-byte aligned.
+ *   s_a     [L] float32 per-token scales out (0 for an all-zero row).
+ *   v_dbg   [L][K] float32 transformed activations out (before rounding),
+ *           16-byte aligned, or NULL.
+ * Shapes: L >= 0, 16 <= K <= 20480, K % 16 == 0.
+ */
+int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                      const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                      int bits, uint8_t* Xq, float* s_a, float* v_dbg, void* stream);
+
+/*
+ * sgat_prepare_weight -- the unified static weight transform, quantised once
+ * (Sec. 3.2 Eq. 12; App. B W_f = Q_w(P^T W^T)), per-output-channel symmetric.
+ *
+ * For every output channel n:
+ *   w = ((W[n] * inv_a_w) H_hb) / hb   (float32, fast transform)
+ *   s_w[n] = amax / 7,  Wq[n] = clamp(rne(w * 7 / amax), -7, 7)
+ *
+ *   W       [N][K] weights, element type w_dtype (F16, BF16 or F32), 16-byte
+ *           aligned.
+ *   inv_a_w [K] float32 weight-side inverse smoothing or NULL (= ones).
+ *   Wq      [N][K/2] packed int4 out; s_w [N] float32 out.
+ * Shapes and hb as for sgat_quantize_act; bits must be 4.
+ */
+int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* inv_a_w, int hb,
+                        int bits, uint8_t* Wq, float* s_w, void* stream);
+
+/*
+ * w4a4_gemm -- the shared-weight integer projection and its dequantisation
+ * (Sec. 3.2 Eq. 13, Sec. 3.1 Eq. 5 and Eq. 3).
+ *
+ *   acc[i][n] = sum_k q_a[i][k] * q_w[n][k]            (exact integer)
+ *   Y[i][n]   = (float)acc * s_a[i] * s_w[n] (+ bias[n]) rounded to y_dtype
+ *               (float32 products in that order, then one rounding).
+ *
+ *   Xq [L][K/2], Wq [N][K/2] packed int4, 16-byte aligned.
+ *   s_a [L], s_w [N] float32; bias [N] float32 or NULL.
+ *   Y  [L][N] out, y_dtype F16, BF16 or F32, 16-byte aligned.
+ *   acc_dbg [L][N] int32 out (the exact accumulators) or NULL.
+ * Shapes: L >= 0, N >= 32 with N % 32 == 0, K >= 128 with K % 128 == 0,
+ * K <= 65536 (so |acc| <= 49 K < 2^22).
+ */
+int w4a4_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
+              const float* bias, int L, int N, int K, void* Y, int y_dtype, int32_t* acc_dbg,
+              void* stream);
+
+/*
+ * tac_apply -- block-wise affine compensation of the quantised attention
+ * output before the output projection (Sec. 3.3 Eq. 17; App. C row-major
+ * form Z_b M_b^T + 1 d_b^T).
+ *
+ *   out[i][b*g + r] = sum_j M[b][r][j] * Z[i][b*g + j] + d[b][r]
+ *
+ *   Z   [L][C] element type z_dtype (F16, BF16 or F32), 16-byte aligned.
+ *   M   [C/g][g][g] float32 (row r = output channel r of block b); d [C/g][g]
+ *       float32 (NULL = zeros). Both 16-byte aligned.
+ *   out [L][C] element type out_dtype (F16, BF16 or F32), 16-byte aligned;
+ *       must not overlap Z.
+ * Shapes: L >= 0, g in {4, 8, 16, 32, 64, 128}, C % g == 0, C % 8 == 0.
+ */
+int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d,
+              void* out, int out_dtype, void* stream);
+
+/*
+ * sgat_linear -- the fused SGAT W4A4 linear of one quantised layer: optional
+ * TAC on the input (Eq. 17), the state-guided transform and A4 quantisation
+ * (Eq. 11), and the shared-weight integer GEMM with its dequantisation
+ * epilogue (Eq. 13). Equivalent to tac_apply (to float32) ->
+ * sgat_quantize_act -> w4a4_gemm, with the intermediates in `workspace`.
+ *
+ *   tac_M, tac_d, tac_g: TAC parameters as for tac_apply, or tac_M = NULL
+ *   for no TAC. Wq/s_w come from sgat_prepare_weight. Other arguments as in
+ *   the calls above. K % 128 == 0.
+ *   workspace: device buffer of at least sgat_linear_workspace_size(L, K,
+ *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller.
+ */
+size_t sgat_linear_workspace_size(int L, int K, int with_tac);
+int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                const float* tac_M, const float* tac_d, int tac_g,
+                const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
+                void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* STARQ_H */

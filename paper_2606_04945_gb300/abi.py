@@ -1,0 +1,127 @@
+"""Python binding of libstarq.so (include/starq.h): argument marshalling only.
+
+Every function takes torch CUDA tensors, passes their device pointers and
+sizes to the C ABI, and raises ``StarqError`` with the library's message on
+a non-zero return. No step of the computation runs in Python: if the
+library is missing or fails to load, importing this module raises.
+"""
+
+import ctypes
+import os
+
+import torch
+
+from .build import LIB
+
+F16, BF16, F32 = 0, 1, 2
+OK, ERR_ARG, ERR_SHAPE, ERR_ALIGN, ERR_BITS, ERR_CUDA, ERR_TIMEOUT = 0, -1, -2, -3, -4, -5, -6
+
+EXPORTED = (
+    "starq_version", "starq_last_error", "starq_check_status",
+    "sgat_quantize_act", "sgat_prepare_weight", "w4a4_gemm", "tac_apply",
+    "sgat_linear_workspace_size", "sgat_linear",
+)
+
+
+class StarqError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"starq error {code}: {msg}")
+        self.code = code
+
+
+def _load():
+    if not os.path.exists(LIB):
+        raise ImportError(
+            f"{LIB} is missing: build it first (python -c 'import __graft_entry__ as g; g.build()')")
+    lib = ctypes.CDLL(LIB)
+    vp, i, f_p, u8p = ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p
+    lib.starq_version.restype = i
+    lib.starq_last_error.restype = ctypes.c_char_p
+    lib.starq_check_status.argtypes = [vp]
+    lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, i, u8p, f_p, f_p, vp]
+    lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
+    lib.w4a4_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, i, vp]
+    lib.sgat_linear_workspace_size.argtypes = [i, i, i]
+    lib.sgat_linear_workspace_size.restype = ctypes.c_size_t
+    lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
+                                u8p, f_p, f_p, i, i, vp, i, vp, ctypes.c_size_t, vp]
+    return lib
+
+
+lib = _load()
+
+
+def _check(rc):
+    if rc != 0:
+        raise StarqError(rc, lib.starq_last_error().decode())
+
+
+def dtype_code(t):
+    return {torch.float16: F16, torch.bfloat16: BF16, torch.float32: F32}[t.dtype]
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _contig(*ts):
+    for t in ts:
+        if t is not None and not t.is_contiguous():
+            raise ValueError("starq expects contiguous tensors")
+
+
+def check_status(stream=None):
+    """Synchronise and raise if a kernel gave up a bounded wait."""
+    _check(lib.starq_check_status(_stream(stream)))
+
+
+def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, bits=4, v_dbg=None,
+                      stream=None):
+    _contig(X, mask, a_m, a_u, Xq, s_a, v_dbg)
+    L, K = X.shape
+    _check(lib.sgat_quantize_act(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb,
+                                 d_sh, d_m, d_u, bits, _p(Xq), _p(s_a), _p(v_dbg), _stream(stream)))
+
+
+def sgat_prepare_weight(W, inv_a_w, hb, Wq, s_w, bits=4, stream=None):
+    _contig(W, inv_a_w, Wq, s_w)
+    N, K = W.shape
+    _check(lib.sgat_prepare_weight(_p(W), dtype_code(W), N, K, _p(inv_a_w), hb, bits,
+                                   _p(Wq), _p(s_w), _stream(stream)))
+
+
+def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, stream=None):
+    _contig(Xq, s_a, Wq, s_w, Y, bias, acc_dbg)
+    L = Xq.shape[0]
+    N = Wq.shape[0]
+    K = 2 * Xq.shape[1]
+    _check(lib.w4a4_gemm(_p(Xq), _p(s_a), _p(Wq), _p(s_w), _p(bias), L, N, K, _p(Y),
+                         dtype_code(Y), _p(acc_dbg), _stream(stream)))
+
+
+def tac_apply(Z, M, d, g, out, stream=None):
+    _contig(Z, M, d, out)
+    L, C = Z.shape
+    _check(lib.tac_apply(_p(Z), dtype_code(Z), L, C, g, _p(M), _p(d), _p(out), dtype_code(out),
+                         _stream(stream)))
+
+
+def sgat_linear_workspace_size(L, K, with_tac):
+    return int(lib.sgat_linear_workspace_size(L, K, 1 if with_tac else 0))
+
+
+def sgat_linear(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, workspace, bias=None,
+                tac_M=None, tac_d=None, tac_g=0, bits=4, stream=None):
+    _contig(X, mask, a_m, a_u, Wq, s_w, Y, workspace, bias, tac_M, tac_d)
+    L, K = X.shape
+    N = Wq.shape[0]
+    _check(lib.sgat_linear(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh, d_m,
+                           d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(s_w), _p(bias), N, bits,
+                           _p(Y), dtype_code(Y), _p(workspace), workspace.numel() * workspace.element_size(),
+                           _stream(stream)))

@@ -1,0 +1,240 @@
+// C ABI of libstarq.so (declared in include/starq.h): argument validation,
+// error reporting, the device status word, and the composition of the
+// kernels into sgat_linear.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "common.cuh"
+
+namespace starq {
+
+// Status word written by kernels whose bounded waits run out.
+__device__ unsigned g_status_word;
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+    return fail(STARQ_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+bool aligned(const void* p, size_t n) { return (reinterpret_cast<uintptr_t>(p) % n) == 0; }
+bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+bool dtype_ok(int t) { return t == STARQ_F16 || t == STARQ_BF16 || t == STARQ_F32; }
+
+unsigned* status_ptr(int* err) {
+    static unsigned* cache[64] = {nullptr};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess || dev >= 64) { *err = cuda_fail(e, "cudaGetDevice"); return nullptr; }
+    if (cache[dev] == nullptr) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_status_word);
+        if (e != cudaSuccess) { *err = cuda_fail(e, "cudaGetSymbolAddress(status)"); return nullptr; }
+        cache[dev] = static_cast<unsigned*>(p);
+    }
+    *err = STARQ_OK;
+    return cache[dev];
+}
+
+int check_transform(int K, int hb, int d_sh, int d_m, int d_u, const float* a_m, const float* a_u) {
+    if (K < 16 || K % 16 != 0 || K > 20480)
+        return fail(STARQ_ERR_SHAPE, "K=%d: need 16 <= K <= 20480 and K %% 16 == 0", K);
+    if (!pow2(hb) || hb > 4096 || K % hb != 0)
+        return fail(STARQ_ERR_SHAPE, "hb=%d: need a power of two <= 4096 dividing K=%d", hb, K);
+    if (d_sh < 0 || d_m < 0 || d_u < 0 || (long)d_sh + d_m + d_u != K)
+        return fail(STARQ_ERR_SHAPE, "gate layout (%d, %d, %d) must be >= 0 and sum to K=%d",
+                    d_sh, d_m, d_u, K);
+    if ((a_m && !aligned(a_m, 16)) || (a_u && !aligned(a_u, 16)))
+        return fail(STARQ_ERR_ALIGN, "smoothing vectors must be 16-byte aligned");
+    return STARQ_OK;
+}
+
+int check_tac(int L, int C, int g, const float* M, const float* d) {
+    if (M == nullptr) return fail(STARQ_ERR_ARG, "TAC matrix M is NULL");
+    if (!(g == 4 || g == 8 || g == 16 || g == 32 || g == 64 || g == 128))
+        return fail(STARQ_ERR_SHAPE, "TAC block g=%d: supported 4, 8, 16, 32, 64, 128", g);
+    if (C <= 0 || C % g != 0 || C % 8 != 0)
+        return fail(STARQ_ERR_SHAPE, "TAC width C=%d must be a positive multiple of g=%d and 8", C, g);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    if (!aligned(M, 16) || (d && !aligned(d, 16)))
+        return fail(STARQ_ERR_ALIGN, "TAC M and d must be 16-byte aligned");
+    return STARQ_OK;
+}
+
+int check_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
+               const float* bias, int L, int N, int K, void* Y, int y_dtype) {
+    if (!Xq || !s_a || !Wq || !s_w || !Y) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL argument");
+    if (!dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "w4a4_gemm: unknown output dtype %d", y_dtype);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    if (N < 32 || N % 32 != 0) return fail(STARQ_ERR_SHAPE, "N=%d: need N >= 32, N %% 32 == 0", N);
+    if (K < 128 || K % 128 != 0 || K > 65536)
+        return fail(STARQ_ERR_SHAPE, "K=%d: need 128 <= K <= 65536 and K %% 128 == 0", K);
+    if (!aligned(Xq, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(s_w, 16) ||
+        (bias && !aligned(bias, 16)) || !aligned(s_a, 4))
+        return fail(STARQ_ERR_ALIGN, "w4a4_gemm: Xq, Wq, Y, s_w, bias must be 16-byte aligned");
+    return STARQ_OK;
+}
+
+constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+}  // namespace
+
+int num_sms() {
+    static int cache[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 64) dev = 63;
+    if (cache[dev] == 0) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        cache[dev] = n > 0 ? n : 1;
+    }
+    return cache[dev];
+}
+
+}  // namespace starq
+
+using namespace starq;
+
+extern "C" {
+
+int starq_version(void) { return 100; }
+
+const char* starq_last_error(void) { return g_err; }
+
+int starq_check_status(void* stream) {
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    unsigned v = 0, zero = 0;
+    e = cudaMemcpyFromSymbol(&v, g_status_word, sizeof(v));
+    if (e != cudaSuccess) return cuda_fail(e, "read status word");
+    if (v != 0) {
+        e = cudaMemcpyToSymbol(g_status_word, &zero, sizeof(zero));
+        if (e != cudaSuccess) return cuda_fail(e, "clear status word");
+        return fail(STARQ_ERR_TIMEOUT, "a kernel gave up a bounded wait (status bits 0x%x)", v);
+    }
+    return STARQ_OK;
+}
+
+int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                      const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                      int bits, uint8_t* Xq, float* s_a, float* v_dbg, void* stream) {
+    if (!X || !Xq || !s_a) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, Xq or s_a");
+    if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: unknown dtype %d", x_dtype);
+    if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
+    if (rc) return rc;
+    if (!aligned(X, 16) || !aligned(Xq, 8) || (v_dbg && !aligned(v_dbg, 16)))
+        return fail(STARQ_ERR_ALIGN, "sgat_quantize_act: X (16 B), Xq (8 B), v_dbg (16 B) alignment");
+    QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, v_dbg};
+    cudaError_t e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "sgat_quantize_act launch");
+    return STARQ_OK;
+}
+
+int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* inv_a_w, int hb,
+                        int bits, uint8_t* Wq, float* s_w, void* stream) {
+    if (!W || !Wq || !s_w) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: NULL W, Wq or s_w");
+    if (!dtype_ok(w_dtype)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: unknown dtype %d", w_dtype);
+    if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
+    if (N < 0) return fail(STARQ_ERR_SHAPE, "N=%d < 0", N);
+    int rc = check_transform(K, hb, K, 0, 0, nullptr, inv_a_w);
+    if (rc) return rc;
+    if (!aligned(W, 16) || !aligned(Wq, 8))
+        return fail(STARQ_ERR_ALIGN, "sgat_prepare_weight: W (16 B), Wq (8 B) alignment");
+    QuantArgs a{W, w_dtype, N, K, nullptr, nullptr, inv_a_w, hb, K, 0, 0, 7, 1.f / (float)hb,
+                Wq, s_w, nullptr};
+    cudaError_t e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "sgat_prepare_weight launch");
+    return STARQ_OK;
+}
+
+int w4a4_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
+              const float* bias, int L, int N, int K, void* Y, int y_dtype, int32_t* acc_dbg,
+              void* stream) {
+    int rc = check_gemm(Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
+    if (rc) return rc;
+    if (acc_dbg && !aligned(acc_dbg, 16)) return fail(STARQ_ERR_ALIGN, "acc_dbg must be 16-byte aligned");
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st};
+    cudaError_t e = launch_w4a4_gemm(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm launch");
+    return STARQ_OK;
+}
+
+int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d,
+              void* out, int out_dtype, void* stream) {
+    if (!Z || !out) return fail(STARQ_ERR_ARG, "tac_apply: NULL Z or out");
+    if (!dtype_ok(z_dtype) || !dtype_ok(out_dtype)) return fail(STARQ_ERR_ARG, "tac_apply: unknown dtype");
+    int rc = check_tac(L, C, g, M, d);
+    if (rc) return rc;
+    if (!aligned(Z, 16) || !aligned(out, 16)) return fail(STARQ_ERR_ALIGN, "tac_apply: Z, out alignment");
+    TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype};
+    cudaError_t e = launch_tac(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "tac_apply launch");
+    return STARQ_OK;
+}
+
+size_t sgat_linear_workspace_size(int L, int K, int with_tac) {
+    if (L < 0 || K < 0) return 0;
+    size_t n = align256((size_t)L * K / 2) + align256((size_t)L * 4);
+    if (with_tac) n += align256((size_t)L * K * 4);
+    return n;
+}
+
+int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                const float* tac_M, const float* tac_d, int tac_g,
+                const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
+                void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
+    if (!X || !Wq || !s_w || !Y || !workspace) return fail(STARQ_ERR_ARG, "sgat_linear: NULL argument");
+    if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear: unknown dtype");
+    if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
+    if (rc) return rc;
+    if (tac_M && (rc = check_tac(L, K, tac_g, tac_M, tac_d))) return rc;
+    const size_t need = sgat_linear_workspace_size(L, K, tac_M != nullptr);
+    if (workspace_bytes < need)
+        return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu needed", workspace_bytes, need);
+    if (!aligned(workspace, 256) || !aligned(X, 16)) return fail(STARQ_ERR_ALIGN, "sgat_linear alignment");
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    uint8_t* Xq = ws;
+    float* s_a = reinterpret_cast<float*>(ws + align256((size_t)L * K / 2));
+    float* zt = tac_M ? reinterpret_cast<float*>(ws + align256((size_t)L * K / 2) + align256((size_t)L * 4))
+                      : nullptr;
+    rc = check_gemm(Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
+    if (rc) return rc;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const void* qin = X;
+    int qin_dtype = x_dtype;
+    cudaError_t e;
+    if (tac_M) {
+        TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, STARQ_F32};
+        if ((e = launch_tac(t, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: tac launch");
+        qin = zt;
+        qin_dtype = STARQ_F32;
+    }
+    QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr};
+    if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");
+    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st};
+    if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: gemm launch");
+    return STARQ_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,237 @@
+// Device-side helpers shared by the libstarq kernels (sm_103a only):
+// mbarrier and tcgen05 PTX wrappers, bounded waits, shared-memory matrix
+// descriptors, and the launcher interface between the C ABI and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_fp16.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/starq.h"
+
+namespace starq {
+
+// Bits of the device status word (set with atomicOr, read and cleared by
+// starq_check_status).
+constexpr unsigned STATUS_TIMEOUT_GEMM = 1u << 0;
+constexpr unsigned STATUS_TIMEOUT_FP16_GEMM = 1u << 1;
+constexpr unsigned STATUS_TIMEOUT_TEST = 1u << 2;
+
+// Upper bound of any single wait inside a kernel. Kernels of this library
+// finish in milliseconds; a wait this long means a broken pipeline, and the
+// kernel gives up, records it and returns instead of hanging the GPU.
+constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;  // 2 s
+
+// ---------------------------------------------------------------------------
+// Launchers (host functions in each kernel translation unit). Arguments are
+// validated by the C ABI before these are called.
+// ---------------------------------------------------------------------------
+struct QuantArgs {
+    const void* X; int x_dtype; int L; int K;
+    const uint8_t* mask; const float* a_m; const float* a_u;
+    int hb; int d_sh; int d_m; int d_u;
+    int qmax; float post_scale;
+    uint8_t* Xq; float* s; float* v_dbg;
+};
+cudaError_t launch_sgat_quant(const QuantArgs& a, cudaStream_t stream);
+
+struct GemmArgs {
+    const uint8_t* Xq; const float* s_a; const uint8_t* Wq; const float* s_w;
+    const float* bias; int L; int N; int K;
+    void* Y; int y_dtype; int32_t* acc_dbg;
+    unsigned* status;
+};
+cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+
+struct TacArgs {
+    const void* Z; int z_dtype; int L; int C; int g;
+    const float* M; const float* d; void* out; int out_dtype;
+};
+cudaError_t launch_tac(const TacArgs& a, cudaStream_t stream);
+
+int num_sms();  // SM count of the current device (cached per device)
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("{\n\t.reg .b64 st;\n\tmbarrier.arrive.shared::cta.b64 st, [%0];\n\t}"
+                 :: "r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile("{\n\t.reg .pred p;\n\t"
+                 "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}"
+                 : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase of `bar` with the given parity to complete. Gives up
+// (returns false) after WAIT_LIMIT_NS, or early when *abort is set by another
+// role of the same CTA that has already given up.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
+                                                  volatile int* abort) {
+    #pragma unroll 1
+    for (int i = 0; i < 256; ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    #pragma unroll 1
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort) return false;
+        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) return false;
+    }
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// ---- tcgen05 (5th-generation tensor core, tensor memory) -----------------
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                 :: "r"(dst_smem), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;"
+                 :: "r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Arrive once on `bar` when every tcgen05 operation issued so far by this
+// thread has completed.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];"
+                 :: "r"(bar) : "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, E4M3 x E4M3 -> F32 (kind::f8f6f4).
+__device__ __forceinline__ void mma_f8f6f4(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                           uint32_t idesc, uint32_t accumulate) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}"
+                 :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+                 : "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, F16/BF16 inputs -> F32 (kind::f16).
+__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                        uint32_t idesc, uint32_t accumulate) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+                 :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+                 : "memory");
+}
+
+// 32 consecutive 32-bit columns of one TMEM lane per thread (lanes = the
+// warp's 32-lane quarter).
+__device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+          "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
+          "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]),
+          "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]),
+          "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor for a K-major operand tile stored in the
+// 128-byte swizzle layout: rows of 128 bytes, 8-row atoms of 1024 bytes
+// (stride-dimension byte offset), 16-byte chunks XOR-ed with the row index
+// within the atom. `addr` is the byte address of the tile's first row plus
+// the K offset (in bytes, < 128) of the sub-block the MMA reads; the atom
+// base must be 1024-byte aligned.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((addr & 0x3FFFFu) >> 4);          // start address
+    d |= (uint64_t)1 << 16;                            // leading byte offset (unused)
+    d |= (uint64_t)(1024u >> 4) << 32;                 // stride byte offset
+    d |= (uint64_t)1 << 46;                            // descriptor version
+    d |= (uint64_t)2 << 61;                            // 128-byte swizzle
+    return d;
+}
+
+// Byte offset of logical 16-byte chunk `c` (0..7) of row `row` inside a
+// 128-byte-swizzled K-major tile.
+__device__ __forceinline__ uint32_t sw128_offset(uint32_t row, uint32_t c) {
+    return (row >> 3) * 1024u + (row & 7u) * 128u + ((c ^ (row & 7u)) << 4);
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b,
+                                             uint32_t c, uint32_t d) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};"
+                 :: "r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+
+__device__ __forceinline__ uint4 ld_global_nc_v4(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+    return v;
+}
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+
+// Eight int4 codes (two's complement nibbles, code k in bits 4k..4k+3) to
+// eight E4M3 bytes (byte k = code k). Every integer in [-8, 7] is exact in
+// E4M3. Two byte-permutes look the magnitude up in 8-entry tables (the
+// selector's top bit replicates a zero sign for the other half of the codes),
+// a third spreads the nibble sign bits to the byte sign bits.
+__device__ __forceinline__ void int4x8_to_e4m3x8(uint32_t x, uint32_t& lo, uint32_t& hi) {
+    // positive codes 0..7: 0x00 0x38 0x40 0x44 | 0x48 0x4A 0x4C 0x4E
+    constexpr uint32_t P0 = 0x44403800u, P1 = 0x4E4C4A48u;
+    // negative codes -8..-1 indexed by the low three bits (magnitude bytes,
+    // sign added separately): 8 7 6 5 | 4 3 2 1
+    constexpr uint32_t N0 = 0x4A4C4E50u, N1 = 0x38404448u;
+    const uint32_t xn = x ^ 0x88888888u;
+    const uint32_t xh = x >> 16, xnh = xn >> 16;
+    const uint32_t mlo = prmt(P0, P1, x) | prmt(N0, N1, xn);
+    const uint32_t mhi = prmt(P0, P1, xh) | prmt(N0, N1, xnh);
+    const uint32_t ylo = prmt(x, 0, 0x1100u);   // bytes: x0 x0 x1 x1
+    const uint32_t yhi = prmt(x, 0, 0x3322u);   // bytes: x2 x2 x3 x3
+    const uint32_t slo = ((ylo << 4) & 0x00800080u) | (ylo & 0x80008000u);
+    const uint32_t shi = ((yhi << 4) & 0x00800080u) | (yhi & 0x80008000u);
+    lo = mlo | slo;
+    hi = mhi | shi;
+}
+
+}  // namespace starq

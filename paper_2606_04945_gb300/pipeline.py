@@ -1,0 +1,103 @@
+"""Device-resident SGAT W4A4 layers built on the C ABI.
+
+``SgatLinear`` holds one quantised linear on the GPU: the folded int4
+weight (Eq. 12, prepared once by ``sgat_prepare_weight``), the two state
+transforms, optional TAC parameters and a workspace. ``run`` is one call to
+``sgat_linear`` (TAC -> state-guided quantisation -> W4A4 GEMM + dequant).
+
+``AttentionProjections`` is the attention-side hot path of one denoising
+step of a LLaDA-shaped layer: the fused QKV projection of the layer input,
+then TAC on the attention output followed by the O projection (Sec. 3.3: TAC
+sits between the softmax-value product and W_o). ``capture`` records the step
+in a CUDA graph so a replay issues all five kernels with one launch.
+"""
+
+import numpy as np
+import torch
+
+from . import abi
+
+
+def _dev(x, dtype=None, device="cuda"):
+    t = torch.from_numpy(np.ascontiguousarray(x))
+    if dtype is not None:
+        t = t.to(dtype)
+    return t.to(device)
+
+
+TORCH_DTYPE = {"f16": torch.float16, "bf16": torch.bfloat16, "f32": torch.float32}
+
+
+class SgatLinear:
+    def __init__(self, case, device="cuda", out_dtype=None):
+        xf = case.xf
+        self.L, self.K, self.N = case.L, case.K, case.N
+        self.dtype = TORCH_DTYPE[case.dtype]
+        self.out_dtype = TORCH_DTYPE[out_dtype or case.dtype]
+        self.hb, self.d_sh, self.d_m, self.d_u = xf.hb, xf.d_sh, xf.d_m, xf.d_u
+        self.a_m = _dev(xf.a_m, device=device)
+        self.a_u = _dev(xf.a_u, device=device)
+        self.bias = _dev(case.bias, device=device) if case.bias is not None else None
+        self.tac = case.tac
+        if case.tac is not None:
+            self.tac_M = _dev(case.tac.M, device=device)
+            self.tac_d = _dev(case.tac.d, device=device)
+            self.tac_g = case.tac.g
+        else:
+            self.tac_M = self.tac_d = None
+            self.tac_g = 0
+        W = _dev(case.W, self.dtype, device)
+        self.Wq = torch.empty(self.N, self.K // 2, dtype=torch.uint8, device=device)
+        self.s_w = torch.empty(self.N, dtype=torch.float32, device=device)
+        abi.sgat_prepare_weight(W, _dev(xf.inv_a_w, device=device), self.hb, self.Wq, self.s_w)
+        del W
+        self.workspace = torch.empty(abi.sgat_linear_workspace_size(self.L, self.K, self.tac is not None),
+                                     dtype=torch.uint8, device=device)
+
+    def run(self, X, mask, Y, stream=None):
+        abi.sgat_linear(X, mask, self.a_m, self.a_u, self.hb, self.d_sh, self.d_m, self.d_u,
+                        self.Wq, self.s_w, Y, self.workspace, bias=self.bias, tac_M=self.tac_M,
+                        tac_d=self.tac_d, tac_g=self.tac_g, stream=stream)
+
+    def int_ops(self, L=None):
+        return 2 * (L or self.L) * self.N * self.K
+
+
+class AttentionProjections:
+    """QKV projection of X and TAC + O projection of Z for one step."""
+
+    def __init__(self, qkv_case, o_case, device="cuda"):
+        self.qkv = SgatLinear(qkv_case, device)
+        self.o = SgatLinear(o_case, device)
+        self.L = qkv_case.L
+        self.X = _dev(qkv_case.X, self.qkv.dtype, device)
+        self.Z = _dev(o_case.X, self.o.dtype, device)
+        self.mask = _dev(qkv_case.mask, device=device)
+        self.Y_qkv = torch.empty(self.L, self.qkv.N, dtype=self.qkv.out_dtype, device=device)
+        self.Y_o = torch.empty(self.L, self.o.N, dtype=self.o.out_dtype, device=device)
+        self.graph = None
+
+    def step(self, stream=None):
+        self.qkv.run(self.X, self.mask, self.Y_qkv, stream)
+        self.o.run(self.Z, self.mask, self.Y_o, stream)
+
+    def capture(self):
+        """Record one step in a CUDA graph (call after a warm-up step)."""
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.step()
+        torch.cuda.current_stream().wait_stream(s)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.step()
+        self.graph = g
+        return g
+
+    def replay(self):
+        self.graph.replay()
+
+    def int_ops(self):
+        return self.qkv.int_ops() + self.o.int_ops()
+
+    KERNELS_PER_STEP = 5   # quant + GEMM (QKV); TAC + quant + GEMM (O)

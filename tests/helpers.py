@@ -1,0 +1,102 @@
+"""Shared test plumbing: device transfer, oracle runs, tolerances.
+
+Tolerances (spec bar; the readings are listed in the design doc):
+  * int codes, scales and integer accumulators: bit-exact.
+  * dequantised outputs in float16: |gpu - ref| <= 1e-3 |ref| + 2^-25 (the
+    absolute half-spacing of float16 subnormals), ref = float64 oracle.
+  * bfloat16 outputs: one bfloat16 rounding alone exceeds 1e-3, so the bound
+    is 1e-3 |ref| + half a bfloat16 spacing at |ref|.
+  * float32 outputs: 1e-6 |ref| + 1e-30.
+  * TAC outputs: |gpu - ref| / max(|ref|, 1e-2 rms(ref)) <= 1e-3 (plus the
+    output type's half-spacing for 16-bit outputs).
+"""
+
+import numpy as np
+import torch
+
+from oracle import sgat as osg
+
+F32 = np.float32
+
+
+def dev(x, dtype=None):
+    """numpy -> contiguous CUDA tensor (bf16 values stored as float32 are cast
+    exactly)."""
+    t = torch.from_numpy(np.ascontiguousarray(x))
+    if dtype is not None:
+        t = t.to(dtype)
+    return t.cuda()
+
+
+def torch_dtype(name):
+    return {"f16": torch.float16, "bf16": torch.bfloat16, "f32": torch.float32}[name]
+
+
+def host(t):
+    return t.detach().float().cpu().numpy() if t.dtype in (torch.float16, torch.bfloat16) else t.detach().cpu().numpy()
+
+
+def unpack(t):
+    return osg.unpack_int4(t.cpu().numpy())
+
+
+def half_spacing(ref, dtype):
+    a = np.abs(ref).astype(np.float64)
+    if dtype == "f16":
+        return np.full_like(a, 2.0 ** -25)
+    if dtype == "bf16":
+        e = np.floor(np.log2(np.maximum(a, 2.0 ** -126)))
+        return 0.5 * 2.0 ** (e - 7)
+    return np.zeros_like(a)
+
+
+def assert_output_close(gpu, ref, dtype, what="Y"):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert gpu.shape == ref.shape
+    if dtype == "f32":
+        tol = 1e-6 * np.abs(ref) + 1e-30
+    else:
+        tol = 1e-3 * np.abs(ref) + half_spacing(ref, dtype)
+        if dtype == "f16":
+            tol = 1e-3 * np.abs(ref) + 2.0 ** -25
+    err = np.abs(gpu - ref)
+    bad = err > tol
+    if bad.any():
+        i = np.unravel_index(np.argmax(err - tol), err.shape)
+        raise AssertionError(f"{what}: {bad.sum()} of {bad.size} outside tolerance; worst at {i}: "
+                             f"gpu={gpu[i]!r} ref={ref[i]!r} tol={tol[i]!r}")
+
+
+def assert_tac_close(gpu, ref, dtype="f32"):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    floor = 1e-2 * np.sqrt(np.mean(ref ** 2)) if ref.size else 0.0
+    denom = np.maximum(np.abs(ref), floor)
+    err = np.abs(gpu - ref) - half_spacing(ref, dtype) if dtype != "f32" else np.abs(gpu - ref)
+    rel = np.max(np.maximum(err, 0) / denom) if ref.size else 0.0
+    assert rel <= 1e-3, f"TAC max relative error {rel:.3e} > 1e-3"
+
+
+def gemm_codes(seed, L, N, K, lo=-7, hi=7):
+    rng = np.random.default_rng(seed)
+    qa = rng.integers(lo, hi + 1, (L, K)).astype(np.int32)
+    qw = rng.integers(lo, hi + 1, (N, K)).astype(np.int32)
+    s_a = rng.uniform(0.01, 2.0, L).astype(F32)
+    s_w = rng.uniform(0.001, 0.05, N).astype(F32)
+    return qa, qw, s_a, s_w
+
+
+def workspace_views(ws, L, K, with_tac):
+    """Views of the intermediates sgat_linear leaves in its workspace
+    (packed codes, per-token scales, float32 TAC output), following the
+    layout documented at sgat_linear_workspace_size."""
+    a256 = lambda x: (x + 255) // 256 * 256
+    o1 = a256(L * K // 2)
+    Xq = ws[: L * K // 2].view(L, K // 2)
+    s_a = ws[o1: o1 + 4 * L].view(torch.float32)
+    zt = None
+    if with_tac:
+        o2 = o1 + a256(4 * L)
+        zt = ws[o2: o2 + 4 * L * K].view(torch.float32).view(L, K)
+    return Xq, s_a, zt

@@ -1,0 +1,103 @@
+"""Host-side checks of libstarq.so that need no GPU.
+
+The library builds for sm_103a, loads, exports every function declared in
+include/*.h, and rejects bad arguments with the documented error code before
+any CUDA call (only validation paths run here: no compute call is made).
+"""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from tests.conftest import ROOT
+
+
+def declared_functions():
+    names = []
+    inc = os.path.join(ROOT, "include")
+    for fn in sorted(os.listdir(inc)):
+        if not fn.endswith(".h"):
+            continue
+        src = open(os.path.join(inc, fn)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        for m in re.finditer(r"^[A-Za-z_][\w \*]*?\b([A-Za-z_]\w*)\s*\(", src, flags=re.M):
+            if not src[m.start():].startswith(("typedef", "enum", "struct", "#")):
+                names.append(m.group(1))
+    return sorted(set(names))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_04945_gb300 import build
+    build.build()
+    from paper_2606_04945_gb300 import abi
+    return abi
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert "sgat_linear" in names and "w4a4_gemm" in names and len(names) >= 9
+    for n in names:
+        assert hasattr(lib.lib, n), n
+    assert set(lib.EXPORTED) <= set(names)
+
+
+def test_version_and_last_error(lib):
+    assert lib.lib.starq_version() >= 100
+    assert isinstance(lib.lib.starq_last_error(), bytes)
+
+
+P = ctypes.c_void_p(4096)  # a non-null, 16-byte-aligned stand-in; never dereferenced
+
+
+@pytest.mark.parametrize("args,code", [
+    ((None, 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -1),   # NULL X
+    ((P, 9, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -1),      # dtype
+    ((P, 0, 4, 512, None, None, None, 512, 512, 0, 0, 8, P, P, None, None), -4),      # bits
+    ((P, 0, 4, 100, None, None, None, 4, 100, 0, 0, 4, P, P, None, None), -2),        # K % 16
+    ((P, 0, 4, 512, None, None, None, 384, 512, 0, 0, 4, P, P, None, None), -2),      # hb not pow2
+    ((P, 0, 4, 512, None, None, None, 8192, 512, 0, 0, 4, P, P, None, None), -2),     # hb > K
+    ((P, 0, 4, 512, None, None, None, 512, 500, 6, 0, 4, P, P, None, None), -2),      # gate sum
+    ((P, 0, -1, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -2),     # L < 0
+    ((ctypes.c_void_p(4100), 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -3),
+])
+def test_quantize_act_validation(lib, args, code):
+    assert lib.lib.sgat_quantize_act(*args) == code
+    assert lib.lib.starq_last_error()
+
+
+@pytest.mark.parametrize("L,N,K,code", [(4, 100, 512, -2), (4, 256, 200, -2), (4, 256, 131072, -2),
+                                        (-1, 256, 512, -2)])
+def test_gemm_validation(lib, L, N, K, code):
+    assert lib.lib.w4a4_gemm(P, P, P, P, None, L, N, K, P, 0, None, None) == code
+
+
+def test_gemm_null_and_alignment(lib):
+    assert lib.lib.w4a4_gemm(None, P, P, P, None, 4, 256, 512, P, 0, None, None) == -1
+    assert lib.lib.w4a4_gemm(ctypes.c_void_p(4104), P, P, P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert lib.lib.w4a4_gemm(P, P, P, P, None, 4, 256, 512, P, 7, None, None) == -1
+
+
+@pytest.mark.parametrize("g,C,code", [(12, 96, -2), (16, 100, -2), (256, 4096, -2)])
+def test_tac_validation(lib, g, C, code):
+    assert lib.lib.tac_apply(P, 0, 4, C, g, P, P, P, 0, None) == code
+
+
+def test_tac_null_matrix(lib):
+    assert lib.lib.tac_apply(P, 0, 4, 64, 16, None, P, P, 0, None) == -1
+
+
+def test_linear_workspace_and_validation(lib):
+    n = lib.sgat_linear_workspace_size(1024, 4096, False)
+    assert n == 1024 * 2048 + 4096
+    assert lib.sgat_linear_workspace_size(1024, 4096, True) == n + 1024 * 4096 * 4
+    # workspace too small
+    rc = lib.lib.sgat_linear(P, 0, 1024, 4096, None, None, None, 4096, 4096, 0, 0, None, None, 0,
+                             P, P, None, 256, 4, P, 0, P, 16, None)
+    assert rc == -2 and b"workspace" in lib.lib.starq_last_error()
+    # TAC block that does not divide K
+    rc = lib.lib.sgat_linear(P, 0, 16, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 48,
+                             P, P, None, 256, 4, P, 0, P, 1 << 30, None)
+    assert rc == -2

@@ -1,0 +1,261 @@
+"""GPU (libstarq.so through its C ABI) against the CPU oracle.
+
+Bit-exact: packed int4 codes, per-row scales, float32 transformed values and
+the integer accumulators. Tolerance (tests/helpers.py): dequantised outputs
+and TAC. Sizes run from one token to several tiles with ragged tails, plus
+the edge cases of the method (all-zero rows, all-masked / all-unmasked
+batches, no mask, identity transform, gates off).
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import sgat as osg
+from oracle import tac as otac
+from paper_2606_04945_gb300 import inputs
+from tests import helpers as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def abi():
+    from paper_2606_04945_gb300 import abi as a
+    return a
+
+
+def run_quant(abi, case, mask=True, dbg=True):
+    xf = case.xf
+    X = H.dev(case.X, H.torch_dtype(case.dtype))
+    L, K = case.X.shape
+    m = H.dev(case.mask) if mask else None
+    a_m, a_u = H.dev(xf.a_m), H.dev(xf.a_u)
+    Xq = torch.empty(L, K // 2, dtype=torch.uint8, device="cuda")
+    s_a = torch.empty(L, dtype=torch.float32, device="cuda")
+    v = torch.empty(L, K, dtype=torch.float32, device="cuda") if dbg else None
+    abi.sgat_quantize_act(X, m, a_m, a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, Xq, s_a, v_dbg=v)
+    abi.check_status()
+    return Xq, s_a, v
+
+
+QUANT_CASES = [
+    # (L, K, hb, dtype, gates_on)
+    (1, 512, 512, "f16", True),
+    (7, 128, 128, "f16", True),
+    (33, 3584, 512, "bf16", True),
+    (129, 4096, 4096, "f16", True),
+    (5, 12288, 4096, "f16", True),
+    (3, 18944, 512, "bf16", True),
+    (64, 1024, 1024, "f16", False),
+    (40, 2048, 2048, "f32", True),
+    (9, 256, 16, "f16", True),
+    (9, 256, 1, "f16", False),
+    (300, 640, 128, "f16", True),
+]
+
+
+@pytest.mark.parametrize("L,K,hb,dtype,gates", QUANT_CASES)
+def test_quantize_act_bitexact(abi, L, K, hb, dtype, gates):
+    case = inputs.random_linear(L + K + hb, L, K, 128, dtype=dtype, gates_on=gates, hb=hb)
+    xf = case.xf
+    Xq, s_a, v = run_quant(abi, case)
+    codes, s = osg.sgat_quantize_act(case.X, case.mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, 4)
+    V = osg.sgat_transform(case.X, case.mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u)
+    assert np.array_equal(v.cpu().numpy(), V), "transformed activations differ"
+    assert np.array_equal(H.unpack(Xq), codes), "int4 codes differ"
+    assert np.array_equal(s_a.cpu().numpy(), s), "scales differ"
+
+
+def test_quantize_act_edge_cases(abi):
+    """No mask (all unmasked), all masked, mixed; an all-zero row in each."""
+    case = inputs.random_linear(5, 24, 512, 128, hb=512)
+    case.X[3] = 0
+    xf = case.xf
+    mixed = case.mask.copy()
+    for mode in ("none", "all", "mixed"):
+        if mode == "none":
+            mask_np = np.zeros(case.L, np.uint8)
+            Xq, s_a, _ = run_quant(abi, case, mask=False)
+        else:
+            mask_np = np.ones(case.L, np.uint8) if mode == "all" else mixed
+            case.mask = mask_np
+            Xq, s_a, _ = run_quant(abi, case)
+        codes, s = osg.sgat_quantize_act(case.X, mask_np, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, 4)
+        assert np.array_equal(H.unpack(Xq), codes), mode
+        assert np.array_equal(s_a.cpu().numpy(), s), mode
+        assert s[3] == 0 and not codes[3].any()
+
+
+@pytest.mark.parametrize("N,K,hb,dtype", [(256, 512, 512, "f16"), (96, 4096, 4096, "bf16"),
+                                          (64, 18944, 512, "bf16"), (32, 128, 1, "f32")])
+def test_prepare_weight_bitexact(abi, N, K, hb, dtype):
+    case = inputs.random_linear(N + K, 16, K, N, dtype=dtype, hb=hb)
+    W = H.dev(case.W, H.torch_dtype(dtype))
+    inv = H.dev(case.xf.inv_a_w)
+    Wq = torch.empty(N, K // 2, dtype=torch.uint8, device="cuda")
+    s_w = torch.empty(N, dtype=torch.float32, device="cuda")
+    abi.sgat_prepare_weight(W, inv, hb, Wq, s_w)
+    abi.check_status()
+    q, s = osg.prepare_weight(case.W, case.xf.inv_a_w, hb, 4)
+    assert np.array_equal(H.unpack(Wq), q)
+    assert np.array_equal(s_w.cpu().numpy(), s)
+
+
+def run_gemm(abi, qa, qw, s_a, s_w, out="f16", bias=None):
+    L, K = qa.shape
+    N = qw.shape[0]
+    Xq = H.dev(osg.pack_int4(qa))
+    Wq = H.dev(osg.pack_int4(qw))
+    Y = torch.empty(L, N, dtype=H.torch_dtype(out), device="cuda")
+    acc = torch.empty(L, N, dtype=torch.int32, device="cuda")
+    abi.w4a4_gemm(Xq, H.dev(s_a), Wq, H.dev(s_w), Y, bias=None if bias is None else H.dev(bias), acc_dbg=acc)
+    abi.check_status()
+    return H.host(Y), acc.cpu().numpy()
+
+
+@pytest.mark.parametrize("L,N,K,out", [(1, 256, 128, "f16"), (129, 512, 512, "f16"), (300, 288, 1024, "bf16"),
+                                       (128, 256, 4096, "f32"), (1000, 768, 384, "f16"),
+                                       (257, 4096, 256, "f16")])
+def test_w4a4_gemm_exact(abi, L, N, K, out):
+    qa, qw, s_a, s_w = H.gemm_codes(L * 7 + N + K, L, N, K)
+    bias = np.random.default_rng(1).normal(0, 0.1, N).astype(np.float32) if out == "bf16" else None
+    Y, acc = run_gemm(abi, qa, qw, s_a, s_w, out, bias)
+    ref_acc = osg.int_gemm(qa, qw)
+    assert np.array_equal(acc, ref_acc), "integer accumulators differ"
+    H.assert_output_close(Y, osg.dequant(ref_acc, s_a, s_w, bias), out)
+
+
+@pytest.mark.parametrize("K", [18944, 65536])
+def test_w4a4_gemm_adversarial_exactness(abi, K):
+    """Integer exactness of the float32 tensor-core accumulation: all codes
+    +-7 (largest accumulators), alternating signs, and a large running sum
+    followed by increments of exactly 1 per 32-element MMA step (a truncating
+    accumulator would drop them)."""
+    L, N = 128, 256
+    half = K // 2
+    qa = np.zeros((L, K), np.int32)
+    qw = np.zeros((N, K), np.int32)
+    qa[0] = 7
+    qw[0] = 7
+    qw[1] = -7
+    qa[1] = np.where(np.arange(K) % 2 == 0, 7, -7)
+    qw[2] = np.where(np.arange(K) % 3 == 0, 7, -6)
+    ramp_a = np.zeros(K, np.int32)
+    ramp_a[:half] = 7
+    ramp_a[half::32] = 1
+    qa[2] = ramp_a
+    qw[3] = ramp_a
+    qw[4] = -ramp_a
+    rng = np.random.default_rng(K)
+    qa[3:] = rng.integers(-7, 8, (L - 3, K))
+    qw[5:] = rng.integers(-7, 8, (N - 5, K))
+    s_a = np.ones(L, np.float32)
+    s_w = np.ones(N, np.float32)
+    _, acc = run_gemm(abi, qa, qw, s_a, s_w, "f32")
+    ref = osg.int_gemm(qa, qw)
+    assert ref[0, 0] == 49 * K and ref[2, 3] == 49 * half + half // 32
+    assert np.array_equal(acc, ref)
+
+
+@pytest.mark.parametrize("g,L,C,zin,zout", [(4, 33, 64, "f16", "f32"), (8, 100, 256, "f16", "f16"),
+                                            (16, 1025, 512, "bf16", "f32"), (32, 7, 96, "f32", "f32"),
+                                            (64, 256, 512, "f16", "f32"), (128, 130, 4096, "f16", "f32"),
+                                            (128, 64, 4096, "bf16", "bf16")])
+def test_tac_apply(abi, g, L, C, zin, zout):
+    rng = np.random.default_rng(g * 1000 + L)
+    Z = rng.standard_normal((L, C)).astype(np.float32)
+    Z = Z.astype(np.float16).astype(np.float32) if zin == "f16" else (inputs.round_to_bf16(Z) if zin == "bf16" else Z)
+    tp = inputs.make_tac(rng, C, g, noise=0.05)
+    out = torch.empty(L, C, dtype=H.torch_dtype(zout), device="cuda")
+    abi.tac_apply(H.dev(Z, H.torch_dtype(zin)), H.dev(tp.M), H.dev(tp.d), g, out)
+    abi.check_status()
+    ref = otac.tac_apply(Z, tp.M, tp.d, g)
+    H.assert_tac_close(H.host(out), ref, zout)
+
+
+def _oracle_linear_from_codes(qa, s_a, qw, s_w, bias):
+    acc = osg.int_gemm(qa, qw)
+    return osg.dequant(acc, s_a, s_w, bias), acc
+
+
+def run_linear_case(abi, case, out_dtype=None, check_rows=None):
+    """sgat_prepare_weight + sgat_linear on the GPU against the oracle's
+    literal split / quantise / GEMM / scatter. With TAC, the TAC output is
+    compared within tolerance and the rest of the chain is teacher-forced on
+    the GPU's float32 TAC output (left in the workspace)."""
+    xf = case.xf
+    dt = H.torch_dtype(case.dtype)
+    out_dtype = out_dtype or case.dtype
+    L, K, N = case.L, case.K, case.N
+    W = H.dev(case.W, dt)
+    Wq = torch.empty(N, K // 2, dtype=torch.uint8, device="cuda")
+    s_w = torch.empty(N, dtype=torch.float32, device="cuda")
+    abi.sgat_prepare_weight(W, H.dev(xf.inv_a_w), xf.hb, Wq, s_w)
+    with_tac = case.tac is not None
+    ws = torch.empty(abi.sgat_linear_workspace_size(L, K, with_tac), dtype=torch.uint8, device="cuda")
+    Y = torch.empty(L, N, dtype=H.torch_dtype(out_dtype), device="cuda")
+    kw = {}
+    if with_tac:
+        kw = dict(tac_M=H.dev(case.tac.M), tac_d=H.dev(case.tac.d), tac_g=case.tac.g)
+    bias = H.dev(case.bias) if case.bias is not None else None
+    abi.sgat_linear(H.dev(case.X, dt), H.dev(case.mask), H.dev(xf.a_m), H.dev(xf.a_u), xf.hb, xf.d_sh,
+                    xf.d_m, xf.d_u, Wq, s_w, Y, ws, bias=bias, **kw)
+    abi.check_status()
+    qw, sw = osg.prepare_weight(case.W, xf.inv_a_w, xf.hb, 4)
+    assert np.array_equal(H.unpack(Wq), qw) and np.array_equal(s_w.cpu().numpy(), sw)
+    Xq_g, s_a_g, zt = H.workspace_views(ws, L, K, with_tac)
+    rows = np.arange(L) if check_rows is None else np.asarray(check_rows)
+    X_in = case.X
+    if with_tac:
+        z_gpu = zt.cpu().numpy()
+        ref_tac = otac.tac_apply(case.X[rows], case.tac.M, case.tac.d, case.tac.g)
+        H.assert_tac_close(z_gpu[rows], ref_tac, "f32")
+        X_in = z_gpu                      # teacher forcing on the GPU's TAC output
+    Y_ref, codes, s_a, acc = osg.sgat_linear(X_in[rows], case.mask[rows], xf.a_m, xf.a_u, xf.hb, xf.d_sh,
+                                             xf.d_m, xf.d_u, qw, sw, case.bias, 4)
+    assert np.array_equal(H.unpack(Xq_g)[rows], codes), "activation codes differ"
+    assert np.array_equal(s_a_g.cpu().numpy()[rows], s_a), "activation scales differ"
+    H.assert_output_close(H.host(Y)[rows], Y_ref, out_dtype)
+    return Y
+
+
+@pytest.mark.parametrize("gates", [True, False])
+def test_single_linear_full(abi, gates):
+    """Single SGAT linear, 256 x 512 -> 512, with and without gates, with
+    and without TAC (block 64)."""
+    case = inputs.single_linear(0, gates_on=gates)
+    run_linear_case(abi, case)
+    case.tac = None
+    run_linear_case(abi, case)
+
+
+def test_llada_attention_full(abi):
+    """LLaDA-8B attention projections at one step: QKV 1024 x 4096 -> 12288
+    and O 4096 -> 4096 with TAC (block 128), full size, every row."""
+    qkv, o = inputs.llada_attention(0)
+    run_linear_case(abi, qkv)
+    run_linear_case(abi, o)
+
+
+@pytest.mark.parametrize("L,K,N,dtype,tac_g,bias", [(1, 128, 32, "f16", None, False),
+                                                    (77, 512, 320, "bf16", 16, True),
+                                                    (129, 1024, 256, "f16", 128, False),
+                                                    (513, 3584, 512, "bf16", 128, True)])
+def test_sgat_linear_ragged(abi, L, K, N, dtype, tac_g, bias):
+    case = inputs.random_linear(L * 3 + K, L, K, N, dtype=dtype, tac_g=tac_g, bias=bias)
+    run_linear_case(abi, case)
+
+
+def test_empty_batch(abi):
+    """L = 0 is a valid no-op for every entry point."""
+    K, N = 512, 256
+    X = torch.empty(0, K, dtype=torch.float16, device="cuda")
+    Xq = torch.empty(0, K // 2, dtype=torch.uint8, device="cuda")
+    s = torch.empty(0, dtype=torch.float32, device="cuda")
+    abi.sgat_quantize_act(X, None, None, None, 512, K, 0, 0, Xq, s)
+    Wq = torch.zeros(N, K // 2, dtype=torch.uint8, device="cuda")
+    sw = torch.ones(N, dtype=torch.float32, device="cuda")
+    Y = torch.empty(0, N, dtype=torch.float16, device="cuda")
+    abi.w4a4_gemm(Xq, s, Wq, sw, Y)
+    abi.check_status()
