@@ -149,11 +149,18 @@ def profiled_traffic():
         return None
 
 
+def gpu_delay(torch):
+    """Keep the GPU busy ~50 us after the flush so that the host has enqueued
+    the start event and the timed launches before the GPU reaches them."""
+    torch.cuda._sleep(100000)
+
+
 def time_kernel(fn, flush, reps, torch):
     s = torch.cuda.current_stream()
     ts = []
     for _ in range(reps):
         flush()
+        gpu_delay(torch)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(s)
@@ -228,6 +235,7 @@ def run_ours(args):
     evs = []
     for _ in range(args.steps):
         flush()
+        gpu_delay(torch)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(s)
@@ -264,6 +272,7 @@ def run_ours(args):
     ets = []
     for _ in range(args.steps):
         flush()
+        gpu_delay(torch)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(s)

@@ -14,6 +14,8 @@
  *     message of the last error on the calling thread is returned by
  *     starq_last_error().
  *   - Matrices are row-major and dense (row stride = number of columns).
+ *   - L = 0 (no tokens) is a valid no-op; pointers to arrays with L rows may
+ *     then be NULL.
  *   - Packed int4: a [rows][K] code matrix is stored as uint8 [rows][K/2];
  *     code k lives in byte k/2, even k in the low nibble, odd k in the high
  *     nibble, each nibble in two's complement. Codes lie in [-7, 7].
@@ -154,7 +156,10 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  *   for no TAC. Wq/s_w come from sgat_prepare_weight. Other arguments as in
  *   the calls above. K % 128 == 0.
  *   workspace: device buffer of at least sgat_linear_workspace_size(L, K,
- *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller.
+ *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller. On return it
+ *   holds the intermediates, laid out as [packed codes Xq: L*K/2 bytes,
+ *   padded to 256][s_a: 4*L bytes, padded to 256][TAC output: float32 L*K,
+ *   only with TAC].
  */
 size_t sgat_linear_workspace_size(int L, int K, int with_tac);
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,

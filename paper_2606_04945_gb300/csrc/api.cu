@@ -74,12 +74,14 @@ int check_tac(int L, int C, int g, const float* M, const float* d) {
 
 int check_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
                const float* bias, int L, int N, int K, void* Y, int y_dtype) {
-    if (!Xq || !s_a || !Wq || !s_w || !Y) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL argument");
+    if (!Wq || !s_w) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Wq or s_w");
+    if (L > 0 && (!Xq || !s_a || !Y)) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Xq, s_a or Y");
     if (!dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "w4a4_gemm: unknown output dtype %d", y_dtype);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
     if (N < 32 || N % 32 != 0) return fail(STARQ_ERR_SHAPE, "N=%d: need N >= 32, N %% 32 == 0", N);
     if (K < 128 || K % 128 != 0 || K > 65536)
         return fail(STARQ_ERR_SHAPE, "K=%d: need 128 <= K <= 65536 and K %% 128 == 0", K);
+    if (L == 0) return STARQ_OK;  // nothing is read or written
     if (!aligned(Xq, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(s_w, 16) ||
         (bias && !aligned(bias, 16)) || !aligned(s_a, 4))
         return fail(STARQ_ERR_ALIGN, "w4a4_gemm: Xq, Wq, Y, s_w, bias must be 16-byte aligned");
@@ -130,12 +132,13 @@ int starq_check_status(void* stream) {
 int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
                       int bits, uint8_t* Xq, float* s_a, float* v_dbg, void* stream) {
-    if (!X || !Xq || !s_a) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, Xq or s_a");
+    if (L > 0 && (!X || !Xq || !s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, Xq or s_a");
     if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: unknown dtype %d", x_dtype);
     if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
     int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
     if (rc) return rc;
+    if (L == 0) return STARQ_OK;
     if (!aligned(X, 16) || !aligned(Xq, 8) || (v_dbg && !aligned(v_dbg, 16)))
         return fail(STARQ_ERR_ALIGN, "sgat_quantize_act: X (16 B), Xq (8 B), v_dbg (16 B) alignment");
     QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, v_dbg};
@@ -146,12 +149,13 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
 
 int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* inv_a_w, int hb,
                         int bits, uint8_t* Wq, float* s_w, void* stream) {
-    if (!W || !Wq || !s_w) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: NULL W, Wq or s_w");
+    if (N > 0 && (!W || !Wq || !s_w)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: NULL W, Wq or s_w");
     if (!dtype_ok(w_dtype)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: unknown dtype %d", w_dtype);
     if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
     if (N < 0) return fail(STARQ_ERR_SHAPE, "N=%d < 0", N);
     int rc = check_transform(K, hb, K, 0, 0, nullptr, inv_a_w);
     if (rc) return rc;
+    if (N == 0) return STARQ_OK;
     if (!aligned(W, 16) || !aligned(Wq, 8))
         return fail(STARQ_ERR_ALIGN, "sgat_prepare_weight: W (16 B), Wq (8 B) alignment");
     QuantArgs a{W, w_dtype, N, K, nullptr, nullptr, inv_a_w, hb, K, 0, 0, 7, 1.f / (float)hb,
@@ -177,10 +181,11 @@ int w4a4_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const floa
 
 int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d,
               void* out, int out_dtype, void* stream) {
-    if (!Z || !out) return fail(STARQ_ERR_ARG, "tac_apply: NULL Z or out");
+    if (L > 0 && (!Z || !out)) return fail(STARQ_ERR_ARG, "tac_apply: NULL Z or out");
     if (!dtype_ok(z_dtype) || !dtype_ok(out_dtype)) return fail(STARQ_ERR_ARG, "tac_apply: unknown dtype");
     int rc = check_tac(L, C, g, M, d);
     if (rc) return rc;
+    if (L == 0) return STARQ_OK;
     if (!aligned(Z, 16) || !aligned(out, 16)) return fail(STARQ_ERR_ALIGN, "tac_apply: Z, out alignment");
     TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype};
     cudaError_t e = launch_tac(a, static_cast<cudaStream_t>(stream));
@@ -200,13 +205,15 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const float* tac_M, const float* tac_d, int tac_g,
                 const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
                 void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
-    if (!X || !Wq || !s_w || !Y || !workspace) return fail(STARQ_ERR_ARG, "sgat_linear: NULL argument");
+    if (!Wq || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear: NULL Wq or s_w");
+    if (L > 0 && (!X || !Y || !workspace)) return fail(STARQ_ERR_ARG, "sgat_linear: NULL X, Y or workspace");
     if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear: unknown dtype");
     if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
     int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
     if (rc) return rc;
     if (tac_M && (rc = check_tac(L, K, tac_g, tac_M, tac_d))) return rc;
+    if (L == 0) return STARQ_OK;
     const size_t need = sgat_linear_workspace_size(L, K, tac_M != nullptr);
     if (workspace_bytes < need)
         return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu needed", workspace_bytes, need);
