@@ -168,6 +168,42 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
                 void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * sgat_linear_noalloc -- sgat_linear for callers that cannot allocate device
+ * memory. (The paper has no counterpart: this is a deployment convenience.)
+ *
+ * Some callers may not call cudaMalloc at all: a serving runtime that plans
+ * all device memory at start-up and owns the pool, a plugin or custom-op
+ * interface that passes an operator only its inputs and outputs, or a
+ * latency-critical path where cudaMalloc's implicit device synchronisation
+ * is not acceptable. They cannot supply sgat_linear's workspace. This entry
+ * point instead keeps the intermediates in a fixed scratch array of
+ * STARQ_NOALLOC_SCRATCH_BYTES bytes inside the library's device image
+ * (every GPU that loads the library holds it until the process exits), and
+ * allocates nothing: no cudaMalloc, no cudaFree, no allocating library call.
+ * The caller still passes all inputs and outputs; arguments and results are
+ * exactly those of sgat_linear without `workspace` / `workspace_bytes`.
+ *
+ *   - Limit: sgat_linear_workspace_size(L, K, tac_M != NULL) must not
+ *     exceed STARQ_NOALLOC_SCRATCH_BYTES (32 MiB: e.g. 1024 tokens x 4096
+ *     features with TAC need about 18.9 MB); larger calls return
+ *     STARQ_ERR_SHAPE with a message and launch nothing.
+ *   - The first call on each device looks up the scratch array's device
+ *     address (cudaGetSymbolAddress, with that device current) and caches
+ *     it; make that first call before any stream capture on that device.
+ *   - All calls on a device share the one array, which keeps the last call's
+ *     contents. Nothing in it needs to start at zero: every byte a call reads
+ *     back was written earlier in the same call. Calls whose work overlaps on
+ *     the GPU (concurrent streams, or several host threads) race on the
+ *     array and corrupt each other's results: serialise them.
+ */
+#define STARQ_NOALLOC_SCRATCH_BYTES (32u << 20)
+int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                        const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                        const float* tac_M, const float* tac_d, int tac_g,
+                        const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
+                        void* Y, int y_dtype, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -46,6 +46,9 @@ def _load():
     lib.sgat_linear_workspace_size.restype = ctypes.c_size_t
     lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
                                 u8p, f_p, f_p, i, i, vp, i, vp, ctypes.c_size_t, vp]
+    if hasattr(lib, "sgat_linear_noalloc"):
+        lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
+                                            u8p, f_p, f_p, i, i, vp, i, vp]
     return lib
 
 
@@ -125,3 +128,18 @@ def sgat_linear(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, workspace, bi
                            d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(s_w), _p(bias), N, bits,
                            _p(Y), dtype_code(Y), _p(workspace), workspace.numel() * workspace.element_size(),
                            _stream(stream)))
+
+
+NOALLOC_SCRATCH_BYTES = 32 << 20
+
+
+def sgat_linear_noalloc(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, bias=None,
+                        tac_M=None, tac_d=None, tac_g=0, bits=4, stream=None):
+    """sgat_linear without a workspace: the library's fixed device scratch
+    array holds the intermediates (see include/starq.h)."""
+    _contig(X, mask, a_m, a_u, Wq, s_w, Y, bias, tac_M, tac_d)
+    L, K = X.shape
+    N = Wq.shape[0]
+    _check(lib.sgat_linear_noalloc(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh,
+                                   d_m, d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(s_w), _p(bias), N,
+                                   bits, _p(Y), dtype_code(Y), _stream(stream)))

@@ -92,6 +92,8 @@ constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 }  // namespace
 
+int report_error(int code, const char* msg) { return fail(code, "%s", msg); }
+
 int num_sms() {
     static int cache[64] = {0};
     int dev = 0;

@@ -51,6 +51,7 @@ struct TacArgs {
 cudaError_t launch_tac(const TacArgs& a, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached per device)
+int report_error(int code, const char* msg);  // record msg for starq_last_error(), return code
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
