@@ -125,7 +125,7 @@ class ClockSampler:
 def kernel_source_hash():
     p = os.path.join(ROOT, "paper_2606_04945_gb300", "csrc")
     h = hashlib.sha256()
-    for f in ("w4a4_gemm.cu", "common.cuh"):
+    for f in ("w4a4_gemm.cu", "common.cuh"):  # the GEMM's sources
         with open(os.path.join(p, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -212,17 +212,18 @@ def run_ours(args):
 
     # per-kernel durations (each kernel alone, L2 flushed before every launch)
     Xq = torch.empty(L, K // 2, dtype=torch.uint8, device="cuda")
+    Xe = torch.empty(L, K, dtype=torch.uint8, device="cuda")
     s_a = torch.empty(L, dtype=torch.float32, device="cuda")
     zt = torch.empty(L, K, dtype=torch.float32, device="cuda")
     q, o = step.qkv, step.o
     reps = 20
     t_quant_x = time_kernel(lambda: abi.sgat_quantize_act(step.X, step.mask, q.a_m, q.a_u, q.hb, q.d_sh, q.d_m,
-                                                          q.d_u, Xq, s_a), flush, reps, torch)
-    t_gemm_qkv = time_kernel(lambda: abi.w4a4_gemm(Xq, s_a, q.Wq, q.s_w, step.Y_qkv), flush, reps, torch)
+                                                          q.d_u, Xq, s_a, Xe=Xe), flush, reps, torch)
+    t_gemm_qkv = time_kernel(lambda: abi.w4a4_gemm(None, s_a, q.Wq, q.s_w, step.Y_qkv, Xe=Xe), flush, reps, torch)
     t_tac = time_kernel(lambda: abi.tac_apply(step.Z, o.tac_M, o.tac_d, o.tac_g, zt), flush, reps, torch)
     t_quant_z = time_kernel(lambda: abi.sgat_quantize_act(zt, step.mask, o.a_m, o.a_u, o.hb, o.d_sh, o.d_m,
-                                                          o.d_u, Xq, s_a), flush, reps, torch)
-    t_gemm_o = time_kernel(lambda: abi.w4a4_gemm(Xq, s_a, o.Wq, o.s_w, step.Y_o), flush, reps, torch)
+                                                          o.d_u, Xq, s_a, Xe=Xe), flush, reps, torch)
+    t_gemm_o = time_kernel(lambda: abi.w4a4_gemm(None, s_a, o.Wq, o.s_w, step.Y_o, Xe=Xe), flush, reps, torch)
     abi.check_status()
 
     # timed region: exactly `steps` steps, device-timed per step
@@ -296,12 +297,12 @@ def run_ours(args):
     achieved = gemm_ops / (gemm_ms * 1e-3) / 1e12
     peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]) * FP8_PER_BF16
     hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
-    quant_x_bytes = L * K * 2 + L * K // 2 + 4 * L
-    quant_z_bytes = L * K * 4 + L * K // 2 + 4 * L
+    quant_x_bytes = L * K * 2 + L * K // 2 + L * K + 4 * L     # X in; packed + E4M3 codes, scales out
+    quant_z_bytes = L * K * 4 + L * K // 2 + L * K + 4 * L
     tac_bytes = L * K * 2 + L * K * 4 + K * o.tac_g * 4 + K * 4
     traffic = profiled_traffic()
-    gemm_bytes = [L * K // 2 + q.N * K // 2 + 2 * L * q.N + 4 * (L + q.N),
-                  L * K // 2 + o.N * K // 2 + 2 * L * o.N + 4 * (L + o.N)]
+    gemm_bytes = [L * K + q.N * K // 2 + 2 * L * q.N + 4 * (L + q.N),    # E4M3 codes, packed weights, fp16 out
+                  L * K + o.N * K // 2 + 2 * L * o.N + 4 * (L + o.N)]
 
     if rank != 0:
         return None
@@ -317,7 +318,7 @@ def run_ours(args):
         "config": config_dict(graph),
         "tokens_per_s": round(tokens_s, 1),
         "roofline": {
-            "bound": "tensor", "kernel": "w4a4_gemm_kernel (QKV + O launches)",
+            "bound": "tensor", "kernel": "w4a4_gemm_pair_kernel (QKV + O launches)",
             "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
             "frac": round(achieved / peak, 4), "traffic": traffic,
             "peak_source": f"{peak_src} bf16 dense burst x {FP8_PER_BF16} (fp8 kind::f8f6f4 path; "

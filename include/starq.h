@@ -84,13 +84,15 @@ int starq_check_status(void* stream);
  *   bits    must be 4.
  *   Xq      [L][K/2] packed int4 codes out, 8-byte aligned.
  *   s_a     [L] float32 per-token scales out (0 for an all-zero row).
+ *   Xe      [L][K] the same codes as E4M3 bytes out (the form w4a4_gemm
+ *           streams by TMA), 16-byte aligned, or NULL.
  *   v_dbg   [L][K] float32 transformed activations out (before rounding),
  *           16-byte aligned, or NULL.
  * Shapes: L >= 0, 16 <= K <= 20480, K % 16 == 0.
  */
 int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                      int bits, uint8_t* Xq, float* s_a, float* v_dbg, void* stream);
+                      int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg, void* stream);
 
 /*
  * sgat_prepare_weight -- the unified static weight transform, quantised once
@@ -118,15 +120,19 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
  *               (float32 products in that order, then one rounding).
  *
  *   Xq [L][K/2], Wq [N][K/2] packed int4, 16-byte aligned.
+ *   Xe [L][K] the activation codes as E4M3 bytes (sgat_quantize_act's Xe
+ *      output), 16-byte aligned, or NULL. When given, Xq may be NULL and the
+ *      kernel streams Xe by TMA to CTA pairs (tcgen05 cta_group::2) that
+ *      convert only the weights; otherwise it converts both operands.
  *   s_a [L], s_w [N] float32; bias [N] float32 or NULL.
  *   Y  [L][N] out, y_dtype F16, BF16 or F32, 16-byte aligned.
  *   acc_dbg [L][N] int32 out (the exact accumulators) or NULL.
  * Shapes: L >= 0, N >= 32 with N % 32 == 0, K >= 128 with K % 128 == 0,
  * K <= 65536 (so |acc| <= 49 K < 2^22).
  */
-int w4a4_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
-              const float* bias, int L, int N, int K, void* Y, int y_dtype, int32_t* acc_dbg,
-              void* stream);
+int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq,
+              const float* s_w, const float* bias, int L, int N, int K, void* Y, int y_dtype,
+              int32_t* acc_dbg, void* stream);
 
 /*
  * tac_apply -- block-wise affine compensation of the quantised attention
@@ -158,8 +164,8 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  *   workspace: device buffer of at least sgat_linear_workspace_size(L, K,
  *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller. On return it
  *   holds the intermediates, laid out as [packed codes Xq: L*K/2 bytes,
- *   padded to 256][s_a: 4*L bytes, padded to 256][TAC output: float32 L*K,
- *   only with TAC].
+ *   padded to 256][s_a: 4*L bytes, padded to 256][E4M3 codes Xe: L*K bytes,
+ *   padded to 256][TAC output: float32 L*K, only with TAC].
  */
 size_t sgat_linear_workspace_size(int L, int K, int with_tac);
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,

@@ -38,9 +38,9 @@ def _load():
     lib.starq_version.restype = i
     lib.starq_last_error.restype = ctypes.c_char_p
     lib.starq_check_status.argtypes = [vp]
-    lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, i, u8p, f_p, f_p, vp]
+    lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, i, u8p, f_p, u8p, f_p, vp]
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
-    lib.w4a4_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, i, vp]
     lib.sgat_linear_workspace_size.argtypes = [i, i, i]
     lib.sgat_linear_workspace_size.restype = ctypes.c_size_t
@@ -84,12 +84,13 @@ def check_status(stream=None):
     _check(lib.starq_check_status(_stream(stream)))
 
 
-def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, bits=4, v_dbg=None,
+def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, bits=4, Xe=None, v_dbg=None,
                       stream=None):
-    _contig(X, mask, a_m, a_u, Xq, s_a, v_dbg)
+    _contig(X, mask, a_m, a_u, Xq, s_a, Xe, v_dbg)
     L, K = X.shape
     _check(lib.sgat_quantize_act(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb,
-                                 d_sh, d_m, d_u, bits, _p(Xq), _p(s_a), _p(v_dbg), _stream(stream)))
+                                 d_sh, d_m, d_u, bits, _p(Xq), _p(s_a), _p(Xe), _p(v_dbg),
+                                 _stream(stream)))
 
 
 def sgat_prepare_weight(W, inv_a_w, hb, Wq, s_w, bits=4, stream=None):
@@ -99,12 +100,14 @@ def sgat_prepare_weight(W, inv_a_w, hb, Wq, s_w, bits=4, stream=None):
                                    _p(Wq), _p(s_w), _stream(stream)))
 
 
-def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, stream=None):
-    _contig(Xq, s_a, Wq, s_w, Y, bias, acc_dbg)
-    L = Xq.shape[0]
+def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, stream=None):
+    """Xq: packed int4 codes [L][K/2] (may be None when Xe is given);
+    Xe: the same codes as E4M3 bytes [L][K] (selects the TMA CTA-pair kernel)."""
+    _contig(Xq, Xe, s_a, Wq, s_w, Y, bias, acc_dbg)
+    L = Y.shape[0]
     N = Wq.shape[0]
-    K = 2 * Xq.shape[1]
-    _check(lib.w4a4_gemm(_p(Xq), _p(s_a), _p(Wq), _p(s_w), _p(bias), L, N, K, _p(Y),
+    K = 2 * Wq.shape[1]
+    _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(s_w), _p(bias), L, N, K, _p(Y),
                          dtype_code(Y), _p(acc_dbg), _stream(stream)))
 
 

@@ -72,19 +72,19 @@ int check_tac(int L, int C, int g, const float* M, const float* d) {
     return STARQ_OK;
 }
 
-int check_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
+int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq, const float* s_w,
                const float* bias, int L, int N, int K, void* Y, int y_dtype) {
     if (!Wq || !s_w) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Wq or s_w");
-    if (L > 0 && (!Xq || !s_a || !Y)) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Xq, s_a or Y");
+    if (L > 0 && ((!Xq && !Xe) || !s_a || !Y)) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Xq/Xe, s_a or Y");
     if (!dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "w4a4_gemm: unknown output dtype %d", y_dtype);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
     if (N < 32 || N % 32 != 0) return fail(STARQ_ERR_SHAPE, "N=%d: need N >= 32, N %% 32 == 0", N);
     if (K < 128 || K % 128 != 0 || K > 65536)
         return fail(STARQ_ERR_SHAPE, "K=%d: need 128 <= K <= 65536 and K %% 128 == 0", K);
     if (L == 0) return STARQ_OK;  // nothing is read or written
-    if (!aligned(Xq, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(s_w, 16) ||
+    if (!aligned(Xq, 16) || !aligned(Xe, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(s_w, 16) ||
         (bias && !aligned(bias, 16)) || !aligned(s_a, 4))
-        return fail(STARQ_ERR_ALIGN, "w4a4_gemm: Xq, Wq, Y, s_w, bias must be 16-byte aligned");
+        return fail(STARQ_ERR_ALIGN, "w4a4_gemm: Xq, Xe, Wq, Y, s_w, bias must be 16-byte aligned");
     return STARQ_OK;
 }
 
@@ -133,7 +133,7 @@ int starq_check_status(void* stream) {
 
 int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                      int bits, uint8_t* Xq, float* s_a, float* v_dbg, void* stream) {
+                      int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg, void* stream) {
     if (L > 0 && (!X || !Xq || !s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, Xq or s_a");
     if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: unknown dtype %d", x_dtype);
     if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
@@ -141,9 +141,9 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
     int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
     if (rc) return rc;
     if (L == 0) return STARQ_OK;
-    if (!aligned(X, 16) || !aligned(Xq, 8) || (v_dbg && !aligned(v_dbg, 16)))
-        return fail(STARQ_ERR_ALIGN, "sgat_quantize_act: X (16 B), Xq (8 B), v_dbg (16 B) alignment");
-    QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, v_dbg};
+    if (!aligned(X, 16) || !aligned(Xq, 8) || (v_dbg && !aligned(v_dbg, 16)) || (Xe && !aligned(Xe, 16)))
+        return fail(STARQ_ERR_ALIGN, "sgat_quantize_act: X (16 B), Xq (8 B), Xe (16 B), v_dbg (16 B) alignment");
+    QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, v_dbg, Xe};
     cudaError_t e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "sgat_quantize_act launch");
     return STARQ_OK;
@@ -167,15 +167,15 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
     return STARQ_OK;
 }
 
-int w4a4_gemm(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
-              const float* bias, int L, int N, int K, void* Y, int y_dtype, int32_t* acc_dbg,
-              void* stream) {
-    int rc = check_gemm(Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
+int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq,
+              const float* s_w, const float* bias, int L, int N, int K, void* Y, int y_dtype,
+              int32_t* acc_dbg, void* stream) {
+    int rc = check_gemm(Xq, Xe, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     if (acc_dbg && !aligned(acc_dbg, 16)) return fail(STARQ_ERR_ALIGN, "acc_dbg must be 16-byte aligned");
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
-    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st};
+    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe};
     cudaError_t e = launch_w4a4_gemm(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm launch");
     return STARQ_OK;
@@ -197,7 +197,7 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
 
 size_t sgat_linear_workspace_size(int L, int K, int with_tac) {
     if (L < 0 || K < 0) return 0;
-    size_t n = align256((size_t)L * K / 2) + align256((size_t)L * 4);
+    size_t n = align256((size_t)L * K / 2) + align256((size_t)L * 4) + align256((size_t)L * K);
     if (with_tac) n += align256((size_t)L * K * 4);
     return n;
 }
@@ -223,9 +223,9 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     uint8_t* ws = static_cast<uint8_t*>(workspace);
     uint8_t* Xq = ws;
     float* s_a = reinterpret_cast<float*>(ws + align256((size_t)L * K / 2));
-    float* zt = tac_M ? reinterpret_cast<float*>(ws + align256((size_t)L * K / 2) + align256((size_t)L * 4))
-                      : nullptr;
-    rc = check_gemm(Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
+    uint8_t* Xe = ws + align256((size_t)L * K / 2) + align256((size_t)L * 4);
+    float* zt = tac_M ? reinterpret_cast<float*>(Xe + align256((size_t)L * K)) : nullptr;
+    rc = check_gemm(Xq, Xe, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
@@ -239,9 +239,9 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
         qin = zt;
         qin_dtype = STARQ_F32;
     }
-    QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr};
+    QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");
-    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st};
+    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe};
     if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: gemm launch");
     return STARQ_OK;
 }

@@ -33,6 +33,7 @@ struct QuantArgs {
     int hb; int d_sh; int d_m; int d_u;
     int qmax; float post_scale;
     uint8_t* Xq; float* s; float* v_dbg;
+    uint8_t* Xe = nullptr;   // optional E4M3 byte copy of the codes [L][K]
 };
 cudaError_t launch_sgat_quant(const QuantArgs& a, cudaStream_t stream);
 
@@ -41,6 +42,7 @@ struct GemmArgs {
     const float* bias; int L; int N; int K;
     void* Y; int y_dtype; int32_t* acc_dbg;
     unsigned* status;
+    const uint8_t* Xe = nullptr;   // optional E4M3 bytes of the codes [L][K]
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
 
@@ -212,27 +214,105 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
     return d;
 }
 
+// ---- clusters and CTA pairs ----------------------------------------------
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// shared::cluster address of the variable at `addr` (a shared::cta address)
+// in the CTA of the cluster with rank `rank`.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+    uint32_t d;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(addr), "r"(rank));
+    return d;
+}
+// Arrive on an mbarrier given by its shared::cluster address (any CTA of
+// the cluster), with release semantics at cluster scope.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];"
+                 :: "r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
+                 :: "r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+                 ::: "memory");
+}
+// 2-D TMA tile load global -> this CTA's shared memory, completion counted
+// on `bar` (bytes).
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int x, int y,
+                                            uint32_t bar) {
+    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+                 " [%0], [%1, {%2, %3}], [%4];"
+                 :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar) : "memory");
+}
+// Same, with the tile (and the completion on `bar`) delivered to the same
+// shared-memory offsets in every CTA of `cta_mask`.
+__device__ __forceinline__ void tma_load_2d_multicast(uint32_t dst, const void* tmap, int x, int y,
+                                                      uint32_t bar, uint16_t cta_mask) {
+    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+                 " [%0], [%1, {%2, %3}], [%4], %5;"
+                 :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar), "h"(cta_mask) : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;"
+                 :: "r"(dst_smem), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;"
+                 :: "r"(taddr), "r"(ncols) : "memory");
+}
+// D[tmem of both CTAs] (+)= A[smem, M rows split over the pair] *
+// B[smem, N rows split over the pair]^T, E4M3 -> F32; issued by the leader.
+__device__ __forceinline__ void mma_f8f6f4_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                                uint32_t idesc, uint32_t accumulate) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}"
+                 :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+                 : "memory");
+}
+// Arrive once on the barrier at shared offset `bar` in every CTA of
+// `cta_mask` when the issuing thread's tcgen05 operations have completed.
+__device__ __forceinline__ void tc_commit_pair_multicast(uint32_t bar, uint16_t cta_mask) {
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+                 " [%0], %1;" :: "r"(bar), "h"(cta_mask) : "memory");
+}
+
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
 // Eight int4 codes (two's complement nibbles, code k in bits 4k..4k+3) to
 // eight E4M3 bytes (byte k = code k). Every integer in [-8, 7] is exact in
-// E4M3. Two byte-permutes look the magnitude up in 8-entry tables (the
-// selector's top bit replicates a zero sign for the other half of the codes),
-// a third spreads the nibble sign bits to the byte sign bits.
+// E4M3. Per four codes three byte-permutes do the work: one looks the code
+// up in the table of non-negative values (a negative code's selector has its
+// top bit set, which replicates the zero sign bit of the table byte: 0x00),
+// one looks the low three bits up in the table of negative values (selector
+// top bits flipped, so non-negative codes yield 0xFF), and one replicates
+// each code's sign bit into a byte mask that picks between the two.
 __device__ __forceinline__ void int4x8_to_e4m3x8(uint32_t x, uint32_t& lo, uint32_t& hi) {
-    // positive codes 0..7: 0x00 0x38 0x40 0x44 | 0x48 0x4A 0x4C 0x4E
+    // codes 0..7: 0x00 0x38 0x40 0x44 | 0x48 0x4A 0x4C 0x4E
     constexpr uint32_t P0 = 0x44403800u, P1 = 0x4E4C4A48u;
-    // negative codes -8..-1 indexed by the low three bits (magnitude bytes,
-    // sign added separately): 8 7 6 5 | 4 3 2 1
-    constexpr uint32_t N0 = 0x4A4C4E50u, N1 = 0x38404448u;
+    // codes -8..-1 by their low three bits: 0xD0 0xCE 0xCC 0xCA | 0xC8 0xC4 0xC0 0xB8
+    constexpr uint32_t N0 = 0xCACCCED0u, N1 = 0xB8C0C4C8u;
+    const uint32_t xs = x << 4;                 // low-nibble sign bits -> byte msb
     const uint32_t xn = x ^ 0x88888888u;
     const uint32_t xh = x >> 16, xnh = xn >> 16;
-    const uint32_t mlo = prmt(P0, P1, x) | prmt(N0, N1, xn);
-    const uint32_t mhi = prmt(P0, P1, xh) | prmt(N0, N1, xnh);
-    const uint32_t ylo = prmt(x, 0, 0x1100u);   // bytes: x0 x0 x1 x1
-    const uint32_t yhi = prmt(x, 0, 0x3322u);   // bytes: x2 x2 x3 x3
-    const uint32_t slo = ((ylo << 4) & 0x00800080u) | (ylo & 0x80008000u);
-    const uint32_t shi = ((yhi << 4) & 0x00800080u) | (yhi & 0x80008000u);
-    lo = mlo | slo;
-    hi = mhi | shi;
+    // sign masks: byte k = 0xFF iff code k < 0 (sign of code 2j in xs byte j,
+    // of code 2j+1 in x byte j)
+    const uint32_t mlo = prmt(xs, x, 0xD9C8u);
+    const uint32_t mhi = prmt(xs, x, 0xFBEAu);
+    lo = prmt(P0, P1, x) | (prmt(N0, N1, xn) & mlo);
+    hi = prmt(P0, P1, xh) | (prmt(N0, N1, xnh) & mhi);
 }
 
 }  // namespace starq

@@ -1,38 +1,42 @@
 // SGAT activation transform + per-row symmetric int4 quantisation.
 //
-// One CTA per row (a token for Q_a, an output channel for Q_w). Each thread
-// owns 16 consecutive elements per pass of 16 * blockDim elements; rows
-// longer than 4096 take up to five passes, all held in registers so the row
-// is read from HBM once.
-//
-// Per row (Sec. 3.2 Eq. 11 with P = diag(a_s) H_hb, Sec. 3.1 Eq. 2):
+// Per row (a token for Q_a, an output channel for Q_w); Sec. 3.2 Eq. 11 with
+// P = diag(a_s) H_hb, Sec. 3.1 Eq. 2:
 //   v = fl32(x * a_s)                      state picked by the row's mask bit
 //   v = v H_hb                             fast Walsh-Hadamard transform
 //   v = v * gate_s                          binary subspace gate (Eq. 9)
 //   v = fl32(v * post_scale)               1/hb on the weight side (Eq. 12)
-//   amax = max |v|; s = amax / qmax; r = qmax / amax; q = clamp(rne(v*r))
-//
-// The transform's butterfly network is the one of the fast Walsh-Hadamard
+//   amax = max |v|; s = amax / qmax; r = qmax / amax; q = rne(v * r)
+// The transform is the butterfly network of the fast Walsh-Hadamard
 // transform in stage order h = 1, 2, 4, ..., hb/2, each butterfly
-// (a, b) -> (a + b, a - b) in float32 round-to-nearest. Stages h <= 8 run
-// inside a thread, 16 <= h <= 256 across lanes by shuffles, h >= 512 across
-// warps through shared memory. Every float operation is an explicit
-// round-to-nearest intrinsic so that no multiply is contracted into an add.
+// (a, b) -> (a + b, a - b) in float32 round-to-nearest; every float operation
+// is an explicit round-to-nearest intrinsic, so nothing is contracted into an
+// FMA and the values match the reference network bit for bit. With qmax = 7
+// no clamp is needed: |fl(v * r)| <= 7 (1 + 2^-24)^2 < 7.5.
+//
+// Work split: a warp owns a chunk of C = 32 E consecutive elements of a row
+// (E = hb / 32, or E = 16 with several Hadamard blocks per chunk when
+// hb < 512). In layout A lane l holds elements E l .. E l + E - 1, so stages
+// h < E are butterflies between registers of one thread. One transpose
+// through shared memory (layout B: lane l holds elements l + 32 i) makes the
+// stages h >= 32 register-local too; a transpose back gives each lane E
+// contiguous values again for gating, scaling and packing.
+//
+// Rows of one chunk (K == C) take one warp each, four rows per CTA; longer
+// rows take a CTA of up to 8 warps, each keeping up to NC chunks in
+// registers, and reduce amax across warps through shared memory.
 #include "common.cuh"
 
 namespace starq {
 namespace {
 
-constexpr int EPT = 16;          // elements per thread per pass
-constexpr int MAX_THREADS = 256; // threads per CTA for rows >= 4096
-constexpr int MAX_PASSES = 5;    // rows up to 5 * 4096 = 20480 elements
-
 template <typename T> struct In;
 template <> struct In<__half> {
-    static __device__ __forceinline__ void load16(const __half* p, float (&v)[EPT]) {
+    template <int E>
+    static __device__ __forceinline__ void load(const __half* p, float (&v)[E]) {
         const uint4* q = reinterpret_cast<const uint4*>(p);
         #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < E / 8; ++u) {
             uint4 w = __ldg(q + u);
             const __half2* h = reinterpret_cast<const __half2*>(&w);
             #pragma unroll
@@ -45,10 +49,11 @@ template <> struct In<__half> {
     }
 };
 template <> struct In<__nv_bfloat16> {
-    static __device__ __forceinline__ void load16(const __nv_bfloat16* p, float (&v)[EPT]) {
+    template <int E>
+    static __device__ __forceinline__ void load(const __nv_bfloat16* p, float (&v)[E]) {
         const uint4* q = reinterpret_cast<const uint4*>(p);
         #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < E / 8; ++u) {
             uint4 w = __ldg(q + u);
             const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&w);
             #pragma unroll
@@ -61,10 +66,11 @@ template <> struct In<__nv_bfloat16> {
     }
 };
 template <> struct In<float> {
-    static __device__ __forceinline__ void load16(const float* p, float (&v)[EPT]) {
+    template <int E>
+    static __device__ __forceinline__ void load(const float* p, float (&v)[E]) {
         const float4* q = reinterpret_cast<const float4*>(p);
         #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < E / 4; ++u) {
             float4 w = __ldg(q + u);
             v[4 * u] = w.x; v[4 * u + 1] = w.y; v[4 * u + 2] = w.z; v[4 * u + 3] = w.w;
         }
@@ -77,148 +83,243 @@ __device__ __forceinline__ void butterfly(float& lo, float& hi) {
     hi = __fsub_rn(a, b);
 }
 
-template <int PASSES, typename Tin>
-__global__ void __launch_bounds__(MAX_THREADS)
-sgat_quant_kernel(QuantArgs a) {
-    __shared__ float xchg[EPT * MAX_THREADS];   // cross-warp butterfly exchange
-    __shared__ float red[MAX_THREADS / 32];
-    const int T = blockDim.x;
-    const int t = threadIdx.x;
-    const int lane = t & 31;
-    const int row = blockIdx.x;
+// Butterflies between registers i and i + s for every i with (i & s) == 0,
+// for s = s_lo, 2 s_lo, ... while s < s_end.
+template <int E>
+__device__ __forceinline__ void inlane_stages(float (&v)[E], int s_lo, int s_end) {
+    #pragma unroll
+    for (int s = 1; s < E; s <<= 1) {
+        if (s >= s_lo && s < s_end) {
+            #pragma unroll
+            for (int i = 0; i < E; ++i)
+                if ((i & s) == 0) butterfly(v[i], v[i + s]);
+        }
+    }
+}
+
+// Shared-buffer index of chunk element e: one padding float after every E
+// elements. Layout A (lane stride E + 1, odd) and layout B (consecutive
+// lanes, consecutive words) are then both free of bank conflicts, and every
+// access is a per-lane base plus a compile-time offset.
+template <int E>
+__device__ __forceinline__ int pad_idx(int e) { return e + e / E; }
+
+// Full transform of one chunk held in layout A; `buf` is this warp's
+// 32 E-float shared buffer.
+template <int E>
+__device__ __forceinline__ void chunk_fwht(float (&v)[E], int hb, int lane, float* buf) {
+    inlane_stages<E>(v, 1, hb < E ? hb : E);                  // h = 1 .. min(hb, E)/2
+    if (hb <= E) return;
+    if (E < 32) {                                            // h = E .. 16 across lanes
+        #pragma unroll
+        for (int h = E; h < 32; h <<= 1) {
+            if (h < hb) {
+                const int m = h / E;
+                const float sgn = (lane & m) ? -1.f : 1.f;
+                #pragma unroll
+                for (int i = 0; i < E; ++i) {
+                    const float o = __shfl_xor_sync(0xffffffffu, v[i], m);
+                    // lower lane: v + o; upper lane: o - v (the product by -1 is exact)
+                    v[i] = __fmaf_rn(sgn, v[i], o);
+                }
+            }
+        }
+    }
+    if (hb <= 32) return;
+    // layout A -> B
+    float* a_base = buf + (E + 1) * lane;      // = buf + pad_idx(E * lane)
+    #pragma unroll
+    for (int i = 0; i < E; ++i) a_base[i] = v[i];
+    __syncwarp();
+    #pragma unroll
+    for (int i = 0; i < E; ++i) v[i] = buf[pad_idx<E>(lane + 32 * i)];
+    // stages h = max(E, 32) .. hb/2: register distance h / 32 in layout B
+    inlane_stages<E>(v, (E > 32 ? E : 32) / 32, hb / 32);
+    __syncwarp();
+    #pragma unroll
+    for (int i = 0; i < E; ++i) buf[pad_idx<E>(lane + 32 * i)] = v[i];
+    __syncwarp();
+    #pragma unroll
+    for (int i = 0; i < E; ++i) v[i] = a_base[i];
+    __syncwarp();
+}
+
+// Eight codes (int, |q| <= 7) -> packed nibbles, code k in bits 4k..4k+3.
+__device__ __forceinline__ uint32_t pack8(const int* q) {
+    uint32_t w = 0;
+    #pragma unroll
+    for (int k = 0; k < 8; ++k) w |= (uint32_t)(q[k] & 0xF) << (4 * k);
+    return w;
+}
+
+template <int E, int NC, typename Tin>
+__global__ void __launch_bounds__(256)
+sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
+    extern __shared__ float qsm[];
+    constexpr int C = 32 * E;
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int wr = warp % warps_per_row;                 // warp index within its row
+    const int row = blockIdx.x * rows_per_cta + warp / warps_per_row;
+    float* buf = qsm + warp * (C + 32);
+    float* red = qsm + (blockDim.x >> 5) * (C + 32);     // [warps] partial amax
+    const bool row_ok = row < a.L;
     const int K = a.K;
-    const int hb = a.hb;
-    const Tin* X = static_cast<const Tin*>(a.X) + (size_t)row * K;
-    const bool masked = a.mask != nullptr && a.mask[row] != 0;
+    const int nchunks = (K + C - 1) / C;   // a partial last chunk only when hb < 512
+
+    const bool masked = row_ok && a.mask != nullptr && a.mask[row] != 0;
     const float* sm = masked ? a.a_m : a.a_u;
     // Active coordinates of the row's state (Eq. 9): masked rows keep
     // [0, d_sh + d_m), unmasked rows keep [0, d_sh) and [d_sh + d_m, K).
     const int own_lo = masked ? a.d_sh : a.d_sh + a.d_m;
-    const int own_hi = masked ? a.d_sh + a.d_m : a.K;
+    const int own_hi = masked ? a.d_sh + a.d_m : K;
+    const Tin* X = static_cast<const Tin*>(a.X) + (size_t)(row_ok ? row : 0) * K;
 
-    float v[PASSES][EPT];
+    float v[NC][E];
     float amax = 0.f;
     #pragma unroll
-    for (int p = 0; p < PASSES; ++p) {
-        const int e0 = p * EPT * T + EPT * t;
-        const bool live = e0 < K;
+    for (int j = 0; j < NC; ++j) {
+        const int c = wr + j * warps_per_row;
+        const int lo = c * C + E * lane;                 // first element of this lane
+        // lanes lie wholly inside or outside the row: E | K when hb < 512
+        const bool live = c < nchunks && row_ok && lo < K;
         if (live) {
-            In<Tin>::load16(X + e0, v[p]);
+            In<Tin>::template load<E>(X + lo, v[j]);
             if (sm != nullptr) {
-                const float4* s4 = reinterpret_cast<const float4*>(sm + e0);
+                const float4* s4 = reinterpret_cast<const float4*>(sm + lo);
                 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
+                for (int u = 0; u < E / 4; ++u) {
                     const float4 w = __ldg(s4 + u);
-                    v[p][4 * u] = __fmul_rn(v[p][4 * u], w.x);
-                    v[p][4 * u + 1] = __fmul_rn(v[p][4 * u + 1], w.y);
-                    v[p][4 * u + 2] = __fmul_rn(v[p][4 * u + 2], w.z);
-                    v[p][4 * u + 3] = __fmul_rn(v[p][4 * u + 3], w.w);
+                    v[j][4 * u] = __fmul_rn(v[j][4 * u], w.x);
+                    v[j][4 * u + 1] = __fmul_rn(v[j][4 * u + 1], w.y);
+                    v[j][4 * u + 2] = __fmul_rn(v[j][4 * u + 2], w.z);
+                    v[j][4 * u + 3] = __fmul_rn(v[j][4 * u + 3], w.w);
                 }
             }
         } else {
             #pragma unroll
-            for (int i = 0; i < EPT; ++i) v[p][i] = 0.f;
+            for (int i = 0; i < E; ++i) v[j][i] = 0.f;
         }
-        // stages h = 1, 2, 4, 8 inside the thread
-        #pragma unroll
-        for (int h = 1; h < EPT; h <<= 1) {
-            if (h < hb) {
-                #pragma unroll
-                for (int i = 0; i < EPT; ++i)
-                    if ((i & h) == 0) butterfly(v[p][i], v[p][i + h]);
-            }
-        }
-        // stages h = 16 .. 256 across lanes: partner lane = lane ^ (h / 16)
-        #pragma unroll
-        for (int m = 1; m < 32; m <<= 1) {
-            if (EPT * m < hb) {
-                const bool upper = (lane & m) != 0;
-                #pragma unroll
-                for (int i = 0; i < EPT; ++i) {
-                    const float o = __shfl_xor_sync(0xffffffffu, v[p][i], m);
-                    v[p][i] = upper ? __fsub_rn(o, v[p][i]) : __fadd_rn(v[p][i], o);
-                }
-            }
-        }
-        // stages h = 512 .. 2048 across warps: partner thread = t ^ (h / 16)
-        for (int m = 32; EPT * m < hb; m <<= 1) {
+        if (c < nchunks) chunk_fwht<E>(v[j], a.hb, lane, buf);   // warp-uniform condition
+        // gate: whole-lane decisions first, per element only where a lane
+        // straddles a subspace boundary
+        const bool all_keep = (lo + E <= a.d_sh) || (lo >= own_lo && lo + E <= own_hi);
+        if (!all_keep) {
             #pragma unroll
-            for (int i = 0; i < EPT; ++i) xchg[i * T + t] = v[p][i];
-            __syncthreads();
-            const bool upper = (t & m) != 0;
-            #pragma unroll
-            for (int i = 0; i < EPT; ++i) {
-                const float o = xchg[i * T + (t ^ m)];
-                v[p][i] = upper ? __fsub_rn(o, v[p][i]) : __fadd_rn(v[p][i], o);
+            for (int i = 0; i < E; ++i) {
+                const int e = lo + i;
+                if (!(e < a.d_sh || (e >= own_lo && e < own_hi))) v[j][i] = 0.f;
             }
-            __syncthreads();
         }
-        // gate, post-scale, optional debug copy, running amax
+        if (a.post_scale != 1.f) {
+            #pragma unroll
+            for (int i = 0; i < E; ++i) v[j][i] = __fmul_rn(v[j][i], a.post_scale);
+        }
         #pragma unroll
-        for (int i = 0; i < EPT; ++i) {
-            const int e = e0 + i;
-            const bool keep = live && (e < a.d_sh || (e >= own_lo && e < own_hi));
-            float w = keep ? v[p][i] : 0.f;
-            if (a.post_scale != 1.f) w = __fmul_rn(w, a.post_scale);
-            v[p][i] = w;
-            amax = fmaxf(amax, fabsf(w));
-        }
+        for (int i = 0; i < E; ++i) amax = fmaxf(amax, fabsf(v[j][i]));
         if (a.v_dbg != nullptr && live) {
-            float4* d4 = reinterpret_cast<float4*>(a.v_dbg + (size_t)row * K + e0);
+            float4* d4 = reinterpret_cast<float4*>(a.v_dbg + (size_t)row * K + lo);
             #pragma unroll
-            for (int u = 0; u < 4; ++u)
-                d4[u] = make_float4(v[p][4 * u], v[p][4 * u + 1], v[p][4 * u + 2], v[p][4 * u + 3]);
+            for (int u = 0; u < E / 4; ++u)
+                d4[u] = make_float4(v[j][4 * u], v[j][4 * u + 1], v[j][4 * u + 2], v[j][4 * u + 3]);
         }
     }
-    // row amax: warp shuffle, then across warps
     #pragma unroll
     for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
-    if (lane == 0) red[t >> 5] = amax;
-    __syncthreads();
-    amax = 0.f;
-    for (int w = 0; w < (T >> 5); ++w) amax = fmaxf(amax, red[w]);
+    if (warps_per_row > 1) {
+        if (lane == 0) red[warp] = amax;
+        __syncthreads();
+        amax = 0.f;
+        for (int w = 0; w < warps_per_row; ++w) amax = fmaxf(amax, red[w]);
+    }
+    if (!row_ok) return;
 
     const float qmax = (float)a.qmax;
     const bool nz = amax > 0.f;
     const float s = nz ? __fdiv_rn(amax, qmax) : 0.f;
     const float r = nz ? __fdiv_rn(qmax, amax) : 0.f;
-    if (t == 0) a.s[row] = s;
+    if (wr == 0 && lane == 0) a.s[row] = s;
     #pragma unroll
-    for (int p = 0; p < PASSES; ++p) {
-        const int e0 = p * EPT * T + EPT * t;
-        if (e0 >= K) continue;
-        uint32_t packed[2] = {0u, 0u};
+    for (int j = 0; j < NC; ++j) {
+        const int c = wr + j * warps_per_row;
+        const int lo = c * C + E * lane;
+        if (c >= nchunks || lo >= K) continue;
+        uint32_t packed[E / 8];
         #pragma unroll
-        for (int i = 0; i < EPT; ++i) {
-            int q = __float2int_rn(__fmul_rn(v[p][i], r));
-            q = max(-a.qmax, min(a.qmax, q));
-            packed[i >> 3] |= (uint32_t)(q & 0xF) << (4 * (i & 7));
+        for (int u = 0; u < E / 8; ++u) {
+            int q[8];
+            #pragma unroll
+            for (int k = 0; k < 8; ++k) q[k] = __float2int_rn(__fmul_rn(v[j][8 * u + k], r));
+            packed[u] = pack8(q);
         }
-        *reinterpret_cast<uint2*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) =
-            make_uint2(packed[0], packed[1]);
+        uint8_t* dst = a.Xq + (size_t)row * (K / 2) + lo / 2;
+        if (E == 16) {
+            *reinterpret_cast<uint2*>(dst) = make_uint2(packed[0], packed[1]);
+        } else {
+            #pragma unroll
+            for (int u = 0; u < E / 32; ++u)
+                reinterpret_cast<uint4*>(dst)[u] =
+                    make_uint4(packed[4 * u], packed[4 * u + 1], packed[4 * u + 2], packed[4 * u + 3]);
+        }
+        if (a.Xe != nullptr) {   // E4M3 bytes of the same codes
+            uint4* e4 = reinterpret_cast<uint4*>(a.Xe + (size_t)row * K + lo);
+            #pragma unroll
+            for (int u = 0; u < E / 16; ++u) {
+                uint32_t o[4];
+                int4x8_to_e4m3x8(packed[2 * u], o[0], o[1]);
+                int4x8_to_e4m3x8(packed[2 * u + 1], o[2], o[3]);
+                e4[u] = make_uint4(o[0], o[1], o[2], o[3]);
+            }
+        }
     }
+}
+
+template <int E, typename Tin>
+cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
+    constexpr int C = 32 * E;
+    const int n = (a.K + C - 1) / C;
+    int wpr, rpc, nc;
+    if (n == 1) { wpr = 1; rpc = 4; nc = 1; }
+    else { wpr = n < 8 ? n : 8; rpc = 1; nc = (n + wpr - 1) / wpr; }
+    const int warps = wpr * rpc;
+    const size_t smem = (size_t)warps * (C + 32) * 4 + 8 * 4;
+    dim3 grid((a.L + rpc - 1) / rpc), block(32 * warps);
+    #define STARQ_QUANT_LAUNCH(NCV)                                                            \
+        {                                                                                      \
+            static bool attr[64] = {false};                                                    \
+            int dev = 0; cudaGetDevice(&dev);                                                  \
+            if (smem > 48 * 1024 && dev < 64 && !attr[dev]) {                                  \
+                cudaError_t e = cudaFuncSetAttribute(sgat_quant_kernel<E, NCV, Tin>,           \
+                        cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);              \
+                if (e != cudaSuccess) return e;                                                \
+                attr[dev] = true;                                                              \
+            }                                                                                  \
+            sgat_quant_kernel<E, NCV, Tin><<<grid, block, smem, stream>>>(a, wpr, rpc);        \
+        }
+    if (E * nc > 128 || nc > 5) return cudaErrorInvalidValue;
+    switch (nc) {
+        case 1: STARQ_QUANT_LAUNCH(1); break;
+        case 2: if constexpr (E <= 64) STARQ_QUANT_LAUNCH(2); break;
+        case 3: if constexpr (E <= 32) STARQ_QUANT_LAUNCH(3); break;
+        case 4: if constexpr (E <= 32) STARQ_QUANT_LAUNCH(4); break;
+        case 5: if constexpr (E <= 16) STARQ_QUANT_LAUNCH(5); break;
+        default: return cudaErrorInvalidValue;
+    }
+    #undef STARQ_QUANT_LAUNCH
+    return cudaGetLastError();
 }
 
 template <typename Tin>
 cudaError_t launch_typed(const QuantArgs& a, cudaStream_t stream) {
-    int threads, passes;
-    if (a.K <= EPT * MAX_THREADS) {
-        threads = ((a.K / EPT) + 31) / 32 * 32;
-        passes = 1;
-    } else {
-        threads = MAX_THREADS;
-        passes = (a.K + EPT * MAX_THREADS - 1) / (EPT * MAX_THREADS);
-    }
-    dim3 grid(a.L), block(threads);
-    switch (passes) {
-        case 1: sgat_quant_kernel<1, Tin><<<grid, block, 0, stream>>>(a); break;
-        case 2: sgat_quant_kernel<2, Tin><<<grid, block, 0, stream>>>(a); break;
-        case 3: sgat_quant_kernel<3, Tin><<<grid, block, 0, stream>>>(a); break;
-        case 4: sgat_quant_kernel<4, Tin><<<grid, block, 0, stream>>>(a); break;
-        case 5: sgat_quant_kernel<5, Tin><<<grid, block, 0, stream>>>(a); break;
+    // chunk = one Hadamard block when hb >= 512, else 512 elements
+    const int C = a.hb >= 512 ? a.hb : 512;
+    switch (C) {
+        case 512: return launch_e<16, Tin>(a, stream);
+        case 1024: return launch_e<32, Tin>(a, stream);
+        case 2048: return launch_e<64, Tin>(a, stream);
+        case 4096: return launch_e<128, Tin>(a, stream);
         default: return cudaErrorInvalidValue;
     }
-    return cudaGetLastError();
 }
 
 }  // namespace

@@ -21,6 +21,9 @@
 // accumulators in TMEM let the epilogue of tile t overlap the MMAs of t+1.
 // Every mbarrier wait is bounded; a CTA that gives up records it in the
 // status word, drains its MMAs and frees TMEM before returning.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "common.cuh"
 
 namespace starq {
@@ -336,6 +339,417 @@ w4a4_gemm_kernel(GemmArgs a) {
     if (warp == MMA_WARP) tmem_dealloc(tmem_base, TMEM_COLS);
 }
 
+// ---------------------------------------------------------------------------
+// CTA-pair kernel: activation codes as E4M3 bytes by TMA, packed int4
+// weights by TMA into a staging buffer and converted in shared memory.
+//
+// Two CTAs of a cluster share one 256 x 256 output tile through
+// tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 32 per instruction): CTA r
+// holds tokens m0 + 128 r .. + 127 of A and output channels n0 + 128 r ..
+// + 127 of B, and receives rows 128 r .. of the accumulator in its own TMEM.
+// Each CTA therefore converts only its half of the weight tile. The leader
+// (rank 0) issues the MMAs once both CTAs' converters have arrived on its
+// stage barrier, and its commits arrive on the stage / accumulator barriers
+// of both CTAs. Roles per CTA (20 warps): 0-7 epilogue, 8 TMA producers
+// (activations; raw weights), 9 TMEM allocation + (leader) MMA issue, 10-19
+// converters, two per stage buffer. When the output has at least two
+// channel tiles, clusters hold two pairs that share the activation tile:
+// CTAs r and r ^ 2 each load half of it and multicast it to both.
+// ---------------------------------------------------------------------------
+namespace pairk {
+constexpr int BM = 128;                    // token rows per CTA (M = 256 per pair)
+constexpr int BN = 256;                    // output channels per pair tile
+constexpr int BN_CTA = 128;                // ... per CTA
+constexpr int BK = 128;                    // K elements per stage
+constexpr int UMMA_K = 32;
+constexpr int STAGES = 5;
+constexpr int A_BYTES = BM * BK;                       // 16 KB E4M3
+constexpr int B_BYTES = BN_CTA * BK;                   // 16 KB E4M3 (converted)
+constexpr int BRAW_BYTES = BN_CTA * BK / 2;            // 8 KB packed int4
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES + BRAW_BYTES;
+constexpr int NUM_EPI_WARPS = 8;           // lane quarter w % 4, column half w / 4
+constexpr int TMA_WARP = 8;                // lane 0: activation tiles, lane 1: raw weight tiles
+constexpr int MMA_WARP = 9;
+constexpr int FIRST_CONV_WARP = 10;
+constexpr int CONV_WARPS_PER_STAGE = 2;    // each converts half of a stage's rows
+constexpr int NUM_CONV_WARPS = CONV_WARPS_PER_STAGE * STAGES;
+constexpr int THREADS = (FIRST_CONV_WARP + NUM_CONV_WARPS) * 32;   // 640
+constexpr int TMEM_COLS = 512;
+constexpr int EPI_PARAM_BYTES = NUM_EPI_WARPS * 2 * (BN / 2) * 4;   // s_w and bias, 128 columns per warp
+constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
+constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
+static_assert(BRAW_BYTES % (16 * 32 * CONV_WARPS_PER_STAGE) == 0, "");
+
+struct Smem {
+    uint64_t a_full[STAGES];      // activation tile landed (TMA bytes)
+    uint64_t raw_full[STAGES];    // packed weight tile landed (TMA bytes)
+    uint64_t raw_empty[STAGES];   // converters done reading the packed tile
+    uint64_t full[STAGES];        // leader: converter warps of the pair
+    uint64_t empty[STAGES];       // MMA commit of every pair (multicast)
+    uint64_t tmem_full[2];        // MMA commit (multicast to the pair)
+    uint64_t tmem_empty[2];       // leader: epilogue warps of the pair
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+};
+}  // namespace pairk
+
+template <typename TOut, int CL>
+__global__ void __launch_bounds__(pairk::THREADS, 1)
+w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
+                      const __grid_constant__ CUtensorMap tmap_b) {
+    constexpr int BM = pairk::BM, BN = pairk::BN, BN_CTA = pairk::BN_CTA, BK = pairk::BK;
+    constexpr int UMMA_K = pairk::UMMA_K, STAGES = pairk::STAGES, STAGE_BYTES = pairk::STAGE_BYTES;
+    constexpr int A_BYTES = pairk::A_BYTES, B_BYTES = pairk::B_BYTES, BRAW_BYTES = pairk::BRAW_BYTES;
+    constexpr int TMA_WARP = pairk::TMA_WARP, MMA_WARP = pairk::MMA_WARP;
+    constexpr int FIRST_CONV_WARP = pairk::FIRST_CONV_WARP;
+    constexpr int CONV_WARPS_PER_STAGE = pairk::CONV_WARPS_PER_STAGE;
+    constexpr int NUM_EPI_WARPS = pairk::NUM_EPI_WARPS;
+    constexpr int TMEM_COLS = pairk::TMEM_COLS;
+    constexpr uint32_t IDESC = pairk::IDESC;
+    constexpr int PAIRS = CL / 2;                 // CTA pairs per cluster
+    constexpr uint16_t ALL = (uint16_t)((1u << CL) - 1u);
+    using Smem = pairk::Smem;
+    static_assert(CL == 2 || CL == 4, "");
+
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_addr(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    Smem* sh = reinterpret_cast<Smem*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES);
+    volatile int* abort = &sh->abort;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const uint32_t half = rank & 1u;             // position inside the CTA pair
+    const uint32_t pr = rank >> 1;               // which pair of the cluster
+    const uint32_t leader = rank & ~1u;
+    const uint16_t pair_mask = (uint16_t)(3u << (2 * pr));
+    const int L = a.L, N = a.N, K = a.K;
+    // Cluster tile: 256 tokens x PAIRS * 256 channels. Pair p takes
+    // channels p * 256 .. + 255 of it; the pairs share the activation tile,
+    // which CTAs r and r ^ 2 (same token rows) load half each and multicast.
+    const int num_m = (L + 2 * BM - 1) / (2 * BM);
+    const int num_n = (N + BN - 1) / BN;
+    const int num_np = (num_n + PAIRS - 1) / PAIRS;
+    const int num_tiles = num_m * num_np;
+    const int num_k = K / BK;
+    const int cluster = blockIdx.x / CL;
+    const int num_clusters = gridDim.x / CL;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_addr(&sh->a_full[s]), 1);
+            mbar_init(smem_addr(&sh->raw_full[s]), 1);
+            mbar_init(smem_addr(&sh->raw_empty[s]), CONV_WARPS_PER_STAGE);
+            mbar_init(smem_addr(&sh->full[s]), 2 * CONV_WARPS_PER_STAGE);  // converter warps of the pair
+            mbar_init(smem_addr(&sh->empty[s]), PAIRS);                    // every pair's MMA commit
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_addr(&sh->tmem_full[b]), 1);
+            mbar_init(smem_addr(&sh->tmem_empty[b]), 2 * NUM_EPI_WARPS);
+        }
+        mbar_init(smem_addr(&sh->drain), 1);
+        sh->abort = 0;
+        mbar_fence_init();
+    }
+    if (warp == MMA_WARP) {
+        tmem_alloc_pair(smem_addr(&sh->tmem_base), TMEM_COLS);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    cluster_sync();              // barriers of every CTA initialised, TMEM allocated
+    tc_fence_after();
+    const uint32_t tmem_base = sh->tmem_base;
+
+    if (warp == TMA_WARP) {
+        // Lane 0 streams activation tiles into a stage once every pair of
+        // the cluster has finished the MMAs on it; lane 1 streams packed
+        // weight tiles into the staging buffer as soon as the converters have
+        // read the previous one, so the raw weights of a stage arrive well
+        // before its MMA slot frees.
+        if (lane < 2) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            // With two pairs, CTAs r and r ^ 2 hold the same token rows: each
+            // loads half of them and multicasts it to both.
+            const uint16_t a_mask = (uint16_t)((1u << rank) | (1u << ((rank ^ 2u) % CL)));
+            for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters) {
+                const int m_rows = (tile % num_m) * 2 * BM + (int)half * BM;
+                const int n_rows = ((tile / num_m) * PAIRS + (int)pr) * BN + (int)half * BN_CTA;
+                for (int kc = 0; kc < num_k; ++kc) {
+                    const uint32_t st = base + stage * STAGE_BYTES;
+                    if (lane == 0) {
+                        if (!mbar_wait_bounded(smem_addr(&sh->empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
+                        const uint32_t bar = smem_addr(&sh->a_full[stage]);
+                        mbar_arrive_expect_tx(bar, A_BYTES);
+                        if (CL == 2) {
+                            tma_load_2d(st, &tmap_a, kc * BK, m_rows, bar);
+                        } else {
+                            tma_load_2d_multicast(st + pr * (A_BYTES / 2), &tmap_a, kc * BK,
+                                                  m_rows + (int)pr * (BM / 2), bar, a_mask);
+                        }
+                    } else {
+                        if (!mbar_wait_bounded(smem_addr(&sh->raw_empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
+                        const uint32_t bar = smem_addr(&sh->raw_full[stage]);
+                        mbar_arrive_expect_tx(bar, BRAW_BYTES);
+                        tma_load_2d(st + A_BYTES + B_BYTES, &tmap_b, kc * (BK / 2), n_rows, bar);
+                    }
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
+        }
+        __syncwarp();
+    } else if (warp >= FIRST_CONV_WARP) {
+        // Converter warps (cw % STAGES) own stage buffer cw % STAGES and
+        // convert its phases in order (stages g = buffer, buffer + STAGES,
+        // ... of the CTA's sequence), each the half of the rows given by
+        // cw / STAGES. All stage buffers convert concurrently, and a parity
+        // wait can never be two phases ahead of its barrier. One
+        // cluster-scope arrive per warp and stage tells the pair's leader
+        // that its rows are ready.
+        const int cw = warp - FIRST_CONV_WARP;
+        const int buf = cw % STAGES;
+        const int row0 = (cw / STAGES) * (BN_CTA / CONV_WARPS_PER_STAGE);
+        const uint32_t leader_full0 = mapa_shared(smem_addr(&sh->full[0]), leader);
+        const int my_tiles = cluster < num_tiles ? (num_tiles - 1 - cluster) / num_clusters + 1 : 0;
+        const int total = my_tiles * num_k;
+        bool ok = true;
+        for (int g = buf; g < total; g += STAGES) {
+            const int stage = buf;
+            const uint32_t k = (uint32_t)(g / STAGES);          // phase index of this buffer
+            if (!mbar_wait_bounded(smem_addr(&sh->raw_full[stage]), k & 1u, abort)) { ok = false; break; }
+            // the converted tile overwrites the previous phase's MMA operand
+            if (k > 0 && !mbar_wait_bounded(smem_addr(&sh->empty[stage]), (k - 1) & 1u, abort)) { ok = false; break; }
+            const uint32_t st = base + stage * STAGE_BYTES;
+            const uint32_t sB = st + A_BYTES, sRaw = st + A_BYTES + B_BYTES;
+            #pragma unroll 4
+            for (int u = 0; u < BRAW_BYTES / 16 / 32 / CONV_WARPS_PER_STAGE; ++u) {
+                const int idx = lane + 32 * u;
+                const int r = row0 + (idx >> 2), q = idx & 3;
+                convert_store(sB, r, q, ld_shared_v4(sRaw + r * (BK / 2) + q * 16));
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_addr(&sh->raw_empty[stage]));
+            fence_proxy_async_smem();
+            // the stage is ready for the MMA once this CTA's activation tile landed too
+            if (!mbar_wait_bounded(smem_addr(&sh->a_full[stage]), k & 1u, abort)) { ok = false; break; }
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(leader_full0 + stage * 8);
+        }
+        if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
+    } else if (warp == MMA_WARP) {
+        if (lane == 0 && half == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            int it = 0;
+            for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters, ++it) {
+                const int acc = it & 1;
+                const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+                if (!mbar_wait_bounded(smem_addr(&sh->tmem_empty[acc]), acc_phase ^ 1u, abort)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+                for (int kc = 0; kc < num_k; ++kc) {
+                    if (!mbar_wait_bounded(smem_addr(&sh->full[stage]), phase, abort)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t sA = base + stage * STAGE_BYTES;
+                    const uint32_t sB = sA + A_BYTES;
+                    #pragma unroll
+                    for (int ks = 0; ks < BK / UMMA_K; ++ks)
+                        mma_f8f6f4_pair(d_tmem, smem_desc_sw128(sA + ks * UMMA_K),
+                                        smem_desc_sw128(sB + ks * UMMA_K), IDESC,
+                                        (kc > 0 || ks > 0) ? 1u : 0u);
+                    // the stage may be refilled once every pair of the cluster is done with it
+                    tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), ALL);
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                tc_commit_pair_multicast(smem_addr(&sh->tmem_full[acc]), pair_mask);
+            }
+            tc_commit_pair_multicast(smem_addr(&sh->drain), pair_mask);
+            if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
+        }
+        __syncwarp();
+    } else {
+        // epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31 of this CTA,
+        // columns (w / 4) * 128 .. + 127 of the tile. Its per-channel scales
+        // and biases are staged in its own shared slice while the tile's
+        // MMAs run, so no global-load latency follows the accumulator.
+        const uint32_t leader_tmem_empty0 = mapa_shared(smem_addr(&sh->tmem_empty[0]), leader);
+        float* epi_sw = reinterpret_cast<float*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES + sizeof(Smem) +
+                                                 (16 - sizeof(Smem) % 16) % 16) + warp * 2 * (BN / 2);
+        float* epi_b = epi_sw + BN / 2;
+        const int quarter = warp & 3, chalf = warp >> 2;
+        bool ok = true;
+        int it = 0;
+        TOut* Y = static_cast<TOut*>(a.Y);
+        for (int tile = cluster; tile < num_tiles; tile += num_clusters, ++it) {
+            const int m0 = (tile % num_m) * 2 * BM + (int)half * BM;
+            const int n0 = ((tile / num_m) * PAIRS + (int)pr) * BN;
+            const int acc = it & 1;
+            const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+            const int row = m0 + quarter * 32 + lane;
+            const bool valid = row < L;
+            const float sa = valid ? __ldg(a.s_a + row) : 0.f;
+            {
+                const int ncol = n0 + chalf * (BN / 2) + 4 * lane;      // 4 columns per lane
+                float4 w = make_float4(0.f, 0.f, 0.f, 0.f), b = w;
+                if (ncol < N) {
+                    w = __ldg(reinterpret_cast<const float4*>(a.s_w + ncol));
+                    if (a.bias != nullptr) b = __ldg(reinterpret_cast<const float4*>(a.bias + ncol));
+                }
+                __syncwarp();          // the previous tile's reads of the slice are done
+                reinterpret_cast<float4*>(epi_sw)[lane] = w;
+                reinterpret_cast<float4*>(epi_b)[lane] = b;
+                __syncwarp();
+            }
+            if (!mbar_wait_bounded(smem_addr(&sh->tmem_full[acc]), acc_phase, abort)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t t_row = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+            #pragma unroll 1
+            for (int cc = 0; cc < BN / 64; ++cc) {
+                const int c = chalf * (BN / 64) + cc;
+                const int nc = n0 + c * 32;
+                if (nc >= N) break;
+                uint32_t r[32];
+                tmem_ld_32x32b_x32(t_row + c * 32, r);
+                tmem_ld_wait();
+                if (valid) {
+                    float y[32];
+                    const float4* sw4 = reinterpret_cast<const float4*>(epi_sw + cc * 32);
+                    const float4* b4 = reinterpret_cast<const float4*>(epi_b + cc * 32);
+                    #pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const float4 sw = sw4[u];
+                        y[4 * u] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u]), sa), sw.x);
+                        y[4 * u + 1] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 1]), sa), sw.y);
+                        y[4 * u + 2] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 2]), sa), sw.z);
+                        y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
+                    }
+                    if (a.bias != nullptr) {
+                        #pragma unroll
+                        for (int u = 0; u < 8; ++u) {
+                            const float4 b = b4[u];
+                            y[4 * u] = __fadd_rn(y[4 * u], b.x);
+                            y[4 * u + 1] = __fadd_rn(y[4 * u + 1], b.y);
+                            y[4 * u + 2] = __fadd_rn(y[4 * u + 2], b.z);
+                            y[4 * u + 3] = __fadd_rn(y[4 * u + 3], b.w);
+                        }
+                    }
+                    Out<TOut>::store32(Y + (size_t)row * N + nc, y);
+                    if (a.acc_dbg != nullptr) {
+                        int4* d4 = reinterpret_cast<int4*>(a.acc_dbg + (size_t)row * N + nc);
+                        #pragma unroll
+                        for (int u = 0; u < 8; ++u)
+                            d4[u] = make_int4(__float2int_rn(__uint_as_float(r[4 * u])),
+                                              __float2int_rn(__uint_as_float(r[4 * u + 1])),
+                                              __float2int_rn(__uint_as_float(r[4 * u + 2])),
+                                              __float2int_rn(__uint_as_float(r[4 * u + 3])));
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + acc * 8);
+        }
+        if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
+    }
+
+    // every MMA the pair's leader issued has completed before TMEM is released
+    if (warp == MMA_WARP && lane == 0) {
+        volatile int never = 0;
+        if (!mbar_wait_bounded(smem_addr(&sh->drain), 0, &never)) atomicOr(a.status, STATUS_TIMEOUT_GEMM);
+    }
+    __syncwarp();
+    tc_fence_before();
+    cluster_sync();              // no CTA leaves while another may still signal it
+    tc_fence_after();
+    if (warp == MMA_WARP) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+}
+
+// Tensor map of a row-major uint8 matrix [rows][cols] with a box of
+// box_rows x box_cols bytes.
+bool encode_u8_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                    uint32_t box_cols, CUtensorMapSwizzle swz) {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (fn == nullptr) {
+        cudaDriverEntryPointQueryResult q;
+        void* f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
+            return false;
+        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols};
+    const cuuint32_t box[2] = {box_cols, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Cluster size of the CTA-pair GEMM: 4 (two pairs sharing the activation
+// tile by multicast) unless fewer than two clusters of 4 fit, then 2.
+template <typename TOut, int CL>
+cudaError_t launch_pair_cl(const GemmArgs& a, cudaStream_t stream, const CUtensorMap& ta,
+                           const CUtensorMap& tb) {
+    constexpr int BM = pairk::BM, BN = pairk::BN;
+    constexpr int THREADS = pairk::THREADS;
+    constexpr size_t SMEM_BYTES = pairk::SMEM_BYTES;
+    auto kernel = w4a4_gemm_pair_kernel<TOut, CL>;
+    static bool attr_set[64] = {false};
+    static int max_clusters[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (dev < 64 && !attr_set[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        cfg.gridDim = dim3(CL * 64);
+        int n = 0;
+        e = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg);
+        if (e != cudaSuccess) return e;
+        max_clusters[dev] = n;
+        attr_set[dev] = true;
+    }
+    const int pairs_per_cluster = CL / 2;
+    const int num_tiles = ((a.L + 2 * BM - 1) / (2 * BM)) *
+                          (((a.N + BN - 1) / BN + pairs_per_cluster - 1) / pairs_per_cluster);
+    int clusters = dev < 64 ? max_clusters[dev] : 1;
+    if (clusters < 1) clusters = 1;
+    if (num_tiles < clusters) clusters = num_tiles;
+    cfg.gridDim = dim3(CL * clusters);
+    return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb);
+}
+
+template <typename TOut>
+cudaError_t launch_pair_typed(const GemmArgs& a, cudaStream_t stream) {
+    constexpr int BM = pairk::BM, BN_CTA = pairk::BN_CTA, BK = pairk::BK;
+    CUtensorMap ta2, ta4, tb;
+    if (!encode_u8_tmap(&ta2, a.Xe, (uint64_t)a.L, (uint64_t)a.K, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_u8_tmap(&ta4, a.Xe, (uint64_t)a.L, (uint64_t)a.K, BM / 2, BK, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_u8_tmap(&tb, a.Wq, (uint64_t)a.N, (uint64_t)a.K / 2, BN_CTA, BK / 2, CU_TENSOR_MAP_SWIZZLE_NONE))
+        return cudaErrorInvalidValue;
+    // two pairs per cluster (sharing the activation tile) when the
+    // channel tiles come in pairs
+    const bool quad = ((a.N + pairk::BN - 1) / pairk::BN) >= 2;
+    return quad ? launch_pair_cl<TOut, 4>(a, stream, ta4, tb) : launch_pair_cl<TOut, 2>(a, stream, ta2, tb);
+}
+
 template <typename TOut>
 cudaError_t launch_typed(const GemmArgs& a, cudaStream_t stream) {
     static bool attr_set[64] = {false};
@@ -358,6 +772,14 @@ cudaError_t launch_typed(const GemmArgs& a, cudaStream_t stream) {
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
     if (a.L == 0) return cudaSuccess;
+    if (a.Xe != nullptr) {
+        switch (a.y_dtype) {
+            case STARQ_F16: return launch_pair_typed<__half>(a, stream);
+            case STARQ_BF16: return launch_pair_typed<__nv_bfloat16>(a, stream);
+            case STARQ_F32: return launch_pair_typed<float>(a, stream);
+            default: return cudaErrorInvalidValue;
+        }
+    }
     switch (a.y_dtype) {
         case STARQ_F16: return launch_typed<__half>(a, stream);
         case STARQ_BF16: return launch_typed<__nv_bfloat16>(a, stream);

@@ -89,14 +89,26 @@ def gemm_codes(seed, L, N, K, lo=-7, hi=7):
 
 def workspace_views(ws, L, K, with_tac):
     """Views of the intermediates sgat_linear leaves in its workspace
-    (packed codes, per-token scales, float32 TAC output), following the
-    layout documented at sgat_linear_workspace_size."""
+    (packed codes, per-token scales, E4M3 codes, float32 TAC output),
+    following the layout documented for sgat_linear in include/starq.h."""
     a256 = lambda x: (x + 255) // 256 * 256
     o1 = a256(L * K // 2)
+    o2 = o1 + a256(4 * L)
+    o3 = o2 + a256(L * K)
     Xq = ws[: L * K // 2].view(L, K // 2)
     s_a = ws[o1: o1 + 4 * L].view(torch.float32)
-    zt = None
-    if with_tac:
-        o2 = o1 + a256(4 * L)
-        zt = ws[o2: o2 + 4 * L * K].view(torch.float32).view(L, K)
-    return Xq, s_a, zt
+    Xe = ws[o2: o2 + L * K].view(L, K)
+    zt = ws[o3: o3 + 4 * L * K].view(torch.float32).view(L, K) if with_tac else None
+    return Xq, s_a, Xe, zt
+
+
+def e4m3_bytes(q):
+    """E4M3 encoding (1 sign, 4 exponent bits with bias 7, 3 mantissa bits) of
+    integer codes in [-8, 8], written from the format's definition:
+    |q| = 2^e (1 + m/8) gives byte = sign << 7 | (e + 7) << 3 | m."""
+    q = np.asarray(q, dtype=np.int64)
+    a = np.abs(q)
+    e = np.where(a > 0, np.floor(np.log2(np.maximum(a, 1))).astype(np.int64), 0)
+    m = np.where(a > 0, (a * 8 // (1 << e)) - 8, 0)
+    b = np.where(a > 0, ((e + 7) << 3) | m, 0)
+    return (b | np.where(q < 0, 0x80, 0)).astype(np.uint8)

@@ -53,15 +53,15 @@ P = ctypes.c_void_p(4096)  # a non-null, 16-byte-aligned stand-in; never derefer
 
 
 @pytest.mark.parametrize("args,code", [
-    ((None, 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -1),   # NULL X
-    ((P, 9, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -1),      # dtype
-    ((P, 0, 4, 512, None, None, None, 512, 512, 0, 0, 8, P, P, None, None), -4),      # bits
-    ((P, 0, 4, 100, None, None, None, 4, 100, 0, 0, 4, P, P, None, None), -2),        # K % 16
-    ((P, 0, 4, 512, None, None, None, 384, 512, 0, 0, 4, P, P, None, None), -2),      # hb not pow2
-    ((P, 0, 4, 512, None, None, None, 8192, 512, 0, 0, 4, P, P, None, None), -2),     # hb > K
-    ((P, 0, 4, 512, None, None, None, 512, 500, 6, 0, 4, P, P, None, None), -2),      # gate sum
-    ((P, 0, -1, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -2),     # L < 0
-    ((ctypes.c_void_p(4100), 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None), -3),
+    ((None, 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -1),   # NULL X
+    ((P, 9, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -1),      # dtype
+    ((P, 0, 4, 512, None, None, None, 512, 512, 0, 0, 8, P, P, None, None, None), -4),      # bits
+    ((P, 0, 4, 100, None, None, None, 4, 100, 0, 0, 4, P, P, None, None, None), -2),        # K % 16
+    ((P, 0, 4, 512, None, None, None, 384, 512, 0, 0, 4, P, P, None, None, None), -2),      # hb not pow2
+    ((P, 0, 4, 512, None, None, None, 8192, 512, 0, 0, 4, P, P, None, None, None), -2),     # hb > K
+    ((P, 0, 4, 512, None, None, None, 512, 500, 6, 0, 4, P, P, None, None, None), -2),      # gate sum
+    ((P, 0, -1, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -2),     # L < 0
+    ((ctypes.c_void_p(4100), 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -3),
 ])
 def test_quantize_act_validation(lib, args, code):
     assert lib.lib.sgat_quantize_act(*args) == code
@@ -71,13 +71,14 @@ def test_quantize_act_validation(lib, args, code):
 @pytest.mark.parametrize("L,N,K,code", [(4, 100, 512, -2), (4, 256, 200, -2), (4, 256, 131072, -2),
                                         (-1, 256, 512, -2)])
 def test_gemm_validation(lib, L, N, K, code):
-    assert lib.lib.w4a4_gemm(P, P, P, P, None, L, N, K, P, 0, None, None) == code
+    assert lib.lib.w4a4_gemm(P, None, P, P, P, None, L, N, K, P, 0, None, None) == code
 
 
 def test_gemm_null_and_alignment(lib):
-    assert lib.lib.w4a4_gemm(None, P, P, P, None, 4, 256, 512, P, 0, None, None) == -1
-    assert lib.lib.w4a4_gemm(ctypes.c_void_p(4104), P, P, P, None, 4, 256, 512, P, 0, None, None) == -3
-    assert lib.lib.w4a4_gemm(P, P, P, P, None, 4, 256, 512, P, 7, None, None) == -1
+    assert lib.lib.w4a4_gemm(None, None, P, P, P, None, 4, 256, 512, P, 0, None, None) == -1
+    assert lib.lib.w4a4_gemm(ctypes.c_void_p(4104), None, P, P, P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert lib.lib.w4a4_gemm(None, ctypes.c_void_p(4104), P, P, P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert lib.lib.w4a4_gemm(P, None, P, P, P, None, 4, 256, 512, P, 7, None, None) == -1
 
 
 @pytest.mark.parametrize("g,C,code", [(12, 96, -2), (16, 100, -2), (256, 4096, -2)])
@@ -91,7 +92,7 @@ def test_tac_null_matrix(lib):
 
 def test_linear_workspace_and_validation(lib):
     n = lib.sgat_linear_workspace_size(1024, 4096, False)
-    assert n == 1024 * 2048 + 4096
+    assert n == 1024 * 2048 + 4096 + 1024 * 4096
     assert lib.sgat_linear_workspace_size(1024, 4096, True) == n + 1024 * 4096 * 4
     # workspace too small
     rc = lib.lib.sgat_linear(P, 0, 1024, 4096, None, None, None, 4096, 4096, 0, 0, None, None, 0,

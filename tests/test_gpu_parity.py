@@ -33,9 +33,11 @@ def run_quant(abi, case, mask=True, dbg=True):
     a_m, a_u = H.dev(xf.a_m), H.dev(xf.a_u)
     Xq = torch.empty(L, K // 2, dtype=torch.uint8, device="cuda")
     s_a = torch.empty(L, dtype=torch.float32, device="cuda")
+    Xe = torch.empty(L, K, dtype=torch.uint8, device="cuda")
     v = torch.empty(L, K, dtype=torch.float32, device="cuda") if dbg else None
-    abi.sgat_quantize_act(X, m, a_m, a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, Xq, s_a, v_dbg=v)
+    abi.sgat_quantize_act(X, m, a_m, a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, Xq, s_a, Xe=Xe, v_dbg=v)
     abi.check_status()
+    assert np.array_equal(Xe.cpu().numpy(), H.e4m3_bytes(H.unpack(Xq))), "E4M3 copy differs from the codes"
     return Xq, s_a, v
 
 
@@ -102,32 +104,40 @@ def test_prepare_weight_bitexact(abi, N, K, hb, dtype):
     assert np.array_equal(s_w.cpu().numpy(), s)
 
 
-def run_gemm(abi, qa, qw, s_a, s_w, out="f16", bias=None):
+def run_gemm(abi, qa, qw, s_a, s_w, out="f16", bias=None, path="e4m3"):
+    """path "packed": packed int4 activations (both operands converted in the
+    kernel); path "e4m3": E4M3 activation codes streamed by TMA to CTA pairs."""
     L, K = qa.shape
     N = qw.shape[0]
-    Xq = H.dev(osg.pack_int4(qa))
     Wq = H.dev(osg.pack_int4(qw))
     Y = torch.empty(L, N, dtype=H.torch_dtype(out), device="cuda")
     acc = torch.empty(L, N, dtype=torch.int32, device="cuda")
-    abi.w4a4_gemm(Xq, H.dev(s_a), Wq, H.dev(s_w), Y, bias=None if bias is None else H.dev(bias), acc_dbg=acc)
+    if path == "packed":
+        Xq, Xe = H.dev(osg.pack_int4(qa)), None
+    else:
+        Xq, Xe = None, H.dev(H.e4m3_bytes(qa))
+    abi.w4a4_gemm(Xq, H.dev(s_a), Wq, H.dev(s_w), Y, bias=None if bias is None else H.dev(bias),
+                  acc_dbg=acc, Xe=Xe)
     abi.check_status()
     return H.host(Y), acc.cpu().numpy()
 
 
+@pytest.mark.parametrize("path", ["e4m3", "packed"])
 @pytest.mark.parametrize("L,N,K,out", [(1, 256, 128, "f16"), (129, 512, 512, "f16"), (300, 288, 1024, "bf16"),
                                        (128, 256, 4096, "f32"), (1000, 768, 384, "f16"),
-                                       (257, 4096, 256, "f16")])
-def test_w4a4_gemm_exact(abi, L, N, K, out):
+                                       (257, 4096, 256, "f16"), (513, 160, 640, "f16")])
+def test_w4a4_gemm_exact(abi, L, N, K, out, path):
     qa, qw, s_a, s_w = H.gemm_codes(L * 7 + N + K, L, N, K)
     bias = np.random.default_rng(1).normal(0, 0.1, N).astype(np.float32) if out == "bf16" else None
-    Y, acc = run_gemm(abi, qa, qw, s_a, s_w, out, bias)
+    Y, acc = run_gemm(abi, qa, qw, s_a, s_w, out, bias, path)
     ref_acc = osg.int_gemm(qa, qw)
     assert np.array_equal(acc, ref_acc), "integer accumulators differ"
     H.assert_output_close(Y, osg.dequant(ref_acc, s_a, s_w, bias), out)
 
 
+@pytest.mark.parametrize("path", ["e4m3", "packed"])
 @pytest.mark.parametrize("K", [18944, 65536])
-def test_w4a4_gemm_adversarial_exactness(abi, K):
+def test_w4a4_gemm_adversarial_exactness(abi, K, path):
     """Integer exactness of the float32 tensor-core accumulation: all codes
     +-7 (largest accumulators), alternating signs, and a large running sum
     followed by increments of exactly 1 per 32-element MMA step (a truncating
@@ -152,7 +162,7 @@ def test_w4a4_gemm_adversarial_exactness(abi, K):
     qw[5:] = rng.integers(-7, 8, (N - 5, K))
     s_a = np.ones(L, np.float32)
     s_w = np.ones(N, np.float32)
-    _, acc = run_gemm(abi, qa, qw, s_a, s_w, "f32")
+    _, acc = run_gemm(abi, qa, qw, s_a, s_w, "f32", path=path)
     ref = osg.int_gemm(qa, qw)
     assert ref[0, 0] == 49 * K and ref[2, 3] == 49 * half + half // 32
     assert np.array_equal(acc, ref)
@@ -204,7 +214,7 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None):
     abi.check_status()
     qw, sw = osg.prepare_weight(case.W, xf.inv_a_w, xf.hb, 4)
     assert np.array_equal(H.unpack(Wq), qw) and np.array_equal(s_w.cpu().numpy(), sw)
-    Xq_g, s_a_g, zt = H.workspace_views(ws, L, K, with_tac)
+    Xq_g, s_a_g, Xe_g, zt = H.workspace_views(ws, L, K, with_tac)
     rows = np.arange(L) if check_rows is None else np.asarray(check_rows)
     X_in = case.X
     if with_tac:
@@ -215,6 +225,7 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None):
     Y_ref, codes, s_a, acc = osg.sgat_linear(X_in[rows], case.mask[rows], xf.a_m, xf.a_u, xf.hb, xf.d_sh,
                                              xf.d_m, xf.d_u, qw, sw, case.bias, 4)
     assert np.array_equal(H.unpack(Xq_g)[rows], codes), "activation codes differ"
+    assert np.array_equal(Xe_g.cpu().numpy()[rows], H.e4m3_bytes(codes)), "E4M3 codes differ"
     assert np.array_equal(s_a_g.cpu().numpy()[rows], s_a), "activation scales differ"
     H.assert_output_close(H.host(Y)[rows], Y_ref, out_dtype)
     return Y
@@ -258,4 +269,5 @@ def test_empty_batch(abi):
     sw = torch.ones(N, dtype=torch.float32, device="cuda")
     Y = torch.empty(0, N, dtype=torch.float16, device="cuda")
     abi.w4a4_gemm(Xq, s, Wq, sw, Y)
+    abi.w4a4_gemm(None, s, Wq, sw, Y, Xe=torch.empty(0, K, dtype=torch.uint8, device="cuda"))
     abi.check_status()
