@@ -189,7 +189,9 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
     if (rc) return rc;
     if (L == 0) return STARQ_OK;
     if (!aligned(Z, 16) || !aligned(out, 16)) return fail(STARQ_ERR_ALIGN, "tac_apply: Z, out alignment");
-    TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype};
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype, st};
     cudaError_t e = launch_tac(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "tac_apply launch");
     return STARQ_OK;
@@ -234,7 +236,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     int qin_dtype = x_dtype;
     cudaError_t e;
     if (tac_M) {
-        TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, STARQ_F32};
+        TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, STARQ_F32, st};
         if ((e = launch_tac(t, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: tac launch");
         qin = zt;
         qin_dtype = STARQ_F32;

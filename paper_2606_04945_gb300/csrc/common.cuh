@@ -17,6 +17,7 @@ namespace starq {
 constexpr unsigned STATUS_TIMEOUT_GEMM = 1u << 0;
 constexpr unsigned STATUS_TIMEOUT_FP16_GEMM = 1u << 1;
 constexpr unsigned STATUS_TIMEOUT_TEST = 1u << 2;
+constexpr unsigned STATUS_TIMEOUT_TAC = 1u << 3;
 
 // Upper bound of any single wait inside a kernel. Kernels of this library
 // finish in milliseconds; a wait this long means a broken pipeline, and the
@@ -49,6 +50,7 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
 struct TacArgs {
     const void* Z; int z_dtype; int L; int C; int g;
     const float* M; const float* d; void* out; int out_dtype;
+    unsigned* status = nullptr;   // device status word (tensor-core path)
 };
 cudaError_t launch_tac(const TacArgs& a, cudaStream_t stream);
 
@@ -256,6 +258,29 @@ __device__ __forceinline__ void tma_load_2d_multicast(uint32_t dst, const void* 
     asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
                  " [%0], [%1, {%2, %3}], [%4], %5;"
                  :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar), "h"(cta_mask) : "memory");
+}
+// Contiguous global -> shared bulk copy (16-byte aligned, size % 16 == 0),
+// completion counted on `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+// 2-D TMA tile store shared -> global (bulk group of the calling thread).
+__device__ __forceinline__ void tma_store_2d(const void* tmap, int x, int y, uint32_t src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];"
+                 :: "l"(tmap), "r"(x), "r"(y), "r"(src) : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Wait until the calling thread's committed bulk stores have read their
+// shared-memory sources.
+__device__ __forceinline__ void bulk_wait_read0() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+// Wait until the calling thread's committed bulk stores are complete.
+__device__ __forceinline__ void bulk_wait0() {
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;"

@@ -2,11 +2,17 @@
 //
 //   out[i][b*g + r] = sum_j M[b][r][j] * Z[i][b*g + j] + d[b][r]
 //
-// Grid: (token tiles, blocks b). A CTA stages M_b transposed (Mt[j][r]) and a
-// tile of TM tokens of block b in shared memory, then each thread computes
+// 16-bit inputs with g = 64 or 128 run on the tensor cores (tac_tc_kernel
+// below). Otherwise, the CUDA-core kernel: grid (token tiles, blocks b). A
+// CTA stages M_b transposed (Mt[j][r]) and a tile of TM tokens of block b in shared memory, then each thread computes
 // RT = 4 tokens x RC = 8 channels with float32 FMAs, reading four j at a time
 // (float4) from both tiles. TM = 8192 / g tokens, so the token tile is
 // 32 KB (fp32) and the CTA holds g*g*4 + 32 KB of shared memory.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <type_traits>
+
 #include "common.cuh"
 
 namespace starq {
@@ -118,8 +124,315 @@ cudaError_t launch_g(const TacArgs& a, cudaStream_t stream) {
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Tensor-core TAC for g in {64, 128} with 16-bit inputs.
+//
+// Block b is a GEMM out_b[L x g] = Z_b[L x g] M_b^T[g x g] + d_b with the
+// contraction over the block's g channels. Z is exact in its 16-bit type; M
+// is split into M_hi = 16bit(M) and M_lo = 16bit(M - M_hi) of the same type
+// (the MMA takes equal A and B types), and the tensor core accumulates
+// Z M_hi^T + Z M_lo^T in float32 in TMEM; the residual of the split is
+// below 2^-22 |M| for fp16 and 2^-16 |M| for bf16. A CTA owns one block b and
+// a run of 128-token tiles: it converts M_b once into 128-byte-swizzled
+// K-major shared tiles, streams the Z tiles by TMA (two buffers), runs
+// 2 g/16 MMAs (M = 128, N = g, K = 16) per tile, and its four warps add d_b
+// to the rows read back from TMEM. float32 outputs are staged as
+// 128-byte-swizzled 32 x 32 boxes and written by TMA stores; 16-bit outputs
+// by 16-byte row stores.
+// ---------------------------------------------------------------------------
+constexpr int TC_TM = 128;              // tokens per tile (MMA M)
+constexpr int TC_THREADS = 128;
+
+template <int G>
+struct TacTc {
+    static constexpr int ATOMS = G / 64;                      // 64 16-bit elements = 128 B per atom row
+    static constexpr int Z_BYTES = TC_TM * G * 2;             // one Z tile
+    static constexpr int M_BYTES = G * G * 2;                 // one of M_hi / M_lo
+    static constexpr int MF32_BYTES = G * G * 4;              // M_b in float32
+    static constexpr int STAGE_OUT_BYTES = TC_TM * G * 4;     // float32 output tile
+    // M_b in float32 first, the output staging afterwards
+    static constexpr int RAW_BYTES = MF32_BYTES > STAGE_OUT_BYTES ? MF32_BYTES : STAGE_OUT_BYTES;
+    static constexpr size_t SMEM = 2 * (size_t)Z_BYTES + 2 * (size_t)M_BYTES + RAW_BYTES + 1024 + 256;
+    static constexpr int TMEM_COLS = 2 * G;                   // two accumulators
+};
+
+template <typename T> struct Split16;
+template <> struct Split16<__half> {
+    static __device__ __forceinline__ void split(float m, uint16_t& hi, uint16_t& lo) {
+        const __half h = __float2half_rn(m);
+        const __half l = __float2half_rn(m - __half2float(h));
+        hi = __half_as_ushort(h);
+        lo = __half_as_ushort(l);
+    }
+    static constexpr uint32_t KIND = 0;
+};
+template <> struct Split16<__nv_bfloat16> {
+    static __device__ __forceinline__ void split(float m, uint16_t& hi, uint16_t& lo) {
+        const __nv_bfloat16 h = __float2bfloat16_rn(m);
+        const __nv_bfloat16 l = __float2bfloat16_rn(m - __bfloat162float(h));
+        hi = __bfloat16_as_ushort(h);
+        lo = __bfloat16_as_ushort(l);
+    }
+    static constexpr uint32_t KIND = 1;
+};
+
+template <typename TOut> struct TacStore;
+// float32 output: 32 x 32 boxes staged 128-byte-swizzled and written by TMA
+template <> struct TacStore<float> {
+    static constexpr bool TMA = true;
+};
+template <> struct TacStore<__half> { static constexpr bool TMA = false; };
+template <> struct TacStore<__nv_bfloat16> { static constexpr bool TMA = false; };
+
+template <int G, typename TIn, typename TOut>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+tac_tc_kernel(TacArgs a, int tiles_per_cta, const __grid_constant__ CUtensorMap tmap_z,
+              const __grid_constant__ CUtensorMap tmap_out, unsigned* status) {
+    using P = TacTc<G>;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t zfull[2], mdone[2], mbar_raw;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_flag;
+    const uint32_t raw = smem_addr(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    const uint32_t sZ = base;                                  // 2 x Z tile
+    const uint32_t sMh = base + 2 * P::Z_BYTES, sMl = sMh + P::M_BYTES;
+    const uint32_t sRaw = sMl + P::M_BYTES;                    // M_b float32, then output staging
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = blockIdx.x;
+    const int t0 = blockIdx.y * tiles_per_cta;
+    const int n_tiles_total = (a.L + TC_TM - 1) / TC_TM;
+    const int nt = min(tiles_per_cta, n_tiles_total - t0);
+    volatile int* abort = &abort_flag;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(smem_addr(&zfull[i]), 1);
+            mbar_init(smem_addr(&mdone[i]), 1);
+        }
+        mbar_init(smem_addr(&mbar_raw), 1);
+        abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_addr(&tmem_slot), P::TMEM_COLS);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        // M_b (float32, contiguous) and the first Z tiles in flight together
+        mbar_arrive_expect_tx(smem_addr(&mbar_raw), P::MF32_BYTES);
+        bulk_load(sRaw, a.M + (size_t)b * G * G, P::MF32_BYTES, smem_addr(&mbar_raw));
+        for (int i = 0; i < 2 && i < nt; ++i) {
+            const uint32_t bar = smem_addr(&zfull[i]);
+            mbar_arrive_expect_tx(bar, P::Z_BYTES);
+            for (int at = 0; at < P::ATOMS; ++at)
+                tma_load_2d(sZ + i * P::Z_BYTES + at * (TC_TM * 128), &tmap_z, b * G + at * 64, (t0 + i) * TC_TM, bar);
+        }
+    }
+    bool ok = mbar_wait_bounded(smem_addr(&mbar_raw), 0, abort);
+    // M_b -> hi / lo 16-bit tiles, K-major (row r = output channel, 8 inputs per 16-byte chunk)
+    for (int idx = threadIdx.x; ok && idx < G * G / 8; idx += TC_THREADS) {
+        const int r = idx / (G / 8), jc = idx % (G / 8);      // inputs j = 8 jc .. 8 jc + 7
+        const uint4 w0 = ld_shared_v4(sRaw + (uint32_t)(r * G + 8 * jc) * 4);
+        const uint4 w1 = ld_shared_v4(sRaw + (uint32_t)(r * G + 8 * jc + 4) * 4);
+        const float mv[8] = {__uint_as_float(w0.x), __uint_as_float(w0.y), __uint_as_float(w0.z),
+                             __uint_as_float(w0.w), __uint_as_float(w1.x), __uint_as_float(w1.y),
+                             __uint_as_float(w1.z), __uint_as_float(w1.w)};
+        uint32_t hi[4], lo[4];
+        #pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            uint16_t h0, l0, h1, l1;
+            Split16<TIn>::split(mv[2 * e], h0, l0);
+            Split16<TIn>::split(mv[2 * e + 1], h1, l1);
+            hi[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+            lo[e] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+        }
+        const int at = jc / 8, c = jc % 8;                    // atom, 16-byte chunk in the 128-byte row
+        const uint32_t off = at * (G * 128) + sw128_offset(r, c);
+        st_shared_v4(sMh + off, hi[0], hi[1], hi[2], hi[3]);
+        st_shared_v4(sMl + off, lo[0], lo[1], lo[2], lo[3]);
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    constexpr uint32_t IDESC = (1u << 4) | (Split16<TIn>::KIND << 7) | (Split16<TIn>::KIND << 10) |
+                               ((uint32_t)(G >> 3) << 17) | ((uint32_t)(TC_TM >> 4) << 24);
+    TOut* out = static_cast<TOut*>(a.out);
+    // per-warp staging of its 32 rows: G/32 boxes of 32 x 32 float32
+    const uint32_t stage_w = sRaw + warp * (32 * G * 4);
+    for (int i = 0; i < nt && ok; ++i) {
+        const int buf = i & 1;
+        const uint32_t ph = (uint32_t)(i >> 1) & 1u;
+        if (threadIdx.x == 0) {
+            if (!mbar_wait_bounded(smem_addr(&zfull[buf]), ph, abort)) { ok = false; *abort = 1; }
+            else {
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(buf * G);
+                #pragma unroll
+                for (int ks = 0; ks < G / 16; ++ks) {
+                    const uint32_t koff = (ks / 4) * (TC_TM * 128) + (ks % 4) * 32;
+                    const uint32_t moff = (ks / 4) * (G * 128) + (ks % 4) * 32;
+                    const uint64_t ad = smem_desc_sw128(sZ + buf * P::Z_BYTES + koff);
+                    mma_f16(d, ad, smem_desc_sw128(sMh + moff), IDESC, ks > 0 ? 1u : 0u);
+                    mma_f16(d, ad, smem_desc_sw128(sMl + moff), IDESC, 1u);
+                }
+                tc_commit(smem_addr(&mdone[buf]));
+            }
+        }
+        if (!mbar_wait_bounded(smem_addr(&mdone[buf]), ph, abort)) ok = false;
+        __syncthreads();
+        if (!ok || *abort) { ok = false; break; }
+        tc_fence_after();
+        // the Z buffer is free again: fetch the tile after next
+        if (threadIdx.x == 0 && i + 2 < nt) {
+            const uint32_t bar = smem_addr(&zfull[buf]);
+            mbar_arrive_expect_tx(bar, P::Z_BYTES);
+            for (int at = 0; at < P::ATOMS; ++at)
+                tma_load_2d(sZ + buf * P::Z_BYTES + at * (TC_TM * 128), &tmap_z, b * G + at * 64, (t0 + i + 2) * TC_TM, bar);
+        }
+        const int row0 = (t0 + i) * TC_TM + warp * 32;
+        const int tok = row0 + lane;
+        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * G);
+        const float* dp = a.d ? a.d + (size_t)b * G : nullptr;
+        if (TacStore<TOut>::TMA && lane == 0) bulk_wait_read0();   // previous tile's stores left the staging
+        __syncwarp();
+        #pragma unroll 1
+        for (int c = 0; c < G / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld_32x32b_x32(trow + c * 32, r);
+            tmem_ld_wait();
+            float v[32];
+            #pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+                float4 dd = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (dp) dd = __ldg(reinterpret_cast<const float4*>(dp + c * 32 + j));
+                v[j] = __uint_as_float(r[j]) + dd.x;
+                v[j + 1] = __uint_as_float(r[j + 1]) + dd.y;
+                v[j + 2] = __uint_as_float(r[j + 2]) + dd.z;
+                v[j + 3] = __uint_as_float(r[j + 3]) + dd.w;
+            }
+            if (TacStore<TOut>::TMA) {
+                // box c of this warp: row `lane`, 16-byte chunk q at (q ^ (lane & 7))
+                const uint32_t box = stage_w + c * (32 * 128);
+                #pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    st_shared_v4(box + lane * 128 + ((q ^ (lane & 7)) << 4), __float_as_uint(v[4 * q]),
+                                 __float_as_uint(v[4 * q + 1]), __float_as_uint(v[4 * q + 2]),
+                                 __float_as_uint(v[4 * q + 3]));
+            } else if (tok < a.L) {
+                TOut* o = out + (size_t)tok * a.C + b * G + c * 32;
+                #pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    uint32_t w[4];
+                    #pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        TOut x0 = from_f<TOut>(v[8 * u + 2 * e]), x1 = from_f<TOut>(v[8 * u + 2 * e + 1]);
+                        w[e] = (uint32_t)(*reinterpret_cast<uint16_t*>(&x0)) |
+                               ((uint32_t)(*reinterpret_cast<uint16_t*>(&x1)) << 16);
+                    }
+                    reinterpret_cast<uint4*>(o)[u] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+            }
+        }
+        if (TacStore<TOut>::TMA) {
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                for (int c = 0; c < G / 32; ++c)
+                    tma_store_2d(&tmap_out, b * G + c * 32, row0, stage_w + c * (32 * 128));
+                bulk_commit();
+            }
+        }
+        tc_fence_before();
+        __syncthreads();
+    }
+    if (TacStore<TOut>::TMA && lane == 0) bulk_wait0();
+    if (!ok && threadIdx.x == 0) atomicOr(status, STATUS_TIMEOUT_TAC);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, P::TMEM_COLS);
+}
+
+bool encode_u16_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                     uint32_t box_cols) {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (fn == nullptr) {
+        cudaDriverEntryPointQueryResult q;
+        void* f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
+            return false;
+        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols * 2};
+    const cuuint32_t box[2] = {box_cols, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_f32_out_tmap(CUtensorMap* m, void* ptr, uint64_t rows, uint64_t cols) {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (fn == nullptr) {
+        cudaDriverEntryPointQueryResult q;
+        void* f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
+            return false;
+        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols * 4};
+    const cuuint32_t box[2] = {32, 32};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, ptr, dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int G, typename TIn, typename TOut>
+cudaError_t launch_tc(const TacArgs& a, cudaStream_t stream) {
+    using P = TacTc<G>;
+    static bool attr_set[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 64 && !attr_set[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(tac_tc_kernel<G, TIn, TOut>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::SMEM);
+        if (e != cudaSuccess) return e;
+        attr_set[dev] = true;
+    }
+    CUtensorMap tz, to;
+    if (!encode_u16_tmap(&tz, a.Z, (uint64_t)a.L, (uint64_t)a.C, TC_TM, 64)) return cudaErrorInvalidValue;
+    if (TacStore<TOut>::TMA) {
+        if (!encode_f32_out_tmap(&to, a.out, (uint64_t)a.L, (uint64_t)a.C)) return cudaErrorInvalidValue;
+    } else {
+        to = tz;   // unused
+    }
+    const int blocks = a.C / G;
+    const int tiles = (a.L + TC_TM - 1) / TC_TM;
+    // about two CTAs' worth of work per SM, at least two tiles per CTA when possible
+    int per = (blocks * tiles + 2 * num_sms() - 1) / (2 * num_sms());
+    if (per < 2) per = tiles < 2 ? tiles : 2;
+    if (per > tiles) per = tiles;
+    dim3 grid(blocks, (tiles + per - 1) / per);
+    tac_tc_kernel<G, TIn, TOut><<<grid, TC_THREADS, P::SMEM, stream>>>(a, per, tz, to, a.status);
+    return cudaGetLastError();
+}
+
 template <typename TIn, typename TOut>
 cudaError_t launch_io(const TacArgs& a, cudaStream_t stream) {
+    if constexpr (!std::is_same<TIn, float>::value) {
+        if (a.status != nullptr && (a.g == 64 || a.g == 128)) {
+            return a.g == 64 ? launch_tc<64, TIn, TOut>(a, stream) : launch_tc<128, TIn, TOut>(a, stream);
+        }
+    }
     switch (a.g) {
         case 4: return launch_g<4, TIn, TOut>(a, stream);
         case 8: return launch_g<8, TIn, TOut>(a, stream);
