@@ -15,16 +15,17 @@
 // no clamp is needed: |fl(v * r)| <= 7 (1 + 2^-24)^2 < 7.5.
 //
 // Work split: a warp owns a chunk of C = 32 E consecutive elements of a row
-// (E = hb / 32, or E = 16 with several Hadamard blocks per chunk when
-// hb < 512). In layout A lane l holds elements E l .. E l + E - 1, so stages
-// h < E are butterflies between registers of one thread. One transpose
-// through shared memory (layout B: lane l holds elements l + 32 i) makes the
-// stages h >= 32 register-local too; a transpose back gives each lane E
-// contiguous values again for gating, scaling and packing.
+// (C = 1024 when hb >= 1024, else C = 512 holding 512 / hb Hadamard blocks).
+// In layout A lane l holds elements E l .. E l + E - 1, so stages h < E are
+// butterflies between registers of one thread. One transpose through shared
+// memory (layout B: lane l holds elements l + 32 i) makes the stages
+// 32 <= h < C register-local too; a transpose back gives each lane E
+// contiguous values again. Stages h >= C (hb = 2048, 4096) pair chunks held
+// by different warps of the row and exchange through shared memory.
 //
-// Rows of one chunk (K == C) take one warp each, four rows per CTA; longer
-// rows take a CTA of up to 8 warps, each keeping up to NC chunks in
-// registers, and reduce amax across warps through shared memory.
+// A row takes min(K / C, 8) warps, each keeping up to NC chunks in
+// registers; short rows share a CTA of 8 warps. amax is reduced across a
+// row's warps through shared memory.
 #include "common.cuh"
 
 namespace starq {
@@ -201,6 +202,24 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
             for (int i = 0; i < E; ++i) v[j][i] = 0.f;
         }
         if (c < nchunks) chunk_fwht<E>(v[j], a.hb, lane, buf);   // warp-uniform condition
+        // Stages h = C .. hb/2 pair chunk c with chunk c ^ (h / C), held by
+        // warp wr ^ (h / C) of the same row in the same round j (the warp
+        // count of a row is a multiple of hb / C). Exchange in layout A
+        // through the warps' padded buffers; all warps of the CTA take part.
+        for (int m = 1; m * C < a.hb; m <<= 1) {
+            float* mine = buf + (E + 1) * lane;
+            const float* other = qsm + (warp ^ m) * (C + 32) + (E + 1) * lane;
+            #pragma unroll
+            for (int i = 0; i < E; ++i) mine[i] = v[j][i];
+            __syncthreads();
+            const bool upper = (wr & m) != 0;
+            #pragma unroll
+            for (int i = 0; i < E; ++i) {
+                const float o = other[i];
+                v[j][i] = upper ? __fsub_rn(o, v[j][i]) : __fadd_rn(v[j][i], o);
+            }
+            __syncthreads();
+        }
         // gate: whole-lane decisions first, per element only where a lane
         // straddles a subspace boundary
         const bool all_keep = (lo + E <= a.d_sh) || (lo >= own_lo && lo + E <= own_hi);
@@ -230,7 +249,8 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
         if (lane == 0) red[warp] = amax;
         __syncthreads();
         amax = 0.f;
-        for (int w = 0; w < warps_per_row; ++w) amax = fmaxf(amax, red[w]);
+        const int first = warp - wr;                     // first warp of this row
+        for (int w = 0; w < warps_per_row; ++w) amax = fmaxf(amax, red[first + w]);
     }
     if (!row_ok) return;
 
@@ -277,10 +297,10 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
 template <int E, typename Tin>
 cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
     constexpr int C = 32 * E;
-    const int n = (a.K + C - 1) / C;
-    int wpr, rpc, nc;
-    if (n == 1) { wpr = 1; rpc = 4; nc = 1; }
-    else { wpr = n < 8 ? n : 8; rpc = 1; nc = (n + wpr - 1) / wpr; }
+    const int n = (a.K + C - 1) / C;                 // chunks per row
+    const int wpr = n < 8 ? n : 8;                   // warps per row (a multiple of hb / C)
+    const int rpc = wpr <= 4 ? 8 / wpr : 1;          // rows per CTA
+    const int nc = (n + wpr - 1) / wpr;              // rounds
     const int warps = wpr * rpc;
     const size_t smem = (size_t)warps * (C + 32) * 4 + 8 * 4;
     dim3 grid((a.L + rpc - 1) / rpc), block(32 * warps);
@@ -296,12 +316,11 @@ cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
             }                                                                                  \
             sgat_quant_kernel<E, NCV, Tin><<<grid, block, smem, stream>>>(a, wpr, rpc);        \
         }
-    if (E * nc > 128 || nc > 5) return cudaErrorInvalidValue;
     switch (nc) {
         case 1: STARQ_QUANT_LAUNCH(1); break;
-        case 2: if constexpr (E <= 64) STARQ_QUANT_LAUNCH(2); break;
-        case 3: if constexpr (E <= 32) STARQ_QUANT_LAUNCH(3); break;
-        case 4: if constexpr (E <= 32) STARQ_QUANT_LAUNCH(4); break;
+        case 2: STARQ_QUANT_LAUNCH(2); break;
+        case 3: STARQ_QUANT_LAUNCH(3); break;
+        case 4: STARQ_QUANT_LAUNCH(4); break;
         case 5: if constexpr (E <= 16) STARQ_QUANT_LAUNCH(5); break;
         default: return cudaErrorInvalidValue;
     }
@@ -311,15 +330,9 @@ cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
 
 template <typename Tin>
 cudaError_t launch_typed(const QuantArgs& a, cudaStream_t stream) {
-    // chunk = one Hadamard block when hb >= 512, else 512 elements
-    const int C = a.hb >= 512 ? a.hb : 512;
-    switch (C) {
-        case 512: return launch_e<16, Tin>(a, stream);
-        case 1024: return launch_e<32, Tin>(a, stream);
-        case 2048: return launch_e<64, Tin>(a, stream);
-        case 4096: return launch_e<128, Tin>(a, stream);
-        default: return cudaErrorInvalidValue;
-    }
+    // a warp's chunk: 1024 elements when hb >= 1024 (larger blocks finish
+    // across warps), else 512 elements holding 512 / hb blocks
+    return a.hb >= 1024 ? launch_e<32, Tin>(a, stream) : launch_e<16, Tin>(a, stream);
 }
 
 }  // namespace
