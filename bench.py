@@ -219,11 +219,11 @@ def run_ours(args):
     reps = 20
     t_quant_x = time_kernel(lambda: abi.sgat_quantize_act(step.X, step.mask, q.a_m, q.a_u, q.hb, q.d_sh, q.d_m,
                                                           q.d_u, Xq, s_a, Xe=Xe), flush, reps, torch)
-    t_gemm_qkv = time_kernel(lambda: abi.w4a4_gemm(None, s_a, q.Wq, q.s_w, step.Y_qkv, Xe=Xe), flush, reps, torch)
+    t_gemm_qkv = time_kernel(lambda: abi.w4a4_gemm(None, s_a, q.Wq, q.s_w, step.Y_qkv, Xe=Xe, We=q.We), flush, reps, torch)
     t_tac = time_kernel(lambda: abi.tac_apply(step.Z, o.tac_M, o.tac_d, o.tac_g, zt), flush, reps, torch)
     t_quant_z = time_kernel(lambda: abi.sgat_quantize_act(zt, step.mask, o.a_m, o.a_u, o.hb, o.d_sh, o.d_m,
                                                           o.d_u, Xq, s_a, Xe=Xe), flush, reps, torch)
-    t_gemm_o = time_kernel(lambda: abi.w4a4_gemm(None, s_a, o.Wq, o.s_w, step.Y_o, Xe=Xe), flush, reps, torch)
+    t_gemm_o = time_kernel(lambda: abi.w4a4_gemm(None, s_a, o.Wq, o.s_w, step.Y_o, Xe=Xe, We=o.We), flush, reps, torch)
     abi.check_status()
 
     # timed region: exactly `steps` steps, device-timed per step
@@ -301,8 +301,9 @@ def run_ours(args):
     quant_z_bytes = L * K * 4 + L * K // 2 + L * K + 4 * L
     tac_bytes = L * K * 2 + L * K * 4 + K * o.tac_g * 4 + K * 4
     traffic = profiled_traffic()
-    gemm_bytes = [L * K + q.N * K // 2 + 2 * L * q.N + 4 * (L + q.N),    # E4M3 codes, packed weights, fp16 out
-                  L * K + o.N * K // 2 + 2 * L * o.N + 4 * (L + o.N)]
+    wbytes = lambda lin: lin.N * K if lin.We is not None else lin.N * K // 2
+    gemm_bytes = [L * K + wbytes(q) + 2 * L * q.N + 4 * (L + q.N),    # E4M3 codes, weights, fp16 out
+                  L * K + wbytes(o) + 2 * L * o.N + 4 * (L + o.N)]
 
     if rank != 0:
         return None
@@ -318,7 +319,7 @@ def run_ours(args):
         "config": config_dict(graph),
         "tokens_per_s": round(tokens_s, 1),
         "roofline": {
-            "bound": "tensor", "kernel": "w4a4_gemm_pair_kernel (QKV + O launches)",
+            "bound": "tensor", "kernel": "w4a4_gemm_tma_pair_kernel (QKV + O launches)",
             "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
             "frac": round(achieved / peak, 4), "traffic": traffic,
             "peak_source": f"{peak_src} bf16 dense burst x {FP8_PER_BF16} (fp8 kind::f8f6f4 path; "

@@ -112,6 +112,21 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
                         int bits, uint8_t* Wq, float* s_w, void* stream);
 
 /*
+ * w4_unpack_e4m3 -- the prepared weight codes in the byte form the tensor
+ * cores read: each int4 code q of Wq becomes the E4M3 byte of the value q
+ * (exact: every integer of [-8, 8] is an E4M3 number). Run once per weight
+ * after sgat_prepare_weight and keep We with Wq and s_w; w4a4_gemm and
+ * sgat_linear then stream both operands by TMA without converting them.
+ * (The paper has no counterpart: its int4 codes are unchanged, only their
+ * storage for this GPU's FP8 tensor-core kind.)
+ *
+ *   Wq [N][K/2] packed int4 (low nibble = even k), 16-byte aligned.
+ *   We [N][K] out, 16-byte aligned, caller-owned (N*K bytes).
+ * Shapes: N >= 0, K >= 32 with K % 32 == 0.
+ */
+int w4_unpack_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
+
+/*
  * w4a4_gemm -- the shared-weight integer projection and its dequantisation
  * (Sec. 3.2 Eq. 13, Sec. 3.1 Eq. 5 and Eq. 3).
  *
@@ -121,9 +136,13 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
  *
  *   Xq [L][K/2], Wq [N][K/2] packed int4, 16-byte aligned.
  *   Xe [L][K] the activation codes as E4M3 bytes (sgat_quantize_act's Xe
- *      output), 16-byte aligned, or NULL. When given, Xq may be NULL and the
- *      kernel streams Xe by TMA to CTA pairs (tcgen05 cta_group::2) that
- *      convert only the weights; otherwise it converts both operands.
+ *      output), 16-byte aligned, or NULL (then Xq is read).
+ *   We [N][K] the weight codes as E4M3 bytes (w4_unpack_e4m3), 16-byte
+ *      aligned, or NULL (then Wq is read). Used only together with Xe.
+ *   Kernels: Xe and We: TMA streams both operands to CTA pairs (tcgen05
+ *   cta_group::2, FP8 kind, float32 accumulators that hold the integer sums
+ *   exactly); Xe only: the pairs convert the packed weights on the fly;
+ *   neither: one CTA per tile converts both.
  *   s_a [L], s_w [N] float32; bias [N] float32 or NULL.
  *   Y  [L][N] out, y_dtype F16, BF16 or F32, 16-byte aligned.
  *   acc_dbg [L][N] int32 out (the exact accumulators) or NULL.
@@ -131,8 +150,8 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
  * K <= 65536 (so |acc| <= 49 K < 2^22).
  */
 int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq,
-              const float* s_w, const float* bias, int L, int N, int K, void* Y, int y_dtype,
-              int32_t* acc_dbg, void* stream);
+              const uint8_t* We, const float* s_w, const float* bias, int L, int N, int K, void* Y,
+              int y_dtype, int32_t* acc_dbg, void* stream);
 
 /*
  * tac_apply -- block-wise affine compensation of the quantised attention
@@ -159,8 +178,9 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  * sgat_quantize_act -> w4a4_gemm, with the intermediates in `workspace`.
  *
  *   tac_M, tac_d, tac_g: TAC parameters as for tac_apply, or tac_M = NULL
- *   for no TAC. Wq/s_w come from sgat_prepare_weight. Other arguments as in
- *   the calls above. K % 128 == 0.
+ *   for no TAC. Wq/s_w come from sgat_prepare_weight, We (optional, NULL =
+ *   convert Wq on the fly) from w4_unpack_e4m3. Other arguments as in the
+ *   calls above. K % 128 == 0.
  *   workspace: device buffer of at least sgat_linear_workspace_size(L, K,
  *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller. On return it
  *   holds the intermediates, laid out as [packed codes Xq: L*K/2 bytes,
@@ -171,8 +191,8 @@ size_t sgat_linear_workspace_size(int L, int K, int with_tac);
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
                 const float* tac_M, const float* tac_d, int tac_g,
-                const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
-                void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
+                const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N,
+                int bits, void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * sgat_linear_noalloc -- sgat_linear for callers that cannot allocate device
@@ -207,8 +227,8 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
 int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                         const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
                         const float* tac_M, const float* tac_d, int tac_g,
-                        const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
-                        void* Y, int y_dtype, void* stream);
+                        const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias,
+                        int N, int bits, void* Y, int y_dtype, void* stream);
 
 #ifdef __cplusplus
 }

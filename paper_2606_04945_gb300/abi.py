@@ -18,7 +18,7 @@ OK, ERR_ARG, ERR_SHAPE, ERR_ALIGN, ERR_BITS, ERR_CUDA, ERR_TIMEOUT = 0, -1, -2, 
 
 EXPORTED = (
     "starq_version", "starq_last_error", "starq_check_status",
-    "sgat_quantize_act", "sgat_prepare_weight", "w4a4_gemm", "tac_apply",
+    "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "tac_apply",
     "sgat_linear_workspace_size", "sgat_linear",
 )
 
@@ -40,15 +40,16 @@ def _load():
     lib.starq_check_status.argtypes = [vp]
     lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, i, u8p, f_p, u8p, f_p, vp]
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
-    lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
+    lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, i, vp]
     lib.sgat_linear_workspace_size.argtypes = [i, i, i]
     lib.sgat_linear_workspace_size.restype = ctypes.c_size_t
     lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
-                                u8p, f_p, f_p, i, i, vp, i, vp, ctypes.c_size_t, vp]
+                                u8p, u8p, f_p, f_p, i, i, vp, i, vp, ctypes.c_size_t, vp]
     if hasattr(lib, "sgat_linear_noalloc"):
         lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
-                                            u8p, f_p, f_p, i, i, vp, i, vp]
+                                            u8p, u8p, f_p, f_p, i, i, vp, i, vp]
     return lib
 
 
@@ -100,14 +101,27 @@ def sgat_prepare_weight(W, inv_a_w, hb, Wq, s_w, bits=4, stream=None):
                                    _p(Wq), _p(s_w), _stream(stream)))
 
 
-def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, stream=None):
+def _weight_shape(Wq, We):
+    if Wq is not None:
+        return Wq.shape[0], 2 * Wq.shape[1]
+    return We.shape[0], We.shape[1]
+
+
+def w4_unpack_e4m3(Wq, We, stream=None):
+    """Packed int4 weight codes [N][K/2] -> E4M3 bytes [N][K] (once per weight)."""
+    _contig(Wq, We)
+    N, K = We.shape
+    _check(lib.w4_unpack_e4m3(_p(Wq), N, K, _p(We), _stream(stream)))
+
+
+def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, stream=None):
     """Xq: packed int4 codes [L][K/2] (may be None when Xe is given);
-    Xe: the same codes as E4M3 bytes [L][K] (selects the TMA CTA-pair kernel)."""
-    _contig(Xq, Xe, s_a, Wq, s_w, Y, bias, acc_dbg)
+    Xe: the same codes as E4M3 bytes [L][K] (selects a TMA CTA-pair kernel);
+    We: the weight codes as E4M3 bytes [N][K] (with Xe: both operands by TMA)."""
+    _contig(Xq, Xe, s_a, Wq, We, s_w, Y, bias, acc_dbg)
     L = Y.shape[0]
-    N = Wq.shape[0]
-    K = 2 * Wq.shape[1]
-    _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(s_w), _p(bias), L, N, K, _p(Y),
+    N, K = _weight_shape(Wq, We)
+    _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y),
                          dtype_code(Y), _p(acc_dbg), _stream(stream)))
 
 
@@ -123,12 +137,12 @@ def sgat_linear_workspace_size(L, K, with_tac):
 
 
 def sgat_linear(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, workspace, bias=None,
-                tac_M=None, tac_d=None, tac_g=0, bits=4, stream=None):
-    _contig(X, mask, a_m, a_u, Wq, s_w, Y, workspace, bias, tac_M, tac_d)
+                tac_M=None, tac_d=None, tac_g=0, bits=4, We=None, stream=None):
+    _contig(X, mask, a_m, a_u, Wq, We, s_w, Y, workspace, bias, tac_M, tac_d)
     L, K = X.shape
-    N = Wq.shape[0]
+    N = _weight_shape(Wq, We)[0]
     _check(lib.sgat_linear(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh, d_m,
-                           d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(s_w), _p(bias), N, bits,
+                           d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(We), _p(s_w), _p(bias), N, bits,
                            _p(Y), dtype_code(Y), _p(workspace), workspace.numel() * workspace.element_size(),
                            _stream(stream)))
 
@@ -137,12 +151,12 @@ NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
 def sgat_linear_noalloc(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, bias=None,
-                        tac_M=None, tac_d=None, tac_g=0, bits=4, stream=None):
+                        tac_M=None, tac_d=None, tac_g=0, bits=4, We=None, stream=None):
     """sgat_linear without a workspace: the library's fixed device scratch
     array holds the intermediates (see include/starq.h)."""
-    _contig(X, mask, a_m, a_u, Wq, s_w, Y, bias, tac_M, tac_d)
+    _contig(X, mask, a_m, a_u, Wq, We, s_w, Y, bias, tac_M, tac_d)
     L, K = X.shape
-    N = Wq.shape[0]
+    N = _weight_shape(Wq, We)[0]
     _check(lib.sgat_linear_noalloc(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh,
-                                   d_m, d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(s_w), _p(bias), N,
+                                   d_m, d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(We), _p(s_w), _p(bias), N,
                                    bits, _p(Y), dtype_code(Y), _stream(stream)))

@@ -72,9 +72,10 @@ int check_tac(int L, int C, int g, const float* M, const float* d) {
     return STARQ_OK;
 }
 
-int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq, const float* s_w,
-               const float* bias, int L, int N, int K, void* Y, int y_dtype) {
-    if (!Wq || !s_w) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Wq or s_w");
+int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq, const uint8_t* We,
+               const float* s_w, const float* bias, int L, int N, int K, void* Y, int y_dtype) {
+    if ((!Wq && !We) || !s_w) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Wq/We or s_w");
+    if (L > 0 && !Wq && !Xe) return fail(STARQ_ERR_ARG, "w4a4_gemm: We without Xe needs Wq");
     if (L > 0 && ((!Xq && !Xe) || !s_a || !Y)) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Xq/Xe, s_a or Y");
     if (!dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "w4a4_gemm: unknown output dtype %d", y_dtype);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
@@ -82,9 +83,9 @@ int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uin
     if (K < 128 || K % 128 != 0 || K > 65536)
         return fail(STARQ_ERR_SHAPE, "K=%d: need 128 <= K <= 65536 and K %% 128 == 0", K);
     if (L == 0) return STARQ_OK;  // nothing is read or written
-    if (!aligned(Xq, 16) || !aligned(Xe, 16) || !aligned(Wq, 16) || !aligned(Y, 16) || !aligned(s_w, 16) ||
-        (bias && !aligned(bias, 16)) || !aligned(s_a, 4))
-        return fail(STARQ_ERR_ALIGN, "w4a4_gemm: Xq, Xe, Wq, Y, s_w, bias must be 16-byte aligned");
+    if (!aligned(Xq, 16) || !aligned(Xe, 16) || !aligned(Wq, 16) || !aligned(We, 16) || !aligned(Y, 16) ||
+        !aligned(s_w, 16) || (bias && !aligned(bias, 16)) || !aligned(s_a, 4))
+        return fail(STARQ_ERR_ALIGN, "w4a4_gemm: Xq, Xe, Wq, We, Y, s_w, bias must be 16-byte aligned");
     return STARQ_OK;
 }
 
@@ -167,15 +168,25 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
     return STARQ_OK;
 }
 
-int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq,
+int w4_unpack_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream) {
+    if (N > 0 && (!Wq || !We)) return fail(STARQ_ERR_ARG, "w4_unpack_e4m3: NULL Wq or We");
+    if (N < 0 || K < 32 || K % 32 != 0) return fail(STARQ_ERR_SHAPE, "w4_unpack_e4m3: N=%d K=%d (K %% 32 == 0)", N, K);
+    if (N == 0) return STARQ_OK;
+    if (!aligned(Wq, 16) || !aligned(We, 16)) return fail(STARQ_ERR_ALIGN, "w4_unpack_e4m3: Wq, We alignment");
+    cudaError_t e = launch_unpack_e4m3(Wq, We, (size_t)N, K, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w4_unpack_e4m3 launch");
+    return STARQ_OK;
+}
+
+int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq, const uint8_t* We,
               const float* s_w, const float* bias, int L, int N, int K, void* Y, int y_dtype,
               int32_t* acc_dbg, void* stream) {
-    int rc = check_gemm(Xq, Xe, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
+    int rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     if (acc_dbg && !aligned(acc_dbg, 16)) return fail(STARQ_ERR_ALIGN, "acc_dbg must be 16-byte aligned");
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
-    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe};
+    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe, Xe ? We : nullptr};
     cudaError_t e = launch_w4a4_gemm(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm launch");
     return STARQ_OK;
@@ -207,9 +218,9 @@ size_t sgat_linear_workspace_size(int L, int K, int with_tac) {
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
                 const float* tac_M, const float* tac_d, int tac_g,
-                const uint8_t* Wq, const float* s_w, const float* bias, int N, int bits,
+                const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
                 void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
-    if (!Wq || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear: NULL Wq or s_w");
+    if ((!Wq && !We) || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear: NULL Wq/We or s_w");
     if (L > 0 && (!X || !Y || !workspace)) return fail(STARQ_ERR_ARG, "sgat_linear: NULL X, Y or workspace");
     if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear: unknown dtype");
     if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
@@ -227,7 +238,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     float* s_a = reinterpret_cast<float*>(ws + align256((size_t)L * K / 2));
     uint8_t* Xe = ws + align256((size_t)L * K / 2) + align256((size_t)L * 4);
     float* zt = tac_M ? reinterpret_cast<float*>(Xe + align256((size_t)L * K)) : nullptr;
-    rc = check_gemm(Xq, Xe, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype);
+    rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
@@ -243,7 +254,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     }
     QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");
-    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe};
+    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
     if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: gemm launch");
     return STARQ_OK;
 }

@@ -43,9 +43,12 @@ struct GemmArgs {
     const float* bias; int L; int N; int K;
     void* Y; int y_dtype; int32_t* acc_dbg;
     unsigned* status;
-    const uint8_t* Xe = nullptr;   // optional E4M3 bytes of the codes [L][K]
+    const uint8_t* Xe = nullptr;   // optional E4M3 bytes of the activation codes [L][K]
+    const uint8_t* We = nullptr;   // optional E4M3 bytes of the weight codes [N][K]
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+// Packed int4 codes [rows][K/2] -> E4M3 bytes [rows][K].
+cudaError_t launch_unpack_e4m3(const uint8_t* packed, uint8_t* e4m3, size_t rows, int K, cudaStream_t stream);
 
 struct TacArgs {
     const void* Z; int z_dtype; int L; int C; int g;
@@ -92,6 +95,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// One lane of a converged warp (the lowest active lane) gets true.
+__device__ __forceinline__ bool elect_one() {
+    uint32_t pred;
+    asm volatile("{\n\t.reg .pred p;\n\t.reg .b32 r;\n\t"
+                 "elect.sync r|p, 0xffffffff;\n\t"
+                 "selp.u32 %0, 1, 0, p;\n\t}" : "=r"(pred));
+    return pred != 0;
+}
+
 // Wait for the phase of `bar` with the given parity to complete. Gives up
 // (returns false) after WAIT_LIMIT_NS, or early when *abort is set by another
 // role of the same CTA that has already given up.
@@ -107,6 +119,12 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
         if (*abort) return false;
         if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) return false;
     }
+}
+
+// Whole-warp form: every lane waits; the result is the same in every lane.
+__device__ __forceinline__ bool mbar_wait_bounded_warp(uint32_t bar, uint32_t parity, volatile int* abort) {
+    const bool ok = mbar_wait_bounded(bar, parity, abort);
+    return __all_sync(0xffffffffu, ok);
 }
 
 __device__ __forceinline__ void fence_proxy_async_smem() {
@@ -250,6 +268,24 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, int 
     asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
                  " [%0], [%1, {%2, %3}], [%4];"
                  :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar) : "memory");
+}
+// 2-D TMA tile load into this CTA's shared memory whose completion is
+// counted on an mbarrier of either CTA of the pair (shared::cluster
+// address `bar`).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap, int x, int y,
+                                                 uint32_t bar) {
+    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2"
+                 " [%0], [%1, {%2, %3}], [%4];"
+                 :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar) : "memory");
+}
+// Pair form with cluster multicast: the tile lands at `dst` in every CTA of
+// `cta_mask`; each destination's bytes are counted on the barrier at `bar`'s
+// offset in the even (leader) CTA of that destination's pair.
+__device__ __forceinline__ void tma_load_2d_pair_multicast(uint32_t dst, const void* tmap, int x, int y,
+                                                           uint32_t bar, uint16_t cta_mask) {
+    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+                 ".cta_group::2 [%0], [%1, {%2, %3}], [%4], %5;"
+                 :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar), "h"(cta_mask) : "memory");
 }
 // Same, with the tile (and the completion on `bar`) delivered to the same
 // shared-memory offsets in every CTA of `cta_mask`.

@@ -692,6 +692,326 @@ bool encode_u8_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// ---------------------------------------------------------------------------
+// CTA-pair GEMM with both operands as E4M3 bytes by TMA (activation codes
+// from the quantiser, weight codes from w4_unpack_e4m3).
+//
+// The standard two-barrier pipeline: the TMA producer of each CTA waits for
+// the stage to be free (the MMA commits, multicast to the cluster) and loads
+// its 128 activation rows and 128 weight rows, the bytes counted on the
+// pair leader's stage barrier (cta_group::2); the leader's MMA thread waits
+// there and issues the four K = 32 MMAs of the stage (M 256, N 256).
+// CL = 4: two pairs on the same token rows and neighbouring channel tiles;
+// CTAs r and r ^ 2 need the same activation rows, so each loads half of
+// them and multicasts it to both, and a stage is free once both pairs'
+// MMAs have read it. 6 stages of 32 KB; 8 epilogue warps.
+// ---------------------------------------------------------------------------
+namespace tmak {
+constexpr int BM = 128, BN = 256, BN_CTA = 128, BK = 128, UMMA_K = 32;
+constexpr int STAGES = 6;
+constexpr int A_BYTES = BM * BK, B_BYTES = BN_CTA * BK;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;             // 32 KB
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int TMA_WARP = 8, MMA_WARP = 9;
+constexpr int THREADS = 10 * 32;
+constexpr int TMEM_COLS = 512;
+constexpr int EPI_PARAM_BYTES = NUM_EPI_WARPS * 2 * (BN / 2) * 4;
+constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
+constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
+struct Smem {
+    uint64_t full[STAGES];        // pair leader: both CTAs' TMA bytes
+    uint64_t empty[STAGES];       // MMA commits of every pair of the cluster
+    uint64_t tmem_full[2];
+    uint64_t tmem_empty[2];       // pair leader: epilogue warps of the pair
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+};
+}  // namespace tmak
+
+template <typename TOut, int CL>
+__global__ void __launch_bounds__(tmak::THREADS, 1)
+w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
+                          const __grid_constant__ CUtensorMap tmap_b) {
+    constexpr int BM = tmak::BM, BN = tmak::BN, BN_CTA = tmak::BN_CTA, BK = tmak::BK;
+    constexpr int UMMA_K = tmak::UMMA_K, STAGES = tmak::STAGES, STAGE_BYTES = tmak::STAGE_BYTES;
+    constexpr int A_BYTES = tmak::A_BYTES, B_BYTES = tmak::B_BYTES;
+    constexpr int TMA_WARP = tmak::TMA_WARP, MMA_WARP = tmak::MMA_WARP;
+    constexpr int NUM_EPI_WARPS = tmak::NUM_EPI_WARPS, TMEM_COLS = tmak::TMEM_COLS;
+    constexpr uint32_t IDESC = tmak::IDESC;
+    constexpr int PAIRS = CL / 2;
+    constexpr uint16_t ALL = (uint16_t)((1u << CL) - 1u);
+    using Smem = tmak::Smem;
+    static_assert(CL == 2 || CL == 4, "one or two CTA pairs per cluster");
+
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_addr(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    Smem* sh = reinterpret_cast<Smem*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES);
+    volatile int* abort = &sh->abort;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const uint32_t half = rank & 1u, pr = rank >> 1, leader = rank & ~1u;
+    const uint16_t pair_mask = (uint16_t)(3u << (2 * pr));
+    const int L = a.L, N = a.N, K = a.K;
+    const int num_m = (L + 2 * BM - 1) / (2 * BM);
+    const int num_n = (N + BN - 1) / BN;
+    const int num_tiles = num_m * ((num_n + PAIRS - 1) / PAIRS);
+    const int num_k = K / BK;
+    const int cluster = blockIdx.x / CL, num_clusters = gridDim.x / CL;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(smem_addr(&sh->full[s]), 1);
+            mbar_init(smem_addr(&sh->empty[s]), PAIRS);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_addr(&sh->tmem_full[b]), 1);
+            mbar_init(smem_addr(&sh->tmem_empty[b]), 2 * NUM_EPI_WARPS);
+        }
+        mbar_init(smem_addr(&sh->drain), 1);
+        sh->abort = 0;
+        mbar_fence_init();
+    }
+    if (warp == MMA_WARP) {
+        tmem_alloc_pair(smem_addr(&sh->tmem_base), TMEM_COLS);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    cluster_sync();              // barriers of every CTA initialised, TMEM allocated
+    tc_fence_after();
+    const uint32_t tmem_base = sh->tmem_base;
+
+    // The producer and MMA roles run their loops with the whole warp (warp-
+    // uniform control flow and descriptors); one elected lane issues.
+    if (warp == TMA_WARP) {
+        const uint32_t leader_full0 = mapa_shared(smem_addr(&sh->full[0]), leader);
+        const uint16_t a_mask = (uint16_t)((1u << rank) | (1u << ((rank ^ 2u) % CL)));
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters) {
+            const int m_rows = (tile % num_m) * 2 * BM + (int)half * BM;
+            const int n_rows = ((tile / num_m) * PAIRS + (int)pr) * BN + (int)half * BN_CTA;
+            for (int kc = 0; kc < num_k; ++kc) {
+                if (!mbar_wait_bounded_warp(smem_addr(&sh->empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
+                const uint32_t st = base + stage * STAGE_BYTES;
+                const uint32_t bar = leader_full0 + stage * 8;
+                if (elect_one()) {
+                    if (half == 0) mbar_arrive_expect_tx(smem_addr(&sh->full[stage]), 2 * (A_BYTES + B_BYTES));
+                    if (CL == 2) {
+                        tma_load_2d_pair(st, &tmap_a, kc * BK, m_rows, bar);
+                    } else {
+                        tma_load_2d_pair_multicast(st + pr * (A_BYTES / 2), &tmap_a, kc * BK,
+                                                   m_rows + (int)pr * (BM / 2), bar, a_mask);
+                    }
+                    tma_load_2d_pair(st + A_BYTES, &tmap_b, kc * BK, n_rows, bar);
+                }
+                __syncwarp();
+                if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+            }
+        }
+        if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
+        __syncwarp();
+    } else if (warp == MMA_WARP) {
+        if (half == 0) {
+            const uint64_t desc0 = smem_desc_sw128(base);     // start-address field: base >> 4
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            int it = 0;
+            for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters, ++it) {
+                const int acc = it & 1;
+                const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+                if (!mbar_wait_bounded_warp(smem_addr(&sh->tmem_empty[acc]), acc_phase ^ 1u, abort)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+                for (int kc = 0; kc < num_k; ++kc) {
+                    if (!mbar_wait_bounded_warp(smem_addr(&sh->full[stage]), phase, abort)) { ok = false; break; }
+                    tc_fence_after();
+                    // stage offsets stay below 2^18 bytes, so adding them to
+                    // the start-address field never carries out of it
+                    const uint64_t ad = desc0 + (uint64_t)((stage * STAGE_BYTES) >> 4);
+                    const uint64_t bd = ad + (uint64_t)(A_BYTES >> 4);
+                    if (elect_one()) {
+                        #pragma unroll
+                        for (int ks = 0; ks < BK / UMMA_K; ++ks)
+                            mma_f8f6f4_pair(d_tmem, ad + (uint64_t)(ks * UMMA_K / 16), bd + (uint64_t)(ks * UMMA_K / 16),
+                                            IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
+                        tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), ALL);
+                    }
+                    __syncwarp();
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->tmem_full[acc]), pair_mask);
+                __syncwarp();
+            }
+            if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->drain), pair_mask);
+            __syncwarp();
+            if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
+        }
+        __syncwarp();
+    } else {
+        // epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31, columns
+        // (w / 4) * 128 .. + 127; scales and biases staged before the wait
+        const uint32_t leader_tmem_empty0 = mapa_shared(smem_addr(&sh->tmem_empty[0]), leader);
+        float* epi_sw = reinterpret_cast<float*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES + sizeof(Smem) +
+                                                 (16 - sizeof(Smem) % 16) % 16) + warp * 2 * (BN / 2);
+        float* epi_b = epi_sw + BN / 2;
+        const int quarter = warp & 3, chalf = warp >> 2;
+        bool ok = true;
+        int it = 0;
+        TOut* Y = static_cast<TOut*>(a.Y);
+        for (int tile = cluster; tile < num_tiles; tile += num_clusters, ++it) {
+            const int m0 = (tile % num_m) * 2 * BM + (int)half * BM;
+            const int n0 = ((tile / num_m) * PAIRS + (int)pr) * BN;
+            const int acc = it & 1;
+            const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+            const int row = m0 + quarter * 32 + lane;
+            const bool valid = row < L;
+            const float sa = valid ? __ldg(a.s_a + row) : 0.f;
+            {
+                const int ncol = n0 + chalf * (BN / 2) + 4 * lane;
+                float4 w = make_float4(0.f, 0.f, 0.f, 0.f), bb = w;
+                if (ncol < N) {
+                    w = __ldg(reinterpret_cast<const float4*>(a.s_w + ncol));
+                    if (a.bias != nullptr) bb = __ldg(reinterpret_cast<const float4*>(a.bias + ncol));
+                }
+                __syncwarp();
+                reinterpret_cast<float4*>(epi_sw)[lane] = w;
+                reinterpret_cast<float4*>(epi_b)[lane] = bb;
+                __syncwarp();
+            }
+            if (!mbar_wait_bounded(smem_addr(&sh->tmem_full[acc]), acc_phase, abort)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t t_row = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+            #pragma unroll 1
+            for (int cc = 0; cc < BN / 64; ++cc) {
+                const int c = chalf * (BN / 64) + cc;
+                const int nc = n0 + c * 32;
+                if (nc >= N) break;
+                uint32_t r[32];
+                tmem_ld_32x32b_x32(t_row + c * 32, r);
+                tmem_ld_wait();
+                if (valid) {
+                    float y[32];
+                    const float4* sw4 = reinterpret_cast<const float4*>(epi_sw + cc * 32);
+                    const float4* b4 = reinterpret_cast<const float4*>(epi_b + cc * 32);
+                    #pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const float4 sw = sw4[u];
+                        y[4 * u] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u]), sa), sw.x);
+                        y[4 * u + 1] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 1]), sa), sw.y);
+                        y[4 * u + 2] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 2]), sa), sw.z);
+                        y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
+                    }
+                    if (a.bias != nullptr) {
+                        #pragma unroll
+                        for (int u = 0; u < 8; ++u) {
+                            const float4 bq = b4[u];
+                            y[4 * u] = __fadd_rn(y[4 * u], bq.x);
+                            y[4 * u + 1] = __fadd_rn(y[4 * u + 1], bq.y);
+                            y[4 * u + 2] = __fadd_rn(y[4 * u + 2], bq.z);
+                            y[4 * u + 3] = __fadd_rn(y[4 * u + 3], bq.w);
+                        }
+                    }
+                    Out<TOut>::store32(Y + (size_t)row * N + nc, y);
+                    if (a.acc_dbg != nullptr) {
+                        int4* d4 = reinterpret_cast<int4*>(a.acc_dbg + (size_t)row * N + nc);
+                        #pragma unroll
+                        for (int u = 0; u < 8; ++u)
+                            d4[u] = make_int4(__float2int_rn(__uint_as_float(r[4 * u])),
+                                              __float2int_rn(__uint_as_float(r[4 * u + 1])),
+                                              __float2int_rn(__uint_as_float(r[4 * u + 2])),
+                                              __float2int_rn(__uint_as_float(r[4 * u + 3])));
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + acc * 8);
+        }
+        if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
+    }
+
+    // every MMA the pair's leader issued has completed before TMEM is released
+    if (warp == MMA_WARP && lane == 0) {
+        volatile int never = 0;
+        if (!mbar_wait_bounded(smem_addr(&sh->drain), 0, &never)) atomicOr(a.status, STATUS_TIMEOUT_GEMM);
+    }
+    __syncwarp();
+    tc_fence_before();
+    cluster_sync();              // no CTA leaves while another may still signal it
+    tc_fence_after();
+    if (warp == MMA_WARP) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+}
+
+template <typename TOut, int CL>
+cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
+    constexpr int BM = tmak::BM, BN = tmak::BN, BN_CTA = tmak::BN_CTA, BK = tmak::BK;
+    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL>;
+    static bool attr_set[64] = {false};
+    static int max_clusters[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(tmak::THREADS);
+    cfg.dynamicSmemBytes = tmak::SMEM_BYTES;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (dev < 64 && !attr_set[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)tmak::SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        cfg.gridDim = dim3(CL * 32);
+        int n = 0;
+        e = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg);
+        if (e != cudaSuccess) return e;
+        max_clusters[dev] = n;
+        attr_set[dev] = true;
+    }
+    CUtensorMap ta, tb;
+    if (!encode_u8_tmap(&ta, a.Xe, (uint64_t)a.L, (uint64_t)a.K, CL == 2 ? BM : BM / 2, BK,
+                        CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_u8_tmap(&tb, a.We, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK, CU_TENSOR_MAP_SWIZZLE_128B))
+        return cudaErrorInvalidValue;
+    const int num_n = (a.N + BN - 1) / BN;
+    const int num_tiles = ((a.L + 2 * BM - 1) / (2 * BM)) * ((num_n + CL / 2 - 1) / (CL / 2));
+    int clusters = dev < 64 ? max_clusters[dev] : 1;
+    if (clusters < 1) clusters = 1;
+    if (num_tiles < clusters) clusters = num_tiles;
+    cfg.gridDim = dim3(CL * clusters);
+    return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb);
+}
+
+template <typename TOut>
+cudaError_t launch_tma_typed(const GemmArgs& a, cudaStream_t stream) {
+    const int num_n = (a.N + tmak::BN - 1) / tmak::BN;
+    return num_n >= 2 ? launch_tma_cl<TOut, 4>(a, stream) : launch_tma_cl<TOut, 2>(a, stream);
+}
+
+// Packed int4 -> E4M3: each thread turns 16 packed bytes into 32 E4M3 bytes.
+__global__ void __launch_bounds__(256) unpack_e4m3_kernel(const uint4* __restrict__ packed,
+                                                          uint4* __restrict__ out, size_t n16) {
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += (size_t)gridDim.x * blockDim.x) {
+        const uint4 w = ld_global_nc_v4(packed + i);
+        uint32_t o[8];
+        int4x8_to_e4m3x8(w.x, o[0], o[1]);
+        int4x8_to_e4m3x8(w.y, o[2], o[3]);
+        int4x8_to_e4m3x8(w.z, o[4], o[5]);
+        int4x8_to_e4m3x8(w.w, o[6], o[7]);
+        out[2 * i] = make_uint4(o[0], o[1], o[2], o[3]);
+        out[2 * i + 1] = make_uint4(o[4], o[5], o[6], o[7]);
+    }
+}
+
 // Cluster size of the CTA-pair GEMM: 4 (two pairs sharing the activation
 // tile by multicast) unless fewer than two clusters of 4 fit, then 2.
 template <typename TOut, int CL>
@@ -770,8 +1090,27 @@ cudaError_t launch_typed(const GemmArgs& a, cudaStream_t stream) {
 
 }  // namespace
 
+cudaError_t launch_unpack_e4m3(const uint8_t* packed, uint8_t* e4m3, size_t rows, int K, cudaStream_t stream) {
+    const size_t n16 = rows * (size_t)K / 32;
+    if (n16 == 0) return cudaSuccess;
+    size_t blocks = (n16 + 255) / 256;
+    const size_t cap = (size_t)num_sms() * 8;
+    if (blocks > cap) blocks = cap;
+    unpack_e4m3_kernel<<<(unsigned)blocks, 256, 0, stream>>>(reinterpret_cast<const uint4*>(packed),
+                                                               reinterpret_cast<uint4*>(e4m3), n16);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {
     if (a.L == 0) return cudaSuccess;
+    if (a.Xe != nullptr && a.We != nullptr) {
+        switch (a.y_dtype) {
+            case STARQ_F16: return launch_tma_typed<__half>(a, stream);
+            case STARQ_BF16: return launch_tma_typed<__nv_bfloat16>(a, stream);
+            case STARQ_F32: return launch_tma_typed<float>(a, stream);
+            default: return cudaErrorInvalidValue;
+        }
+    }
     if (a.Xe != nullptr) {
         switch (a.y_dtype) {
             case STARQ_F16: return launch_pair_typed<__half>(a, stream);

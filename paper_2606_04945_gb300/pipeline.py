@@ -1,8 +1,9 @@
 """Device-resident SGAT W4A4 layers built on the C ABI.
 
 ``SgatLinear`` holds one quantised linear on the GPU: the folded int4
-weight (Eq. 12, prepared once by ``sgat_prepare_weight``), the two state
-transforms, optional TAC parameters and a workspace. ``run`` is one call to
+weight (Eq. 12, prepared once by ``sgat_prepare_weight``) and, by default,
+the same codes as E4M3 bytes for the tensor cores (``w4_unpack_e4m3``), the
+two state transforms, optional TAC parameters and a workspace. ``run`` is one call to
 ``sgat_linear`` (TAC -> state-guided quantisation -> W4A4 GEMM + dequant).
 
 ``AttentionProjections`` is the attention-side hot path of one denoising
@@ -29,7 +30,7 @@ TORCH_DTYPE = {"f16": torch.float16, "bf16": torch.bfloat16, "f32": torch.float3
 
 
 class SgatLinear:
-    def __init__(self, case, device="cuda", out_dtype=None):
+    def __init__(self, case, device="cuda", out_dtype=None, e4m3_weights=True):
         xf = case.xf
         self.L, self.K, self.N = case.L, case.K, case.N
         self.dtype = TORCH_DTYPE[case.dtype]
@@ -51,13 +52,17 @@ class SgatLinear:
         self.s_w = torch.empty(self.N, dtype=torch.float32, device=device)
         abi.sgat_prepare_weight(W, _dev(xf.inv_a_w, device=device), self.hb, self.Wq, self.s_w)
         del W
+        self.We = None
+        if e4m3_weights:
+            self.We = torch.empty(self.N, self.K, dtype=torch.uint8, device=device)
+            abi.w4_unpack_e4m3(self.Wq, self.We)
         self.workspace = torch.empty(abi.sgat_linear_workspace_size(self.L, self.K, self.tac is not None),
                                      dtype=torch.uint8, device=device)
 
     def run(self, X, mask, Y, stream=None):
         abi.sgat_linear(X, mask, self.a_m, self.a_u, self.hb, self.d_sh, self.d_m, self.d_u,
                         self.Wq, self.s_w, Y, self.workspace, bias=self.bias, tac_M=self.tac_M,
-                        tac_d=self.tac_d, tac_g=self.tac_g, stream=stream)
+                        tac_d=self.tac_d, tac_g=self.tac_g, We=self.We, stream=stream)
 
     def int_ops(self, L=None):
         return 2 * (L or self.L) * self.N * self.K
@@ -66,9 +71,9 @@ class SgatLinear:
 class AttentionProjections:
     """QKV projection of X and TAC + O projection of Z for one step."""
 
-    def __init__(self, qkv_case, o_case, device="cuda"):
-        self.qkv = SgatLinear(qkv_case, device)
-        self.o = SgatLinear(o_case, device)
+    def __init__(self, qkv_case, o_case, device="cuda", e4m3_weights=True):
+        self.qkv = SgatLinear(qkv_case, device, e4m3_weights=e4m3_weights)
+        self.o = SgatLinear(o_case, device, e4m3_weights=e4m3_weights)
         self.L = qkv_case.L
         self.X = _dev(qkv_case.X, self.qkv.dtype, device)
         self.Z = _dev(o_case.X, self.o.dtype, device)

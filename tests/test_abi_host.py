@@ -71,14 +71,29 @@ def test_quantize_act_validation(lib, args, code):
 @pytest.mark.parametrize("L,N,K,code", [(4, 100, 512, -2), (4, 256, 200, -2), (4, 256, 131072, -2),
                                         (-1, 256, 512, -2)])
 def test_gemm_validation(lib, L, N, K, code):
-    assert lib.lib.w4a4_gemm(P, None, P, P, P, None, L, N, K, P, 0, None, None) == code
+    assert lib.lib.w4a4_gemm(P, None, P, P, None, P, None, L, N, K, P, 0, None, None) == code
 
 
 def test_gemm_null_and_alignment(lib):
-    assert lib.lib.w4a4_gemm(None, None, P, P, P, None, 4, 256, 512, P, 0, None, None) == -1
-    assert lib.lib.w4a4_gemm(ctypes.c_void_p(4104), None, P, P, P, None, 4, 256, 512, P, 0, None, None) == -3
-    assert lib.lib.w4a4_gemm(None, ctypes.c_void_p(4104), P, P, P, None, 4, 256, 512, P, 0, None, None) == -3
-    assert lib.lib.w4a4_gemm(P, None, P, P, P, None, 4, 256, 512, P, 7, None, None) == -1
+    assert lib.lib.w4a4_gemm(None, None, P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -1
+    assert lib.lib.w4a4_gemm(P, None, P, None, None, P, None, 4, 256, 512, P, 0, None, None) == -1
+    # E4M3 weights need E4M3 activations when there are no packed weights
+    assert lib.lib.w4a4_gemm(P, None, P, None, P, P, None, 4, 256, 512, P, 0, None, None) == -1
+    assert lib.lib.w4a4_gemm(ctypes.c_void_p(4104), None, P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert lib.lib.w4a4_gemm(None, ctypes.c_void_p(4104), P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert lib.lib.w4a4_gemm(None, P, P, None, ctypes.c_void_p(4104), P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert lib.lib.w4a4_gemm(P, None, P, P, None, P, None, 4, 256, 512, P, 7, None, None) == -1
+
+
+@pytest.mark.parametrize("N,K,code", [(-1, 512, -2), (4, 48, -2), (4, 16, -2)])
+def test_unpack_validation(lib, N, K, code):
+    assert lib.lib.w4_unpack_e4m3(P, N, K, P, None) == code
+
+
+def test_unpack_null_and_alignment(lib):
+    assert lib.lib.w4_unpack_e4m3(None, 4, 512, P, None) == -1
+    assert lib.lib.w4_unpack_e4m3(P, 4, 512, ctypes.c_void_p(4100), None) == -3
+    assert lib.lib.w4_unpack_e4m3(None, 0, 512, None, None) == 0
 
 
 @pytest.mark.parametrize("g,C,code", [(12, 96, -2), (16, 100, -2), (256, 4096, -2)])
@@ -96,9 +111,9 @@ def test_linear_workspace_and_validation(lib):
     assert lib.sgat_linear_workspace_size(1024, 4096, True) == n + 1024 * 4096 * 4
     # workspace too small
     rc = lib.lib.sgat_linear(P, 0, 1024, 4096, None, None, None, 4096, 4096, 0, 0, None, None, 0,
-                             P, P, None, 256, 4, P, 0, P, 16, None)
+                             P, None, P, None, 256, 4, P, 0, P, 16, None)
     assert rc == -2 and b"workspace" in lib.lib.starq_last_error()
     # TAC block that does not divide K
     rc = lib.lib.sgat_linear(P, 0, 16, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 48,
-                             P, P, None, 256, 4, P, 0, P, 1 << 30, None)
+                             P, None, P, None, 256, 4, P, 0, P, 1 << 30, None)
     assert rc == -2

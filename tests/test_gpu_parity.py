@@ -104,25 +104,52 @@ def test_prepare_weight_bitexact(abi, N, K, hb, dtype):
     assert np.array_equal(s_w.cpu().numpy(), s)
 
 
+def unpacked_weight(abi, Wq):
+    """The E4M3 weight bytes of packed codes, by w4_unpack_e4m3."""
+    We = torch.empty(Wq.shape[0], 2 * Wq.shape[1], dtype=torch.uint8, device="cuda")
+    abi.w4_unpack_e4m3(Wq, We)
+    return We
+
+
 def run_gemm(abi, qa, qw, s_a, s_w, out="f16", bias=None, path="e4m3"):
     """path "packed": packed int4 activations (both operands converted in the
-    kernel); path "e4m3": E4M3 activation codes streamed by TMA to CTA pairs."""
+    kernel); "e4m3": E4M3 activation codes by TMA to CTA pairs that convert
+    the weights; "tma": both operands as E4M3 bytes by TMA (weights unpacked
+    by w4_unpack_e4m3, checked against the format's definition)."""
     L, K = qa.shape
     N = qw.shape[0]
     Wq = H.dev(osg.pack_int4(qw))
     Y = torch.empty(L, N, dtype=H.torch_dtype(out), device="cuda")
     acc = torch.empty(L, N, dtype=torch.int32, device="cuda")
+    We = None
     if path == "packed":
         Xq, Xe = H.dev(osg.pack_int4(qa)), None
     else:
         Xq, Xe = None, H.dev(H.e4m3_bytes(qa))
+    if path == "tma":
+        We = unpacked_weight(abi, Wq)
+        assert np.array_equal(We.cpu().numpy(), H.e4m3_bytes(qw)), "unpacked weight bytes differ"
+        Wq = None
     abi.w4a4_gemm(Xq, H.dev(s_a), Wq, H.dev(s_w), Y, bias=None if bias is None else H.dev(bias),
-                  acc_dbg=acc, Xe=Xe)
+                  acc_dbg=acc, Xe=Xe, We=We)
     abi.check_status()
     return H.host(Y), acc.cpu().numpy()
 
 
-@pytest.mark.parametrize("path", ["e4m3", "packed"])
+@pytest.mark.parametrize("N,K", [(1, 32), (3, 96), (1000, 4096), (4096, 64)])
+def test_w4_unpack_e4m3(abi, N, K):
+    """Every byte value of the packed codes (both nibbles, -8 included) maps
+    to the E4M3 byte of its integer."""
+    rng = np.random.default_rng(N * 7 + K)
+    packed = rng.integers(0, 256, (N, K // 2), dtype=np.uint8)
+    flat = packed.reshape(-1)
+    flat[: min(256, flat.size)] = np.arange(min(256, flat.size), dtype=np.uint8)
+    We = unpacked_weight(abi, H.dev(packed))
+    abi.check_status()
+    assert np.array_equal(We.cpu().numpy(), H.e4m3_bytes(osg.unpack_int4(packed)))
+
+
+@pytest.mark.parametrize("path", ["tma", "e4m3", "packed"])
 @pytest.mark.parametrize("L,N,K,out", [(1, 256, 128, "f16"), (129, 512, 512, "f16"), (300, 288, 1024, "bf16"),
                                        (128, 256, 4096, "f32"), (1000, 768, 384, "f16"),
                                        (257, 4096, 256, "f16"), (513, 160, 640, "f16")])
@@ -135,7 +162,7 @@ def test_w4a4_gemm_exact(abi, L, N, K, out, path):
     H.assert_output_close(Y, osg.dequant(ref_acc, s_a, s_w, bias), out)
 
 
-@pytest.mark.parametrize("path", ["e4m3", "packed"])
+@pytest.mark.parametrize("path", ["tma", "e4m3", "packed"])
 @pytest.mark.parametrize("K", [18944, 65536])
 def test_w4a4_gemm_adversarial_exactness(abi, K, path):
     """Integer exactness of the float32 tensor-core accumulation: all codes
@@ -189,7 +216,7 @@ def _oracle_linear_from_codes(qa, s_a, qw, s_w, bias):
     return osg.dequant(acc, s_a, s_w, bias), acc
 
 
-def run_linear_case(abi, case, out_dtype=None, check_rows=None):
+def run_linear_case(abi, case, out_dtype=None, check_rows=None, weights="e4m3"):
     """sgat_prepare_weight + sgat_linear on the GPU against the oracle's
     literal split / quantise / GEMM / scatter. With TAC, the TAC output is
     compared within tolerance and the rest of the chain is teacher-forced on
@@ -202,6 +229,7 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None):
     Wq = torch.empty(N, K // 2, dtype=torch.uint8, device="cuda")
     s_w = torch.empty(N, dtype=torch.float32, device="cuda")
     abi.sgat_prepare_weight(W, H.dev(xf.inv_a_w), xf.hb, Wq, s_w)
+    We = unpacked_weight(abi, Wq) if weights == "e4m3" else None
     with_tac = case.tac is not None
     ws = torch.empty(abi.sgat_linear_workspace_size(L, K, with_tac), dtype=torch.uint8, device="cuda")
     Y = torch.empty(L, N, dtype=H.torch_dtype(out_dtype), device="cuda")
@@ -210,7 +238,7 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None):
         kw = dict(tac_M=H.dev(case.tac.M), tac_d=H.dev(case.tac.d), tac_g=case.tac.g)
     bias = H.dev(case.bias) if case.bias is not None else None
     abi.sgat_linear(H.dev(case.X, dt), H.dev(case.mask), H.dev(xf.a_m), H.dev(xf.a_u), xf.hb, xf.d_sh,
-                    xf.d_m, xf.d_u, Wq, s_w, Y, ws, bias=bias, **kw)
+                    xf.d_m, xf.d_u, Wq, s_w, Y, ws, bias=bias, We=We, **kw)
     abi.check_status()
     qw, sw = osg.prepare_weight(case.W, xf.inv_a_w, xf.hb, 4)
     assert np.array_equal(H.unpack(Wq), qw) and np.array_equal(s_w.cpu().numpy(), sw)
@@ -231,31 +259,34 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None):
     return Y
 
 
+@pytest.mark.parametrize("weights", ["e4m3", "packed"])
 @pytest.mark.parametrize("gates", [True, False])
-def test_single_linear_full(abi, gates):
+def test_single_linear_full(abi, gates, weights):
     """Single SGAT linear, 256 x 512 -> 512, with and without gates, with
     and without TAC (block 64)."""
     case = inputs.single_linear(0, gates_on=gates)
-    run_linear_case(abi, case)
+    run_linear_case(abi, case, weights=weights)
     case.tac = None
-    run_linear_case(abi, case)
+    run_linear_case(abi, case, weights=weights)
 
 
-def test_llada_attention_full(abi):
+@pytest.mark.parametrize("weights", ["e4m3", "packed"])
+def test_llada_attention_full(abi, weights):
     """LLaDA-8B attention projections at one step: QKV 1024 x 4096 -> 12288
     and O 4096 -> 4096 with TAC (block 128), full size, every row."""
     qkv, o = inputs.llada_attention(0)
-    run_linear_case(abi, qkv)
-    run_linear_case(abi, o)
+    run_linear_case(abi, qkv, weights=weights)
+    run_linear_case(abi, o, weights=weights)
 
 
 @pytest.mark.parametrize("L,K,N,dtype,tac_g,bias", [(1, 128, 32, "f16", None, False),
                                                     (77, 512, 320, "bf16", 16, True),
                                                     (129, 1024, 256, "f16", 128, False),
                                                     (513, 3584, 512, "bf16", 128, True)])
-def test_sgat_linear_ragged(abi, L, K, N, dtype, tac_g, bias):
+@pytest.mark.parametrize("weights", ["e4m3", "packed"])
+def test_sgat_linear_ragged(abi, L, K, N, dtype, tac_g, bias, weights):
     case = inputs.random_linear(L * 3 + K, L, K, N, dtype=dtype, tac_g=tac_g, bias=bias)
-    run_linear_case(abi, case)
+    run_linear_case(abi, case, weights=weights)
 
 
 def test_empty_batch(abi):
@@ -269,5 +300,9 @@ def test_empty_batch(abi):
     sw = torch.ones(N, dtype=torch.float32, device="cuda")
     Y = torch.empty(0, N, dtype=torch.float16, device="cuda")
     abi.w4a4_gemm(Xq, s, Wq, sw, Y)
-    abi.w4a4_gemm(None, s, Wq, sw, Y, Xe=torch.empty(0, K, dtype=torch.uint8, device="cuda"))
+    Xe0 = torch.empty(0, K, dtype=torch.uint8, device="cuda")
+    abi.w4a4_gemm(None, s, Wq, sw, Y, Xe=Xe0)
+    abi.w4a4_gemm(None, s, None, sw, Y, Xe=Xe0, We=unpacked_weight(abi, Wq))
+    abi.w4_unpack_e4m3(torch.empty(0, K // 2, dtype=torch.uint8, device="cuda"),
+                       torch.empty(0, K, dtype=torch.uint8, device="cuda"))
     abi.check_status()

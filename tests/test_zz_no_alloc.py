@@ -81,5 +81,5 @@ def test_noalloc_symbol_and_limit_declared():
     # the size check runs before any CUDA call
     P = ctypes.c_void_p(4096)
     rc = abi.lib.sgat_linear_noalloc(P, 0, 4096, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 128,
-                                     P, P, None, 256, 4, P, 0, None)
+                                     P, None, P, None, 256, 4, P, 0, None)
     assert rc == abi.ERR_SHAPE
