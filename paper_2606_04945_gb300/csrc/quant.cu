@@ -294,6 +294,246 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Rows with Hadamard blocks of 1024 elements or more (hb >= 1024, K a
+// multiple of 1024, K <= 4096 NR): one CTA of four warps per row, in rounds
+// of 4096 elements (four 1024-element chunks, chunk j of a round in warp j).
+//
+//   layout A  lane l holds elements 32 l .. 32 l + 31 of its warp's chunk:
+//             stages h = 1 .. 16 are between registers;
+//   layout B  lane l holds elements l + 32 i (i = 0 .. 31) of the chunk,
+//             after a transpose through the chunk's shared slice: stages
+//             h = 32 .. 512 are between registers;
+//   layout C  after the round's four chunks are in shared memory, lane l of
+//             warp w holds elements j 1024 + 256 w + 8 l .. + 7 of every
+//             chunk j: stages h = 1024, 2048 are between registers, and the
+//             eight consecutive codes per chunk pack into one 32-bit word.
+// Butterflies on pairs of registers use the packed f32x2 add and subtract
+// (each half rounds like the scalar operation). The shared slice of a chunk
+// holds its 32 x 32 floats with 16-byte column groups XOR-swizzled by the
+// row (row & 7), so the row-wise 16-byte accesses (layouts A and C) and the
+// column-wise 4-byte accesses (layout B) are all free of bank conflicts.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int swz(int row, int col) {      // float index in a 32 x 32 slice
+    return row * 32 + ((((col >> 2) ^ (row & 7))) << 2) + (col & 3);
+}
+
+// Two butterflies (a0, b0) and (a1, b1) with one packed add and one packed
+// subtract: a' = a + b, b' = a - b.
+__device__ __forceinline__ void butterfly2(float& a0, float& a1, float& b0, float& b1) {
+    asm("{\n\t.reg .b64 A, B, S, D;\n\t"
+        "mov.b64 A, {%0, %1};\n\t"
+        "mov.b64 B, {%2, %3};\n\t"
+        "add.rn.f32x2 S, A, B;\n\t"
+        "sub.rn.f32x2 D, A, B;\n\t"
+        "mov.b64 {%0, %1}, S;\n\t"
+        "mov.b64 {%2, %3}, D;\n\t}"
+        : "+f"(a0), "+f"(a1), "+f"(b0), "+f"(b1));
+}
+
+// In-register stages of a 32-value array for register distances
+// s = s_lo .. s_end / 2 (s = 1 scalar, s >= 2 on packed pairs).
+__device__ __forceinline__ void reg_stages32(float (&v)[32], int s_lo, int s_end) {
+    if (s_lo <= 1 && 1 < s_end) {
+        #pragma unroll
+        for (int i = 0; i < 32; i += 2) butterfly(v[i], v[i + 1]);
+    }
+    #pragma unroll
+    for (int s = 2; s < 32; s <<= 1) {
+        if (s >= s_lo && s < s_end) {
+            #pragma unroll
+            for (int i = 0; i < 32; i += 2)
+                if ((i & s) == 0) butterfly2(v[i], v[i + 1], v[i + s], v[i + s + 1]);
+        }
+    }
+}
+
+// Codes of two values: q = rne(fl(v * r)). The product is a scalar
+// round-to-nearest multiply (never contracted: a fused multiply-add would
+// round the exact product and break ties differently). Adding M = 1.5 * 2^23
+// then rounds it to an integer in one step (floats in [2^23, 2^24) are the
+// integers, ties to even), fl(t - M) is that integer as a float (+0 for
+// zero), and the low mantissa bits of t are the integer itself.
+__device__ __forceinline__ void quant_pair(float v0, float v1, float r, float& q0, float& q1, int& i0, int& i1) {
+    const float p0 = __fmul_rn(v0, r), p1 = __fmul_rn(v1, r);
+    asm("{\n\t.reg .b64 V, M, T;\n\t"
+        "mov.b64 V, {%4, %5};\n\t"
+        "mov.b64 M, {%6, %6};\n\t"
+        "add.rn.f32x2 T, V, M;\n\t"
+        "sub.rn.f32x2 V, T, M;\n\t"
+        "mov.b64 {%0, %1}, V;\n\t"
+        "mov.b64 {%2, %3}, T;\n\t}"
+        : "=f"(q0), "=f"(q1), "=r"(i0), "=r"(i1) : "f"(p0), "f"(p1), "f"(12582912.0f));
+    i0 -= 0x4B400000;
+    i1 -= 0x4B400000;
+}
+
+// Eight codes -> packed nibbles (code k in bits 4k .. 4k + 3) and their
+// eight E4M3 bytes (byte k = code k); qf are the codes as floats, qi as ints.
+__device__ __forceinline__ void pack_codes8(const float* qf, const int* qi, uint32_t& nib, uint2& e4) {
+    uint32_t w = 0;
+    #pragma unroll
+    for (int k = 6; k >= 0; k -= 2)      // d = c << 8 | sat4(a) << 4 | sat4(b)
+        asm("cvt.pack.sat.s4.s32.b32 %0, %1, %2, %0;" : "+r"(w) : "r"(qi[k + 1]), "r"(qi[k]));
+    nib = w;
+    uint16_t h[4];
+    #pragma unroll
+    for (int k = 0; k < 4; ++k)          // upper byte from the first operand
+        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(h[k]) : "f"(qf[2 * k + 1]), "f"(qf[2 * k]));
+    e4.x = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
+    e4.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
+}
+
+template <int NR, typename Tin>
+__global__ void __launch_bounds__(128)
+sgat_quant_rows_kernel(QuantArgs a) {
+    __shared__ __align__(16) float buf[4096];
+    __shared__ float red[4];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int row = blockIdx.x;
+    const int K = a.K;
+    const bool masked = a.mask != nullptr && a.mask[row] != 0;
+    const float* sm = masked ? a.a_m : a.a_u;
+    const int own_lo = masked ? a.d_sh : a.d_sh + a.d_m;
+    const int own_hi = masked ? a.d_sh + a.d_m : K;
+    const Tin* X = static_cast<const Tin*>(a.X) + (size_t)row * K;
+    float* slice = buf + warp * 1024;
+
+    float v[NR][32];                      // layout C: v[R][8 j + k]
+    float amax = 0.f;
+    #pragma unroll
+    for (int R = 0; R < NR; ++R) {
+        const int base = R * 4096;
+        const int nch = min(4, (K - base) >> 10);        // chunks in this round (>= 1)
+        float u[32];
+        const int lo = base + warp * 1024 + 32 * lane;
+        if (warp < nch) {
+            In<Tin>::template load<32>(X + lo, u);
+            if (sm != nullptr) {
+                const float4* s4 = reinterpret_cast<const float4*>(sm + lo);
+                #pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float4 w = __ldg(s4 + q);
+                    u[4 * q] = __fmul_rn(u[4 * q], w.x);
+                    u[4 * q + 1] = __fmul_rn(u[4 * q + 1], w.y);
+                    u[4 * q + 2] = __fmul_rn(u[4 * q + 2], w.z);
+                    u[4 * q + 3] = __fmul_rn(u[4 * q + 3], w.w);
+                }
+            }
+            reg_stages32(u, 1, 32);                              // h = 1 .. 16
+            #pragma unroll
+            for (int q = 0; q < 8; ++q)                          // layout A -> slice
+                *reinterpret_cast<float4*>(slice + swz(lane, 4 * q)) =
+                    make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
+            __syncwarp();
+            #pragma unroll
+            for (int i = 0; i < 32; ++i) u[i] = slice[swz(i, lane)];   // layout B
+            reg_stages32(u, 1, a.hb / 32);                       // h = 32 .. min(hb, 1024) / 2
+            #pragma unroll
+            for (int i = 0; i < 32; ++i) slice[swz(i, lane)] = u[i];
+        }
+        __syncthreads();
+        #pragma unroll
+        for (int j = 0; j < 4; ++j) {                            // layout C
+            if (j < nch) {
+                const int r = warp * 8 + (lane >> 2), c = (lane & 3) * 8;
+                const float4 p0 = *reinterpret_cast<const float4*>(buf + j * 1024 + swz(r, c));
+                const float4 p1 = *reinterpret_cast<const float4*>(buf + j * 1024 + swz(r, c + 4));
+                v[R][8 * j] = p0.x; v[R][8 * j + 1] = p0.y; v[R][8 * j + 2] = p0.z; v[R][8 * j + 3] = p0.w;
+                v[R][8 * j + 4] = p1.x; v[R][8 * j + 5] = p1.y; v[R][8 * j + 6] = p1.z; v[R][8 * j + 7] = p1.w;
+            } else {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) v[R][8 * j + k] = 0.f;
+            }
+        }
+        if (NR > 1) __syncthreads();                             // the next round reuses buf
+        if (a.hb > 1024) {                                       // h = 1024: chunks j, j ^ 1
+            #pragma unroll
+            for (int k = 0; k < 8; k += 2) {
+                butterfly2(v[R][k], v[R][k + 1], v[R][8 + k], v[R][9 + k]);
+                butterfly2(v[R][16 + k], v[R][17 + k], v[R][24 + k], v[R][25 + k]);
+            }
+        }
+        if (a.hb > 2048) {                                       // h = 2048: chunks j, j ^ 2
+            #pragma unroll
+            for (int k = 0; k < 8; k += 2) {
+                butterfly2(v[R][k], v[R][k + 1], v[R][16 + k], v[R][17 + k]);
+                butterfly2(v[R][8 + k], v[R][9 + k], v[R][24 + k], v[R][25 + k]);
+            }
+        }
+        #pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int e0 = base + j * 1024 + warp * 256 + 8 * lane;    // first element of the group
+            if (j >= nch) continue;
+            const bool all_keep = (e0 + 8 <= a.d_sh) || (e0 >= own_lo && e0 + 8 <= own_hi);
+            if (!all_keep) {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const int e = e0 + k;
+                    if (!(e < a.d_sh || (e >= own_lo && e < own_hi))) v[R][8 * j + k] = 0.f;
+                }
+            }
+            if (a.post_scale != 1.f) {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) v[R][8 * j + k] = __fmul_rn(v[R][8 * j + k], a.post_scale);
+            }
+            #pragma unroll
+            for (int k = 0; k < 8; ++k) amax = fmaxf(amax, fabsf(v[R][8 * j + k]));
+            if (a.v_dbg != nullptr) {
+                float4* d4 = reinterpret_cast<float4*>(a.v_dbg + (size_t)row * K + e0);
+                d4[0] = make_float4(v[R][8 * j], v[R][8 * j + 1], v[R][8 * j + 2], v[R][8 * j + 3]);
+                d4[1] = make_float4(v[R][8 * j + 4], v[R][8 * j + 5], v[R][8 * j + 6], v[R][8 * j + 7]);
+            }
+        }
+    }
+    #pragma unroll
+    for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
+    if (lane == 0) red[warp] = amax;
+    __syncthreads();
+    amax = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+
+    const float qmax = (float)a.qmax;
+    const bool nz = amax > 0.f;
+    const float s = nz ? __fdiv_rn(amax, qmax) : 0.f;
+    const float r = nz ? __fdiv_rn(qmax, amax) : 0.f;
+    if (threadIdx.x == 0) a.s[row] = s;
+    #pragma unroll
+    for (int R = 0; R < NR; ++R) {
+        const int base = R * 4096;
+        const int nch = min(4, (K - base) >> 10);
+        #pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (j >= nch) continue;
+            const int e0 = base + j * 1024 + warp * 256 + 8 * lane;
+            float qf[8];
+            int qi[8];
+            #pragma unroll
+            for (int k = 0; k < 8; k += 2)
+                quant_pair(v[R][8 * j + k], v[R][8 * j + k + 1], r, qf[k], qf[k + 1], qi[k], qi[k + 1]);
+            uint32_t nib;
+            uint2 e4;
+            pack_codes8(qf, qi, nib, e4);
+            *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = nib;
+            if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * K + e0) = e4;
+        }
+    }
+}
+
+template <typename Tin>
+cudaError_t launch_rows(const QuantArgs& a, cudaStream_t stream) {
+    const int nr = (a.K + 4095) / 4096;
+    dim3 grid(a.L), block(128);
+    switch (nr) {
+        case 1: sgat_quant_rows_kernel<1, Tin><<<grid, block, 0, stream>>>(a); break;
+        case 2: sgat_quant_rows_kernel<2, Tin><<<grid, block, 0, stream>>>(a); break;
+        case 3: sgat_quant_rows_kernel<3, Tin><<<grid, block, 0, stream>>>(a); break;
+        case 4: sgat_quant_rows_kernel<4, Tin><<<grid, block, 0, stream>>>(a); break;
+        default: return cudaErrorInvalidValue;
+    }
+    return cudaGetLastError();
+}
+
 template <int E, typename Tin>
 cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
     constexpr int C = 32 * E;
@@ -330,8 +570,10 @@ cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
 
 template <typename Tin>
 cudaError_t launch_typed(const QuantArgs& a, cudaStream_t stream) {
-    // a warp's chunk: 1024 elements when hb >= 1024 (larger blocks finish
-    // across warps), else 512 elements holding 512 / hb blocks
+    // hb >= 1024 and up to 16384 features: a CTA per row; otherwise a warp's
+    // chunk is 1024 elements (hb >= 1024, blocks finish across warps) or 512
+    // elements holding 512 / hb blocks
+    if (a.hb >= 1024 && a.K % 1024 == 0 && a.K <= 16384) return launch_rows<Tin>(a, stream);
     return a.hb >= 1024 ? launch_e<32, Tin>(a, stream) : launch_e<16, Tin>(a, stream);
 }
 

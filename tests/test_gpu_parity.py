@@ -54,6 +54,12 @@ QUANT_CASES = [
     (9, 256, 16, "f16", True),
     (9, 256, 1, "f16", False),
     (300, 640, 128, "f16", True),
+    # rows of 1024-or-larger blocks: one CTA per row, rounds of 4096 features
+    (17, 8192, 2048, "bf16", True),       # two rounds
+    (6, 16384, 4096, "f16", True),        # four rounds
+    (11, 5120, 1024, "f32", True),        # last round holds one chunk
+    (4, 6144, 2048, "f16", False),        # last round holds one 2048 block
+    (3, 20480, 4096, "f16", True),        # beyond 16384 features: warp-per-chunk kernel
 ]
 
 
@@ -69,9 +75,43 @@ def test_quantize_act_bitexact(abi, L, K, hb, dtype, gates):
     assert np.array_equal(s_a.cpu().numpy(), s), "scales differ"
 
 
-def test_quantize_act_edge_cases(abi):
+@pytest.mark.parametrize("K,hb", [(4096, 4096), (2048, 1024), (1024, 512), (256, 16)])
+def test_quantize_act_exact_ties(abi, K, hb):
+    """Transformed values that sit exactly on a rounding tie (x.5 after the
+    scaling by r = 7 / amax, an exact power of two here): the codes round
+    half to even. X = v H / hb per block is exact in float32, and the
+    float32 butterflies of X reproduce v exactly (dyadic partial sums)."""
+    rng = np.random.default_rng(K + hb)
+    L = 12
+    V = np.zeros((L, K))
+    ties = np.array([0.5, 1.5, 2.5, 3.5, 4.5, 5.5, 6.5])
+    for i in range(L):
+        scale = 2.0 ** (i - 4)                       # amax = 7 * scale, r = 1 / scale
+        pos = rng.choice(K, 2 * len(ties) + 1, replace=False)
+        V[i, pos[0]] = 7 * scale * (-1) ** i
+        V[i, pos[1:1 + len(ties)]] = ties * scale
+        V[i, pos[1 + len(ties):]] = -ties * scale
+    Hh = osg.hadamard_sylvester(hb).astype(np.float64)
+    X = (V.reshape(L, K // hb, hb) @ Hh / hb).reshape(L, K).astype(np.float32)
+    Xq = torch.empty(L, K // 2, dtype=torch.uint8, device="cuda")
+    s_a = torch.empty(L, dtype=torch.float32, device="cuda")
+    Xe = torch.empty(L, K, dtype=torch.uint8, device="cuda")
+    abi.sgat_quantize_act(H.dev(X), None, None, None, hb, K, 0, 0, Xq, s_a, Xe=Xe)
+    abi.check_status()
+    codes, s = osg.sgat_quantize_act(X, np.zeros(L, np.uint8), None, None, hb, K, 0, 0, 4)
+    nz = V != 0
+    expect = np.where(np.abs(V / (np.abs(V).max(1, keepdims=True) / 7)) % 1 == 0.5, 0, 1)
+    assert (nz & (expect == 0)).sum() == L * 2 * len(ties)          # the ties are there
+    assert np.array_equal(codes[nz], np.rint(V[nz] / (np.abs(V).max(1, keepdims=True) / 7).repeat(K, 1)[nz]))
+    assert np.array_equal(H.unpack(Xq), codes), "codes at exact ties differ"
+    assert np.array_equal(s_a.cpu().numpy(), s)
+    assert np.array_equal(Xe.cpu().numpy(), H.e4m3_bytes(codes))
+
+
+@pytest.mark.parametrize("K,hb", [(512, 512), (4096, 4096)])
+def test_quantize_act_edge_cases(abi, K, hb):
     """No mask (all unmasked), all masked, mixed; an all-zero row in each."""
-    case = inputs.random_linear(5, 24, 512, 128, hb=512)
+    case = inputs.random_linear(5, 24, K, 128, hb=hb)
     case.X[3] = 0
     xf = case.xf
     mixed = case.mask.copy()
