@@ -16,6 +16,7 @@ data path). `--impl reference` times the CPU oracle on the same workload.
 """
 
 import argparse
+import datetime
 import hashlib
 import json
 import os
@@ -73,7 +74,11 @@ def config_dict(graph):
 # Clocks during the timed region
 # ---------------------------------------------------------------------------
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi clocks and throttle reasons every 100 ms from before the
+    warm-up to after the timed region; the summary keeps the samples taken
+    within 250 ms of the timed region (the two nearest ones when the region
+    is shorter than the sampling period)."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -81,6 +86,7 @@ class ClockSampler:
         self.gpu = gpu_index
         self.proc = None
         self.path = None
+        self.t0 = self.t1 = None
 
     def start(self):
         try:
@@ -88,15 +94,21 @@ class ClockSampler:
             os.close(fd)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
 
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+
     def stop(self):
         if self.proc is None:
             return None
-        time.sleep(0.25)
+        time.sleep(0.3)
         self.proc.terminate()
         try:
             self.proc.wait(timeout=5)
@@ -106,22 +118,28 @@ class ClockSampler:
         with open(self.path) as f:
             for line in f:
                 parts = [x.strip() for x in line.split(",")]
-                if len(parts) >= 9:
-                    rows.append(parts)
+                if len(parts) >= 10:
+                    try:
+                        ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                    except ValueError:
+                        continue
+                    rows.append((ts, parts[1:]))
         os.unlink(self.path)
-        if not rows:
+        if not rows or self.t0 is None or self.t1 is None:
             return None
-        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
-        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        sel = [r for t, r in rows if self.t0 - 0.25 <= t <= self.t1 + 0.25]
+        if not sel:
+            mid = 0.5 * (self.t0 + self.t1)
+            sel = [r for t, r in sorted(rows, key=lambda tr: abs(tr[0] - mid))[:2]]
+        num = lambda x: float(x) if x.replace(".", "").isdigit() else None
+        sm = [num(r[1]) for r in sel if num(r[1]) is not None]
+        mx = [num(r[2]) for r in sel if num(r[2]) is not None]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower().startswith("active")})
+        reasons = sorted({n for r in sel for n, v in zip(names, r[5:9]) if v.lower().startswith("active")})
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(rows)}
+                "reasons": reasons, "samples": len(sel),
+                "timed_region_s": round(self.t1 - self.t0, 3)}
 
-
-# ---------------------------------------------------------------------------
-# GPU arm
-# ---------------------------------------------------------------------------
 def kernel_source_hash():
     p = os.path.join(ROOT, "paper_2606_04945_gb300", "csrc")
     h = hashlib.sha256()
@@ -195,6 +213,8 @@ def run_ours(args):
     L, K = step.L, step.qkv.K
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     flush = lambda: flush_buf.zero_()
+    clocks = ClockSampler(local)
+    clocks.start()
 
     # warm-up, then capture the step in a CUDA graph
     for _ in range(max(args.warmup, 3)):
@@ -227,11 +247,10 @@ def run_ours(args):
     abi.check_status()
 
     # timed region: exactly `steps` steps, device-timed per step
-    clocks = ClockSampler(local)
-    clocks.start()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    clocks.mark_start()
     s = torch.cuda.current_stream()
     evs = []
     for _ in range(args.steps):
@@ -244,6 +263,7 @@ def run_ours(args):
         e1.record(s)
         evs.append((e0, e1))
     torch.cuda.synchronize()
+    clocks.mark_end()
     if world > 1:
         dist.barrier()
     clk = clocks.stop()

@@ -294,10 +294,18 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
     }
 }
 
+template <typename T> struct To;
+template <> struct To<__half> { static __device__ __forceinline__ float f(__half h) { return __half2float(h); } };
+template <> struct To<__nv_bfloat16> { static __device__ __forceinline__ float f(__nv_bfloat16 h) { return __bfloat162float(h); } };
+template <> struct To<float> { static __device__ __forceinline__ float f(float h) { return h; } };
+
 // ---------------------------------------------------------------------------
 // Rows with Hadamard blocks of 1024 elements or more (hb >= 1024, K a
 // multiple of 1024, K <= 4096 NR): one CTA of four warps per row, in rounds
 // of 4096 elements (four 1024-element chunks, chunk j of a round in warp j).
+// A warp reads its chunk of x and of the smoothing vector with coalesced
+// 16-byte loads (lane l at 16 l + 512 q) into shared memory and takes it
+// back in layout A.
 //
 //   layout A  lane l holds elements 32 l .. 32 l + 31 of its warp's chunk:
 //             stages h = 1 .. 16 are between registers;
@@ -385,9 +393,10 @@ __device__ __forceinline__ void pack_codes8(const float* qf, const int* qi, uint
 }
 
 template <int NR, typename Tin>
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
 sgat_quant_rows_kernel(QuantArgs a) {
     __shared__ __align__(16) float buf[4096];
+    __shared__ __align__(16) float xst[4096];
     __shared__ float red[4];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
@@ -407,20 +416,74 @@ sgat_quant_rows_kernel(QuantArgs a) {
         const int base = R * 4096;
         const int nch = min(4, (K - base) >> 10);        // chunks in this round (>= 1)
         float u[32];
-        const int lo = base + warp * 1024 + 32 * lane;
         if (warp < nch) {
-            In<Tin>::template load<32>(X + lo, u);
-            if (sm != nullptr) {
-                const float4* s4 = reinterpret_cast<const float4*>(sm + lo);
+            // coalesced loads (lane l: 16 bytes at 16 l + 512 q), staged
+            // through shared memory and read back in layout A
+            const int c0 = base + warp * 1024;                   // first element of the chunk
+            float* stage = xst + warp * 1024;                    // 4 KB per warp
+            if (sizeof(Tin) == 2) {
+                uint4 xr[4];
+                #pragma unroll
+                for (int q = 0; q < 4; ++q) xr[q] = __ldg(reinterpret_cast<const uint4*>(X + c0) + lane + 32 * q);
+                float4 sr[8];
+                if (sm != nullptr) {
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
+                }
+                // fp16 staging: 32 rows of 64 bytes, 16-byte group g of row R at g ^ ((R >> 1) & 3)
+                uint8_t* st8 = reinterpret_cast<uint8_t*>(stage);
+                #pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int R = (lane >> 2) + 8 * q, g = lane & 3;
+                    *reinterpret_cast<uint4*>(st8 + R * 64 + 16 * (g ^ ((R >> 1) & 3))) = xr[q];
+                }
+                if (sm != nullptr) {
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
+                }
+                __syncwarp();
+                #pragma unroll
+                for (int g = 0; g < 4; ++g) {
+                    const uint4 w = *reinterpret_cast<const uint4*>(st8 + lane * 64 + 16 * (g ^ ((lane >> 1) & 3)));
+                    const Tin* h = reinterpret_cast<const Tin*>(&w);
+                    #pragma unroll
+                    for (int k = 0; k < 8; ++k) u[8 * g + k] = To<Tin>::f(h[k]);
+                }
+            } else {
+                float4 xr[8], sr[8];
+                #pragma unroll
+                for (int q = 0; q < 8; ++q) xr[q] = __ldg(reinterpret_cast<const float4*>(X + c0) + lane + 32 * q);
+                if (sm != nullptr) {
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
+                }
+                #pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    *reinterpret_cast<float4*>(stage + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = xr[q];
+                if (sm != nullptr) {
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
+                }
+                __syncwarp();
                 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
-                    const float4 w = __ldg(s4 + q);
+                    const float4 w = *reinterpret_cast<const float4*>(stage + swz(lane, 4 * q));
+                    u[4 * q] = w.x; u[4 * q + 1] = w.y; u[4 * q + 2] = w.z; u[4 * q + 3] = w.w;
+                }
+            }
+            if (sm != nullptr) {
+                #pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float4 w = *reinterpret_cast<const float4*>(slice + swz(lane, 4 * q));
                     u[4 * q] = __fmul_rn(u[4 * q], w.x);
                     u[4 * q + 1] = __fmul_rn(u[4 * q + 1], w.y);
                     u[4 * q + 2] = __fmul_rn(u[4 * q + 2], w.z);
                     u[4 * q + 3] = __fmul_rn(u[4 * q + 3], w.w);
                 }
             }
+            __syncwarp();
             reg_stages32(u, 1, 32);                              // h = 1 .. 16
             #pragma unroll
             for (int q = 0; q < 8; ++q)                          // layout A -> slice

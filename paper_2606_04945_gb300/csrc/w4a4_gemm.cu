@@ -80,7 +80,30 @@ __device__ __forceinline__ void convert_store(uint32_t tile, int row, int q, uin
 }
 
 template <typename TOut> struct Out;
+// Row `row` (32 values) of a 32 x 32 output box staged for a TMA store:
+// 16-bit types use 64-byte rows with the 64-byte swizzle (16-byte group g at
+// g ^ ((row >> 1) & 3)), float uses 128-byte rows with the 128-byte swizzle
+// (g ^ (row & 7)); either way the 32 lanes of a warp write without bank
+// conflicts.
+template <typename T2, typename Cvt>
+__device__ __forceinline__ void stage_row16(uint32_t box, int row, const float (&y)[32], Cvt cvt) {
+    #pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        uint32_t w[4];
+        #pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            T2 h = cvt(y[8 * g + 2 * j], y[8 * g + 2 * j + 1]);
+            w[j] = *reinterpret_cast<uint32_t*>(&h);
+        }
+        st_shared_v4(box + row * 64 + 16 * (g ^ ((row >> 1) & 3)), w[0], w[1], w[2], w[3]);
+    }
+}
 template <> struct Out<__half> {
+    static constexpr CUtensorMapDataType TMAP_TYPE = CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+    static constexpr CUtensorMapSwizzle TMAP_SWIZZLE = CU_TENSOR_MAP_SWIZZLE_64B;
+    static __device__ __forceinline__ void stage32(uint32_t box, int row, const float (&y)[32]) {
+        stage_row16<__half2>(box, row, y, [](float a, float b) { return __floats2half2_rn(a, b); });
+    }
     static __device__ __forceinline__ void store32(__half* p, const float (&y)[32]) {
         uint4* q = reinterpret_cast<uint4*>(p);
         #pragma unroll
@@ -96,6 +119,11 @@ template <> struct Out<__half> {
     }
 };
 template <> struct Out<__nv_bfloat16> {
+    static constexpr CUtensorMapDataType TMAP_TYPE = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    static constexpr CUtensorMapSwizzle TMAP_SWIZZLE = CU_TENSOR_MAP_SWIZZLE_64B;
+    static __device__ __forceinline__ void stage32(uint32_t box, int row, const float (&y)[32]) {
+        stage_row16<__nv_bfloat162>(box, row, y, [](float a, float b) { return __floats2bfloat162_rn(a, b); });
+    }
     static __device__ __forceinline__ void store32(__nv_bfloat16* p, const float (&y)[32]) {
         uint4* q = reinterpret_cast<uint4*>(p);
         #pragma unroll
@@ -111,6 +139,14 @@ template <> struct Out<__nv_bfloat16> {
     }
 };
 template <> struct Out<float> {
+    static constexpr CUtensorMapDataType TMAP_TYPE = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    static constexpr CUtensorMapSwizzle TMAP_SWIZZLE = CU_TENSOR_MAP_SWIZZLE_128B;
+    static __device__ __forceinline__ void stage32(uint32_t box, int row, const float (&y)[32]) {
+        #pragma unroll
+        for (int g = 0; g < 8; ++g)
+            st_shared_v4(box + row * 128 + 16 * (g ^ (row & 7)), __float_as_uint(y[4 * g]),
+                         __float_as_uint(y[4 * g + 1]), __float_as_uint(y[4 * g + 2]), __float_as_uint(y[4 * g + 3]));
+    }
     static __device__ __forceinline__ void store32(float* p, const float (&y)[32]) {
         float4* q = reinterpret_cast<float4*>(p);
         #pragma unroll
@@ -692,6 +728,26 @@ bool encode_u8_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tensor map of the row-major output Y [rows][cols] with 32 x 32 boxes.
+bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t elem, uint64_t rows,
+                     uint64_t cols, CUtensorMapSwizzle swz) {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (fn == nullptr) {
+        cudaDriverEntryPointQueryResult q;
+        void* f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
+            return false;
+        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols * elem};
+    const cuuint32_t box[2] = {32, 32};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, type, 2, ptr, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+              CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // ---------------------------------------------------------------------------
 // CTA-pair GEMM with both operands as E4M3 bytes by TMA (activation codes
 // from the quantiser, weight codes from w4_unpack_e4m3).
@@ -708,7 +764,7 @@ bool encode_u8_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
 // ---------------------------------------------------------------------------
 namespace tmak {
 constexpr int BM = 128, BN = 256, BN_CTA = 128, BK = 128, UMMA_K = 32;
-constexpr int STAGES = 6;
+constexpr int STAGES = 5;
 constexpr int A_BYTES = BM * BK, B_BYTES = BN_CTA * BK;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;             // 32 KB
 constexpr int NUM_EPI_WARPS = 8;
@@ -716,7 +772,9 @@ constexpr int TMA_WARP = 8, MMA_WARP = 9;
 constexpr int THREADS = 10 * 32;
 constexpr int TMEM_COLS = 512;
 constexpr int EPI_PARAM_BYTES = NUM_EPI_WARPS * 2 * (BN / 2) * 4;
-constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
+constexpr int EPI_BOX_WARP_BYTES = 4096;                  // two 32 x 32 16-bit boxes or one float box
+constexpr int EPI_STAGE_BYTES = NUM_EPI_WARPS * EPI_BOX_WARP_BYTES;
+constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + EPI_STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
 constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
 struct Smem {
     uint64_t full[STAGES];        // pair leader: both CTAs' TMA bytes
@@ -732,7 +790,7 @@ struct Smem {
 template <typename TOut, int CL>
 __global__ void __launch_bounds__(tmak::THREADS, 1)
 w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
-                          const __grid_constant__ CUtensorMap tmap_b) {
+                          const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y) {
     constexpr int BM = tmak::BM, BN = tmak::BN, BN_CTA = tmak::BN_CTA, BK = tmak::BK;
     constexpr int UMMA_K = tmak::UMMA_K, STAGES = tmak::STAGES, STAGE_BYTES = tmak::STAGE_BYTES;
     constexpr int A_BYTES = tmak::A_BYTES, B_BYTES = tmak::B_BYTES;
@@ -747,7 +805,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
-    Smem* sh = reinterpret_cast<Smem*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES);
+    constexpr int EPI_STAGE_BYTES = tmak::EPI_STAGE_BYTES, EPI_BOX_WARP_BYTES = tmak::EPI_BOX_WARP_BYTES;
+    Smem* sh = reinterpret_cast<Smem*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES + EPI_STAGE_BYTES);
     volatile int* abort = &sh->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = cluster_ctarank();
@@ -854,15 +913,21 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         __syncwarp();
     } else {
         // epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31, columns
-        // (w / 4) * 128 .. + 127; scales and biases staged before the wait
+        // (w / 4) * 128 .. + 127, in 32 x 32 boxes; scales and biases are
+        // staged before the accumulator wait. Each box is dequantised into
+        // the warp's swizzled staging buffer and written by one TMA store
+        // (rows past L and columns past N are clipped by the tensor map).
+        constexpr int BOX_BYTES = 32 * 32 * (int)sizeof(TOut);
+        constexpr int NBUF = EPI_BOX_WARP_BYTES / BOX_BYTES;
         const uint32_t leader_tmem_empty0 = mapa_shared(smem_addr(&sh->tmem_empty[0]), leader);
-        float* epi_sw = reinterpret_cast<float*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES + sizeof(Smem) +
+        const uint32_t ybox0 = base + STAGES * STAGE_BYTES + warp * EPI_BOX_WARP_BYTES;
+        float* epi_sw = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sh) + sizeof(Smem) +
                                                  (16 - sizeof(Smem) % 16) % 16) + warp * 2 * (BN / 2);
         float* epi_b = epi_sw + BN / 2;
         const int quarter = warp & 3, chalf = warp >> 2;
         bool ok = true;
         int it = 0;
-        TOut* Y = static_cast<TOut*>(a.Y);
+        int nbox = 0;
         for (int tile = cluster; tile < num_tiles; tile += num_clusters, ++it) {
             const int m0 = (tile % num_m) * 2 * BM + (int)half * BM;
             const int n0 = ((tile / num_m) * PAIRS + (int)pr) * BN;
@@ -894,44 +959,59 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 uint32_t r[32];
                 tmem_ld_32x32b_x32(t_row + c * 32, r);
                 tmem_ld_wait();
-                if (valid) {
-                    float y[32];
-                    const float4* sw4 = reinterpret_cast<const float4*>(epi_sw + cc * 32);
-                    const float4* b4 = reinterpret_cast<const float4*>(epi_b + cc * 32);
+                float y[32];
+                const float4* sw4 = reinterpret_cast<const float4*>(epi_sw + cc * 32);
+                const float4* b4 = reinterpret_cast<const float4*>(epi_b + cc * 32);
+                #pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const float4 sw = sw4[u];
+                    y[4 * u] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u]), sa), sw.x);
+                    y[4 * u + 1] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 1]), sa), sw.y);
+                    y[4 * u + 2] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 2]), sa), sw.z);
+                    y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
+                }
+                if (a.bias != nullptr) {
                     #pragma unroll
                     for (int u = 0; u < 8; ++u) {
-                        const float4 sw = sw4[u];
-                        y[4 * u] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u]), sa), sw.x);
-                        y[4 * u + 1] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 1]), sa), sw.y);
-                        y[4 * u + 2] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 2]), sa), sw.z);
-                        y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
+                        const float4 bq = b4[u];
+                        y[4 * u] = __fadd_rn(y[4 * u], bq.x);
+                        y[4 * u + 1] = __fadd_rn(y[4 * u + 1], bq.y);
+                        y[4 * u + 2] = __fadd_rn(y[4 * u + 2], bq.z);
+                        y[4 * u + 3] = __fadd_rn(y[4 * u + 3], bq.w);
                     }
-                    if (a.bias != nullptr) {
-                        #pragma unroll
-                        for (int u = 0; u < 8; ++u) {
-                            const float4 bq = b4[u];
-                            y[4 * u] = __fadd_rn(y[4 * u], bq.x);
-                            y[4 * u + 1] = __fadd_rn(y[4 * u + 1], bq.y);
-                            y[4 * u + 2] = __fadd_rn(y[4 * u + 2], bq.z);
-                            y[4 * u + 3] = __fadd_rn(y[4 * u + 3], bq.w);
-                        }
+                }
+                // the buffer's previous store has read it
+                const uint32_t box = ybox0 + (uint32_t)((nbox % NBUF) * BOX_BYTES);
+                if (nbox >= NBUF) {
+                    if (lane == 0) {
+                        if (NBUF == 2) bulk_wait_read1(); else bulk_wait_read0();
                     }
-                    Out<TOut>::store32(Y + (size_t)row * N + nc, y);
-                    if (a.acc_dbg != nullptr) {
-                        int4* d4 = reinterpret_cast<int4*>(a.acc_dbg + (size_t)row * N + nc);
-                        #pragma unroll
-                        for (int u = 0; u < 8; ++u)
-                            d4[u] = make_int4(__float2int_rn(__uint_as_float(r[4 * u])),
-                                              __float2int_rn(__uint_as_float(r[4 * u + 1])),
-                                              __float2int_rn(__uint_as_float(r[4 * u + 2])),
-                                              __float2int_rn(__uint_as_float(r[4 * u + 3])));
-                    }
+                    __syncwarp();
+                }
+                Out<TOut>::stage32(box, lane, y);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&tmap_y, nc, m0 + quarter * 32, box);
+                    bulk_commit();
+                }
+                ++nbox;
+                if (a.acc_dbg != nullptr && valid) {
+                    int4* d4 = reinterpret_cast<int4*>(a.acc_dbg + (size_t)row * N + nc);
+                    #pragma unroll
+                    for (int u = 0; u < 8; ++u)
+                        d4[u] = make_int4(__float2int_rn(__uint_as_float(r[4 * u])),
+                                          __float2int_rn(__uint_as_float(r[4 * u + 1])),
+                                          __float2int_rn(__uint_as_float(r[4 * u + 2])),
+                                          __float2int_rn(__uint_as_float(r[4 * u + 3])));
                 }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + acc * 8);
         }
+        if (lane == 0) bulk_wait0();     // this warp's stores are complete
+        __syncwarp();
         if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
     }
 
@@ -977,10 +1057,12 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
         max_clusters[dev] = n;
         attr_set[dev] = true;
     }
-    CUtensorMap ta, tb;
+    CUtensorMap ta, tb, ty;
     if (!encode_u8_tmap(&ta, a.Xe, (uint64_t)a.L, (uint64_t)a.K, CL == 2 ? BM : BM / 2, BK,
                         CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_u8_tmap(&tb, a.We, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK, CU_TENSOR_MAP_SWIZZLE_128B))
+        !encode_u8_tmap(&tb, a.We, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N,
+                         Out<TOut>::TMAP_SWIZZLE))
         return cudaErrorInvalidValue;
     const int num_n = (a.N + BN - 1) / BN;
     const int num_tiles = ((a.L + 2 * BM - 1) / (2 * BM)) * ((num_n + CL / 2 - 1) / (CL / 2));
@@ -988,7 +1070,7 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
     if (clusters < 1) clusters = 1;
     if (num_tiles < clusters) clusters = num_tiles;
     cfg.gridDim = dim3(CL * clusters);
-    return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb);
+    return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb, ty);
 }
 
 template <typename TOut>
