@@ -319,6 +319,47 @@ def test_llada_attention_full(abi, weights):
     run_linear_case(abi, o, weights=weights)
 
 
+def _sample_rows(rng, L, n, mask):
+    """Sorted sample of n rows with both states and both ends of the batch."""
+    rows = set(rng.choice(L, n - 4, replace=False).tolist()) | {0, L - 1}
+    rows |= {int(np.argmax(mask)), int(np.argmin(mask))}
+    return np.array(sorted(rows))
+
+
+@pytest.mark.parametrize("ratio", [0.1, 0.5, 0.9])
+def test_llada_mlp(abi, ratio):
+    """LLaDA-8B MLP at one step: gate+up 4096 -> 24576 with SGAT, SwiGLU
+    (test glue on the GPU, in float32, rounded to float16), down 12288 ->
+    4096 with SGAT on its own input (hb = 4096, three 4096-feature rounds
+    per row). The mask is semi-autoregressive: the last round(32 ratio)
+    blocks of 32 tokens are masked. Weight codes are compared for every
+    channel, activations on 256 sampled tokens; the down projection is
+    teacher-forced on the GPU's SwiGLU output."""
+    gu, W_down, mask = inputs.llada_mlp(0, ratio)
+    rng = np.random.default_rng(int(ratio * 10))
+    rows = _sample_rows(rng, gu.L, 256, mask)
+    Y = run_linear_case(abi, gu, check_rows=rows)
+    F = gu.N // 2
+    h = (torch.nn.functional.silu(Y[:, :F].float()) * Y[:, F:].float()).half()
+    hx = h.float().cpu().numpy()
+    down = inputs.LinearCase(f"llada_down_1024x12288x4096_r{ratio}", hx, "f16", mask, W_down,
+                             inputs.make_sgat(hx, mask))
+    assert down.xf.hb == 4096
+    run_linear_case(abi, down, check_rows=rows)
+
+
+def test_dream_block_linears(abi):
+    """Dream-7B (Qwen2.5-7B shape) block linears on 4 x 2048 tokens in
+    bfloat16: QKV with bias, O with TAC (block 128), gate+up 3584 -> 37888,
+    down 18944 -> 3584 (hb = 512). Full-size launches; weight codes compared
+    for every channel, activations and outputs on 256 sampled tokens."""
+    cases = inputs.dream_block_linears(0)
+    rng = np.random.default_rng(7)
+    rows = _sample_rows(rng, cases[0].L, 256, cases[0].mask)
+    for case in cases:
+        run_linear_case(abi, case, check_rows=rows)
+
+
 @pytest.mark.parametrize("L,K,N,dtype,tac_g,bias", [(1, 128, 32, "f16", None, False),
                                                     (77, 512, 320, "bf16", 16, True),
                                                     (129, 1024, 256, "f16", 128, False),
