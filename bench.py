@@ -267,6 +267,16 @@ def run_ours(args):
     t_gemm_o = time_kernel(lambda: abi.w4a4_gemm(None, s_a, o.Wq, o.s_w, step.Y_o, Xe=Xe, We=o.We), flush, reps, torch)
     abi.check_status()
 
+    # the unquantised baseline: the same two projections as 16-bit GEMMs
+    # (fp16 weights and activations, float32 accumulation) -- context for
+    # the paper's speed-up over FP16, not part of the step
+    W16_qkv = torch.from_numpy(qkv_case.W).to(torch.float16).cuda()
+    W16_o = torch.from_numpy(o_case.W).to(torch.float16).cuda()
+    t_f16_qkv = time_kernel(lambda: abi.fp16_gemm_ref(step.X, W16_qkv, step.Y_qkv), flush, reps, torch)
+    t_f16_o = time_kernel(lambda: abi.fp16_gemm_ref(step.Z, W16_o, step.Y_o), flush, reps, torch)
+    abi.check_status()
+    del W16_qkv, W16_o
+
     # timed region: exactly `steps` steps, device-timed per step
     if world > 1:
         dist.barrier()
@@ -377,6 +387,15 @@ def run_ours(args):
             "sgat_quantize_act_f32": {"ms": round(t_quant_z, 5), "bytes": quant_z_bytes,
                                       "gbs": round(quant_z_bytes / t_quant_z / 1e6, 1),
                                       "frac": round(quant_z_bytes / t_quant_z / 1e6 / hbm, 4)},
+        },
+        "fp16_baseline": {
+            "kernel": "fp16_gemm_ref (tcgen05 kind::f16 CTA pairs, fp16 in/out, fp32 accumulate)",
+            "launch_ms": {"qkv": round(t_f16_qkv, 5), "o": round(t_f16_o, 5)},
+            "tflops": round(gemm_ops / ((t_f16_qkv + t_f16_o) * 1e-3) / 1e12, 2),
+            "speedup_gemms": round((t_f16_qkv + t_f16_o) / gemm_ms, 3),
+            "speedup_step": round((t_f16_qkv + t_f16_o) / ms, 3),
+            "note": "W4A4 GEMMs vs fp16 GEMMs of the same shapes; step = W4A4 step (quantisers and TAC "
+                    "included) vs the two fp16 GEMMs alone. The paper's 1.69x (A40, Sec. 4.4) is context only.",
         },
         "e2e": {"value": round(job_tops(ops, ms_e2e, world), 3), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms_e2e, 5)},

@@ -154,6 +154,19 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
               int y_dtype, int32_t* acc_dbg, void* stream);
 
 /*
+ * fp16_gemm_ref -- the 16-bit baseline of the projections: C = A B^T with
+ * float32 accumulation and one rounding to the element type. It is the
+ * unquantised model's linear layer that Sec. 4.4 measures its speed-up
+ * against; here it serves only as that denominator (the same CTA-pair
+ * tcgen05 kernel structure as w4a4_gemm, kind::f16, no cuBLAS).
+ *
+ *   A [M][K], B [N][K] row-major, C [M][N] out; all of element type dtype
+ *   (F16 or BF16), 16-byte aligned.
+ * Shapes: M >= 0, N >= 32 with N % 32 == 0, K >= 64 with K % 64 == 0.
+ */
+int fp16_gemm_ref(const void* A, const void* B, int dtype, int M, int N, int K, void* C, void* stream);
+
+/*
  * tac_apply -- block-wise affine compensation of the quantised attention
  * output before the output projection (Sec. 3.3 Eq. 17; App. C row-major
  * form Z_b M_b^T + 1 d_b^T).

@@ -18,7 +18,7 @@ OK, ERR_ARG, ERR_SHAPE, ERR_ALIGN, ERR_BITS, ERR_CUDA, ERR_TIMEOUT = 0, -1, -2, 
 
 EXPORTED = (
     "starq_version", "starq_last_error", "starq_check_status",
-    "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "tac_apply",
+    "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "fp16_gemm_ref", "tac_apply",
     "sgat_linear_workspace_size", "sgat_linear",
 )
 
@@ -43,6 +43,7 @@ def _load():
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, i, vp]
+    lib.fp16_gemm_ref.argtypes = [vp, vp, i, i, i, i, vp, vp]
     lib.sgat_linear_workspace_size.argtypes = [i, i, i]
     lib.sgat_linear_workspace_size.restype = ctypes.c_size_t
     lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
@@ -123,6 +124,14 @@ def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, st
     N, K = _weight_shape(Wq, We)
     _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y),
                          dtype_code(Y), _p(acc_dbg), _stream(stream)))
+
+
+def fp16_gemm_ref(A, B, C, stream=None):
+    """C = A B^T for 16-bit A [M][K], B [N][K] (the unquantised baseline)."""
+    _contig(A, B, C)
+    M, K = A.shape
+    N = B.shape[0]
+    _check(lib.fp16_gemm_ref(_p(A), _p(B), dtype_code(A), M, N, K, _p(C), _stream(stream)))
 
 
 def tac_apply(Z, M, d, g, out, stream=None):

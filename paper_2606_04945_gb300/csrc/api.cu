@@ -192,6 +192,25 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
     return STARQ_OK;
 }
 
+int fp16_gemm_ref(const void* A, const void* B, int dtype, int M, int N, int K, void* C, void* stream) {
+    if (M > 0 && (!A || !B || !C)) return fail(STARQ_ERR_ARG, "fp16_gemm_ref: NULL A, B or C");
+    if (dtype != STARQ_F16 && dtype != STARQ_BF16) return fail(STARQ_ERR_ARG, "fp16_gemm_ref: dtype must be F16 or BF16");
+    if (M < 0) return fail(STARQ_ERR_SHAPE, "M=%d < 0", M);
+    if (N < 32 || N % 32 != 0) return fail(STARQ_ERR_SHAPE, "fp16_gemm_ref: N=%d: need N >= 32, N %% 32 == 0", N);
+    if (K < 64 || K % 64 != 0) return fail(STARQ_ERR_SHAPE, "fp16_gemm_ref: K=%d: need K >= 64, K %% 64 == 0", K);
+    if (M == 0) return STARQ_OK;
+    if (!aligned(A, 16) || !aligned(B, 16) || !aligned(C, 16))
+        return fail(STARQ_ERR_ALIGN, "fp16_gemm_ref: A, B, C must be 16-byte aligned");
+    int rc = STARQ_OK;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    GemmArgs a{nullptr, nullptr, nullptr, nullptr, nullptr, M, N, K, C, dtype, nullptr, st,
+               static_cast<const uint8_t*>(A), static_cast<const uint8_t*>(B)};
+    cudaError_t e = launch_fp16_gemm(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "fp16_gemm_ref launch");
+    return STARQ_OK;
+}
+
 int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d,
               void* out, int out_dtype, void* stream) {
     if (L > 0 && (!Z || !out)) return fail(STARQ_ERR_ARG, "tac_apply: NULL Z or out");

@@ -47,6 +47,9 @@ struct GemmArgs {
     const uint8_t* We = nullptr;   // optional E4M3 bytes of the weight codes [N][K]
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+// Plain 16-bit GEMM C = A B^T (A = a.Xe [L][K], B = a.We [N][K], both of
+// type a.y_dtype, float32 accumulation, C = a.Y), no scales.
+cudaError_t launch_fp16_gemm(const GemmArgs& a, cudaStream_t stream);
 // Packed int4 codes [rows][K/2] -> E4M3 bytes [rows][K].
 cudaError_t launch_unpack_e4m3(const uint8_t* packed, uint8_t* e4m3, size_t rows, int K, cudaStream_t stream);
 
@@ -170,6 +173,15 @@ __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t a_desc, uint64
                                         uint32_t idesc, uint32_t accumulate) {
     asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
                  "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+                 :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+                 : "memory");
+}
+
+// CTA-pair form (M = 256 across the pair) of the 16-bit MMA.
+__device__ __forceinline__ void mma_f16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                             uint32_t idesc, uint32_t accumulate) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}"
                  :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
                  : "memory");
 }

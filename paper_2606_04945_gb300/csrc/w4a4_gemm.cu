@@ -728,6 +728,28 @@ bool encode_u8_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tensor map of a row-major K-major operand [rows][cols] of 1- or 2-byte
+// elements, box box_rows x box_cols elements, 128-byte swizzle.
+bool encode_operand_tmap(CUtensorMap* m, const void* ptr, CUtensorMapDataType type, size_t elem, uint64_t rows,
+                         uint64_t cols, uint32_t box_rows, uint32_t box_cols) {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (fn == nullptr) {
+        cudaDriverEntryPointQueryResult q;
+        void* f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
+            return false;
+        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }
+    const cuuint64_t dims[2] = {cols, rows};
+    const cuuint64_t strides[1] = {cols * elem};
+    const cuuint32_t box[2] = {box_cols, box_rows};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(m, type, 2, const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Tensor map of the row-major output Y [rows][cols] with 32 x 32 boxes.
 bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t elem, uint64_t rows,
                      uint64_t cols, CUtensorMapSwizzle swz) {
@@ -787,7 +809,10 @@ struct Smem {
 };
 }  // namespace tmak
 
-template <typename TOut, int CL>
+// OPK: operand kind -- 0 = E4M3 codes (dequantising epilogue), 1 = fp16,
+// 2 = bf16 (plain float32 accumulator cast to the output type). Every kind
+// reads 128-byte K rows and advances 32 bytes of K per MMA.
+template <typename TOut, int CL, int OPK>
 __global__ void __launch_bounds__(tmak::THREADS, 1)
 w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
                           const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y) {
@@ -796,7 +821,9 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     constexpr int A_BYTES = tmak::A_BYTES, B_BYTES = tmak::B_BYTES;
     constexpr int TMA_WARP = tmak::TMA_WARP, MMA_WARP = tmak::MMA_WARP;
     constexpr int NUM_EPI_WARPS = tmak::NUM_EPI_WARPS, TMEM_COLS = tmak::TMEM_COLS;
-    constexpr uint32_t IDESC = tmak::IDESC;
+    constexpr uint32_t IDESC = tmak::IDESC | (OPK == 2 ? ((1u << 7) | (1u << 10)) : 0u);
+    constexpr int BKE = OPK == 0 ? BK : BK / 2;          // K elements per stage row
+    constexpr bool DEQUANT = OPK == 0;
     constexpr int PAIRS = CL / 2;
     constexpr uint16_t ALL = (uint16_t)((1u << CL) - 1u);
     using Smem = tmak::Smem;
@@ -816,7 +843,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     const int num_m = (L + 2 * BM - 1) / (2 * BM);
     const int num_n = (N + BN - 1) / BN;
     const int num_tiles = num_m * ((num_n + PAIRS - 1) / PAIRS);
-    const int num_k = K / BK;
+    const int num_k = K / BKE;
     const int cluster = blockIdx.x / CL, num_clusters = gridDim.x / CL;
 
     if (threadIdx.x == 0) {
@@ -859,12 +886,12 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 if (elect_one()) {
                     if (half == 0) mbar_arrive_expect_tx(smem_addr(&sh->full[stage]), 2 * (A_BYTES + B_BYTES));
                     if (CL == 2) {
-                        tma_load_2d_pair(st, &tmap_a, kc * BK, m_rows, bar);
+                        tma_load_2d_pair(st, &tmap_a, kc * BKE, m_rows, bar);
                     } else {
-                        tma_load_2d_pair_multicast(st + pr * (A_BYTES / 2), &tmap_a, kc * BK,
+                        tma_load_2d_pair_multicast(st + pr * (A_BYTES / 2), &tmap_a, kc * BKE,
                                                    m_rows + (int)pr * (BM / 2), bar, a_mask);
                     }
-                    tma_load_2d_pair(st + A_BYTES, &tmap_b, kc * BK, n_rows, bar);
+                    tma_load_2d_pair(st + A_BYTES, &tmap_b, kc * BKE, n_rows, bar);
                 }
                 __syncwarp();
                 if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -894,9 +921,11 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                     const uint64_t bd = ad + (uint64_t)(A_BYTES >> 4);
                     if (elect_one()) {
                         #pragma unroll
-                        for (int ks = 0; ks < BK / UMMA_K; ++ks)
-                            mma_f8f6f4_pair(d_tmem, ad + (uint64_t)(ks * UMMA_K / 16), bd + (uint64_t)(ks * UMMA_K / 16),
-                                            IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
+                        for (int ks = 0; ks < BK / UMMA_K; ++ks) {
+                            const uint64_t adk = ad + (uint64_t)(ks * UMMA_K / 16), bdk = bd + (uint64_t)(ks * UMMA_K / 16);
+                            if (OPK == 0) mma_f8f6f4_pair(d_tmem, adk, bdk, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
+                            else mma_f16_pair(d_tmem, adk, bdk, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
+                        }
                         tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), ALL);
                     }
                     __syncwarp();
@@ -935,8 +964,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
             const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
             const int row = m0 + quarter * 32 + lane;
             const bool valid = row < L;
-            const float sa = valid ? __ldg(a.s_a + row) : 0.f;
-            {
+            const float sa = (DEQUANT && valid) ? __ldg(a.s_a + row) : 0.f;
+            if (DEQUANT) {
                 const int ncol = n0 + chalf * (BN / 2) + 4 * lane;
                 float4 w = make_float4(0.f, 0.f, 0.f, 0.f), bb = w;
                 if (ncol < N) {
@@ -963,14 +992,21 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 const float4* sw4 = reinterpret_cast<const float4*>(epi_sw + cc * 32);
                 const float4* b4 = reinterpret_cast<const float4*>(epi_b + cc * 32);
                 #pragma unroll
-                for (int u = 0; u < 8; ++u) {
+                for (int u = 0; u < 8 && !DEQUANT; ++u) {
+                    y[4 * u] = __uint_as_float(r[4 * u]);
+                    y[4 * u + 1] = __uint_as_float(r[4 * u + 1]);
+                    y[4 * u + 2] = __uint_as_float(r[4 * u + 2]);
+                    y[4 * u + 3] = __uint_as_float(r[4 * u + 3]);
+                }
+                #pragma unroll
+                for (int u = 0; u < 8 && DEQUANT; ++u) {
                     const float4 sw = sw4[u];
                     y[4 * u] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u]), sa), sw.x);
                     y[4 * u + 1] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 1]), sa), sw.y);
                     y[4 * u + 2] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 2]), sa), sw.z);
                     y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
                 }
-                if (a.bias != nullptr) {
+                if (DEQUANT && a.bias != nullptr) {
                     #pragma unroll
                     for (int u = 0; u < 8; ++u) {
                         const float4 bq = b4[u];
@@ -1027,10 +1063,11 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     if (warp == MMA_WARP) tmem_dealloc_pair(tmem_base, TMEM_COLS);
 }
 
-template <typename TOut, int CL>
+template <typename TOut, int CL, int OPK>
 cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
     constexpr int BM = tmak::BM, BN = tmak::BN, BN_CTA = tmak::BN_CTA, BK = tmak::BK;
-    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL>;
+    constexpr int ELEM = OPK == 0 ? 1 : 2;
+    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL, OPK>;
     static bool attr_set[64] = {false};
     static int max_clusters[64] = {0};
     int dev = 0;
@@ -1058,9 +1095,9 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
         attr_set[dev] = true;
     }
     CUtensorMap ta, tb, ty;
-    if (!encode_u8_tmap(&ta, a.Xe, (uint64_t)a.L, (uint64_t)a.K, CL == 2 ? BM : BM / 2, BK,
-                        CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_u8_tmap(&tb, a.We, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK, CU_TENSOR_MAP_SWIZZLE_128B) ||
+    const CUtensorMapDataType opt = OPK == 0 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
+    if (!encode_operand_tmap(&ta, a.Xe, opt, ELEM, (uint64_t)a.L, (uint64_t)a.K, CL == 2 ? BM : BM / 2, BK / ELEM) ||
+        !encode_operand_tmap(&tb, a.We, opt, ELEM, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK / ELEM) ||
         !encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N,
                          Out<TOut>::TMAP_SWIZZLE))
         return cudaErrorInvalidValue;
@@ -1073,10 +1110,10 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
     return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb, ty);
 }
 
-template <typename TOut>
+template <typename TOut, int OPK = 0>
 cudaError_t launch_tma_typed(const GemmArgs& a, cudaStream_t stream) {
     const int num_n = (a.N + tmak::BN - 1) / tmak::BN;
-    return num_n >= 2 ? launch_tma_cl<TOut, 4>(a, stream) : launch_tma_cl<TOut, 2>(a, stream);
+    return num_n >= 2 ? launch_tma_cl<TOut, 4, OPK>(a, stream) : launch_tma_cl<TOut, 2, OPK>(a, stream);
 }
 
 // Packed int4 -> E4M3: each thread turns 16 packed bytes into 32 E4M3 bytes.
@@ -1181,6 +1218,15 @@ cudaError_t launch_unpack_e4m3(const uint8_t* packed, uint8_t* e4m3, size_t rows
     unpack_e4m3_kernel<<<(unsigned)blocks, 256, 0, stream>>>(reinterpret_cast<const uint4*>(packed),
                                                                reinterpret_cast<uint4*>(e4m3), n16);
     return cudaGetLastError();
+}
+
+cudaError_t launch_fp16_gemm(const GemmArgs& a, cudaStream_t stream) {
+    if (a.L == 0) return cudaSuccess;
+    switch (a.y_dtype) {
+        case STARQ_F16: return launch_tma_typed<__half, 1>(a, stream);
+        case STARQ_BF16: return launch_tma_typed<__nv_bfloat16, 2>(a, stream);
+        default: return cudaErrorInvalidValue;
+    }
 }
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {

@@ -96,6 +96,17 @@ def test_unpack_null_and_alignment(lib):
     assert lib.lib.w4_unpack_e4m3(None, 0, 512, None, None) == 0
 
 
+@pytest.mark.parametrize("M,N,K,dt,code", [(4, 100, 512, 0, -2), (4, 256, 96, 0, -2), (-1, 256, 512, 0, -2),
+                                            (4, 256, 512, 2, -1), (0, 256, 512, 0, 0)])
+def test_fp16_gemm_validation(lib, M, N, K, dt, code):
+    assert lib.lib.fp16_gemm_ref(P, P, dt, M, N, K, P, None) == code
+
+
+def test_fp16_gemm_alignment(lib):
+    assert lib.lib.fp16_gemm_ref(ctypes.c_void_p(4098), P, 0, 4, 256, 512, P, None) == -3
+    assert lib.lib.fp16_gemm_ref(None, P, 0, 4, 256, 512, P, None) == -1
+
+
 @pytest.mark.parametrize("g,C,code", [(12, 96, -2), (16, 100, -2), (256, 4096, -2)])
 def test_tac_validation(lib, g, C, code):
     assert lib.lib.tac_apply(P, 0, 4, C, g, P, P, P, 0, None) == code

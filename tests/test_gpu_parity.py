@@ -202,6 +202,31 @@ def test_w4a4_gemm_exact(abi, L, N, K, out, path):
     H.assert_output_close(Y, osg.dequant(ref_acc, s_a, s_w, bias), out)
 
 
+@pytest.mark.parametrize("M,N,K,dt", [(1, 32, 64, "f16"), (129, 288, 640, "f16"), (300, 512, 1024, "bf16"),
+                                      (1024, 4096, 4096, "f16"), (77, 768, 4096, "bf16")])
+def test_fp16_gemm_ref(abi, M, N, K, dt):
+    """The 16-bit baseline GEMM against the exact product: float64 sums of
+    the 16-bit inputs; bound = one rounding to the element type plus float32
+    accumulation error (2^-22 K^(1/2) of the sum of |a b| per output)."""
+    rng = np.random.default_rng(M + N + K)
+    A = rng.standard_normal((M, K)).astype(np.float32)
+    B = rng.standard_normal((N, K)).astype(np.float32)
+    if dt == "f16":
+        A, B = A.astype(np.float16).astype(np.float32), B.astype(np.float16).astype(np.float32)
+    else:
+        A, B = inputs.round_to_bf16(A), inputs.round_to_bf16(B)
+    C = torch.empty(M, N, dtype=H.torch_dtype(dt), device="cuda")
+    abi.fp16_gemm_ref(H.dev(A, H.torch_dtype(dt)), H.dev(B, H.torch_dtype(dt)), C)
+    abi.check_status()
+    ref = A.astype(np.float64) @ B.astype(np.float64).T
+    mag = np.abs(A).astype(np.float64) @ np.abs(B).astype(np.float64).T
+    got = H.host(C).astype(np.float64)
+    tol = H.half_spacing(ref, dt) + 2.0 ** -22 * np.sqrt(K) * mag
+    if dt == "f16":
+        tol = np.maximum(tol, 2.0 ** -11 * np.abs(ref)) + 2.0 ** -22 * np.sqrt(K) * mag
+    assert np.all(np.abs(got - ref) <= tol), f"max excess {np.max(np.abs(got - ref) - tol)}"
+
+
 @pytest.mark.parametrize("path", ["tma", "e4m3", "packed"])
 @pytest.mark.parametrize("K", [18944, 65536])
 def test_w4a4_gemm_adversarial_exactness(abi, K, path):
