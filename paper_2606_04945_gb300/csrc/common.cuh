@@ -53,6 +53,15 @@ cudaError_t launch_fp16_gemm(const GemmArgs& a, cudaStream_t stream);
 // Packed int4 codes [rows][K/2] -> E4M3 bytes [rows][K].
 cudaError_t launch_unpack_e4m3(const uint8_t* packed, uint8_t* e4m3, size_t rows, int K, cudaStream_t stream);
 
+// Launch attribute that lets a kernel overlap its launch and prologue with
+// the tail of the previous kernel in the stream (see grid_dependency_wait).
+inline cudaLaunchAttribute pdl_attribute() {
+    cudaLaunchAttribute at;
+    at.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at.val.programmaticStreamSerializationAllowed = 1;
+    return at;
+}
+
 struct TacArgs {
     const void* Z; int z_dtype; int L; int C; int g;
     const float* M; const float* d; void* out; int out_dtype;
@@ -96,6 +105,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
                  "selp.u32 %0, 1, 0, p;\n\t}"
                  : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
     return ok != 0;
+}
+
+// Programmatic dependent launch. A kernel launched with the programmatic
+// stream-serialisation attribute may start while the previous kernel of the
+// stream is still running; it must call grid_dependency_wait() before its
+// first global-memory access (that waits until the previous grid has
+// completed and its writes are visible; a no-op without a programmatic
+// predecessor). grid_launch_dependents() lets the next such launch begin
+// once every CTA of this grid has called it or exited.
+__device__ __forceinline__ void grid_dependency_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // One lane of a converged warp (the lowest active lane) gets true.

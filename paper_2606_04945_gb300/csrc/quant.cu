@@ -398,6 +398,8 @@ sgat_quant_rows_kernel(QuantArgs a) {
     __shared__ __align__(16) float buf[4096];
     __shared__ __align__(16) float xst[4096];
     __shared__ float red[4];
+    grid_dependency_wait();            // launched with programmatic serialisation
+    grid_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int row = blockIdx.x;
@@ -583,18 +585,27 @@ sgat_quant_rows_kernel(QuantArgs a) {
     }
 }
 
+template <int NR, typename Tin>
+cudaError_t launch_rows_nr(const QuantArgs& a, cudaStream_t stream) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1] = {pdl_attribute()};
+    cfg.gridDim = dim3(a.L);
+    cfg.blockDim = dim3(128);
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin>, a);
+}
+
 template <typename Tin>
 cudaError_t launch_rows(const QuantArgs& a, cudaStream_t stream) {
-    const int nr = (a.K + 4095) / 4096;
-    dim3 grid(a.L), block(128);
-    switch (nr) {
-        case 1: sgat_quant_rows_kernel<1, Tin><<<grid, block, 0, stream>>>(a); break;
-        case 2: sgat_quant_rows_kernel<2, Tin><<<grid, block, 0, stream>>>(a); break;
-        case 3: sgat_quant_rows_kernel<3, Tin><<<grid, block, 0, stream>>>(a); break;
-        case 4: sgat_quant_rows_kernel<4, Tin><<<grid, block, 0, stream>>>(a); break;
+    switch ((a.K + 4095) / 4096) {
+        case 1: return launch_rows_nr<1, Tin>(a, stream);
+        case 2: return launch_rows_nr<2, Tin>(a, stream);
+        case 3: return launch_rows_nr<3, Tin>(a, stream);
+        case 4: return launch_rows_nr<4, Tin>(a, stream);
         default: return cudaErrorInvalidValue;
     }
-    return cudaGetLastError();
 }
 
 template <int E, typename Tin>

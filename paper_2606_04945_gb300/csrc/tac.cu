@@ -219,6 +219,9 @@ tac_tc_kernel(TacArgs a, int tiles_per_cta, const __grid_constant__ CUtensorMap 
         tmem_relinquish();
     }
     __syncthreads();
+    // the prologue above may overlap the previous kernel (programmatic launch)
+    grid_dependency_wait();
+    grid_launch_dependents();
     if (threadIdx.x == 0) {
         // M_b (float32, contiguous) and the first Z tiles in flight together
         mbar_arrive_expect_tx(smem_addr(&mbar_raw), P::MF32_BYTES);
@@ -421,9 +424,15 @@ cudaError_t launch_tc(const TacArgs& a, cudaStream_t stream) {
     int per = (blocks * tiles + 2 * num_sms() - 1) / (2 * num_sms());
     if (per < 2) per = tiles < 2 ? tiles : 2;
     if (per > tiles) per = tiles;
-    dim3 grid(blocks, (tiles + per - 1) / per);
-    tac_tc_kernel<G, TIn, TOut><<<grid, TC_THREADS, P::SMEM, stream>>>(a, per, tz, to, a.status);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1] = {pdl_attribute()};
+    cfg.gridDim = dim3(blocks, (tiles + per - 1) / per);
+    cfg.blockDim = dim3(TC_THREADS);
+    cfg.dynamicSmemBytes = P::SMEM;
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, tac_tc_kernel<G, TIn, TOut>, a, per, tz, to, a.status);
 }
 
 template <typename TIn, typename TOut>

@@ -867,6 +867,10 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     cluster_sync();              // barriers of every CTA initialised, TMEM allocated
     tc_fence_after();
     const uint32_t tmem_base = sh->tmem_base;
+    // the prologue above may overlap the previous kernel; no global memory
+    // is touched before its results are visible
+    grid_dependency_wait();
+    grid_launch_dependents();
 
     // The producer and MMA roles run their loops with the whole warp (warp-
     // uniform control flow and descriptors); one elected lane issues.
@@ -1073,16 +1077,17 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = CL;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1] = pdl_attribute();
     cfg.blockDim = dim3(tmak::THREADS);
     cfg.dynamicSmemBytes = tmak::SMEM_BYTES;
     cfg.stream = stream;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 1;                // the occupancy query takes the cluster shape only
     if (dev < 64 && !attr_set[dev]) {
         cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)tmak::SMEM_BYTES);
@@ -1107,6 +1112,7 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
     if (clusters < 1) clusters = 1;
     if (num_tiles < clusters) clusters = num_tiles;
     cfg.gridDim = dim3(CL * clusters);
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb, ty);
 }
 
