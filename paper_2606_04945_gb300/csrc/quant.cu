@@ -304,8 +304,9 @@ template <> struct To<float> { static __device__ __forceinline__ float f(float h
 // multiple of 1024, K <= 4096 NR): one CTA of four warps per row, in rounds
 // of 4096 elements (four 1024-element chunks, chunk j of a round in warp j).
 // A warp reads its chunk of x and of the smoothing vector with coalesced
-// 16-byte loads (lane l at 16 l + 512 q) into shared memory and takes it
-// back in layout A.
+// 16-byte loads (lane l at 16 l + 512 q) and passes each through its
+// shared slice to take it back in layout A (16 KB of shared memory per CTA,
+// so registers, not shared memory, bound the CTAs per SM).
 //
 //   layout A  lane l holds elements 32 l .. 32 l + 31 of its warp's chunk:
 //             stages h = 1 .. 16 are between registers;
@@ -396,7 +397,6 @@ template <int NR, typename Tin>
 __global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
 sgat_quant_rows_kernel(QuantArgs a) {
     __shared__ __align__(16) float buf[4096];
-    __shared__ __align__(16) float xst[4096];
     __shared__ float red[4];
     grid_dependency_wait();            // launched with programmatic serialisation
     grid_launch_dependents();
@@ -419,21 +419,17 @@ sgat_quant_rows_kernel(QuantArgs a) {
         const int nch = min(4, (K - base) >> 10);        // chunks in this round (>= 1)
         float u[32];
         if (warp < nch) {
-            // coalesced loads (lane l: 16 bytes at 16 l + 512 q), staged
-            // through shared memory and read back in layout A
+            // coalesced loads (lane l: 16 bytes at 16 l + 512 q); x and then
+            // the smoothing vector pass through the warp's slice and come
+            // back in layout A
             const int c0 = base + warp * 1024;                   // first element of the chunk
-            float* stage = xst + warp * 1024;                    // 4 KB per warp
+            float4 sr[8];
             if (sizeof(Tin) == 2) {
                 uint4 xr[4];
                 #pragma unroll
                 for (int q = 0; q < 4; ++q) xr[q] = __ldg(reinterpret_cast<const uint4*>(X + c0) + lane + 32 * q);
-                float4 sr[8];
-                if (sm != nullptr) {
-                    #pragma unroll
-                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
-                }
-                // fp16 staging: 32 rows of 64 bytes, 16-byte group g of row R at g ^ ((R >> 1) & 3)
-                uint8_t* st8 = reinterpret_cast<uint8_t*>(stage);
+                // 16-bit staging: 32 rows of 64 bytes, 16-byte group g of row R at g ^ ((R >> 1) & 3)
+                uint8_t* st8 = reinterpret_cast<uint8_t*>(slice);
                 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     const int R = (lane >> 2) + 8 * q, g = lane & 3;
@@ -441,8 +437,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 }
                 if (sm != nullptr) {
                     #pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
+                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
                 }
                 __syncwarp();
                 #pragma unroll
@@ -453,29 +448,29 @@ sgat_quant_rows_kernel(QuantArgs a) {
                     for (int k = 0; k < 8; ++k) u[8 * g + k] = To<Tin>::f(h[k]);
                 }
             } else {
-                float4 xr[8], sr[8];
+                float4 xr[8];
                 #pragma unroll
                 for (int q = 0; q < 8; ++q) xr[q] = __ldg(reinterpret_cast<const float4*>(X + c0) + lane + 32 * q);
+                #pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = xr[q];
                 if (sm != nullptr) {
                     #pragma unroll
                     for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
                 }
-                #pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    *reinterpret_cast<float4*>(stage + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = xr[q];
-                if (sm != nullptr) {
-                    #pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
-                }
                 __syncwarp();
                 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
-                    const float4 w = *reinterpret_cast<const float4*>(stage + swz(lane, 4 * q));
+                    const float4 w = *reinterpret_cast<const float4*>(slice + swz(lane, 4 * q));
                     u[4 * q] = w.x; u[4 * q + 1] = w.y; u[4 * q + 2] = w.z; u[4 * q + 3] = w.w;
                 }
             }
             if (sm != nullptr) {
+                __syncwarp();                                    // x has left the slice
+                #pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
+                __syncwarp();
                 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
                     const float4 w = *reinterpret_cast<const float4*>(slice + swz(lane, 4 * q));

@@ -80,6 +80,19 @@ __device__ __forceinline__ void convert_store(uint32_t tile, int row, int q, uin
 }
 
 template <typename TOut> struct Out;
+// (a s, b s) then (. * t0, . * t1): two packed round-to-nearest multiplies,
+// each half rounding like the scalar operation.
+__device__ __forceinline__ void mul2_rn(float a, float b, float s, float t0, float t1, float& y0, float& y1) {
+    asm("{\n\t.reg .b64 V, S, T;\n\t"
+        "mov.b64 V, {%2, %3};\n\t"
+        "mov.b64 S, {%4, %4};\n\t"
+        "mov.b64 T, {%5, %6};\n\t"
+        "mul.rn.f32x2 V, V, S;\n\t"
+        "mul.rn.f32x2 V, V, T;\n\t"
+        "mov.b64 {%0, %1}, V;\n\t}"
+        : "=f"(y0), "=f"(y1) : "f"(a), "f"(b), "f"(s), "f"(t0), "f"(t1));
+}
+
 // Row `row` (32 values) of a 32 x 32 output box staged for a TMA store:
 // 16-bit types use 64-byte rows with the 64-byte swizzle (16-byte group g at
 // g ^ ((row >> 1) & 3)), float uses 128-byte rows with the 128-byte swizzle
@@ -786,7 +799,6 @@ bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t
 // ---------------------------------------------------------------------------
 namespace tmak {
 constexpr int BM = 128, BN = 256, BN_CTA = 128, BK = 128, UMMA_K = 32;
-constexpr int STAGES = 5;
 constexpr int A_BYTES = BM * BK, B_BYTES = BN_CTA * BK;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;             // 32 KB
 constexpr int NUM_EPI_WARPS = 8;
@@ -794,18 +806,27 @@ constexpr int TMA_WARP = 8, MMA_WARP = 9;
 constexpr int THREADS = 10 * 32;
 constexpr int TMEM_COLS = 512;
 constexpr int EPI_PARAM_BYTES = NUM_EPI_WARPS * 2 * (BN / 2) * 4;
-constexpr int EPI_BOX_WARP_BYTES = 4096;                  // two 32 x 32 16-bit boxes or one float box
-constexpr int EPI_STAGE_BYTES = NUM_EPI_WARPS * EPI_BOX_WARP_BYTES;
-constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + EPI_STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
 constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
+template <int S>
 struct Smem {
-    uint64_t full[STAGES];        // pair leader: both CTAs' TMA bytes
-    uint64_t empty[STAGES];       // MMA commits of every pair of the cluster
+    uint64_t full[S];             // pair leader: both CTAs' TMA bytes
+    uint64_t empty[S];            // MMA commits of every pair of the cluster
     uint64_t tmem_full[2];
     uint64_t tmem_empty[2];       // pair leader: epilogue warps of the pair
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
+};
+// Per output element size: one 32 x 32 staging box per epilogue warp, and
+// as many 32 KB stages as the rest of the 227 KB allows (6 for 16-bit
+// outputs, 5 for float).
+template <int OUT_BYTES>
+struct Cfg {
+    static constexpr int EPI_BOX_WARP_BYTES = 32 * 32 * OUT_BYTES;
+    static constexpr int EPI_STAGE_BYTES = NUM_EPI_WARPS * EPI_BOX_WARP_BYTES;
+    static constexpr int STAGES = OUT_BYTES == 4 ? 5 : 6;
+    static constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + EPI_STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
+    static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
 };
 }  // namespace tmak
 
@@ -817,7 +838,7 @@ __global__ void __launch_bounds__(tmak::THREADS, 1)
 w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
                           const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y) {
     constexpr int BM = tmak::BM, BN = tmak::BN, BN_CTA = tmak::BN_CTA, BK = tmak::BK;
-    constexpr int UMMA_K = tmak::UMMA_K, STAGES = tmak::STAGES, STAGE_BYTES = tmak::STAGE_BYTES;
+    constexpr int UMMA_K = tmak::UMMA_K, STAGES = tmak::Cfg<sizeof(TOut)>::STAGES, STAGE_BYTES = tmak::STAGE_BYTES;
     constexpr int A_BYTES = tmak::A_BYTES, B_BYTES = tmak::B_BYTES;
     constexpr int TMA_WARP = tmak::TMA_WARP, MMA_WARP = tmak::MMA_WARP;
     constexpr int NUM_EPI_WARPS = tmak::NUM_EPI_WARPS, TMEM_COLS = tmak::TMEM_COLS;
@@ -826,13 +847,14 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     constexpr bool DEQUANT = OPK == 0;
     constexpr int PAIRS = CL / 2;
     constexpr uint16_t ALL = (uint16_t)((1u << CL) - 1u);
-    using Smem = tmak::Smem;
+    using Smem = tmak::Smem<STAGES>;
     static_assert(CL == 2 || CL == 4, "one or two CTA pairs per cluster");
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
-    constexpr int EPI_STAGE_BYTES = tmak::EPI_STAGE_BYTES, EPI_BOX_WARP_BYTES = tmak::EPI_BOX_WARP_BYTES;
+    constexpr int EPI_STAGE_BYTES = tmak::Cfg<sizeof(TOut)>::EPI_STAGE_BYTES;
+    constexpr int EPI_BOX_WARP_BYTES = tmak::Cfg<sizeof(TOut)>::EPI_BOX_WARP_BYTES;
     Smem* sh = reinterpret_cast<Smem*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES + EPI_STAGE_BYTES);
     volatile int* abort = &sh->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1002,13 +1024,25 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                     y[4 * u + 2] = __uint_as_float(r[4 * u + 2]);
                     y[4 * u + 3] = __uint_as_float(r[4 * u + 3]);
                 }
-                #pragma unroll
-                for (int u = 0; u < 8 && DEQUANT; ++u) {
-                    const float4 sw = sw4[u];
-                    y[4 * u] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u]), sa), sw.x);
-                    y[4 * u + 1] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 1]), sa), sw.y);
-                    y[4 * u + 2] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 2]), sa), sw.z);
-                    y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
+                if (DEQUANT && a.bias == nullptr) {
+                    // fl(fl(acc s_a) s_w) on packed pairs (two multiplies: nothing to contract)
+                    #pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const float4 sw = sw4[u];
+                        mul2_rn(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]), sa, sw.x, sw.y,
+                                y[4 * u], y[4 * u + 1]);
+                        mul2_rn(__uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]), sa, sw.z, sw.w,
+                                y[4 * u + 2], y[4 * u + 3]);
+                    }
+                } else if (DEQUANT) {
+                    #pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const float4 sw = sw4[u];
+                        y[4 * u] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u]), sa), sw.x);
+                        y[4 * u + 1] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 1]), sa), sw.y);
+                        y[4 * u + 2] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 2]), sa), sw.z);
+                        y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
+                    }
                 }
                 if (DEQUANT && a.bias != nullptr) {
                     #pragma unroll
@@ -1084,13 +1118,13 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
     attr[0].val.clusterDim.z = 1;
     attr[1] = pdl_attribute();
     cfg.blockDim = dim3(tmak::THREADS);
-    cfg.dynamicSmemBytes = tmak::SMEM_BYTES;
+    cfg.dynamicSmemBytes = tmak::Cfg<sizeof(TOut)>::SMEM_BYTES;
     cfg.stream = stream;
     cfg.attrs = attr;
     cfg.numAttrs = 1;                // the occupancy query takes the cluster shape only
     if (dev < 64 && !attr_set[dev]) {
         cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)tmak::SMEM_BYTES);
+                                             (int)tmak::Cfg<sizeof(TOut)>::SMEM_BYTES);
         if (e != cudaSuccess) return e;
         cfg.gridDim = dim3(CL * 32);
         int n = 0;
