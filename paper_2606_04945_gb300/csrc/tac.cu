@@ -141,19 +141,18 @@ cudaError_t launch_g(const TacArgs& a, cudaStream_t stream) {
 // by 16-byte row stores.
 // ---------------------------------------------------------------------------
 constexpr int TC_TM = 128;              // tokens per tile (MMA M)
-constexpr int TC_THREADS = 128;
+constexpr int TC_THREADS = 256;
 
 template <int G>
 struct TacTc {
     static constexpr int ATOMS = G / 64;                      // 64 16-bit elements = 128 B per atom row
-    static constexpr int Z_BYTES = TC_TM * G * 2;             // one Z tile
+    static constexpr int Z_BYTES = TC_TM * G * 2;             // the Z tile
     static constexpr int M_BYTES = G * G * 2;                 // one of M_hi / M_lo
-    static constexpr int MF32_BYTES = G * G * 4;              // M_b in float32
-    static constexpr int STAGE_OUT_BYTES = TC_TM * G * 4;     // float32 output tile
-    // M_b in float32 first, the output staging afterwards
-    static constexpr int RAW_BYTES = MF32_BYTES > STAGE_OUT_BYTES ? MF32_BYTES : STAGE_OUT_BYTES;
-    static constexpr size_t SMEM = 2 * (size_t)Z_BYTES + 2 * (size_t)M_BYTES + RAW_BYTES + 1024 + 256;
-    static constexpr int TMEM_COLS = 2 * G;                   // two accumulators
+    static constexpr int OUT_BYTES = (TC_THREADS / 32) * 32 * 32 * 4;   // one float 32 x 32 box per warp
+    // the Z tile's space holds the output boxes once the MMAs have read it
+    static constexpr int REGION = Z_BYTES > OUT_BYTES ? Z_BYTES : OUT_BYTES;
+    static constexpr size_t SMEM = (size_t)REGION + 2 * (size_t)M_BYTES + 1024;
+    static constexpr int TMEM_COLS = G;
 };
 
 template <typename T> struct Split16;
@@ -184,33 +183,39 @@ template <> struct TacStore<float> {
 template <> struct TacStore<__half> { static constexpr bool TMA = false; };
 template <> struct TacStore<__nv_bfloat16> { static constexpr bool TMA = false; };
 
+// Tensor-core TAC: one CTA per (block b, tile of 128 tokens), 8 warps.
+//   * the tile Z[rows][b g .. b g + g) arrives by TMA (128-byte swizzle);
+//   * meanwhile all threads read M_b (float32) with coalesced 32-byte loads
+//     and write its two 16-bit halves hi = rn(M), lo = rn(M - hi) (the
+//     input's type) into the K-major swizzled operand layout;
+//   * one thread issues g/16 pairs of kind::f16 MMAs (Z hi^T and Z lo^T,
+//     float32 accumulation in TMEM: relative error about 2^-22);
+//   * each warp reads 32 tokens x g/2 channels of the accumulator, adds d,
+//     and stores: float output through 32 x 32 boxes (staged in the Z
+//     tile's space, which the MMAs no longer need) and TMA stores, 16-bit
+//     output with direct row stores.
+// About 97 KB of shared memory at g = 128, so two CTAs share an SM.
 template <int G, typename TIn, typename TOut>
-__global__ void __launch_bounds__(TC_THREADS, 1)
-tac_tc_kernel(TacArgs a, int tiles_per_cta, const __grid_constant__ CUtensorMap tmap_z,
-              const __grid_constant__ CUtensorMap tmap_out, unsigned* status) {
+__global__ void __launch_bounds__(TC_THREADS)
+tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __grid_constant__ CUtensorMap tmap_out,
+              unsigned* status) {
     using P = TacTc<G>;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t zfull[2], mdone[2], mbar_raw;
+    __shared__ __align__(8) uint64_t zfull, mdone;
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
-    const uint32_t sZ = base;                                  // 2 x Z tile
-    const uint32_t sMh = base + 2 * P::Z_BYTES, sMl = sMh + P::M_BYTES;
-    const uint32_t sRaw = sMl + P::M_BYTES;                    // M_b float32, then output staging
+    const uint32_t sZ = base;                                  // Z tile, then output boxes
+    const uint32_t sMh = base + P::REGION, sMl = sMh + P::M_BYTES;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int b = blockIdx.x;
-    const int t0 = blockIdx.y * tiles_per_cta;
-    const int n_tiles_total = (a.L + TC_TM - 1) / TC_TM;
-    const int nt = min(tiles_per_cta, n_tiles_total - t0);
+    const int row0 = blockIdx.y * TC_TM;
     volatile int* abort = &abort_flag;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(smem_addr(&zfull[i]), 1);
-            mbar_init(smem_addr(&mdone[i]), 1);
-        }
-        mbar_init(smem_addr(&mbar_raw), 1);
+        mbar_init(smem_addr(&zfull), 1);
+        mbar_init(smem_addr(&mdone), 1);
         abort_flag = 0;
         mbar_fence_init();
     }
@@ -223,25 +228,18 @@ tac_tc_kernel(TacArgs a, int tiles_per_cta, const __grid_constant__ CUtensorMap 
     grid_dependency_wait();
     grid_launch_dependents();
     if (threadIdx.x == 0) {
-        // M_b (float32, contiguous) and the first Z tiles in flight together
-        mbar_arrive_expect_tx(smem_addr(&mbar_raw), P::MF32_BYTES);
-        bulk_load(sRaw, a.M + (size_t)b * G * G, P::MF32_BYTES, smem_addr(&mbar_raw));
-        for (int i = 0; i < 2 && i < nt; ++i) {
-            const uint32_t bar = smem_addr(&zfull[i]);
-            mbar_arrive_expect_tx(bar, P::Z_BYTES);
-            for (int at = 0; at < P::ATOMS; ++at)
-                tma_load_2d(sZ + i * P::Z_BYTES + at * (TC_TM * 128), &tmap_z, b * G + at * 64, (t0 + i) * TC_TM, bar);
-        }
+        mbar_arrive_expect_tx(smem_addr(&zfull), P::Z_BYTES);
+        for (int at = 0; at < P::ATOMS; ++at)
+            tma_load_2d(sZ + at * (TC_TM * 128), &tmap_z, b * G + at * 64, row0, smem_addr(&zfull));
     }
-    bool ok = mbar_wait_bounded(smem_addr(&mbar_raw), 0, abort);
-    // M_b -> hi / lo 16-bit tiles, K-major (row r = output channel, 8 inputs per 16-byte chunk)
-    for (int idx = threadIdx.x; ok && idx < G * G / 8; idx += TC_THREADS) {
+    // M_b -> hi / lo, K-major (row r = output channel, 8 inputs per 16-byte chunk)
+    const float* Mb = a.M + (size_t)b * G * G;
+    #pragma unroll 2
+    for (int idx = threadIdx.x; idx < G * G / 8; idx += TC_THREADS) {
         const int r = idx / (G / 8), jc = idx % (G / 8);      // inputs j = 8 jc .. 8 jc + 7
-        const uint4 w0 = ld_shared_v4(sRaw + (uint32_t)(r * G + 8 * jc) * 4);
-        const uint4 w1 = ld_shared_v4(sRaw + (uint32_t)(r * G + 8 * jc + 4) * 4);
-        const float mv[8] = {__uint_as_float(w0.x), __uint_as_float(w0.y), __uint_as_float(w0.z),
-                             __uint_as_float(w0.w), __uint_as_float(w1.x), __uint_as_float(w1.y),
-                             __uint_as_float(w1.z), __uint_as_float(w1.w)};
+        const float4 w0 = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc));
+        const float4 w1 = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc + 4));
+        const float mv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
         uint32_t hi[4], lo[4];
         #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -251,8 +249,7 @@ tac_tc_kernel(TacArgs a, int tiles_per_cta, const __grid_constant__ CUtensorMap 
             hi[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
             lo[e] = (uint32_t)l0 | ((uint32_t)l1 << 16);
         }
-        const int at = jc / 8, c = jc % 8;                    // atom, 16-byte chunk in the 128-byte row
-        const uint32_t off = at * (G * 128) + sw128_offset(r, c);
+        const uint32_t off = (jc / 8) * (G * 128) + sw128_offset(r, jc % 8);
         st_shared_v4(sMh + off, hi[0], hi[1], hi[2], hi[3]);
         st_shared_v4(sMl + off, lo[0], lo[1], lo[2], lo[3]);
     }
@@ -263,70 +260,65 @@ tac_tc_kernel(TacArgs a, int tiles_per_cta, const __grid_constant__ CUtensorMap 
     const uint32_t tmem = tmem_slot;
     constexpr uint32_t IDESC = (1u << 4) | (Split16<TIn>::KIND << 7) | (Split16<TIn>::KIND << 10) |
                                ((uint32_t)(G >> 3) << 17) | ((uint32_t)(TC_TM >> 4) << 24);
-    TOut* out = static_cast<TOut*>(a.out);
-    // per-warp staging of its 32 rows: G/32 boxes of 32 x 32 float32
-    const uint32_t stage_w = sRaw + warp * (32 * G * 4);
-    for (int i = 0; i < nt && ok; ++i) {
-        const int buf = i & 1;
-        const uint32_t ph = (uint32_t)(i >> 1) & 1u;
-        if (threadIdx.x == 0) {
-            if (!mbar_wait_bounded(smem_addr(&zfull[buf]), ph, abort)) { ok = false; *abort = 1; }
-            else {
-                tc_fence_after();
-                const uint32_t d = tmem + (uint32_t)(buf * G);
-                #pragma unroll
-                for (int ks = 0; ks < G / 16; ++ks) {
-                    const uint32_t koff = (ks / 4) * (TC_TM * 128) + (ks % 4) * 32;
-                    const uint32_t moff = (ks / 4) * (G * 128) + (ks % 4) * 32;
-                    const uint64_t ad = smem_desc_sw128(sZ + buf * P::Z_BYTES + koff);
-                    mma_f16(d, ad, smem_desc_sw128(sMh + moff), IDESC, ks > 0 ? 1u : 0u);
-                    mma_f16(d, ad, smem_desc_sw128(sMl + moff), IDESC, 1u);
-                }
-                tc_commit(smem_addr(&mdone[buf]));
+    if (threadIdx.x == 0) {
+        if (!mbar_wait_bounded(smem_addr(&zfull), 0, abort)) {
+            *abort = 1;
+        } else {
+            tc_fence_after();
+            #pragma unroll
+            for (int ks = 0; ks < G / 16; ++ks) {
+                const uint32_t koff = (ks / 4) * (TC_TM * 128) + (ks % 4) * 32;
+                const uint32_t moff = (ks / 4) * (G * 128) + (ks % 4) * 32;
+                const uint64_t ad = smem_desc_sw128(sZ + koff);
+                mma_f16(tmem, ad, smem_desc_sw128(sMh + moff), IDESC, ks > 0 ? 1u : 0u);
+                mma_f16(tmem, ad, smem_desc_sw128(sMl + moff), IDESC, 1u);
             }
         }
-        if (!mbar_wait_bounded(smem_addr(&mdone[buf]), ph, abort)) ok = false;
-        __syncthreads();
-        if (!ok || *abort) { ok = false; break; }
-        tc_fence_after();
-        // the Z buffer is free again: fetch the tile after next
-        if (threadIdx.x == 0 && i + 2 < nt) {
-            const uint32_t bar = smem_addr(&zfull[buf]);
-            mbar_arrive_expect_tx(bar, P::Z_BYTES);
-            for (int at = 0; at < P::ATOMS; ++at)
-                tma_load_2d(sZ + buf * P::Z_BYTES + at * (TC_TM * 128), &tmap_z, b * G + at * 64, (t0 + i + 2) * TC_TM, bar);
-        }
-        const int row0 = (t0 + i) * TC_TM + warp * 32;
-        const int tok = row0 + lane;
-        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * G);
+        tc_commit(smem_addr(&mdone));       // also after a failed wait: nothing was issued
+    }
+    bool ok = mbar_wait_bounded(smem_addr(&mdone), 0, abort) && !*abort;
+    tc_fence_after();
+    if (ok) {
+        const int quarter = warp & 3, chalf = warp >> 2;
+        const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+        const int tok = row0 + quarter * 32 + lane;
         const float* dp = a.d ? a.d + (size_t)b * G : nullptr;
-        if (TacStore<TOut>::TMA && lane == 0) bulk_wait_read0();   // previous tile's stores left the staging
-        __syncwarp();
+        const uint32_t box = sZ + warp * (32 * 32 * 4);
+        TOut* out = static_cast<TOut*>(a.out);
         #pragma unroll 1
-        for (int c = 0; c < G / 32; ++c) {
+        for (int c = 0; c < G / 64; ++c) {
+            const int col = chalf * (G / 2) + c * 32;
             uint32_t r[32];
-            tmem_ld_32x32b_x32(trow + c * 32, r);
+            tmem_ld_32x32b_x32(trow + col, r);
             tmem_ld_wait();
             float v[32];
             #pragma unroll
             for (int j = 0; j < 32; j += 4) {
                 float4 dd = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (dp) dd = __ldg(reinterpret_cast<const float4*>(dp + c * 32 + j));
+                if (dp) dd = __ldg(reinterpret_cast<const float4*>(dp + col + j));
                 v[j] = __uint_as_float(r[j]) + dd.x;
                 v[j + 1] = __uint_as_float(r[j + 1]) + dd.y;
                 v[j + 2] = __uint_as_float(r[j + 2]) + dd.z;
                 v[j + 3] = __uint_as_float(r[j + 3]) + dd.w;
             }
             if (TacStore<TOut>::TMA) {
-                // box c of this warp: row `lane`, 16-byte chunk q at (q ^ (lane & 7))
-                const uint32_t box = stage_w + c * (32 * 128);
+                if (c > 0) {                                     // the previous box has been read
+                    if (lane == 0) bulk_wait_read0();
+                    __syncwarp();
+                }
                 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     st_shared_v4(box + lane * 128 + ((q ^ (lane & 7)) << 4), __float_as_uint(v[4 * q]),
                                  __float_as_uint(v[4 * q + 1]), __float_as_uint(v[4 * q + 2]),
                                  __float_as_uint(v[4 * q + 3]));
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&tmap_out, b * G + col, row0 + quarter * 32, box);
+                    bulk_commit();
+                }
             } else if (tok < a.L) {
-                TOut* o = out + (size_t)tok * a.C + b * G + c * 32;
+                TOut* o = out + (size_t)tok * a.C + b * G + col;
                 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     uint32_t w[4];
@@ -340,20 +332,11 @@ tac_tc_kernel(TacArgs a, int tiles_per_cta, const __grid_constant__ CUtensorMap 
                 }
             }
         }
-        if (TacStore<TOut>::TMA) {
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                for (int c = 0; c < G / 32; ++c)
-                    tma_store_2d(&tmap_out, b * G + c * 32, row0, stage_w + c * (32 * 128));
-                bulk_commit();
-            }
-        }
-        tc_fence_before();
-        __syncthreads();
+        if (TacStore<TOut>::TMA && lane == 0) bulk_wait0();
+        __syncwarp();
+    } else if (threadIdx.x == 0) {
+        atomicOr(status, STATUS_TIMEOUT_TAC);
     }
-    if (TacStore<TOut>::TMA && lane == 0) bulk_wait0();
-    if (!ok && threadIdx.x == 0) atomicOr(status, STATUS_TIMEOUT_TAC);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -418,21 +401,15 @@ cudaError_t launch_tc(const TacArgs& a, cudaStream_t stream) {
     } else {
         to = tz;   // unused
     }
-    const int blocks = a.C / G;
-    const int tiles = (a.L + TC_TM - 1) / TC_TM;
-    // about two CTAs' worth of work per SM, at least two tiles per CTA when possible
-    int per = (blocks * tiles + 2 * num_sms() - 1) / (2 * num_sms());
-    if (per < 2) per = tiles < 2 ? tiles : 2;
-    if (per > tiles) per = tiles;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute at[1] = {pdl_attribute()};
-    cfg.gridDim = dim3(blocks, (tiles + per - 1) / per);
+    cfg.gridDim = dim3(a.C / G, (a.L + TC_TM - 1) / TC_TM);
     cfg.blockDim = dim3(TC_THREADS);
     cfg.dynamicSmemBytes = P::SMEM;
     cfg.stream = stream;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, tac_tc_kernel<G, TIn, TOut>, a, per, tz, to, a.status);
+    return cudaLaunchKernelEx(&cfg, tac_tc_kernel<G, TIn, TOut>, a, tz, to, a.status);
 }
 
 template <typename TIn, typename TOut>
