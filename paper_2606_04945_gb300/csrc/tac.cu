@@ -145,6 +145,7 @@ constexpr int TC_THREADS = 256;
 
 template <int G>
 struct TacTc {
+    static_assert(G * G / 8 % TC_THREADS == 0, "whole load rounds per thread");
     static constexpr int ATOMS = G / 64;                      // 64 16-bit elements = 128 B per atom row
     static constexpr int Z_BYTES = TC_TM * G * 2;             // the Z tile
     static constexpr int M_BYTES = G * G * 2;                 // one of M_hi / M_lo
@@ -232,14 +233,23 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
         for (int at = 0; at < P::ATOMS; ++at)
             tma_load_2d(sZ + at * (TC_TM * 128), &tmap_z, b * G + at * 64, row0, smem_addr(&zfull));
     }
-    // M_b -> hi / lo, K-major (row r = output channel, 8 inputs per 16-byte chunk)
+    // M_b -> hi / lo, K-major (row r = output channel, 8 inputs per 16-byte
+    // chunk); every load of the thread is issued before the first convert
     const float* Mb = a.M + (size_t)b * G * G;
-    #pragma unroll 2
-    for (int idx = threadIdx.x; idx < G * G / 8; idx += TC_THREADS) {
+    constexpr int NIT = G * G / 8 / TC_THREADS;
+    float4 w0[NIT], w1[NIT];
+    #pragma unroll
+    for (int it = 0; it < NIT; ++it) {
+        const int idx = threadIdx.x + it * TC_THREADS;
+        const int r = idx / (G / 8), jc = idx % (G / 8);
+        w0[it] = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc));
+        w1[it] = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc + 4));
+    }
+    #pragma unroll
+    for (int it = 0; it < NIT; ++it) {
+        const int idx = threadIdx.x + it * TC_THREADS;
         const int r = idx / (G / 8), jc = idx % (G / 8);      // inputs j = 8 jc .. 8 jc + 7
-        const float4 w0 = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc));
-        const float4 w1 = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc + 4));
-        const float mv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+        const float mv[8] = {w0[it].x, w0[it].y, w0[it].z, w0[it].w, w1[it].x, w1[it].y, w1[it].z, w1[it].w};
         uint32_t hi[4], lo[4];
         #pragma unroll
         for (int e = 0; e < 4; ++e) {
