@@ -27,3 +27,10 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+@pytest.fixture(scope="module")
+def abi():
+    """The ctypes binding of libstarq.so (GPU tests)."""
+    from paper_2606_04945_gb300 import abi as a
+    return a

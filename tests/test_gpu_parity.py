@@ -19,12 +19,6 @@ from tests import helpers as H
 pytestmark = pytest.mark.gpu
 
 
-@pytest.fixture(scope="module")
-def abi():
-    from paper_2606_04945_gb300 import abi as a
-    return a
-
-
 def run_quant(abi, case, mask=True, dbg=True):
     xf = case.xf
     X = H.dev(case.X, H.torch_dtype(case.dtype))
