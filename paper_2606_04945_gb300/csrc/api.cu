@@ -274,6 +274,9 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");
     GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
+    // the GEMM's predecessor is the quantiser launched above, which waits for
+    // everything before it and does not write the weights
+    g.weights_ready = 1;
     if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: gemm launch");
     return STARQ_OK;
 }

@@ -45,6 +45,10 @@ struct GemmArgs {
     unsigned* status;
     const uint8_t* Xe = nullptr;   // optional E4M3 bytes of the activation codes [L][K]
     const uint8_t* We = nullptr;   // optional E4M3 bytes of the weight codes [N][K]
+    // The caller guarantees that no kernel still running when this one is
+    // launched writes the weights: their first tiles are fetched before
+    // the wait for the previous kernel (programmatic launch).
+    int weights_ready = 0;
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
 // Plain 16-bit GEMM C = A B^T (A = a.Xe [L][K], B = a.We [N][K], both of

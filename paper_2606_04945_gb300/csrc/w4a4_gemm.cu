@@ -890,8 +890,9 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     tc_fence_after();
     const uint32_t tmem_base = sh->tmem_base;
     // the prologue above may overlap the previous kernel; no global memory
-    // is touched before its results are visible
-    grid_dependency_wait();
+    // is touched before its results are visible (except the weight tiles
+    // of the first stages when the caller vouches for them: see below)
+    if (warp != TMA_WARP) grid_dependency_wait();
     grid_launch_dependents();
 
     // The producer and MMA roles run their loops with the whole warp (warp-
@@ -899,6 +900,22 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     if (warp == TMA_WARP) {
         const uint32_t leader_full0 = mapa_shared(smem_addr(&sh->full[0]), leader);
         const uint16_t a_mask = (uint16_t)((1u << rank) | (1u << ((rank ^ 2u) % CL)));
+        // weight tiles of the first stages ahead of the wait for the previous
+        // kernel (their stage barriers are fresh, so no empty wait is due)
+        int pre = 0;
+        if (a.weights_ready && cluster < num_tiles) {
+            pre = num_k < STAGES ? num_k : STAGES;
+            const int n_rows = ((cluster / num_m) * PAIRS + (int)pr) * BN + (int)half * BN_CTA;
+            for (int kc = 0; kc < pre; ++kc) {
+                if (elect_one()) {
+                    if (half == 0) mbar_arrive_expect_tx(smem_addr(&sh->full[kc]), 2 * (A_BYTES + B_BYTES));
+                    tma_load_2d_pair(base + kc * STAGE_BYTES + A_BYTES, &tmap_b, kc * BKE, n_rows,
+                                     leader_full0 + kc * 8);
+                }
+                __syncwarp();
+            }
+        }
+        grid_dependency_wait();
         int stage = 0;
         uint32_t phase = 0;
         bool ok = true;
@@ -906,18 +923,19 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
             const int m_rows = (tile % num_m) * 2 * BM + (int)half * BM;
             const int n_rows = ((tile / num_m) * PAIRS + (int)pr) * BN + (int)half * BN_CTA;
             for (int kc = 0; kc < num_k; ++kc) {
-                if (!mbar_wait_bounded_warp(smem_addr(&sh->empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
+                const bool early = tile == cluster && kc < pre;  // weights already in flight
+                if (!early && !mbar_wait_bounded_warp(smem_addr(&sh->empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
                 const uint32_t st = base + stage * STAGE_BYTES;
                 const uint32_t bar = leader_full0 + stage * 8;
                 if (elect_one()) {
-                    if (half == 0) mbar_arrive_expect_tx(smem_addr(&sh->full[stage]), 2 * (A_BYTES + B_BYTES));
+                    if (half == 0 && !early) mbar_arrive_expect_tx(smem_addr(&sh->full[stage]), 2 * (A_BYTES + B_BYTES));
                     if (CL == 2) {
                         tma_load_2d_pair(st, &tmap_a, kc * BKE, m_rows, bar);
                     } else {
                         tma_load_2d_pair_multicast(st + pr * (A_BYTES / 2), &tmap_a, kc * BKE,
                                                    m_rows + (int)pr * (BM / 2), bar, a_mask);
                     }
-                    tma_load_2d_pair(st + A_BYTES, &tmap_b, kc * BKE, n_rows, bar);
+                    if (!early) tma_load_2d_pair(st + A_BYTES, &tmap_b, kc * BKE, n_rows, bar);
                 }
                 __syncwarp();
                 if (++stage == STAGES) { stage = 0; phase ^= 1u; }
