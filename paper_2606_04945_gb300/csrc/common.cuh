@@ -151,6 +151,20 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
     }
 }
 
+// Same, polling every `sleep_ns` nanoseconds: for waits that are not on a
+// critical path, so the spinning warp leaves issue slots to its neighbours.
+__device__ __forceinline__ bool mbar_wait_bounded_sleepy(uint32_t bar, uint32_t parity, volatile int* abort,
+                                                         unsigned sleep_ns) {
+    const unsigned long long t0 = globaltimer_ns();
+    #pragma unroll 1
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort) return false;
+        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) return false;
+        __nanosleep(sleep_ns);
+    }
+}
+
 // Whole-warp form: every lane waits; the result is the same in every lane.
 __device__ __forceinline__ bool mbar_wait_bounded_warp(uint32_t bar, uint32_t parity, volatile int* abort) {
     const bool ok = mbar_wait_bounded(bar, parity, abort);

@@ -1021,7 +1021,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 reinterpret_cast<float4*>(epi_b)[lane] = bb;
                 __syncwarp();
             }
-            if (!mbar_wait_bounded(smem_addr(&sh->tmem_full[acc]), acc_phase, abort)) { ok = false; break; }
+            // a whole tile of MMAs away: poll gently, the MMA warp shares the scheduler
+            if (!mbar_wait_bounded_sleepy(smem_addr(&sh->tmem_full[acc]), acc_phase, abort, 256)) { ok = false; break; }
             tc_fence_after();
             const uint32_t t_row = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
             #pragma unroll 1
