@@ -285,7 +285,7 @@ def run_ours(args):
     t_quant_x = time_kernel(lambda: abi.sgat_quantize_act(step.X, step.mask, q.a_m, q.a_u, q.hb, q.d_sh, q.d_m,
                                                           q.d_u, Xq, s_a, Xe=Xe), flush, reps, torch)
     t_gemm_qkv = time_kernel(lambda: abi.w4a4_gemm(None, s_a, q.Wq, q.s_w, step.Y_qkv, Xe=Xe, We=q.We), flush, reps, torch)
-    t_tac = time_kernel(lambda: abi.tac_apply(step.Z, o.tac_M, o.tac_d, o.tac_g, zt), flush, reps, torch)
+    t_tac = time_kernel(lambda: abi.tac_apply(step.Z, o.tac_M, o.tac_d, o.tac_g, zt, Mp=o.tac_Mp), flush, reps, torch)
     t_quant_z = time_kernel(lambda: abi.sgat_quantize_act(zt, step.mask, o.a_m, o.a_u, o.hb, o.d_sh, o.d_m,
                                                           o.d_u, Xq, s_a, Xe=Xe), flush, reps, torch)
     t_gemm_o = time_kernel(lambda: abi.w4a4_gemm(None, s_a, o.Wq, o.s_w, step.Y_o, Xe=Xe, We=o.We), flush, reps, torch)
@@ -298,7 +298,7 @@ def run_ours(args):
     Zr = [step.Z.clone() for _ in range(R)]
     Zf = [torch.empty(L, K, dtype=torch.float32, device="cuda") for _ in range(R // 2)]   # 10 x 16 MB
     for i in range(R // 2):
-        abi.tac_apply(Zr[i], o.tac_M, o.tac_d, o.tac_g, Zf[i])
+        abi.tac_apply(Zr[i], o.tac_M, o.tac_d, o.tac_g, Zf[i], Mp=o.tac_Mp)
     Wr_q = [q.We] + [q.We.clone() for _ in range(2)]               # 3 x 50 MB
     Wr_o = [o.We] + [o.We.clone() for _ in range(7)]               # 8 x 17 MB
     Xer = [Xe] + [Xe.clone() for _ in range(2)]
@@ -306,8 +306,8 @@ def run_ours(args):
                                                                  q.d_u, Xq, s_a, Xe=Xe) for i in range(R)], flush, torch)
     s_gemm_qkv = time_stream([lambda i=i: abi.w4a4_gemm(None, s_a, q.Wq, q.s_w, step.Y_qkv, Xe=Xer[i], We=Wr_q[i])
                               for i in range(3)], flush, torch, rounds=4)
-    s_tac = time_stream([lambda i=i: abi.tac_apply(Zr[i], o.tac_M, o.tac_d, o.tac_g, zt) for i in range(R)],
-                        flush, torch)
+    s_tac = time_stream([lambda i=i: abi.tac_apply(Zr[i], o.tac_M, o.tac_d, o.tac_g, zt, Mp=o.tac_Mp)
+                         for i in range(R)], flush, torch)
     s_quant_z = time_stream([lambda i=i: abi.sgat_quantize_act(Zf[i], step.mask, o.a_m, o.a_u, o.hb, o.d_sh, o.d_m,
                                                                  o.d_u, Xq, s_a, Xe=Xe) for i in range(R // 2)],
                             flush, torch, rounds=4)
@@ -433,7 +433,7 @@ def run_ours(args):
     hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
     quant_x_bytes = L * K * 2 + L * K // 2 + L * K + 4 * L     # X in; packed + E4M3 codes, scales out
     quant_z_bytes = L * K * 4 + L * K // 2 + L * K + 4 * L
-    tac_bytes = L * K * 2 + L * K * 4 + K * o.tac_g * 4 + K * 4
+    tac_bytes = L * K * 2 + L * K * 4 + K * o.tac_g * 4 + K * 4      # Z in, float32 out, M (prepared: 4 C g B), d
     traffic = profiled_traffic()
     wbytes = lambda lin: lin.N * K if lin.We is not None else lin.N * K // 2
     gemm_bytes = [L * K + wbytes(q) + 2 * L * q.N + 4 * (L + q.N),    # E4M3 codes, weights, fp16 out

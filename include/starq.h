@@ -167,6 +167,23 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
 int fp16_gemm_ref(const void* A, const void* B, int dtype, int M, int N, int K, void* C, void* stream);
 
 /*
+ * tac_prepare -- the TAC matrices in the form the tensor-core TAC reads
+ * (the paper has no counterpart: a storage form, like w4_unpack_e4m3).
+ * Every block M_b is split into two 16-bit matrices of Z's type,
+ * hi = rn(M_b) and lo = rn(M_b - hi) (Z hi^T + Z lo^T reproduces Z M_b^T
+ * with float32 accumulation to about 2^-22 relative), laid out K-major with
+ * the 128-byte swizzle. Run once per set of TAC parameters; pass the result
+ * as Mp to tac_apply / sgat_linear, which then copy it instead of splitting
+ * M in every CTA.
+ *
+ *   M  [C/g][g][g] float32, 16-byte aligned.
+ *   Mp out, 4*C*g bytes, 16-byte aligned, caller-owned.
+ *   z_dtype: F16 or BF16, the type of the Z it will be applied to.
+ * Shapes: g in {64, 128}, C % g == 0.
+ */
+int tac_prepare(const float* M, int C, int g, int z_dtype, void* Mp, void* stream);
+
+/*
  * tac_apply -- block-wise affine compensation of the quantised attention
  * output before the output projection (Sec. 3.3 Eq. 17; App. C row-major
  * form Z_b M_b^T + 1 d_b^T).
@@ -176,12 +193,15 @@ int fp16_gemm_ref(const void* A, const void* B, int dtype, int M, int N, int K, 
  *   Z   [L][C] element type z_dtype (F16, BF16 or F32), 16-byte aligned.
  *   M   [C/g][g][g] float32 (row r = output channel r of block b); d [C/g][g]
  *       float32 (NULL = zeros). Both 16-byte aligned.
+ *   Mp  tac_prepare(M, C, g, z_dtype) output or NULL; only with 16-bit Z and
+ *       g = 64 or 128 (the tensor-core path), which otherwise splits M in
+ *       every CTA.
  *   out [L][C] element type out_dtype (F16, BF16 or F32), 16-byte aligned;
  *       must not overlap Z.
  * Shapes: L >= 0, g in {4, 8, 16, 32, 64, 128}, C % g == 0, C % 8 == 0.
  */
 int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d,
-              void* out, int out_dtype, void* stream);
+              const void* Mp, void* out, int out_dtype, void* stream);
 
 /*
  * sgat_linear -- the fused SGAT W4A4 linear of one quantised layer: optional
@@ -190,10 +210,11 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  * epilogue (Eq. 13). Equivalent to tac_apply (to float32) ->
  * sgat_quantize_act -> w4a4_gemm, with the intermediates in `workspace`.
  *
- *   tac_M, tac_d, tac_g: TAC parameters as for tac_apply, or tac_M = NULL
- *   for no TAC. Wq/s_w come from sgat_prepare_weight, We (optional, NULL =
- *   convert Wq on the fly) from w4_unpack_e4m3. Other arguments as in the
- *   calls above. K % 128 == 0.
+ *   tac_M, tac_d, tac_g, tac_Mp: TAC parameters as for tac_apply (tac_Mp =
+ *   tac_prepare output or NULL), or tac_M = NULL for no TAC. Wq/s_w come
+ *   from sgat_prepare_weight, We (optional, NULL = convert Wq on the fly)
+ *   from w4_unpack_e4m3. Other arguments as in the calls above.
+ *   K % 128 == 0.
  *   workspace: device buffer of at least sgat_linear_workspace_size(L, K,
  *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller. On return it
  *   holds the intermediates, laid out as [packed codes Xq: L*K/2 bytes,
@@ -203,7 +224,7 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
 size_t sgat_linear_workspace_size(int L, int K, int with_tac);
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                const float* tac_M, const float* tac_d, int tac_g,
+                const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
                 const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N,
                 int bits, void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
@@ -239,7 +260,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
 #define STARQ_NOALLOC_SCRATCH_BYTES (32u << 20)
 int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                         const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                        const float* tac_M, const float* tac_d, int tac_g,
+                        const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
                         const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias,
                         int N, int bits, void* Y, int y_dtype, void* stream);
 

@@ -18,7 +18,7 @@ OK, ERR_ARG, ERR_SHAPE, ERR_ALIGN, ERR_BITS, ERR_CUDA, ERR_TIMEOUT = 0, -1, -2, 
 
 EXPORTED = (
     "starq_version", "starq_last_error", "starq_check_status",
-    "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "fp16_gemm_ref", "tac_apply",
+    "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "fp16_gemm_ref", "tac_prepare", "tac_apply",
     "sgat_linear_workspace_size", "sgat_linear",
 )
 
@@ -42,14 +42,15 @@ def _load():
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
-    lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, i, vp]
+    lib.tac_prepare.argtypes = [f_p, i, i, i, vp, vp]
+    lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, vp, i, vp]
     lib.fp16_gemm_ref.argtypes = [vp, vp, i, i, i, i, vp, vp]
     lib.sgat_linear_workspace_size.argtypes = [i, i, i]
     lib.sgat_linear_workspace_size.restype = ctypes.c_size_t
-    lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
+    lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
                                 u8p, u8p, f_p, f_p, i, i, vp, i, vp, ctypes.c_size_t, vp]
     if hasattr(lib, "sgat_linear_noalloc"):
-        lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i,
+        lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
                                             u8p, u8p, f_p, f_p, i, i, vp, i, vp]
     return lib
 
@@ -134,10 +135,23 @@ def fp16_gemm_ref(A, B, C, stream=None):
     _check(lib.fp16_gemm_ref(_p(A), _p(B), dtype_code(A), M, N, K, _p(C), _stream(stream)))
 
 
-def tac_apply(Z, M, d, g, out, stream=None):
-    _contig(Z, M, d, out)
+def tac_prepare(M, g, z_dtype, Mp, stream=None):
+    """M [C/g][g][g] float32 -> the tensor-core form (4 C g bytes) for Z of
+    type z_dtype (torch.float16 or torch.bfloat16)."""
+    _contig(M, Mp)
+    C = M.shape[0] * g
+    code = {torch.float16: F16, torch.bfloat16: BF16}[z_dtype]
+    _check(lib.tac_prepare(_p(M), C, g, code, _p(Mp), _stream(stream)))
+
+
+def tac_prepared_bytes(C, g):
+    return 4 * C * g
+
+
+def tac_apply(Z, M, d, g, out, Mp=None, stream=None):
+    _contig(Z, M, d, out, Mp)
     L, C = Z.shape
-    _check(lib.tac_apply(_p(Z), dtype_code(Z), L, C, g, _p(M), _p(d), _p(out), dtype_code(out),
+    _check(lib.tac_apply(_p(Z), dtype_code(Z), L, C, g, _p(M), _p(d), _p(Mp), _p(out), dtype_code(out),
                          _stream(stream)))
 
 
@@ -146,12 +160,12 @@ def sgat_linear_workspace_size(L, K, with_tac):
 
 
 def sgat_linear(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, workspace, bias=None,
-                tac_M=None, tac_d=None, tac_g=0, bits=4, We=None, stream=None):
-    _contig(X, mask, a_m, a_u, Wq, We, s_w, Y, workspace, bias, tac_M, tac_d)
+                tac_M=None, tac_d=None, tac_g=0, bits=4, We=None, tac_Mp=None, stream=None):
+    _contig(X, mask, a_m, a_u, Wq, We, s_w, Y, workspace, bias, tac_M, tac_d, tac_Mp)
     L, K = X.shape
     N = _weight_shape(Wq, We)[0]
     _check(lib.sgat_linear(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh, d_m,
-                           d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(We), _p(s_w), _p(bias), N, bits,
+                           d_u, _p(tac_M), _p(tac_d), tac_g, _p(tac_Mp), _p(Wq), _p(We), _p(s_w), _p(bias), N, bits,
                            _p(Y), dtype_code(Y), _p(workspace), workspace.numel() * workspace.element_size(),
                            _stream(stream)))
 
@@ -160,12 +174,12 @@ NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
 def sgat_linear_noalloc(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, bias=None,
-                        tac_M=None, tac_d=None, tac_g=0, bits=4, We=None, stream=None):
+                        tac_M=None, tac_d=None, tac_g=0, bits=4, We=None, tac_Mp=None, stream=None):
     """sgat_linear without a workspace: the library's fixed device scratch
     array holds the intermediates (see include/starq.h)."""
-    _contig(X, mask, a_m, a_u, Wq, We, s_w, Y, bias, tac_M, tac_d)
+    _contig(X, mask, a_m, a_u, Wq, We, s_w, Y, bias, tac_M, tac_d, tac_Mp)
     L, K = X.shape
     N = _weight_shape(Wq, We)[0]
     _check(lib.sgat_linear_noalloc(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh,
-                                   d_m, d_u, _p(tac_M), _p(tac_d), tac_g, _p(Wq), _p(We), _p(s_w), _p(bias), N,
+                                   d_m, d_u, _p(tac_M), _p(tac_d), tac_g, _p(tac_Mp), _p(Wq), _p(We), _p(s_w), _p(bias), N,
                                    bits, _p(Y), dtype_code(Y), _stream(stream)))

@@ -211,17 +211,41 @@ int fp16_gemm_ref(const void* A, const void* B, int dtype, int M, int N, int K, 
     return STARQ_OK;
 }
 
-int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d,
+int tac_prepare(const float* M, int C, int g, int z_dtype, void* Mp, void* stream) {
+    if (C > 0 && (!M || !Mp)) return fail(STARQ_ERR_ARG, "tac_prepare: NULL M or Mp");
+    if (z_dtype != STARQ_F16 && z_dtype != STARQ_BF16)
+        return fail(STARQ_ERR_ARG, "tac_prepare: z_dtype must be F16 or BF16 (the tensor-core path)");
+    if (g != 64 && g != 128) return fail(STARQ_ERR_SHAPE, "tac_prepare: g=%d: the tensor-core path takes 64 or 128", g);
+    if (C < 0 || C % g != 0) return fail(STARQ_ERR_SHAPE, "tac_prepare: C=%d must be a multiple of g=%d", C, g);
+    if (C == 0) return STARQ_OK;
+    if (!aligned(M, 16) || !aligned(Mp, 16)) return fail(STARQ_ERR_ALIGN, "tac_prepare: M, Mp alignment");
+    cudaError_t e = launch_tac_prepare(M, C, g, z_dtype, Mp, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "tac_prepare launch");
+    return STARQ_OK;
+}
+
+namespace {
+int check_tac_prepared(const void* Mp, int z_dtype, int g) {
+    if (!Mp) return STARQ_OK;
+    if ((z_dtype != STARQ_F16 && z_dtype != STARQ_BF16) || (g != 64 && g != 128))
+        return fail(STARQ_ERR_ARG, "prepared TAC matrix: 16-bit Z and g = 64 or 128 only");
+    if (!aligned(Mp, 16)) return fail(STARQ_ERR_ALIGN, "prepared TAC matrix must be 16-byte aligned");
+    return STARQ_OK;
+}
+}  // namespace
+
+int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d, const void* Mp,
               void* out, int out_dtype, void* stream) {
     if (L > 0 && (!Z || !out)) return fail(STARQ_ERR_ARG, "tac_apply: NULL Z or out");
     if (!dtype_ok(z_dtype) || !dtype_ok(out_dtype)) return fail(STARQ_ERR_ARG, "tac_apply: unknown dtype");
     int rc = check_tac(L, C, g, M, d);
     if (rc) return rc;
+    if ((rc = check_tac_prepared(Mp, z_dtype, g))) return rc;
     if (L == 0) return STARQ_OK;
     if (!aligned(Z, 16) || !aligned(out, 16)) return fail(STARQ_ERR_ALIGN, "tac_apply: Z, out alignment");
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
-    TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype, st};
+    TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype, st, Mp};
     cudaError_t e = launch_tac(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "tac_apply launch");
     return STARQ_OK;
@@ -236,7 +260,7 @@ size_t sgat_linear_workspace_size(int L, int K, int with_tac) {
 
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                const float* tac_M, const float* tac_d, int tac_g,
+                const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
                 const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
                 void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
     if ((!Wq && !We) || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear: NULL Wq/We or s_w");
@@ -247,6 +271,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
     if (rc) return rc;
     if (tac_M && (rc = check_tac(L, K, tac_g, tac_M, tac_d))) return rc;
+    if (tac_M && (rc = check_tac_prepared(tac_Mp, x_dtype, tac_g))) return rc;
     if (L == 0) return STARQ_OK;
     const size_t need = sgat_linear_workspace_size(L, K, tac_M != nullptr);
     if (workspace_bytes < need)
@@ -266,7 +291,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     int qin_dtype = x_dtype;
     cudaError_t e;
     if (tac_M) {
-        TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, STARQ_F32, st};
+        TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, STARQ_F32, st, tac_Mp};
         if ((e = launch_tac(t, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: tac launch");
         qin = zt;
         qin_dtype = STARQ_F32;

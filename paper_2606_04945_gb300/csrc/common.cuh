@@ -70,8 +70,13 @@ struct TacArgs {
     const void* Z; int z_dtype; int L; int C; int g;
     const float* M; const float* d; void* out; int out_dtype;
     unsigned* status = nullptr;   // device status word (tensor-core path)
+    const void* Mp = nullptr;     // optional tac_prepare output (tensor-core path)
 };
 cudaError_t launch_tac(const TacArgs& a, cudaStream_t stream);
+// M [C/g][g][g] float32 -> its 16-bit halves (hi = rn(M), lo = rn(M - hi), of
+// type z_dtype) in the tensor-core operand layout: per block b, 2 g g 16-bit
+// values (hi then lo, each K-major with the 128-byte swizzle).
+cudaError_t launch_tac_prepare(const float* M, int C, int g, int z_dtype, void* Mp, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached per device)
 int report_error(int code, const char* msg);  // record msg for starq_last_error(), return code

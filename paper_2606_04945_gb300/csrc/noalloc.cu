@@ -58,7 +58,7 @@ void* scratch_address(int* rc, cudaError_t* err) {
 
 extern "C" int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                                    const float* a_m, const float* a_u, int hb, int d_sh, int d_m,
-                                   int d_u, const float* tac_M, const float* tac_d, int tac_g,
+                                   int d_u, const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
                                    const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N,
                                    int bits, void* Y, int y_dtype, void* stream) {
     const size_t need = sgat_linear_workspace_size(L, K, tac_M != nullptr);
@@ -78,7 +78,7 @@ extern "C" int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, con
                  cudaGetErrorString(err));
         return starq::report_error(rc, msg);
     }
-    return sgat_linear(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g,
+    return sgat_linear(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g, tac_Mp,
                        Wq, We, s_w, bias, N, bits, Y, y_dtype, scratch,
                        (size_t)STARQ_NOALLOC_SCRATCH_BYTES, stream);
 }

@@ -184,11 +184,77 @@ template <> struct TacStore<float> {
 template <> struct TacStore<__half> { static constexpr bool TMA = false; };
 template <> struct TacStore<__nv_bfloat16> { static constexpr bool TMA = false; };
 
+// M_b (float32 [g][g]) -> its two 16-bit halves, K-major (row r = output
+// channel, 8 inputs per 16-byte chunk, 128-byte swizzle) at shared
+// addresses sMh / sMl; every load of the thread is issued before the first
+// convert.
+template <int G, typename TIn>
+__device__ __forceinline__ void tac_split_block(const float* Mb, uint32_t sMh, uint32_t sMl) {
+    constexpr int NIT = G * G / 8 / TC_THREADS;
+    float4 w0[NIT], w1[NIT];
+    #pragma unroll
+    for (int it = 0; it < NIT; ++it) {
+        const int idx = threadIdx.x + it * TC_THREADS;
+        const int r = idx / (G / 8), jc = idx % (G / 8);
+        w0[it] = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc));
+        w1[it] = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc + 4));
+    }
+    #pragma unroll
+    for (int it = 0; it < NIT; ++it) {
+        const int idx = threadIdx.x + it * TC_THREADS;
+        const int r = idx / (G / 8), jc = idx % (G / 8);      // inputs j = 8 jc .. 8 jc + 7
+        const float mv[8] = {w0[it].x, w0[it].y, w0[it].z, w0[it].w, w1[it].x, w1[it].y, w1[it].z, w1[it].w};
+        uint32_t hi[4], lo[4];
+        #pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            uint16_t h0, l0, h1, l1;
+            Split16<TIn>::split(mv[2 * e], h0, l0);
+            Split16<TIn>::split(mv[2 * e + 1], h1, l1);
+            hi[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+            lo[e] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+        }
+        const uint32_t off = (jc / 8) * (G * 128) + sw128_offset(r, jc % 8);
+        st_shared_v4(sMh + off, hi[0], hi[1], hi[2], hi[3]);
+        st_shared_v4(sMl + off, lo[0], lo[1], lo[2], lo[3]);
+    }
+}
+
+// The same halves written once to global memory, byte for byte the shared
+// image tac_tc_kernel builds (hi then lo per block), for a bulk copy.
+template <int G, typename TIn>
+__global__ void __launch_bounds__(256)
+tac_prepare_kernel(const float* __restrict__ M, uint8_t* __restrict__ Mp) {
+    constexpr int M_BYTES = G * G * 2;
+    const int b = blockIdx.x;
+    const float* Mb = M + (size_t)b * G * G;
+    uint8_t* hi = Mp + (size_t)b * 2 * M_BYTES;
+    uint8_t* lo = hi + M_BYTES;
+    for (int idx = threadIdx.x; idx < G * G / 8; idx += blockDim.x) {
+        const int r = idx / (G / 8), jc = idx % (G / 8);
+        const float4 w0 = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc));
+        const float4 w1 = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc + 4));
+        const float mv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+        uint32_t h[4], l[4];
+        #pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            uint16_t h0, l0, h1, l1;
+            Split16<TIn>::split(mv[2 * e], h0, l0);
+            Split16<TIn>::split(mv[2 * e + 1], h1, l1);
+            h[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+            l[e] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+        }
+        const uint32_t off = (jc / 8) * (G * 128) + sw128_offset(r, jc % 8);
+        *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
+        *reinterpret_cast<uint4*>(lo + off) = make_uint4(l[0], l[1], l[2], l[3]);
+    }
+}
+
 // Tensor-core TAC: one CTA per (block b, tile of 128 tokens), 8 warps.
 //   * the tile Z[rows][b g .. b g + g) arrives by TMA (128-byte swizzle);
 //   * meanwhile all threads read M_b (float32) with coalesced 32-byte loads
 //     and write its two 16-bit halves hi = rn(M), lo = rn(M - hi) (the
-//     input's type) into the K-major swizzled operand layout;
+//     input's type) into the K-major swizzled operand layout -- or, with a
+//     prepared M (tac_prepare), one bulk copy brings both halves;
 //   * one thread issues g/16 pairs of kind::f16 MMAs (Z hi^T and Z lo^T,
 //     float32 accumulation in TMEM: relative error about 2^-22);
 //   * each warp reads 32 tokens x g/2 channels of the accumulator, adds d,
@@ -220,6 +286,7 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
         abort_flag = 0;
         mbar_fence_init();
     }
+    const bool prepared = a.Mp != nullptr;
     if (warp == 0) {
         tmem_alloc(smem_addr(&tmem_slot), P::TMEM_COLS);
         tmem_relinquish();
@@ -229,40 +296,17 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
     grid_dependency_wait();
     grid_launch_dependents();
     if (threadIdx.x == 0) {
-        mbar_arrive_expect_tx(smem_addr(&zfull), P::Z_BYTES);
+        // Z tile (and, when prepared, both 16-bit halves of M_b) on one barrier
+        mbar_arrive_expect_tx(smem_addr(&zfull), P::Z_BYTES + (prepared ? 2 * P::M_BYTES : 0));
         for (int at = 0; at < P::ATOMS; ++at)
             tma_load_2d(sZ + at * (TC_TM * 128), &tmap_z, b * G + at * 64, row0, smem_addr(&zfull));
+        if (prepared)
+            bulk_load(sMh, static_cast<const uint8_t*>(a.Mp) + (size_t)b * 2 * P::M_BYTES, 2 * P::M_BYTES,
+                      smem_addr(&zfull));
     }
-    // M_b -> hi / lo, K-major (row r = output channel, 8 inputs per 16-byte
-    // chunk); every load of the thread is issued before the first convert
-    const float* Mb = a.M + (size_t)b * G * G;
-    constexpr int NIT = G * G / 8 / TC_THREADS;
-    float4 w0[NIT], w1[NIT];
-    #pragma unroll
-    for (int it = 0; it < NIT; ++it) {
-        const int idx = threadIdx.x + it * TC_THREADS;
-        const int r = idx / (G / 8), jc = idx % (G / 8);
-        w0[it] = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc));
-        w1[it] = __ldg(reinterpret_cast<const float4*>(Mb + (size_t)r * G + 8 * jc + 4));
-    }
-    #pragma unroll
-    for (int it = 0; it < NIT; ++it) {
-        const int idx = threadIdx.x + it * TC_THREADS;
-        const int r = idx / (G / 8), jc = idx % (G / 8);      // inputs j = 8 jc .. 8 jc + 7
-        const float mv[8] = {w0[it].x, w0[it].y, w0[it].z, w0[it].w, w1[it].x, w1[it].y, w1[it].z, w1[it].w};
-        uint32_t hi[4], lo[4];
-        #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            uint16_t h0, l0, h1, l1;
-            Split16<TIn>::split(mv[2 * e], h0, l0);
-            Split16<TIn>::split(mv[2 * e + 1], h1, l1);
-            hi[e] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-            lo[e] = (uint32_t)l0 | ((uint32_t)l1 << 16);
-        }
-        const uint32_t off = (jc / 8) * (G * 128) + sw128_offset(r, jc % 8);
-        st_shared_v4(sMh + off, hi[0], hi[1], hi[2], hi[3]);
-        st_shared_v4(sMl + off, lo[0], lo[1], lo[2], lo[3]);
-    }
+    if (!prepared)
+        tac_split_block<G, TIn>(a.M + (size_t)b * G * G, sMh, sMl);
+
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
@@ -451,6 +495,20 @@ cudaError_t launch_in(const TacArgs& a, cudaStream_t stream) {
 }
 
 }  // namespace
+
+cudaError_t launch_tac_prepare(const float* M, int C, int g, int z_dtype, void* Mp, cudaStream_t stream) {
+    if (C == 0) return cudaSuccess;
+    uint8_t* out = static_cast<uint8_t*>(Mp);
+    dim3 grid(C / g);
+    if (z_dtype == STARQ_F16) {
+        if (g == 64) tac_prepare_kernel<64, __half><<<grid, 256, 0, stream>>>(M, out);
+        else tac_prepare_kernel<128, __half><<<grid, 256, 0, stream>>>(M, out);
+    } else {
+        if (g == 64) tac_prepare_kernel<64, __nv_bfloat16><<<grid, 256, 0, stream>>>(M, out);
+        else tac_prepare_kernel<128, __nv_bfloat16><<<grid, 256, 0, stream>>>(M, out);
+    }
+    return cudaGetLastError();
+}
 
 cudaError_t launch_tac(const TacArgs& a, cudaStream_t stream) {
     if (a.L == 0) return cudaSuccess;

@@ -40,10 +40,16 @@ class SgatLinear:
         self.a_u = _dev(xf.a_u, device=device)
         self.bias = _dev(case.bias, device=device) if case.bias is not None else None
         self.tac = case.tac
+        self.tac_Mp = None
         if case.tac is not None:
             self.tac_M = _dev(case.tac.M, device=device)
             self.tac_d = _dev(case.tac.d, device=device)
             self.tac_g = case.tac.g
+            if self.dtype != torch.float32 and self.tac_g in (64, 128):
+                # TAC matrices in the tensor-core form, once
+                self.tac_Mp = torch.empty(abi.tac_prepared_bytes(self.K, self.tac_g), dtype=torch.uint8,
+                                          device=device)
+                abi.tac_prepare(self.tac_M, self.tac_g, self.dtype, self.tac_Mp)
         else:
             self.tac_M = self.tac_d = None
             self.tac_g = 0
@@ -62,7 +68,7 @@ class SgatLinear:
     def run(self, X, mask, Y, stream=None):
         abi.sgat_linear(X, mask, self.a_m, self.a_u, self.hb, self.d_sh, self.d_m, self.d_u,
                         self.Wq, self.s_w, Y, self.workspace, bias=self.bias, tac_M=self.tac_M,
-                        tac_d=self.tac_d, tac_g=self.tac_g, We=self.We, stream=stream)
+                        tac_d=self.tac_d, tac_g=self.tac_g, We=self.We, tac_Mp=self.tac_Mp, stream=stream)
 
     def int_ops(self, L=None):
         return 2 * (L or self.L) * self.N * self.K

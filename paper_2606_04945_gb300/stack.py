@@ -77,16 +77,18 @@ class QLinear:
         self.L = L
         self.tac = tac
         self.sgat = None
-        self.tac_M = self.tac_d = None
+        self.tac_M = self.tac_d = self.tac_Mp = None
         if tac is not None:
             dev = W16.device
             self.tac_M = torch.from_numpy(tac.M).to(dev)
             self.tac_d = torch.from_numpy(tac.d).to(dev)
+            self.tac_Mp = torch.empty(abi.tac_prepared_bytes(self.K, tac.g), dtype=torch.uint8, device=dev)
+            abi.tac_prepare(self.tac_M, tac.g, W16.dtype, self.tac_Mp)
 
     def tac_out(self, X):
         """TAC of the linear's input (float32), as sgat_linear applies it."""
         Z = torch.empty(X.shape, dtype=torch.float32, device=X.device)
-        abi.tac_apply(X, self.tac_M, self.tac_d, self.tac.g, Z)
+        abi.tac_apply(X, self.tac_M, self.tac_d, self.tac.g, Z, Mp=self.tac_Mp)
         return Z
 
     def calibrate(self, X, mask):
@@ -107,7 +109,7 @@ class QLinear:
         xf = self.sgat
         abi.sgat_linear(X, mask, self.a_m, self.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, self.Wq, self.s_w, Y,
                         self.workspace, tac_M=self.tac_M, tac_d=self.tac_d,
-                        tac_g=self.tac.g if self.tac is not None else 0, We=self.We)
+                        tac_g=self.tac.g if self.tac is not None else 0, We=self.We, tac_Mp=self.tac_Mp)
 
     def fp16(self, X, Y):
         abi.fp16_gemm_ref(X, self.W16, Y)

@@ -109,11 +109,27 @@ def test_fp16_gemm_alignment(lib):
 
 @pytest.mark.parametrize("g,C,code", [(12, 96, -2), (16, 100, -2), (256, 4096, -2)])
 def test_tac_validation(lib, g, C, code):
-    assert lib.lib.tac_apply(P, 0, 4, C, g, P, P, P, 0, None) == code
+    assert lib.lib.tac_apply(P, 0, 4, C, g, P, P, None, P, 0, None) == code
 
 
 def test_tac_null_matrix(lib):
-    assert lib.lib.tac_apply(P, 0, 4, 64, 16, None, P, P, 0, None) == -1
+    assert lib.lib.tac_apply(P, 0, 4, 64, 16, None, P, None, P, 0, None) == -1
+
+
+def test_tac_prepared_only_on_the_tensor_core_path(lib):
+    assert lib.lib.tac_apply(P, 2, 4, 256, 128, P, P, P, P, 2, None) == -1      # float32 Z
+    assert lib.lib.tac_apply(P, 0, 4, 256, 32, P, P, P, P, 2, None) == -1      # g = 32
+    assert lib.lib.tac_apply(P, 0, 4, 256, 128, P, P, ctypes.c_void_p(4104), P, 2, None) == -3
+
+
+@pytest.mark.parametrize("C,g,dt,code", [(256, 32, 0, -2), (200, 64, 0, -2), (256, 128, 2, -1), (0, 128, 1, 0)])
+def test_tac_prepare_validation(lib, C, g, dt, code):
+    assert lib.lib.tac_prepare(P, C, g, dt, P, None) == code
+
+
+def test_tac_prepare_null_and_alignment(lib):
+    assert lib.lib.tac_prepare(None, 256, 128, 0, P, None) == -1
+    assert lib.lib.tac_prepare(P, 256, 128, 0, ctypes.c_void_p(4100), None) == -3
 
 
 def test_linear_workspace_and_validation(lib):
@@ -121,10 +137,10 @@ def test_linear_workspace_and_validation(lib):
     assert n == 1024 * 2048 + 4096 + 1024 * 4096
     assert lib.sgat_linear_workspace_size(1024, 4096, True) == n + 1024 * 4096 * 4
     # workspace too small
-    rc = lib.lib.sgat_linear(P, 0, 1024, 4096, None, None, None, 4096, 4096, 0, 0, None, None, 0,
+    rc = lib.lib.sgat_linear(P, 0, 1024, 4096, None, None, None, 4096, 4096, 0, 0, None, None, 0, None,
                              P, None, P, None, 256, 4, P, 0, P, 16, None)
     assert rc == -2 and b"workspace" in lib.lib.starq_last_error()
     # TAC block that does not divide K
-    rc = lib.lib.sgat_linear(P, 0, 16, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 48,
+    rc = lib.lib.sgat_linear(P, 0, 16, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 48, None,
                              P, None, P, None, 256, 4, P, 0, P, 1 << 30, None)
     assert rc == -2

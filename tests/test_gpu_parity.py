@@ -264,10 +264,19 @@ def test_tac_apply(abi, g, L, C, zin, zout):
     Z = Z.astype(np.float16).astype(np.float32) if zin == "f16" else (inputs.round_to_bf16(Z) if zin == "bf16" else Z)
     tp = inputs.make_tac(rng, C, g, noise=0.05)
     out = torch.empty(L, C, dtype=H.torch_dtype(zout), device="cuda")
-    abi.tac_apply(H.dev(Z, H.torch_dtype(zin)), H.dev(tp.M), H.dev(tp.d), g, out)
+    Zd, Md = H.dev(Z, H.torch_dtype(zin)), H.dev(tp.M)
+    abi.tac_apply(Zd, Md, H.dev(tp.d), g, out)
     abi.check_status()
     ref = otac.tac_apply(Z, tp.M, tp.d, g)
     H.assert_tac_close(H.host(out), ref, zout)
+    if zin != "f32" and g in (64, 128):
+        # the prepared matrices (tac_prepare) give the same shared image, hence the same bits
+        Mp = torch.empty(abi.tac_prepared_bytes(C, g), dtype=torch.uint8, device="cuda")
+        abi.tac_prepare(Md, g, H.torch_dtype(zin), Mp)
+        out2 = torch.empty_like(out)
+        abi.tac_apply(Zd, Md, H.dev(tp.d), g, out2, Mp=Mp)
+        abi.check_status()
+        assert torch.equal(out2, out), "prepared TAC differs"
 
 
 def _oracle_linear_from_codes(qa, s_a, qw, s_w, bias):
@@ -295,6 +304,10 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None, weights="e4m3"):
     kw = {}
     if with_tac:
         kw = dict(tac_M=H.dev(case.tac.M), tac_d=H.dev(case.tac.d), tac_g=case.tac.g)
+        if weights == "e4m3" and case.dtype != "f32" and case.tac.g in (64, 128):
+            # the main path also takes the prepared TAC matrices
+            kw["tac_Mp"] = torch.empty(abi.tac_prepared_bytes(K, case.tac.g), dtype=torch.uint8, device="cuda")
+            abi.tac_prepare(kw["tac_M"], case.tac.g, dt, kw["tac_Mp"])
     bias = H.dev(case.bias) if case.bias is not None else None
     abi.sgat_linear(H.dev(case.X, dt), H.dev(case.mask), H.dev(xf.a_m), H.dev(xf.a_u), xf.hb, xf.d_sh,
                     xf.d_m, xf.d_u, Wq, s_w, Y, ws, bias=bias, We=We, **kw)

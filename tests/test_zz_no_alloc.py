@@ -80,6 +80,6 @@ def test_noalloc_symbol_and_limit_declared():
     assert abi.NOALLOC_SCRATCH_BYTES == 32 << 20
     # the size check runs before any CUDA call
     P = ctypes.c_void_p(4096)
-    rc = abi.lib.sgat_linear_noalloc(P, 0, 4096, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 128,
+    rc = abi.lib.sgat_linear_noalloc(P, 0, 4096, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 128, None,
                                      P, None, P, None, 256, 4, P, 0, None)
     assert rc == abi.ERR_SHAPE
