@@ -219,7 +219,9 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller. On return it
  *   holds the intermediates, laid out as [packed codes Xq: L*K/2 bytes,
  *   padded to 256][s_a: 4*L bytes, padded to 256][E4M3 codes Xe: L*K bytes,
- *   padded to 256][TAC output: float32 L*K, only with TAC].
+ *   padded to 256][TAC output: L*K values of x_dtype (room for float32), only
+ *   with TAC]. The TAC output is rounded to x_dtype once, as the unquantised
+ *   model stores attention outputs, and the quantiser reads it.
  */
 size_t sgat_linear_workspace_size(int L, int K, int with_tac);
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,

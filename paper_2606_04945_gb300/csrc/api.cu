@@ -281,7 +281,8 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     uint8_t* Xq = ws;
     float* s_a = reinterpret_cast<float*>(ws + align256((size_t)L * K / 2));
     uint8_t* Xe = ws + align256((size_t)L * K / 2) + align256((size_t)L * 4);
-    float* zt = tac_M ? reinterpret_cast<float*>(Xe + align256((size_t)L * K)) : nullptr;
+    // TAC output in the input's type (the region has room for float32)
+    void* zt = tac_M ? static_cast<void*>(Xe + align256((size_t)L * K)) : nullptr;
     rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     unsigned* st = status_ptr(&rc);
@@ -291,10 +292,10 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     int qin_dtype = x_dtype;
     cudaError_t e;
     if (tac_M) {
-        TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, STARQ_F32, st, tac_Mp};
+        TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, x_dtype, st, tac_Mp};
         if ((e = launch_tac(t, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: tac launch");
         qin = zt;
-        qin_dtype = STARQ_F32;
+        qin_dtype = x_dtype;
     }
     QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");

@@ -181,8 +181,9 @@ template <typename TOut> struct TacStore;
 template <> struct TacStore<float> {
     static constexpr bool TMA = true;
 };
-template <> struct TacStore<__half> { static constexpr bool TMA = false; };
-template <> struct TacStore<__nv_bfloat16> { static constexpr bool TMA = false; };
+// 16-bit output: 32 x 32 boxes of 64-byte rows with the 64-byte swizzle
+template <> struct TacStore<__half> { static constexpr bool TMA = true; };
+template <> struct TacStore<__nv_bfloat16> { static constexpr bool TMA = true; };
 
 // M_b (float32 [g][g]) -> its two 16-bit halves, K-major (row r = output
 // channel, 8 inputs per 16-byte chunk, 128-byte swizzle) at shared
@@ -360,11 +361,25 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
                     if (lane == 0) bulk_wait_read0();
                     __syncwarp();
                 }
-                #pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    st_shared_v4(box + lane * 128 + ((q ^ (lane & 7)) << 4), __float_as_uint(v[4 * q]),
-                                 __float_as_uint(v[4 * q + 1]), __float_as_uint(v[4 * q + 2]),
-                                 __float_as_uint(v[4 * q + 3]));
+                if (sizeof(TOut) == 4) {                         // 128-byte rows: group q at q ^ (row & 7)
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        st_shared_v4(box + lane * 128 + ((q ^ (lane & 7)) << 4), __float_as_uint(v[4 * q]),
+                                     __float_as_uint(v[4 * q + 1]), __float_as_uint(v[4 * q + 2]),
+                                     __float_as_uint(v[4 * q + 3]));
+                } else {                                         // 64-byte rows: group q at q ^ ((row >> 1) & 3)
+                    #pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint32_t w[4];
+                        #pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            TOut x0 = from_f<TOut>(v[8 * q + 2 * e]), x1 = from_f<TOut>(v[8 * q + 2 * e + 1]);
+                            w[e] = (uint32_t)(*reinterpret_cast<uint16_t*>(&x0)) |
+                                   ((uint32_t)(*reinterpret_cast<uint16_t*>(&x1)) << 16);
+                        }
+                        st_shared_v4(box + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4), w[0], w[1], w[2], w[3]);
+                    }
+                }
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) {
@@ -417,7 +432,9 @@ bool encode_u16_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t co
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-bool encode_f32_out_tmap(CUtensorMap* m, void* ptr, uint64_t rows, uint64_t cols) {
+// Output tensor map with 32 x 32 boxes: float (128-byte rows, 128-byte
+// swizzle) or a 16-bit type (64-byte rows, 64-byte swizzle).
+bool encode_out_tmap16or32(CUtensorMap* m, void* ptr, size_t elem, bool is_f16, uint64_t rows, uint64_t cols) {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (fn == nullptr) {
         cudaDriverEntryPointQueryResult q;
@@ -428,11 +445,13 @@ bool encode_f32_out_tmap(CUtensorMap* m, void* ptr, uint64_t rows, uint64_t cols
         fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
     }
     const cuuint64_t dims[2] = {cols, rows};
-    const cuuint64_t strides[1] = {cols * 4};
+    const cuuint64_t strides[1] = {cols * elem};
     const cuuint32_t box[2] = {32, 32};
     const cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, ptr, dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+    const CUtensorMapDataType type = elem == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+                                     : (is_f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16);
+    return fn(m, type, 2, ptr, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              elem == 4 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -450,11 +469,9 @@ cudaError_t launch_tc(const TacArgs& a, cudaStream_t stream) {
     }
     CUtensorMap tz, to;
     if (!encode_u16_tmap(&tz, a.Z, (uint64_t)a.L, (uint64_t)a.C, TC_TM, 64)) return cudaErrorInvalidValue;
-    if (TacStore<TOut>::TMA) {
-        if (!encode_f32_out_tmap(&to, a.out, (uint64_t)a.L, (uint64_t)a.C)) return cudaErrorInvalidValue;
-    } else {
-        to = tz;   // unused
-    }
+    if (!encode_out_tmap16or32(&to, a.out, sizeof(TOut), std::is_same<TOut, __half>::value, (uint64_t)a.L,
+                               (uint64_t)a.C))
+        return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute at[1] = {pdl_attribute()};
     cfg.gridDim = dim3(a.C / G, (a.L + TC_TM - 1) / TC_TM);

@@ -87,10 +87,11 @@ def gemm_codes(seed, L, N, K, lo=-7, hi=7):
     return qa, qw, s_a, s_w
 
 
-def workspace_views(ws, L, K, with_tac):
+def workspace_views(ws, L, K, with_tac, x_dtype=torch.float32):
     """Views of the intermediates sgat_linear leaves in its workspace
-    (packed codes, per-token scales, E4M3 codes, float32 TAC output),
-    following the layout documented for sgat_linear in include/starq.h."""
+    (packed codes, per-token scales, E4M3 codes, the TAC output in the input's
+    type x_dtype), following the layout documented for sgat_linear in
+    include/starq.h."""
     a256 = lambda x: (x + 255) // 256 * 256
     o1 = a256(L * K // 2)
     o2 = o1 + a256(4 * L)
@@ -98,7 +99,8 @@ def workspace_views(ws, L, K, with_tac):
     Xq = ws[: L * K // 2].view(L, K // 2)
     s_a = ws[o1: o1 + 4 * L].view(torch.float32)
     Xe = ws[o2: o2 + L * K].view(L, K)
-    zt = ws[o3: o3 + 4 * L * K].view(torch.float32).view(L, K) if with_tac else None
+    esz = torch.empty(0, dtype=x_dtype).element_size()
+    zt = ws[o3: o3 + esz * L * K].view(x_dtype).view(L, K) if with_tac else None
     return Xq, s_a, Xe, zt
 
 

@@ -288,7 +288,7 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None, weights="e4m3"):
     """sgat_prepare_weight + sgat_linear on the GPU against the oracle's
     literal split / quantise / GEMM / scatter. With TAC, the TAC output is
     compared within tolerance and the rest of the chain is teacher-forced on
-    the GPU's float32 TAC output (left in the workspace)."""
+    the GPU's TAC output (left in the workspace in the input's type)."""
     xf = case.xf
     dt = H.torch_dtype(case.dtype)
     out_dtype = out_dtype or case.dtype
@@ -314,13 +314,13 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None, weights="e4m3"):
     abi.check_status()
     qw, sw = osg.prepare_weight(case.W, xf.inv_a_w, xf.hb, 4)
     assert np.array_equal(H.unpack(Wq), qw) and np.array_equal(s_w.cpu().numpy(), sw)
-    Xq_g, s_a_g, Xe_g, zt = H.workspace_views(ws, L, K, with_tac)
+    Xq_g, s_a_g, Xe_g, zt = H.workspace_views(ws, L, K, with_tac, dt)
     rows = np.arange(L) if check_rows is None else np.asarray(check_rows)
     X_in = case.X
     if with_tac:
-        z_gpu = zt.cpu().numpy()
+        z_gpu = H.host(zt)
         ref_tac = otac.tac_apply(case.X[rows], case.tac.M, case.tac.d, case.tac.g)
-        H.assert_tac_close(z_gpu[rows], ref_tac, "f32")
+        H.assert_tac_close(z_gpu[rows], ref_tac, case.dtype)
         X_in = z_gpu                      # teacher forcing on the GPU's TAC output
     Y_ref, codes, s_a, acc = osg.sgat_linear(X_in[rows], case.mask[rows], xf.a_m, xf.a_u, xf.hb, xf.d_sh,
                                              xf.d_m, xf.d_u, qw, sw, case.bias, 4)
