@@ -154,6 +154,17 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
               int y_dtype, int32_t* acc_dbg, void* stream);
 
 /*
+ * Tile of the last Xe + We (or fp16_gemm_ref) launch on the calling thread,
+ * as BN * 10 + cluster size: 2564 (256-channel pair tiles, two pairs per
+ * cluster sharing the activation tile), 2562, or 2242 (224-channel tiles on
+ * single pairs); 0 before the first. The launcher estimates each shape's
+ * time as ceil(tiles / resident clusters) rounds of a stage cost bound by
+ * shared-memory traffic and takes the cheaper. A diagnostic for tests and
+ * tuning; the results do not depend on it.
+ */
+int starq_last_gemm_tile(void);
+
+/*
  * fp16_gemm_ref -- the 16-bit baseline of the projections: C = A B^T with
  * float32 accumulation and one rounding to the element type. It is the
  * unquantised model's linear layer that Sec. 4.4 measures its speed-up

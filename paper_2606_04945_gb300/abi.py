@@ -19,7 +19,7 @@ OK, ERR_ARG, ERR_SHAPE, ERR_ALIGN, ERR_BITS, ERR_CUDA, ERR_TIMEOUT = 0, -1, -2, 
 EXPORTED = (
     "starq_version", "starq_last_error", "starq_check_status",
     "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "fp16_gemm_ref", "tac_prepare", "tac_apply",
-    "sgat_linear_workspace_size", "sgat_linear",
+    "sgat_linear_workspace_size", "sgat_linear", "starq_last_gemm_tile",
 )
 
 
@@ -43,6 +43,7 @@ def _load():
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.tac_prepare.argtypes = [f_p, i, i, i, vp, vp]
+    lib.starq_last_gemm_tile.restype = i
     lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, vp, i, vp]
     lib.fp16_gemm_ref.argtypes = [vp, vp, i, i, i, i, vp, vp]
     lib.sgat_linear_workspace_size.argtypes = [i, i, i]
@@ -125,6 +126,13 @@ def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, st
     N, K = _weight_shape(Wq, We)
     _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y),
                          dtype_code(Y), _p(acc_dbg), _stream(stream)))
+
+
+def last_gemm_tile():
+    """(channels per pair tile, CTAs per cluster) of the calling thread's
+    last TMA pair GEMM launch, or None before the first."""
+    t = int(lib.starq_last_gemm_tile())
+    return (t // 10, t % 10) if t else None
 
 
 def fp16_gemm_ref(A, B, C, stream=None):

@@ -116,6 +116,8 @@ extern "C" {
 
 int starq_version(void) { return 100; }
 
+int starq_last_gemm_tile(void) { return last_gemm_tile(); }
+
 const char* starq_last_error(void) { return g_err; }
 
 int starq_check_status(void* stream) {

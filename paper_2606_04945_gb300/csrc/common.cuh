@@ -51,6 +51,9 @@ struct GemmArgs {
     int weights_ready = 0;
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+// Tile of the calling thread's last TMA pair GEMM launch (BN * 10 + cluster
+// size; 0 before the first).
+int last_gemm_tile();
 // Plain 16-bit GEMM C = A B^T (A = a.Xe [L][K], B = a.We [N][K], both of
 // type a.y_dtype, float32 accumulation, C = a.Y), no scales.
 cudaError_t launch_fp16_gemm(const GemmArgs& a, cudaStream_t stream);

@@ -798,15 +798,26 @@ bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t
 // MMAs have read it. 6 stages of 32 KB; 8 epilogue warps.
 // ---------------------------------------------------------------------------
 namespace tmak {
-constexpr int BM = 128, BN = 256, BN_CTA = 128, BK = 128, UMMA_K = 32;
-constexpr int A_BYTES = BM * BK, B_BYTES = BN_CTA * BK;
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;             // 32 KB
+constexpr int BM = 128, BK = 128, UMMA_K = 32;
+constexpr int A_BYTES = BM * BK;
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int TMA_WARP = 8, MMA_WARP = 9;
 constexpr int THREADS = 10 * 32;
 constexpr int TMEM_COLS = 512;
-constexpr int EPI_PARAM_BYTES = NUM_EPI_WARPS * 2 * (BN / 2) * 4;
-constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
+constexpr int ACC_STRIDE = 256;                // TMEM columns from one accumulator to the other
+constexpr int EPI_CHUNKS = 4;                  // 32-column chunks per epilogue warp and tile
+constexpr int EPI_PARAM_BYTES = NUM_EPI_WARPS * 2 * (EPI_CHUNKS * 32) * 4;
+// A CTA pair's output tile is 256 tokens x BN channels; each CTA holds
+// BN / 2 weight rows of every stage.
+template <int BN>
+struct Tile {
+    static_assert(BN % 32 == 0 && BN >= 64 && BN <= 256, "pair tile width");
+    static constexpr int BN_CTA = BN / 2;
+    static constexpr int B_BYTES = BN_CTA * BK;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;       // 32 KB at BN = 256
+    static_assert(STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
+    static constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((2 * BM) >> 4) << 24);
+};
 template <int S>
 struct Smem {
     uint64_t full[S];             // pair leader: both CTAs' TMA bytes
@@ -817,32 +828,57 @@ struct Smem {
     uint32_t tmem_base;
     int abort;
 };
-// Per output element size: one 32 x 32 staging box per epilogue warp, and
-// as many 32 KB stages as the rest of the 227 KB allows (6 for 16-bit
-// outputs, 5 for float).
-template <int OUT_BYTES>
+// Per output element size and tile width: one 32 x 32 staging box per
+// epilogue warp, and as many stages (up to 6) as the rest of the 227 KB
+// allows: at BN = 256, 6 for 16-bit outputs and 5 for float; at BN = 224, 6.
+template <int OUT_BYTES, int BN>
 struct Cfg {
     static constexpr int EPI_BOX_WARP_BYTES = 32 * 32 * OUT_BYTES;
     static constexpr int EPI_STAGE_BYTES = NUM_EPI_WARPS * EPI_BOX_WARP_BYTES;
-    static constexpr int STAGES = OUT_BYTES == 4 ? 5 : 6;
-    static constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + EPI_STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
-    static_assert(SMEM_BYTES <= 227 * 1024, "shared memory");
+    static constexpr int FIXED = EPI_STAGE_BYTES + EPI_PARAM_BYTES + 1024 + 512;
+    static constexpr int FIT = (227 * 1024 - FIXED) / Tile<BN>::STAGE_BYTES;
+    static constexpr int STAGES = FIT < 6 ? FIT : 6;
+    static constexpr size_t SMEM_BYTES = (size_t)STAGES * Tile<BN>::STAGE_BYTES + FIXED;
+    static_assert(STAGES >= 4 && SMEM_BYTES <= 227 * 1024, "shared memory");
 };
 }  // namespace tmak
 
 // OPK: operand kind -- 0 = E4M3 codes (dequantising epilogue), 1 = fp16,
 // 2 = bf16 (plain float32 accumulator cast to the output type). Every kind
 // reads 128-byte K rows and advances 32 bytes of K per MMA.
-template <typename TOut, int CL, int OPK>
+// Tile of the calling thread's last TMA pair GEMM launch: BN * 10 + CL.
+thread_local int g_last_tile = 0;
+
+// Output tiles of the pair GEMM: 256-token rows x BN-channel pair tiles,
+// CL / 2 pairs side by side per cluster tile.
+int tma_tiles(int L, int N, int BN, int CL) {
+    const int num_n = (N + BN - 1) / BN;
+    return ((L + 2 * tmak::BM - 1) / (2 * tmak::BM)) * ((num_n + CL / 2 - 1) / (CL / 2));
+}
+// Estimated cycles of a launch (twice the model's stage cycles per round).
+long long tma_round_cost(int L, int N, int BN, int CL, int clusters) {
+    const long long tiles = tma_tiles(L, N, BN, CL);
+    const long long used = clusters < 1 ? 1 : clusters;
+    const long long rounds = (tiles + used - 1) / used;
+    const long long stage2 = 4LL * BN > 512LL + 3LL * BN ? 4LL * BN : 512LL + 3LL * BN;
+    return rounds * stage2;
+}
+
+template <typename TOut, int CL, int OPK, int BN>
 __global__ void __launch_bounds__(tmak::THREADS, 1)
 w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
                           const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y) {
-    constexpr int BM = tmak::BM, BN = tmak::BN, BN_CTA = tmak::BN_CTA, BK = tmak::BK;
-    constexpr int UMMA_K = tmak::UMMA_K, STAGES = tmak::Cfg<sizeof(TOut)>::STAGES, STAGE_BYTES = tmak::STAGE_BYTES;
-    constexpr int A_BYTES = tmak::A_BYTES, B_BYTES = tmak::B_BYTES;
+    using Tile = tmak::Tile<BN>;
+    using Cfg = tmak::Cfg<sizeof(TOut), BN>;
+    constexpr int BM = tmak::BM, BN_CTA = Tile::BN_CTA, BK = tmak::BK;
+    constexpr int UMMA_K = tmak::UMMA_K, STAGES = Cfg::STAGES, STAGE_BYTES = Tile::STAGE_BYTES;
+    constexpr int A_BYTES = tmak::A_BYTES, B_BYTES = Tile::B_BYTES;
     constexpr int TMA_WARP = tmak::TMA_WARP, MMA_WARP = tmak::MMA_WARP;
     constexpr int NUM_EPI_WARPS = tmak::NUM_EPI_WARPS, TMEM_COLS = tmak::TMEM_COLS;
-    constexpr uint32_t IDESC = tmak::IDESC | (OPK == 2 ? ((1u << 7) | (1u << 10)) : 0u);
+    constexpr int ACC_STRIDE = tmak::ACC_STRIDE, EPI_CHUNKS = tmak::EPI_CHUNKS;
+    static_assert(ACC_STRIDE >= BN && ACC_STRIDE + BN <= TMEM_COLS, "two accumulators in TMEM");
+    static_assert(2 * EPI_CHUNKS * 32 >= BN, "two epilogue warps per row quarter cover the tile");
+    constexpr uint32_t IDESC = Tile::IDESC | (OPK == 2 ? ((1u << 7) | (1u << 10)) : 0u);
     constexpr int BKE = OPK == 0 ? BK : BK / 2;          // K elements per stage row
     constexpr bool DEQUANT = OPK == 0;
     constexpr int PAIRS = CL / 2;
@@ -853,8 +889,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
-    constexpr int EPI_STAGE_BYTES = tmak::Cfg<sizeof(TOut)>::EPI_STAGE_BYTES;
-    constexpr int EPI_BOX_WARP_BYTES = tmak::Cfg<sizeof(TOut)>::EPI_BOX_WARP_BYTES;
+    constexpr int EPI_STAGE_BYTES = Cfg::EPI_STAGE_BYTES;
+    constexpr int EPI_BOX_WARP_BYTES = Cfg::EPI_BOX_WARP_BYTES;
     Smem* sh = reinterpret_cast<Smem*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES + EPI_STAGE_BYTES);
     volatile int* abort = &sh->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -955,7 +991,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
                 if (!mbar_wait_bounded_warp(smem_addr(&sh->tmem_empty[acc]), acc_phase ^ 1u, abort)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * ACC_STRIDE);
                 for (int kc = 0; kc < num_k; ++kc) {
                     if (!mbar_wait_bounded_warp(smem_addr(&sh->full[stage]), phase, abort)) { ok = false; break; }
                     tc_fence_after();
@@ -986,7 +1022,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         __syncwarp();
     } else {
         // epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31, columns
-        // (w / 4) * 128 .. + 127, in 32 x 32 boxes; scales and biases are
+        // (w / 4) * 128 .. + 127 below BN, in 32 x 32 boxes; scales and biases are
         // staged before the accumulator wait. Each box is dequantised into
         // the warp's swizzled staging buffer and written by one TMA store
         // (rows past L and columns past N are clipped by the tensor map).
@@ -995,8 +1031,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         const uint32_t leader_tmem_empty0 = mapa_shared(smem_addr(&sh->tmem_empty[0]), leader);
         const uint32_t ybox0 = base + STAGES * STAGE_BYTES + warp * EPI_BOX_WARP_BYTES;
         float* epi_sw = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sh) + sizeof(Smem) +
-                                                 (16 - sizeof(Smem) % 16) % 16) + warp * 2 * (BN / 2);
-        float* epi_b = epi_sw + BN / 2;
+                                                 (16 - sizeof(Smem) % 16) % 16) + warp * 2 * (EPI_CHUNKS * 32);
+        float* epi_b = epi_sw + EPI_CHUNKS * 32;
         const int quarter = warp & 3, chalf = warp >> 2;
         bool ok = true;
         int it = 0;
@@ -1010,7 +1046,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
             const bool valid = row < L;
             const float sa = (DEQUANT && valid) ? __ldg(a.s_a + row) : 0.f;
             if (DEQUANT) {
-                const int ncol = n0 + chalf * (BN / 2) + 4 * lane;
+                const int ncol = n0 + chalf * (EPI_CHUNKS * 32) + 4 * lane;
                 float4 w = make_float4(0.f, 0.f, 0.f, 0.f), bb = w;
                 if (ncol < N) {
                     w = __ldg(reinterpret_cast<const float4*>(a.s_w + ncol));
@@ -1024,12 +1060,12 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
             // a whole tile of MMAs away: poll gently, the MMA warp shares the scheduler
             if (!mbar_wait_bounded_sleepy(smem_addr(&sh->tmem_full[acc]), acc_phase, abort, 256)) { ok = false; break; }
             tc_fence_after();
-            const uint32_t t_row = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+            const uint32_t t_row = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * ACC_STRIDE);
             #pragma unroll 1
-            for (int cc = 0; cc < BN / 64; ++cc) {
-                const int c = chalf * (BN / 64) + cc;
+            for (int cc = 0; cc < EPI_CHUNKS; ++cc) {
+                const int c = chalf * EPI_CHUNKS + cc;
                 const int nc = n0 + c * 32;
-                if (nc >= N) break;
+                if (c * 32 >= BN || nc >= N) break;
                 uint32_t r[32];
                 tmem_ld_32x32b_x32(t_row + c * 32, r);
                 tmem_ld_wait();
@@ -1120,15 +1156,43 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     if (warp == MMA_WARP) tmem_dealloc_pair(tmem_base, TMEM_COLS);
 }
 
-template <typename TOut, int CL, int OPK>
-cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
-    constexpr int BM = tmak::BM, BN = tmak::BN, BN_CTA = tmak::BN_CTA, BK = tmak::BK;
-    constexpr int ELEM = OPK == 0 ? 1 : 2;
-    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL, OPK>;
-    static bool attr_set[64] = {false};
+// Clusters of this instantiation resident at once on the current device
+// (queried once per device; also sets the kernel's shared-memory limit).
+template <typename TOut, int CL, int OPK, int BN>
+cudaError_t tma_max_clusters(int* clusters) {
+    constexpr size_t SMEM_BYTES = tmak::Cfg<sizeof(TOut), BN>::SMEM_BYTES;
+    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN>;
     static int max_clusters[64] = {0};
     int dev = 0;
     cudaGetDevice(&dev);
+    if (dev < 0 || dev >= 64) dev = 63;
+    if (max_clusters[dev] == 0) {
+        cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = CL;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.blockDim = dim3(tmak::THREADS);
+        cfg.dynamicSmemBytes = SMEM_BYTES;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;                // the occupancy query takes the cluster shape only
+        cfg.gridDim = dim3(CL * 32);
+        int n = 0;
+        e = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg);
+        if (e != cudaSuccess) return e;
+        max_clusters[dev] = n > 0 ? n : 1;
+    }
+    *clusters = max_clusters[dev];
+    return cudaSuccess;
+}
+
+template <typename TOut, int CL, int OPK, int BN>
+cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) {
+    constexpr int BM = tmak::BM, BN_CTA = tmak::Tile<BN>::BN_CTA, BK = tmak::BK;
+    constexpr int ELEM = OPK == 0 ? 1 : 2;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -1137,21 +1201,10 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
     attr[0].val.clusterDim.z = 1;
     attr[1] = pdl_attribute();
     cfg.blockDim = dim3(tmak::THREADS);
-    cfg.dynamicSmemBytes = tmak::Cfg<sizeof(TOut)>::SMEM_BYTES;
+    cfg.dynamicSmemBytes = tmak::Cfg<sizeof(TOut), BN>::SMEM_BYTES;
     cfg.stream = stream;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;                // the occupancy query takes the cluster shape only
-    if (dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)tmak::Cfg<sizeof(TOut)>::SMEM_BYTES);
-        if (e != cudaSuccess) return e;
-        cfg.gridDim = dim3(CL * 32);
-        int n = 0;
-        e = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg);
-        if (e != cudaSuccess) return e;
-        max_clusters[dev] = n;
-        attr_set[dev] = true;
-    }
+    cfg.numAttrs = 2;
     CUtensorMap ta, tb, ty;
     const CUtensorMapDataType opt = OPK == 0 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
     if (!encode_operand_tmap(&ta, a.Xe, opt, ELEM, (uint64_t)a.L, (uint64_t)a.K, CL == 2 ? BM : BM / 2, BK / ELEM) ||
@@ -1159,20 +1212,36 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream) {
         !encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N,
                          Out<TOut>::TMAP_SWIZZLE))
         return cudaErrorInvalidValue;
-    const int num_n = (a.N + BN - 1) / BN;
-    const int num_tiles = ((a.L + 2 * BM - 1) / (2 * BM)) * ((num_n + CL / 2 - 1) / (CL / 2));
-    int clusters = dev < 64 ? max_clusters[dev] : 1;
-    if (clusters < 1) clusters = 1;
+    const int num_tiles = tma_tiles(a.L, a.N, BN, CL);
     if (num_tiles < clusters) clusters = num_tiles;
     cfg.gridDim = dim3(CL * clusters);
-    cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb, ty);
+    return cudaLaunchKernelEx(&cfg, w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN>, a, ta, tb, ty);
 }
 
+// Tile shape per problem. A stage's steady state is bound by shared memory:
+// per CTA the MMAs read the 16 KB activation tile and the CTA's weight half
+// twice (for itself and for its pair peer) while TMA writes both, i.e.
+// 256 + 1.5 BN cycles at 128 bytes per clock against 2 BN cycles of tensor
+// work. A launch takes ceil(tiles / clusters) rounds of a tile's stages.
+// Candidates: 256-wide pair tiles (two pairs per cluster sharing the
+// activation tile when there are at least two channel tiles) and 224-wide
+// tiles on single pairs, whose tile counts fill the 76 pairs of the LLaDA
+// projections better; the cheaper estimate wins, ties keep 256.
 template <typename TOut, int OPK = 0>
 cudaError_t launch_tma_typed(const GemmArgs& a, cudaStream_t stream) {
-    const int num_n = (a.N + tmak::BN - 1) / tmak::BN;
-    return num_n >= 2 ? launch_tma_cl<TOut, 4, OPK>(a, stream) : launch_tma_cl<TOut, 2, OPK>(a, stream);
+    const bool quad = (a.N + 255) / 256 >= 2;
+    int c256 = 0, c224 = 0;
+    cudaError_t e = quad ? tma_max_clusters<TOut, 4, OPK, 256>(&c256) : tma_max_clusters<TOut, 2, OPK, 256>(&c256);
+    if (e != cudaSuccess) return e;
+    if ((e = tma_max_clusters<TOut, 2, OPK, 224>(&c224)) != cudaSuccess) return e;
+    const long long t256 = tma_round_cost(a.L, a.N, 256, quad ? 4 : 2, c256);
+    const long long t224 = tma_round_cost(a.L, a.N, 224, 2, c224);
+    if (t224 < t256) {
+        g_last_tile = 224 * 10 + 2;
+        return launch_tma_cl<TOut, 2, OPK, 224>(a, stream, c224);
+    }
+    g_last_tile = 256 * 10 + (quad ? 4 : 2);
+    return quad ? launch_tma_cl<TOut, 4, OPK, 256>(a, stream, c256) : launch_tma_cl<TOut, 2, OPK, 256>(a, stream, c256);
 }
 
 // Packed int4 -> E4M3: each thread turns 16 packed bytes into 32 E4M3 bytes.
@@ -1278,6 +1347,8 @@ cudaError_t launch_unpack_e4m3(const uint8_t* packed, uint8_t* e4m3, size_t rows
                                                                reinterpret_cast<uint4*>(e4m3), n16);
     return cudaGetLastError();
 }
+
+int last_gemm_tile() { return g_last_tile; }
 
 cudaError_t launch_fp16_gemm(const GemmArgs& a, cudaStream_t stream) {
     if (a.L == 0) return cudaSuccess;

@@ -196,7 +196,27 @@ def test_w4a4_gemm_exact(abi, L, N, K, out, path):
     H.assert_output_close(Y, osg.dequant(ref_acc, s_a, s_w, bias), out)
 
 
-@pytest.mark.parametrize("M,N,K,dt", [(1, 32, 64, "f16"), (129, 288, 640, "f16"), (300, 512, 1024, "bf16"),
+@pytest.mark.parametrize("out", ["f16", "f32"])
+def test_w4a4_gemm_tile_widths(abi, out):
+    """The launcher takes 256-channel pair tiles (two pairs per cluster) or
+    224-channel tiles on single pairs, whichever its estimate makes cheaper.
+    4608 x 1024 fills 36 clusters exactly with 256-wide tiles (224 would need
+    a second round); 97 x 256 is one round either way, and the narrower tile
+    has the cheaper stage; the LLaDA widths 4096 and 12288 (at a short K)
+    favour 224. Every product is exact, and both widths occur."""
+    seen = set()
+    for L, N, K in [(4608, 1024, 128), (97, 256, 128), (1024, 4096, 256), (1024, 12288, 256), (300, 4128, 384)]:
+        qa, qw, s_a, s_w = H.gemm_codes(L + N + K, L, N, K)
+        Y, acc = run_gemm(abi, qa, qw, s_a, s_w, out, path="tma")
+        bn, cl = abi.last_gemm_tile()
+        seen.add(bn)
+        ref = osg.int_gemm(qa, qw)
+        assert np.array_equal(acc, ref), f"integer accumulators differ ({L}x{N}x{K}, tile {bn}/{cl})"
+        H.assert_output_close(Y, osg.dequant(ref, s_a, s_w, None), out)
+    assert seen == {224, 256}, seen
+
+
+@pytest.mark.parametrize("M,N,K,dt", [(1, 32, 64, "f16"), (129, 288, 640, "f16"), (300, 512, 1024, "bf16"), (4608, 1024, 128, "bf16"),
                                       (1024, 4096, 4096, "f16"), (77, 768, 4096, "bf16")])
 def test_fp16_gemm_ref(abi, M, N, K, dt):
     """The 16-bit baseline GEMM against the exact product: float64 sums of
