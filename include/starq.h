@@ -233,6 +233,15 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  *   padded to 256][TAC output: L*K values of x_dtype (room for float32), only
  *   with TAC]. The TAC output is rounded to x_dtype once, as the unquantised
  *   model stores attention outputs, and the quantiser reads it.
+ *
+ *   Programmatic launch: the kernels of sgat_linear may start while the
+ *   previous kernel of the stream is still running (CUDA programmatic
+ *   dependent launch) and read the layer's parameters (Wq/We, s_w, bias,
+ *   tac_M, tac_d, tac_Mp) before waiting for it; the inputs and the
+ *   workspace are read only after it has completed. Parameters must
+ *   therefore not be written by a kernel that lets its dependents start
+ *   early; no kernel of this library does, and the preparation calls
+ *   (sgat_prepare_weight, w4_unpack_e4m3, tac_prepare) never let them.
  */
 size_t sgat_linear_workspace_size(int L, int K, int with_tac);
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,

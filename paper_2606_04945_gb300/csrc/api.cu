@@ -295,6 +295,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     cudaError_t e;
     if (tac_M) {
         TacArgs t{X, x_dtype, L, K, tac_g, tac_M, tac_d, zt, x_dtype, st, tac_Mp};
+        t.params_ready = 1;      // layer parameters: see the header's note on programmatic launch
         if ((e = launch_tac(t, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: tac launch");
         qin = zt;
         qin_dtype = x_dtype;

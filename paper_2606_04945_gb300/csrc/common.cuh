@@ -74,6 +74,10 @@ struct TacArgs {
     const float* M; const float* d; void* out; int out_dtype;
     unsigned* status = nullptr;   // device status word (tensor-core path)
     const void* Mp = nullptr;     // optional tac_prepare output (tensor-core path)
+    // The caller guarantees that no kernel still running when this one is
+    // launched writes Mp or d: they are fetched before the wait for the
+    // previous kernel (programmatic launch).
+    int params_ready = 0;
 };
 cudaError_t launch_tac(const TacArgs& a, cudaStream_t stream);
 // M [C/g][g][g] float32 -> its 16-bit halves (hi = rn(M), lo = rn(M - hi), of

@@ -269,7 +269,8 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
               unsigned* status) {
     using P = TacTc<G>;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t zfull, mdone;
+    __shared__ __align__(8) uint64_t zfull, mfull, mdone;
+    __shared__ __align__(16) float dsm[G];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_flag;
     const uint32_t raw = smem_addr(smem_raw);
@@ -283,6 +284,7 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
 
     if (threadIdx.x == 0) {
         mbar_init(smem_addr(&zfull), 1);
+        mbar_init(smem_addr(&mfull), 1);
         mbar_init(smem_addr(&mdone), 1);
         abort_flag = 0;
         mbar_fence_init();
@@ -293,21 +295,31 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
         tmem_relinquish();
     }
     __syncthreads();
+    // both 16-bit halves of M_b (prepared) on their own barrier, and d_b in
+    // shared memory; ahead of the wait for the previous kernel when the
+    // caller vouches that it does not write them
+    auto fetch_params = [&]() {
+        if (threadIdx.x == 0 && prepared) {
+            mbar_arrive_expect_tx(smem_addr(&mfull), 2 * P::M_BYTES);
+            bulk_load(sMh, static_cast<const uint8_t*>(a.Mp) + (size_t)b * 2 * P::M_BYTES, 2 * P::M_BYTES,
+                      smem_addr(&mfull));
+        }
+        if (!prepared) tac_split_block<G, TIn>(a.M + (size_t)b * G * G, sMh, sMl);
+        if (threadIdx.x < G / 4)
+            reinterpret_cast<float4*>(dsm)[threadIdx.x] =
+                a.d ? __ldg(reinterpret_cast<const float4*>(a.d + (size_t)b * G) + threadIdx.x)
+                    : make_float4(0.f, 0.f, 0.f, 0.f);
+    };
+    if (a.params_ready) fetch_params();
     // the prologue above may overlap the previous kernel (programmatic launch)
     grid_dependency_wait();
     grid_launch_dependents();
+    if (!a.params_ready) fetch_params();
     if (threadIdx.x == 0) {
-        // Z tile (and, when prepared, both 16-bit halves of M_b) on one barrier
-        mbar_arrive_expect_tx(smem_addr(&zfull), P::Z_BYTES + (prepared ? 2 * P::M_BYTES : 0));
+        mbar_arrive_expect_tx(smem_addr(&zfull), P::Z_BYTES);
         for (int at = 0; at < P::ATOMS; ++at)
             tma_load_2d(sZ + at * (TC_TM * 128), &tmap_z, b * G + at * 64, row0, smem_addr(&zfull));
-        if (prepared)
-            bulk_load(sMh, static_cast<const uint8_t*>(a.Mp) + (size_t)b * 2 * P::M_BYTES, 2 * P::M_BYTES,
-                      smem_addr(&zfull));
     }
-    if (!prepared)
-        tac_split_block<G, TIn>(a.M + (size_t)b * G * G, sMh, sMl);
-
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
@@ -316,7 +328,8 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
     constexpr uint32_t IDESC = (1u << 4) | (Split16<TIn>::KIND << 7) | (Split16<TIn>::KIND << 10) |
                                ((uint32_t)(G >> 3) << 17) | ((uint32_t)(TC_TM >> 4) << 24);
     if (threadIdx.x == 0) {
-        if (!mbar_wait_bounded(smem_addr(&zfull), 0, abort)) {
+        if (!mbar_wait_bounded(smem_addr(&zfull), 0, abort) ||
+            (prepared && !mbar_wait_bounded(smem_addr(&mfull), 0, abort))) {
             *abort = 1;
         } else {
             tc_fence_after();
@@ -337,7 +350,6 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
         const int quarter = warp & 3, chalf = warp >> 2;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
         const int tok = row0 + quarter * 32 + lane;
-        const float* dp = a.d ? a.d + (size_t)b * G : nullptr;
         const uint32_t box = sZ + warp * (32 * 32 * 4);
         TOut* out = static_cast<TOut*>(a.out);
         #pragma unroll 1
@@ -349,8 +361,7 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
             float v[32];
             #pragma unroll
             for (int j = 0; j < 32; j += 4) {
-                float4 dd = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (dp) dd = __ldg(reinterpret_cast<const float4*>(dp + col + j));
+                const float4 dd = reinterpret_cast<const float4*>(dsm + col)[j / 4];
                 v[j] = __uint_as_float(r[j]) + dd.x;
                 v[j + 1] = __uint_as_float(r[j + 1]) + dd.y;
                 v[j + 2] = __uint_as_float(r[j + 2]) + dd.z;
