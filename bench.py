@@ -532,19 +532,68 @@ def cpu_cores():
     return os.cpu_count() or 1
 
 
-def cpu_baseline(qkv_case, o_case, tokens):
+def cpu_model():
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.machine()
+
+
+def oracle_sample(qkv_case, o_case, tokens):
+    """Seconds and int ops of one full oracle step on the first `tokens`
+    tokens (weight folding untimed)."""
     import numpy as np
     w = oracle_prepare(qkv_case, o_case)
     rows = np.arange(min(tokens, qkv_case.L))
     t0 = time.perf_counter()
     oracle_step(qkv_case, o_case, w, rows)
     dt = time.perf_counter() - t0
-    ops = 2 * len(rows) * (qkv_case.N + o_case.N) * qkv_case.K
-    return {"value": round(ops / dt / 1e12, 6), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-            "sample": f"one full oracle step on {len(rows)} of {qkv_case.L} tokens "
-                      f"(TAC + SGAT quantise + exact int GEMM + dequant, both projections; "
-                      f"weight folding untimed); {dt:.2f} s",
-            "seconds": round(dt, 3)}
+    return dt, 2 * len(rows) * (qkv_case.N + o_case.N) * qkv_case.K
+
+
+def single_thread_sample(tokens):
+    """The same oracle step in a child process whose BLAS and OpenMP pools
+    have one thread each."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = ("import json, bench\n"
+            "from paper_2606_04945_gb300 import inputs\n"
+            "q, o = inputs.llada_attention(seed=0)\n"
+            f"print(json.dumps(bench.oracle_sample(q, o, {int(tokens)})))\n")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True,
+                       timeout=900)
+    if r.returncode != 0:
+        return None
+    dt, ops = json.loads(r.stdout.strip().splitlines()[-1])
+    return dt, ops
+
+
+def cpu_baseline(qkv_case, o_case, tokens, single_tokens=128):
+    dt, ops = oracle_sample(qkv_case, o_case, tokens)
+    out = {"value": round(ops / dt / 1e12, 6), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+           "sample": f"one full oracle step on {min(tokens, qkv_case.L)} of {qkv_case.L} tokens "
+                     f"(TAC + SGAT quantise + exact int GEMM + dequant, both projections; "
+                     f"weight folding untimed); {dt:.2f} s",
+           "seconds": round(dt, 3), "nproc": os.cpu_count(), "cpu_model": cpu_model()}
+    st = single_thread_sample(single_tokens)
+    if st is not None:
+        sdt, sops = st
+        out["single_thread"] = {"value": round(sops / sdt / 1e12, 6), "unit": UNIT, "cores": 1,
+                                "sample": f"the same step on {single_tokens} tokens, one BLAS/OpenMP "
+                                          f"thread (child process); {sdt:.2f} s",
+                                "seconds": round(sdt, 3)}
+    return out
 
 
 def run_reference(args):
