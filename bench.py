@@ -50,9 +50,11 @@ def parse():
     p.add_argument("--cpu-sample-tokens", type=int, default=1024)
     p.add_argument("--ref-sample-tokens", type=int, default=128)
     p.add_argument("--skip-cpu-baseline", action="store_true")
-    p.add_argument("--workload", default="attention_step", choices=["attention_step", "denoise_stack"],
+    p.add_argument("--workload", default="attention_step",
+                   choices=["attention_step", "denoise_stack", "tac_calibration"],
                    help="attention_step: the LLaDA attention projections (default); denoise_stack: the "
-                        "64-step 4-layer LLaDA-shaped stack (per-step tokens/s, latency, drift vs fp16)")
+                        "64-step 4-layer LLaDA-shaped stack (per-step tokens/s, latency, drift vs fp16); "
+                        "tac_calibration: App. C's closed-form TAC calibration on the GPU vs the oracle")
     return p.parse_args()
 
 
@@ -705,8 +707,63 @@ def run_stack(args):
     }
 
 
+def run_tac_calibration(args):
+    """TAC's closed-form calibration (App. C) on the GPU against the oracle,
+    on paired calibration outputs of the LLaDA attention width (8 samples of
+    1024 tokens, C = 4096) at g = 128 (the block size tac_apply runs in the
+    attention step) and g = 16 (the paper's default)."""
+    import numpy as np
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi, inputs
+    from oracle import tac as otac
+    torch.cuda.set_device(0)
+    N, C = 8192, 4096
+    Zf, Zq = inputs.tac_calibration_pairs(0, N, C, 128)
+    zf, zq = torch.from_numpy(Zf).cuda(), torch.from_numpy(Zq).cuda()
+    res = {}
+    for g in (128, 16):
+        M = torch.empty(C // g, g, g, dtype=torch.float32, device="cuda")
+        d = torch.empty(C // g, g, dtype=torch.float32, device="cuda")
+        ws = torch.empty(abi.tac_calibrate_workspace_size(C, g), dtype=torch.uint8, device="cuda")
+        for _ in range(max(args.warmup, 1)):
+            abi.tac_calibrate(zf, zq, g, M, d, ws)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 5
+        e0.record()
+        for _ in range(reps):
+            abi.tac_calibrate(zf, zq, g, M, d, ws)
+        e1.record()
+        e1.synchronize()
+        abi.check_status()
+        ms = e0.elapsed_time(e1) / reps
+        t0 = time.perf_counter()
+        Mo, do = otac.tac_calibrate(Zf.astype(np.float64), Zq.astype(np.float64), g)
+        t_orc = time.perf_counter() - t0
+        Mg = M.cpu().numpy().astype(np.float64)
+        err = float(np.abs(Mg - Mo).max() / max(1.0, np.abs(Mo).max()))
+        # the token reduction's float64 work: both representations' sums and
+        # upper-triangle second moments, 2 flops per multiply-add
+        flops = 2 * 2 * N * (C // g) * (g * (g + 4) / 2 + g)
+        res[f"g{g}"] = {"ms": round(ms, 3), "oracle_s": round(t_orc, 3), "speedup_vs_oracle": round(t_orc * 1e3 / ms, 1),
+                        "max_rel_err_M_vs_oracle": err, "stats_fp64_gflop": round(flops / 1e9, 2)}
+    return {"metric": "TAC closed-form calibration time (App. C)", "unit": "ms", "higher_is_better": False,
+            "data": "synthetic paired calibration outputs (seeded)", "dtype": "fp16 in, float64 math, float32 out",
+            "config": {"workload": "tac_calibration", "tokens": N, "channels": C}, "n_gpus": 1,
+            "cpu_baseline": {"kind": "oracle", "cores": cpu_cores(), "nproc": os.cpu_count(),
+                             "cpu_model": cpu_model(), "sample": "the full calibration of each g"},
+            "results": res}
+
+
 def main():
     args = parse()
+    if args.workload == "tac_calibration":
+        out = run_tac_calibration(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
+                                                                    "the oracle arm times the attention-step workload"}
+        print(json.dumps(out), flush=True)
+        return
     if args.workload == "denoise_stack":
         out = run_stack(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
                                                            "the oracle arm times the attention-step workload"}

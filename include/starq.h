@@ -215,6 +215,37 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
               const void* Mp, void* out, int out_dtype, void* stream);
 
 /*
+ * tac_calibrate -- the closed-form TAC parameters (App. C, "Block-wise
+ * statistics" through "Bias estimation"), on the GPU in float64.
+ *
+ *   For every block b of g channels, from the N paired calibration tokens:
+ *     mu_b, Sigma_b = population mean and covariance of Z_fp and of Z_q;
+ *     lambda_b = rho * max(Tr(Sigma^Q_b) / g, eps);
+ *     M_b = (Sigma^FP_b)^(1/2) (Sigma^Q_b + lambda_b I)^(-1/2), each power
+ *           Q diag(max(lambda_i, 1e-12)^p) Q^T of a symmetric
+ *           eigendecomposition;
+ *     singular values of M_b replaced by (1 - eta) sigma_i + eta mean(sigma);
+ *     M_b <- (1 - alpha) M_b + alpha I;  d_b = mu^FP_b - M_b mu^Q_b.
+ *   The paper's defaults: rho = 3e-4, eps = 1e-8, eta = 0.15, alpha = 0.55.
+ *
+ *   Z_fp, Z_q [N][C] of element type z_dtype (F16, BF16 or F32), the full-
+ *     precision and quantised attention outputs of the same N tokens,
+ *     16-byte aligned.
+ *   M out [C/g][g][g] float32 (row r = output channel r of block b), d out
+ *     [C/g][g] float32: tac_apply's parameter layout. 16-byte aligned.
+ *   workspace: tac_calibrate_workspace_size(C, g) bytes of device memory,
+ *     256-byte aligned, caller-owned; its contents do not matter.
+ * Shapes: N >= 1, g in {4, 8, 16, 32, 64, 128}, C % g == 0.
+ * Kernels: a token reduction (fp64 sums and second moments per block) and
+ * one CTA per block for the matrix functions (parallel cyclic Jacobi) and
+ * the SVD of M (one-sided Jacobi on the same schedule).
+ */
+size_t tac_calibrate_workspace_size(int C, int g);
+int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, int g, double rho, double eps,
+                  double eta, double alpha, float* M, float* d, void* workspace, size_t workspace_bytes,
+                  void* stream);
+
+/*
  * sgat_linear -- the fused SGAT W4A4 linear of one quantised layer: optional
  * TAC on the input (Eq. 17), the state-guided transform and A4 quantisation
  * (Eq. 11), and the shared-weight integer GEMM with its dequantisation

@@ -20,6 +20,7 @@ EXPORTED = (
     "starq_version", "starq_last_error", "starq_check_status",
     "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "fp16_gemm_ref", "tac_prepare", "tac_apply",
     "sgat_linear_workspace_size", "sgat_linear", "starq_last_gemm_tile",
+    "tac_calibrate_workspace_size", "tac_calibrate",
 )
 
 
@@ -44,6 +45,10 @@ def _load():
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.tac_prepare.argtypes = [f_p, i, i, i, vp, vp]
     lib.starq_last_gemm_tile.restype = i
+    dbl = ctypes.c_double
+    lib.tac_calibrate_workspace_size.argtypes = [i, i]
+    lib.tac_calibrate_workspace_size.restype = ctypes.c_size_t
+    lib.tac_calibrate.argtypes = [vp, vp, i, i, i, i, dbl, dbl, dbl, dbl, f_p, f_p, vp, ctypes.c_size_t, vp]
     lib.tac_apply.argtypes = [vp, i, i, i, i, f_p, f_p, vp, vp, i, vp]
     lib.fp16_gemm_ref.argtypes = [vp, vp, i, i, i, i, vp, vp]
     lib.sgat_linear_workspace_size.argtypes = [i, i, i]
@@ -161,6 +166,22 @@ def tac_apply(Z, M, d, g, out, Mp=None, stream=None):
     L, C = Z.shape
     _check(lib.tac_apply(_p(Z), dtype_code(Z), L, C, g, _p(M), _p(d), _p(Mp), _p(out), dtype_code(out),
                          _stream(stream)))
+
+
+def tac_calibrate_workspace_size(C, g):
+    return int(lib.tac_calibrate_workspace_size(C, g))
+
+
+def tac_calibrate(Z_fp, Z_q, g, M, d, workspace=None, rho=3e-4, eps=1e-8, eta=0.15, alpha=0.55, stream=None):
+    """Closed-form TAC parameters (App. C) from paired calibration outputs
+    Z_fp, Z_q [N][C] into M [C/g][g][g] and d [C/g][g] (float32)."""
+    _contig(Z_fp, Z_q, M, d, workspace)
+    N, C = Z_fp.shape
+    assert Z_q.shape == Z_fp.shape and Z_q.dtype == Z_fp.dtype
+    if workspace is None:
+        workspace = torch.empty(tac_calibrate_workspace_size(C, g), dtype=torch.uint8, device=Z_fp.device)
+    _check(lib.tac_calibrate(_p(Z_fp), _p(Z_q), dtype_code(Z_fp), N, C, g, rho, eps, eta, alpha, _p(M), _p(d),
+                             _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def sgat_linear_workspace_size(L, K, with_tac):

@@ -6,6 +6,7 @@
 #include <cstring>
 
 #include "common.cuh"
+#include "tac_calib.cuh"
 
 namespace starq {
 
@@ -250,6 +251,35 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
     TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype, st, Mp};
     cudaError_t e = launch_tac(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "tac_apply launch");
+    return STARQ_OK;
+}
+
+size_t tac_calibrate_workspace_size(int C, int g) {
+    if (C <= 0 || g <= 0 || C % g != 0) return 0;
+    return tac_calib_workspace_doubles(C, g) * sizeof(double);
+}
+
+int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, int g, double rho, double eps,
+                  double eta, double alpha, float* M, float* d, void* workspace, size_t workspace_bytes,
+                  void* stream) {
+    if (!Z_fp || !Z_q || !M || !d || !workspace) return fail(STARQ_ERR_ARG, "tac_calibrate: NULL pointer");
+    if (!dtype_ok(z_dtype)) return fail(STARQ_ERR_ARG, "tac_calibrate: unknown dtype %d", z_dtype);
+    if (!(g == 4 || g == 8 || g == 16 || g == 32 || g == 64 || g == 128))
+        return fail(STARQ_ERR_SHAPE, "tac_calibrate: g=%d: supported 4, 8, 16, 32, 64, 128", g);
+    if (C <= 0 || C % g != 0) return fail(STARQ_ERR_SHAPE, "tac_calibrate: C=%d must be a positive multiple of g=%d", C, g);
+    if (N < 1) return fail(STARQ_ERR_SHAPE, "tac_calibrate: N=%d: at least one token", N);
+    if (!(rho >= 0.0) || !(eps > 0.0) || !(eta >= 0.0 && eta <= 1.0) || !(alpha >= 0.0 && alpha <= 1.0))
+        return fail(STARQ_ERR_ARG, "tac_calibrate: need rho >= 0, eps > 0, eta and alpha in [0, 1]");
+    const size_t need = tac_calibrate_workspace_size(C, g);
+    if (workspace_bytes < need) return fail(STARQ_ERR_SHAPE, "tac_calibrate: workspace %zu bytes < %zu", workspace_bytes, need);
+    if (!aligned(Z_fp, 16) || !aligned(Z_q, 16) || !aligned(M, 16) || !aligned(d, 16) || !aligned(workspace, 256))
+        return fail(STARQ_ERR_ALIGN, "tac_calibrate: Z_fp, Z_q, M, d 16-byte and workspace 256-byte alignment");
+    int rc = STARQ_OK;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    CalArgs a{Z_fp, Z_q, z_dtype, N, C, g, rho, eps, eta, alpha, M, d, static_cast<double*>(workspace), st};
+    cudaError_t e = launch_tac_calibrate(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "tac_calibrate launch");
     return STARQ_OK;
 }
 

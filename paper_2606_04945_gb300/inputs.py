@@ -288,3 +288,21 @@ def random_linear(seed, L, K, N, dtype="f16", gates_on=True, tac_g=None, bias=Fa
     b = rng.normal(0, 0.02, N).astype(np.float32) if bias else None
     tac = make_tac(rng, K, tac_g) if tac_g else None
     return LinearCase(f"random_{L}x{K}x{N}", X, dtype, mask, W, xf, bias=b, tac=tac)
+
+
+def tac_calibration_pairs(seed, N, C, g, dtype="f16"):
+    """Paired calibration outputs for TAC (App. C): Z_fp [N][C] with
+    correlated channels inside each g-block (Gaussian tokens through a
+    random g x g mixing near I) and per-channel means, and Z_q = Z_fp plus
+    per-token noise as wide as a 4-bit step (uniform over one step of
+    amax / 7, the width of a 4-bit quantiser's rounding error) and a small
+    Gaussian term. Both are rounded to `dtype` (float16 arrays, or bfloat16
+    values held in float32)."""
+    rng = np.random.default_rng(seed)
+    B = C // g
+    mix = rng.standard_normal((B, g, g)) / np.sqrt(g) + np.eye(g)[None]
+    Z = np.einsum("nbi,bij->nbj", rng.standard_normal((N, B, g)), mix).reshape(N, C)
+    Z = Z + rng.normal(0.0, 0.5, C)[None, :]
+    step = np.abs(Z).max(axis=1, keepdims=True) / 7.0
+    Zq = Z + step * rng.uniform(-0.5, 0.5, Z.shape) + rng.normal(0.0, 0.01, Z.shape)
+    return _store(Z, dtype), _store(Zq, dtype)

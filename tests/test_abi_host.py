@@ -144,3 +144,25 @@ def test_linear_workspace_and_validation(lib):
     rc = lib.lib.sgat_linear(P, 0, 16, 4096, None, None, None, 4096, 4096, 0, 0, P, None, 48, None,
                              P, None, P, None, 256, 4, P, 0, P, 1 << 30, None)
     assert rc == -2
+
+
+def test_tac_calibrate_validation(lib):
+    """Argument checks of tac_calibrate run before any CUDA call."""
+    L = lib.lib
+    ws = lib.tac_calibrate_workspace_size(4096, 128)
+    assert ws == (4096 // 128) * (2 * 128 + 5 * 128 * 128) * 8
+    assert lib.tac_calibrate_workspace_size(100, 16) == 0                          # C % g != 0
+    good = dict(zf=P, zq=P, dt=0, N=64, C=256, g=16, rho=3e-4, eps=1e-8, eta=0.15, alpha=0.55, M=P, d=P,
+                w=ctypes.c_void_p(4096), wb=lib.tac_calibrate_workspace_size(256, 16))
+
+    def call(**kw):
+        a = dict(good, **kw)
+        return L.tac_calibrate(a["zf"], a["zq"], a["dt"], a["N"], a["C"], a["g"], a["rho"], a["eps"], a["eta"],
+                               a["alpha"], a["M"], a["d"], a["w"], a["wb"], None)
+    assert call(zf=None) == -1 and call(M=None) == -1 and call(w=None) == -1
+    assert call(dt=5) == -1
+    assert call(g=12) == -2 and call(g=256) == -2 and call(C=100) == -2 and call(N=0) == -2
+    assert call(eps=0.0) == -1 and call(eta=1.5) == -1 and call(alpha=-0.1) == -1 and call(rho=-1.0) == -1
+    assert call(wb=good["wb"] - 8) == -2
+    assert call(zq=ctypes.c_void_p(4104)) == -3 and call(w=ctypes.c_void_p(4104)) == -3
+    assert "tac_calibrate" in L.starq_last_error().decode()
