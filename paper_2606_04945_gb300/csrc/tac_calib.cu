@@ -10,14 +10,15 @@
 //                      memory and keeps 4 x 4 tiles of the upper triangle of
 //                      S_b in registers, then adds them to the float64
 //                      accumulators in the workspace.
-//   tac_solve_kernel   one CTA per block: mu = s / N, Sigma = S / N - mu mu^T
-//                      (population statistics); lambda_b = rho max(Tr
-//                      Sigma^Q / g, eps); M = (Sigma^FP)^(1/2)
-//                      (Sigma^Q + lambda_b I)^(-1/2) with A^p = Q diag(max(
-//                      lambda_i, 1e-12)^p) Q^T from a symmetric
-//                      eigendecomposition; singular values of M smoothed
-//                      toward their mean by eta; M_final = (1 - alpha) M_sv +
-//                      alpha I; d = mu^FP - M_final mu^Q.
+//   tac_power_kernel   one CTA per block and representation: mu = s / N,
+//                      Sigma = S / N - mu mu^T (population statistics);
+//                      F1 = (Sigma^FP)^(1/2), F2 = (Sigma^Q + lambda_b I)^(-1/2)
+//                      with lambda_b = rho max(Tr Sigma^Q / g, eps) and
+//                      A^p = Q diag(max(lambda_i, 1e-12)^p) Q^T from a
+//                      symmetric eigendecomposition;
+//   tac_final_kernel   one CTA per block: M = F1 F2, its singular values
+//                      smoothed toward their mean by eta, M_final =
+//                      (1 - alpha) M_sv + alpha I, d = mu^FP - M_final mu^Q.
 //
 // The eigendecompositions are parallel cyclic Jacobi: each sweep visits
 // every index pair once in n - 1 steps of n / 2 disjoint rotations (round-
@@ -68,12 +69,18 @@ __global__ void __launch_bounds__(CAL_THREADS) tac_stats_kernel(CalArgs a, int p
     const int t0 = blockIdx.y * per, t1 = min(a.N, t0 + per);
     const Ws w(a.ws, B, g);
     const int T4 = g / 4, ntiles = T4 * (T4 + 1) / 2;
+    // up to STAT_TPT tiles per thread when there are more tiles than
+    // threads; with fewer (small g), `groups` threads share each tile and
+    // split the batch's tokens between them
+    const int groups = ntiles >= CAL_THREADS ? 1 : CAL_THREADS / ntiles;
+    const int grp = groups > 1 ? threadIdx.x / ntiles : 0;
     int ti[STAT_TPT], tj[STAT_TPT];
     double acc[STAT_TPT][16];
     #pragma unroll
     for (int k = 0; k < STAT_TPT; ++k) {
-        int t = threadIdx.x + k * CAL_THREADS;          // column-major upper triangle: t = j (j + 1) / 2 + i
-        int j = 0;
+        int t = groups == 1 ? threadIdx.x + k * CAL_THREADS
+                            : (k == 0 && grp < groups ? threadIdx.x % ntiles : ntiles);
+        int j = 0;                                      // column-major upper triangle: t = j (j + 1) / 2 + i
         while (t >= 0 && (j + 1) * (j + 2) / 2 <= t) ++j;
         ti[k] = t < ntiles ? t - j * (j + 1) / 2 : -1;
         tj[k] = j;
@@ -96,7 +103,7 @@ __global__ void __launch_bounds__(CAL_THREADS) tac_stats_kernel(CalArgs a, int p
             if (ti[k] < 0) continue;
             const double* zi = zs + 4 * ti[k];
             const double* zj = zs + 4 * tj[k];
-            for (int r = 0; r < nt; ++r) {
+            for (int r = grp; r < nt; r += groups) {
                 double x[4], y[4];
                 #pragma unroll
                 for (int u = 0; u < 4; ++u) { x[u] = zi[r * g + u]; y[u] = zj[r * g + u]; }
@@ -313,75 +320,95 @@ __device__ void load_cov(double* A, const double* S, const double* mu, double in
     __syncthreads();
 }
 
-__global__ void __launch_bounds__(CAL_THREADS) tac_solve_kernel(CalArgs a) {
+// Shared-memory layout of the solve kernels: A (g x (g + 1) doubles), five
+// g-vectors and the reduction scratch (doubles), the rotation pairs (ints),
+// then V (g x (g + 1) floats).
+struct SolveSmem {
+    double *A, *mu_fp, *mu_q, *lam, *f, *cs, *red;
+    int* pq;
+    float* V;
+    __device__ SolveSmem(uint8_t* raw, int g) {
+        A = reinterpret_cast<double*>(raw);
+        mu_fp = A + g * (g + 1);
+        mu_q = mu_fp + g;
+        lam = mu_q + g;
+        f = lam + g;
+        cs = f + g;
+        red = cs + g;
+        pq = reinterpret_cast<int*>(red + CAL_THREADS / 32);
+        V = reinterpret_cast<float*>(pq + g);
+    }
+};
+
+// grid (B, 2): the matrix functions of block b, F1 = (Sigma^FP)^(1/2)
+// (blockIdx.y = 0) and F2 = (Sigma^Q + lambda_b I)^(-1/2) (blockIdx.y = 1),
+// each Q diag(max(lambda_i, 1e-12)^p) Q^T.
+__global__ void __launch_bounds__(CAL_THREADS) tac_power_kernel(CalArgs a) {
     extern __shared__ __align__(16) uint8_t cal_smem[];
-    const int g = a.g, B = a.C / g, b = blockIdx.x, ld = g + 1;
-    double* A = reinterpret_cast<double*>(cal_smem);                 // g x (g + 1)
-    double* mu_fp = A + g * ld;
-    double* mu_q = mu_fp + g;
-    double* lam = mu_q + g;
-    double* f = lam + g;
-    double* cs = f + g;                                              // g: cosines, sines
-    double* red = cs + g;                                            // CAL_THREADS / 32
-    int* pq = reinterpret_cast<int*>(red + CAL_THREADS / 32);        // g
-    float* V = reinterpret_cast<float*>(pq + g);                     // g x (g + 1)
+    const int g = a.g, B = a.C / g, b = blockIdx.x, rep = blockIdx.y, ld = g + 1;
+    SolveSmem sm(cal_smem, g);
     const Ws w(a.ws, B, g);
     const double invN = 1.0 / (double)a.N;
-    const double* s_fp = w.s + (size_t)b * g;
-    const double* s_q = w.s + ((size_t)B + b) * g;
-    const double* S_fp = w.S + (size_t)b * g * g;
-    const double* S_q = w.S + ((size_t)B + b) * g * g;
+    const double* sv = w.s + ((size_t)rep * B + b) * g;
+    for (int i = threadIdx.x; i < g; i += CAL_THREADS) sm.mu_fp[i] = sv[i] * invN;
+    __syncthreads();
+    load_cov(sm.A, w.S + ((size_t)rep * B + b) * g * g, sm.mu_fp, invN, 0.0, g);
+    if (rep == 1) {                                   // damping (App. C)
+        double tr = 0.0;
+        for (int i = threadIdx.x; i < g; i += CAL_THREADS) tr += sm.A[i * ld + i];
+        tr = block_sum(tr, sm.red);
+        const double damp = a.rho * fmax(tr / (double)g, a.eps);
+        for (int i = threadIdx.x; i < g; i += CAL_THREADS) sm.A[i * ld + i] += damp;
+        __syncthreads();
+    }
+    jacobi(sm.A, sm.V, sm.lam, sm.cs, sm.pq, sm.red, g);
+    for (int i = threadIdx.x; i < g; i += CAL_THREADS) {
+        const double l = fmax(sm.lam[i], 1e-12);
+        sm.f[i] = rep == 0 ? sqrt(l) : 1.0 / sqrt(l);
+    }
+    __syncthreads();
+    spectral((rep == 0 ? w.F1 : w.F2) + (size_t)b * g * g, sm.V, sm.f, g);
+}
+
+// grid B: M = F1 F2, its SVD M V = U diag(sigma), the smoothed singular
+// values, the identity shrinkage and the bias of block b.
+__global__ void __launch_bounds__(CAL_THREADS) tac_final_kernel(CalArgs a) {
+    extern __shared__ __align__(16) uint8_t cal_smem[];
+    const int g = a.g, B = a.C / g, b = blockIdx.x, ld = g + 1;
+    SolveSmem sm(cal_smem, g);
+    const Ws w(a.ws, B, g);
+    const double invN = 1.0 / (double)a.N;
+    for (int i = threadIdx.x; i < g; i += CAL_THREADS) {
+        sm.mu_fp[i] = w.s[(size_t)b * g + i] * invN;
+        sm.mu_q[i] = w.s[((size_t)B + b) * g + i] * invN;
+    }
     double* F1 = w.F1 + (size_t)b * g * g;
     double* F2 = w.F2 + (size_t)b * g * g;
     double* MM = w.MM + (size_t)b * g * g;
-
-    for (int i = threadIdx.x; i < g; i += CAL_THREADS) {
-        mu_fp[i] = s_fp[i] * invN;
-        mu_q[i] = s_q[i] * invN;
-    }
-    __syncthreads();
-    // (Sigma^FP)^(1/2)
-    load_cov(A, S_fp, mu_fp, invN, 0.0, g);
-    jacobi(A, V, lam, cs, pq, red, g);
-    for (int i = threadIdx.x; i < g; i += CAL_THREADS) f[i] = sqrt(fmax(lam[i], 1e-12));
-    __syncthreads();
-    spectral(F1, V, f, g);
-    // damping and (Sigma^Q + lambda_b I)^(-1/2)
-    load_cov(A, S_q, mu_q, invN, 0.0, g);
-    double tr = 0.0;
-    for (int i = threadIdx.x; i < g; i += CAL_THREADS) tr += A[i * ld + i];
-    tr = block_sum(tr, red);
-    const double damp = a.rho * fmax(tr / (double)g, a.eps);
-    for (int i = threadIdx.x; i < g; i += CAL_THREADS) A[i * ld + i] += damp;
-    __syncthreads();
-    jacobi(A, V, lam, cs, pq, red, g);
-    for (int i = threadIdx.x; i < g; i += CAL_THREADS) f[i] = 1.0 / sqrt(fmax(lam[i], 1e-12));
-    __syncthreads();
-    spectral(F2, V, f, g);
-    // covariance matching, and the SVD of M: M V = U diag(sigma)
+    double* A = sm.A;
     matmul(MM, F1, F2, false, A, g);
     for (int e = threadIdx.x; e < g * g; e += CAL_THREADS) A[(e / g) * ld + e % g] = MM[e];
     __syncthreads();
-    svd_onesided(A, V, cs, pq, red, g);
+    svd_onesided(A, sm.V, sm.cs, sm.pq, sm.red, g);
     double ssum = 0.0;
     for (int j = threadIdx.x; j < g; j += CAL_THREADS) {
         double t = 0.0;
         for (int i = 0; i < g; ++i) t = fma(A[i * ld + j], A[i * ld + j], t);
-        lam[j] = sqrt(t);
-        ssum += lam[j];
+        sm.lam[j] = sqrt(t);
+        ssum += sm.lam[j];
     }
-    const double sbar = block_sum(ssum, red) / (double)g;
+    const double sbar = block_sum(ssum, sm.red) / (double)g;
     // singular values smoothed toward their mean: column j of U diag(sigma)
     // scaled by ((1 - eta) sigma_j + eta sbar) / sigma_j
     for (int j = threadIdx.x; j < g; j += CAL_THREADS)
-        f[j] = lam[j] > 0.0 ? ((1.0 - a.eta) * lam[j] + a.eta * sbar) / lam[j] : 0.0;
+        sm.f[j] = sm.lam[j] > 0.0 ? ((1.0 - a.eta) * sm.lam[j] + a.eta * sbar) / sm.lam[j] : 0.0;
     __syncthreads();
     // M_final = (1 - alpha) U diag(sigma') V^T + alpha I, and d
     float* Mo = a.M + (size_t)b * g * g;
     for (int e = threadIdx.x; e < g * g; e += CAL_THREADS) {
         const int i = e / g, k = e - i * g;
         double t = 0.0;
-        for (int j = 0; j < g; ++j) t = fma(A[i * ld + j] * f[j], (double)V[k * ld + j], t);
+        for (int j = 0; j < g; ++j) t = fma(A[i * ld + j] * sm.f[j], (double)sm.V[k * ld + j], t);
         const double mf = (1.0 - a.alpha) * t + (i == k ? a.alpha : 0.0);
         F1[e] = mf;
         Mo[e] = (float)mf;
@@ -389,8 +416,8 @@ __global__ void __launch_bounds__(CAL_THREADS) tac_solve_kernel(CalArgs a) {
     __syncthreads();
     for (int i = threadIdx.x; i < g; i += CAL_THREADS) {
         double t = 0.0;
-        for (int j = 0; j < g; ++j) t = fma(F1[(size_t)i * g + j], mu_q[j], t);
-        a.d[(size_t)b * g + i] = (float)(mu_fp[i] - t);
+        for (int j = 0; j < g; ++j) t = fma(F1[(size_t)i * g + j], sm.mu_q[j], t);
+        a.d[(size_t)b * g + i] = (float)(sm.mu_fp[i] - t);
     }
 }
 
@@ -432,12 +459,17 @@ cudaError_t launch_tac_calibrate(const CalArgs& a, cudaStream_t stream) {
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev < 64 && !attr_set[dev]) {
-        e = cudaFuncSetAttribute(tac_solve_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(tac_power_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)solve_smem(CAL_MAX_G));
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(tac_final_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)solve_smem(CAL_MAX_G));
         if (e != cudaSuccess) return e;
         attr_set[dev] = true;
     }
-    tac_solve_kernel<<<B, CAL_THREADS, smem, stream>>>(a);
+    tac_power_kernel<<<dim3(B, 2), CAL_THREADS, smem, stream>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    tac_final_kernel<<<B, CAL_THREADS, smem, stream>>>(a);
     return cudaGetLastError();
 }
 
