@@ -282,6 +282,29 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 int bits, void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * sgat_linear_swiglu -- sgat_linear for the gate and up projections of a
+ * SwiGLU MLP, with the activation fused into the GEMM's epilogue. Gate and
+ * up share one quantised input (Sec. 3.2: every quantised linear, the MLP's
+ * included, runs through the SGAT transform). The activation is the MLP's
+ * own, silu(gate) * up, not part of the paper's method.
+ *
+ *   Wq, We, s_w, bias: the 2F output channels with gate and up rows
+ *     interleaved in groups of 16: rows 32 k .. 32 k + 15 are gate channels
+ *     16 k .. 16 k + 15, rows 32 k + 16 .. 32 k + 31 the matching up
+ *     channels. Prepare them from the weight rows in that order.
+ *   N = 2F, N % 32 == 0; We is required.
+ *   H [L][F] out, h_dtype F16 or BF16:
+ *     H[i][f] = silu(y_gate) * y_up rounded once to h_dtype, y = the float32
+ *     dequantised outputs, silu(x) = x / (1 + exp(-x)).
+ * Other arguments and the workspace are exactly sgat_linear's.
+ */
+int sgat_linear_swiglu(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                       const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
+                       const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N,
+                       int bits, void* H, int h_dtype, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * sgat_linear_noalloc -- sgat_linear for callers that cannot allocate device
  * memory. (The paper has no counterpart: this is a deployment convenience.)
  *

@@ -20,7 +20,7 @@ EXPORTED = (
     "starq_version", "starq_last_error", "starq_check_status",
     "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "fp16_gemm_ref", "tac_prepare", "tac_apply",
     "sgat_linear_workspace_size", "sgat_linear", "starq_last_gemm_tile",
-    "tac_calibrate_workspace_size", "tac_calibrate",
+    "tac_calibrate_workspace_size", "tac_calibrate", "sgat_linear_swiglu",
 )
 
 
@@ -55,6 +55,7 @@ def _load():
     lib.sgat_linear_workspace_size.restype = ctypes.c_size_t
     lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
                                 u8p, u8p, f_p, f_p, i, i, vp, i, vp, ctypes.c_size_t, vp]
+    lib.sgat_linear_swiglu.argtypes = lib.sgat_linear.argtypes
     if hasattr(lib, "sgat_linear_noalloc"):
         lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
                                             u8p, u8p, f_p, f_p, i, i, vp, i, vp]
@@ -197,6 +198,28 @@ def sgat_linear(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, workspace, bi
                            d_u, _p(tac_M), _p(tac_d), tac_g, _p(tac_Mp), _p(Wq), _p(We), _p(s_w), _p(bias), N, bits,
                            _p(Y), dtype_code(Y), _p(workspace), workspace.numel() * workspace.element_size(),
                            _stream(stream)))
+
+
+def swiglu_row_order(F, device="cpu"):
+    """Row order of a gate+up weight [2F][K] (gate rows 0..F-1, up rows
+    F..2F-1) for sgat_linear_swiglu: groups of 16 gate rows, each followed by
+    the matching 16 up rows."""
+    assert F % 16 == 0
+    g = torch.arange(F, device=device).view(-1, 16)
+    return torch.stack([g, g + F], dim=1).reshape(-1)
+
+
+def sgat_linear_swiglu(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, H, workspace, bias=None,
+                       tac_M=None, tac_d=None, tac_g=0, bits=4, We=None, tac_Mp=None, stream=None):
+    """sgat_linear with silu(gate) * up fused into the GEMM epilogue: the
+    weights' rows in swiglu_row_order, H [L][N / 2]."""
+    _contig(X, mask, a_m, a_u, Wq, We, s_w, H, workspace, bias, tac_M, tac_d, tac_Mp)
+    L, K = X.shape
+    N = _weight_shape(Wq, We)[0]
+    _check(lib.sgat_linear_swiglu(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh, d_m,
+                                  d_u, _p(tac_M), _p(tac_d), tac_g, _p(tac_Mp), _p(Wq), _p(We), _p(s_w), _p(bias),
+                                  N, bits, _p(H), dtype_code(H), _p(workspace),
+                                  workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 NOALLOC_SCRATCH_BYTES = 32 << 20

@@ -290,11 +290,14 @@ size_t sgat_linear_workspace_size(int L, int K, int with_tac) {
     return n;
 }
 
-int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
-                const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
-                const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
-                void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
+}  // extern "C"
+
+namespace {
+int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                     const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                     const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
+                     const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
+                     void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream, int swiglu) {
     if ((!Wq && !We) || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear: NULL Wq/We or s_w");
     if (L > 0 && (!X || !Y || !workspace)) return fail(STARQ_ERR_ARG, "sgat_linear: NULL X, Y or workspace");
     if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear: unknown dtype");
@@ -336,8 +339,35 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
     // the GEMM's predecessor is the quantiser launched above, which waits for
     // everything before it and does not write the weights
     g.weights_ready = 1;
+    g.swiglu = swiglu;
     if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: gemm launch");
     return STARQ_OK;
+}
+}  // namespace
+
+extern "C" {
+
+int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
+                const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
+                void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
+    return sgat_linear_impl(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g, tac_Mp, Wq,
+                            We, s_w, bias, N, bits, Y, y_dtype, workspace, workspace_bytes, stream, 0);
+}
+
+int sgat_linear_swiglu(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
+                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
+                       const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
+                       const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
+                       void* H, int h_dtype, void* workspace, size_t workspace_bytes, void* stream) {
+    if (!We) return fail(STARQ_ERR_ARG, "sgat_linear_swiglu: needs the E4M3 weights We");
+    if (h_dtype != STARQ_F16 && h_dtype != STARQ_BF16)
+        return fail(STARQ_ERR_ARG, "sgat_linear_swiglu: output dtype must be F16 or BF16");
+    if (N < 32 || N % 32 != 0)
+        return fail(STARQ_ERR_SHAPE, "sgat_linear_swiglu: N=%d: gate and up rows interleaved by 16, N %% 32 == 0", N);
+    return sgat_linear_impl(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g, tac_Mp, Wq,
+                            We, s_w, bias, N, bits, H, h_dtype, workspace, workspace_bytes, stream, 1);
 }
 
 }  // extern "C"

@@ -49,6 +49,9 @@ struct GemmArgs {
     // launched writes the weights: their first tiles are fetched before
     // the wait for the previous kernel (programmatic launch).
     int weights_ready = 0;
+    // Epilogue silu(gate) * up over weight rows interleaved in groups of 16
+    // (Xe + We path, 16-bit Y of [L][N / 2]).
+    int swiglu = 0;
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
 // Tile of the calling thread's last TMA pair GEMM launch (BN * 10 + cluster

@@ -111,11 +111,30 @@ __device__ __forceinline__ void stage_row16(uint32_t box, int row, const float (
         st_shared_v4(box + row * 64 + 16 * (g ^ ((row >> 1) & 3)), w[0], w[1], w[2], w[3]);
     }
 }
+// Row `row` (16 values) of a 32 x 16 box of a 16-bit type: 32-byte rows
+// with the 32-byte swizzle (16-byte group g at g ^ ((row >> 2) & 1)), which
+// keeps the 32 lanes' stores free of bank conflicts.
+template <typename T2, typename Cvt>
+__device__ __forceinline__ void stage_row16_half(uint32_t box, int row, const float (&h)[16], Cvt cvt) {
+    #pragma unroll
+    for (int g = 0; g < 2; ++g) {
+        uint32_t w[4];
+        #pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            T2 v = cvt(h[8 * g + 2 * j], h[8 * g + 2 * j + 1]);
+            w[j] = *reinterpret_cast<uint32_t*>(&v);
+        }
+        st_shared_v4(box + row * 32 + 16 * (g ^ ((row >> 2) & 1)), w[0], w[1], w[2], w[3]);
+    }
+}
 template <> struct Out<__half> {
     static constexpr CUtensorMapDataType TMAP_TYPE = CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
     static constexpr CUtensorMapSwizzle TMAP_SWIZZLE = CU_TENSOR_MAP_SWIZZLE_64B;
     static __device__ __forceinline__ void stage32(uint32_t box, int row, const float (&y)[32]) {
         stage_row16<__half2>(box, row, y, [](float a, float b) { return __floats2half2_rn(a, b); });
+    }
+    static __device__ __forceinline__ void stage16(uint32_t box, int row, const float (&h)[16]) {
+        stage_row16_half<__half2>(box, row, h, [](float a, float b) { return __floats2half2_rn(a, b); });
     }
     static __device__ __forceinline__ void store32(__half* p, const float (&y)[32]) {
         uint4* q = reinterpret_cast<uint4*>(p);
@@ -137,6 +156,9 @@ template <> struct Out<__nv_bfloat16> {
     static __device__ __forceinline__ void stage32(uint32_t box, int row, const float (&y)[32]) {
         stage_row16<__nv_bfloat162>(box, row, y, [](float a, float b) { return __floats2bfloat162_rn(a, b); });
     }
+    static __device__ __forceinline__ void stage16(uint32_t box, int row, const float (&h)[16]) {
+        stage_row16_half<__nv_bfloat162>(box, row, h, [](float a, float b) { return __floats2bfloat162_rn(a, b); });
+    }
     static __device__ __forceinline__ void store32(__nv_bfloat16* p, const float (&y)[32]) {
         uint4* q = reinterpret_cast<uint4*>(p);
         #pragma unroll
@@ -154,6 +176,7 @@ template <> struct Out<__nv_bfloat16> {
 template <> struct Out<float> {
     static constexpr CUtensorMapDataType TMAP_TYPE = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
     static constexpr CUtensorMapSwizzle TMAP_SWIZZLE = CU_TENSOR_MAP_SWIZZLE_128B;
+    static __device__ __forceinline__ void stage16(uint32_t, int, const float (&)[16]) {}   // 16-bit outputs only
     static __device__ __forceinline__ void stage32(uint32_t box, int row, const float (&y)[32]) {
         #pragma unroll
         for (int g = 0; g < 8; ++g)
@@ -765,7 +788,7 @@ bool encode_operand_tmap(CUtensorMap* m, const void* ptr, CUtensorMapDataType ty
 
 // Tensor map of the row-major output Y [rows][cols] with 32 x 32 boxes.
 bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t elem, uint64_t rows,
-                     uint64_t cols, CUtensorMapSwizzle swz) {
+                     uint64_t cols, CUtensorMapSwizzle swz, uint32_t box_cols = 32) {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (fn == nullptr) {
         cudaDriverEntryPointQueryResult q;
@@ -777,7 +800,7 @@ bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t
     }
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {cols * elem};
-    const cuuint32_t box[2] = {32, 32};
+    const cuuint32_t box[2] = {box_cols, 32};
     const cuuint32_t estr[2] = {1, 1};
     return fn(m, type, 2, ptr, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
               CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -864,7 +887,11 @@ long long tma_round_cost(int L, int N, int BN, int CL, int clusters) {
     return rounds * stage2;
 }
 
-template <typename TOut, int CL, int OPK, int BN>
+// SWIGLU: the weight rows come interleaved in groups of 16 (gate rows
+// 16 k .. 16 k + 15, then the matching up rows), so every 32-column chunk
+// of the accumulator holds 16 gate and 16 up channels; the epilogue writes
+// silu(gate) * up, rounded once, to column nc / 2 of an [L][N / 2] output.
+template <typename TOut, int CL, int OPK, int BN, bool SWIGLU = false>
 __global__ void __launch_bounds__(tmak::THREADS, 1)
 w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
                           const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y) {
@@ -1117,11 +1144,18 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                     }
                     __syncwarp();
                 }
-                Out<TOut>::stage32(box, lane, y);
+                if (SWIGLU) {
+                    float h[16];
+                    #pragma unroll
+                    for (int t = 0; t < 16; ++t) h[t] = y[t] / (1.f + expf(-y[t])) * y[16 + t];
+                    Out<TOut>::stage16(box, lane, h);
+                } else {
+                    Out<TOut>::stage32(box, lane, y);
+                }
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) {
-                    tma_store_2d(&tmap_y, nc, m0 + quarter * 32, box);
+                    tma_store_2d(&tmap_y, SWIGLU ? nc / 2 : nc, m0 + quarter * 32, box);
                     bulk_commit();
                 }
                 ++nbox;
@@ -1158,10 +1192,10 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
 
 // Clusters of this instantiation resident at once on the current device
 // (queried once per device; also sets the kernel's shared-memory limit).
-template <typename TOut, int CL, int OPK, int BN>
+template <typename TOut, int CL, int OPK, int BN, bool SW>
 cudaError_t tma_max_clusters(int* clusters) {
     constexpr size_t SMEM_BYTES = tmak::Cfg<sizeof(TOut), BN>::SMEM_BYTES;
-    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN>;
+    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN, SW>;
     static int max_clusters[64] = {0};
     int dev = 0;
     cudaGetDevice(&dev);
@@ -1189,7 +1223,7 @@ cudaError_t tma_max_clusters(int* clusters) {
     return cudaSuccess;
 }
 
-template <typename TOut, int CL, int OPK, int BN>
+template <typename TOut, int CL, int OPK, int BN, bool SW>
 cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) {
     constexpr int BM = tmak::BM, BN_CTA = tmak::Tile<BN>::BN_CTA, BK = tmak::BK;
     constexpr int ELEM = OPK == 0 ? 1 : 2;
@@ -1209,13 +1243,15 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) 
     const CUtensorMapDataType opt = OPK == 0 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
     if (!encode_operand_tmap(&ta, a.Xe, opt, ELEM, (uint64_t)a.L, (uint64_t)a.K, CL == 2 ? BM : BM / 2, BK / ELEM) ||
         !encode_operand_tmap(&tb, a.We, opt, ELEM, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK / ELEM) ||
-        !encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N,
-                         Out<TOut>::TMAP_SWIZZLE))
+        !(SW ? encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N / 2,
+                               CU_TENSOR_MAP_SWIZZLE_32B, 16)
+             : encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N,
+                               Out<TOut>::TMAP_SWIZZLE)))
         return cudaErrorInvalidValue;
     const int num_tiles = tma_tiles(a.L, a.N, BN, CL);
     if (num_tiles < clusters) clusters = num_tiles;
     cfg.gridDim = dim3(CL * clusters);
-    return cudaLaunchKernelEx(&cfg, w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN>, a, ta, tb, ty);
+    return cudaLaunchKernelEx(&cfg, w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN, SW>, a, ta, tb, ty);
 }
 
 // Tile shape per problem. A stage's steady state is bound by shared memory:
@@ -1227,21 +1263,32 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) 
 // activation tile when there are at least two channel tiles) and 224-wide
 // tiles on single pairs, whose tile counts fill the 76 pairs of the LLaDA
 // projections better; the cheaper estimate wins, ties keep 256.
-template <typename TOut, int OPK = 0>
-cudaError_t launch_tma_typed(const GemmArgs& a, cudaStream_t stream) {
+template <typename TOut, int OPK, bool SW>
+cudaError_t launch_tma_shape(const GemmArgs& a, cudaStream_t stream) {
     const bool quad = (a.N + 255) / 256 >= 2;
     int c256 = 0, c224 = 0;
-    cudaError_t e = quad ? tma_max_clusters<TOut, 4, OPK, 256>(&c256) : tma_max_clusters<TOut, 2, OPK, 256>(&c256);
+    cudaError_t e = quad ? tma_max_clusters<TOut, 4, OPK, 256, SW>(&c256)
+                         : tma_max_clusters<TOut, 2, OPK, 256, SW>(&c256);
     if (e != cudaSuccess) return e;
-    if ((e = tma_max_clusters<TOut, 2, OPK, 224>(&c224)) != cudaSuccess) return e;
+    if ((e = tma_max_clusters<TOut, 2, OPK, 224, SW>(&c224)) != cudaSuccess) return e;
     const long long t256 = tma_round_cost(a.L, a.N, 256, quad ? 4 : 2, c256);
     const long long t224 = tma_round_cost(a.L, a.N, 224, 2, c224);
     if (t224 < t256) {
         g_last_tile = 224 * 10 + 2;
-        return launch_tma_cl<TOut, 2, OPK, 224>(a, stream, c224);
+        return launch_tma_cl<TOut, 2, OPK, 224, SW>(a, stream, c224);
     }
     g_last_tile = 256 * 10 + (quad ? 4 : 2);
-    return quad ? launch_tma_cl<TOut, 4, OPK, 256>(a, stream, c256) : launch_tma_cl<TOut, 2, OPK, 256>(a, stream, c256);
+    return quad ? launch_tma_cl<TOut, 4, OPK, 256, SW>(a, stream, c256)
+                : launch_tma_cl<TOut, 2, OPK, 256, SW>(a, stream, c256);
+}
+
+template <typename TOut, int OPK = 0>
+cudaError_t launch_tma_typed(const GemmArgs& a, cudaStream_t stream) {
+    if constexpr (OPK == 0 && sizeof(TOut) == 2) {
+        if (a.swiglu) return launch_tma_shape<TOut, OPK, true>(a, stream);
+    }
+    if (a.swiglu) return cudaErrorInvalidValue;
+    return launch_tma_shape<TOut, OPK, false>(a, stream);
 }
 
 // Packed int4 -> E4M3: each thread turns 16 packed bytes into 32 E4M3 bytes.

@@ -16,8 +16,10 @@ outputs. Per block:
     x = x + SGAT-W4A4(silu(g) u)            down 12288 -> 4096
 
 Every linear is one `sgat_linear` call of the C ABI with the token's mask
-bit selecting its transform. RMSNorm, RoPE, attention, SwiGLU and the
-residuals are glue (torch ops on the GPU), not part of the quantised path.
+bit selecting its transform; the gate+up projection is `sgat_linear_swiglu`,
+which applies silu(g) u in the GEMM epilogue. RMSNorm, RoPE, attention and
+the residuals are glue (torch ops on the GPU), not part of the quantised
+path; the 16-bit baseline applies SwiGLU as glue too.
 The same stack with 16-bit GEMMs (`fp16_gemm_ref`, no quantisation, no
 TAC) is the unquantised baseline for the per-step output drift.
 
@@ -71,11 +73,14 @@ class QLinear:
     W4A4 form (packed int4 codes, E4M3 copy, per-channel scales), the SGAT
     transforms, optional TAC, and a workspace."""
 
-    def __init__(self, W16, L, tac=None):
+    def __init__(self, W16, L, tac=None, swiglu=False):
         self.W16 = W16
         self.N, self.K = W16.shape
         self.L = L
         self.tac = tac
+        # gate+up of the MLP: the W4A4 form keeps the rows in
+        # swiglu_row_order and writes silu(gate) * up [L][N / 2]
+        self.swiglu = swiglu
         self.sgat = None
         self.tac_M = self.tac_d = self.tac_Mp = None
         if tac is not None:
@@ -99,7 +104,8 @@ class QLinear:
         self.a_m, self.a_u = t(xf.a_m), t(xf.a_u)
         self.Wq = torch.empty(self.N, self.K // 2, dtype=torch.uint8, device=dev)
         self.s_w = torch.empty(self.N, dtype=torch.float32, device=dev)
-        abi.sgat_prepare_weight(self.W16, t(xf.inv_a_w), xf.hb, self.Wq, self.s_w)
+        W = self.W16[abi.swiglu_row_order(self.N // 2, dev)] if self.swiglu else self.W16
+        abi.sgat_prepare_weight(W, t(xf.inv_a_w), xf.hb, self.Wq, self.s_w)
         self.We = torch.empty(self.N, self.K, dtype=torch.uint8, device=dev)
         abi.w4_unpack_e4m3(self.Wq, self.We)
         self.workspace = torch.empty(abi.sgat_linear_workspace_size(self.L, self.K, self.tac is not None),
@@ -107,6 +113,10 @@ class QLinear:
 
     def w4a4(self, X, mask, Y):
         xf = self.sgat
+        if self.swiglu:
+            abi.sgat_linear_swiglu(X, mask, self.a_m, self.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, self.Wq, self.s_w,
+                                   Y, self.workspace, We=self.We)
+            return
         abi.sgat_linear(X, mask, self.a_m, self.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, self.Wq, self.s_w, Y,
                         self.workspace, tac_M=self.tac_M, tac_d=self.tac_d,
                         tac_g=self.tac.g if self.tac is not None else 0, We=self.We, tac_Mp=self.tac_Mp)
@@ -130,7 +140,7 @@ class DenoiseStack:
             self.blocks.append(dict(
                 qkv=QLinear(w(3 * c.hidden, c.hidden), c.seq),
                 o=QLinear(w(c.hidden, c.hidden), c.seq, tac=inputs.make_tac(rng, c.hidden, c.tac_block)),
-                gu=QLinear(w(2 * c.ffn, c.hidden), c.seq),
+                gu=QLinear(w(2 * c.ffn, c.hidden), c.seq, swiglu=True),
                 down=QLinear(w(c.hidden, c.ffn), c.seq)))
         self.cos, self.sin = rope_tables(c.seq, c.hidden // c.heads, device)
         # denoising trajectory: prompt tokens, then masked positions unmasked
@@ -186,9 +196,12 @@ class DenoiseStack:
             self._lin(blk["o"], b["attn"], mask_d, b["o"], quantised, hook, li, "o")
             x = x + b["o"]
             h = rms_norm(x)
-            self._lin(blk["gu"], h, mask_d, b["gu"], quantised, hook, li, "gu")
-            gt, up = b["gu"][:, : c.ffn], b["gu"][:, c.ffn:]
-            b["act"].copy_((torch.nn.functional.silu(gt.float()) * up.float()).half())
+            if quantised:                                 # silu(gate) * up in the GEMM epilogue
+                self._lin(blk["gu"], h, mask_d, b["act"], True, hook, li, "gu")
+            else:
+                blk["gu"].fp16(h, b["gu"])
+                gt, up = b["gu"][:, : c.ffn], b["gu"][:, c.ffn:]
+                b["act"].copy_((torch.nn.functional.silu(gt.float()) * up.float()).half())
             self._lin(blk["down"], b["act"], mask_d, b["down"], quantised, hook, li, "down")
             x = x + b["down"]
         return x

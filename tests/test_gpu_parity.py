@@ -412,6 +412,38 @@ def test_dream_block_linears(abi):
         run_linear_case(abi, case, check_rows=rows)
 
 
+@pytest.mark.parametrize("L,K,F,dtype,bias", [(300, 512, 256, "f16", False), (77, 1024, 512, "bf16", True),
+                                            (1024, 4096, 12288, "f16", False)])
+def test_sgat_linear_swiglu(abi, L, K, F, dtype, bias):
+    """Gate and up projections of a SwiGLU MLP with silu(gate) * up in the
+    GEMM epilogue: the weight rows interleaved by swiglu_row_order, the
+    output [L][F] against silu and the product taken in float64 from the
+    oracle's dequantised gate and up outputs (the same float32 values the
+    epilogue starts from). The last shape is the LLaDA-8B gate+up
+    projection."""
+    case = inputs.random_linear(L * 5 + K + F, L, K, 2 * F, dtype=dtype, bias=bias)
+    xf = case.xf
+    dt = H.torch_dtype(dtype)
+    perm = abi.swiglu_row_order(F).numpy()
+    Wp = case.W[perm]
+    bp = case.bias[perm] if bias else None
+    Wq = torch.empty(2 * F, K // 2, dtype=torch.uint8, device="cuda")
+    s_w = torch.empty(2 * F, dtype=torch.float32, device="cuda")
+    abi.sgat_prepare_weight(H.dev(Wp, dt), H.dev(xf.inv_a_w), xf.hb, Wq, s_w)
+    We = unpacked_weight(abi, Wq)
+    ws = torch.empty(abi.sgat_linear_workspace_size(L, K, False), dtype=torch.uint8, device="cuda")
+    Hout = torch.full((L, F), float("nan"), dtype=dt, device="cuda")
+    abi.sgat_linear_swiglu(H.dev(case.X, dt), H.dev(case.mask), H.dev(xf.a_m), H.dev(xf.a_u), xf.hb, xf.d_sh,
+                           xf.d_m, xf.d_u, Wq, s_w, Hout, ws, bias=None if bp is None else H.dev(bp), We=We)
+    abi.check_status()
+    qw, sw = osg.prepare_weight(Wp, xf.inv_a_w, xf.hb, 4)
+    Y_ref = osg.sgat_linear(case.X, case.mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, qw, sw, bp, 4)[0]
+    Yr = Y_ref.reshape(L, F // 16, 2, 16)
+    gate, up = Yr[:, :, 0, :].reshape(L, F), Yr[:, :, 1, :].reshape(L, F)
+    h_ref = gate / (1.0 + np.exp(-gate)) * up
+    H.assert_output_close(H.host(Hout), h_ref, dtype, what="silu(gate) * up")
+
+
 @pytest.mark.parametrize("L,K,N,dtype,tac_g,bias", [(1, 128, 32, "f16", None, False),
                                                     (77, 512, 320, "bf16", 16, True),
                                                     (129, 1024, 256, "f16", 128, False),

@@ -2,7 +2,8 @@
 
 Hidden 4096, FFN 12288, 32 heads; 1024 positions, the last 256 generated,
 4 unmasked per step; every linear is SGAT W4A4 (the O projection with TAC,
-128 x 128 per head); RMSNorm, RoPE, attention and SwiGLU are glue. At steps
+128 x 128 per head; the gate+up projection with silu(gate) * up in its
+epilogue); RMSNorm, RoPE and attention are glue. At steps
 0, 1, 31 and 63 every linear's activation codes, scales and E4M3 bytes are
 compared bit-exactly with the oracle's quantisation of the GPU's own input
 (teacher forcing; TAC within tolerance); at step 0 every linear's outputs
@@ -60,6 +61,10 @@ def test_denoise_stack(abi):
             if key not in wcodes:
                 wcodes[key] = H.unpack(lin.Wq)
             ref = osg.dequant(osg.int_gemm(codes, wcodes[key]), s, lin.s_w.cpu().numpy(), None)
+            if lin.swiglu:                                # rows interleaved by 16: silu(gate) * up
+                r = ref.reshape(len(rows), -1, 2, 16)
+                gate, up = r[:, :, 0, :].reshape(len(rows), -1), r[:, :, 1, :].reshape(len(rows), -1)
+                ref = gate / (1.0 + np.exp(-gate)) * up
             H.assert_output_close(H.host(Y)[rows], ref, "f16", what=f"layer {li} {name}")
         checked.append((step, li, name))
 
