@@ -16,6 +16,9 @@ Every function is a plain, slow restatement of the paper:
 * ``tac``: Sec. 3.3 (Eq. 17) and App. C block-wise affine compensation, and
   the App. C closed-form calibration (statistics, damping, matrix powers,
   singular-value smoothing, identity shrinkage, bias).
+* ``attention``: the quantised softmax-value product of Sec. 3.3 (Z_hat,
+  8-bit per-row P and 4-bit per-channel V: readings, the paper fixes
+  neither) and TAC on it, one block per head.
 
 Floating point: the transform and the quantiser decision run in float32, the
 precision the CUDA kernels take the integer decision in (a quantised code is
@@ -29,4 +32,4 @@ closed forms, brute force on tiny inputs, hand-worked fixtures in
 "parity unpinned".
 """
 
-from . import sgat, tac  # noqa: F401
+from . import attention, sgat, tac  # noqa: F401

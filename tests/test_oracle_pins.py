@@ -430,3 +430,101 @@ def test_tac_singular_value_smoothing_formula():
         s0 = np.linalg.svd(M0[0], compute_uv=False)
         se = np.linalg.svd(Me[0], compute_uv=False)
         assert np.allclose(se, (1 - eta) * s0 + eta * s0.mean(), rtol=1e-10)
+
+
+# ---------------------------------------------------------------------------
+# The quantised softmax-value product feeding TAC (oracle/attention.py)
+# ---------------------------------------------------------------------------
+
+def test_attention_p_codes_definition():
+    """P's 8-bit codes: each row's largest probability 1 / l maps to 255;
+    uniform scores give 255 everywhere and l = keys; every code is the
+    nearest integer to 255 exp(s - m) by brute force over 0..255."""
+    from oracle import attention as oatt
+    c, l = oatt.p_codes(np.zeros((2, 7)))
+    assert np.all(c == 255) and np.allclose(l, 7.0)
+    rng = np.random.default_rng(3)
+    S = rng.normal(0, 2, (5, 9))
+    c, l = oatt.p_codes(S)
+    assert np.all(c.max(axis=1) == 255)
+    e = np.exp(S - S.max(axis=1, keepdims=True))
+    assert np.allclose(l, e.sum(axis=1))
+    brute = np.argmin(np.abs(255.0 * e[..., None] - np.arange(256)[None, None, :]), axis=-1)
+    assert np.array_equal(c, brute)
+    assert c.min() >= 0 and c.max() <= 255
+
+
+def test_attention_v_codes_per_channel():
+    """V's 4-bit codes run along each channel (column): every column with a
+    non-zero entry reaches |code| 7, and codes are the brute-force nearest
+    multiples of the column's step t = amax / 7."""
+    from oracle import attention as oatt
+    rng = np.random.default_rng(4)
+    V = rng.normal(0, 1, (11, 6)).astype(np.float32)
+    V[:, 2] *= 100.0                                   # one loud channel must not affect the others
+    q, t = oatt.v_codes(V)
+    assert q.shape == V.shape and t.shape == (6,)
+    assert np.all(np.abs(q).max(axis=0) == 7)
+    np.testing.assert_allclose(t, np.abs(V).max(axis=0) / 7, rtol=1e-6)
+    brute = np.argmin(np.abs(V[..., None] / t[None, :, None] - np.arange(-7, 8)[None, None, :]), axis=-1) - 7
+    assert np.array_equal(q, brute)
+
+
+def test_attention_brute_force_tiny():
+    """Z_hat against explicit loops over heads, queries, keys and channels
+    (scores scaled by 1 / sqrt(d), codes per row / per channel)."""
+    from oracle import attention as oatt
+    rng = np.random.default_rng(5)
+    L, H, d = 3, 2, 4
+    Q, K, V = (rng.normal(0, 1, (L, H * d)).astype(np.float32) for _ in range(3))
+    Z, codes, ls, vq, t, acc = oatt.quantised_attention(Q, K, V, H, d)
+    for h in range(H):
+        for i in range(L):
+            s = [sum(float(Q[i, h * d + k]) * float(K[j, h * d + k]) for k in range(d)) / math.sqrt(d)
+                 for j in range(L)]
+            m = max(s)
+            e = [math.exp(x - m) for x in s]
+            lsum = sum(e)
+            cs = [round(255.0 * x) for x in e]          # Python's round is half to even
+            assert cs == list(codes[h, i]) and abs(lsum - ls[h, i]) < 1e-12
+            for c in range(d):
+                a = sum(cs[j] * int(vq[j, h * d + c]) for j in range(L))
+                assert a == acc[h, i, c]
+                want = a / (255.0 * lsum) * float(t[h * d + c])
+                assert abs(want - Z[i, h * d + c]) <= 1e-12 * max(1.0, abs(want))
+
+
+def test_attention_uniform_and_error_bound():
+    """Q = 0 makes attention uniform: Z_hat is the mean of the dequantised
+    V over keys exactly. For general inputs |Z_hat - softmax(s) V| stays
+    within the rounding bound of 8-bit P and 4-bit V."""
+    from oracle import attention as oatt
+    rng = np.random.default_rng(6)
+    L, H, d = 40, 2, 8
+    K = rng.normal(0, 1, (L, H * d)).astype(np.float32)
+    V = rng.normal(0, 1, (L, H * d)).astype(np.float32)
+    Z, _, ls, vq, t, _ = oatt.quantised_attention(np.zeros_like(K), K, V, H, d)
+    assert np.allclose(Z, (vq * t[None, :]).mean(axis=0)[None, :], rtol=1e-12, atol=1e-15)
+    assert np.allclose(ls, L)
+    Q = rng.normal(0, 1, (L, H * d)).astype(np.float32)
+    Z, _, ls, _, t, _ = oatt.quantised_attention(Q, K, V, H, d)
+    for h in range(H):
+        ch = slice(h * d, (h + 1) * d)
+        S = oatt.scores(Q[:, ch], K[:, ch], d)
+        P = np.exp(S - S.max(axis=1, keepdims=True))
+        P /= P.sum(axis=1, keepdims=True)
+        exact = P @ V[:, ch].astype(np.float64)
+        vmax = np.abs(V[:, ch]).max(axis=0)
+        bound = (t[ch][None, :] / 2) * (1 + L / (510 * ls[h][:, None])) + L * vmax[None, :] / (510 * ls[h][:, None])
+        assert np.all(np.abs(Z[:, ch] - exact) <= bound + 1e-12)
+
+
+def test_attention_tac_identity():
+    """TAC with M = I and d = 0 returns Z_hat unchanged (P6 on this path)."""
+    from oracle import attention as oatt
+    rng = np.random.default_rng(7)
+    L, H, d = 16, 2, 8
+    Q, K, V = (rng.normal(0, 1, (L, H * d)).astype(np.float32) for _ in range(3))
+    M = np.broadcast_to(np.eye(d), (H, d, d))
+    Zt, Z = oatt.attention_tac(Q, K, V, M, np.zeros((H, d)), H, d)
+    assert np.array_equal(Zt, Z)
