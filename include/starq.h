@@ -215,6 +215,46 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
               const void* Mp, void* out, int out_dtype, void* stream);
 
 /*
+ * attention_pv_tac -- the quantised softmax-value product of an attention
+ * layer with TAC fused into its dequantisation epilogue (Sec. 3.3: Z_hat is
+ * the quantised counterpart of Softmax(Q K^T / sqrt(d_h)) V, compensated
+ * block-wise before the output projection; App. C places TAC right after
+ * the softmax-value multiplication).
+ *
+ * The paper fixes neither the bit widths nor the granularity of that
+ * multiplication. The readings:
+ *   P per query row, unsigned 8-bit: c_ij = rne(255 exp(s_ij - m_i)), scale
+ *     1 / (255 l_i), with s = q . k / sqrt(128), m_i = max_j s_ij and
+ *     l_i = sum_j exp(s_ij - m_i). The row's largest probability maps to 255;
+ *   V per channel, signed 4-bit: the activation quantiser along each column
+ *     (t_c = amax_c / 7, v_jc = rne(V_jc fl(7 / amax_c)));
+ *   Z_hat_ic = fl(fl(acc_ic fl(1 / fl(255 l_i))) t_c), acc_ic = sum_j c_ij v_jc
+ *     exact (float32 tensor-core accumulation of integers below 2^24);
+ *   Z = Z_hat_h M_h^T + d_h per head h: the head's 128 channels are one TAC
+ *     block (Eq. 17 with g = 128).
+ *
+ *   Q, K, V fp16 [L][ld]: head h is columns 128 h .. 128 h + 127 (e.g. the
+ *     three slices of the QKV projection's output, ld = 3 * 128 H).
+ *   Mp: tac_prepare(M, 128 H, 128, F16) output; d [H][128] float32 or NULL.
+ *   Z out fp16 [L][128 H], the TAC-compensated attention output.
+ *   dbg_codes NULL or uint8 [H][L][L] (P codes), dbg_l NULL or float32 [H][L]
+ *     (row sums l), dbg_acc NULL or int32 [H][L][128] (the exact sums): for
+ *     tests.
+ *   workspace: attention_pv_tac_workspace_size(L, H) bytes, 256-byte aligned
+ *     (V codes transposed and the channel scales).
+ * Shapes: head dimension 128, H >= 1, 128 <= L <= 8192 with L % 128 == 0,
+ * ld >= 128 H with ld % 8 == 0; all pointers 16-byte aligned.
+ * Kernels: a V quantiser (per-channel scales and transposed codes) and one
+ * tcgen05 kernel per (128-query tile, head): two passes of Q K^T over 128-
+ * key chunks (row maxima, then probabilities, codes and sums with P V^T
+ * accumulated one chunk behind), then the dequantisation and TAC epilogue.
+ */
+size_t attention_pv_tac_workspace_size(int L, int H);
+int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L, int H, const void* Mp,
+                     const float* d, void* Z, uint8_t* dbg_codes, float* dbg_l, int32_t* dbg_acc,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * tac_calibrate -- the closed-form TAC parameters (App. C, "Block-wise
  * statistics" through "Bias estimation"), on the GPU in float64.
  *

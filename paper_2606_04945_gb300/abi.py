@@ -21,6 +21,7 @@ EXPORTED = (
     "sgat_quantize_act", "sgat_prepare_weight", "w4_unpack_e4m3", "w4a4_gemm", "fp16_gemm_ref", "tac_prepare", "tac_apply",
     "sgat_linear_workspace_size", "sgat_linear", "starq_last_gemm_tile",
     "tac_calibrate_workspace_size", "tac_calibrate", "sgat_linear_swiglu",
+    "attention_pv_tac_workspace_size", "attention_pv_tac",
 )
 
 
@@ -56,6 +57,9 @@ def _load():
     lib.sgat_linear.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
                                 u8p, u8p, f_p, f_p, i, i, vp, i, vp, ctypes.c_size_t, vp]
     lib.sgat_linear_swiglu.argtypes = lib.sgat_linear.argtypes
+    lib.attention_pv_tac_workspace_size.argtypes = [i, i]
+    lib.attention_pv_tac_workspace_size.restype = ctypes.c_size_t
+    lib.attention_pv_tac.argtypes = [vp, vp, vp, i, i, i, vp, f_p, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
     if hasattr(lib, "sgat_linear_noalloc"):
         lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
                                             u8p, u8p, f_p, f_p, i, i, vp, i, vp]
@@ -183,6 +187,20 @@ def tac_calibrate(Z_fp, Z_q, g, M, d, workspace=None, rho=3e-4, eps=1e-8, eta=0.
         workspace = torch.empty(tac_calibrate_workspace_size(C, g), dtype=torch.uint8, device=Z_fp.device)
     _check(lib.tac_calibrate(_p(Z_fp), _p(Z_q), dtype_code(Z_fp), N, C, g, rho, eps, eta, alpha, _p(M), _p(d),
                              _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def attention_pv_tac(Q, K, V, H, Mp, d, Z, workspace=None, dbg_codes=None, dbg_l=None, dbg_acc=None, stream=None):
+    """Quantised softmax-value product with TAC in its epilogue. Q, K, V are
+    fp16 [L][ld] views (e.g. column slices of the QKV output); Z [L][128 H]."""
+    L = Q.shape[0]
+    ld = Q.stride(0)
+    assert K.stride(0) == ld and V.stride(0) == ld and Q.stride(1) == K.stride(1) == V.stride(1) == 1
+    _contig(Mp, d, Z, workspace, dbg_codes, dbg_l, dbg_acc)
+    if workspace is None:
+        workspace = torch.empty(int(lib.attention_pv_tac_workspace_size(L, H)), dtype=torch.uint8, device=Q.device)
+    _check(lib.attention_pv_tac(_p(Q), _p(K), _p(V), ld, L, H, _p(Mp), _p(d), _p(Z), _p(dbg_codes), _p(dbg_l),
+                                _p(dbg_acc), _p(workspace), workspace.numel() * workspace.element_size(),
+                                _stream(stream)))
 
 
 def sgat_linear_workspace_size(L, K, with_tac):

@@ -6,6 +6,7 @@
 #include <cstring>
 
 #include "common.cuh"
+#include "attn.cuh"
 #include "tac_calib.cuh"
 
 namespace starq {
@@ -251,6 +252,37 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
     TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype, st, Mp};
     cudaError_t e = launch_tac(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "tac_apply launch");
+    return STARQ_OK;
+}
+
+size_t attention_pv_tac_workspace_size(int L, int H) {
+    if (L <= 0 || H <= 0) return 0;
+    return attn_workspace_bytes(L, H);
+}
+
+int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L, int H, const void* Mp,
+                     const float* d, void* Z, uint8_t* dbg_codes, float* dbg_l, int32_t* dbg_acc, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+    if (!Q || !K || !V || !Mp || !Z || !workspace) return fail(STARQ_ERR_ARG, "attention_pv_tac: NULL pointer");
+    if (H < 1) return fail(STARQ_ERR_SHAPE, "attention_pv_tac: H=%d", H);
+    if (L < ATTN_TILE || L % ATTN_TILE != 0 || L > 8192)
+        return fail(STARQ_ERR_SHAPE, "attention_pv_tac: L=%d: need 128 <= L <= 8192, L %% 128 == 0", L);
+    if (ld < ATTN_D * H || ld % 8 != 0)
+        return fail(STARQ_ERR_SHAPE, "attention_pv_tac: ld=%d: need ld >= 128 H and ld %% 8 == 0", ld);
+    const size_t need = attention_pv_tac_workspace_size(L, H);
+    if (workspace_bytes < need) return fail(STARQ_ERR_SHAPE, "attention_pv_tac: workspace %zu bytes < %zu", workspace_bytes, need);
+    if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(Mp, 16) || !aligned(Z, 16) ||
+        (d && !aligned(d, 16)) || !aligned(workspace, 256))
+        return fail(STARQ_ERR_ALIGN, "attention_pv_tac: Q, K, V, Mp, Z, d 16-byte and workspace 256-byte alignment");
+    int rc = STARQ_OK;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    AttnArgs a{Q, K, V, ld, L, H, Mp, d, Z, reinterpret_cast<uint16_t*>(ws),
+               reinterpret_cast<float*>(ws + ((size_t)ATTN_D * H * L * 2 + 255) / 256 * 256),
+               dbg_codes, dbg_l, dbg_acc, st};
+    cudaError_t e = launch_attention_pv_tac(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "attention_pv_tac launch");
     return STARQ_OK;
 }
 
