@@ -19,23 +19,35 @@
 // attn_vquant_kernel   V codes per channel, written as fp16 values into
 //                      Vt [128 H][L] (keys contiguous: the K-major B
 //                      operand of P V^T), and the channel scales t.
-// attn_pv_tac_kernel   one CTA per (128-query tile, head); 8 softmax /
-//                      epilogue warps, a TMA warp and an MMA warp;
-//                      tcgen05 kind::f16 on one CTA (M = N = 128, K = 16).
-//   pass 1  S = Q K^T chunk by chunk (128 keys, double-buffered in TMEM);
-//           each thread keeps the running maximum of its row's half of S.
-//   pass 2  S again; each thread turns its 64 scores into e = exp2((s - m)
-//           log2(e) / sqrt(d)), adds them to l and writes the codes rne(255 e)
-//           as fp16 into the shared A tile of P V^T. The MMA warp
-//           accumulates P V^T one chunk behind the scores (exact integers).
+// attn_pv_tac_kernel   one CTA per (128-query tile, head); 16 softmax /
+//                      epilogue warps (a TMEM lane quarter times 32 of the
+//                      128 columns each), a TMA warp and an MMA warp;
+//                      tcgen05 kind::f16 on one CTA (M = N = 128, K = 16)
+//                      with the A operand (Q, P, Z_hat) in tensor memory
+//                      and B (K, V, M) in shared memory.
+//   prologue  the softmax warps write the Q tile into TMEM.
+//   pass 1  S = Q K^T chunk by chunk (128 keys, three TMEM buffers);
+//           each thread keeps the running maximum of its row's part of S.
+//   pass 2  S again; each thread turns its 32 scores into e = exp2((s - m)
+//           log2(e) / sqrt(d)) (ex2.approx), adds them to l (four partial
+//           sums) and writes the codes rne(255 e), rounded exactly by a
+//           float32 bias whose low bits are fp16 1024 + code, as fp16 over
+//           the S columns it has read (P
+//           double-buffered with S, so the next chunk's probabilities need
+//           not wait for this P V^T). The MMA warp accumulates P V^T one
+//           chunk behind the scores (exact integers).
 //   epilogue  Z_hat from the accumulator, split into fp16 hi + lo (Z_hat =
-//           hi + lo to ~2^-22), written as the A tiles of the TAC product;
-//           Z_hi M_hi^T + Z_hi M_lo^T + Z_lo M_hi^T with M's prepared halves
-//           (tac_prepare); + d; rounded to fp16 and stored by TMA.
-// Shared memory: Q, two K chunks, two V chunks and P (six 32 KB tiles);
-// after the passes the K buffers hold M's halves, the V buffers Z_hat's
-// and the Q tile the output boxes. TMEM: two S buffers, the P V^T and the
-// TAC accumulators (4 x 128 columns). Every wait is bounded.
+//           hi + lo to ~2^-22), written to TMEM as the A operands of the
+//           TAC product Z_hi M_hi^T + Z_hi M_lo^T + Z_lo M_hi^T with M's
+//           prepared halves (tac_prepare); + d; rounded to fp16 and stored
+//           by TMA.
+// Shared memory holds only B operands: a ring of six 32 KB tiles streams
+// pass 1's K chunks and pass 2's K and V chunks in the order the MMAs read
+// them; two of its slots then take M's halves and one the output boxes.
+// (With Q and P in shared memory as well, every chunk moved twice the
+// bytes through shared memory.) TMEM: two S / P buffers, the P V^T
+// accumulator and Q (448 of 512 columns); the TAC accumulator and Z_hat
+// reuse the S buffers. Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -46,107 +58,232 @@ namespace starq {
 namespace {
 
 constexpr unsigned STATUS_TIMEOUT_ATTN = 1u << 4;
-constexpr int ATT_THREADS = 320;
-constexpr int ATT_TMA_WARP = 8, ATT_MMA_WARP = 9, ATT_SOFTMAX_THREADS = 256;
+constexpr int ATT_SOFTMAX_WARPS = 16;           // 4 TMEM lane quarters x 4 column parts of 32
+constexpr int ATT_SOFTMAX_THREADS = ATT_SOFTMAX_WARPS * 32;
+constexpr int ATT_TMA_WARP = ATT_SOFTMAX_WARPS, ATT_MMA_WARP = ATT_SOFTMAX_WARPS + 1;
+constexpr int ATT_THREADS = ATT_SOFTMAX_THREADS + 64;
 constexpr int TILE_BYTES = ATTN_TILE * ATTN_D * 2;            // 128 x 128 fp16, two 128-byte-swizzled atoms
 constexpr int ATOM_BYTES = TILE_BYTES / 2;
-constexpr int OFF_Q = 0, OFF_K = TILE_BYTES, OFF_V = 3 * TILE_BYTES, OFF_P = 5 * TILE_BYTES;
-constexpr int ATT_TILES_BYTES = 6 * TILE_BYTES;
+constexpr int ATT_SLOTS = 6;                                  // the ring of K / V tiles
+constexpr int ATT_TILES_BYTES = ATT_SLOTS * TILE_BYTES;
+// TMEM columns: S in two buffers of 128, the P V^T accumulator O and Q
+// (16-bit, two per column). P overwrites the S it came from: the warp that
+// read S columns [32 p, 32 p + 32) writes their 32 codes to columns
+// [32 p, 32 p + 16). After the passes the TAC accumulator takes the first S
+// buffer and Z_hat's halves the second.
+constexpr uint32_t TM_S = 0, TM_O = 256, TM_Q = 384;
+constexpr uint32_t TM_TAC = 0, TM_ZHI = 128, TM_ZLO = 192;
 
 struct AttSm {
-    uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_empty[2];
-    uint64_t p_full, p_empty, pv_done, z_full, m_full, tac_done;
+    uint64_t q_full, full[ATT_SLOTS], empty[ATT_SLOTS], s_full[3], s_empty[3];
+    uint64_t pv_done, z_full, m_full, tac_done;
     uint32_t tmem_base;
     int abort;
-    float xm[2][ATTN_TILE];            // row maxima / sums of the two column halves
+    float xm[4][ATTN_TILE];            // row maxima / sums of the four column parts
+    float tv[ATTN_D], dv[ATTN_D];      // the head's V channel scales and TAC offsets
 };
 constexpr size_t ATT_SMEM = ATT_TILES_BYTES + 1024 + sizeof(AttSm);
 
 // log2(e) / sqrt(128): S (unscaled Q K^T) to base-2 exponents
 constexpr float EXP_SCALE = (float)(1.4426950408889634 / 11.313708498984761);
+// 1.5 * 2^23 + 0x6400: fma(255, e, ROUND_BIAS) rounds 255 e to the nearest
+// integer n (the spacing of float32 there is 1; the bias is even, so ties
+// go to even n) and leaves 0x6400 + n, the fp16 bits of 1024 + n, in the
+// low half of the result's bits
+constexpr float ROUND_BIAS = 12608512.f;
+
+// 2^x by the PTX approximation (relative error about 2^-22; subnormal
+// results flush to zero, where the code is 0 anyway)
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// D (+)= A B^T, f16 inputs, f32 accumulate, A (128 rows, K-major: a row per
+// TMEM lane, two elements per 32-bit column) in tensor memory, B in shared
+// memory.
+__device__ __forceinline__ void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+    asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                 "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}"
+                 :: "r"(d_tmem), "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate) : "memory");
+}
+
+// 16 consecutive 32-bit columns of one TMEM lane per thread (lanes = the
+// warp's 32-lane quarter).
+__device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+                 "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+                 :: "r"(taddr), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]),
+                    "r"(v[7]), "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+                    "r"(v[15])
+                 : "memory");
+}
+// Arrive once on the barrier at shared offset `bar` in every CTA of
+// `cta_mask` when the issuing thread's tcgen05 operations have completed.
+__device__ __forceinline__ void tc_commit_multicast(uint32_t bar, uint16_t cta_mask) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+                 " [%0], %1;" :: "r"(bar), "h"(cta_mask) : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Both phases complete (warp-uniform result). The two first queries are
+// issued back to back, so their latencies overlap.
+__device__ __forceinline__ bool mbar_wait2_bounded_warp(uint32_t b0, uint32_t p0, uint32_t b1, uint32_t p1,
+                                                        volatile int* abort) {
+    const bool d0 = mbar_try_wait(b0, p0);
+    const bool d1 = mbar_try_wait(b1, p1);
+    bool ok = true;
+    if (!(d0 && d1)) ok = (d0 || mbar_wait_bounded(b0, p0, abort)) && (d1 || mbar_wait_bounded(b1, p1, abort));
+    return __all_sync(0xffffffffu, ok);
+}
 
 __device__ __forceinline__ void named_sync_softmax() {
     asm volatile("bar.sync 1, %0;" :: "r"(ATT_SOFTMAX_THREADS) : "memory");
 }
 
-// Byte offset of element (row, col) of a 128 x 128 fp16 K-major tile (two
-// atoms of 64 columns, 128-byte swizzle).
-__device__ __forceinline__ uint32_t tile_off(int row, int col) {
-    return (uint32_t)(col >> 6) * ATOM_BYTES + sw128_offset((uint32_t)row, (uint32_t)((col & 63) >> 3)) +
-           (uint32_t)(col & 7) * 2;
-}
+// One CTA per 16 channels: two threads per key row, each holding 8
+// channels (16 bytes), 128 rows per sweep. Pass 1 takes the channel maxima,
+// pass 2 (from L2) the codes, transposed through shared memory in tiles of
+// 512 keys and written as 16-byte rows of Vt.
+constexpr int VQ_CH = 16, VQ_KEYS = 512;
 
 __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
-    __shared__ float red[16][32];
-    __shared__ float rcp[32];
-    __shared__ uint16_t tile[32][64 + 2];
-    const __half* V = static_cast<const __half*>(a.V);
-    const int c0 = blockIdx.x * 32;
-    const int tid = threadIdx.x, cp = tid & 15, rg = tid >> 4;
-    float m0 = 0.f, m1 = 0.f;
-    for (int r = rg; r < a.L; r += 16) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(V + (size_t)r * a.ld + c0 + 2 * cp));
-        m0 = fmaxf(m0, fabsf(f.x));
-        m1 = fmaxf(m1, fabsf(f.y));
-    }
-    red[rg][2 * cp] = m0;
-    red[rg][2 * cp + 1] = m1;
-    __syncthreads();
-    if (tid < 32) {
-        float m = 0.f;
+    __shared__ float red[8][VQ_CH];
+    __shared__ float rcp[VQ_CH];
+    __shared__ __align__(16) uint16_t tile[VQ_CH][VQ_KEYS + 8];
+    const int c0 = blockIdx.x * VQ_CH;
+    const int tid = threadIdx.x, hv = tid & 1, rr = tid >> 1, warp = tid >> 5, lane = tid & 31;
+    const __half* col = static_cast<const __half*>(a.V) + c0 + 8 * hv;
+    auto load = [&](int r) {
+        return r < a.L ? __ldg(reinterpret_cast<const uint4*>(col + (size_t)r * a.ld)) : make_uint4(0u, 0u, 0u, 0u);
+    };
+    float m[8];
+    #pragma unroll
+    for (int k = 0; k < 8; ++k) m[k] = 0.f;
+    for (int r0 = 0; r0 < a.L; r0 += VQ_KEYS) {
+        uint4 v[4];
         #pragma unroll
-        for (int g = 0; g < 16; ++g) m = fmaxf(m, red[g][tid]);
-        const bool nz = m > 0.f;
-        a.t[c0 + tid] = nz ? __fdiv_rn(m, 7.f) : 0.f;
-        rcp[tid] = nz ? __fdiv_rn(7.f, m) : 0.f;
+        for (int u = 0; u < 4; ++u) v[u] = load(r0 + rr + 128 * u);
+        #pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const __half2* p = reinterpret_cast<const __half2*>(&v[u]);
+            #pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 f = __half22float2(p[k]);
+                m[2 * k] = fmaxf(m[2 * k], fabsf(f.x));
+                m[2 * k + 1] = fmaxf(m[2 * k + 1], fabsf(f.y));
+            }
+        }
+    }
+    // lanes of equal parity hold the same channels
+    #pragma unroll
+    for (int k = 0; k < 8; ++k)
+        #pragma unroll
+        for (int o = 2; o < 32; o <<= 1) m[k] = fmaxf(m[k], __shfl_xor_sync(0xffffffffu, m[k], o));
+    if (lane < 2) {
+        #pragma unroll
+        for (int k = 0; k < 8; ++k) red[warp][8 * lane + k] = m[k];
     }
     __syncthreads();
-    for (int r0 = 0; r0 < a.L; r0 += 64) {
+    if (tid < VQ_CH) {
+        float mm = 0.f;
         #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int r = r0 + rg + 16 * k;
-            const float2 f = __half22float2(*reinterpret_cast<const __half2*>(V + (size_t)r * a.ld + c0 + 2 * cp));
-            tile[2 * cp][rg + 16 * k] = __half_as_ushort(__float2half_rn(rintf(__fmul_rn(f.x, rcp[2 * cp]))));
-            tile[2 * cp + 1][rg + 16 * k] = __half_as_ushort(__float2half_rn(rintf(__fmul_rn(f.y, rcp[2 * cp + 1]))));
+        for (int w = 0; w < 8; ++w) mm = fmaxf(mm, red[w][tid]);
+        const bool nz = mm > 0.f;
+        a.t[c0 + tid] = nz ? __fdiv_rn(mm, 7.f) : 0.f;
+        rcp[tid] = nz ? __fdiv_rn(7.f, mm) : 0.f;
+    }
+    __syncthreads();
+    float rc[8];
+    #pragma unroll
+    for (int k = 0; k < 8; ++k) rc[k] = rcp[8 * hv + k];
+    for (int r0 = 0; r0 < a.L; r0 += VQ_KEYS) {
+        uint4 v[4];
+        #pragma unroll
+        for (int u = 0; u < 4; ++u) v[u] = load(r0 + rr + 128 * u);
+        #pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const __half2* p = reinterpret_cast<const __half2*>(&v[u]);
+            #pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 f = __half22float2(p[k]);
+                tile[8 * hv + 2 * k][rr + 128 * u] = __half_as_ushort(__float2half_rn(rintf(__fmul_rn(f.x, rc[2 * k]))));
+                tile[8 * hv + 2 * k + 1][rr + 128 * u] =
+                    __half_as_ushort(__float2half_rn(rintf(__fmul_rn(f.y, rc[2 * k + 1]))));
+            }
         }
         __syncthreads();
-        const int c = tid >> 3, rs = (tid & 7) * 8;
-        uint32_t w[4];
-        #pragma unroll
-        for (int u = 0; u < 4; ++u) w[u] = (uint32_t)tile[c][rs + 2 * u] | ((uint32_t)tile[c][rs + 2 * u + 1] << 16);
-        *reinterpret_cast<uint4*>(a.Vt + (size_t)(c0 + c) * a.L + r0 + rs) = make_uint4(w[0], w[1], w[2], w[3]);
+        const int segs = min(VQ_KEYS, a.L - r0) / 8;          // L is a multiple of 128
+        for (int i = tid; i < VQ_CH * segs; i += 256) {
+            const int c = i / segs, sg = i - c * segs;
+            *reinterpret_cast<uint4*>(a.Vt + (size_t)(c0 + c) * a.L + r0 + 8 * sg) =
+                *reinterpret_cast<const uint4*>(&tile[c][8 * sg]);
+        }
         __syncthreads();
     }
 }
 
+// CL CTAs of one head (consecutive query tiles) form a cluster: each loads
+// 128 / CL rows of every K and V tile and multicasts them to all, so each
+// tile leaves L2 once per cluster; a slot is refilled once every CTA's
+// MMAs have read it (its empty barrier counts one commit per CTA).
+template <int CL>
 __global__ void __launch_bounds__(ATT_THREADS, 1)
-attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_z) {
+attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                   const __grid_constant__ CUtensorMap tm_z) {
+    constexpr int SHARE = ATTN_TILE / CL;                    // rows of each tile this CTA loads
+    constexpr uint16_t MASK = (uint16_t)((1u << CL) - 1u);
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     AttSm* sh = reinterpret_cast<AttSm*>(smem_raw + (base - raw) + ATT_TILES_BYTES);
-    const uint32_t sQ = base + OFF_Q, sK = base + OFF_K, sV = base + OFF_V, sP = base + OFF_P;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q0 = blockIdx.x * ATTN_TILE, h = blockIdx.y;
     const int nk = a.L / ATTN_TILE;
     volatile int* abort = &sh->abort;
-    auto B = [&](const uint64_t& bar) { return smem_addr(&bar); };
+    // (the lambdas capture by value: a local captured by reference lives in
+    // memory and is reloaded after every asm with a memory clobber)
+    auto B = [](const uint64_t& bar) { return smem_addr(&bar); };
+    // The ring's loads in order: u = 0 .. nk-1 the K chunks of pass 1, then
+    // u = nk + 2j, nk + 2j + 1 chunk j's K and V tiles for pass 2. Load u
+    // goes to slot u mod 6 (its (u / 6)-th use). M's halves take the slots
+    // of u = U - 6 and U - 5 once those loads are consumed (a negative u
+    // names a slot no load uses), the output boxes the slot of U - 1.
+    const int U = 3 * nk;
+    auto slot_idx = [](int u) { return ((u % ATT_SLOTS) + ATT_SLOTS) % ATT_SLOTS; };
+    auto slot = [=](int u) { return base + (uint32_t)slot_idx(u) * TILE_BYTES; };
+    const uint32_t sMhi = slot(U - 6), sMlo = slot(U - 5), sOut = slot(U - 1);
+    // S buffer of Q K^T number it (pass 1: it = 0 .. nk-1, three buffers,
+    // the third in O's columns, which pass 1 leaves unused; pass 2: it =
+    // nk + j, two buffers) and the number of that buffer's earlier uses
+    auto sbuf = [nk](int it, int& b, int& n) {
+        if (it < nk) {
+            b = it % 3;
+            n = it / 3;
+        } else {
+            const int j = it - nk;
+            b = j & 1;
+            n = (nk - b + 2) / 3 + (j >> 1);
+        }
+    };
 
     if (threadIdx.x == 0) {
-        mbar_init(B(sh->q_full), 1);
-        for (int b = 0; b < 2; ++b) {
-            mbar_init(B(sh->k_full[b]), 1);
-            mbar_init(B(sh->k_empty[b]), 1);
-            mbar_init(B(sh->v_full[b]), 1);
-            mbar_init(B(sh->v_empty[b]), 1);
-            mbar_init(B(sh->s_full[b]), 1);
-            mbar_init(B(sh->s_empty[b]), ATT_SOFTMAX_THREADS / 32);
+        mbar_init(B(sh->q_full), ATT_SOFTMAX_WARPS);
+        for (int k = 0; k < ATT_SLOTS; ++k) {
+            mbar_init(B(sh->full[k]), 1);
+            mbar_init(B(sh->empty[k]), CL);
         }
-        mbar_init(B(sh->p_full), ATT_SOFTMAX_THREADS / 32);
-        mbar_init(B(sh->p_empty), 1);
+        for (int b = 0; b < 3; ++b) {
+            mbar_init(B(sh->s_full[b]), 1);
+            mbar_init(B(sh->s_empty[b]), ATT_SOFTMAX_WARPS);
+        }
         mbar_init(B(sh->pv_done), 1);
-        mbar_init(B(sh->z_full), ATT_SOFTMAX_THREADS / 32);
+        mbar_init(B(sh->z_full), ATT_SOFTMAX_WARPS);
         mbar_init(B(sh->m_full), 1);
         mbar_init(B(sh->tac_done), 1);
         sh->abort = 0;
@@ -158,222 +295,263 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
     }
     tc_fence_before();
     __syncthreads();
+    if (CL > 1) cluster_sync();              // every CTA's barriers exist before any multicast
     tc_fence_after();
     const uint32_t tmem = sh->tmem_base;
+    const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
 
     if (warp == ATT_TMA_WARP) {
         bool ok = true;
-        if (elect_one()) {
-            mbar_arrive_expect_tx(B(sh->q_full), TILE_BYTES);
-            tma_load_2d(sQ, &tm_q, h * ATTN_D, q0, B(sh->q_full));
-            tma_load_2d(sQ + ATOM_BYTES, &tm_q, h * ATTN_D + 64, q0, B(sh->q_full));
-        }
-        __syncwarp();
-        for (int it = 0; it < 2 * nk && ok; ++it) {
-            const int b = it & 1, n = it >> 1, kc = it < nk ? it : it - nk;
-            if (!mbar_wait_bounded_warp(B(sh->k_empty[b]), (uint32_t)(n & 1) ^ 1u, abort)) { ok = false; break; }
-            const uint32_t kt = sK + b * TILE_BYTES;
+        for (int u = 0; u < U && ok; ++u) {
+            const int k = u % ATT_SLOTS, n = u / ATT_SLOTS;
+            if (!mbar_wait_bounded_warp(B(sh->empty[k]), (uint32_t)(n & 1) ^ 1u, abort)) { ok = false; break; }
+            const uint32_t dst = slot(u);
             if (elect_one()) {
-                mbar_arrive_expect_tx(B(sh->k_full[b]), TILE_BYTES);
-                tma_load_2d(kt, &tm_k, h * ATTN_D, kc * ATTN_TILE, B(sh->k_full[b]));
-                tma_load_2d(kt + ATOM_BYTES, &tm_k, h * ATTN_D + 64, kc * ATTN_TILE, B(sh->k_full[b]));
+                mbar_arrive_expect_tx(B(sh->full[k]), TILE_BYTES);
+                const int w = u - nk;
+                const uint32_t d0 = dst + (uint32_t)(rank * SHARE * 128), fb = B(sh->full[k]);
+                const void* tm = (w < 0 || (w & 1) == 0) ? (const void*)&tm_k : (const void*)&tm_v;
+                int x, y;
+                if (w < 0 || (w & 1) == 0) {                 // K chunk: keys are the rows
+                    x = h * ATTN_D;
+                    y = (w < 0 ? u : w >> 1) * ATTN_TILE + rank * SHARE;
+                } else {                                     // V chunk: channels are the rows
+                    x = (w >> 1) * ATTN_TILE;
+                    y = h * ATTN_D + rank * SHARE;
+                }
+                if (CL > 1) {
+                    tma_load_2d_multicast(d0, tm, x, y, fb, MASK);
+                    tma_load_2d_multicast(d0 + ATOM_BYTES, tm, x + 64, y, fb, MASK);
+                } else {
+                    tma_load_2d(d0, tm, x, y, fb);
+                    tma_load_2d(d0 + ATOM_BYTES, tm, x + 64, y, fb);
+                }
             }
             __syncwarp();
-            if (it >= nk) {
-                const int j = it - nk, vb = j & 1, vn = j >> 1;
-                if (!mbar_wait_bounded_warp(B(sh->v_empty[vb]), (uint32_t)(vn & 1) ^ 1u, abort)) { ok = false; break; }
-                const uint32_t vt = sV + vb * TILE_BYTES;
-                if (elect_one()) {
-                    mbar_arrive_expect_tx(B(sh->v_full[vb]), TILE_BYTES);
-                    tma_load_2d(vt, &tm_v, j * ATTN_TILE, h * ATTN_D, B(sh->v_full[vb]));
-                    tma_load_2d(vt + ATOM_BYTES, &tm_v, j * ATTN_TILE + 64, h * ATTN_D, B(sh->v_full[vb]));
-                }
-                __syncwarp();
-            }
         }
-        // M's two halves into the K buffers once the last score MMA has read them
-        for (int b = 0; b < 2 && ok; ++b)
-            ok = mbar_wait_bounded_warp(B(sh->k_empty[b]), (uint32_t)((nk - 1) & 1), abort);
+        // M's halves once their slots' last loads have been consumed
+        for (int u = U - 6; u < U - 4 && ok; ++u)
+            if (u >= 0) ok = mbar_wait_bounded_warp(B(sh->empty[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1), abort);
         if (ok && elect_one()) {
+            const uint8_t* mp = static_cast<const uint8_t*>(a.Mp) + (size_t)h * 2 * TILE_BYTES;
             mbar_arrive_expect_tx(B(sh->m_full), 2 * TILE_BYTES);
-            bulk_load(sK, static_cast<const uint8_t*>(a.Mp) + (size_t)h * 2 * TILE_BYTES, 2 * TILE_BYTES,
-                      B(sh->m_full));
+            bulk_load(sMhi, mp, TILE_BYTES, B(sh->m_full));
+            bulk_load(sMlo, mp + TILE_BYTES, TILE_BYTES, B(sh->m_full));
         }
         __syncwarp();
+        // every CTA's commits for the last use of each slot have arrived
+        // here, so none lands after this CTA has exited
+        for (int u = U - ATT_SLOTS; u < U && ok; ++u)
+            if (u >= 0) ok = mbar_wait_bounded_warp(B(sh->empty[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1), abort);
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     } else if (warp == ATT_MMA_WARP) {
         // f16 A and B, f32 D, N = 128 (bits 17..22), M = 128 (bits 24..28)
         constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(ATTN_TILE >> 3) << 17) | ((uint32_t)(ATTN_TILE >> 4) << 24);
         bool ok = mbar_wait_bounded_warp(B(sh->q_full), 0, abort);
-        auto mma_tile = [&](uint32_t d, uint32_t at, uint32_t bt, bool acc0) {
+        // D (+)= A B^T over K = 128: A from TMEM at a_col (8 columns per K
+        // step; for P, K steps 2p and 2p + 1 sit at 32 p and 32 p + 8), B
+        // the K-major tile at bt
+        auto mma_tile = [=](uint32_t d, uint32_t a_col, uint32_t bt, bool acc0, bool p_layout) {
+            // K step offsets added to the descriptor's start-address field
+            // (addresses below 2^18, so the field never carries)
+            const uint64_t bd = smem_desc_sw128(bt);
+            const uint32_t ta = tmem + a_col;
             if (elect_one()) {
                 #pragma unroll
                 for (int ks = 0; ks < ATTN_D / 16; ++ks) {
                     const uint32_t koff = (uint32_t)(ks >> 2) * ATOM_BYTES + (uint32_t)(ks & 3) * 32;
-                    mma_f16(d, smem_desc_sw128(at + koff), smem_desc_sw128(bt + koff), IDESC, (acc0 || ks > 0) ? 1u : 0u);
+                    const uint32_t ac = p_layout ? 32u * (uint32_t)(ks >> 1) + 8u * (uint32_t)(ks & 1) : 8u * (uint32_t)ks;
+                    mma_f16_ts(d, ta + ac, bd + (uint64_t)(koff >> 4), IDESC, (acc0 || ks > 0) ? 1u : 0u);
                 }
             }
             __syncwarp();
         };
-        auto pv = [&](int j) {                 // P V^T of pass-2 chunk j
-            const int vb = j & 1, vn = j >> 1;
-            ok = ok && mbar_wait_bounded_warp(B(sh->p_full), (uint32_t)(j & 1), abort) &&
-                 mbar_wait_bounded_warp(B(sh->v_full[vb]), (uint32_t)(vn & 1), abort);
-            if (!ok) return;
-            tc_fence_after();
-            mma_tile(tmem + 256, sP, sV + vb * TILE_BYTES, j > 0);
-            if (elect_one()) {
-                tc_commit(B(sh->p_empty));
-                tc_commit(B(sh->v_empty[vb]));
-            }
-            __syncwarp();
+        auto release = [=](int u) {           // this CTA's MMAs are done with ring slot u
+            if (CL > 1) tc_commit_multicast(B(sh->empty[u % ATT_SLOTS]), MASK);
+            else tc_commit(B(sh->empty[u % ATT_SLOTS]));
         };
-        tc_fence_after();
-        for (int it = 0; it < 2 * nk && ok; ++it) {
-            const int b = it & 1, n = it >> 1;
-            ok = mbar_wait_bounded_warp(B(sh->k_full[b]), (uint32_t)(n & 1), abort) &&
-                 mbar_wait_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1) ^ 1u, abort);
-            if (!ok) break;
+        // Q K^T number it, once its K tile has landed and its S buffer's
+        // previous use is consumed (S read by the softmax warps, or P
+        // written by them and read by the P V^T issued before this MMA:
+        // the MMAs of one thread run in issue order)
+        auto qk = [=](int it) -> bool {
+            const int u = it < nk ? it : nk + 2 * (it - nk);
+            int b, n;
+            sbuf(it, b, n);
+            if (!mbar_wait2_bounded_warp(B(sh->full[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1),
+                                         B(sh->s_empty[b]), (uint32_t)(n & 1) ^ 1u, abort))
+                return false;
             tc_fence_after();
-            mma_tile(tmem + b * ATTN_TILE, sQ, sK + b * TILE_BYTES, false);
+            mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(u), false, false);
             if (elect_one()) {
-                tc_commit(B(sh->k_empty[b]));
+                release(u);
                 tc_commit(B(sh->s_full[b]));
             }
             __syncwarp();
-            if (it > nk) pv(it - 1 - nk);        // one chunk behind the scores
-        }
-        if (ok) pv(nk - 1);
-        if (elect_one()) tc_commit(B(sh->pv_done));
-        __syncwarp();
-        ok = ok && mbar_wait_bounded_warp(B(sh->z_full), 0, abort) && mbar_wait_bounded_warp(B(sh->m_full), 0, abort);
-        if (ok) {
+            return true;
+        };
+        // P V^T of pass-2 chunk j, once its P is in its S buffer
+        auto pv = [=](int j) -> bool {
+            const int u = nk + 2 * j + 1;
+            int b, n;
+            sbuf(nk + j, b, n);
+            if (!mbar_wait2_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1), B(sh->full[u % ATT_SLOTS]),
+                                         (uint32_t)((u / ATT_SLOTS) & 1), abort))
+                return false;
             tc_fence_after();
-            const uint32_t dt = tmem + 384;
-            mma_tile(dt, sV, sK, false);                               // Z_hi M_hi^T
-            mma_tile(dt, sV, sK + TILE_BYTES, true);                   // + Z_hi M_lo^T
-            mma_tile(dt, sV + TILE_BYTES, sK, true);                   // + Z_lo M_hi^T
+            mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(u), j > 0, true);
+            if (elect_one()) release(u);
+            __syncwarp();
+            return true;
+        };
+        tc_fence_after();
+        {
+            for (int it = 0; it < 2 * nk && ok; ++it) {
+                ok = qk(it);
+                if (ok && it > nk) ok = pv(it - 1 - nk);   // one chunk behind the scores
+            }
+            if (ok) ok = pv(nk - 1);
+            if (elect_one()) tc_commit(B(sh->pv_done));
+            __syncwarp();
+            ok = ok && mbar_wait2_bounded_warp(B(sh->z_full), 0, B(sh->m_full), 0, abort);
+            if (ok) {
+                tc_fence_after();
+                mma_tile(tmem + TM_TAC, TM_ZHI, sMhi, false, false);       // Z_hi M_hi^T
+                mma_tile(tmem + TM_TAC, TM_ZHI, sMlo, true, false);        // + Z_hi M_lo^T
+                mma_tile(tmem + TM_TAC, TM_ZLO, sMhi, true, false);        // + Z_lo M_hi^T
+            }
+            if (elect_one()) tc_commit(B(sh->tac_done));
+            __syncwarp();
+            if (lane == 0) {
+                // every MMA of this thread has completed before TMEM is released
+                volatile int never = 0;
+                if (!mbar_wait_bounded(B(sh->tac_done), 0, &never)) ok = false;
+            }
+            __syncwarp();
         }
-        if (elect_one()) tc_commit(B(sh->tac_done));
-        __syncwarp();
-        if (lane == 0) {
-            // every MMA of this thread has completed before TMEM is released
-            volatile int never = 0;
-            if (!mbar_wait_bounded(B(sh->tac_done), 0, &never)) ok = false;
-            if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
-        }
-        __syncwarp();
+        if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     } else {
-        const int quarter = warp & 3, hf = warp >> 2;
+        const int quarter = warp & 3, part = warp >> 2, col = part * 32;
         const int row = quarter * 32 + lane;                // query within the tile (TMEM lane)
         const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
         bool ok = true;
         uint32_t r[32];
+        if (threadIdx.x < ATTN_D) {
+            sh->tv[threadIdx.x] = a.t[h * ATTN_D + threadIdx.x];
+        } else if (threadIdx.x < 2 * ATTN_D) {
+            const int c = threadIdx.x - ATTN_D;
+            sh->dv[c] = a.d != nullptr ? a.d[h * ATTN_D + c] : 0.f;
+        }
+        {   // the query row's 32 channels of this part into TMEM (A of Q K^T)
+            const __half* qp = static_cast<const __half*>(a.Q) + (size_t)(q0 + row) * a.ld + h * ATTN_D + col;
+            uint32_t qv[16];
+            #pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const uint4 w = ld_global_nc_v4(qp + 8 * k);
+                qv[4 * k] = w.x;
+                qv[4 * k + 1] = w.y;
+                qv[4 * k + 2] = w.z;
+                qv[4 * k + 3] = w.w;
+            }
+            tmem_st_32x32b_x16(tl + TM_Q + part * 16, qv);
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(B(sh->q_full));
+        }
         // pass 1: row maxima
         float mx = -INFINITY;
         for (int it = 0; it < nk && ok; ++it) {
-            const int b = it & 1, n = it >> 1;
+            int b, n;
+            sbuf(it, b, n);
             if (!mbar_wait_bounded_warp(B(sh->s_full[b]), (uint32_t)(n & 1), abort)) { ok = false; break; }
             tc_fence_after();
-            #pragma unroll
-            for (int c = 0; c < 2; ++c) {
-                tmem_ld_32x32b_x32(tl + b * ATTN_TILE + hf * 64 + c * 32, r);
-                tmem_ld_wait();
-                #pragma unroll
-                for (int k = 0; k < 32; ++k) mx = fmaxf(mx, __uint_as_float(r[k]));
-            }
+            tmem_ld_32x32b_x32(tl + TM_S + b * ATTN_TILE + col, r);
+            tmem_ld_wait();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
+            #pragma unroll
+            for (int k = 0; k < 32; ++k) mx = fmaxf(mx, __uint_as_float(r[k]));
         }
-        sh->xm[hf][row] = mx;
+        sh->xm[part][row] = mx;
         named_sync_softmax();
-        mx = fmaxf(sh->xm[0][row], sh->xm[1][row]);
+        mx = fmaxf(fmaxf(sh->xm[0][row], sh->xm[1][row]), fmaxf(sh->xm[2][row], sh->xm[3][row]));
         named_sync_softmax();
         // pass 2: probabilities, their codes and the row sums
-        float l = 0.f;
+        float lp[4] = {0.f, 0.f, 0.f, 0.f};      // partial row sums (independent chains)
         for (int j = 0; j < nk && ok; ++j) {
-            const int it = nk + j, b = it & 1, n = it >> 1;
+            int b, n;
+            sbuf(nk + j, b, n);
             if (!mbar_wait_bounded_warp(B(sh->s_full[b]), (uint32_t)(n & 1), abort)) { ok = false; break; }
             tc_fence_after();
-            float e[64];
+            tmem_ld_32x32b_x32(tl + TM_S + b * ATTN_TILE + col, r);
+            tmem_ld_wait();
+            // e = 2^((s - m) log2(e) / sqrt(d)); the code n = rne(255 e) in
+            // one rounding: the low halves of fma(255, e, ROUND_BIAS) are the
+            // fp16 values 1024 + n of two codes, and 1024 is subtracted
+            // exactly in fp16
+            uint32_t packed[16];
+            const __half2 minus1024 = __float2half2_rn(-1024.f);
             #pragma unroll
-            for (int c = 0; c < 2; ++c) {
-                tmem_ld_32x32b_x32(tl + b * ATTN_TILE + hf * 64 + c * 32, r);
-                tmem_ld_wait();
-                #pragma unroll
-                for (int k = 0; k < 32; ++k) e[32 * c + k] = exp2f((__uint_as_float(r[k]) - mx) * EXP_SCALE);
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
-            uint32_t packed[32];
-            #pragma unroll
-            for (int k = 0; k < 64; k += 2) {
-                l += e[k];
-                l += e[k + 1];
-                const __half c0 = __float2half_rn(rintf(__fmul_rn(255.f, e[k])));
-                const __half c1 = __float2half_rn(rintf(__fmul_rn(255.f, e[k + 1])));
-                packed[k / 2] = (uint32_t)__half_as_ushort(c0) | ((uint32_t)__half_as_ushort(c1) << 16);
+            for (int k = 0; k < 32; k += 2) {
+                const float e0 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k]), mx), EXP_SCALE));
+                const float e1 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k + 1]), mx), EXP_SCALE));
+                lp[(k >> 1) & 1] += e0;
+                lp[2 + ((k >> 1) & 1)] += e1;
+                const uint32_t t0 = __float_as_uint(fmaf(255.f, e0, ROUND_BIAS));
+                const uint32_t t1 = __float_as_uint(fmaf(255.f, e1, ROUND_BIAS));
+                const uint32_t biased = prmt(t0, t1, 0x5410u);           // {1024 + n0, 1024 + n1}
+                const __half2 hc = __hadd2(*reinterpret_cast<const __half2*>(&biased), minus1024);
+                packed[k / 2] = *reinterpret_cast<const uint32_t*>(&hc);
             }
             if (a.dbg_codes != nullptr) {
-                uint8_t* dc = a.dbg_codes + ((size_t)h * a.L + q0 + row) * a.L + j * ATTN_TILE + hf * 64;
+                uint8_t* dc = a.dbg_codes + ((size_t)h * a.L + q0 + row) * a.L + j * ATTN_TILE + col;
                 #pragma unroll
-                for (int k = 0; k < 32; ++k) {
+                for (int k = 0; k < 16; ++k) {
                     dc[2 * k] = (uint8_t)__half2float(__ushort_as_half((uint16_t)(packed[k] & 0xFFFFu)));
                     dc[2 * k + 1] = (uint8_t)__half2float(__ushort_as_half((uint16_t)(packed[k] >> 16)));
                 }
             }
-            // the previous chunk's P V^T has read the P tile
-            if (!mbar_wait_bounded_warp(B(sh->p_empty), (uint32_t)(j & 1) ^ 1u, abort)) { ok = false; break; }
-            #pragma unroll
-            for (int c = 0; c < 8; ++c)
-                st_shared_v4(sP + tile_off(row, hf * 64 + 8 * c), packed[4 * c], packed[4 * c + 1], packed[4 * c + 2],
-                             packed[4 * c + 3]);
-            fence_proxy_async_smem();
+            // P over the S columns this warp has read
+            tmem_st_32x32b_x16(tl + TM_S + b * ATTN_TILE + col, packed);
+            tmem_st_wait();
+            tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(B(sh->p_full));
+            if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
         }
-        sh->xm[hf][row] = l;
+        sh->xm[part][row] = (lp[0] + lp[1]) + (lp[2] + lp[3]);
         named_sync_softmax();
-        l = sh->xm[0][row] + sh->xm[1][row];
+        const float l = (sh->xm[0][row] + sh->xm[1][row]) + (sh->xm[2][row] + sh->xm[3][row]);
         const float sp = __fdiv_rn(1.f, __fmul_rn(255.f, l));
-        if (a.dbg_l != nullptr && hf == 0) a.dbg_l[(size_t)h * a.L + q0 + row] = l;
-        // epilogue 1: Z_hat = (acc sp) t as fp16 hi + lo A tiles of the TAC product
+        if (a.dbg_l != nullptr && part == 0) a.dbg_l[(size_t)h * a.L + q0 + row] = l;
+        // epilogue 1: Z_hat = (acc sp) t as fp16 hi + lo, the A operands of
+        // the TAC product, into TMEM
         ok = ok && mbar_wait_bounded_warp(B(sh->pv_done), 0, abort);
         if (ok) {
             tc_fence_after();
-            #pragma unroll 1
-            for (int c = 0; c < 2; ++c) {
-                const int ch = hf * 64 + c * 32;
-                tmem_ld_32x32b_x32(tl + 256 + ch, r);
-                tmem_ld_wait();
-                if (a.dbg_acc != nullptr) {
-                    int32_t* da = a.dbg_acc + ((size_t)h * a.L + q0 + row) * ATTN_D + ch;
-                    #pragma unroll
-                    for (int k = 0; k < 32; ++k) da[k] = __float2int_rn(__uint_as_float(r[k]));
-                }
-                uint32_t hi[16], lo[16];
+            tmem_ld_32x32b_x32(tl + TM_O + col, r);
+            tmem_ld_wait();
+            if (a.dbg_acc != nullptr) {
+                int32_t* da = a.dbg_acc + ((size_t)h * a.L + q0 + row) * ATTN_D + col;
                 #pragma unroll
-                for (int k = 0; k < 32; k += 2) {
-                    float z[2];
-                    #pragma unroll
-                    for (int u = 0; u < 2; ++u)
-                        z[u] = __fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), __ldg(a.t + h * ATTN_D + ch + k + u));
-                    const __half h0 = __float2half_rn(z[0]), h1 = __float2half_rn(z[1]);
-                    const __half l0 = __float2half_rn(z[0] - __half2float(h0)), l1 = __float2half_rn(z[1] - __half2float(h1));
-                    hi[k / 2] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-                    lo[k / 2] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
-                }
-                #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint32_t off = tile_off(row, ch + 8 * q);
-                    st_shared_v4(sV + off, hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
-                    st_shared_v4(sV + TILE_BYTES + off, lo[4 * q], lo[4 * q + 1], lo[4 * q + 2], lo[4 * q + 3]);
-                }
+                for (int k = 0; k < 32; ++k) da[k] = __float2int_rn(__uint_as_float(r[k]));
             }
+            uint32_t hi[16], lo[16];
+            #pragma unroll
+            for (int k = 0; k < 32; k += 2) {
+                float z[2];
+                #pragma unroll
+                for (int u = 0; u < 2; ++u) z[u] = __fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), sh->tv[col + k + u]);
+                const __half h0 = __float2half_rn(z[0]), h1 = __float2half_rn(z[1]);
+                const __half l0 = __float2half_rn(z[0] - __half2float(h0)), l1 = __float2half_rn(z[1] - __half2float(h1));
+                hi[k / 2] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
+                lo[k / 2] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+            }
+            tmem_st_32x32b_x16(tl + TM_ZHI + part * 16, hi);
+            tmem_st_32x32b_x16(tl + TM_ZLO + part * 16, lo);
+            tmem_st_wait();
             tc_fence_before();
-            fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(B(sh->z_full));
         }
@@ -381,42 +559,41 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
         ok = ok && mbar_wait_bounded_warp(B(sh->tac_done), 0, abort);
         if (ok) {
             tc_fence_after();
-            #pragma unroll 1
-            for (int c = 0; c < 2; ++c) {
-                const int ch = hf * 64 + c * 32;
-                tmem_ld_32x32b_x32(tl + 384 + ch, r);
-                tmem_ld_wait();
-                const uint32_t box = sQ + (uint32_t)(warp * 2 + c) * 2048;
+            tmem_ld_32x32b_x32(tl + TM_TAC + col, r);
+            tmem_ld_wait();
+            const uint32_t box = sOut + (uint32_t)warp * 2048;
+            const bool add_d = a.d != nullptr;
+            #pragma unroll
+            for (int g = 0; g < 4; ++g) {
+                uint32_t w[4];
                 #pragma unroll
-                for (int g = 0; g < 4; ++g) {
-                    uint32_t w[4];
-                    #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int k = 8 * g + 2 * u;
-                        float y0 = __uint_as_float(r[k]), y1 = __uint_as_float(r[k + 1]);
-                        if (a.d != nullptr) {
-                            y0 = __fadd_rn(y0, __ldg(a.d + h * ATTN_D + ch + k));
-                            y1 = __fadd_rn(y1, __ldg(a.d + h * ATTN_D + ch + k + 1));
-                        }
-                        const __half2 hv = __floats2half2_rn(y0, y1);
-                        w[u] = *reinterpret_cast<const uint32_t*>(&hv);
+                for (int u = 0; u < 4; ++u) {
+                    const int k = 8 * g + 2 * u;
+                    float y0 = __uint_as_float(r[k]), y1 = __uint_as_float(r[k + 1]);
+                    if (add_d) {
+                        y0 = __fadd_rn(y0, sh->dv[col + k]);
+                        y1 = __fadd_rn(y1, sh->dv[col + k + 1]);
                     }
-                    st_shared_v4(box + lane * 64 + 16 * (g ^ ((lane >> 1) & 3)), w[0], w[1], w[2], w[3]);
+                    const __half2 hv = __floats2half2_rn(y0, y1);
+                    w[u] = *reinterpret_cast<const uint32_t*>(&hv);
                 }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    tma_store_2d(&tm_z, h * ATTN_D + ch, q0 + quarter * 32, box);
-                    bulk_commit();
-                }
+                st_shared_v4(box + lane * 64 + 16 * (g ^ ((lane >> 1) & 3)), w[0], w[1], w[2], w[3]);
             }
-            if (lane == 0) bulk_wait0();
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                tma_store_2d(&tm_z, h * ATTN_D + col, q0 + quarter * 32, box);
+                bulk_commit();
+                bulk_wait0();
+            }
             __syncwarp();
         }
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     }
     tc_fence_before();
     __syncthreads();
+    // no CTA leaves while another may still commit to its barriers
+    if (CL > 1) cluster_sync();
     tc_fence_after();
     if (warp == ATT_MMA_WARP) tmem_dealloc(tmem, 512);
 }
@@ -443,27 +620,48 @@ bool encode_2d(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, ui
 
 }  // namespace
 
-cudaError_t launch_attention_pv_tac(const AttnArgs& a, cudaStream_t stream) {
+template <int CL>
+cudaError_t launch_pv_tac(const AttnArgs& a, cudaStream_t stream) {
     const int C = ATTN_D * a.H;
-    attn_vquant_kernel<<<C / 32, 256, 0, stream>>>(a);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    CUtensorMap tq, tk, tv, tz;
-    if (!encode_2d(&tq, a.Q, (uint64_t)a.L, (uint64_t)C, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)C, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_2d(&tv, a.Vt, (uint64_t)C, (uint64_t)a.L, (uint64_t)a.L, ATTN_D, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
+    CUtensorMap tk, tv, tz;
+    if (!encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)C, (uint64_t)a.ld, ATTN_TILE / CL, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_2d(&tv, a.Vt, (uint64_t)C, (uint64_t)a.L, (uint64_t)a.L, ATTN_D / CL, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !encode_2d(&tz, a.Z, (uint64_t)a.L, (uint64_t)C, (uint64_t)C, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
         return cudaErrorInvalidValue;
     static bool attr_set[64] = {false};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev < 64 && !attr_set[dev]) {
-        e = cudaFuncSetAttribute(attn_pv_tac_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ATT_SMEM);
+        const cudaError_t e =
+            cudaFuncSetAttribute(attn_pv_tac_kernel<CL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ATT_SMEM);
         if (e != cudaSuccess) return e;
         attr_set[dev] = true;
     }
-    attn_pv_tac_kernel<<<dim3(a.L / ATTN_TILE, a.H), ATT_THREADS, ATT_SMEM, stream>>>(a, tq, tk, tv, tz);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3(a.L / ATTN_TILE, a.H);
+    cfg.blockDim = dim3(ATT_THREADS);
+    cfg.dynamicSmemBytes = ATT_SMEM;
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, attn_pv_tac_kernel<CL>, a, tk, tv, tz);
+}
+
+cudaError_t launch_attention_pv_tac(const AttnArgs& a, cudaStream_t stream) {
+    const int C = ATTN_D * a.H;
+    attn_vquant_kernel<<<C / VQ_CH, 256, 0, stream>>>(a);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // clusters of 4 (or 2) query tiles of a head share the K / V loads
+    const int tiles = a.L / ATTN_TILE;
+    if (tiles % 4 == 0) return launch_pv_tac<4>(a, stream);
+    if (tiles % 2 == 0) return launch_pv_tac<2>(a, stream);
+    return launch_pv_tac<1>(a, stream);
 }
 
 }  // namespace starq

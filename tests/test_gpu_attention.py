@@ -5,9 +5,10 @@ Q, K and V are the three column slices of one fp16 [L][3 * 128 H] QKV
 output (the layout the QKV projection writes), N(0, 1). The TAC blocks
 are I + N(0, 0.01), one per head. The comparisons:
 
-- P codes at every position. The kernel takes exp in float32 and the
-  oracle in float64, so a code may differ by one, but only where 255 e lies
-  within 1e-3 of a half-integer (the decision is a floating-point
+- P codes at every position. The kernel takes exp in float32 (the PTX
+  approximation, relative error about 2^-22, so 255 e to about 1e-4) and
+  the oracle in float64, so a code may differ by one, but only where 255 e
+  lies within 1e-3 of a half-integer (the decision is a floating-point
   rounding; elsewhere the codes are equal);
 - row sums l to 1e-5 relative;
 - the exact integer sums, bit for bit, against the oracle's integer product
