@@ -245,9 +245,12 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  * Shapes: head dimension 128, H >= 1, 128 <= L <= 8192 with L % 128 == 0,
  * ld >= 128 H with ld % 8 == 0; all pointers 16-byte aligned.
  * Kernels: a V quantiser (per-channel scales and transposed codes) and one
- * tcgen05 kernel per (128-query tile, head): two passes of Q K^T over 128-
- * key chunks (row maxima, then probabilities, codes and sums with P V^T
- * accumulated one chunk behind), then the dequantisation and TAC epilogue.
+ * tcgen05 kernel with a CTA per (128-query tile, head): two passes of
+ * Q K^T over 128-key chunks (row maxima, then probabilities, codes and sums
+ * with P V^T accumulated one chunk behind), then the dequantisation and TAC
+ * epilogue. Clusters of 4 (or 2) query tiles of a head share each K / V
+ * tile load by multicast. The call is asynchronous on `stream`; a wait that
+ * gives up inside the kernel is reported by starq_check_status.
  */
 size_t attention_pv_tac_workspace_size(int L, int H);
 int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L, int H, const void* Mp,

@@ -351,39 +351,39 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         // D (+)= A B^T over K = 128: A from TMEM at a_col (8 columns per K
         // step; for P, K steps 2p and 2p + 1 sit at 32 p and 32 p + 8), B
         // the K-major tile at bt
+        // (issued by the elected lane)
         auto mma_tile = [=](uint32_t d, uint32_t a_col, uint32_t bt, bool acc0, bool p_layout) {
             // K step offsets added to the descriptor's start-address field
             // (addresses below 2^18, so the field never carries)
             const uint64_t bd = smem_desc_sw128(bt);
             const uint32_t ta = tmem + a_col;
-            if (elect_one()) {
-                #pragma unroll
-                for (int ks = 0; ks < ATTN_D / 16; ++ks) {
-                    const uint32_t koff = (uint32_t)(ks >> 2) * ATOM_BYTES + (uint32_t)(ks & 3) * 32;
-                    const uint32_t ac = p_layout ? 32u * (uint32_t)(ks >> 1) + 8u * (uint32_t)(ks & 1) : 8u * (uint32_t)ks;
-                    mma_f16_ts(d, ta + ac, bd + (uint64_t)(koff >> 4), IDESC, (acc0 || ks > 0) ? 1u : 0u);
-                }
+            #pragma unroll
+            for (int ks = 0; ks < ATTN_D / 16; ++ks) {
+                const uint32_t koff = (uint32_t)(ks >> 2) * ATOM_BYTES + (uint32_t)(ks & 3) * 32;
+                const uint32_t ac = p_layout ? 32u * (uint32_t)(ks >> 1) + 8u * (uint32_t)(ks & 1) : 8u * (uint32_t)ks;
+                mma_f16_ts(d, ta + ac, bd + (uint64_t)(koff >> 4), IDESC, (acc0 || ks > 0) ? 1u : 0u);
             }
-            __syncwarp();
         };
         auto release = [=](int u) {           // this CTA's MMAs are done with ring slot u
             if (CL > 1) tc_commit_multicast(B(sh->empty[u % ATT_SLOTS]), MASK);
             else tc_commit(B(sh->empty[u % ATT_SLOTS]));
         };
         // Q K^T number it, once its K tile has landed and its S buffer's
-        // previous use is consumed (S read by the softmax warps, or P
-        // written by them and read by the P V^T issued before this MMA:
-        // the MMAs of one thread run in issue order)
+        // previous use is consumed: S read by the softmax warps, or P
+        // written by them and read by the P V^T issued before this MMA (the
+        // MMAs of one thread run in issue order). For pass-2 chunks from 2
+        // on, that P V^T's own wait has already seen the P written.
         auto qk = [=](int it) -> bool {
             const int u = it < nk ? it : nk + 2 * (it - nk);
             int b, n;
             sbuf(it, b, n);
-            if (!mbar_wait2_bounded_warp(B(sh->full[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1),
-                                         B(sh->s_empty[b]), (uint32_t)(n & 1) ^ 1u, abort))
+            const uint32_t fb = B(sh->full[u % ATT_SLOTS]), fp = (uint32_t)((u / ATT_SLOTS) & 1);
+            if (!(it >= nk + 2 ? mbar_wait_bounded_warp(fb, fp, abort)
+                               : mbar_wait2_bounded_warp(fb, fp, B(sh->s_empty[b]), (uint32_t)(n & 1) ^ 1u, abort)))
                 return false;
             tc_fence_after();
-            mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(u), false, false);
             if (elect_one()) {
+                mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(u), false, false);
                 release(u);
                 tc_commit(B(sh->s_full[b]));
             }
@@ -399,8 +399,10 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                                          (uint32_t)((u / ATT_SLOTS) & 1), abort))
                 return false;
             tc_fence_after();
-            mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(u), j > 0, true);
-            if (elect_one()) release(u);
+            if (elect_one()) {
+                mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(u), j > 0, true);
+                release(u);
+            }
             __syncwarp();
             return true;
         };
@@ -414,13 +416,15 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             if (elect_one()) tc_commit(B(sh->pv_done));
             __syncwarp();
             ok = ok && mbar_wait2_bounded_warp(B(sh->z_full), 0, B(sh->m_full), 0, abort);
-            if (ok) {
-                tc_fence_after();
-                mma_tile(tmem + TM_TAC, TM_ZHI, sMhi, false, false);       // Z_hi M_hi^T
-                mma_tile(tmem + TM_TAC, TM_ZHI, sMlo, true, false);        // + Z_hi M_lo^T
-                mma_tile(tmem + TM_TAC, TM_ZLO, sMhi, true, false);        // + Z_lo M_hi^T
+            tc_fence_after();
+            if (elect_one()) {
+                if (ok) {
+                    mma_tile(tmem + TM_TAC, TM_ZHI, sMhi, false, false);   // Z_hi M_hi^T
+                    mma_tile(tmem + TM_TAC, TM_ZHI, sMlo, true, false);    // + Z_hi M_lo^T
+                    mma_tile(tmem + TM_TAC, TM_ZLO, sMhi, true, false);    // + Z_lo M_hi^T
+                }
+                tc_commit(B(sh->tac_done));
             }
-            if (elect_one()) tc_commit(B(sh->tac_done));
             __syncwarp();
             if (lane == 0) {
                 // every MMA of this thread has completed before TMEM is released
@@ -436,13 +440,8 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
         bool ok = true;
         uint32_t r[32];
-        if (threadIdx.x < ATTN_D) {
-            sh->tv[threadIdx.x] = a.t[h * ATTN_D + threadIdx.x];
-        } else if (threadIdx.x < 2 * ATTN_D) {
-            const int c = threadIdx.x - ATTN_D;
-            sh->dv[c] = a.d != nullptr ? a.d[h * ATTN_D + c] : 0.f;
-        }
-        {   // the query row's 32 channels of this part into TMEM (A of Q K^T)
+        {   // the query row's 32 channels of this part into TMEM (A of Q K^T);
+            // the loads of Q, t and d are all in flight together
             const __half* qp = static_cast<const __half*>(a.Q) + (size_t)(q0 + row) * a.ld + h * ATTN_D + col;
             uint32_t qv[16];
             #pragma unroll
@@ -452,6 +451,10 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 qv[4 * k + 1] = w.y;
                 qv[4 * k + 2] = w.z;
                 qv[4 * k + 3] = w.w;
+            }
+            if (threadIdx.x >= ATTN_D && threadIdx.x < 2 * ATTN_D) {
+                const int c = threadIdx.x - ATTN_D;
+                sh->dv[c] = a.d != nullptr ? a.d[h * ATTN_D + c] : 0.f;
             }
             tmem_st_32x32b_x16(tl + TM_Q + part * 16, qv);
             tmem_st_wait();
@@ -474,6 +477,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             #pragma unroll
             for (int k = 0; k < 32; ++k) mx = fmaxf(mx, __uint_as_float(r[k]));
         }
+        if (threadIdx.x < ATTN_D) sh->tv[threadIdx.x] = a.t[h * ATTN_D + threadIdx.x];   // V channel scales
         sh->xm[part][row] = mx;
         named_sync_softmax();
         mx = fmaxf(fmaxf(sh->xm[0][row], sh->xm[1][row]), fmaxf(sh->xm[2][row], sh->xm[3][row]));
@@ -584,7 +588,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             if (lane == 0) {
                 tma_store_2d(&tm_z, h * ATTN_D + col, q0 + quarter * 32, box);
                 bulk_commit();
-                bulk_wait0();
+                bulk_wait_read0();           // the box has been read; the write completes with the grid
             }
             __syncwarp();
         }
