@@ -81,11 +81,17 @@ int starq_check_status(void* stream);
  *   d_sh,d_m,d_u  gate layout over transformed coordinates (Eq. 8-9):
  *           [0, d_sh) shared, [d_sh, d_sh + d_m) masked-only, the rest
  *           unmasked-only; each >= 0 and d_sh + d_m + d_u == K.
- *   bits    must be 4.
- *   Xq      [L][K/2] packed int4 codes out, 8-byte aligned.
+ *   bits    4, or 8 for the W8A8 setting (Tab. 5): the same quantiser with
+ *           127 in place of 7.
+ *   Xq      codes out, 8-byte aligned: bits 4: [L][K/2] packed int4 (low
+ *           nibble = even k); bits 8: [L][K] int8.
  *   s_a     [L] float32 per-token scales out (0 for an all-zero row).
- *   Xe      [L][K] the same codes as E4M3 bytes out (the form w4a4_gemm
- *           streams by TMA), 16-byte aligned, or NULL.
+ *   Xe      the GEMM operand out, 16-byte aligned, or NULL. bits 4: [L][K]
+ *           the codes as E4M3 bytes (the form w4a4_gemm streams by TMA).
+ *           bits 8: [L][2K], each code c split as c = 16 h + l with
+ *           l = ((c + 8) mod 16) - 8 in [-8, 7] and h in [-8, 8]: the E4M3
+ *           bytes of h in columns 0..K-1 and of l in columns K..2K-1 (the
+ *           operand of w8a8_gemm).
  *   v_dbg   [L][K] float32 transformed activations out (before rounding),
  *           16-byte aligned, or NULL.
  * Shapes: L >= 0, 16 <= K <= 20480, K % 16 == 0.
@@ -105,8 +111,9 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
  *   W       [N][K] weights, element type w_dtype (F16, BF16 or F32), 16-byte
  *           aligned.
  *   inv_a_w [K] float32 weight-side inverse smoothing or NULL (= ones).
- *   Wq      [N][K/2] packed int4 out; s_w [N] float32 out.
- * Shapes and hb as for sgat_quantize_act; bits must be 4.
+ *   Wq      codes out: bits 4: [N][K/2] packed int4; bits 8: [N][K] int8.
+ *   s_w     [N] float32 out.
+ * Shapes and hb as for sgat_quantize_act; bits 4 or 8 (127 in place of 7).
  */
 int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* inv_a_w, int hb,
                         int bits, uint8_t* Wq, float* s_w, void* stream);
@@ -125,6 +132,40 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
  * Shapes: N >= 0, K >= 32 with K % 32 == 0.
  */
 int w4_unpack_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
+
+/*
+ * w8_split_e4m3 -- 8-bit weight codes in the form w8a8_gemm reads: each code
+ * c of Wq [N][K] (int8) split as c = 16 h + l (l = ((c + 8) mod 16) - 8),
+ * We [N][2K] = E4M3 bytes of h in columns 0..K-1 and of l in K..2K-1 (both
+ * exact E4M3 numbers). Run once per weight after sgat_prepare_weight with
+ * bits = 8.
+ *   Wq, We 16-byte aligned; We caller-owned (2 N K bytes).
+ * Shapes: N >= 0, K >= 128 with K % 128 == 0.
+ */
+int w8_split_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
+
+/*
+ * w8a8_gemm -- the integer projection and its dequantisation at 8 bits (the
+ * W8A8 setting of Tab. 5; Sec. 3.2 Eq. 13, Sec. 3.1 Eq. 3):
+ *
+ *   acc[i][n] = sum_k q_a[i][k] * q_w[n][k]            (exact integer)
+ *   Y[i][n]   = (float)acc * s_a[i] * s_w[n] (+ bias[n]) rounded to y_dtype
+ *               (float32 products in that order, then one rounding).
+ *
+ *   Xe [L][2K] activation code halves (sgat_quantize_act, bits 8), We [N][2K]
+ *      weight code halves (w8_split_e4m3), 16-byte aligned.
+ *   acc = 256 (H_a H_w^T) + 16 (H_a L_w^T + L_a H_w^T) + L_a L_w^T: four FP8
+ *   tensor-core products (tcgen05 kind::f8f6f4) into three float32
+ *   accumulators, each an integer below 2^24 and so exact, combined in
+ *   int32 by the epilogue.
+ *   s_a [L], s_w [N] float32; bias [N] float32 or NULL.
+ *   Y  [L][N] out, y_dtype F16, BF16 or F32, 16-byte aligned.
+ *   acc_dbg [L][N] int32 out (the exact accumulators) or NULL.
+ * Shapes: L >= 0, N >= 128 with N % 128 == 0, 128 <= K <= 65536 with
+ * K % 128 == 0 (|acc| <= 127^2 K < 2^31).
+ */
+int w8a8_gemm(const uint8_t* Xe, const float* s_a, const uint8_t* We, const float* s_w, const float* bias, int L,
+              int N, int K, void* Y, int y_dtype, int32_t* acc_dbg, void* stream);
 
 /*
  * w4a4_gemm -- the shared-weight integer projection and its dequantisation
@@ -301,12 +342,16 @@ int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, 
  *   from w4_unpack_e4m3. Other arguments as in the calls above.
  *   K % 128 == 0.
  *   workspace: device buffer of at least sgat_linear_workspace_size(L, K,
- *   tac_M != NULL) bytes, 256-byte aligned, owned by the caller. On return it
- *   holds the intermediates, laid out as [packed codes Xq: L*K/2 bytes,
- *   padded to 256][s_a: 4*L bytes, padded to 256][E4M3 codes Xe: L*K bytes,
- *   padded to 256][TAC output: L*K values of x_dtype (room for float32), only
- *   with TAC]. The TAC output is rounded to x_dtype once, as the unquantised
- *   model stores attention outputs, and the quantiser reads it.
+ *   tac_M != NULL) bytes (bits 4) or sgat_linear_workspace_size_bits(L, K,
+ *   tac_M != NULL, bits), 256-byte aligned, owned by the caller. On return
+ *   it holds the intermediates, laid out as [codes Xq: L*K/2 bytes (bits 4)
+ *   or L*K (bits 8), padded to 256][s_a: 4*L bytes, padded to 256][GEMM
+ *   operand Xe: L*K bytes (bits 4) or 2*L*K (bits 8), padded to 256][TAC
+ *   output: L*K values of x_dtype (room for float32), only with TAC]. The
+ *   TAC output is rounded to x_dtype once, as the unquantised model stores
+ *   attention outputs, and the quantiser reads it.
+ *   bits 8 (the W8A8 setting): Wq may be NULL; We is the w8_split_e4m3
+ *   output and the GEMM is w8a8_gemm's; N % 128 == 0.
  *
  *   Programmatic launch: the kernels of sgat_linear may start while the
  *   previous kernel of the stream is still running (CUDA programmatic
@@ -318,6 +363,7 @@ int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, 
  *   (sgat_prepare_weight, w4_unpack_e4m3, tac_prepare) never let them.
  */
 size_t sgat_linear_workspace_size(int L, int K, int with_tac);
+size_t sgat_linear_workspace_size_bits(int L, int K, int with_tac, int bits);
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
                 const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,

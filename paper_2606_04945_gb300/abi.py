@@ -22,6 +22,7 @@ EXPORTED = (
     "sgat_linear_workspace_size", "sgat_linear", "starq_last_gemm_tile",
     "tac_calibrate_workspace_size", "tac_calibrate", "sgat_linear_swiglu",
     "attention_pv_tac_workspace_size", "attention_pv_tac",
+    "w8_split_e4m3", "w8a8_gemm", "sgat_linear_workspace_size_bits",
 )
 
 
@@ -44,6 +45,10 @@ def _load():
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.w8_split_e4m3.argtypes = [u8p, i, i, u8p, vp]
+    lib.w8a8_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.sgat_linear_workspace_size_bits.argtypes = [i, i, i, i]
+    lib.sgat_linear_workspace_size_bits.restype = ctypes.c_size_t
     lib.tac_prepare.argtypes = [f_p, i, i, i, vp, vp]
     lib.starq_last_gemm_tile.restype = i
     dbl = ctypes.c_double
@@ -127,6 +132,23 @@ def w4_unpack_e4m3(Wq, We, stream=None):
     _check(lib.w4_unpack_e4m3(_p(Wq), N, K, _p(We), _stream(stream)))
 
 
+def w8_split_e4m3(Wq, We, stream=None):
+    """8-bit weight codes [N][K] (int8) -> their E4M3 halves [N][2K] (once per weight)."""
+    _contig(Wq, We)
+    N, K = Wq.shape
+    _check(lib.w8_split_e4m3(_p(Wq), N, K, _p(We), _stream(stream)))
+
+
+def w8a8_gemm(Xe, s_a, We, s_w, Y, bias=None, acc_dbg=None, stream=None):
+    """Xe: activation code halves [L][2K] (sgat_quantize_act with bits=8);
+    We: weight code halves [N][2K] (w8_split_e4m3); Y [L][N]."""
+    _contig(Xe, s_a, We, s_w, Y, bias, acc_dbg)
+    L, N = Y.shape
+    K = We.shape[1] // 2
+    _check(lib.w8a8_gemm(_p(Xe), _p(s_a), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y), dtype_code(Y), _p(acc_dbg),
+                         _stream(stream)))
+
+
 def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, stream=None):
     """Xq: packed int4 codes [L][K/2] (may be None when Xe is given);
     Xe: the same codes as E4M3 bytes [L][K] (selects a TMA CTA-pair kernel);
@@ -203,8 +225,10 @@ def attention_pv_tac(Q, K, V, H, Mp, d, Z, workspace=None, dbg_codes=None, dbg_l
                                 _stream(stream)))
 
 
-def sgat_linear_workspace_size(L, K, with_tac):
-    return int(lib.sgat_linear_workspace_size(L, K, 1 if with_tac else 0))
+def sgat_linear_workspace_size(L, K, with_tac, bits=4):
+    if bits == 4:
+        return int(lib.sgat_linear_workspace_size(L, K, 1 if with_tac else 0))
+    return int(lib.sgat_linear_workspace_size_bits(L, K, 1 if with_tac else 0, bits))
 
 
 def sgat_linear(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, Y, workspace, bias=None,

@@ -8,6 +8,7 @@
 #include "common.cuh"
 #include "attn.cuh"
 #include "tac_calib.cuh"
+#include "w8a8.cuh"
 
 namespace starq {
 
@@ -93,6 +94,22 @@ int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uin
 
 constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
+int check_w8a8(const uint8_t* Xe, const float* s_a, const uint8_t* We, const float* s_w, const float* bias, int L,
+               int N, int K, void* Y, int y_dtype) {
+    if (!We || !s_w) return fail(STARQ_ERR_ARG, "w8a8_gemm: NULL We or s_w");
+    if (L > 0 && (!Xe || !s_a || !Y)) return fail(STARQ_ERR_ARG, "w8a8_gemm: NULL Xe, s_a or Y");
+    if (!dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "w8a8_gemm: unknown output dtype %d", y_dtype);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    if (N < 128 || N % 128 != 0) return fail(STARQ_ERR_SHAPE, "w8a8_gemm: N=%d: need N >= 128, N %% 128 == 0", N);
+    if (K < 128 || K % 128 != 0 || K > 65536)
+        return fail(STARQ_ERR_SHAPE, "w8a8_gemm: K=%d: need 128 <= K <= 65536 and K %% 128 == 0", K);
+    if (L == 0) return STARQ_OK;
+    if (!aligned(Xe, 16) || !aligned(We, 16) || !aligned(Y, 16) || !aligned(s_w, 16) || (bias && !aligned(bias, 16)) ||
+        !aligned(s_a, 4))
+        return fail(STARQ_ERR_ALIGN, "w8a8_gemm: Xe, We, Y, s_w, bias must be 16-byte aligned");
+    return STARQ_OK;
+}
+
 }  // namespace
 
 int report_error(int code, const char* msg) { return fail(code, "%s", msg); }
@@ -141,14 +158,14 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
                       int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg, void* stream) {
     if (L > 0 && (!X || !Xq || !s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, Xq or s_a");
     if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: unknown dtype %d", x_dtype);
-    if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
+    if (bits != 4 && bits != 8) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4- and 8-bit codes", bits);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
     int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
     if (rc) return rc;
     if (L == 0) return STARQ_OK;
     if (!aligned(X, 16) || !aligned(Xq, 8) || (v_dbg && !aligned(v_dbg, 16)) || (Xe && !aligned(Xe, 16)))
         return fail(STARQ_ERR_ALIGN, "sgat_quantize_act: X (16 B), Xq (8 B), Xe (16 B), v_dbg (16 B) alignment");
-    QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, v_dbg, Xe};
+    QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits == 8 ? 127 : 7, 1.f, Xq, s_a, v_dbg, Xe};
     cudaError_t e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "sgat_quantize_act launch");
     return STARQ_OK;
@@ -158,14 +175,14 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
                         int bits, uint8_t* Wq, float* s_w, void* stream) {
     if (N > 0 && (!W || !Wq || !s_w)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: NULL W, Wq or s_w");
     if (!dtype_ok(w_dtype)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: unknown dtype %d", w_dtype);
-    if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
+    if (bits != 4 && bits != 8) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4- and 8-bit codes", bits);
     if (N < 0) return fail(STARQ_ERR_SHAPE, "N=%d < 0", N);
     int rc = check_transform(K, hb, K, 0, 0, nullptr, inv_a_w);
     if (rc) return rc;
     if (N == 0) return STARQ_OK;
     if (!aligned(W, 16) || !aligned(Wq, 8))
         return fail(STARQ_ERR_ALIGN, "sgat_prepare_weight: W (16 B), Wq (8 B) alignment");
-    QuantArgs a{W, w_dtype, N, K, nullptr, nullptr, inv_a_w, hb, K, 0, 0, 7, 1.f / (float)hb,
+    QuantArgs a{W, w_dtype, N, K, nullptr, nullptr, inv_a_w, hb, K, 0, 0, bits == 8 ? 127 : 7, 1.f / (float)hb,
                 Wq, s_w, nullptr};
     cudaError_t e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "sgat_prepare_weight launch");
@@ -193,6 +210,30 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
     GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe, Xe ? We : nullptr};
     cudaError_t e = launch_w4a4_gemm(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm launch");
+    return STARQ_OK;
+}
+
+int w8_split_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream) {
+    if (N > 0 && (!Wq || !We)) return fail(STARQ_ERR_ARG, "w8_split_e4m3: NULL Wq or We");
+    if (N < 0 || K < 128 || K % 128 != 0) return fail(STARQ_ERR_SHAPE, "w8_split_e4m3: N=%d K=%d (K %% 128 == 0)", N, K);
+    if (N == 0) return STARQ_OK;
+    if (!aligned(Wq, 16) || !aligned(We, 16)) return fail(STARQ_ERR_ALIGN, "w8_split_e4m3: Wq, We alignment");
+    cudaError_t e = launch_w8_split(Wq, We, (size_t)N, K, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w8_split_e4m3 launch");
+    return STARQ_OK;
+}
+
+int w8a8_gemm(const uint8_t* Xe, const float* s_a, const uint8_t* We, const float* s_w, const float* bias, int L,
+              int N, int K, void* Y, int y_dtype, int32_t* acc_dbg, void* stream) {
+    int rc = check_w8a8(Xe, s_a, We, s_w, bias, L, N, K, Y, y_dtype);
+    if (rc) return rc;
+    if (L == 0) return STARQ_OK;
+    if (acc_dbg && !aligned(acc_dbg, 16)) return fail(STARQ_ERR_ALIGN, "acc_dbg must be 16-byte aligned");
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    GemmArgs a{nullptr, s_a, nullptr, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe, We};
+    cudaError_t e = launch_w8a8_gemm(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w8a8_gemm launch");
     return STARQ_OK;
 }
 
@@ -315,11 +356,19 @@ int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, 
     return STARQ_OK;
 }
 
-size_t sgat_linear_workspace_size(int L, int K, int with_tac) {
-    if (L < 0 || K < 0) return 0;
-    size_t n = align256((size_t)L * K / 2) + align256((size_t)L * 4) + align256((size_t)L * K);
+size_t sgat_linear_workspace_size_bits(int L, int K, int with_tac, int bits) {
+    if (L < 0 || K < 0 || (bits != 4 && bits != 8)) return 0;
+    // codes (packed nibbles or bytes), s_a, the GEMM operand (E4M3 codes or
+    // the E4M3 halves of 8-bit codes), TAC output
+    const size_t q = bits == 8 ? (size_t)L * K : (size_t)L * K / 2;
+    const size_t e = bits == 8 ? (size_t)L * K * 2 : (size_t)L * K;
+    size_t n = align256(q) + align256((size_t)L * 4) + align256(e);
     if (with_tac) n += align256((size_t)L * K * 4);
     return n;
+}
+
+size_t sgat_linear_workspace_size(int L, int K, int with_tac) {
+    return sgat_linear_workspace_size_bits(L, K, with_tac, 4);
 }
 
 }  // extern "C"
@@ -333,24 +382,28 @@ int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* ma
     if ((!Wq && !We) || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear: NULL Wq/We or s_w");
     if (L > 0 && (!X || !Y || !workspace)) return fail(STARQ_ERR_ARG, "sgat_linear: NULL X, Y or workspace");
     if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear: unknown dtype");
-    if (bits != 4) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4-bit codes", bits);
+    if (bits != 4 && bits != 8) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4- and 8-bit codes", bits);
+    if (bits == 8 && swiglu) return fail(STARQ_ERR_BITS, "sgat_linear_swiglu: 4-bit codes only");
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
     int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
     if (rc) return rc;
     if (tac_M && (rc = check_tac(L, K, tac_g, tac_M, tac_d))) return rc;
     if (tac_M && (rc = check_tac_prepared(tac_Mp, x_dtype, tac_g))) return rc;
     if (L == 0) return STARQ_OK;
-    const size_t need = sgat_linear_workspace_size(L, K, tac_M != nullptr);
+    const size_t need = sgat_linear_workspace_size_bits(L, K, tac_M != nullptr, bits);
     if (workspace_bytes < need)
         return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu needed", workspace_bytes, need);
     if (!aligned(workspace, 256) || !aligned(X, 16)) return fail(STARQ_ERR_ALIGN, "sgat_linear alignment");
+    const size_t qbytes = bits == 8 ? (size_t)L * K : (size_t)L * K / 2;
+    const size_t ebytes = bits == 8 ? (size_t)L * K * 2 : (size_t)L * K;
     uint8_t* ws = static_cast<uint8_t*>(workspace);
     uint8_t* Xq = ws;
-    float* s_a = reinterpret_cast<float*>(ws + align256((size_t)L * K / 2));
-    uint8_t* Xe = ws + align256((size_t)L * K / 2) + align256((size_t)L * 4);
+    float* s_a = reinterpret_cast<float*>(ws + align256(qbytes));
+    uint8_t* Xe = ws + align256(qbytes) + align256((size_t)L * 4);
     // TAC output in the input's type (the region has room for float32)
-    void* zt = tac_M ? static_cast<void*>(Xe + align256((size_t)L * K)) : nullptr;
-    rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
+    void* zt = tac_M ? static_cast<void*>(Xe + align256(ebytes)) : nullptr;
+    rc = bits == 8 ? check_w8a8(Xe, s_a, We, s_w, bias, L, N, K, Y, y_dtype)
+                   : check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
@@ -365,8 +418,13 @@ int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* ma
         qin = zt;
         qin_dtype = x_dtype;
     }
-    QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
+    QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits == 8 ? 127 : 7, 1.f, Xq, s_a, nullptr, Xe};
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");
+    if (bits == 8) {
+        GemmArgs g8{nullptr, s_a, nullptr, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
+        if ((e = launch_w8a8_gemm(g8, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: w8a8 gemm launch");
+        return STARQ_OK;
+    }
     GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
     // the GEMM's predecessor is the quantiser launched above, which waits for
     // everything before it and does not write the weights

@@ -61,7 +61,7 @@ extern "C" int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, con
                                    int d_u, const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
                                    const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N,
                                    int bits, void* Y, int y_dtype, void* stream) {
-    const size_t need = sgat_linear_workspace_size(L, K, tac_M != nullptr);
+    const size_t need = sgat_linear_workspace_size_bits(L, K, tac_M != nullptr, bits);
     if (L > 0 && need > (size_t)STARQ_NOALLOC_SCRATCH_BYTES) {
         char msg[160];
         snprintf(msg, sizeof(msg),

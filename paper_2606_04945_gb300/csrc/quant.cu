@@ -12,7 +12,16 @@
 // (a, b) -> (a + b, a - b) in float32 round-to-nearest; every float operation
 // is an explicit round-to-nearest intrinsic, so nothing is contracted into an
 // FMA and the values match the reference network bit for bit. With qmax = 7
-// no clamp is needed: |fl(v * r)| <= 7 (1 + 2^-24)^2 < 7.5.
+// no clamp is needed: |fl(v * r)| <= 7 (1 + 2^-24)^2 < 7.5 (likewise 127.5
+// for qmax = 127).
+//
+// Storage by code width. qmax <= 7 (4-bit): Xq packs two codes per byte and
+// Xe holds each code as an E4M3 byte [rows][K]. qmax = 127 (8-bit, the W8A8
+// setting of Tab. 5): Xq holds one code per byte (two's complement) and Xe
+// [rows][2K] holds the nibble split c = 16 h + l, l = ((c + 8) mod 16) - 8 in
+// [-8, 7], h = (c - l) / 16 in [-8, 8]: E4M3 bytes of h in columns 0..K-1
+// and of l in columns K..2K-1 (both exact in E4M3), the operands of the
+// 8-bit GEMM.
 //
 // Work split: a warp owns a chunk of C = 32 E consecutive elements of a row
 // (C = 1024 when hb >= 1024, else C = 512 holding 512 / hb Hadamard blocks).
@@ -145,6 +154,28 @@ __device__ __forceinline__ void chunk_fwht(float (&v)[E], int hb, int lane, floa
     __syncwarp();
 }
 
+// Eight 8-bit codes -> their bytes (two's complement, code k in byte k) and
+// the E4M3 bytes of their split c = 16 h + l (see the file comment).
+__device__ __forceinline__ void split_codes8(const int* q, uint2& bytes, uint2& eh, uint2& el) {
+    uint32_t b0 = 0, b1 = 0;
+    #pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        b0 |= (uint32_t)(q[k] & 0xFF) << (8 * k);
+        b1 |= (uint32_t)(q[k + 4] & 0xFF) << (8 * k);
+    }
+    bytes = make_uint2(b0, b1);
+    uint16_t hh[4], ll[4];
+    #pragma unroll
+    for (int k = 0; k < 4; ++k) {        // upper byte from the first operand
+        const int l0 = ((q[2 * k] + 8) & 15) - 8, l1 = ((q[2 * k + 1] + 8) & 15) - 8;
+        const int h0 = (q[2 * k] - l0) >> 4, h1 = (q[2 * k + 1] - l1) >> 4;
+        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(hh[k]) : "f"((float)h1), "f"((float)h0));
+        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(ll[k]) : "f"((float)l1), "f"((float)l0));
+    }
+    eh = make_uint2((uint32_t)hh[0] | ((uint32_t)hh[1] << 16), (uint32_t)hh[2] | ((uint32_t)hh[3] << 16));
+    el = make_uint2((uint32_t)ll[0] | ((uint32_t)ll[1] << 16), (uint32_t)ll[2] | ((uint32_t)ll[3] << 16));
+}
+
 // Eight codes (int, |q| <= 7) -> packed nibbles, code k in bits 4k..4k+3.
 __device__ __forceinline__ uint32_t pack8(const int* q) {
     uint32_t w = 0;
@@ -264,6 +295,22 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
         const int c = wr + j * warps_per_row;
         const int lo = c * C + E * lane;
         if (c >= nchunks || lo >= K) continue;
+        if (a.qmax > 7) {                // 8-bit codes: bytes and their E4M3 split
+            #pragma unroll
+            for (int u = 0; u < E / 8; ++u) {
+                int q[8];
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) q[k] = __float2int_rn(__fmul_rn(v[j][8 * u + k], r));
+                uint2 bytes, eh, el;
+                split_codes8(q, bytes, eh, el);
+                *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + lo + 8 * u) = bytes;
+                if (a.Xe != nullptr) {
+                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + lo + 8 * u) = eh;
+                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + lo + 8 * u) = el;
+                }
+            }
+            continue;
+        }
         uint32_t packed[E / 8];
         #pragma unroll
         for (int u = 0; u < E / 8; ++u) {
@@ -571,6 +618,16 @@ sgat_quant_rows_kernel(QuantArgs a) {
             #pragma unroll
             for (int k = 0; k < 8; k += 2)
                 quant_pair(v[R][8 * j + k], v[R][8 * j + k + 1], r, qf[k], qf[k + 1], qi[k], qi[k + 1]);
+            if (a.qmax > 7) {            // 8-bit codes: bytes and their E4M3 split
+                uint2 bytes, eh, el;
+                split_codes8(qi, bytes, eh, el);
+                *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + e0) = bytes;
+                if (a.Xe != nullptr) {
+                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + e0) = eh;
+                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + e0) = el;
+                }
+                continue;
+            }
             uint32_t nib;
             uint2 e4;
             pack_codes8(qf, qi, nib, e4);

@@ -55,7 +55,7 @@ P = ctypes.c_void_p(4096)  # a non-null, 16-byte-aligned stand-in; never derefer
 @pytest.mark.parametrize("args,code", [
     ((None, 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -1),   # NULL X
     ((P, 9, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -1),      # dtype
-    ((P, 0, 4, 512, None, None, None, 512, 512, 0, 0, 8, P, P, None, None, None), -4),      # bits
+    ((P, 0, 4, 512, None, None, None, 512, 512, 0, 0, 6, P, P, None, None, None), -4),      # bits (4 or 8)
     ((P, 0, 4, 100, None, None, None, 4, 100, 0, 0, 4, P, P, None, None, None), -2),        # K % 16
     ((P, 0, 4, 512, None, None, None, 384, 512, 0, 0, 4, P, P, None, None, None), -2),      # hb not pow2
     ((P, 0, 4, 512, None, None, None, 8192, 512, 0, 0, 4, P, P, None, None, None), -2),     # hb > K
@@ -66,6 +66,33 @@ P = ctypes.c_void_p(4096)  # a non-null, 16-byte-aligned stand-in; never derefer
 def test_quantize_act_validation(lib, args, code):
     assert lib.lib.sgat_quantize_act(*args) == code
     assert lib.lib.starq_last_error()
+
+
+@pytest.mark.parametrize("L,N,K,code", [(4, 96, 512, -2), (4, 256, 200, -2), (4, 256, 131072, -2),
+                                        (-1, 256, 512, -2), (4, 256, 512, -1)])
+def test_w8a8_gemm_validation(lib, L, N, K, code):
+    """8-bit GEMM: N % 128, K % 128, K <= 65536, L >= 0; NULL Xe with L > 0."""
+    Xe = None if code == -1 else P
+    assert lib.lib.w8a8_gemm(Xe, P, P, P, None, L, N, K, P, 0, None, None) == code
+    assert lib.lib.starq_last_error()
+
+
+def test_w8_split_validation(lib):
+    assert lib.lib.w8_split_e4m3(P, 4, 200, P, None) == -2          # K % 128
+    assert lib.lib.w8_split_e4m3(ctypes.c_void_p(4100), 4, 256, P, None) == -3
+    assert lib.lib.w8_split_e4m3(P, 0, 256, P, None) == 0           # nothing to do
+
+
+def test_linear_workspace_by_bits(lib):
+    """8-bit codes take a byte each and their E4M3 halves two; 4-bit codes
+    half a byte and one."""
+    L, K = 1000, 4096
+    a256 = lambda x: (x + 255) // 256 * 256
+    assert lib.lib.sgat_linear_workspace_size_bits(L, K, 0, 4) == lib.lib.sgat_linear_workspace_size(L, K, 0)
+    assert lib.lib.sgat_linear_workspace_size_bits(L, K, 0, 8) == a256(L * K) + a256(4 * L) + a256(2 * L * K)
+    assert lib.lib.sgat_linear_workspace_size_bits(L, K, 1, 8) == (a256(L * K) + a256(4 * L) + a256(2 * L * K)
+                                                                   + a256(4 * L * K))
+    assert lib.lib.sgat_linear_workspace_size_bits(L, K, 0, 6) == 0
 
 
 @pytest.mark.parametrize("L,N,K,code", [(4, 100, 512, -2), (4, 256, 200, -2), (4, 256, 131072, -2),
