@@ -15,10 +15,16 @@
 // float32 accumulation of the tensor cores is exact. The combination runs in
 // int32 (|acc| <= 127^2 K < 2^31).
 //
-// One CTA per 128 x 128 output tile: four epilogue warps (one TMEM lane
-// quarter each), a TMA warp and an MMA warp. A pipeline stage holds the
-// four 128 x 128-byte tiles (H_a, L_a, H_w, L_w) of one 128-wide K block
-// (64 KB, 128-byte swizzle); three stages. Every wait is bounded.
+// One CTA per 128 x 128 output tile; the row tiles of one weight tile are
+// consecutive in the grid, so a weight tile leaves DRAM once. Four epilogue
+// warps (one TMEM lane quarter each), a TMA warp and an MMA warp. A
+// pipeline stage holds the four 128 x 128-byte tiles (H_a, L_a, H_w, L_w)
+// of one 128-wide K block (64 KB, 128-byte swizzle); three stages. Every
+// MMA reads both operands from shared memory, whose bandwidth bounds the
+// kernel: 192 KB per K block (16 MMAs of 8 KB, 64 KB of TMA writes) against
+// 1024 cycles of MMA. (Copying the activation halves into TMEM first, so
+// the MMAs read them there, was slower: eight more tcgen05 instructions per
+// K block made the single issuing thread the bound.) Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -91,7 +97,7 @@ w8a8_gemm_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tm_a, const __g
     const uint32_t base = (raw + 1023u) & ~1023u;
     W8Sm* sh = reinterpret_cast<W8Sm*>(smem_raw + (base - raw) + (size_t)W8_STAGES * W8_STAGE);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n0 = blockIdx.x * W8_BN, m0 = blockIdx.y * W8_BM;
+    const int m0 = blockIdx.x * W8_BM, n0 = blockIdx.y * W8_BN;
     const int K = a.K, nkb = K / W8_BK;
     volatile int* abort = &sh->abort;
     auto B = [](const uint64_t& bar) { return smem_addr(&bar); };
@@ -266,7 +272,7 @@ cudaError_t launch_typed(const GemmArgs& a, const CUtensorMap& ta, const CUtenso
         if (e != cudaSuccess) return e;
         attr_set[dev] = true;
     }
-    const dim3 grid(a.N / W8_BN, (a.L + W8_BM - 1) / W8_BM);
+    const dim3 grid((a.L + W8_BM - 1) / W8_BM, a.N / W8_BN);
     w8a8_gemm_kernel<TOut><<<grid, W8_THREADS, W8_SMEM, stream>>>(a, ta, tw);
     return cudaGetLastError();
 }
