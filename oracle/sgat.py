@@ -15,6 +15,12 @@ Readings of the paper taken here (each is listed in the design doc):
   ``round`` is round-half-to-even. The scale form is s = amax / qmax and the
   code is rne(v * r) with r = qmax / amax, both in float32. An all-zero row
   gets s = 0 and all-zero codes.
+* The asymmetric member (Eq. 2-4), for activations: per row, X_min and
+  X_max are the row's extremes with zero included (X_min <= 0 <= X_max, so
+  z stays in [0, 2^b - 1]); s = fl(fl(X_max - X_min) / (2^b - 1)); X / s is
+  taken as fl(v * r) with r = fl((2^b - 1) / fl(X_max - X_min)), like the
+  symmetric reading; z = rne(fl(-X_min * r)); codes clamp(rne(fl(v r)) + z,
+  0, 2^b - 1). An all-zero row gets s = 0, z = 0 and all-zero codes.
 * P is the block-diagonal Sylvester Hadamard matrix of block ``hb`` preceded
   by a per-state diagonal smoothing ``a_s``: Phi_s(x) = ((x * a_s) H) G_s with
   the unnormalised H; the 1/hb that makes H^-1 = H / hb is folded into the
@@ -115,6 +121,29 @@ def quantize_rows_sym(v, bits):
     return q, s
 
 
+def quantize_rows_asym(v, bits):
+    """Per-row asymmetric quantiser (Eq. 2-4, read as in the module notes).
+
+    Returns (codes int32 [rows, K] in [0, 2^b - 1], s float32 [rows],
+    z int32 [rows]); X_hat = s (codes - z) (Eq. 3).
+    """
+    v = np.asarray(v, dtype=F32)
+    assert v.ndim == 2
+    assert np.all(np.isfinite(v)), "the quantiser is defined on finite inputs"
+    levels = F32((1 << bits) - 1)
+    vmax = np.maximum(v.max(axis=1), F32(0)) if v.shape[1] else np.zeros(v.shape[0], F32)
+    vmin = np.minimum(v.min(axis=1), F32(0)) if v.shape[1] else np.zeros(v.shape[0], F32)
+    d = (vmax - vmin).astype(F32)
+    nz = d > 0
+    safe = np.where(nz, d, F32(1))
+    s = np.where(nz, safe / levels, F32(0)).astype(F32)
+    r = np.where(nz, levels / safe, F32(0)).astype(F32)
+    z = np.clip(np.rint((-vmin * r).astype(F32)), 0, levels).astype(np.int32)
+    prod = (v * r[:, None]).astype(F32)
+    q = np.clip(np.rint(prod) + z[:, None], 0, levels).astype(np.int32)
+    return q, s, z
+
+
 def pack_int4(q):
     """Pack int4 codes [rows, K] into bytes [rows, K/2].
 
@@ -211,6 +240,25 @@ def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits):
     return codes, s_a
 
 
+def sgat_quantize_act_asym(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits=4):
+    """As sgat_quantize_act with the asymmetric activation quantiser.
+    Returns (codes int32 [L, K] in [0, 2^b - 1], s_a float32 [L], z_a int32
+    [L])."""
+    X = np.asarray(X)
+    L, K = X.shape
+    g_m, g_u = state_gates(K, d_sh, d_m, d_u)
+    I_m, I_u = state_index_sets(mask)
+    codes = np.zeros((L, K), dtype=np.int32)
+    s_a = np.zeros(L, dtype=F32)
+    z_a = np.zeros(L, dtype=np.int32)
+    for I, a, g in ((I_m, a_m, g_m), (I_u, a_u, g_u)):
+        if len(I) == 0:
+            continue
+        q, s, z = quantize_rows_asym(phi_state(X[I], a, g, hb), bits)
+        codes[I], s_a[I], z_a[I] = q, s, z
+    return codes, s_a, z_a
+
+
 def sgat_transform(X, mask, a_m, a_u, hb, d_sh, d_m, d_u):
     """Phi_s(X^s) for both states in token order, float32, unquantised."""
     X = np.asarray(X)
@@ -251,6 +299,15 @@ def dequant(acc, s_a, s_w, bias=None):
     if bias is not None:
         y = y + np.asarray(bias, dtype=np.float64)[None, :]
     return y
+
+
+def sgat_linear_asym(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, qw, s_w, bias=None, bits=4):
+    """Y_hat with asymmetric activation codes and symmetric weight codes:
+    Y = s_a s_w sum_k (q_a - z_a) q_w (Eq. 3 and Eq. 5). Returns (Y float64
+    [L, N], codes, s_a, z_a, acc int64 [L, N] = sum_k (q_a - z_a) q_w)."""
+    codes, s_a, z_a = sgat_quantize_act_asym(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits)
+    acc = int_gemm(codes - z_a[:, None], qw)
+    return dequant(acc, s_a, s_w, bias), codes, s_a, z_a, acc
 
 
 def sgat_linear(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, qw, s_w, bias=None, bits=4):

@@ -528,3 +528,106 @@ def test_attention_tac_identity():
     M = np.broadcast_to(np.eye(d), (H, d, d))
     Zt, Z = oatt.attention_tac(Q, K, V, M, np.zeros((H, d)), H, d)
     assert np.array_equal(Zt, Z)
+
+
+# ---------------------------------------------------------------------------
+# Asymmetric activation quantiser (Eq. 2-4) and its linear
+# ---------------------------------------------------------------------------
+
+def test_asym_quant_worked_example():
+    """Eq. 4 on v = (-1, 0.5, 2, 0), b = 4, worked by hand: X_max - X_min = 3,
+    s = 3/15 = 0.2, X / s = 5 v, z = round(1 / 0.2) = 5; Eq. 2 gives
+    round(-5) + 5 = 0, round(2.5) + 5 = 2 + 5 (half to even), round(10) + 5 =
+    15, 0 + 5 = 5."""
+    q, s, z = sgat.quantize_rows_asym(np.array([[-1.0, 0.5, 2.0, 0.0]], F32), 4)
+    assert q.tolist() == [[0, 7, 15, 5]] and z.tolist() == [5]
+    assert s[0] == F32(0.2)
+
+
+def _brute_asym_row(a, k, m, bits):
+    """Row with X_min = -a 2^-k, X_max = (L - a) 2^-k (L = 2^b - 1) and inner
+    values m 2^-k / 2, all exact: v / s = v 2^k is exact. The code of v is the
+    integer of [0, L] minimising |s (q - z) - v| = 2^-k |q - a - v 2^k|,
+    ties to the even integer before the shift by z = a, which is Eq. 2 with
+    round-half-even."""
+    levels = (1 << bits) - 1
+    vals = [-a, levels - a] + [mm / 2 for mm in m]
+    v = np.array([x * 2.0 ** -k for x in vals], dtype=F32)
+    want = []
+    for x in vals:
+        best = None
+        for n in range(-2 * levels, 2 * levels + 1):            # n = round(v / s) candidate
+            d = abs(n - x)
+            if best is None or d < best[0] - 1e-12 or (abs(d - best[0]) <= 1e-12 and n % 2 == 0):
+                best = (d, n)
+        want.append(min(max(best[1] + a, 0), levels))
+    return v, want, a
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+def test_asym_quant_brute_force(bits):
+    rng = np.random.default_rng(40 + bits)
+    levels = (1 << bits) - 1
+    for _ in range(60):
+        a = int(rng.integers(0, levels + 1))
+        k = int(rng.integers(-3, 6))
+        m = rng.integers(-2 * a, 2 * (levels - a) + 1, 9)
+        v, want, z_want = _brute_asym_row(a, k, m, bits)
+        q, s, z = sgat.quantize_rows_asym(v[None], bits)
+        assert q[0].tolist() == want and z[0] == z_want, (a, k, m.tolist(), bits)
+        assert s[0] == F32(2.0 ** -k)
+
+
+def test_asym_quant_invariants():
+    """Random rows: codes in [0, 15], z in [0, 15]; dequantisation (Eq. 3)
+    within half a step (no clamping: the range holds every value); an
+    all-zero row gives s = 0, z = 0, codes 0; a row with X_max = -X_min has
+    z = round(7.5) = 8; a row of positive values has z = 0 (zero is in the
+    range)."""
+    rng = np.random.default_rng(7)
+    v = (rng.standard_normal((64, 96)) * rng.uniform(0.01, 10, (64, 1))).astype(F32)
+    v[3] = 0
+    v[5] = np.abs(v[5])
+    v[6, :2] = [2.5, -2.5]
+    v[6, 2:] = np.clip(v[6, 2:], -2.5, 2.5)
+    q, s, z = sgat.quantize_rows_asym(v, 4)
+    assert q.min() >= 0 and q.max() <= 15 and z.min() >= 0 and z.max() <= 15
+    deq = s.astype(np.float64)[:, None] * (q - z[:, None])
+    assert np.all(np.abs(deq - v) <= 0.5 * s.astype(np.float64)[:, None] * (1 + 1e-5) + 1e-30)
+    assert s[3] == 0 and z[3] == 0 and not q[3].any()
+    assert z[5] == 0 and q[5].min() == 0
+    assert z[6] == 8
+
+
+def test_asym_linear_16bit_reproduces_fp_matmul():
+    """P = I, all gates on, b = 16 for both quantisers: Y_hat = s_a s_w
+    sum_k (q_a - z_a) q_w must equal X W^T within the quantisation bound.
+    Dropping the zero point, or subtracting it with the wrong sign, misses
+    by the size of z times the weight row sums."""
+    X, W, mask = _case()
+    K = X.shape[1]
+    qw, s_w = sgat.prepare_weight(W, None, 1, 16)
+    Y, codes, s_a, z_a, acc = sgat.sgat_linear_asym(X, mask, None, None, 1, K, 0, 0, qw, s_w, bits=16)
+    ref = X.astype(np.float64) @ W.astype(np.float64).T
+    ea = 0.5 * s_a.astype(np.float64)[:, None]
+    ew = 0.5 * s_w.astype(np.float64)[None, :]
+    bound = (ea * np.abs(W).astype(np.float64).sum(1)[None, :]
+             + ew * np.abs(X).astype(np.float64).sum(1)[:, None] + K * ea * ew)
+    assert np.all(np.abs(Y - ref) <= bound * 1.0001 + 1e-12)
+    assert np.linalg.norm(Y - ref) / np.linalg.norm(ref) < 2e-4
+    assert z_a.max() > 1000                                  # the zero point matters here
+
+
+def test_asym_linear_triple_loop():
+    """acc = sum_k (q_a - z_a) q_w by explicit loops on a tiny case."""
+    rng = np.random.default_rng(3)
+    X = rng.standard_normal((5, 16)).astype(F32)
+    W = rng.standard_normal((3, 16)).astype(F32)
+    qw, s_w = sgat.prepare_weight(W, None, 16, 4)
+    mask = np.array([0, 1, 0, 1, 1], np.uint8)
+    Y, codes, s_a, z_a, acc = sgat.sgat_linear_asym(X, mask, None, None, 16, 8, 4, 4, qw, s_w)
+    for i in range(5):
+        for n in range(3):
+            want = sum((int(codes[i, k]) - int(z_a[i])) * int(qw[n, k]) for k in range(16))
+            assert acc[i, n] == want
+            assert Y[i, n] == float(want) * float(s_a[i]) * float(s_w[n])
