@@ -168,6 +168,45 @@ int w8a8_gemm(const uint8_t* Xe, const float* s_a, const uint8_t* We, const floa
               int N, int K, void* Y, int y_dtype, int32_t* acc_dbg, void* stream);
 
 /*
+ * Asymmetric activation quantisation (Eq. 2-4) with symmetric per-channel
+ * weights, through the 4-bit GEMM.
+ *
+ * sgat_quantize_act_asym -- sgat_quantize_act with the asymmetric 4-bit
+ * quantiser per token: X_min = min(min v, 0), X_max = max(max v, 0) (zero
+ * is inside the range), s = (X_max - X_min) / 15, r = 15 / (X_max - X_min),
+ * z = rne(-X_min r) in [0, 15], q = clamp(rne(v r) + z, 0, 15), all in
+ * float32; an all-zero row gets s = 0, z = 0, codes 0. X_hat = s (q - z).
+ *   Xq  [L][K/2] packed unsigned nibbles out (low nibble = even k).
+ *   s_a [L] float32 out, z_a [L] int32 out.
+ *   Xe  [L][K + 128] out or NULL: the codes as E4M3 bytes, then 128 bytes
+ *       of E4M3(-z) (the zero-point columns); K % 128 == 0 and K <= 7680.
+ * Other arguments as for sgat_quantize_act.
+ *
+ * w4_zero_point_columns -- symmetric 4-bit weight codes Wq [N][K/2] (from
+ * sgat_prepare_weight) to We [N][K + 128]: the codes as E4M3 bytes, then
+ * 128 E4M3 values whose sum is exactly sum_k q_w[n][k]. With the
+ * activations' zero-point columns, the GEMM over K + 128 computes
+ * sum_k (q_a - z) q_w exactly. K % 128 == 0, K <= 7680 (128 E4M3 values of
+ * at most 448 hold |sum| <= 7 K).
+ *
+ * sgat_linear_asym -- the fused linear with asymmetric activation codes:
+ *   Y = (float)acc * s_a[i] * s_w[n] (+ bias), acc = sum_k (q_a - z_a) q_w,
+ * i.e. sgat_quantize_act_asym then w4a4_gemm(Xe, We, K + 128). workspace:
+ * sgat_linear_asym_workspace_size(L, K) bytes, 256-byte aligned, laid out
+ * as [Xq L*K/2][s_a 4L][z_a 4L][Xe L*(K+128)], each part padded to 256.
+ * N >= 32 with N % 32 == 0.
+ */
+int sgat_quantize_act_asym(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                           const float* a_u, int hb, int d_sh, int d_m, int d_u, uint8_t* Xq, float* s_a,
+                           int32_t* z_a, uint8_t* Xe, void* stream);
+int w4_zero_point_columns(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
+size_t sgat_linear_asym_workspace_size(int L, int K);
+int sgat_linear_asym(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                     const float* a_u, int hb, int d_sh, int d_m, int d_u, const uint8_t* We, const float* s_w,
+                     const float* bias, int N, void* Y, int y_dtype, void* workspace, size_t workspace_bytes,
+                     void* stream);
+
+/*
  * w4a4_gemm -- the shared-weight integer projection and its dequantisation
  * (Sec. 3.2 Eq. 13, Sec. 3.1 Eq. 5 and Eq. 3).
  *

@@ -23,6 +23,7 @@ EXPORTED = (
     "tac_calibrate_workspace_size", "tac_calibrate", "sgat_linear_swiglu",
     "attention_pv_tac_workspace_size", "attention_pv_tac",
     "w8_split_e4m3", "w8a8_gemm", "sgat_linear_workspace_size_bits",
+    "sgat_quantize_act_asym", "w4_zero_point_columns", "sgat_linear_asym_workspace_size", "sgat_linear_asym",
 )
 
 
@@ -49,6 +50,12 @@ def _load():
     lib.w8a8_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.sgat_linear_workspace_size_bits.argtypes = [i, i, i, i]
     lib.sgat_linear_workspace_size_bits.restype = ctypes.c_size_t
+    lib.sgat_quantize_act_asym.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, u8p, f_p, vp, u8p, vp]
+    lib.w4_zero_point_columns.argtypes = [u8p, i, i, u8p, vp]
+    lib.sgat_linear_asym_workspace_size.argtypes = [i, i]
+    lib.sgat_linear_asym_workspace_size.restype = ctypes.c_size_t
+    lib.sgat_linear_asym.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, u8p, f_p, f_p, i, vp, i, vp,
+                                     ctypes.c_size_t, vp]
     lib.tac_prepare.argtypes = [f_p, i, i, i, vp, vp]
     lib.starq_last_gemm_tile.restype = i
     dbl = ctypes.c_double
@@ -130,6 +137,38 @@ def w4_unpack_e4m3(Wq, We, stream=None):
     _contig(Wq, We)
     N, K = We.shape
     _check(lib.w4_unpack_e4m3(_p(Wq), N, K, _p(We), _stream(stream)))
+
+
+def sgat_quantize_act_asym(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, z_a, Xe=None, stream=None):
+    """Asymmetric 4-bit activation codes (Eq. 2-4): Xq [L][K/2] unsigned
+    nibbles, s_a [L], z_a [L] int32; Xe [L][K + 128] E4M3 codes + zero-point
+    columns."""
+    _contig(X, mask, a_m, a_u, Xq, s_a, z_a, Xe)
+    L, K = X.shape
+    _check(lib.sgat_quantize_act_asym(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh, d_m, d_u,
+                                      _p(Xq), _p(s_a), _p(z_a), _p(Xe), _stream(stream)))
+
+
+def w4_zero_point_columns(Wq, We, stream=None):
+    """Packed 4-bit weight codes [N][K/2] -> E4M3 rows [N][K + 128] (codes,
+    then 128 values summing to the row's code sum)."""
+    _contig(Wq, We)
+    N = Wq.shape[0]
+    K = We.shape[1] - 128
+    _check(lib.w4_zero_point_columns(_p(Wq), N, K, _p(We), _stream(stream)))
+
+
+def sgat_linear_asym_workspace_size(L, K):
+    return int(lib.sgat_linear_asym_workspace_size(L, K))
+
+
+def sgat_linear_asym(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, We, s_w, Y, workspace, bias=None, stream=None):
+    _contig(X, mask, a_m, a_u, We, s_w, Y, workspace, bias)
+    L, K = X.shape
+    N = We.shape[0]
+    _check(lib.sgat_linear_asym(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh, d_m, d_u,
+                                _p(We), _p(s_w), _p(bias), N, _p(Y), dtype_code(Y), _p(workspace),
+                                workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def w8_split_e4m3(Wq, We, stream=None):

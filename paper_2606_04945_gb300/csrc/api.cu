@@ -9,6 +9,7 @@
 #include "attn.cuh"
 #include "tac_calib.cuh"
 #include "w8a8.cuh"
+#include "asym.cuh"
 
 namespace starq {
 
@@ -210,6 +211,81 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
     GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe, Xe ? We : nullptr};
     cudaError_t e = launch_w4a4_gemm(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm launch");
+    return STARQ_OK;
+}
+
+int sgat_quantize_act_asym(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                           const float* a_u, int hb, int d_sh, int d_m, int d_u, uint8_t* Xq, float* s_a,
+                           int32_t* z_a, uint8_t* Xe, void* stream) {
+    if (L > 0 && (!X || !Xq || !s_a || !z_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act_asym: NULL X, Xq, s_a or z_a");
+    if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act_asym: unknown dtype %d", x_dtype);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
+    if (rc) return rc;
+    if (Xe && (K % 128 != 0 || K > ASYM_MAX_K))
+        return fail(STARQ_ERR_SHAPE, "sgat_quantize_act_asym: K=%d: Xe needs K %% 128 == 0 and K <= %d", K, ASYM_MAX_K);
+    if (L == 0) return STARQ_OK;
+    if (!aligned(X, 16) || !aligned(Xq, 8) || !aligned(z_a, 4) || (Xe && !aligned(Xe, 16)))
+        return fail(STARQ_ERR_ALIGN, "sgat_quantize_act_asym: X (16 B), Xq (8 B), z_a (4 B), Xe (16 B) alignment");
+    QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 15, 1.f, Xq, s_a, nullptr, Xe};
+    a.asym = 1;
+    a.z = z_a;
+    cudaError_t e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "sgat_quantize_act_asym launch");
+    return STARQ_OK;
+}
+
+int w4_zero_point_columns(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream) {
+    if (N > 0 && (!Wq || !We)) return fail(STARQ_ERR_ARG, "w4_zero_point_columns: NULL Wq or We");
+    if (N < 0 || K < 128 || K % 128 != 0 || K > ASYM_MAX_K)
+        return fail(STARQ_ERR_SHAPE, "w4_zero_point_columns: N=%d K=%d (K %% 128 == 0, K <= %d)", N, K, ASYM_MAX_K);
+    if (N == 0) return STARQ_OK;
+    if (!aligned(Wq, 16) || !aligned(We, 16)) return fail(STARQ_ERR_ALIGN, "w4_zero_point_columns: Wq, We alignment");
+    cudaError_t e = launch_zero_point_columns(Wq, We, N, K, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w4_zero_point_columns launch");
+    return STARQ_OK;
+}
+
+size_t sgat_linear_asym_workspace_size(int L, int K) {
+    if (L < 0 || K < 0) return 0;
+    return align256((size_t)L * K / 2) + 2 * align256((size_t)L * 4) + align256((size_t)L * (K + 128));
+}
+
+int sgat_linear_asym(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                     const float* a_u, int hb, int d_sh, int d_m, int d_u, const uint8_t* We, const float* s_w,
+                     const float* bias, int N, void* Y, int y_dtype, void* workspace, size_t workspace_bytes,
+                     void* stream) {
+    if (!We || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear_asym: NULL We or s_w");
+    if (L > 0 && (!X || !Y || !workspace)) return fail(STARQ_ERR_ARG, "sgat_linear_asym: NULL X, Y or workspace");
+    if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear_asym: unknown dtype");
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    int rc = check_transform(K, hb, d_sh, d_m, d_u, a_m, a_u);
+    if (rc) return rc;
+    if (K % 128 != 0 || K > ASYM_MAX_K)
+        return fail(STARQ_ERR_SHAPE, "sgat_linear_asym: K=%d: need K %% 128 == 0 and K <= %d", K, ASYM_MAX_K);
+    if (L == 0) return STARQ_OK;
+    const size_t need = sgat_linear_asym_workspace_size(L, K);
+    if (workspace_bytes < need) return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu needed", workspace_bytes, need);
+    if (!aligned(workspace, 256) || !aligned(X, 16)) return fail(STARQ_ERR_ALIGN, "sgat_linear_asym alignment");
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    uint8_t* Xq = ws;
+    float* s_a = reinterpret_cast<float*>(ws + align256((size_t)L * K / 2));
+    int32_t* z_a = reinterpret_cast<int32_t*>(ws + align256((size_t)L * K / 2) + align256((size_t)L * 4));
+    uint8_t* Xe = ws + align256((size_t)L * K / 2) + 2 * align256((size_t)L * 4);
+    const int K2 = K + 128;                       // the augmented contraction
+    rc = check_gemm(nullptr, Xe, s_a, nullptr, We, s_w, bias, L, N, K2, Y, y_dtype);
+    if (rc) return rc;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    QuantArgs q{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, 15, 1.f, Xq, s_a, nullptr, Xe};
+    q.asym = 1;
+    q.z = z_a;
+    cudaError_t e;
+    if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear_asym: quant launch");
+    GemmArgs g{nullptr, s_a, nullptr, s_w, bias, L, N, K2, Y, y_dtype, nullptr, st, Xe, We};
+    g.weights_ready = 1;
+    if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear_asym: gemm launch");
     return STARQ_OK;
 }
 

@@ -35,6 +35,11 @@ struct QuantArgs {
     int qmax; float post_scale;
     uint8_t* Xq; float* s; float* v_dbg;
     uint8_t* Xe = nullptr;   // optional E4M3 byte copy of the codes [L][K]
+    // asymmetric activation quantiser (Eq. 2-4): codes in [0, qmax], zero
+    // points out to z [L]; Xe rows are K + 128 long, the last 128 bytes the
+    // E4M3 of -z (the zero-point columns of the augmented contraction)
+    int asym = 0;
+    int32_t* z = nullptr;
 };
 cudaError_t launch_sgat_quant(const QuantArgs& a, cudaStream_t stream);
 

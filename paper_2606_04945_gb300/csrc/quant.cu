@@ -23,6 +23,14 @@
 // and of l in columns K..2K-1 (both exact in E4M3), the operands of the
 // 8-bit GEMM.
 //
+// Asymmetric mode (a.asym, Eq. 2-4, activations): per row X_max = max(max v,
+// 0) and -X_min = max(max -v, 0); s = fl(fl(X_max - X_min) / qmax), r =
+// fl(qmax / fl(X_max - X_min)), z = rne(fl(-X_min r)) in [0, qmax], codes
+// clamp(rne(fl(v r)) + z, 0, qmax) (qmax = 15: unsigned nibbles in Xq, E4M3
+// bytes in Xe, whose rows are K + 128 long and end in 128 bytes of E4M3(-z):
+// with weight rows ending in E4M3 values that sum to sum_k q_w, the 4-bit
+// GEMM over K + 128 then gives sum_k (q_a - z) q_w exactly).
+//
 // Work split: a warp owns a chunk of C = 32 E consecutive elements of a row
 // (C = 1024 when hb >= 1024, else C = 512 holding 512 / hb Hadamard blocks).
 // In layout A lane l holds elements E l .. E l + E - 1, so stages h < E are
@@ -176,6 +184,25 @@ __device__ __forceinline__ void split_codes8(const int* q, uint2& bytes, uint2& 
     el = make_uint2((uint32_t)ll[0] | ((uint32_t)ll[1] << 16), (uint32_t)ll[2] | ((uint32_t)ll[3] << 16));
 }
 
+// Eight codes in [0, 15] -> E4M3 bytes (byte k = code k).
+__device__ __forceinline__ uint2 e4m3_of8(const int* q) {
+    uint16_t h[4];
+    #pragma unroll
+    for (int k = 0; k < 4; ++k)          // upper byte from the first operand
+        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(h[k]) : "f"((float)q[2 * k + 1]), "f"((float)q[2 * k]));
+    return make_uint2((uint32_t)h[0] | ((uint32_t)h[1] << 16), (uint32_t)h[2] | ((uint32_t)h[3] << 16));
+}
+
+// The zero-point columns of an asymmetric row: 128 bytes of E4M3(-z) after
+// its K codes, eight threads of 16 bytes each (t = 0 .. 7).
+__device__ __forceinline__ void store_zero_point_columns(uint8_t* row_end, int z, int t) {
+    uint16_t h;
+    const float m = (float)(-z);
+    asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %1;" : "=h"(h) : "f"(m));
+    const uint32_t w = (uint32_t)h | ((uint32_t)h << 16);
+    reinterpret_cast<uint4*>(row_end)[t] = make_uint4(w, w, w, w);
+}
+
 // Eight codes (int, |q| <= 7) -> packed nibbles, code k in bits 4k..4k+3.
 __device__ __forceinline__ uint32_t pack8(const int* q) {
     uint32_t w = 0;
@@ -208,7 +235,7 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
     const Tin* X = static_cast<const Tin*>(a.X) + (size_t)(row_ok ? row : 0) * K;
 
     float v[NC][E];
-    float amax = 0.f;
+    float amax = 0.f, nmin = 0.f;                        // asym: X_max and -X_min
     #pragma unroll
     for (int j = 0; j < NC; ++j) {
         const int c = wr + j * warps_per_row;
@@ -265,8 +292,16 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
             #pragma unroll
             for (int i = 0; i < E; ++i) v[j][i] = __fmul_rn(v[j][i], a.post_scale);
         }
-        #pragma unroll
-        for (int i = 0; i < E; ++i) amax = fmaxf(amax, fabsf(v[j][i]));
+        if (a.asym) {
+            #pragma unroll
+            for (int i = 0; i < E; ++i) {
+                amax = fmaxf(amax, v[j][i]);
+                nmin = fmaxf(nmin, -v[j][i]);
+            }
+        } else {
+            #pragma unroll
+            for (int i = 0; i < E; ++i) amax = fmaxf(amax, fabsf(v[j][i]));
+        }
         if (a.v_dbg != nullptr && live) {
             float4* d4 = reinterpret_cast<float4*>(a.v_dbg + (size_t)row * K + lo);
             #pragma unroll
@@ -275,27 +310,56 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
         }
     }
     #pragma unroll
-    for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
+    for (int m = 16; m > 0; m >>= 1) {
+        amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
+        nmin = fmaxf(nmin, __shfl_xor_sync(0xffffffffu, nmin, m));
+    }
     if (warps_per_row > 1) {
-        if (lane == 0) red[warp] = amax;
+        if (lane == 0) {
+            red[warp] = amax;
+            red[8 + warp] = nmin;
+        }
         __syncthreads();
         amax = 0.f;
+        nmin = 0.f;
         const int first = warp - wr;                     // first warp of this row
-        for (int w = 0; w < warps_per_row; ++w) amax = fmaxf(amax, red[first + w]);
+        for (int w = 0; w < warps_per_row; ++w) {
+            amax = fmaxf(amax, red[first + w]);
+            nmin = fmaxf(nmin, red[8 + first + w]);
+        }
     }
     if (!row_ok) return;
 
     const float qmax = (float)a.qmax;
-    const bool nz = amax > 0.f;
-    const float s = nz ? __fdiv_rn(amax, qmax) : 0.f;
-    const float r = nz ? __fdiv_rn(qmax, amax) : 0.f;
-    if (wr == 0 && lane == 0) a.s[row] = s;
+    const float range = a.asym ? __fadd_rn(amax, nmin) : amax;     // X_max - X_min, or amax
+    const bool nz = range > 0.f;
+    const float s = nz ? __fdiv_rn(range, qmax) : 0.f;
+    const float r = nz ? __fdiv_rn(qmax, range) : 0.f;
+    const int zp = a.asym ? min(max(__float2int_rn(__fmul_rn(nmin, r)), 0), a.qmax) : 0;
+    if (wr == 0 && lane == 0) {
+        a.s[row] = s;
+        if (a.asym) a.z[row] = zp;
+    }
+    if (a.asym && a.Xe != nullptr && wr == 0 && lane < 8)
+        store_zero_point_columns(a.Xe + (size_t)row * (K + 128) + K, zp, lane);
     #pragma unroll
     for (int j = 0; j < NC; ++j) {
         const int c = wr + j * warps_per_row;
         const int lo = c * C + E * lane;
         if (c >= nchunks || lo >= K) continue;
-        if (a.qmax > 7) {                // 8-bit codes: bytes and their E4M3 split
+        if (a.asym) {                    // codes in [0, qmax]: unsigned nibbles and E4M3 bytes
+            #pragma unroll
+            for (int u = 0; u < E / 8; ++u) {
+                int q[8];
+                #pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    q[k] = min(max(__float2int_rn(__fmul_rn(v[j][8 * u + k], r)) + zp, 0), a.qmax);
+                *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + lo / 2 + 4 * u) = pack8(q);
+                if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * (K + 128) + lo + 8 * u) = e4m3_of8(q);
+            }
+            continue;
+        }
+        if (a.qmax > 15) {               // 8-bit codes: bytes and their E4M3 split
             #pragma unroll
             for (int u = 0; u < E / 8; ++u) {
                 int q[8];
@@ -444,7 +508,7 @@ template <int NR, typename Tin>
 __global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
 sgat_quant_rows_kernel(QuantArgs a) {
     __shared__ __align__(16) float buf[4096];
-    __shared__ float red[4];
+    __shared__ float red[8];              // [0, 4) amax or X_max, [4, 8) -X_min (asym)
     grid_dependency_wait();            // launched with programmatic serialisation
     grid_launch_dependents();
     const int lane = threadIdx.x & 31;
@@ -459,7 +523,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
     float* slice = buf + warp * 1024;
 
     float v[NR][32];                      // layout C: v[R][8 j + k]
-    float amax = 0.f;
+    float amax = 0.f, nmin = 0.f;         // asym: X_max and -X_min
     #pragma unroll
     for (int R = 0; R < NR; ++R) {
         const int base = R * 4096;
@@ -585,8 +649,16 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 #pragma unroll
                 for (int k = 0; k < 8; ++k) v[R][8 * j + k] = __fmul_rn(v[R][8 * j + k], a.post_scale);
             }
-            #pragma unroll
-            for (int k = 0; k < 8; ++k) amax = fmaxf(amax, fabsf(v[R][8 * j + k]));
+            if (a.asym) {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    amax = fmaxf(amax, v[R][8 * j + k]);
+                    nmin = fmaxf(nmin, -v[R][8 * j + k]);
+                }
+            } else {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) amax = fmaxf(amax, fabsf(v[R][8 * j + k]));
+            }
             if (a.v_dbg != nullptr) {
                 float4* d4 = reinterpret_cast<float4*>(a.v_dbg + (size_t)row * K + e0);
                 d4[0] = make_float4(v[R][8 * j], v[R][8 * j + 1], v[R][8 * j + 2], v[R][8 * j + 3]);
@@ -595,16 +667,30 @@ sgat_quant_rows_kernel(QuantArgs a) {
         }
     }
     #pragma unroll
-    for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
-    if (lane == 0) red[warp] = amax;
+    for (int m = 16; m > 0; m >>= 1) {
+        amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
+        nmin = fmaxf(nmin, __shfl_xor_sync(0xffffffffu, nmin, m));
+    }
+    if (lane == 0) {
+        red[warp] = amax;
+        red[4 + warp] = nmin;
+    }
     __syncthreads();
     amax = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+    nmin = fmaxf(fmaxf(red[4], red[5]), fmaxf(red[6], red[7]));
 
     const float qmax = (float)a.qmax;
-    const bool nz = amax > 0.f;
-    const float s = nz ? __fdiv_rn(amax, qmax) : 0.f;
-    const float r = nz ? __fdiv_rn(qmax, amax) : 0.f;
-    if (threadIdx.x == 0) a.s[row] = s;
+    const float range = a.asym ? __fadd_rn(amax, nmin) : amax;     // X_max - X_min, or amax
+    const bool nz = range > 0.f;
+    const float s = nz ? __fdiv_rn(range, qmax) : 0.f;
+    const float r = nz ? __fdiv_rn(qmax, range) : 0.f;
+    const int zp = a.asym ? min(max(__float2int_rn(__fmul_rn(nmin, r)), 0), a.qmax) : 0;
+    if (threadIdx.x == 0) {
+        a.s[row] = s;
+        if (a.asym) a.z[row] = zp;
+    }
+    if (a.asym && a.Xe != nullptr && threadIdx.x < 8)
+        store_zero_point_columns(a.Xe + (size_t)row * (K + 128) + K, zp, threadIdx.x);
     #pragma unroll
     for (int R = 0; R < NR; ++R) {
         const int base = R * 4096;
@@ -618,7 +704,15 @@ sgat_quant_rows_kernel(QuantArgs a) {
             #pragma unroll
             for (int k = 0; k < 8; k += 2)
                 quant_pair(v[R][8 * j + k], v[R][8 * j + k + 1], r, qf[k], qf[k + 1], qi[k], qi[k + 1]);
-            if (a.qmax > 7) {            // 8-bit codes: bytes and their E4M3 split
+            if (a.asym) {                // codes in [0, qmax]: unsigned nibbles and E4M3 bytes
+                int q[8];
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) q[k] = min(max(qi[k] + zp, 0), a.qmax);
+                *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = pack8(q);
+                if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * (K + 128) + e0) = e4m3_of8(q);
+                continue;
+            }
+            if (a.qmax > 15) {           // 8-bit codes: bytes and their E4M3 split
                 uint2 bytes, eh, el;
                 split_codes8(qi, bytes, eh, el);
                 *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + e0) = bytes;
@@ -668,7 +762,7 @@ cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
     const int rpc = wpr <= 4 ? 8 / wpr : 1;          // rows per CTA
     const int nc = (n + wpr - 1) / wpr;              // rounds
     const int warps = wpr * rpc;
-    const size_t smem = (size_t)warps * (C + 32) * 4 + 8 * 4;
+    const size_t smem = (size_t)warps * (C + 32) * 4 + 16 * 4;
     dim3 grid((a.L + rpc - 1) / rpc), block(32 * warps);
     #define STARQ_QUANT_LAUNCH(NCV)                                                            \
         {                                                                                      \
