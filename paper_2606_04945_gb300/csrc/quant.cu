@@ -504,7 +504,9 @@ __device__ __forceinline__ void pack_codes8(const float* qf, const int* qi, uint
     e4.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
 }
 
-template <int NR, typename Tin>
+// ASYM: the asymmetric mode (a compile-time copy, so that the symmetric
+// kernel carries none of its reductions)
+template <int NR, typename Tin, bool ASYM>
 __global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
 sgat_quant_rows_kernel(QuantArgs a) {
     __shared__ __align__(16) float buf[4096];
@@ -649,7 +651,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 #pragma unroll
                 for (int k = 0; k < 8; ++k) v[R][8 * j + k] = __fmul_rn(v[R][8 * j + k], a.post_scale);
             }
-            if (a.asym) {
+            if (ASYM) {
                 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
                     amax = fmaxf(amax, v[R][8 * j + k]);
@@ -667,29 +669,30 @@ sgat_quant_rows_kernel(QuantArgs a) {
         }
     }
     #pragma unroll
-    for (int m = 16; m > 0; m >>= 1) {
-        amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
-        nmin = fmaxf(nmin, __shfl_xor_sync(0xffffffffu, nmin, m));
+    for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
+    if (ASYM) {
+        #pragma unroll
+        for (int m = 16; m > 0; m >>= 1) nmin = fmaxf(nmin, __shfl_xor_sync(0xffffffffu, nmin, m));
     }
     if (lane == 0) {
         red[warp] = amax;
-        red[4 + warp] = nmin;
+        if (ASYM) red[4 + warp] = nmin;
     }
     __syncthreads();
     amax = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
-    nmin = fmaxf(fmaxf(red[4], red[5]), fmaxf(red[6], red[7]));
+    if (ASYM) nmin = fmaxf(fmaxf(red[4], red[5]), fmaxf(red[6], red[7]));
 
     const float qmax = (float)a.qmax;
-    const float range = a.asym ? __fadd_rn(amax, nmin) : amax;     // X_max - X_min, or amax
+    const float range = ASYM ? __fadd_rn(amax, nmin) : amax;     // X_max - X_min, or amax
     const bool nz = range > 0.f;
     const float s = nz ? __fdiv_rn(range, qmax) : 0.f;
     const float r = nz ? __fdiv_rn(qmax, range) : 0.f;
-    const int zp = a.asym ? min(max(__float2int_rn(__fmul_rn(nmin, r)), 0), a.qmax) : 0;
+    const int zp = ASYM ? min(max(__float2int_rn(__fmul_rn(nmin, r)), 0), a.qmax) : 0;
     if (threadIdx.x == 0) {
         a.s[row] = s;
-        if (a.asym) a.z[row] = zp;
+        if (ASYM) a.z[row] = zp;
     }
-    if (a.asym && a.Xe != nullptr && threadIdx.x < 8)
+    if (ASYM && a.Xe != nullptr && threadIdx.x < 8)
         store_zero_point_columns(a.Xe + (size_t)row * (K + 128) + K, zp, threadIdx.x);
     #pragma unroll
     for (int R = 0; R < NR; ++R) {
@@ -704,7 +707,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
             #pragma unroll
             for (int k = 0; k < 8; k += 2)
                 quant_pair(v[R][8 * j + k], v[R][8 * j + k + 1], r, qf[k], qf[k + 1], qi[k], qi[k + 1]);
-            if (a.asym) {                // codes in [0, qmax]: unsigned nibbles and E4M3 bytes
+            if (ASYM) {                  // codes in [0, qmax]: unsigned nibbles and E4M3 bytes
                 int q[8];
                 #pragma unroll
                 for (int k = 0; k < 8; ++k) q[k] = min(max(qi[k] + zp, 0), a.qmax);
@@ -740,7 +743,8 @@ cudaError_t launch_rows_nr(const QuantArgs& a, cudaStream_t stream) {
     cfg.stream = stream;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin>, a);
+    return a.asym ? cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, true>, a)
+                  : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, false>, a);
 }
 
 template <typename Tin>
