@@ -21,6 +21,13 @@ Readings of the paper taken here (each is listed in the design doc):
   taken as fl(v * r) with r = fl((2^b - 1) / fl(X_max - X_min)), like the
   symmetric reading; z = rne(fl(-X_min * r)); codes clamp(rne(fl(v r)) + z,
   0, 2^b - 1). An all-zero row gets s = 0, z = 0 and all-zero codes.
+* The dense basis (SGAT's learned P, kept orthogonal, App. B: W_f =
+  Q_w(P^T W^T)): the transform is a 16-bit GEMM. Its operands are the
+  scaled rows fl32(x * a_s) and P, both rounded to float16; the product is
+  exact here (float64) and rounded to float16 once (the stored result),
+  then gated and quantised. The weight side is the same product on
+  fl32(w * inv_a_w): w_f = fl16(fl16(w * inv_a_w) P), the row form of
+  P^T W^T.
 * P is the block-diagonal Sylvester Hadamard matrix of block ``hb`` preceded
   by a per-state diagonal smoothing ``a_s``: Phi_s(x) = ((x * a_s) H) G_s with
   the unnormalised H; the 1/hb that makes H^-1 = H / hb is folded into the
@@ -257,6 +264,51 @@ def sgat_quantize_act_asym(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits=4):
         q, s, z = quantize_rows_asym(phi_state(X[I], a, g, hb), bits)
         codes[I], s_a[I], z_a[I] = q, s, z
     return codes, s_a, z_a
+
+
+def dense_basis_product(A, P16):
+    """fl16(fl16(A) P) for rows A [rows][K] (float32) and the dense basis P
+    [K][K] (float16 values): float64 product of the float16 operands, one
+    rounding to float16. Returned as float32."""
+    a16 = np.asarray(A, dtype=F32).astype(np.float16).astype(np.float64)
+    p = np.asarray(P16, dtype=np.float16).astype(np.float64)
+    return (a16 @ p).astype(np.float16).astype(F32)
+
+
+def sgat_quantize_act_dense(X, mask, a_m, a_u, P16, d_sh, d_m, d_u, bits=4):
+    """Q_a(X^s P G_s) with the dense basis (per state: scaled rows, the 16-bit
+    product, the gate, the symmetric quantiser). Returns (codes int32 [L, K],
+    s_a float32 [L], V float32 [L, K] = the ungated product)."""
+    X = np.asarray(X)
+    L, K = X.shape
+    g_m, g_u = state_gates(K, d_sh, d_m, d_u)
+    I_m, I_u = state_index_sets(mask)
+    codes = np.zeros((L, K), dtype=np.int32)
+    s_a = np.zeros(L, dtype=F32)
+    V = np.zeros((L, K), dtype=F32)
+    for I, a, g in ((I_m, a_m, g_m), (I_u, a_u, g_u)):
+        if len(I) == 0:
+            continue
+        x = np.asarray(X[I]).astype(F32)
+        if a is not None:
+            x = (x * np.asarray(a, dtype=F32)[None, :]).astype(F32)
+        v = dense_basis_product(x, P16)
+        V[I] = v
+        q, s = quantize_rows_sym(np.where(np.asarray(g)[None, :] != 0, v, F32(0)).astype(F32), bits)
+        codes[I], s_a[I] = q, s
+    return codes, s_a, V
+
+
+def prepare_weight_dense(W, inv_a_w, P16, bits=4):
+    """W_f = Q_w(P^T W^T) in row form: rows fl16(fl16(w * inv_a_w) P),
+    per-channel symmetric. Returns (codes int32 [N, K], s_w float32 [N],
+    Wf float32 [N, K])."""
+    w = np.asarray(W).astype(F32)
+    if inv_a_w is not None:
+        w = (w * np.asarray(inv_a_w, dtype=F32)[None, :]).astype(F32)
+    wf = dense_basis_product(w, P16)
+    q, s = quantize_rows_sym(wf, bits)
+    return q, s, wf
 
 
 def sgat_transform(X, mask, a_m, a_u, hb, d_sh, d_m, d_u):

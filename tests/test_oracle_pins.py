@@ -631,3 +631,60 @@ def test_asym_linear_triple_loop():
             want = sum((int(codes[i, k]) - int(z_a[i])) * int(qw[n, k]) for k in range(16))
             assert acc[i, n] == want
             assert Y[i, n] == float(want) * float(s_a[i]) * float(s_w[n])
+
+
+# ---------------------------------------------------------------------------
+# Dense basis (the learned orthogonal P of App. B) as a 16-bit product
+# ---------------------------------------------------------------------------
+
+def test_dense_basis_permutation_is_exact():
+    """A permutation is orthogonal and exact in float16: the dense path then
+    permutes the float16-rounded scaled rows and quantises them, which a
+    direct computation gives exactly."""
+    rng = np.random.default_rng(8)
+    L, K = 12, 64
+    X = rng.standard_normal((L, K)).astype(F32)
+    perm = rng.permutation(K)
+    P = np.zeros((K, K), np.float16)
+    P[perm, np.arange(K)] = 1                        # (x P)[j] = x[perm[j]]
+    mask = np.zeros(L, np.uint8)
+    codes, s, V = sgat.sgat_quantize_act_dense(X, mask, None, None, P, K, 0, 0)
+    want = X.astype(np.float16).astype(F32)[:, perm]
+    assert np.array_equal(V, want)
+    q, s2 = sgat.quantize_rows_sym(want, 4)
+    assert np.array_equal(codes, q) and np.array_equal(s, s2)
+
+
+def test_dense_basis_matches_fast_hadamard_on_exact_inputs():
+    """P = H_4 / 2 (block-diagonal, orthogonal, entries +-1/2 exact in
+    float16) on small-integer inputs: every value is exact in both paths, so
+    the dense product equals the fast transform of hb = 4 scaled by 1/2."""
+    rng = np.random.default_rng(9)
+    L, K = 6, 32
+    X = rng.integers(-8, 9, (L, K)).astype(F32)
+    H4 = sgat.hadamard_sylvester(4).astype(np.float64)
+    P = np.kron(np.eye(K // 4), H4 / 2).astype(np.float16)
+    V = sgat.dense_basis_product(X, P)
+    assert np.array_equal(V, sgat.fwht_f32(X, 4) * F32(0.5))
+
+
+def test_dense_basis_cancellation_16bit():
+    """A random orthogonal P (QR of a Gaussian, rounded to float16): the
+    16-bit dense linear reproduces X W^T up to the float16 roundings of the
+    transform. Applying P^T instead of P on one side, or P on both sides
+    transposed, breaks the cancellation by order one."""
+    rng = np.random.default_rng(10)
+    L, K, N = 16, 128, 24
+    X = rng.standard_normal((L, K)).astype(F32)
+    W = (rng.standard_normal((N, K)) * 0.1).astype(F32)
+    Q, _ = np.linalg.qr(rng.standard_normal((K, K)))
+    P = Q.astype(np.float16)
+    mask = (rng.random(L) < 0.5).astype(np.uint8)
+    codes, s_a, _ = sgat.sgat_quantize_act_dense(X, mask, None, None, P, K, 0, 0, bits=16)
+    qw, s_w, _ = sgat.prepare_weight_dense(W, None, P, bits=16)
+    Y = sgat.dequant(sgat.int_gemm(codes, qw), s_a, s_w)
+    ref = X.astype(np.float64) @ W.astype(np.float64).T
+    assert np.linalg.norm(Y - ref) / np.linalg.norm(ref) < 4e-3
+    qt, st, _ = sgat.prepare_weight_dense(W, None, P.T.copy(), bits=16)
+    Yt = sgat.dequant(sgat.int_gemm(codes, qt), s_a, st)
+    assert np.linalg.norm(Yt - ref) / np.linalg.norm(ref) > 0.5
