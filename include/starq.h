@@ -201,6 +201,42 @@ int sgat_quantize_act_asym(const void* X, int x_dtype, int L, int K, const uint8
                            int32_t* z_a, uint8_t* Xe, void* stream);
 int w4_zero_point_columns(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
 size_t sgat_linear_asym_workspace_size(int L, int K);
+
+/*
+ * Dense orthogonal basis (the learned P of App. B; W_f = Q_w(P^T W^T)) in
+ * place of the block Hadamard transform. The transform X^s P is a 16-bit
+ * GEMM: its operands are the scaled rows fl16(fl32(x * a_s)) and P, both
+ * float16, accumulated in float32 on the tensor cores, and the result is
+ * stored as float16. The gate and the symmetric 4-bit quantiser (hb = 1)
+ * then run on it.
+ *
+ *   Pt [K][K] float16: the basis transposed (row j holds column j of P),
+ *      16-byte aligned. P must be orthogonal: the weight side then uses the
+ *      same matrix (w_f = w P, the row form of P^T W^T).
+ *   Shapes: 128 <= K <= 16384 with K % 128 == 0.
+ *
+ * sgat_quantize_act_dense -- Q_a(X^s P G_s) per token: Xq [L][K/2] packed
+ *   int4, s_a [L], Xe [L][K] E4M3 or NULL, as for sgat_quantize_act.
+ *   workspace: sgat_dense_workspace_size(L, K) bytes, 256-byte aligned; it
+ *   holds [scaled rows fp16 L*K][V = X^s P fp16 L*K], each padded to 256.
+ * sgat_prepare_weight_dense -- Wq [N][K/2], s_w [N] from the rows
+ *   fl16(fl16(w * inv_a_w) P); workspace sgat_dense_workspace_size(N, K).
+ * sgat_linear_dense -- the fused linear: sgat_quantize_act_dense then
+ *   w4a4_gemm (Wq/We from sgat_prepare_weight_dense and w4_unpack_e4m3).
+ *   workspace: sgat_linear_dense_workspace_size(L, K) bytes: the dense
+ *   workspace, then [Xq][s_a][Xe] as in sgat_linear.
+ */
+size_t sgat_dense_workspace_size(int rows, int K);
+int sgat_quantize_act_dense(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                            const float* a_u, const void* Pt, int d_sh, int d_m, int d_u, uint8_t* Xq, float* s_a,
+                            uint8_t* Xe, void* workspace, size_t workspace_bytes, void* stream);
+int sgat_prepare_weight_dense(const void* W, int w_dtype, int N, int K, const float* inv_a_w, const void* Pt,
+                              uint8_t* Wq, float* s_w, void* workspace, size_t workspace_bytes, void* stream);
+size_t sgat_linear_dense_workspace_size(int L, int K);
+int sgat_linear_dense(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                      const float* a_u, const void* Pt, int d_sh, int d_m, int d_u, const uint8_t* Wq,
+                      const uint8_t* We, const float* s_w, const float* bias, int N, void* Y, int y_dtype,
+                      void* workspace, size_t workspace_bytes, void* stream);
 int sgat_linear_asym(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
                      const float* a_u, int hb, int d_sh, int d_m, int d_u, const uint8_t* We, const float* s_w,
                      const float* bias, int N, void* Y, int y_dtype, void* workspace, size_t workspace_bytes,

@@ -24,6 +24,8 @@ EXPORTED = (
     "attention_pv_tac_workspace_size", "attention_pv_tac",
     "w8_split_e4m3", "w8a8_gemm", "sgat_linear_workspace_size_bits",
     "sgat_quantize_act_asym", "w4_zero_point_columns", "sgat_linear_asym_workspace_size", "sgat_linear_asym",
+    "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
+    "sgat_linear_dense_workspace_size", "sgat_linear_dense",
 )
 
 
@@ -56,6 +58,15 @@ def _load():
     lib.sgat_linear_asym_workspace_size.restype = ctypes.c_size_t
     lib.sgat_linear_asym.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, u8p, f_p, f_p, i, vp, i, vp,
                                      ctypes.c_size_t, vp]
+    lib.sgat_dense_workspace_size.argtypes = [i, i]
+    lib.sgat_dense_workspace_size.restype = ctypes.c_size_t
+    lib.sgat_quantize_act_dense.argtypes = [vp, i, i, i, u8p, f_p, f_p, vp, i, i, i, u8p, f_p, u8p, vp,
+                                            ctypes.c_size_t, vp]
+    lib.sgat_prepare_weight_dense.argtypes = [vp, i, i, i, f_p, vp, u8p, f_p, vp, ctypes.c_size_t, vp]
+    lib.sgat_linear_dense_workspace_size.argtypes = [i, i]
+    lib.sgat_linear_dense_workspace_size.restype = ctypes.c_size_t
+    lib.sgat_linear_dense.argtypes = [vp, i, i, i, u8p, f_p, f_p, vp, i, i, i, u8p, u8p, f_p, f_p, i, vp, i, vp,
+                                      ctypes.c_size_t, vp]
     lib.tac_prepare.argtypes = [f_p, i, i, i, vp, vp]
     lib.starq_last_gemm_tile.restype = i
     dbl = ctypes.c_double
@@ -169,6 +180,47 @@ def sgat_linear_asym(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, We, s_w, Y, workspac
     _check(lib.sgat_linear_asym(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb, d_sh, d_m, d_u,
                                 _p(We), _p(s_w), _p(bias), N, _p(Y), dtype_code(Y), _p(workspace),
                                 workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def _ws(n, device):
+    return torch.empty(int(n), dtype=torch.uint8, device=device)
+
+
+def sgat_quantize_act_dense(X, mask, a_m, a_u, Pt, d_sh, d_m, d_u, Xq, s_a, Xe=None, workspace=None, stream=None):
+    """Dense-basis activation codes: Pt = P^T [K][K] float16 (P orthogonal).
+    workspace (optional) holds the scaled rows and V = X^s P (float16)."""
+    L, K = X.shape
+    if workspace is None:
+        workspace = _ws(lib.sgat_dense_workspace_size(L, K), X.device)
+    _contig(X, mask, a_m, a_u, Pt, Xq, s_a, Xe, workspace)
+    _check(lib.sgat_quantize_act_dense(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), _p(Pt), d_sh, d_m,
+                                       d_u, _p(Xq), _p(s_a), _p(Xe), _p(workspace),
+                                       workspace.numel() * workspace.element_size(), _stream(stream)))
+    return workspace
+
+
+def sgat_prepare_weight_dense(W, inv_a_w, Pt, Wq, s_w, workspace=None, stream=None):
+    N, K = W.shape
+    if workspace is None:
+        workspace = _ws(lib.sgat_dense_workspace_size(N, K), W.device)
+    _contig(W, inv_a_w, Pt, Wq, s_w, workspace)
+    _check(lib.sgat_prepare_weight_dense(_p(W), dtype_code(W), N, K, _p(inv_a_w), _p(Pt), _p(Wq), _p(s_w),
+                                         _p(workspace), workspace.numel() * workspace.element_size(),
+                                         _stream(stream)))
+    return workspace
+
+
+def sgat_linear_dense_workspace_size(L, K):
+    return int(lib.sgat_linear_dense_workspace_size(L, K))
+
+
+def sgat_linear_dense(X, mask, a_m, a_u, Pt, d_sh, d_m, d_u, Wq, s_w, Y, workspace, bias=None, We=None, stream=None):
+    _contig(X, mask, a_m, a_u, Pt, Wq, We, s_w, Y, workspace, bias)
+    L, K = X.shape
+    N = _weight_shape(Wq, We)[0]
+    _check(lib.sgat_linear_dense(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), _p(Pt), d_sh, d_m, d_u,
+                                 _p(Wq), _p(We), _p(s_w), _p(bias), N, _p(Y), dtype_code(Y), _p(workspace),
+                                 workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def w8_split_e4m3(Wq, We, stream=None):

@@ -10,6 +10,7 @@
 #include "tac_calib.cuh"
 #include "w8a8.cuh"
 #include "asym.cuh"
+#include "dense.cuh"
 
 namespace starq {
 
@@ -94,6 +95,26 @@ int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uin
 }
 
 constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// The dense-basis transform of `rows` rows into V (float16): the scaled
+// rows fl16(fl32(x * a_s)) into Xs, then V = Xs P on the 16-bit GEMM
+// (B operand Pt = P^T).
+cudaError_t dense_transform(const void* X, int x_dtype, int rows, int K, const uint8_t* mask, const float* a_m,
+                            const float* a_u, const void* Pt, __half* Xs, __half* V, unsigned* st, cudaStream_t s) {
+    cudaError_t e = launch_scale_rows_f16(X, x_dtype, rows, K, mask, a_m, a_u, Xs, s);
+    if (e != cudaSuccess) return e;
+    GemmArgs g{nullptr, nullptr, nullptr, nullptr, nullptr, rows, K, K, V, STARQ_F16, nullptr, st,
+               reinterpret_cast<const uint8_t*>(Xs), static_cast<const uint8_t*>(Pt)};
+    return launch_fp16_gemm(g, s);
+}
+
+int check_dense(int K, const void* Pt) {
+    if (!Pt) return fail(STARQ_ERR_ARG, "dense basis: NULL Pt");
+    if (K < 128 || K % 128 != 0 || K > 16384)
+        return fail(STARQ_ERR_SHAPE, "dense basis: K=%d: need 128 <= K <= 16384, K %% 128 == 0", K);
+    if (!aligned(Pt, 16)) return fail(STARQ_ERR_ALIGN, "dense basis: Pt must be 16-byte aligned");
+    return STARQ_OK;
+}
 
 int check_w8a8(const uint8_t* Xe, const float* s_a, const uint8_t* We, const float* s_w, const float* bias, int L,
                int N, int K, void* Y, int y_dtype) {
@@ -286,6 +307,102 @@ int sgat_linear_asym(const void* X, int x_dtype, int L, int K, const uint8_t* ma
     GemmArgs g{nullptr, s_a, nullptr, s_w, bias, L, N, K2, Y, y_dtype, nullptr, st, Xe, We};
     g.weights_ready = 1;
     if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear_asym: gemm launch");
+    return STARQ_OK;
+}
+
+size_t sgat_dense_workspace_size(int rows, int K) {
+    if (rows < 0 || K < 0) return 0;
+    return 2 * align256((size_t)rows * K * 2);
+}
+
+int sgat_quantize_act_dense(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                            const float* a_u, const void* Pt, int d_sh, int d_m, int d_u, uint8_t* Xq, float* s_a,
+                            uint8_t* Xe, void* workspace, size_t workspace_bytes, void* stream) {
+    if (L > 0 && (!X || !Xq || !s_a || !workspace)) return fail(STARQ_ERR_ARG, "sgat_quantize_act_dense: NULL argument");
+    if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act_dense: unknown dtype %d", x_dtype);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    int rc = check_dense(K, Pt);
+    if (rc) return rc;
+    if ((rc = check_transform(K, 1, d_sh, d_m, d_u, a_m, a_u))) return rc;
+    if (L == 0) return STARQ_OK;
+    if (workspace_bytes < sgat_dense_workspace_size(L, K))
+        return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu", workspace_bytes, sgat_dense_workspace_size(L, K));
+    if (!aligned(X, 16) || !aligned(Xq, 8) || (Xe && !aligned(Xe, 16)) || !aligned(workspace, 256))
+        return fail(STARQ_ERR_ALIGN, "sgat_quantize_act_dense: X, Xe (16 B), Xq (8 B), workspace (256 B) alignment");
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    __half* Xs = static_cast<__half*>(workspace);
+    __half* V = reinterpret_cast<__half*>(static_cast<uint8_t*>(workspace) + align256((size_t)L * K * 2));
+    cudaError_t e = dense_transform(X, x_dtype, L, K, mask, a_m, a_u, Pt, Xs, V, st, s);
+    if (e != cudaSuccess) return cuda_fail(e, "sgat_quantize_act_dense: transform launch");
+    QuantArgs q{V, STARQ_F16, L, K, mask, nullptr, nullptr, 1, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
+    if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_quantize_act_dense: quant launch");
+    return STARQ_OK;
+}
+
+int sgat_prepare_weight_dense(const void* W, int w_dtype, int N, int K, const float* inv_a_w, const void* Pt,
+                              uint8_t* Wq, float* s_w, void* workspace, size_t workspace_bytes, void* stream) {
+    if (N > 0 && (!W || !Wq || !s_w || !workspace)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight_dense: NULL argument");
+    if (!dtype_ok(w_dtype)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight_dense: unknown dtype %d", w_dtype);
+    if (N < 0) return fail(STARQ_ERR_SHAPE, "N=%d < 0", N);
+    int rc = check_dense(K, Pt);
+    if (rc) return rc;
+    if ((rc = check_transform(K, 1, K, 0, 0, nullptr, inv_a_w))) return rc;
+    if (N == 0) return STARQ_OK;
+    if (workspace_bytes < sgat_dense_workspace_size(N, K))
+        return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu", workspace_bytes, sgat_dense_workspace_size(N, K));
+    if (!aligned(W, 16) || !aligned(Wq, 8) || !aligned(workspace, 256))
+        return fail(STARQ_ERR_ALIGN, "sgat_prepare_weight_dense: W (16 B), Wq (8 B), workspace (256 B) alignment");
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    __half* Ws = static_cast<__half*>(workspace);
+    __half* Wf = reinterpret_cast<__half*>(static_cast<uint8_t*>(workspace) + align256((size_t)N * K * 2));
+    cudaError_t e = dense_transform(W, w_dtype, N, K, nullptr, nullptr, inv_a_w, Pt, Ws, Wf, st, s);
+    if (e != cudaSuccess) return cuda_fail(e, "sgat_prepare_weight_dense: transform launch");
+    QuantArgs q{Wf, STARQ_F16, N, K, nullptr, nullptr, nullptr, 1, K, 0, 0, 7, 1.f, Wq, s_w, nullptr};
+    if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_prepare_weight_dense: quant launch");
+    return STARQ_OK;
+}
+
+size_t sgat_linear_dense_workspace_size(int L, int K) {
+    if (L < 0 || K < 0) return 0;
+    return sgat_dense_workspace_size(L, K) + align256((size_t)L * K / 2) + align256((size_t)L * 4) +
+           align256((size_t)L * K);
+}
+
+int sgat_linear_dense(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                      const float* a_u, const void* Pt, int d_sh, int d_m, int d_u, const uint8_t* Wq,
+                      const uint8_t* We, const float* s_w, const float* bias, int N, void* Y, int y_dtype,
+                      void* workspace, size_t workspace_bytes, void* stream) {
+    if (L > 0 && (!X || !Y || !workspace)) return fail(STARQ_ERR_ARG, "sgat_linear_dense: NULL X, Y or workspace");
+    if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear_dense: unknown dtype");
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    int rc = check_dense(K, Pt);
+    if (rc) return rc;
+    if ((rc = check_transform(K, 1, d_sh, d_m, d_u, a_m, a_u))) return rc;
+    if (L == 0) return STARQ_OK;
+    const size_t need = sgat_linear_dense_workspace_size(L, K);
+    if (workspace_bytes < need) return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu needed", workspace_bytes, need);
+    if (!aligned(workspace, 256) || !aligned(X, 16)) return fail(STARQ_ERR_ALIGN, "sgat_linear_dense alignment");
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    __half* Xs = reinterpret_cast<__half*>(ws);
+    __half* V = reinterpret_cast<__half*>(ws + align256((size_t)L * K * 2));
+    uint8_t* Xq = ws + sgat_dense_workspace_size(L, K);
+    float* s_a = reinterpret_cast<float*>(Xq + align256((size_t)L * K / 2));
+    uint8_t* Xe = Xq + align256((size_t)L * K / 2) + align256((size_t)L * 4);
+    if ((rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype))) return rc;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = dense_transform(X, x_dtype, L, K, mask, a_m, a_u, Pt, Xs, V, st, s);
+    if (e != cudaSuccess) return cuda_fail(e, "sgat_linear_dense: transform launch");
+    QuantArgs q{V, STARQ_F16, L, K, mask, nullptr, nullptr, 1, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
+    if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear_dense: quant launch");
+    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
+    g.weights_ready = 1;
+    if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear_dense: gemm launch");
     return STARQ_OK;
 }
 
