@@ -193,3 +193,40 @@ def test_tac_calibrate_validation(lib):
     assert call(wb=good["wb"] - 8) == -2
     assert call(zq=ctypes.c_void_p(4104)) == -3 and call(w=ctypes.c_void_p(4104)) == -3
     assert "tac_calibrate" in L.starq_last_error().decode()
+
+
+def test_asym_validation(lib):
+    """Asymmetric entry points: NULL zero points, the zero-point columns' K
+    limits (K % 128, K <= 7680), alignment; the workspace layout."""
+    L, K = 4, 512
+    args = lambda z, k, xe, x=P: (x, 0, L, k, None, None, None, 1, k, 0, 0, P, P, z, xe, None)
+    assert lib.lib.sgat_quantize_act_asym(*args(None, K, P)) == -1
+    assert lib.lib.sgat_quantize_act_asym(*args(P, 528, P)) == -2          # Xe needs K % 128
+    assert lib.lib.sgat_quantize_act_asym(*args(P, 7808, P)) == -2         # above 7680
+    assert lib.lib.sgat_quantize_act_asym(*args(P, K, ctypes.c_void_p(4104))) == -3
+    assert lib.lib.w4_zero_point_columns(P, 4, 7808, P, None) == -2
+    assert lib.lib.w4_zero_point_columns(P, 4, 200, P, None) == -2
+    assert lib.lib.w4_zero_point_columns(ctypes.c_void_p(4100), 4, 256, P, None) == -3
+    assert lib.lib.w4_zero_point_columns(P, 0, 256, P, None) == 0
+    a256 = lambda x: (x + 255) // 256 * 256
+    assert lib.lib.sgat_linear_asym_workspace_size(1000, 4096) == (a256(1000 * 2048) + 2 * a256(4000)
+                                                                   + a256(1000 * 4224))
+    assert lib.lib.sgat_linear_asym(P, 0, L, 8192, None, None, None, 1, 8192, 0, 0, P, P, None, 64, P, 0, P,
+                                    1 << 30, None) == -2
+
+
+def test_dense_validation(lib):
+    """Dense-basis entry points: NULL basis, K limits (K % 128, K <= 16384),
+    a short workspace; the workspace sizes."""
+    L, K = 4, 512
+    q = lambda pt, k, wsb: lib.lib.sgat_quantize_act_dense(P, 0, L, k, None, None, None, pt, k, 0, 0, P, P, None, P,
+                                                           wsb, None)
+    assert q(None, K, 1 << 20) == -1
+    assert q(P, 576, 1 << 20) == -2
+    assert q(P, 16512, 1 << 30) == -2
+    assert q(P, K, 100) == -2
+    assert lib.lib.sgat_prepare_weight_dense(P, 0, 4, K, None, None, P, P, P, 1 << 20, None) == -1
+    a256 = lambda x: (x + 255) // 256 * 256
+    assert lib.lib.sgat_dense_workspace_size(100, 1024) == 2 * a256(100 * 1024 * 2)
+    assert lib.lib.sgat_linear_dense_workspace_size(100, 1024) == (2 * a256(100 * 1024 * 2) + a256(100 * 512)
+                                                                   + a256(400) + a256(100 * 1024))
