@@ -52,13 +52,14 @@ def parse():
     p.add_argument("--skip-cpu-baseline", action="store_true")
     p.add_argument("--workload", default="attention_step",
                    choices=["attention_step", "denoise_stack", "tac_calibration", "attention_pv_tac", "w8a8_linear",
-                            "asym_linear"],
+                            "asym_linear", "dense_linear"],
                    help="attention_step: the LLaDA attention projections (default); denoise_stack: the "
                         "64-step 4-layer LLaDA-shaped stack (per-step tokens/s, latency, drift vs fp16); "
                         "tac_calibration: App. C's closed-form TAC calibration on the GPU vs the oracle; "
                         "attention_pv_tac: the quantised softmax-value product with the TAC epilogue; "
                         "w8a8_linear: the attention projections at 8 bits (Tab. 5); "
-                        "asym_linear: the attention projections with asymmetric A4 activations (Eq. 2-4)")
+                        "asym_linear: the attention projections with asymmetric A4 activations (Eq. 2-4); "
+                        "dense_linear: the attention projections with a dense orthogonal basis (App. B)")
     return p.parse_args()
 
 
@@ -982,6 +983,78 @@ def run_asym(args):
                              "unit": "TOPS", "cores": cpu_cores(), "sample": f"QKV on {len(rows)} of {L} tokens"}}
 
 
+def run_dense(args):
+    """The dense orthogonal basis (App. B) at the LLaDA-8B attention
+    projections (1024 tokens, QKV 4096->12288, O 4096->4096): sgat_linear_dense
+    (row scaling, the 16-bit GEMM X^s P, the gated quantiser, the W4A4 GEMM)
+    against the Hadamard-basis sgat_linear of the same shapes, each call after
+    an L2 flush."""
+    import numpy as np
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi
+    torch.cuda.set_device(0)
+    L, K, d_m, d_u = 1024, 4096, 128, 128
+    d_sh = K - d_m - d_u
+    shapes = (("qkv", 12288), ("o", 4096))
+    rng = np.random.default_rng(0)
+    X = torch.from_numpy(rng.standard_normal((L, K)).astype(np.float16)).cuda()
+    mask = torch.from_numpy((np.arange(L) >= 640).astype(np.uint8)).cuda()
+    Q, _ = np.linalg.qr(rng.standard_normal((K, K)))
+    Pt = torch.from_numpy(np.ascontiguousarray(Q.T.astype(np.float16))).cuda()
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    flush = lambda: flush_buf.zero_()
+    w = {}
+    for name, N in shapes:
+        W = torch.from_numpy((rng.standard_normal((N, K)) / 64).astype(np.float16)).cuda()
+        e = {}
+        for kind in ("dense", "hadamard"):
+            Wq = torch.empty(N, K // 2, dtype=torch.uint8, device="cuda")
+            s_w = torch.empty(N, dtype=torch.float32, device="cuda")
+            if kind == "dense":
+                abi.sgat_prepare_weight_dense(W, None, Pt, Wq, s_w)
+            else:
+                abi.sgat_prepare_weight(W, None, K, Wq, s_w)
+            We = torch.empty(N, K, dtype=torch.uint8, device="cuda")
+            abi.w4_unpack_e4m3(Wq, We)
+            e[kind] = (Wq, s_w, We)
+        e["Y"] = torch.empty(L, N, dtype=torch.float16, device="cuda")
+        w[name] = e
+    ws_d = torch.empty(abi.sgat_linear_dense_workspace_size(L, K), dtype=torch.uint8, device="cuda")
+    ws_h = torch.empty(abi.sgat_linear_workspace_size(L, K, False), dtype=torch.uint8, device="cuda")
+
+    def dense():
+        for name, _ in shapes:
+            Wq, s_w, We = w[name]["dense"]
+            abi.sgat_linear_dense(X, mask, None, None, Pt, d_sh, d_m, d_u, Wq, s_w, w[name]["Y"], ws_d, We=We)
+
+    def hadamard():
+        for name, _ in shapes:
+            Wq, s_w, We = w[name]["hadamard"]
+            abi.sgat_linear(X, mask, None, None, K, d_sh, d_m, d_u, Wq, s_w, w[name]["Y"], ws_h, We=We)
+
+    for _ in range(max(args.warmup, 3)):
+        dense()
+        hadamard()
+    abi.check_status()
+    t_d = time_kernel(dense, flush, 20, torch)
+    t_h = time_kernel(hadamard, flush, 20, torch)
+    abi.check_status()
+    ops = sum(2 * L * N * K for _, N in shapes)
+    transform_flop = 2 * L * K * K
+    return {"metric": "dense-basis SGAT linear (App. B): integer TOPS of the two attention projections, transform "
+                      "and quantiser included",
+            "value": round(ops / (t_d * 1e-3) / 1e12, 1), "unit": "TOPS", "higher_is_better": True, "n_gpus": 1,
+            "data": "synthetic (seeded N(0, 1) activations, N(0, 1/64^2) weights, QR-orthogonal P in float16)",
+            "dtype": "fp16 transform GEMM, int4 codes, exact integer sums, fp16 out",
+            "config": {"workload": "dense_linear", "tokens": L, "hidden": K, "qkv": "4096->12288", "o": "4096->4096",
+                       "gates": "d_m = d_u = 128", "l2": "flushed before each timed call"},
+            "ms": {"dense_step": round(t_d, 4), "hadamard_step": round(t_h, 4)},
+            "vs_hadamard": round(t_h / t_d, 3),
+            "transform_gflop_per_projection": round(transform_flop / 1e9, 1)}
+
+
 def run_tac_calibration(args):
     """TAC's closed-form calibration (App. C) on the GPU against the oracle,
     on paired calibration outputs of the LLaDA attention width (8 samples of
@@ -1042,6 +1115,11 @@ def main():
     if args.workload == "tac_calibration":
         out = run_tac_calibration(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
                                                                     "the oracle arm times the attention-step workload"}
+        print(json.dumps(out), flush=True)
+        return
+    if args.workload == "dense_linear":
+        out = run_dense(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
+                                                           "the oracle arm times the attention-step workload"}
         print(json.dumps(out), flush=True)
         return
     if args.workload == "asym_linear":
