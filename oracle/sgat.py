@@ -8,7 +8,7 @@ here for the reduction length), ``W`` the weight (C x d, written N x K),
 ``mask`` the per-token state (1 = masked ``m``, 0 = unmasked ``u``), ``P`` the
 transformation basis, ``G_m`` / ``G_u`` the binary subspace gates.
 
-Readings of the paper taken here (each is listed in the design doc):
+Readings of the paper taken here:
 
 * The quantiser is the symmetric signed member of the uniform family of
   Eq. 2-3: zero point 0, codes in [-qmax, qmax] with qmax = 2^(b-1) - 1.

@@ -1,6 +1,6 @@
 """Shared test plumbing: device transfer, oracle runs, tolerances.
 
-Tolerances (spec bar; the readings are listed in the design doc):
+Tolerances:
   * int codes, scales and integer accumulators: bit-exact.
   * dequantised outputs in float16: |gpu - ref| <= 1e-3 |ref| + 2^-25 (the
     absolute half-spacing of float16 subnormals), ref = float64 oracle.
