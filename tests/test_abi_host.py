@@ -230,3 +230,37 @@ def test_dense_validation(lib):
     assert lib.lib.sgat_dense_workspace_size(100, 1024) == 2 * a256(100 * 1024 * 2)
     assert lib.lib.sgat_linear_dense_workspace_size(100, 1024) == (2 * a256(100 * 1024 * 2) + a256(100 * 512)
                                                                    + a256(400) + a256(100 * 1024))
+
+
+def test_zero_point_decomposition_rule_covers_the_k_limit():
+    """The weight-side zero-point columns hold sum_k q_w as 448s plus a
+    greedy remainder of E4M3 numbers (each step takes the largest E4M3
+    value not above what is left). For every |sum| <= 7 K at the API's
+    limit K = 7680 this ends exactly within 128 columns, and every term is
+    an E4M3 number. The rule is written here from the format's definition
+    (3 mantissa bits: above 16, values 2^e (1 + m/8))."""
+    def e4m3_floor(r):
+        if r <= 16:
+            return r
+        e = r.bit_length() - 1
+        step = 1 << (e - 3)
+        return min(r // step * step, 448)
+
+    def is_e4m3(v):
+        if v <= 16:
+            return True
+        e = v.bit_length() - 1
+        return v <= 448 and v % (1 << (e - 3)) == 0
+
+    worst = 0
+    for mag in range(0, 7 * 7680 + 1):
+        n448, rem = divmod(mag, 448)
+        terms = []
+        while rem:
+            t = e4m3_floor(rem)
+            assert is_e4m3(t)
+            terms.append(t)
+            rem -= t
+        assert len(terms) <= 5
+        worst = max(worst, n448 + len(terms))
+    assert worst <= 128
