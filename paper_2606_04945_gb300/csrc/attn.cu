@@ -19,23 +19,27 @@
 // attn_vquant_kernel   V codes per channel, written as fp16 values into
 //                      Vt [128 H][L] (keys contiguous: the K-major B
 //                      operand of P V^T), and the channel scales t.
-// attn_pv_tac_kernel   one CTA per (128-query tile, head); 16 softmax /
-//                      epilogue warps (a TMEM lane quarter times 32 of the
-//                      128 columns each), a TMA warp and an MMA warp;
-//                      tcgen05 kind::f16 on one CTA (M = N = 128, K = 16)
-//                      with the A operand (Q, P, Z_hat) in tensor memory
-//                      and B (K, V, M) in shared memory.
+// attn_pv_tac_kernel   one CTA per (128-query tile, head); clusters of 4
+//                      (or 2) query tiles of a head share every K / V tile
+//                      load by TMA multicast. 16 softmax / epilogue warps (a
+//                      TMEM lane quarter times 32 of the 128 columns each),
+//                      a TMA warp and one MMA warp, which issues every MMA
+//                      (tcgen05 kind::f16 on one CTA, M = N = 128, K = 16)
+//                      with the A operand (Q, P, Z_hat) in tensor memory and
+//                      B (K, V, M) in shared memory.
 //   prologue  the softmax warps write the Q tile into TMEM.
-//   pass 1  S = Q K^T chunk by chunk (128 keys, three TMEM buffers);
-//           each thread keeps the running maximum of its row's part of S.
-//   pass 2  S again; each thread turns its 32 scores into e = exp2((s - m)
-//           log2(e) / sqrt(d)) (ex2.approx), adds them to l (four partial
-//           sums) and writes the codes rne(255 e), rounded exactly by a
-//           float32 bias whose low bits are fp16 1024 + code, as fp16 over
-//           the S columns it has read (P
-//           double-buffered with S, so the next chunk's probabilities need
-//           not wait for this P V^T). The MMA warp accumulates P V^T one
-//           chunk behind the scores (exact integers).
+//   pass 1  S = Q K^T chunk by chunk (128 keys; three TMEM buffers, the
+//           third in the columns of the P V^T accumulator, which pass 1
+//           does not use); each thread keeps the running maximum of its
+//           row's part of S.
+//   pass 2  S again (two buffers); each thread turns its 32 scores into
+//           e = exp2((s - m) log2(e) / sqrt(d)) (ex2.approx), adds them to l
+//           (four partial sums) and writes the codes rne(255 e), rounded
+//           exactly by a float32 bias whose low bits are fp16 1024 + code,
+//           as fp16 over the S columns it has read. P is thus double-
+//           buffered with S, and the next chunk's probabilities need not
+//           wait for this P V^T. The MMA warp accumulates P V^T one chunk
+//           behind the scores (exact integers).
 //   epilogue  Z_hat from the accumulator, split into fp16 hi + lo (Z_hat =
 //           hi + lo to ~2^-22), written to TMEM as the A operands of the
 //           TAC product Z_hi M_hi^T + Z_hi M_lo^T + Z_lo M_hi^T with M's
@@ -44,10 +48,12 @@
 // Shared memory holds only B operands: a ring of six 32 KB tiles streams
 // pass 1's K chunks and pass 2's K and V chunks in the order the MMAs read
 // them; two of its slots then take M's halves and one the output boxes.
-// (With Q and P in shared memory as well, every chunk moved twice the
-// bytes through shared memory.) TMEM: two S / P buffers, the P V^T
-// accumulator and Q (448 of 512 columns); the TAC accumulator and Z_hat
-// reuse the S buffers. Every wait is bounded.
+// TMEM (512 columns): two S / P buffers, the P V^T accumulator and Q; the
+// TAC accumulator and Z_hat reuse the S buffers. The MMA warp queries its
+// two barriers per MMA group back to back, so their latencies overlap: with
+// about 50 cycles per issued MMA and ~160 per barrier query, a single
+// issuing thread is what bounds the tensor pipe here. Every wait is
+// bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
