@@ -5,7 +5,14 @@
  *
  * Conventions for every entry point:
  *   - All array arguments are DEVICE pointers owned by the caller. The library
- *     never allocates, frees or keeps a pointer past the call.
+ *     never allocates, frees or keeps a pointer past the call. Operands that
+ *     the kernels read or write through TMA tensor maps must be memory of
+ *     the current device (cudaSetDevice); calls that build tensor maps check
+ *     this with cudaPointerGetAttributes (outside stream capture) and return
+ *     STARQ_ERR_ARG for host, managed or another device's memory.
+ *   - Host-side state (per-device kernel attributes, occupancy and
+ *     address caches) is initialised once per device under a lock, so the
+ *     entry points may be called from several host threads at once.
  *   - Work is enqueued asynchronously on `stream` (a cudaStream_t passed as
  *     void*; NULL = the legacy default stream). Arguments are validated on
  *     the host before anything is launched; a call that returns an error
@@ -56,6 +63,16 @@ const char* starq_last_error(void);
  * kernels set when a bounded wait inside them runs out. Returns STARQ_OK,
  * STARQ_ERR_TIMEOUT (the kernel returned early; its outputs are undefined)
  * or STARQ_ERR_CUDA.
+ *
+ * Scope: there is ONE status word per device, shared by every stream and
+ * host thread that launches this library's kernels on it. The call waits
+ * for `stream` only, then reads and clears the whole word: a timeout of a
+ * kernel on another stream of the same device is reported (and cleared) by
+ * whichever call reads the word first, and a timeout on another stream that
+ * is still running when the word is read shows up in a later call. A caller
+ * that uses several streams should synchronise all of them before calling
+ * this, and treat a timeout as a failure of every kernel since its last
+ * check on that device.
  */
 int starq_check_status(void* stream);
 
@@ -271,12 +288,12 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
 
 /*
  * Tile of the last Xe + We (or fp16_gemm_ref) launch on the calling thread,
- * as BN * 10 + cluster size: 2564 (256-channel pair tiles, two pairs per
- * cluster sharing the activation tile), 2562, or 2242 (224-channel tiles on
- * single pairs); 0 before the first. The launcher estimates each shape's
- * time as ceil(tiles / resident clusters) rounds of a stage cost bound by
- * shared-memory traffic and takes the cheaper. A diagnostic for tests and
- * tuning; the results do not depend on it.
+ * as BN * 10 + cluster size: 2562 (256-channel pair tiles) or 2242
+ * (224-channel pair tiles); a cluster is one CTA pair, and each CTA loads
+ * its own operand rows. 0 before the first. The launcher estimates each
+ * shape's time as ceil(tiles / resident pairs) rounds of a stage cost bound
+ * by shared-memory traffic and takes the cheaper. A diagnostic for tests
+ * and tuning; the results do not depend on it.
  */
 int starq_last_gemm_tile(void);
 
@@ -364,9 +381,9 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  * tcgen05 kernel with a CTA per (128-query tile, head): two passes of
  * Q K^T over 128-key chunks (row maxima, then probabilities, codes and sums
  * with P V^T accumulated one chunk behind), then the dequantisation and TAC
- * epilogue. Clusters of 4 (or 2) query tiles of a head share each K / V
- * tile load by multicast. The call is asynchronous on `stream`; a wait that
- * gives up inside the kernel is reported by starq_check_status.
+ * epilogue. Every CTA loads its own K / V tiles by TMA. The call is
+ * asynchronous on `stream`; a wait that gives up inside the kernel is
+ * reported by starq_check_status.
  */
 size_t attention_pv_tac_workspace_size(int L, int H);
 int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L, int H, const void* Mp,
@@ -484,13 +501,19 @@ int sgat_linear_swiglu(const void* X, int x_dtype, int L, int K, const uint8_t* 
  * The caller still passes all inputs and outputs; arguments and results are
  * exactly those of sgat_linear without `workspace` / `workspace_bytes`.
  *
- *   - Limit: sgat_linear_workspace_size(L, K, tac_M != NULL) must not
- *     exceed STARQ_NOALLOC_SCRATCH_BYTES (32 MiB: e.g. 1024 tokens x 4096
- *     features with TAC need about 18.9 MB); larger calls return
- *     STARQ_ERR_SHAPE with a message and launch nothing.
+ *   - Limit: sgat_linear_workspace_size_bits(L, K, tac_M != NULL, bits)
+ *     must not exceed STARQ_NOALLOC_SCRATCH_BYTES (32 MiB). At K = 4096 a
+ *     4-bit call with TAC needs 22,532 bytes per token (1024 tokens:
+ *     23,072,768 bytes), so up to 1489 tokens fit; without TAC 6,148 bytes
+ *     per token. 8-bit calls need more (K + 4 + 2K, plus 4K with TAC, bytes
+ *     per token) and reach the limit at fewer tokens (1170 at K = 4096 with
+ *     TAC). Larger calls return STARQ_ERR_SHAPE with a message and launch
+ *     nothing.
  *   - The first call on each device looks up the scratch array's device
  *     address (cudaGetSymbolAddress, with that device current) and caches
  *     it; make that first call before any stream capture on that device.
+ *     The cached address is stale after cudaDeviceReset on that device: do
+ *     not call this entry point there again in the same process.
  *   - All calls on a device share the one array, which keeps the last call's
  *     contents. Nothing in it needs to start at zero: every byte a call reads
  *     back was written earlier in the same call. Calls whose work overlaps on

@@ -25,7 +25,7 @@ EXPORTED = (
     "w8_split_e4m3", "w8a8_gemm", "sgat_linear_workspace_size_bits",
     "sgat_quantize_act_asym", "w4_zero_point_columns", "sgat_linear_asym_workspace_size", "sgat_linear_asym",
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
-    "sgat_linear_dense_workspace_size", "sgat_linear_dense",
+    "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
 )
 
 
@@ -83,9 +83,8 @@ def _load():
     lib.attention_pv_tac_workspace_size.argtypes = [i, i]
     lib.attention_pv_tac_workspace_size.restype = ctypes.c_size_t
     lib.attention_pv_tac.argtypes = [vp, vp, vp, i, i, i, vp, f_p, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
-    if hasattr(lib, "sgat_linear_noalloc"):
-        lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
-                                            u8p, u8p, f_p, f_p, i, i, vp, i, vp]
+    lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
+                                        u8p, u8p, f_p, f_p, i, i, vp, i, vp]
     return lib
 
 

@@ -4,6 +4,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <initializer_list>
 
 #include "common.cuh"
 #include "attn.cuh"
@@ -38,18 +39,17 @@ bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
 bool dtype_ok(int t) { return t == STARQ_F16 || t == STARQ_BF16 || t == STARQ_F32; }
 
 unsigned* status_ptr(int* err) {
-    static unsigned* cache[64] = {nullptr};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess || dev >= 64) { *err = cuda_fail(e, "cudaGetDevice"); return nullptr; }
-    if (cache[dev] == nullptr) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_status_word);
-        if (e != cudaSuccess) { *err = cuda_fail(e, "cudaGetSymbolAddress(status)"); return nullptr; }
-        cache[dev] = static_cast<unsigned*>(p);
-    }
+    static DeviceCache<unsigned*> cache;
+    unsigned* p = nullptr;
+    const cudaError_t e = cache.get(&p, [](int, unsigned** v) {
+        void* a = nullptr;
+        const cudaError_t r = cudaGetSymbolAddress(&a, g_status_word);
+        *v = static_cast<unsigned*>(a);
+        return r;
+    });
+    if (e != cudaSuccess) { *err = cuda_fail(e, "status word address"); return nullptr; }
     *err = STARQ_OK;
-    return cache[dev];
+    return p;
 }
 
 int check_transform(int K, int hb, int d_sh, int d_m, int d_u, const float* a_m, const float* a_u) {
@@ -96,6 +96,36 @@ int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uin
 
 constexpr size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
+// Operands that the kernels reach through TMA tensor maps must be device
+// memory of the current device: a tensor map describes this GPU's own
+// memory. Every non-null pointer is checked with cudaPointerGetAttributes,
+// except while `stream` is capturing a CUDA graph (the eager calls before a
+// capture are checked; a capture records the same pointers).
+int check_local(const char* who, cudaStream_t stream, std::initializer_list<const void*> ptrs) {
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream, &cap) != cudaSuccess) {
+        cudaGetLastError();
+        cap = cudaStreamCaptureStatusNone;
+    }
+    if (cap != cudaStreamCaptureStatusNone) return STARQ_OK;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    for (const void* p : ptrs) {
+        if (p == nullptr) continue;
+        cudaPointerAttributes at;
+        e = cudaPointerGetAttributes(&at, p);
+        if (e != cudaSuccess) {
+            cudaGetLastError();
+            return fail(STARQ_ERR_ARG, "%s: pointer %p is not CUDA memory", who, p);
+        }
+        if (at.type != cudaMemoryTypeDevice || at.device != dev)
+            return fail(STARQ_ERR_ARG, "%s: pointer %p is not device memory of the current device %d "
+                        "(memory type %d, device %d)", who, p, dev, (int)at.type, at.device);
+    }
+    return STARQ_OK;
+}
+
 // The dense-basis transform of `rows` rows into V (float16): the scaled
 // rows fl16(fl32(x * a_s)) into Xs, then V = Xs P on the 16-bit GEMM
 // (B operand Pt = P^T).
@@ -137,16 +167,28 @@ int check_w8a8(const uint8_t* Xe, const float* s_a, const uint8_t* We, const flo
 int report_error(int code, const char* msg) { return fail(code, "%s", msg); }
 
 int num_sms() {
-    static int cache[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev >= 64) dev = 63;
-    if (cache[dev] == 0) {
-        int n = 0;
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        cache[dev] = n > 0 ? n : 1;
-    }
-    return cache[dev];
+    static DeviceCache<int> cache;
+    int n = 1;
+    if (cache.get(&n, [](int dev, int* v) {
+            int c = 0;
+            const cudaError_t r = cudaDeviceGetAttribute(&c, cudaDevAttrMultiProcessorCount, dev);
+            *v = c > 0 ? c : 1;
+            return r;
+        }) != cudaSuccess)
+        return 1;
+    return n;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static const PFN_cuTensorMapEncodeTiled_v12000 fn = []() -> PFN_cuTensorMapEncodeTiled_v12000 {
+        cudaDriverEntryPointQueryResult q;
+        void* f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess || q != cudaDriverEntryPointSuccess)
+            return nullptr;
+        return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }();
+    return fn;
 }
 
 }  // namespace starq
@@ -227,6 +269,8 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
     int rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     if (acc_dbg && !aligned(acc_dbg, 16)) return fail(STARQ_ERR_ALIGN, "acc_dbg must be 16-byte aligned");
+    if (L > 0 && (rc = check_local("w4a4_gemm", static_cast<cudaStream_t>(stream), {Xe, Xe ? We : nullptr, Xe ? Wq : nullptr, Y})))
+        return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe, Xe ? We : nullptr};
@@ -296,6 +340,7 @@ int sgat_linear_asym(const void* X, int x_dtype, int L, int K, const uint8_t* ma
     const int K2 = K + 128;                       // the augmented contraction
     rc = check_gemm(nullptr, Xe, s_a, nullptr, We, s_w, bias, L, N, K2, Y, y_dtype);
     if (rc) return rc;
+    if ((rc = check_local("sgat_linear_asym", static_cast<cudaStream_t>(stream), {workspace, We, Y}))) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -329,6 +374,7 @@ int sgat_quantize_act_dense(const void* X, int x_dtype, int L, int K, const uint
         return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu", workspace_bytes, sgat_dense_workspace_size(L, K));
     if (!aligned(X, 16) || !aligned(Xq, 8) || (Xe && !aligned(Xe, 16)) || !aligned(workspace, 256))
         return fail(STARQ_ERR_ALIGN, "sgat_quantize_act_dense: X, Xe (16 B), Xq (8 B), workspace (256 B) alignment");
+    if ((rc = check_local("sgat_quantize_act_dense", static_cast<cudaStream_t>(stream), {workspace, Pt}))) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -354,6 +400,7 @@ int sgat_prepare_weight_dense(const void* W, int w_dtype, int N, int K, const fl
         return fail(STARQ_ERR_SHAPE, "workspace %zu bytes < %zu", workspace_bytes, sgat_dense_workspace_size(N, K));
     if (!aligned(W, 16) || !aligned(Wq, 8) || !aligned(workspace, 256))
         return fail(STARQ_ERR_ALIGN, "sgat_prepare_weight_dense: W (16 B), Wq (8 B), workspace (256 B) alignment");
+    if ((rc = check_local("sgat_prepare_weight_dense", static_cast<cudaStream_t>(stream), {workspace, Pt}))) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -393,6 +440,7 @@ int sgat_linear_dense(const void* X, int x_dtype, int L, int K, const uint8_t* m
     float* s_a = reinterpret_cast<float*>(Xq + align256((size_t)L * K / 2));
     uint8_t* Xe = Xq + align256((size_t)L * K / 2) + align256((size_t)L * 4);
     if ((rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype))) return rc;
+    if ((rc = check_local("sgat_linear_dense", static_cast<cudaStream_t>(stream), {workspace, Pt, Wq, We, Y}))) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -422,6 +470,7 @@ int w8a8_gemm(const uint8_t* Xe, const float* s_a, const uint8_t* We, const floa
     if (rc) return rc;
     if (L == 0) return STARQ_OK;
     if (acc_dbg && !aligned(acc_dbg, 16)) return fail(STARQ_ERR_ALIGN, "acc_dbg must be 16-byte aligned");
+    if ((rc = check_local("w8a8_gemm", static_cast<cudaStream_t>(stream), {Xe, We}))) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     GemmArgs a{nullptr, s_a, nullptr, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe, We};
@@ -439,7 +488,8 @@ int fp16_gemm_ref(const void* A, const void* B, int dtype, int M, int N, int K, 
     if (M == 0) return STARQ_OK;
     if (!aligned(A, 16) || !aligned(B, 16) || !aligned(C, 16))
         return fail(STARQ_ERR_ALIGN, "fp16_gemm_ref: A, B, C must be 16-byte aligned");
-    int rc = STARQ_OK;
+    int rc = check_local("fp16_gemm_ref", static_cast<cudaStream_t>(stream), {A, B, C});
+    if (rc) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     GemmArgs a{nullptr, nullptr, nullptr, nullptr, nullptr, M, N, K, C, dtype, nullptr, st,
@@ -481,6 +531,7 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
     if ((rc = check_tac_prepared(Mp, z_dtype, g))) return rc;
     if (L == 0) return STARQ_OK;
     if (!aligned(Z, 16) || !aligned(out, 16)) return fail(STARQ_ERR_ALIGN, "tac_apply: Z, out alignment");
+    if ((rc = check_local("tac_apply", static_cast<cudaStream_t>(stream), {Z, out}))) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     TacArgs a{Z, z_dtype, L, C, g, M, d, out, out_dtype, st, Mp};
@@ -508,7 +559,8 @@ int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L,
     if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(Mp, 16) || !aligned(Z, 16) ||
         (d && !aligned(d, 16)) || !aligned(workspace, 256))
         return fail(STARQ_ERR_ALIGN, "attention_pv_tac: Q, K, V, Mp, Z, d 16-byte and workspace 256-byte alignment");
-    int rc = STARQ_OK;
+    int rc = check_local("attention_pv_tac", static_cast<cudaStream_t>(stream), {Q, K, V, Z, workspace});
+    if (rc) return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     uint8_t* ws = static_cast<uint8_t*>(workspace);
@@ -571,7 +623,8 @@ int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* ma
                      const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
                      const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
                      const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
-                     void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream, int swiglu) {
+                     void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream, int swiglu,
+                     bool ws_owned) {
     if ((!Wq && !We) || !s_w) return fail(STARQ_ERR_ARG, "sgat_linear: NULL Wq/We or s_w");
     if (L > 0 && (!X || !Y || !workspace)) return fail(STARQ_ERR_ARG, "sgat_linear: NULL X, Y or workspace");
     if (!dtype_ok(x_dtype) || !dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "sgat_linear: unknown dtype");
@@ -598,6 +651,10 @@ int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* ma
     rc = bits == 8 ? check_w8a8(Xe, s_a, We, s_w, bias, L, N, K, Y, y_dtype)
                    : check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
+    // the scratch of sgat_linear_noalloc is the library's own device array
+    if ((rc = check_local("sgat_linear", static_cast<cudaStream_t>(stream),
+                          {X, ws_owned ? nullptr : workspace, We ? We : Wq, Y})))
+        return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -628,6 +685,17 @@ int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* ma
 }
 }  // namespace
 
+namespace starq {
+int sgat_linear_scratch(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                        const float* a_u, int hb, int d_sh, int d_m, int d_u, const float* tac_M, const float* tac_d,
+                        int tac_g, const void* tac_Mp, const uint8_t* Wq, const uint8_t* We, const float* s_w,
+                        const float* bias, int N, int bits, void* Y, int y_dtype, void* scratch, size_t scratch_bytes,
+                        void* stream) {
+    return sgat_linear_impl(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g, tac_Mp, Wq,
+                            We, s_w, bias, N, bits, Y, y_dtype, scratch, scratch_bytes, stream, 0, true);
+}
+}  // namespace starq
+
 extern "C" {
 
 int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
@@ -636,7 +704,7 @@ int sgat_linear(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                 const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias, int N, int bits,
                 void* Y, int y_dtype, void* workspace, size_t workspace_bytes, void* stream) {
     return sgat_linear_impl(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g, tac_Mp, Wq,
-                            We, s_w, bias, N, bits, Y, y_dtype, workspace, workspace_bytes, stream, 0);
+                            We, s_w, bias, N, bits, Y, y_dtype, workspace, workspace_bytes, stream, 0, false);
 }
 
 int sgat_linear_swiglu(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
@@ -650,7 +718,7 @@ int sgat_linear_swiglu(const void* X, int x_dtype, int L, int K, const uint8_t* 
     if (N < 32 || N % 32 != 0)
         return fail(STARQ_ERR_SHAPE, "sgat_linear_swiglu: N=%d: gate and up rows interleaved by 16, N %% 32 == 0", N);
     return sgat_linear_impl(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g, tac_Mp, Wq,
-                            We, s_w, bias, N, bits, H, h_dtype, workspace, workspace_bytes, stream, 1);
+                            We, s_w, bias, N, bits, H, h_dtype, workspace, workspace_bytes, stream, 1, false);
 }
 
 }  // extern "C"

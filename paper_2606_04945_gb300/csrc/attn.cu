@@ -19,9 +19,8 @@
 // attn_vquant_kernel   V codes per channel, written as fp16 values into
 //                      Vt [128 H][L] (keys contiguous: the K-major B
 //                      operand of P V^T), and the channel scales t.
-// attn_pv_tac_kernel   one CTA per (128-query tile, head); clusters of 4
-//                      (or 2) query tiles of a head share every K / V tile
-//                      load by TMA multicast. 16 softmax / epilogue warps (a
+// attn_pv_tac_kernel   one CTA per (128-query tile, head), each loading its
+//                      own K / V tiles by TMA. 16 softmax / epilogue warps (a
 //                      TMEM lane quarter times 32 of the 128 columns each),
 //                      a TMA warp and one MMA warp, which issues every MMA
 //                      (tcgen05 kind::f16 on one CTA, M = N = 128, K = 16)
@@ -126,13 +125,6 @@ __device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_
                     "r"(v[15])
                  : "memory");
 }
-// Arrive once on the barrier at shared offset `bar` in every CTA of
-// `cta_mask` when the issuing thread's tcgen05 operations have completed.
-__device__ __forceinline__ void tc_commit_multicast(uint32_t bar, uint16_t cta_mask) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-                 " [%0], %1;" :: "r"(bar), "h"(cta_mask) : "memory");
-}
-
 __device__ __forceinline__ void tmem_st_wait() {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
@@ -234,16 +226,11 @@ __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
     }
 }
 
-// CL CTAs of one head (consecutive query tiles) form a cluster: each loads
-// 128 / CL rows of every K and V tile and multicasts them to all, so each
-// tile leaves L2 once per cluster; a slot is refilled once every CTA's
-// MMAs have read it (its empty barrier counts one commit per CTA).
-template <int CL>
+// A ring slot is refilled once this CTA's MMAs have read it (one commit on
+// its empty barrier).
 __global__ void __launch_bounds__(ATT_THREADS, 1)
 attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_z) {
-    constexpr int SHARE = ATTN_TILE / CL;                    // rows of each tile this CTA loads
-    constexpr uint16_t MASK = (uint16_t)((1u << CL) - 1u);
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -282,7 +269,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         mbar_init(B(sh->q_full), ATT_SOFTMAX_WARPS);
         for (int k = 0; k < ATT_SLOTS; ++k) {
             mbar_init(B(sh->full[k]), 1);
-            mbar_init(B(sh->empty[k]), CL);
+            mbar_init(B(sh->empty[k]), 1);
         }
         for (int b = 0; b < 3; ++b) {
             mbar_init(B(sh->s_full[b]), 1);
@@ -301,10 +288,8 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
     }
     tc_fence_before();
     __syncthreads();
-    if (CL > 1) cluster_sync();              // every CTA's barriers exist before any multicast
     tc_fence_after();
     const uint32_t tmem = sh->tmem_base;
-    const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
 
     if (warp == ATT_TMA_WARP) {
         bool ok = true;
@@ -315,23 +300,18 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             if (elect_one()) {
                 mbar_arrive_expect_tx(B(sh->full[k]), TILE_BYTES);
                 const int w = u - nk;
-                const uint32_t d0 = dst + (uint32_t)(rank * SHARE * 128), fb = B(sh->full[k]);
+                const uint32_t fb = B(sh->full[k]);
                 const void* tm = (w < 0 || (w & 1) == 0) ? (const void*)&tm_k : (const void*)&tm_v;
                 int x, y;
                 if (w < 0 || (w & 1) == 0) {                 // K chunk: keys are the rows
                     x = h * ATTN_D;
-                    y = (w < 0 ? u : w >> 1) * ATTN_TILE + rank * SHARE;
+                    y = (w < 0 ? u : w >> 1) * ATTN_TILE;
                 } else {                                     // V chunk: channels are the rows
                     x = (w >> 1) * ATTN_TILE;
-                    y = h * ATTN_D + rank * SHARE;
+                    y = h * ATTN_D;
                 }
-                if (CL > 1) {
-                    tma_load_2d_multicast(d0, tm, x, y, fb, MASK);
-                    tma_load_2d_multicast(d0 + ATOM_BYTES, tm, x + 64, y, fb, MASK);
-                } else {
-                    tma_load_2d(d0, tm, x, y, fb);
-                    tma_load_2d(d0 + ATOM_BYTES, tm, x + 64, y, fb);
-                }
+                tma_load_2d(dst, tm, x, y, fb);
+                tma_load_2d(dst + ATOM_BYTES, tm, x + 64, y, fb);
             }
             __syncwarp();
         }
@@ -345,8 +325,8 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             bulk_load(sMlo, mp + TILE_BYTES, TILE_BYTES, B(sh->m_full));
         }
         __syncwarp();
-        // every CTA's commits for the last use of each slot have arrived
-        // here, so none lands after this CTA has exited
+        // the commits for the last use of each slot have arrived, so none
+        // lands after this CTA has exited
         for (int u = U - ATT_SLOTS; u < U && ok; ++u)
             if (u >= 0) ok = mbar_wait_bounded_warp(B(sh->empty[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1), abort);
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
@@ -371,8 +351,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             }
         };
         auto release = [=](int u) {           // this CTA's MMAs are done with ring slot u
-            if (CL > 1) tc_commit_multicast(B(sh->empty[u % ATT_SLOTS]), MASK);
-            else tc_commit(B(sh->empty[u % ATT_SLOTS]));
+            tc_commit(B(sh->empty[u % ATT_SLOTS]));
         };
         // Q K^T number it, once its K tile has landed and its S buffer's
         // previous use is consumed: S read by the softmax warps, or P
@@ -602,23 +581,14 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
     }
     tc_fence_before();
     __syncthreads();
-    // no CTA leaves while another may still commit to its barriers
-    if (CL > 1) cluster_sync();
     tc_fence_after();
     if (warp == ATT_MMA_WARP) tmem_dealloc(tmem, 512);
 }
 
 bool encode_2d(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint64_t row_elems,
                uint32_t box_rows, uint32_t box_cols, CUtensorMapSwizzle swz) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        cudaDriverEntryPointQueryResult q;
-        void* f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
-            return false;
-        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-    }
+    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+    if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {row_elems * 2};
     const cuuint32_t box[2] = {box_cols, box_rows};
@@ -630,36 +600,22 @@ bool encode_2d(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, ui
 
 }  // namespace
 
-template <int CL>
 cudaError_t launch_pv_tac(const AttnArgs& a, cudaStream_t stream) {
     const int C = ATTN_D * a.H;
     CUtensorMap tk, tv, tz;
-    if (!encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)C, (uint64_t)a.ld, ATTN_TILE / CL, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_2d(&tv, a.Vt, (uint64_t)C, (uint64_t)a.L, (uint64_t)a.L, ATTN_D / CL, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
+    if (!encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)C, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_2d(&tv, a.Vt, (uint64_t)C, (uint64_t)a.L, (uint64_t)a.L, ATTN_D, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !encode_2d(&tz, a.Z, (uint64_t)a.L, (uint64_t)C, (uint64_t)C, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
         return cudaErrorInvalidValue;
-    static bool attr_set[64] = {false};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !attr_set[dev]) {
-        const cudaError_t e =
-            cudaFuncSetAttribute(attn_pv_tac_kernel<CL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ATT_SMEM);
-        if (e != cudaSuccess) return e;
-        attr_set[dev] = true;
-    }
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3(a.L / ATTN_TILE, a.H);
-    cfg.blockDim = dim3(ATT_THREADS);
-    cfg.dynamicSmemBytes = ATT_SMEM;
-    cfg.stream = stream;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, attn_pv_tac_kernel<CL>, a, tk, tv, tz);
+    static DeviceCache<int> attr;
+    int done = 0;
+    const cudaError_t e = attr.get(&done, [](int, int* v) {
+        *v = 1;
+        return cudaFuncSetAttribute(attn_pv_tac_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ATT_SMEM);
+    });
+    if (e != cudaSuccess) return e;
+    attn_pv_tac_kernel<<<dim3(a.L / ATTN_TILE, a.H), ATT_THREADS, ATT_SMEM, stream>>>(a, tk, tv, tz);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_attention_pv_tac(const AttnArgs& a, cudaStream_t stream) {
@@ -667,11 +623,7 @@ cudaError_t launch_attention_pv_tac(const AttnArgs& a, cudaStream_t stream) {
     attn_vquant_kernel<<<C / VQ_CH, 256, 0, stream>>>(a);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    // clusters of 4 (or 2) query tiles of a head share the K / V loads
-    const int tiles = a.L / ATTN_TILE;
-    if (tiles % 4 == 0) return launch_pv_tac<4>(a, stream);
-    if (tiles % 2 == 0) return launch_pv_tac<2>(a, stream);
-    return launch_pv_tac<1>(a, stream);
+    return launch_pv_tac(a, stream);
 }
 
 }  // namespace starq

@@ -3,10 +3,15 @@
 // descriptors, and the launcher interface between the C ABI and the kernels.
 #pragma once
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <cuda_fp16.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
+
+#include <atomic>
+#include <mutex>
 
 #include "../../include/starq.h"
 
@@ -95,6 +100,52 @@ cudaError_t launch_tac_prepare(const float* M, int C, int g, int z_dtype, void* 
 
 int num_sms();  // SM count of the current device (cached per device)
 int report_error(int code, const char* msg);  // record msg for starq_last_error(), return code
+
+// sgat_linear with a workspace that the library owns (the device scratch
+// array of sgat_linear_noalloc), which the device-memory check skips.
+int sgat_linear_scratch(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
+                        const float* a_u, int hb, int d_sh, int d_m, int d_u, const float* tac_M, const float* tac_d,
+                        int tac_g, const void* tac_Mp, const uint8_t* Wq, const uint8_t* We, const float* s_w,
+                        const float* bias, int N, int bits, void* Y, int y_dtype, void* scratch, size_t scratch_bytes,
+                        void* stream);
+
+// cuTensorMapEncodeTiled from the driver (looked up once, thread-safe), or
+// nullptr when the driver does not provide it.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder();
+
+// A value per device, computed once by `init(dev, &value)` with that device
+// current. Several host threads may call get() at once: the first caller for
+// a device computes the value under a lock, the others wait for it or read
+// the published value; a failed init leaves the entry unset for a retry.
+template <typename T>
+class DeviceCache {
+  public:
+    static constexpr int MAX_DEVICES = 64;
+    template <typename F>
+    cudaError_t get(T* out, F&& init) {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return e;
+        if (dev < 0 || dev >= MAX_DEVICES) return cudaErrorInvalidDevice;
+        if (!ready_[dev].load(std::memory_order_acquire)) {
+            std::lock_guard<std::mutex> lock(mu_);
+            if (!ready_[dev].load(std::memory_order_relaxed)) {
+                T v{};
+                e = init(dev, &v);
+                if (e != cudaSuccess) return e;
+                val_[dev] = v;
+                ready_[dev].store(true, std::memory_order_release);
+            }
+        }
+        *out = val_[dev];
+        return cudaSuccess;
+    }
+
+  private:
+    std::mutex mu_;
+    T val_[MAX_DEVICES] = {};
+    std::atomic<bool> ready_[MAX_DEVICES] = {};
+};
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
@@ -350,23 +401,6 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap,
     asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2"
                  " [%0], [%1, {%2, %3}], [%4];"
                  :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar) : "memory");
-}
-// Pair form with cluster multicast: the tile lands at `dst` in every CTA of
-// `cta_mask`; each destination's bytes are counted on the barrier at `bar`'s
-// offset in the even (leader) CTA of that destination's pair.
-__device__ __forceinline__ void tma_load_2d_pair_multicast(uint32_t dst, const void* tmap, int x, int y,
-                                                           uint32_t bar, uint16_t cta_mask) {
-    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-                 ".cta_group::2 [%0], [%1, {%2, %3}], [%4], %5;"
-                 :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar), "h"(cta_mask) : "memory");
-}
-// Same, with the tile (and the completion on `bar`) delivered to the same
-// shared-memory offsets in every CTA of `cta_mask`.
-__device__ __forceinline__ void tma_load_2d_multicast(uint32_t dst, const void* tmap, int x, int y,
-                                                      uint32_t bar, uint16_t cta_mask) {
-    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-                 " [%0], [%1, {%2, %3}], [%4], %5;"
-                 :: "r"(dst), "l"(tmap), "r"(x), "r"(y), "r"(bar), "h"(cta_mask) : "memory");
 }
 // Contiguous global -> shared bulk copy (16-byte aligned, size % 16 == 0),
 // completion counted on `bar`.

@@ -16,7 +16,9 @@
 // Host code cannot use the array's name as a device address, so the device
 // address is looked up with cudaGetSymbolAddress once per device (with that
 // device current) on the first call, cached, and handed to sgat_linear as
-// its workspace.
+// its workspace. The cached address belongs to the device's current primary
+// context: after cudaDeviceReset it is stale, and the process must not call
+// this entry point on that device again.
 #include <cstdio>
 #include <mutex>
 
@@ -78,7 +80,7 @@ extern "C" int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, con
                  cudaGetErrorString(err));
         return starq::report_error(rc, msg);
     }
-    return sgat_linear(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g, tac_Mp,
-                       Wq, We, s_w, bias, N, bits, Y, y_dtype, scratch,
-                       (size_t)STARQ_NOALLOC_SCRATCH_BYTES, stream);
+    return starq::sgat_linear_scratch(X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, tac_M, tac_d, tac_g,
+                                      tac_Mp, Wq, We, s_w, bias, N, bits, Y, y_dtype, scratch,
+                                      (size_t)STARQ_NOALLOC_SCRATCH_BYTES, stream);
 }

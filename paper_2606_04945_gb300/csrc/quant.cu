@@ -770,14 +770,14 @@ cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
     dim3 grid((a.L + rpc - 1) / rpc), block(32 * warps);
     #define STARQ_QUANT_LAUNCH(NCV)                                                            \
         {                                                                                      \
-            static bool attr[64] = {false};                                                    \
-            int dev = 0; cudaGetDevice(&dev);                                                  \
-            if (smem > 48 * 1024 && dev < 64 && !attr[dev]) {                                  \
-                cudaError_t e = cudaFuncSetAttribute(sgat_quant_kernel<E, NCV, Tin>,           \
+            static DeviceCache<int> attr;                                                      \
+            int done = 0;                                                                      \
+            const cudaError_t e = attr.get(&done, [](int, int* v) {                            \
+                *v = 1;                                                                        \
+                return cudaFuncSetAttribute(sgat_quant_kernel<E, NCV, Tin>,                    \
                         cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);              \
-                if (e != cudaSuccess) return e;                                                \
-                attr[dev] = true;                                                              \
-            }                                                                                  \
+            });                                                                                \
+            if (e != cudaSuccess) return e;                                                    \
             sgat_quant_kernel<E, NCV, Tin><<<grid, block, smem, stream>>>(a, wpr, rpc);        \
         }
     switch (nc) {

@@ -110,15 +110,13 @@ cudaError_t launch_g(const TacArgs& a, cudaStream_t stream) {
     constexpr int RC = G < 8 ? G : 8;
     constexpr int TM = (TPB / (G / RC)) * 4;
     constexpr size_t smem = (size_t)G * G * 4 + (size_t)TM * (G + 4) * 4;
-    static bool attr_set[64] = {false};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(tac_kernel<G, TIn, TOut>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        attr_set[dev] = true;
-    }
+    static DeviceCache<int> attr;
+    int done = 0;
+    const cudaError_t e = attr.get(&done, [](int, int* v) {
+        *v = 1;
+        return cudaFuncSetAttribute(tac_kernel<G, TIn, TOut>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    });
+    if (e != cudaSuccess) return e;
     dim3 grid((a.L + TM - 1) / TM, a.C / G);
     tac_kernel<G, TIn, TOut><<<grid, TPB, smem, stream>>>(a);
     return cudaGetLastError();
@@ -425,15 +423,8 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
 
 bool encode_u16_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
                      uint32_t box_cols) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        cudaDriverEntryPointQueryResult q;
-        void* f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
-            return false;
-        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-    }
+    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+    if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {cols * 2};
     const cuuint32_t box[2] = {box_cols, box_rows};
@@ -446,15 +437,8 @@ bool encode_u16_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t co
 // Output tensor map with 32 x 32 boxes: float (128-byte rows, 128-byte
 // swizzle) or a 16-bit type (64-byte rows, 64-byte swizzle).
 bool encode_out_tmap16or32(CUtensorMap* m, void* ptr, size_t elem, bool is_f16, uint64_t rows, uint64_t cols) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        cudaDriverEntryPointQueryResult q;
-        void* f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
-            return false;
-        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-    }
+    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+    if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {cols * elem};
     const cuuint32_t box[2] = {32, 32};
@@ -469,15 +453,14 @@ bool encode_out_tmap16or32(CUtensorMap* m, void* ptr, size_t elem, bool is_f16, 
 template <int G, typename TIn, typename TOut>
 cudaError_t launch_tc(const TacArgs& a, cudaStream_t stream) {
     using P = TacTc<G>;
-    static bool attr_set[64] = {false};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(tac_tc_kernel<G, TIn, TOut>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::SMEM);
-        if (e != cudaSuccess) return e;
-        attr_set[dev] = true;
-    }
+    static DeviceCache<int> attr;
+    int done = 0;
+    const cudaError_t e = attr.get(&done, [](int, int* v) {
+        *v = 1;
+        return cudaFuncSetAttribute(tac_tc_kernel<G, TIn, TOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)P::SMEM);
+    });
+    if (e != cudaSuccess) return e;
     CUtensorMap tz, to;
     if (!encode_u16_tmap(&tz, a.Z, (uint64_t)a.L, (uint64_t)a.C, TC_TM, 64)) return cudaErrorInvalidValue;
     if (!encode_out_tmap16or32(&to, a.out, sizeof(TOut), std::is_same<TOut, __half>::value, (uint64_t)a.L,

@@ -455,18 +455,17 @@ cudaError_t launch_tac_calibrate(const CalArgs& a, cudaStream_t stream) {
     }
     if (e != cudaSuccess) return e;
     const size_t smem = solve_smem(a.g);
-    static bool attr_set[64] = {false};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !attr_set[dev]) {
-        e = cudaFuncSetAttribute(tac_power_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)solve_smem(CAL_MAX_G));
-        if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(tac_final_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)solve_smem(CAL_MAX_G));
-        if (e != cudaSuccess) return e;
-        attr_set[dev] = true;
-    }
+    static DeviceCache<int> attr;
+    int done = 0;
+    e = attr.get(&done, [](int, int* v) {
+        *v = 1;
+        cudaError_t r = cudaFuncSetAttribute(tac_power_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)solve_smem(CAL_MAX_G));
+        if (r != cudaSuccess) return r;
+        return cudaFuncSetAttribute(tac_final_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)solve_smem(CAL_MAX_G));
+    });
+    if (e != cudaSuccess) return e;
     tac_power_kernel<<<dim3(B, 2), CAL_THREADS, smem, stream>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     tac_final_kernel<<<B, CAL_THREADS, smem, stream>>>(a);

@@ -424,9 +424,8 @@ w4a4_gemm_kernel(GemmArgs a) {
 // stage barrier, and its commits arrive on the stage / accumulator barriers
 // of both CTAs. Roles per CTA (20 warps): 0-7 epilogue, 8 TMA producers
 // (activations; raw weights), 9 TMEM allocation + (leader) MMA issue, 10-19
-// converters, two per stage buffer. When the output has at least two
-// channel tiles, clusters hold two pairs that share the activation tile:
-// CTAs r and r ^ 2 each load half of it and multicast it to both.
+// converters, two per stage buffer. Every CTA loads its own activation rows
+// (no cluster multicast).
 // ---------------------------------------------------------------------------
 namespace pairk {
 constexpr int BM = 128;                    // token rows per CTA (M = 256 per pair)
@@ -457,8 +456,8 @@ struct Smem {
     uint64_t raw_full[STAGES];    // packed weight tile landed (TMA bytes)
     uint64_t raw_empty[STAGES];   // converters done reading the packed tile
     uint64_t full[STAGES];        // leader: converter warps of the pair
-    uint64_t empty[STAGES];       // MMA commit of every pair (multicast)
-    uint64_t tmem_full[2];        // MMA commit (multicast to the pair)
+    uint64_t empty[STAGES];       // MMA commit (to both CTAs of the pair)
+    uint64_t tmem_full[2];        // MMA commit (to both CTAs of the pair)
     uint64_t tmem_empty[2];       // leader: epilogue warps of the pair
     uint64_t drain;
     uint32_t tmem_base;
@@ -466,7 +465,7 @@ struct Smem {
 };
 }  // namespace pairk
 
-template <typename TOut, int CL>
+template <typename TOut>
 __global__ void __launch_bounds__(pairk::THREADS, 1)
 w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
                       const __grid_constant__ CUtensorMap tmap_b) {
@@ -479,10 +478,8 @@ w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
     constexpr int NUM_EPI_WARPS = pairk::NUM_EPI_WARPS;
     constexpr int TMEM_COLS = pairk::TMEM_COLS;
     constexpr uint32_t IDESC = pairk::IDESC;
-    constexpr int PAIRS = CL / 2;                 // CTA pairs per cluster
-    constexpr uint16_t ALL = (uint16_t)((1u << CL) - 1u);
+    constexpr uint16_t PAIR = 3u;                 // both CTAs of the cluster (one pair)
     using Smem = pairk::Smem;
-    static_assert(CL == 2 || CL == 4, "");
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
@@ -492,22 +489,16 @@ w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const uint32_t rank = cluster_ctarank();
-    const uint32_t half = rank & 1u;             // position inside the CTA pair
-    const uint32_t pr = rank >> 1;               // which pair of the cluster
-    const uint32_t leader = rank & ~1u;
-    const uint16_t pair_mask = (uint16_t)(3u << (2 * pr));
+    const uint32_t half = cluster_ctarank();     // position inside the CTA pair
+    const uint32_t leader = 0;
     const int L = a.L, N = a.N, K = a.K;
-    // Cluster tile: 256 tokens x PAIRS * 256 channels. Pair p takes
-    // channels p * 256 .. + 255 of it; the pairs share the activation tile,
-    // which CTAs r and r ^ 2 (same token rows) load half each and multicast.
+    // Pair tile: 256 tokens x 256 channels.
     const int num_m = (L + 2 * BM - 1) / (2 * BM);
     const int num_n = (N + BN - 1) / BN;
-    const int num_np = (num_n + PAIRS - 1) / PAIRS;
-    const int num_tiles = num_m * num_np;
+    const int num_tiles = num_m * num_n;
     const int num_k = K / BK;
-    const int cluster = blockIdx.x / CL;
-    const int num_clusters = gridDim.x / CL;
+    const int cluster = blockIdx.x / 2;
+    const int num_clusters = gridDim.x / 2;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -515,7 +506,7 @@ w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
             mbar_init(smem_addr(&sh->raw_full[s]), 1);
             mbar_init(smem_addr(&sh->raw_empty[s]), CONV_WARPS_PER_STAGE);
             mbar_init(smem_addr(&sh->full[s]), 2 * CONV_WARPS_PER_STAGE);  // converter warps of the pair
-            mbar_init(smem_addr(&sh->empty[s]), PAIRS);                    // every pair's MMA commit
+            mbar_init(smem_addr(&sh->empty[s]), 1);                        // the pair's MMA commit
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_addr(&sh->tmem_full[b]), 1);
@@ -544,24 +535,16 @@ w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
-            // With two pairs, CTAs r and r ^ 2 hold the same token rows: each
-            // loads half of them and multicasts it to both.
-            const uint16_t a_mask = (uint16_t)((1u << rank) | (1u << ((rank ^ 2u) % CL)));
             for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters) {
                 const int m_rows = (tile % num_m) * 2 * BM + (int)half * BM;
-                const int n_rows = ((tile / num_m) * PAIRS + (int)pr) * BN + (int)half * BN_CTA;
+                const int n_rows = (tile / num_m) * BN + (int)half * BN_CTA;
                 for (int kc = 0; kc < num_k; ++kc) {
                     const uint32_t st = base + stage * STAGE_BYTES;
                     if (lane == 0) {
                         if (!mbar_wait_bounded(smem_addr(&sh->empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
                         const uint32_t bar = smem_addr(&sh->a_full[stage]);
                         mbar_arrive_expect_tx(bar, A_BYTES);
-                        if (CL == 2) {
-                            tma_load_2d(st, &tmap_a, kc * BK, m_rows, bar);
-                        } else {
-                            tma_load_2d_multicast(st + pr * (A_BYTES / 2), &tmap_a, kc * BK,
-                                                  m_rows + (int)pr * (BM / 2), bar, a_mask);
-                        }
+                        tma_load_2d(st, &tmap_a, kc * BK, m_rows, bar);
                     } else {
                         if (!mbar_wait_bounded(smem_addr(&sh->raw_empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
                         const uint32_t bar = smem_addr(&sh->raw_full[stage]);
@@ -634,14 +617,14 @@ w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
                         mma_f8f6f4_pair(d_tmem, smem_desc_sw128(sA + ks * UMMA_K),
                                         smem_desc_sw128(sB + ks * UMMA_K), IDESC,
                                         (kc > 0 || ks > 0) ? 1u : 0u);
-                    // the stage may be refilled once every pair of the cluster is done with it
-                    tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), ALL);
+                    // the stage may be refilled once the pair's MMAs are done with it
+                    tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), PAIR);
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
-                tc_commit_pair_multicast(smem_addr(&sh->tmem_full[acc]), pair_mask);
+                tc_commit_pair_multicast(smem_addr(&sh->tmem_full[acc]), PAIR);
             }
-            tc_commit_pair_multicast(smem_addr(&sh->drain), pair_mask);
+            tc_commit_pair_multicast(smem_addr(&sh->drain), PAIR);
             if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
         }
         __syncwarp();
@@ -660,7 +643,7 @@ w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
         TOut* Y = static_cast<TOut*>(a.Y);
         for (int tile = cluster; tile < num_tiles; tile += num_clusters, ++it) {
             const int m0 = (tile % num_m) * 2 * BM + (int)half * BM;
-            const int n0 = ((tile / num_m) * PAIRS + (int)pr) * BN;
+            const int n0 = (tile / num_m) * BN;
             const int acc = it & 1;
             const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
             const int row = m0 + quarter * 32 + lane;
@@ -746,15 +729,8 @@ w4a4_gemm_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
 // box_rows x box_cols bytes.
 bool encode_u8_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
                     uint32_t box_cols, CUtensorMapSwizzle swz) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        cudaDriverEntryPointQueryResult q;
-        void* f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
-            return false;
-        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-    }
+    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+    if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {cols};
     const cuuint32_t box[2] = {box_cols, box_rows};
@@ -768,15 +744,8 @@ bool encode_u8_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
 // elements, box box_rows x box_cols elements, 128-byte swizzle.
 bool encode_operand_tmap(CUtensorMap* m, const void* ptr, CUtensorMapDataType type, size_t elem, uint64_t rows,
                          uint64_t cols, uint32_t box_rows, uint32_t box_cols) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        cudaDriverEntryPointQueryResult q;
-        void* f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
-            return false;
-        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-    }
+    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+    if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {cols * elem};
     const cuuint32_t box[2] = {box_cols, box_rows};
@@ -789,15 +758,8 @@ bool encode_operand_tmap(CUtensorMap* m, const void* ptr, CUtensorMapDataType ty
 // Tensor map of the row-major output Y [rows][cols] with 32 x 32 boxes.
 bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t elem, uint64_t rows,
                      uint64_t cols, CUtensorMapSwizzle swz, uint32_t box_cols = 32) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        cudaDriverEntryPointQueryResult q;
-        void* f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
-            return false;
-        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-    }
+    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+    if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {cols * elem};
     const cuuint32_t box[2] = {box_cols, 32};
@@ -811,14 +773,12 @@ bool encode_out_tmap(CUtensorMap* m, void* ptr, CUtensorMapDataType type, size_t
 // from the quantiser, weight codes from w4_unpack_e4m3).
 //
 // The standard two-barrier pipeline: the TMA producer of each CTA waits for
-// the stage to be free (the MMA commits, multicast to the cluster) and loads
-// its 128 activation rows and 128 weight rows, the bytes counted on the
-// pair leader's stage barrier (cta_group::2); the leader's MMA thread waits
-// there and issues the four K = 32 MMAs of the stage (M 256, N 256).
-// CL = 4: two pairs on the same token rows and neighbouring channel tiles;
-// CTAs r and r ^ 2 need the same activation rows, so each loads half of
-// them and multicasts it to both, and a stage is free once both pairs'
-// MMAs have read it. 6 stages of 32 KB; 8 epilogue warps.
+// the stage to be free (the pair's MMA commit, which arrives in both CTAs)
+// and loads its 128 activation rows and BN / 2 weight rows, the bytes
+// counted on the pair leader's stage barrier (cta_group::2); the leader's
+// MMA thread waits there and issues the four K = 32 MMAs of the stage
+// (M 256, N BN). Every CTA loads only its own rows: no cluster multicast.
+// Up to 6 stages of 32 KB; 8 epilogue warps.
 // ---------------------------------------------------------------------------
 namespace tmak {
 constexpr int BM = 128, BK = 128, UMMA_K = 32;
@@ -844,7 +804,7 @@ struct Tile {
 template <int S>
 struct Smem {
     uint64_t full[S];             // pair leader: both CTAs' TMA bytes
-    uint64_t empty[S];            // MMA commits of every pair of the cluster
+    uint64_t empty[S];            // the pair's MMA commit
     uint64_t tmem_full[2];
     uint64_t tmem_empty[2];       // pair leader: epilogue warps of the pair
     uint64_t drain;
@@ -869,18 +829,18 @@ struct Cfg {
 // OPK: operand kind -- 0 = E4M3 codes (dequantising epilogue), 1 = fp16,
 // 2 = bf16 (plain float32 accumulator cast to the output type). Every kind
 // reads 128-byte K rows and advances 32 bytes of K per MMA.
-// Tile of the calling thread's last TMA pair GEMM launch: BN * 10 + CL.
+// Tile of the calling thread's last TMA pair GEMM launch: BN * 10 + 2 (CTAs
+// per cluster).
 thread_local int g_last_tile = 0;
 
-// Output tiles of the pair GEMM: 256-token rows x BN-channel pair tiles,
-// CL / 2 pairs side by side per cluster tile.
-int tma_tiles(int L, int N, int BN, int CL) {
+// Output tiles of the pair GEMM: 256-token rows x BN-channel pair tiles.
+int tma_tiles(int L, int N, int BN) {
     const int num_n = (N + BN - 1) / BN;
-    return ((L + 2 * tmak::BM - 1) / (2 * tmak::BM)) * ((num_n + CL / 2 - 1) / (CL / 2));
+    return ((L + 2 * tmak::BM - 1) / (2 * tmak::BM)) * num_n;
 }
 // Estimated cycles of a launch (twice the model's stage cycles per round).
-long long tma_round_cost(int L, int N, int BN, int CL, int clusters) {
-    const long long tiles = tma_tiles(L, N, BN, CL);
+long long tma_round_cost(int L, int N, int BN, int clusters) {
+    const long long tiles = tma_tiles(L, N, BN);
     const long long used = clusters < 1 ? 1 : clusters;
     const long long rounds = (tiles + used - 1) / used;
     const long long stage2 = 4LL * BN > 512LL + 3LL * BN ? 4LL * BN : 512LL + 3LL * BN;
@@ -891,7 +851,7 @@ long long tma_round_cost(int L, int N, int BN, int CL, int clusters) {
 // 16 k .. 16 k + 15, then the matching up rows), so every 32-column chunk
 // of the accumulator holds 16 gate and 16 up channels; the epilogue writes
 // silu(gate) * up, rounded once, to column nc / 2 of an [L][N / 2] output.
-template <typename TOut, int CL, int OPK, int BN, bool SWIGLU = false>
+template <typename TOut, int OPK, int BN, bool SWIGLU = false>
 __global__ void __launch_bounds__(tmak::THREADS, 1)
 w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
                           const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y) {
@@ -908,10 +868,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     constexpr uint32_t IDESC = Tile::IDESC | (OPK == 2 ? ((1u << 7) | (1u << 10)) : 0u);
     constexpr int BKE = OPK == 0 ? BK : BK / 2;          // K elements per stage row
     constexpr bool DEQUANT = OPK == 0;
-    constexpr int PAIRS = CL / 2;
-    constexpr uint16_t ALL = (uint16_t)((1u << CL) - 1u);
+    constexpr uint16_t PAIR = 3u;                        // both CTAs of the cluster (one pair)
     using Smem = tmak::Smem<STAGES>;
-    static_assert(CL == 2 || CL == 4, "one or two CTA pairs per cluster");
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
@@ -921,20 +879,18 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     Smem* sh = reinterpret_cast<Smem*>(smem_raw + (base - raw) + STAGES * STAGE_BYTES + EPI_STAGE_BYTES);
     volatile int* abort = &sh->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t rank = cluster_ctarank();
-    const uint32_t half = rank & 1u, pr = rank >> 1, leader = rank & ~1u;
-    const uint16_t pair_mask = (uint16_t)(3u << (2 * pr));
+    const uint32_t half = cluster_ctarank(), leader = 0;
     const int L = a.L, N = a.N, K = a.K;
     const int num_m = (L + 2 * BM - 1) / (2 * BM);
     const int num_n = (N + BN - 1) / BN;
-    const int num_tiles = num_m * ((num_n + PAIRS - 1) / PAIRS);
+    const int num_tiles = num_m * num_n;
     const int num_k = K / BKE;
-    const int cluster = blockIdx.x / CL, num_clusters = gridDim.x / CL;
+    const int cluster = blockIdx.x / 2, num_clusters = gridDim.x / 2;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(smem_addr(&sh->full[s]), 1);
-            mbar_init(smem_addr(&sh->empty[s]), PAIRS);
+            mbar_init(smem_addr(&sh->empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(smem_addr(&sh->tmem_full[b]), 1);
@@ -962,13 +918,12 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     // uniform control flow and descriptors); one elected lane issues.
     if (warp == TMA_WARP) {
         const uint32_t leader_full0 = mapa_shared(smem_addr(&sh->full[0]), leader);
-        const uint16_t a_mask = (uint16_t)((1u << rank) | (1u << ((rank ^ 2u) % CL)));
         // weight tiles of the first stages ahead of the wait for the previous
         // kernel (their stage barriers are fresh, so no empty wait is due)
         int pre = 0;
         if (a.weights_ready && cluster < num_tiles) {
             pre = num_k < STAGES ? num_k : STAGES;
-            const int n_rows = ((cluster / num_m) * PAIRS + (int)pr) * BN + (int)half * BN_CTA;
+            const int n_rows = (cluster / num_m) * BN + (int)half * BN_CTA;
             for (int kc = 0; kc < pre; ++kc) {
                 if (elect_one()) {
                     if (half == 0) mbar_arrive_expect_tx(smem_addr(&sh->full[kc]), 2 * (A_BYTES + B_BYTES));
@@ -984,7 +939,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         bool ok = true;
         for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters) {
             const int m_rows = (tile % num_m) * 2 * BM + (int)half * BM;
-            const int n_rows = ((tile / num_m) * PAIRS + (int)pr) * BN + (int)half * BN_CTA;
+            const int n_rows = (tile / num_m) * BN + (int)half * BN_CTA;
             for (int kc = 0; kc < num_k; ++kc) {
                 const bool early = tile == cluster && kc < pre;  // weights already in flight
                 if (!early && !mbar_wait_bounded_warp(smem_addr(&sh->empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
@@ -992,12 +947,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 const uint32_t bar = leader_full0 + stage * 8;
                 if (elect_one()) {
                     if (half == 0 && !early) mbar_arrive_expect_tx(smem_addr(&sh->full[stage]), 2 * (A_BYTES + B_BYTES));
-                    if (CL == 2) {
-                        tma_load_2d_pair(st, &tmap_a, kc * BKE, m_rows, bar);
-                    } else {
-                        tma_load_2d_pair_multicast(st + pr * (A_BYTES / 2), &tmap_a, kc * BKE,
-                                                   m_rows + (int)pr * (BM / 2), bar, a_mask);
-                    }
+                    tma_load_2d_pair(st, &tmap_a, kc * BKE, m_rows, bar);
                     if (!early) tma_load_2d_pair(st + A_BYTES, &tmap_b, kc * BKE, n_rows, bar);
                 }
                 __syncwarp();
@@ -1033,16 +983,16 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                             if (OPK == 0) mma_f8f6f4_pair(d_tmem, adk, bdk, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
                             else mma_f16_pair(d_tmem, adk, bdk, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
                         }
-                        tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), ALL);
+                        tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), PAIR);
                     }
                     __syncwarp();
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
-                if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->tmem_full[acc]), pair_mask);
+                if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->tmem_full[acc]), PAIR);
                 __syncwarp();
             }
-            if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->drain), pair_mask);
+            if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->drain), PAIR);
             __syncwarp();
             if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
         }
@@ -1066,7 +1016,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         int nbox = 0;
         for (int tile = cluster; tile < num_tiles; tile += num_clusters, ++it) {
             const int m0 = (tile % num_m) * 2 * BM + (int)half * BM;
-            const int n0 = ((tile / num_m) * PAIRS + (int)pr) * BN;
+            const int n0 = (tile / num_m) * BN;
             const int acc = it & 1;
             const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
             const int row = m0 + quarter * 32 + lane;
@@ -1190,47 +1140,44 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     if (warp == MMA_WARP) tmem_dealloc_pair(tmem_base, TMEM_COLS);
 }
 
-// Clusters of this instantiation resident at once on the current device
-// (queried once per device; also sets the kernel's shared-memory limit).
-template <typename TOut, int CL, int OPK, int BN, bool SW>
+// Clusters (CTA pairs) of this instantiation resident at once on the current
+// device (queried once per device; also sets the kernel's shared-memory
+// limit).
+template <typename TOut, int OPK, int BN, bool SW>
 cudaError_t tma_max_clusters(int* clusters) {
     constexpr size_t SMEM_BYTES = tmak::Cfg<sizeof(TOut), BN>::SMEM_BYTES;
-    auto kernel = w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN, SW>;
-    static int max_clusters[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 0 || dev >= 64) dev = 63;
-    if (max_clusters[dev] == 0) {
+    static DeviceCache<int> cache;
+    return cache.get(clusters, [](int, int* v) {
+        auto kernel = w4a4_gemm_tma_pair_kernel<TOut, OPK, BN, SW>;
         cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
         if (e != cudaSuccess) return e;
         cudaLaunchConfig_t cfg = {};
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = CL;
+        attr[0].val.clusterDim.x = 2;
         attr[0].val.clusterDim.y = 1;
         attr[0].val.clusterDim.z = 1;
         cfg.blockDim = dim3(tmak::THREADS);
         cfg.dynamicSmemBytes = SMEM_BYTES;
         cfg.attrs = attr;
         cfg.numAttrs = 1;                // the occupancy query takes the cluster shape only
-        cfg.gridDim = dim3(CL * 32);
+        cfg.gridDim = dim3(2 * 32);
         int n = 0;
         e = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg);
         if (e != cudaSuccess) return e;
-        max_clusters[dev] = n > 0 ? n : 1;
-    }
-    *clusters = max_clusters[dev];
-    return cudaSuccess;
+        *v = n > 0 ? n : 1;
+        return cudaSuccess;
+    });
 }
 
-template <typename TOut, int CL, int OPK, int BN, bool SW>
+template <typename TOut, int OPK, int BN, bool SW>
 cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) {
     constexpr int BM = tmak::BM, BN_CTA = tmak::Tile<BN>::BN_CTA, BK = tmak::BK;
     constexpr int ELEM = OPK == 0 ? 1 : 2;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     attr[1] = pdl_attribute();
@@ -1241,45 +1188,40 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) 
     cfg.numAttrs = 2;
     CUtensorMap ta, tb, ty;
     const CUtensorMapDataType opt = OPK == 0 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
-    if (!encode_operand_tmap(&ta, a.Xe, opt, ELEM, (uint64_t)a.L, (uint64_t)a.K, CL == 2 ? BM : BM / 2, BK / ELEM) ||
+    if (!encode_operand_tmap(&ta, a.Xe, opt, ELEM, (uint64_t)a.L, (uint64_t)a.K, BM, BK / ELEM) ||
         !encode_operand_tmap(&tb, a.We, opt, ELEM, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK / ELEM) ||
         !(SW ? encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N / 2,
                                CU_TENSOR_MAP_SWIZZLE_32B, 16)
              : encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N,
                                Out<TOut>::TMAP_SWIZZLE)))
         return cudaErrorInvalidValue;
-    const int num_tiles = tma_tiles(a.L, a.N, BN, CL);
+    const int num_tiles = tma_tiles(a.L, a.N, BN);
     if (num_tiles < clusters) clusters = num_tiles;
-    cfg.gridDim = dim3(CL * clusters);
-    return cudaLaunchKernelEx(&cfg, w4a4_gemm_tma_pair_kernel<TOut, CL, OPK, BN, SW>, a, ta, tb, ty);
+    cfg.gridDim = dim3(2 * clusters);
+    return cudaLaunchKernelEx(&cfg, w4a4_gemm_tma_pair_kernel<TOut, OPK, BN, SW>, a, ta, tb, ty);
 }
 
 // Tile shape per problem. A stage's steady state is bound by shared memory:
 // per CTA the MMAs read the 16 KB activation tile and the CTA's weight half
 // twice (for itself and for its pair peer) while TMA writes both, i.e.
 // 256 + 1.5 BN cycles at 128 bytes per clock against 2 BN cycles of tensor
-// work. A launch takes ceil(tiles / clusters) rounds of a tile's stages.
-// Candidates: 256-wide pair tiles (two pairs per cluster sharing the
-// activation tile when there are at least two channel tiles) and 224-wide
-// tiles on single pairs, whose tile counts fill the 76 pairs of the LLaDA
-// projections better; the cheaper estimate wins, ties keep 256.
+// work. A launch takes ceil(tiles / pairs) rounds of a tile's stages.
+// Candidates: 256- and 224-channel pair tiles (224 fills the 76 pairs of
+// the LLaDA projections better); the cheaper estimate wins, ties keep 256.
 template <typename TOut, int OPK, bool SW>
 cudaError_t launch_tma_shape(const GemmArgs& a, cudaStream_t stream) {
-    const bool quad = (a.N + 255) / 256 >= 2;
     int c256 = 0, c224 = 0;
-    cudaError_t e = quad ? tma_max_clusters<TOut, 4, OPK, 256, SW>(&c256)
-                         : tma_max_clusters<TOut, 2, OPK, 256, SW>(&c256);
+    cudaError_t e = tma_max_clusters<TOut, OPK, 256, SW>(&c256);
     if (e != cudaSuccess) return e;
-    if ((e = tma_max_clusters<TOut, 2, OPK, 224, SW>(&c224)) != cudaSuccess) return e;
-    const long long t256 = tma_round_cost(a.L, a.N, 256, quad ? 4 : 2, c256);
-    const long long t224 = tma_round_cost(a.L, a.N, 224, 2, c224);
+    if ((e = tma_max_clusters<TOut, OPK, 224, SW>(&c224)) != cudaSuccess) return e;
+    const long long t256 = tma_round_cost(a.L, a.N, 256, c256);
+    const long long t224 = tma_round_cost(a.L, a.N, 224, c224);
     if (t224 < t256) {
         g_last_tile = 224 * 10 + 2;
-        return launch_tma_cl<TOut, 2, OPK, 224, SW>(a, stream, c224);
+        return launch_tma_cl<TOut, OPK, 224, SW>(a, stream, c224);
     }
-    g_last_tile = 256 * 10 + (quad ? 4 : 2);
-    return quad ? launch_tma_cl<TOut, 4, OPK, 256, SW>(a, stream, c256)
-                : launch_tma_cl<TOut, 2, OPK, 256, SW>(a, stream, c256);
+    g_last_tile = 256 * 10 + 2;
+    return launch_tma_cl<TOut, OPK, 256, SW>(a, stream, c256);
 }
 
 template <typename TOut, int OPK = 0>
@@ -1306,23 +1248,22 @@ __global__ void __launch_bounds__(256) unpack_e4m3_kernel(const uint4* __restric
     }
 }
 
-// Cluster size of the CTA-pair GEMM: 4 (two pairs sharing the activation
-// tile by multicast) unless fewer than two clusters of 4 fit, then 2.
-template <typename TOut, int CL>
-cudaError_t launch_pair_cl(const GemmArgs& a, cudaStream_t stream, const CUtensorMap& ta,
-                           const CUtensorMap& tb) {
-    constexpr int BM = pairk::BM, BN = pairk::BN;
+// The CTA-pair GEMM that converts packed weights: one pair per cluster, as
+// many clusters as are resident at once (queried once per device).
+template <typename TOut>
+cudaError_t launch_pair_typed(const GemmArgs& a, cudaStream_t stream) {
+    constexpr int BM = pairk::BM, BN = pairk::BN, BN_CTA = pairk::BN_CTA, BK = pairk::BK;
     constexpr int THREADS = pairk::THREADS;
     constexpr size_t SMEM_BYTES = pairk::SMEM_BYTES;
-    auto kernel = w4a4_gemm_pair_kernel<TOut, CL>;
-    static bool attr_set[64] = {false};
-    static int max_clusters[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
+    CUtensorMap ta, tb;
+    if (!encode_u8_tmap(&ta, a.Xe, (uint64_t)a.L, (uint64_t)a.K, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_u8_tmap(&tb, a.Wq, (uint64_t)a.N, (uint64_t)a.K / 2, BN_CTA, BK / 2, CU_TENSOR_MAP_SWIZZLE_NONE))
+        return cudaErrorInvalidValue;
+    auto kernel = w4a4_gemm_pair_kernel<TOut>;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.blockDim = dim3(THREADS);
@@ -1330,52 +1271,36 @@ cudaError_t launch_pair_cl(const GemmArgs& a, cudaStream_t stream, const CUtenso
     cfg.stream = stream;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
-        if (e != cudaSuccess) return e;
-        cfg.gridDim = dim3(CL * 64);
+    static DeviceCache<int> cache;
+    int clusters = 0;
+    cudaError_t e = cache.get(&clusters, [&](int, int* v) {
+        cudaError_t r = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+        if (r != cudaSuccess) return r;
+        cudaLaunchConfig_t q = cfg;
+        q.gridDim = dim3(2 * 64);
         int n = 0;
-        e = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg);
-        if (e != cudaSuccess) return e;
-        max_clusters[dev] = n;
-        attr_set[dev] = true;
-    }
-    const int pairs_per_cluster = CL / 2;
-    const int num_tiles = ((a.L + 2 * BM - 1) / (2 * BM)) *
-                          (((a.N + BN - 1) / BN + pairs_per_cluster - 1) / pairs_per_cluster);
-    int clusters = dev < 64 ? max_clusters[dev] : 1;
-    if (clusters < 1) clusters = 1;
+        r = cudaOccupancyMaxActiveClusters(&n, kernel, &q);
+        if (r != cudaSuccess) return r;
+        *v = n > 0 ? n : 1;
+        return cudaSuccess;
+    });
+    if (e != cudaSuccess) return e;
+    const int num_tiles = ((a.L + 2 * BM - 1) / (2 * BM)) * ((a.N + BN - 1) / BN);
     if (num_tiles < clusters) clusters = num_tiles;
-    cfg.gridDim = dim3(CL * clusters);
+    cfg.gridDim = dim3(2 * clusters);
     return cudaLaunchKernelEx(&cfg, kernel, a, ta, tb);
 }
 
 template <typename TOut>
-cudaError_t launch_pair_typed(const GemmArgs& a, cudaStream_t stream) {
-    constexpr int BM = pairk::BM, BN_CTA = pairk::BN_CTA, BK = pairk::BK;
-    CUtensorMap ta2, ta4, tb;
-    if (!encode_u8_tmap(&ta2, a.Xe, (uint64_t)a.L, (uint64_t)a.K, BM, BK, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_u8_tmap(&ta4, a.Xe, (uint64_t)a.L, (uint64_t)a.K, BM / 2, BK, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_u8_tmap(&tb, a.Wq, (uint64_t)a.N, (uint64_t)a.K / 2, BN_CTA, BK / 2, CU_TENSOR_MAP_SWIZZLE_NONE))
-        return cudaErrorInvalidValue;
-    // two pairs per cluster (sharing the activation tile) when the
-    // channel tiles come in pairs
-    const bool quad = ((a.N + pairk::BN - 1) / pairk::BN) >= 2;
-    return quad ? launch_pair_cl<TOut, 4>(a, stream, ta4, tb) : launch_pair_cl<TOut, 2>(a, stream, ta2, tb);
-}
-
-template <typename TOut>
 cudaError_t launch_typed(const GemmArgs& a, cudaStream_t stream) {
-    static bool attr_set[64] = {false};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<TOut>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)SMEM_BYTES);
-        if (e != cudaSuccess) return e;
-        attr_set[dev] = true;
-    }
+    static DeviceCache<int> attr;
+    int done = 0;
+    cudaError_t e = attr.get(&done, [](int, int* v) {
+        *v = 1;
+        return cudaFuncSetAttribute(w4a4_gemm_kernel<TOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)SMEM_BYTES);
+    });
+    if (e != cudaSuccess) return e;
     const int num_tiles = ((a.L + BM - 1) / BM) * ((a.N + BN - 1) / BN);
     const int grid = num_tiles < num_sms() ? num_tiles : num_sms();
     w4a4_gemm_kernel<TOut><<<grid, THREADS, SMEM_BYTES, stream>>>(a);

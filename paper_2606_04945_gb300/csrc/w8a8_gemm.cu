@@ -243,15 +243,8 @@ __global__ void __launch_bounds__(256) w8_split_kernel(const uint8_t* Wq, uint8_
 }
 
 bool encode_split_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        cudaDriverEntryPointQueryResult q;
-        void* f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess || q != cudaDriverEntryPointSuccess || f == nullptr)
-            return false;
-        fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
-    }
+    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
+    if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {cols};
     const cuuint32_t box[2] = {W8_BK, 128};
@@ -263,15 +256,13 @@ bool encode_split_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t 
 
 template <typename TOut>
 cudaError_t launch_typed(const GemmArgs& a, const CUtensorMap& ta, const CUtensorMap& tw, cudaStream_t stream) {
-    static bool attr_set[64] = {false};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !attr_set[dev]) {
-        const cudaError_t e =
-            cudaFuncSetAttribute(w8a8_gemm_kernel<TOut>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)W8_SMEM);
-        if (e != cudaSuccess) return e;
-        attr_set[dev] = true;
-    }
+    static DeviceCache<int> attr;
+    int done = 0;
+    const cudaError_t e = attr.get(&done, [](int, int* v) {
+        *v = 1;
+        return cudaFuncSetAttribute(w8a8_gemm_kernel<TOut>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)W8_SMEM);
+    });
+    if (e != cudaSuccess) return e;
     const dim3 grid((a.L + W8_BM - 1) / W8_BM, a.N / W8_BN);
     w8a8_gemm_kernel<TOut><<<grid, W8_THREADS, W8_SMEM, stream>>>(a, ta, tw);
     return cudaGetLastError();

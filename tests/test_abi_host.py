@@ -264,3 +264,46 @@ def test_zero_point_decomposition_rule_covers_the_k_limit():
         assert len(terms) <= 5
         worst = max(worst, n448 + len(terms))
     assert worst <= 128
+
+
+def test_validation_from_eight_threads(lib):
+    """Eight host threads call validation-only paths at once. Each thread
+    gets its own return code and its own last-error message (the message is
+    per thread), and calls that pass validation reach the per-device caches
+    (which on a machine without a GPU fail cleanly with STARQ_ERR_CUDA
+    instead of racing)."""
+    import threading
+    import torch
+
+    lib_ = lib.lib
+    gpu = torch.cuda.is_available()
+    errors = []
+    barrier = threading.Barrier(8)
+
+    def worker(t):
+        try:
+            barrier.wait()
+            for it in range(200):
+                K = 100 + 16 * t                     # K % 16 != 0 for every t: a shape error
+                rc = lib_.sgat_quantize_act(P, 0, 4, K, None, None, None, 4, K, 0, 0, 4, P, P, None, None, None)
+                msg = lib_.starq_last_error().decode()
+                if rc != -2 or f"K={K}" not in msg:
+                    errors.append((t, it, rc, msg))
+                rc = lib_.w8a8_gemm(P, P, P, P, None, 4, 96 + 0 * t, 512, P, 0, None, None)
+                if rc != -2:
+                    errors.append((t, it, "w8a8", rc))
+                if not gpu:
+                    # valid arguments: the call reaches the device-side lookups and
+                    # fails there without a device
+                    rc = lib_.tac_prepare(P, 256, 64, 0, P, None)
+                    if rc != lib.ERR_CUDA:
+                        errors.append((t, it, "tac_prepare", rc))
+        except Exception as e:  # pragma: no cover
+            errors.append((t, repr(e)))
+
+    threads = [threading.Thread(target=worker, args=(t,)) for t in range(8)]
+    for th in threads:
+        th.start()
+    for th in threads:
+        th.join()
+    assert not errors, errors[:5]
