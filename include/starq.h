@@ -77,6 +77,20 @@ const char* starq_last_error(void);
 int starq_check_status(void* stream);
 
 /*
+ * starq_selftest_wait_timeout -- failure-detection self-test (the paper has
+ * no counterpart). Launches one kernel whose single thread waits on an
+ * mbarrier that nothing arrives on, through the library's bounded wait,
+ * with a limit of limit_us microseconds (1 .. 100000). The wait runs out,
+ * the kernel sets the status bit 0x4 (self-test timeout) and returns: no
+ * fault, no hang, and the context stays usable. The next
+ * starq_check_status on the device then returns STARQ_ERR_TIMEOUT with the
+ * bit in its message and clears the word. Returns STARQ_OK once launched,
+ * STARQ_ERR_ARG for a limit outside the range, STARQ_ERR_CUDA if the launch
+ * fails.
+ */
+int starq_selftest_wait_timeout(unsigned limit_us, void* stream);
+
+/*
  * sgat_quantize_act -- state-guided activation transform + per-token A4
  * quantisation (Sec. 3.2 Eq. 7-11 and Eq. 13's Q_a; Sec. 3.1 Eq. 2-3).
  *

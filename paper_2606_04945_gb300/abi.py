@@ -26,6 +26,7 @@ EXPORTED = (
     "sgat_quantize_act_asym", "w4_zero_point_columns", "sgat_linear_asym_workspace_size", "sgat_linear_asym",
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
     "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
+    "starq_selftest_wait_timeout",
 )
 
 
@@ -44,6 +45,7 @@ def _load():
     lib.starq_version.restype = i
     lib.starq_last_error.restype = ctypes.c_char_p
     lib.starq_check_status.argtypes = [vp]
+    lib.starq_selftest_wait_timeout.argtypes = [ctypes.c_uint, vp]
     lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, i, u8p, f_p, u8p, f_p, vp]
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
@@ -118,6 +120,13 @@ def _contig(*ts):
 def check_status(stream=None):
     """Synchronise and raise if a kernel gave up a bounded wait."""
     _check(lib.starq_check_status(_stream(stream)))
+
+
+def selftest_wait_timeout(limit_us, stream=None):
+    """Launch the bounded-wait self-test kernel (a wait on a barrier nobody
+    arms, given up after limit_us); the next check_status raises
+    StarqError(ERR_TIMEOUT)."""
+    _check(lib.starq_selftest_wait_timeout(int(limit_us), _stream(stream)))
 
 
 def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, bits=4, Xe=None, v_dbg=None,

@@ -166,6 +166,25 @@ int check_w8a8(const uint8_t* Xe, const float* s_a, const uint8_t* We, const flo
 
 int report_error(int code, const char* msg) { return fail(code, "%s", msg); }
 
+namespace {
+// Failure-detection self-test: one thread waits on an mbarrier that nothing
+// ever arrives on, through the same bounded wait as every pipeline wait of
+// the library (with a short limit), gives up, records STATUS_TIMEOUT_TEST in
+// the status word and returns. Nothing faults and the context stays usable.
+__global__ void selftest_wait_timeout_kernel(unsigned* status, unsigned long long limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort;
+    if (threadIdx.x == 0) {
+        abort = 0;
+        mbar_init(smem_addr(&bar), 1);       // expects one arrival, which never comes
+        mbar_fence_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !mbar_wait_limit(smem_addr(&bar), 0, &abort, limit_ns))
+        atomicOr(status, STATUS_TIMEOUT_TEST);
+}
+}  // namespace
+
 int num_sms() {
     static DeviceCache<int> cache;
     int n = 1;
@@ -214,6 +233,18 @@ int starq_check_status(void* stream) {
         if (e != cudaSuccess) return cuda_fail(e, "clear status word");
         return fail(STARQ_ERR_TIMEOUT, "a kernel gave up a bounded wait (status bits 0x%x)", v);
     }
+    return STARQ_OK;
+}
+
+int starq_selftest_wait_timeout(unsigned limit_us, void* stream) {
+    if (limit_us < 1 || limit_us > 100000)
+        return fail(STARQ_ERR_ARG, "starq_selftest_wait_timeout: limit_us=%u outside [1, 100000]", limit_us);
+    int rc = STARQ_OK;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    selftest_wait_timeout_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(st, 1000ull * limit_us);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "starq_selftest_wait_timeout launch");
     return STARQ_OK;
 }
 

@@ -206,10 +206,10 @@ __device__ __forceinline__ bool elect_one() {
 }
 
 // Wait for the phase of `bar` with the given parity to complete. Gives up
-// (returns false) after WAIT_LIMIT_NS, or early when *abort is set by another
-// role of the same CTA that has already given up.
-__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
-                                                  volatile int* abort) {
+// (returns false) after limit_ns nanoseconds, or early when *abort is set by
+// another role of the same CTA that has already given up.
+__device__ __forceinline__ bool mbar_wait_limit(uint32_t bar, uint32_t parity, volatile int* abort,
+                                                unsigned long long limit_ns) {
     #pragma unroll 1
     for (int i = 0; i < 256; ++i)
         if (mbar_try_wait(bar, parity)) return true;
@@ -218,8 +218,14 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort) return false;
-        if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) return false;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
     }
+}
+
+// The same with the library-wide limit WAIT_LIMIT_NS.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
+                                                  volatile int* abort) {
+    return mbar_wait_limit(bar, parity, abort, WAIT_LIMIT_NS);
 }
 
 // Same, polling every `sleep_ns` nanoseconds: for waits that are not on a

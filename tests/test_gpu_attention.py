@@ -32,12 +32,16 @@ pytestmark = pytest.mark.gpu
 D = 128
 
 
-def run_case(abi, L, Hh, seed, heads=None, zero_q=False):
+def run_case(abi, L, Hh, seed, heads=None, zero_q=False, v_signs=None):
+    """v_signs: per-channel signs [128 H]; V is then +-1 down each column,
+    so every V code is +-7."""
     rng = np.random.default_rng(seed)
     C = D * Hh
     QKV = rng.standard_normal((L, 3 * C)).astype(np.float16)
     if zero_q:
         QKV[:, :C] = 0
+    if v_signs is not None:
+        QKV[:, 2 * C:] = np.broadcast_to(np.asarray(v_signs, np.float16)[None, :], (L, C))
     Y = torch.from_numpy(QKV).cuda()
     Q, K, V = Y[:, :C], Y[:, C:2 * C], Y[:, 2 * C:]
     tac = inputs.make_tac(rng, C, D)
@@ -80,8 +84,46 @@ def test_attention_pv_tac_matches_oracle(abi, L, Hh):
 
 def test_attention_pv_tac_llada_width(abi):
     """1024 tokens, 32 heads of 128 (the LLaDA-8B attention width): every
-    head computed, three checked against the oracle."""
-    run_case(abi, 1024, 32, seed=11, heads=(0, 17, 31))
+    head checked against the oracle."""
+    run_case(abi, 1024, 32, seed=11)
+
+
+@pytest.mark.parametrize("L,Hh", [(2048, 2), (8192, 1)])
+def test_attention_pv_tac_long(abi, L, Hh):
+    """The Dream-7B sequence length (2048) and the longest supported one
+    (8192): 16 and 64 key chunks per query tile, every head checked."""
+    run_case(abi, L, Hh, seed=L + 7 * Hh)
+
+
+def test_attention_pv_tac_exact_at_2_24_edge(abi):
+    """The largest integer sums the kernel can meet: L = 8192 with Q = 0
+    (every P code 255) and V = +-1 down each channel (every V code +-7), so
+    acc = +-255 * 7 * 8192 = +-14,622,720, just below 2^24 = 16,777,216
+    where float32 would stop holding every integer. The sums must come back
+    exact, and Z_hat = acc / (255 l) * t = +-1 before TAC."""
+    L, Hh = 8192, 1
+    signs = np.where(np.random.default_rng(5).random(D * Hh) < 0.5, -1.0, 1.0)
+    rng = np.random.default_rng(9)
+    C = D * Hh
+    QKV = np.zeros((L, 3 * C), np.float16)
+    QKV[:, C:2 * C] = rng.standard_normal((L, C)).astype(np.float16)
+    QKV[:, 2 * C:] = np.broadcast_to(signs.astype(np.float16)[None, :], (L, C))
+    Y = torch.from_numpy(QKV).cuda()
+    tac = inputs.make_tac(rng, C, D)
+    Mp = torch.empty(abi.tac_prepared_bytes(C, D), dtype=torch.uint8, device="cuda")
+    abi.tac_prepare(H.dev(tac.M), D, torch.float16, Mp)
+    Z = torch.full((L, C), float("nan"), dtype=torch.float16, device="cuda")
+    acc = torch.zeros(Hh, L, D, dtype=torch.int32, device="cuda")
+    lsum = torch.zeros(Hh, L, dtype=torch.float32, device="cuda")
+    abi.attention_pv_tac(Y[:, :C], Y[:, C:2 * C], Y[:, 2 * C:], Hh, Mp, H.dev(tac.d), Z, dbg_l=lsum, dbg_acc=acc)
+    abi.check_status()
+    expect = (255 * 7 * L) * signs.astype(np.int64)
+    assert 255 * 7 * L == 14622720 < 2 ** 24
+    assert np.array_equal(acc.cpu().numpy()[0], np.broadcast_to(expect[None, :], (L, D)))
+    assert np.all(lsum.cpu().numpy() == float(L))                  # exp(0) summed exactly
+    zhat = np.broadcast_to(signs[None, :], (L, D)).astype(np.float64)
+    ref = zhat @ tac.M[0].astype(np.float64).T + tac.d[0].astype(np.float64)[None, :]
+    H.assert_tac_close(H.host(Z), ref, "f16")
 
 
 def test_attention_pv_tac_uniform(abi):
