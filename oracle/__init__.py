@@ -18,7 +18,10 @@ Every function is a plain, slow restatement of the paper:
   singular-value smoothing, identity shrinkage, bias).
 * ``attention``: the quantised softmax-value product of Sec. 3.3 (Z_hat,
   8-bit per-row P and 4-bit per-channel V: readings, the paper fixes
-  neither) and TAC on it, one block per head.
+  neither) and TAC on it, one block per head; grouped-query heads.
+* ``glue``: the block's glue around the quantised linears (RMSNorm, rotary
+  embedding, SwiGLU), standard definitions of the model family, not the
+  paper's method.
 
 Floating point: the transform and the quantiser decision run in float32, the
 precision the CUDA kernels take the integer decision in (a quantised code is
@@ -32,4 +35,4 @@ closed forms, brute force on tiny inputs, hand-worked fixtures in
 "parity unpinned".
 """
 
-from . import attention, sgat, tac  # noqa: F401
+from . import attention, glue, sgat, tac  # noqa: F401

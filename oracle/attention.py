@@ -22,6 +22,10 @@ bit widths nor its granularity. The readings here:
 * Z_hat_ic = (1 / (255 l_i)) * t_c * sum_j c_ij v_jc;
 * TAC per head: Z_tac = Z_hat_h M_h^T + 1 d_h^T. The head's d channels are
   one TAC block (g = d).
+* grouped-query attention (the Dream-7B / Qwen2.5 block): H query heads
+  share Hkv key/value heads, query head h reading key/value head
+  h // (H / Hkv); V is quantised per channel of the Hkv heads, so a group of
+  query heads shares one set of V codes and scales.
 """
 
 import numpy as np
@@ -54,14 +58,18 @@ def v_codes(V):
     return q.T.copy(), t
 
 
-def quantised_attention(Q, K, V, H, d):
-    """Z_hat [L][H d] for tokens Q, K, V [L][H d] (head h = channels
-    h d .. h d + d - 1).
+def quantised_attention(Q, K, V, H, d, Hkv=None):
+    """Z_hat [L][H d] for query tokens Q [L][H d] and key/value tokens K, V
+    [L][Hkv d] (head h = channels h d .. h d + d - 1; query head h reads
+    key/value head h // (H / Hkv); Hkv defaults to H).
 
     Returns (Z_hat float64, P codes int32 [H, L, L], l [H, L], V codes int32
-    [L, H d], t float32 [H d], acc int64 [H, L, d]).
+    [L, Hkv d], t float32 [Hkv d], acc int64 [H, L, d]).
     """
     Q, K, V = (np.asarray(x) for x in (Q, K, V))
+    Hkv = H if Hkv is None else Hkv
+    assert H % Hkv == 0 and K.shape[1] == V.shape[1] == Hkv * d
+    group = H // Hkv
     L = Q.shape[0]
     vq, t = v_codes(V)
     Z = np.empty((L, H * d), F64)
@@ -70,16 +78,17 @@ def quantised_attention(Q, K, V, H, d):
     acc = np.empty((H, L, d), np.int64)
     for h in range(H):
         ch = slice(h * d, (h + 1) * d)
-        c, l = p_codes(scores(Q[:, ch], K[:, ch], d))
-        a = sgat.int_gemm(c, vq[:, ch].T)
+        kv = slice((h // group) * d, (h // group + 1) * d)
+        c, l = p_codes(scores(Q[:, ch], K[:, kv], d))
+        a = sgat.int_gemm(c, vq[:, kv].T)
         codes[h], ls[h], acc[h] = c, l, a
-        Z[:, ch] = a.astype(F64) / (255.0 * l[:, None]) * t[ch].astype(F64)[None, :]
+        Z[:, ch] = a.astype(F64) / (255.0 * l[:, None]) * t[kv].astype(F64)[None, :]
     return Z, codes, ls, vq, t, acc
 
 
-def attention_tac(Q, K, V, M, dvec, H, d):
+def attention_tac(Q, K, V, M, dvec, H, d, Hkv=None):
     """TAC of the quantised attention output: Z_hat M_h^T + 1 d_h^T per head
     (Eq. 17 with one block per head). Returns (Z_tac float64 [L][H d],
     Z_hat)."""
-    Z = quantised_attention(Q, K, V, H, d)[0]
+    Z = quantised_attention(Q, K, V, H, d, Hkv)[0]
     return tac.tac_apply(Z, M, dvec, d), Z

@@ -277,6 +277,87 @@ def dream_block_linears(seed=0, batch=4, seq=2048, gen_len=256):
     return cases
 
 
+@dataclass
+class DreamBlockCase:
+    """One Dream-7B (Qwen2.5-7B shape) transformer block at a denoising step:
+    the input hidden states, the mask, the token positions, the block's
+    random-init bf16 weights and the synthetic stand-ins for its calibrated
+    parameters (per-linear SGAT transforms, TAC blocks per head)."""
+    X: np.ndarray            # [L, hidden] float32 holding bf16 values
+    mask: np.ndarray         # [L] uint8
+    pos: np.ndarray          # [L] int32, position within the sequence
+    batch: int
+    seq: int
+    hidden: int
+    ffn: int
+    heads: int
+    kv_heads: int
+    w_ln1: np.ndarray        # [hidden] float32 RMSNorm gains
+    w_ln2: np.ndarray
+    W_qkv: np.ndarray        # [(heads + 2 kv_heads) 128, hidden] bf16 values
+    b_qkv: np.ndarray        # float32 bias
+    W_o: np.ndarray          # [hidden, hidden]
+    W_gate: np.ndarray       # [ffn, hidden]
+    W_up: np.ndarray         # [ffn, hidden]
+    W_down: np.ndarray       # [hidden, ffn]
+    tac: TacParams           # one 128 x 128 block per query head
+    xf_qkv: SgatParams
+    xf_o: SgatParams
+    xf_gu: SgatParams
+    xf_down: SgatParams
+    rope_theta: float = 1e6
+    eps: float = 1e-6
+
+    @property
+    def L(self):
+        return self.X.shape[0]
+
+
+def dream_block(seed=0, batch=4, seq=2048, gen_len=256, hidden=3584, ffn=18944, heads=28, kv_heads=4):
+    """The Dream-7B block workload: 4 sequences of 2048 tokens in bfloat16,
+    the last 256 positions of each generated with 128 still masked
+    (seeded low-confidence remasking). Weights N(0, 0.02), RMSNorm gains
+    1 + N(0, 0.1), QKV bias N(0, 0.02), TAC blocks I + N(0, 0.01) per head.
+    The per-state smoothing of every linear is the synthetic calibration on
+    heavy-tailed activations of that linear's width (the block input itself
+    for the QKV projection); rows of 2048 tokens with the block's mask
+    pattern stand in for the calibration set."""
+    rng = np.random.default_rng(seed)
+    L = batch * seq
+    mask = np.concatenate([remask_schedule(rng, seq, gen_len, gen_len // 2) for _ in range(batch)])
+    pos = np.tile(np.arange(seq, dtype=np.int32), batch)
+    X = heavy_tail_activations(rng, L, hidden, dtype="bf16")
+    nqkv = (heads + 2 * kv_heads) * 128
+    g = lambda n, k: gaussian_weight(rng, n, k, dtype="bf16")
+    W_qkv, W_o, W_gate, W_up, W_down = g(nqkv, hidden), g(hidden, hidden), g(ffn, hidden), g(ffn, hidden), g(hidden, ffn)
+    b_qkv = rng.normal(0, 0.02, nqkv).astype(np.float32)
+    w_ln1 = (1.0 + rng.normal(0, 0.1, hidden)).astype(np.float32)
+    w_ln2 = (1.0 + rng.normal(0, 0.1, hidden)).astype(np.float32)
+    tac = make_tac(rng, hidden, 128)
+    calib_mask = mask[:seq]
+    calib = lambda K: make_sgat(heavy_tail_activations(rng, seq, K, dtype="bf16"), calib_mask)
+    return DreamBlockCase(X=X, mask=mask, pos=pos, batch=batch, seq=seq, hidden=hidden, ffn=ffn, heads=heads,
+                          kv_heads=kv_heads, w_ln1=w_ln1, w_ln2=w_ln2, W_qkv=W_qkv, b_qkv=b_qkv, W_o=W_o,
+                          W_gate=W_gate, W_up=W_up, W_down=W_down, tac=tac, xf_qkv=make_sgat(X, mask),
+                          xf_o=calib(hidden), xf_gu=calib(hidden), xf_down=calib(ffn))
+
+
+def basis_calibration_set(seed, d, n_samples=16, tokens=64, N=None, mask_p=0.5):
+    """Synthetic calibration set for the dense basis (App. B): n_samples
+    activation matrices of `tokens` tokens each (one per denoising step,
+    N(0, 1) with 0.5% Student-t(3) channels, float32), each with its own
+    Bernoulli(mask_p) mask, and a weight N(0, 0.02) [N][d] (N = d by
+    default). Returns (samples [(X, mask)], W)."""
+    rng = np.random.default_rng(seed)
+    samples = []
+    for _ in range(n_samples):
+        mask = (rng.random(tokens) < mask_p).astype(np.uint8)
+        X = heavy_tail_activations(rng, tokens, d, dtype="f16").astype(np.float32)
+        samples.append((X, mask))
+    W = gaussian_weight(rng, N or d, d).astype(np.float32)
+    return samples, W
+
+
 def random_linear(seed, L, K, N, dtype="f16", gates_on=True, tac_g=None, bias=False,
                   mask_p=0.5, hb=None):
     """Small random case for shape sweeps (ragged L, several tiles)."""

@@ -519,6 +519,28 @@ def test_attention_uniform_and_error_bound():
         assert np.all(np.abs(Z[:, ch] - exact) <= bound + 1e-12)
 
 
+def test_attention_gqa_equals_mha_on_repeated_heads():
+    """Grouped-query attention with H query heads over Hkv key/value heads
+    equals multi-head attention whose K and V repeat every key/value head
+    H / Hkv times (query head h reads key/value head h // (H / Hkv)): the
+    repeated channels carry identical columns, so their per-channel V codes
+    and scales are identical too. Swapping the group order (a plausible
+    indexing slip, h % Hkv) gives a different result."""
+    from oracle import attention as oatt
+    rng = np.random.default_rng(17)
+    L, H, Hkv, d = 24, 6, 2, 8
+    Q = rng.normal(0, 1, (L, H * d)).astype(np.float32)
+    K, V = (rng.normal(0, 1, (L, Hkv * d)).astype(np.float32) for _ in range(2))
+    rep = np.concatenate([np.arange(k * d, (k + 1) * d) for k in np.repeat(np.arange(Hkv), H // Hkv)])
+    Zg, cg, lg, vqg, tg, ag = oatt.quantised_attention(Q, K, V, H, d, Hkv)
+    Zm, cm, lm, vqm, tm, am = oatt.quantised_attention(Q, K[:, rep], V[:, rep], H, d)
+    assert np.array_equal(cg, cm) and np.array_equal(ag, am) and np.array_equal(lg, lm)
+    assert np.array_equal(Zg, Zm) and np.array_equal(tg[rep], tm) and np.array_equal(vqg[:, rep], vqm)
+    wrong = np.concatenate([np.arange(k * d, (k + 1) * d) for k in np.tile(np.arange(Hkv), H // Hkv)])
+    Zw = oatt.quantised_attention(Q, K[:, wrong], V[:, wrong], H, d)[0]
+    assert not np.allclose(Zg, Zw)
+
+
 def test_attention_tac_identity():
     """TAC with M = I and d = 0 returns Z_hat unchanged (P6 on this path)."""
     from oracle import attention as oatt
@@ -688,3 +710,170 @@ def test_dense_basis_cancellation_16bit():
     qt, st, _ = sgat.prepare_weight_dense(W, None, P.T.copy(), bits=16)
     Yt = sgat.dequant(sgat.int_gemm(codes, qt), s_a, st)
     assert np.linalg.norm(Yt - ref) / np.linalg.norm(ref) > 0.5
+
+
+# ---------------------------------------------------------------------------
+# Block glue (RMSNorm, rotary embedding, SwiGLU): standard definitions
+# ---------------------------------------------------------------------------
+
+def test_rmsnorm_worked_example_and_invariants():
+    """h = (3, 4): mean square 12.5, so y = h / sqrt(12.5) * w (by hand:
+    (0.848528..., 1.131370...) for w = 1). A constant row c gives w * c /
+    |c| up to eps; scaling a row does not change its normalised values
+    (eps = 0); the gain multiplies per column (a transposed gain fails)."""
+    from oracle import glue
+    y = glue.rmsnorm([[3.0, 4.0]], [1.0, 1.0], 0.0)
+    assert np.allclose(y, [[3 / math.sqrt(12.5), 4 / math.sqrt(12.5)]], rtol=1e-15)
+    assert abs(y[0, 0] - 0.8485281374238570) < 1e-15 and abs(y[0, 1] - 1.1313708498984760) < 1e-15
+    w = np.array([0.5, 2.0, -1.0, 3.0])
+    assert np.allclose(glue.rmsnorm(np.full((1, 4), -2.5), w, 1e-12), -w[None, :], atol=1e-12)
+    rng = np.random.default_rng(3)
+    h = rng.normal(0, 1, (5, 16))
+    w = rng.normal(1, 0.1, 16)
+    assert np.allclose(glue.rmsnorm(7.0 * h, w, 0.0), glue.rmsnorm(h, w, 0.0), rtol=1e-13)
+    y = glue.rmsnorm(h, w, 0.0)
+    assert np.allclose(np.mean((y / w[None, :]) ** 2, axis=1), 1.0, rtol=1e-13)
+
+
+def test_rope_identity_rotation_and_composition():
+    """Position 0 is the identity; each rotated pair keeps its norm; two
+    rotations compose (rotating by p1 then p2 equals rotating by p1 + p2);
+    the first frequency is 1, so pair 0 turns by pos radians (worked by hand
+    at pos = 1: (1, 0) -> (cos 1, sin 1)); columns past the rotated heads
+    are untouched."""
+    from oracle import glue
+    rng = np.random.default_rng(4)
+    L, heads, d = 6, 3, 128
+    x = rng.normal(0, 1, (L, heads * d + 64))
+    assert np.array_equal(glue.rope(x, np.zeros(L), heads, 1e6), x)
+    pos = rng.integers(0, 2048, L)
+    y = glue.rope(x, pos, heads, 1e6)
+    for h in range(heads):
+        a, b = x[:, h * d:h * d + 64], x[:, h * d + 64:(h + 1) * d]
+        ya, yb = y[:, h * d:h * d + 64], y[:, h * d + 64:(h + 1) * d]
+        assert np.allclose(a * a + b * b, ya * ya + yb * yb, rtol=1e-12)
+    p1, p2 = rng.integers(0, 1000, L), rng.integers(0, 1000, L)
+    assert np.allclose(glue.rope(glue.rope(x, p1, heads, 1e4), p2, heads, 1e4),
+                       glue.rope(x, p1 + p2, heads, 1e4), atol=1e-9)
+    assert np.array_equal(y[:, heads * d:], x[:, heads * d:])
+    e = np.zeros((1, d))
+    e[0, 0] = 1.0
+    r = glue.rope(e, [1], 1, 1e6)
+    assert abs(r[0, 0] - math.cos(1.0)) < 1e-15 and abs(r[0, 64] - math.sin(1.0)) < 1e-15
+    assert glue.rope_frequencies(1e6)[0] == 1.0
+    assert abs(glue.rope_frequencies(1e6)[32] - 1e6 ** -0.5) < 1e-18
+
+
+def test_swiglu_values():
+    """silu(0) = 0, silu(x) -> x for large x, silu(-x) = silu(x) - x."""
+    from oracle import glue
+    x = np.array([0.0, 30.0, -2.0, 1.5])
+    s = glue.swiglu(x, np.ones(4))
+    assert s[0] == 0.0 and abs(s[1] - 30.0) < 1e-11
+    assert abs(glue.swiglu([2.0], [1.0])[0] - glue.swiglu([-2.0], [1.0])[0] - 2.0) < 1e-15
+    assert abs(s[3] - 1.5 / (1 + math.exp(-1.5))) < 1e-15
+
+
+# ---------------------------------------------------------------------------
+# Calibration of the dense orthogonal basis (App. B, Eq. 15)
+# ---------------------------------------------------------------------------
+
+def test_cayley_map_is_orthogonal():
+    """C(0) = I; C(A) is orthogonal with determinant +1 for any A; a
+    transposed solve (C = (I + S)(I - S)^-1 computed wrongly as (I + S)^-1
+    (I - S)) would give C(A)^T instead, so C(A) is checked against the
+    explicit formula on a worked 2 x 2 case: S = [[0, -t], [t, 0]] gives the
+    rotation by 2 atan(t)."""
+    import torch
+    from oracle import calibration as oc
+    assert torch.equal(oc.cayley(torch.zeros(5, 5, dtype=torch.float64)), torch.eye(5, dtype=torch.float64))
+    A = torch.as_tensor(np.random.default_rng(2).normal(0, 1, (7, 7)))
+    C = oc.cayley(A).numpy()
+    assert np.abs(C.T @ C - np.eye(7)).max() < 1e-13 and abs(np.linalg.det(C) - 1.0) < 1e-12
+    t = 0.3
+    C2 = oc.cayley(torch.tensor([[0.0, 0.0], [t, 0.0]], dtype=torch.float64)).numpy()   # S = [[0, -t], [t, 0]]
+    th = 2 * math.atan(t)
+    assert np.allclose(C2, [[math.cos(th), -math.sin(th)], [math.sin(th), math.cos(th)]], atol=1e-15)
+
+
+def test_state_objective_brute_force():
+    """Eq. 15 against explicit numpy loops on a tiny case: per state, the
+    gated transformed rows quantised per row, the weight quantised per
+    output channel of P^T W^T, the squared Frobenius error summed."""
+    from oracle import calibration as oc
+    rng = np.random.default_rng(8)
+    d, N = 8, 5
+    d_sh, d_m, d_u = 4, 2, 2
+    P = oc.orthogonal_init(d, 3)
+    W = rng.normal(0, 1, (N, d))
+    samples = [(rng.normal(0, 1, (6, d)), np.array([1, 0, 1, 1, 0, 0])), (rng.normal(0, 1, (3, d)), np.array([0, 0, 0]))]
+    g_m, g_u = oc.gates(d, d_sh, d_m, d_u)
+
+    def q_rows(v, bits):
+        qmax = 2 ** (bits - 1) - 1
+        out = np.zeros_like(v)
+        for i in range(v.shape[0]):
+            a = np.abs(v[i]).max()
+            if a > 0:
+                s = a / qmax
+                out[i] = np.array([round(x / s) for x in v[i]]) * s      # half to even
+        return out
+    Wt = q_rows(W @ P, 4)
+    want = 0.0
+    for X, mask in samples:
+        for state, g in ((1, g_m), (0, g_u)):
+            Xs = X[mask == state]
+            if len(Xs):
+                want += float(((Xs @ W.T - q_rows((Xs @ P) * g[None, :], 4) @ Wt.T) ** 2).sum())
+    got = float(oc.state_objective(P, samples, W, d_sh, d_m, d_u))
+    assert abs(got - want) <= 1e-10 * want
+
+
+def test_calibration_recovers_planted_subspaces():
+    """Activations built to satisfy Eq. 25 for a planted basis P*: masked
+    tokens live in span(U*_sh, U*_m), unmasked ones in span(U*_sh, U*_u).
+    With 16-bit quantisers and an orthogonal W the objective is the energy
+    of Delta_s of Eq. 28, || X^s P G_s^perp P^T W^T ||^2 = || X^s P G_s^perp ||^2
+    (the leakage), up to rounding; so calibration from a random orthogonal
+    start must drive the leakage toward zero: below 2% of its start, with P
+    orthogonal to round-off after every step and the objective below its
+    start after every epoch. (With a general W the objective can also fall
+    by hiding the leakage in W's small singular directions.)"""
+    from oracle import calibration as oc
+    rng = np.random.default_rng(11)
+    d, d_sh, d_m, d_u = 16, 12, 2, 2
+    Ps = oc.orthogonal_init(d, 99)
+    Um, Uu, Ush = Ps[:, d_sh:d_sh + d_m], Ps[:, d_sh + d_m:], Ps[:, :d_sh]
+    samples = []
+    for _ in range(8):
+        mask = (rng.random(24) < 0.5).astype(np.uint8)
+        X = np.empty((24, d))
+        for i in range(24):
+            B = np.concatenate([Ush, Um if mask[i] else Uu], axis=1)
+            X[i] = B @ rng.normal(0, 1, d_sh + d_m)
+        samples.append((X, mask))
+    W = 2.0 * oc.orthogonal_init(d, 7)
+    P, hist = oc.calibrate_basis(samples, W, d_sh, d_m, d_u, bits_a=16, bits_w=16, lr=2e-2, epochs=80, seed=5)
+    assert max(hist["orth_err"]) < 1e-12
+    assert oc.leakage(Ps, samples, d_sh, d_m, d_u) < 1e-20            # the planted basis has none
+    assert hist["leakage"][-1] < 0.02 * hist["leakage"][0]
+    assert all(o <= hist["objective"][0] for o in hist["objective"][1:])
+
+
+def test_calibration_paper_settings_reduce_objective():
+    """App. B's settings (AdamW lr 1e-3, batch 4, 15 epochs, 4-bit codes) on
+    the synthetic calibration set: P stays orthogonal to round-off after
+    every step, starts at the orthogonalised Gaussian (the objective's first
+    entry is the objective of that start), and the objective after every
+    epoch is below its value at the start."""
+    from oracle import calibration as oc
+    from paper_2606_04945_gb300 import inputs
+    d = 64
+    samples, W = inputs.basis_calibration_set(4, d, n_samples=8, tokens=32)
+    d_m = d_u = d // 32
+    d_sh = d - 2 * d_m
+    P, hist = oc.calibrate_basis(samples, W, d_sh, d_m, d_u, seed=1)
+    assert len(hist["orth_err"]) == 15 * 2 and max(hist["orth_err"]) < 1e-12
+    start = float(oc.state_objective(oc.orthogonal_init(d, 1), samples, W, d_sh, d_m, d_u))
+    assert abs(hist["objective"][0] - start) <= 1e-12 * start
+    assert all(o < hist["objective"][0] for o in hist["objective"][1:])
