@@ -50,16 +50,18 @@ def parse():
     p.add_argument("--cpu-sample-tokens", type=int, default=1024)
     p.add_argument("--ref-sample-tokens", type=int, default=128)
     p.add_argument("--skip-cpu-baseline", action="store_true")
+    p.add_argument("--skip-stack", action="store_true", help="leave out the short denoising-stack run")
     p.add_argument("--workload", default="attention_step",
                    choices=["attention_step", "denoise_stack", "tac_calibration", "attention_pv_tac", "w8a8_linear",
-                            "asym_linear", "dense_linear"],
+                            "asym_linear", "dense_linear", "dream_block"],
                    help="attention_step: the LLaDA attention projections (default); denoise_stack: the "
                         "64-step 4-layer LLaDA-shaped stack (per-step tokens/s, latency, drift vs fp16); "
                         "tac_calibration: App. C's closed-form TAC calibration on the GPU vs the oracle; "
                         "attention_pv_tac: the quantised softmax-value product with the TAC epilogue; "
                         "w8a8_linear: the attention projections at 8 bits (Tab. 5); "
                         "asym_linear: the attention projections with asymmetric A4 activations (Eq. 2-4); "
-                        "dense_linear: the attention projections with a dense orthogonal basis (App. B)")
+                        "dense_linear: the attention projections with a dense orthogonal basis (App. B); "
+                        "dream_block: the full Dream-7B-shaped block (GQA 28/4 heads, bf16, 4 x 2048 tokens)")
     return p.parse_args()
 
 
@@ -241,6 +243,83 @@ def time_kernel(fn, flush, reps, torch):
     return statistics.mean(ts)
 
 
+def probe_peaks(abi, torch, iters=2048, reps=3):
+    """Tensor-core rates of the instruction kinds (starq_probe_mma), each the
+    best of `reps` launches timed with CUDA events after one warm-up launch:
+    TFLOP/s (2 multiply-adds per MAC), multiply-adds per clock and SM from
+    the CTAs' own cycle counts, and the exactness check's mismatch count."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    cycles = torch.zeros(4 * sms, dtype=torch.int64, device="cuda")
+    errors = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = {}
+    s = torch.cuda.current_stream()
+    for kind, name in abi.PROBE_KINDS.items():
+        errors.zero_()
+        abi.probe_mma(kind, iters, cycles, errors)
+        best = None
+        for _ in range(reps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            ctas, macs = abi.probe_mma(kind, iters, cycles, errors)
+            e1.record(s)
+            e1.synchronize()
+            ms = e0.elapsed_time(e1)
+            best = ms if best is None else min(best, ms)
+        cyc = cycles[:ctas].double()
+        # macs_per_cta is per CTA (one SM; a CTA pair's MMA counts half per CTA)
+        ctas_per_sm = ctas / sms if kind >= 3 else 1
+        out[name] = {"tflops": round(2 * macs * ctas / (best * 1e-3) / 1e12, 1), "ms": round(best, 5),
+                     "mac_per_clk_sm": round(macs * ctas_per_sm / float(cyc.max()), 1),
+                     "errors": int(errors.item()), "ctas": ctas}
+    abi.check_status()
+    return out
+
+
+def hbm_passes_large(abi, o, flush, torch, L=8192):
+    """The HBM-bound passes at L = 8192 tokens (the Dream block's token
+    count), each timed back to back over three rotating input sets larger
+    than L2 together. Bytes per token follow the algorithmic counts: the
+    quantiser reads 2K (16-bit X) and writes K/2 + 4 (packed codes, scale);
+    with the E4M3 operand it writes K more; TAC reads and writes 2C and reads
+    its parameters once."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(8192)
+    out = {}
+
+    def quant_entry(name, K, hb, dt, a_m, a_u, e4m3):
+        Xs = [torch.randn(L, K, device="cuda", dtype=torch.float32, generator=g).to(dt) for _ in range(3)]
+        mask = (torch.rand(L, device="cuda", generator=g) < 0.25).to(torch.uint8)
+        Xq = torch.empty(L, K // 2, dtype=torch.uint8, device="cuda")
+        Xe = torch.empty(L, K, dtype=torch.uint8, device="cuda") if e4m3 else None
+        s_a = torch.empty(L, dtype=torch.float32, device="cuda")
+        d_m = d_u = K // 32
+        ms = time_stream([lambda i=i: abi.sgat_quantize_act(Xs[i], mask, a_m, a_u, hb, K - d_m - d_u, d_m, d_u, Xq,
+                                                            s_a, Xe=Xe) for i in range(3)], flush, torch, rounds=4)
+        alg = L * (2 * K + K // 2 + 4)
+        moved = alg + (L * K if e4m3 else 0)
+        out[name] = {"ms": round(ms, 5), "tokens": L, "K": K, "hb": hb, "dtype": str(dt).replace("torch.", ""),
+                     "bytes_algorithmic": alg, "bytes_moved": moved,
+                     "gbs": round(alg / ms / 1e6, 1), "gbs_moved": round(moved / ms / 1e6, 1)}
+        del Xs
+
+    K = o.K
+    quant_entry(f"sgat_quantize_act_{L}x{K}_f16", K, o.hb, torch.float16, o.a_m, o.a_u, False)
+    quant_entry(f"sgat_quantize_act_{L}x{K}_f16_e4m3", K, o.hb, torch.float16, o.a_m, o.a_u, True)
+    Kd = 3584
+    a_d = [torch.exp(0.3 * torch.randn(Kd, device="cuda", generator=g)) for _ in range(2)]
+    quant_entry(f"sgat_quantize_act_{L}x{Kd}_bf16_hb512", Kd, 512, torch.bfloat16, a_d[0], a_d[1], False)
+    Zs = [torch.randn(L, K, device="cuda", dtype=torch.float32, generator=g).to(torch.float16) for _ in range(3)]
+    Zo = torch.empty(L, K, dtype=torch.float16, device="cuda")
+    ms = time_stream([lambda i=i: abi.tac_apply(Zs[i], o.tac_M, o.tac_d, o.tac_g, Zo, Mp=o.tac_Mp) for i in range(3)],
+                     flush, torch, rounds=4)
+    alg = L * K * 4 + K * o.tac_g * 4 + K * 4
+    out[f"tac_apply_{L}x{K}_g{o.tac_g}"] = {"ms": round(ms, 5), "tokens": L, "C": K, "g": o.tac_g,
+                                           "bytes_algorithmic": alg, "gbs": round(alg / ms / 1e6, 1)}
+    del Zs
+    return out
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -322,6 +401,11 @@ def run_ours(args):
                             for i in range(8)], flush, torch, rounds=3)
     abi.check_status()
     del Xr, Zr, Zf, Wr_q, Wr_o, Xer
+    large = hbm_passes_large(abi, o, flush, torch)
+    abi.check_status()
+    probes = probe_peaks(abi, torch)
+    denoise = stack_steps(torch) if not args.skip_stack else None
+    abi.check_status()
 
     # the unquantised baseline: the same two projections as 16-bit GEMMs
     # (fp16 weights and activations, float32 accumulation) -- context for
@@ -436,7 +520,9 @@ def run_ours(args):
     gemm_ops = q.int_ops() + o.int_ops()
     gemm_ms = s_gemm_qkv + s_gemm_o
     achieved = gemm_ops / (gemm_ms * 1e-3) / 1e12
-    peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]) * FP8_PER_BF16
+    peak_bf16x2 = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]) * FP8_PER_BF16
+    pair_probe = probes[abi.PROBE_KINDS[1]]
+    peak = pair_probe["tflops"] if pair_probe["errors"] == 0 else peak_bf16x2
     hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
     quant_x_bytes = L * K * 2 + L * K // 2 + L * K + 4 * L     # X in; packed + E4M3 codes, scales out
     quant_z_bytes = L * K * 2 + L * K // 2 + L * K + 4 * L             # the TAC output (16-bit) in
@@ -463,8 +549,13 @@ def run_ours(args):
             "bound": "tensor", "kernel": "w4a4_gemm_tma_pair_kernel (QKV + O launches)",
             "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
             "frac": round(achieved / peak, 4), "traffic": traffic,
-            "peak_source": f"{peak_src} bf16 dense burst x {FP8_PER_BF16} (fp8 kind::f8f6f4 path; "
-                           f"sm_103a has no integer tcgen05 MMA)",
+            "peak_source": "starq_probe_mma kind 1 (tcgen05 kind::f8f6f4 cta_group::2 back-to-back MMAs on "
+                           "on-chip operands, this run, best of 3; csrc/probe.cu): the instruction the GEMM "
+                           "issues; sm_103a has no integer tcgen05 MMA",
+            "peak_bf16x2": round(peak_bf16x2, 1), "frac_bf16x2": round(achieved / peak_bf16x2, 4),
+            "peak_bf16x2_source": f"{peak_src} bf16 dense burst x {FP8_PER_BF16} (nominal fp8 / bf16 ratio)",
+            "per_launch_frac": {"qkv": round(q.int_ops() / (s_gemm_qkv * 1e-3) / 1e12 / peak, 4),
+                                "o": round(o.int_ops() / (s_gemm_o * 1e-3) / 1e12 / peak, 4)},
             "algorithmic": f"{gemm_ops} int ops per step over 2 launches; "
                            f"{sum(gemm_bytes)} algorithmic bytes per step",
             "stream_ms": {"qkv": round(s_gemm_qkv, 5), "o": round(s_gemm_o, 5)},
@@ -474,6 +565,7 @@ def run_ours(args):
         },
         "roofline_hbm_kernels": {
             "peak_gbs": hbm, "peak_source": peak_src,
+            "large": {k: dict(v, frac=round(v["gbs"] / hbm, 4)) for k, v in large.items()},
             "timing": "ms: back-to-back launches over rotating inputs larger than L2; launch_ms: one "
                       "launch after an L2 flush (launch latency included)",
             "sgat_quantize_act_f16": {"ms": round(s_quant_x, 5), "launch_ms": round(t_quant_x, 5), "bytes": quant_x_bytes,
@@ -486,6 +578,8 @@ def run_ours(args):
                                       "gbs": round(quant_z_bytes / s_quant_z / 1e6, 1),
                                       "frac": round(quant_z_bytes / s_quant_z / 1e6 / hbm, 4)},
         },
+        "tensor_probes": probes,
+        "denoise_step": denoise,
         "fp16_baseline": {
             "kernel": "fp16_gemm_ref (tcgen05 kind::f16 CTA pairs, fp16 in/out, fp32 accumulate)",
             "stream_ms": {"qkv": round(s_f16_qkv, 5), "o": round(s_f16_o, 5)},
@@ -636,6 +730,45 @@ def run_reference(args):
     }
 
 
+def stack_steps(torch, steps=8):
+    """A short run of the 64-step denoising trajectory of the 4-layer
+    LLaDA-8B-shaped stack (quantised path: SGAT W4A4 linears, quantised
+    attention with TAC, glue kernels; each step one CUDA graph replay) and
+    of the same stack on 16-bit GEMMs with unquantised attention: the first
+    `steps` steps of each, device-timed per step."""
+    from paper_2606_04945_gb300.stack import DenoiseStack, StackConfig
+    cfg = StackConfig()
+    st = DenoiseStack(cfg)
+    st.calibrate()
+    s = torch.cuda.current_stream()
+    out = {}
+    for q in (True, False):
+        g, tok_s, mask_s, _ = st.capture(q)
+        for step in range(2):                        # warm-up replays
+            st.set_state(step, tok_s, mask_s)
+            g.replay()
+        evs = []
+        for step in range(steps):
+            st.set_state(step, tok_s, mask_s)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            g.replay()
+            e1.record(s)
+            evs.append((e0, e1))
+        torch.cuda.synchronize()
+        out[q] = statistics.mean(a.elapsed_time(b) for a, b in evs)
+        del g
+    ms, ms16 = out[True], out[False]
+    res = {"workload": "llada8b_4layer_denoise (hidden 4096, FFN 12288, 32 heads, 1024 tokens, 256 generated)",
+           "steps_timed": steps, "ms_per_step": round(ms, 4), "tokens_per_s": round(cfg.seq / (ms * 1e-3), 1),
+           "fp16_stack_ms_per_step": round(ms16, 4), "speedup_vs_fp16_stack": round(ms16 / ms, 3),
+           "note": "first steps of the 64-step trajectory, one CUDA graph per step; the fp16 stack runs "
+                   "fp16_gemm_ref linears and torch SDPA attention"}
+    del st
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_stack(args):
     """The 64-step denoising trajectory of the 4-layer LLaDA-8B-shaped stack
     (every linear SGAT W4A4, TAC on O, glue ops in torch), timed per step,
@@ -709,6 +842,75 @@ def run_stack(args):
         "fp16_stack": {"ms_per_step": round(statistics.mean(tf), 4),
                        "speedup": round(statistics.mean(tf) / ms, 3)},
         "drift_vs_fp16": {"first": round(drift[0], 4), "max": round(max(drift), 4), "last": round(drift[-1], 4)},
+    }
+
+
+def run_dream_block(args):
+    """The full Dream-7B-shaped transformer block (Qwen2.5-7B shape, bf16,
+    4 sequences x 2048 tokens, 28 query / 4 key-value heads, FFN 18944):
+    RMSNorm, SGAT W4A4 QKV with bias, RoPE, the quantised GQA attention with
+    TAC, SGAT W4A4 O, residual + RMSNorm, SGAT W4A4 gate/up with SwiGLU,
+    down, residual; one CUDA graph per pass, timed per pass (the block's
+    operands are several times larger than L2)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi, inputs
+    from paper_2606_04945_gb300.dream import DreamBlock
+    torch.cuda.set_device(0)
+    case = inputs.dream_block(seed=0)
+    blk = DreamBlock(case)
+    for _ in range(max(args.warmup, 3)):
+        blk.forward()
+    abi.check_status()
+    blk.capture()
+    for _ in range(2):
+        blk.replay()
+    s = torch.cuda.current_stream()
+    evs = []
+    for _ in range(args.steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        blk.replay()
+        e1.record(s)
+        evs.append((e0, e1))
+    torch.cuda.synchronize()
+    abi.check_status()
+    ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+    # one eager pass with events around the linears and the attention
+    parts = {}
+    b = blk.buf
+
+    def timed(name, fn):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(s)
+        fn()
+        e1.record(s)
+        parts[name] = (e0, e1)
+    timed("qkv", lambda: blk.qkv.run(b["a"], blk.mask, b["qkv"]))
+    timed("attention", lambda: blk.attention(b["qkv"], b["z"]))
+    timed("o", lambda: blk.o.run(b["z"], blk.mask, b["o"]))
+    timed("gate_up_swiglu", lambda: blk.gu.run(b["a2"], blk.mask, b["g"]))
+    timed("down", lambda: blk.down.run(b["g"], blk.mask, b["d"]))
+    torch.cuda.synchronize()
+    part_ms = {k: round(a.elapsed_time(e), 4) for k, (a, e) in parts.items()}
+    lin_ms = sum(v for k, v in part_ms.items() if k != "attention")
+    ops = blk.int_ops()
+    L = case.L
+    return {
+        "metric": "Dream-7B-shaped block tokens/s (W4A4 SGAT linears, quantised GQA attention with TAC)",
+        "value": round(L / (ms * 1e-3), 1), "unit": "tokens/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int4 (W4A4 codes, SGAT) linears; 8-bit P / 4-bit V attention with TAC; bf16 I/O and glue",
+        "data": "synthetic (seeded; random-init Dream-7B-shaped weights)",
+        "config": {"workload": "dream7b_block", "batch": case.batch, "seq": case.seq, "tokens": L,
+                   "hidden": case.hidden, "ffn": case.ffn, "heads": case.heads, "kv_heads": case.kv_heads,
+                   "cuda_graph": True, "l2": "operands several times larger than L2"},
+        "linears": {"int_ops_per_pass": ops, "ms": round(lin_ms, 4), "tops": round(ops / (lin_ms * 1e-3) / 1e12, 1),
+                    "tops_whole_block": round(ops / (ms * 1e-3) / 1e12, 1)},
+        "parts_ms_eager": part_ms,
+        "gpu_launches": args.steps * blk.kernel_launches(),
     }
 
 
@@ -1131,6 +1333,13 @@ def main():
         out = run_w8a8(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
                                                           "the oracle arm times the attention-step workload"}
         print(json.dumps(out), flush=True)
+        return
+    if args.workload == "dream_block":
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable": "the oracle arm times the attention-step workload"}))
+            return
+        out = run_dream_block(args)
+        print(json.dumps(out))
         return
     if args.workload == "denoise_stack":
         out = run_stack(args) if args.impl == "ours" else {"impl": "reference", "unavailable":

@@ -91,6 +91,37 @@ int starq_check_status(void* stream);
 int starq_selftest_wait_timeout(unsigned limit_us, void* stream);
 
 /*
+ * starq_probe_mma -- rate probe of the tensor-core instruction kinds, the
+ * measured denominators of the GEMM rooflines (the paper has no
+ * counterpart; sm_103a has no integer tcgen05 MMA, so the W4A4 path runs on
+ * the FP8 kind and its peak has to be measured, not looked up).
+ *
+ * Every CTA issues `iters` rounds of back-to-back MMAs on operands resident
+ * on chip, waits (bounded) for them, writes its cycle count to cycles[cta]
+ * and adds the number of accumulators that differ from the exact expected
+ * value to *errors. The caller times the launch with events on `stream`
+ * and computes 2 * macs_per_cta * ctas / time.
+ *   kind 0  tcgen05.mma cta_group::1 kind::f8f6f4, E4M3 x E4M3 -> F32,
+ *           M 128 N 256 K 32 per instruction, one CTA per SM; operands all
+ *           E4M3(7), so every accumulator must equal 49 * 128 * iters
+ *           exactly (integer sums below 2^24 through the FP8 path).
+ *   kind 1  the same on CTA pairs (cta_group::2, M 256 over the pair), the
+ *           form w4a4_gemm issues.
+ *   kind 2  tcgen05.mma cta_group::1 kind::f16, bf16 operands 1.0,
+ *           M 128 N 256 K 16; accumulators 64 * iters.
+ *   kind 3  mma.sync m16n8k32 s8.s8.s32 (warp-level integer MMA), four CTAs
+ *           per SM of four warps, eight independent accumulator chains per
+ *           warp; accumulators 32 * iters.
+ *   kind 4  mma.sync m16n8k64 s4.s4.s32, likewise; accumulators 64 * iters.
+ *   iters   1 .. 2048.
+ *   cycles  device u64 [4 * SM count] (room for every kind), out.
+ *   errors  device int32, zeroed by the caller; mismatch count added.
+ *   ctas, macs_per_cta  host outputs: CTAs launched, multiply-adds per CTA.
+ */
+int starq_probe_mma(int kind, int iters, unsigned long long* cycles, int* errors, int* ctas,
+                    double* macs_per_cta, void* stream);
+
+/*
  * sgat_quantize_act -- state-guided activation transform + per-token A4
  * quantisation (Sec. 3.2 Eq. 7-11 and Eq. 13's Q_a; Sec. 3.1 Eq. 2-3).
  *
@@ -388,7 +419,8 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  *     (row sums l), dbg_acc NULL or int32 [H][L][128] (the exact sums): for
  *     tests.
  *   workspace: attention_pv_tac_workspace_size(L, H) bytes, 256-byte aligned
- *     (V codes transposed and the channel scales).
+ *     (V codes transposed and the channel scales; the size takes the number
+ *     of key/value heads, which is H here).
  * Shapes: head dimension 128, H >= 1, 128 <= L <= 8192 with L % 128 == 0,
  * ld >= 128 H with ld % 8 == 0; all pointers 16-byte aligned.
  * Kernels: a V quantiser (per-channel scales and transposed codes) and one
@@ -399,10 +431,30 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
  * asynchronous on `stream`; a wait that gives up inside the kernel is
  * reported by starq_check_status.
  */
-size_t attention_pv_tac_workspace_size(int L, int H);
+size_t attention_pv_tac_workspace_size(int L, int Hkv);
 int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L, int H, const void* Mp,
                      const float* d, void* Z, uint8_t* dbg_codes, float* dbg_l, int32_t* dbg_acc,
                      void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * attention_pv_tac_gqa -- attention_pv_tac with grouped-query attention and
+ * a choice of element type (the Dream-7B / Qwen2.5 block: 28 query heads
+ * over 4 key/value heads, bf16). Query head h reads key/value head
+ * h / (H / Hkv): K and V hold Hkv heads (columns 128 k .. 128 k + 127 of
+ * head k), Q and Z hold H heads. V is quantised per channel of the Hkv
+ * heads, so the query heads of a group share one set of V codes and scales.
+ *   dtype  STARQ_F16 or STARQ_BF16: the type of Q, K, V and Z. Q K^T runs in
+ *          that type; the P and V codes are integers (exact in fp16); the
+ *          TAC product runs on fp16 halves of Z_hat (scaled per head by an
+ *          exact power of two into fp16's range) against M's fp16 halves,
+ *          so Mp = tac_prepare(M, 128 H, 128, STARQ_F16) for either dtype.
+ *   workspace  attention_pv_tac_workspace_size(L, Hkv) bytes.
+ *   Other arguments, shapes and outputs as attention_pv_tac; H % Hkv == 0.
+ * attention_pv_tac is this call with Hkv = H and dtype = STARQ_F16.
+ */
+int attention_pv_tac_gqa(const void* Q, const void* K, const void* V, int ld, int L, int H, int Hkv, int dtype,
+                         const void* Mp, const float* d, void* Z, uint8_t* dbg_codes, float* dbg_l,
+                         int32_t* dbg_acc, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * tac_calibrate -- the closed-form TAC parameters (App. C, "Block-wise
@@ -540,6 +592,34 @@ int sgat_linear_noalloc(const void* X, int x_dtype, int L, int K, const uint8_t*
                         const float* tac_M, const float* tac_d, int tac_g, const void* tac_Mp,
                         const uint8_t* Wq, const uint8_t* We, const float* s_w, const float* bias,
                         int N, int bits, void* Y, int y_dtype, void* stream);
+
+/*
+ * Glue of the quantised transformer blocks (not part of the paper's method:
+ * Sec. 3 quantises the linears and the softmax-value product; the block
+ * runs these element-wise passes between them, on this GPU like the rest).
+ *
+ * glue_add_rmsnorm -- residual add and RMSNorm of rows of K values:
+ *   h = fl_T(X + R)                     (R = NULL: h = X)
+ *   Y = fl_T(fl32(h * inv) * w),  inv = 1 / sqrt(mean_k(h^2) + eps)
+ * with the sum of squares, mean and reciprocal square root in float32.
+ *   X, R, h_out, Y  [L][K] of element type dtype (F16 or BF16), 16-byte
+ *   aligned; R, h_out and Y may be NULL (h_out needs R; at least one of
+ *   h_out, Y). h_out may be X or R (in place).
+ *   w  [K] float32 gain (needed with Y).
+ * Shapes: L >= 0, 8 <= K <= 20480, K % 8 == 0.
+ *
+ * glue_rope -- rotary position embedding, in place, on the first `heads`
+ * heads of 128 channels of each row of QK [L][ld] (the query and key heads
+ * of a fused QKV output): for i < 64 the pair (x_i, x_{i+64}) of a head is
+ * rotated by the angle pos[token] * f_i, f_i = theta^(-2 i / 128) (float64,
+ * rounded to float32), as (x_i c - x_{i+64} s, x_{i+64} c + x_i s) in
+ * float32 with one rounding to dtype (the rotate-half form of the LLaMA and
+ * Qwen2 families). pos: int32 [L] device array; theta > 1 (1e6 for Qwen2.5).
+ * Shapes: L >= 0, heads >= 1, ld >= 128 heads.
+ */
+int glue_add_rmsnorm(const void* X, const void* R, int dtype, int L, int K, const float* w, float eps,
+                     void* h_out, void* Y, void* stream);
+int glue_rope(void* QK, int dtype, int L, int ld, int heads, const int32_t* pos, double theta, void* stream);
 
 #ifdef __cplusplus
 }

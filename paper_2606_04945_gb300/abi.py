@@ -26,7 +26,7 @@ EXPORTED = (
     "sgat_quantize_act_asym", "w4_zero_point_columns", "sgat_linear_asym_workspace_size", "sgat_linear_asym",
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
     "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
-    "starq_selftest_wait_timeout",
+    "starq_selftest_wait_timeout", "starq_probe_mma", "attention_pv_tac_gqa", "glue_add_rmsnorm", "glue_rope",
 )
 
 
@@ -46,6 +46,9 @@ def _load():
     lib.starq_last_error.restype = ctypes.c_char_p
     lib.starq_check_status.argtypes = [vp]
     lib.starq_selftest_wait_timeout.argtypes = [ctypes.c_uint, vp]
+    lib.glue_add_rmsnorm.argtypes = [vp, vp, i, i, i, f_p, ctypes.c_float, vp, vp, vp]
+    lib.glue_rope.argtypes = [vp, i, i, i, i, vp, ctypes.c_double, vp]
+    lib.starq_probe_mma.argtypes = [i, i, vp, vp, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double), vp]
     lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, i, u8p, f_p, u8p, f_p, vp]
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
@@ -85,6 +88,8 @@ def _load():
     lib.attention_pv_tac_workspace_size.argtypes = [i, i]
     lib.attention_pv_tac_workspace_size.restype = ctypes.c_size_t
     lib.attention_pv_tac.argtypes = [vp, vp, vp, i, i, i, vp, f_p, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+    lib.attention_pv_tac_gqa.argtypes = [vp, vp, vp, i, i, i, i, i, vp, f_p, vp, vp, vp, vp, vp, ctypes.c_size_t,
+                                         vp]
     lib.sgat_linear_noalloc.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, f_p, f_p, i, vp,
                                         u8p, u8p, f_p, f_p, i, i, vp, i, vp]
     return lib
@@ -127,6 +132,23 @@ def selftest_wait_timeout(limit_us, stream=None):
     arms, given up after limit_us); the next check_status raises
     StarqError(ERR_TIMEOUT)."""
     _check(lib.starq_selftest_wait_timeout(int(limit_us), _stream(stream)))
+
+
+PROBE_KINDS = {0: "tcgen05 kind::f8f6f4 cta_group::1 M128 N256 K32 (E4M3)",
+               1: "tcgen05 kind::f8f6f4 cta_group::2 M256 N256 K32 (E4M3, CTA pairs)",
+               2: "tcgen05 kind::f16 cta_group::1 M128 N256 K16 (bf16)",
+               3: "mma.sync m16n8k32 s8.s8.s32",
+               4: "mma.sync m16n8k64 s4.s4.s32"}
+
+
+def probe_mma(kind, iters, cycles, errors, stream=None):
+    """Launch the tensor-core rate probe; cycles (int64 [4 * SMs]) and errors
+    (int32 [1], zeroed) are device tensors. Returns (ctas, macs_per_cta)."""
+    ctas = ctypes.c_int(0)
+    macs = ctypes.c_double(0.0)
+    _check(lib.starq_probe_mma(int(kind), int(iters), _p(cycles), _p(errors), ctypes.byref(ctas),
+                               ctypes.byref(macs), _stream(stream)))
+    return ctas.value, macs.value
 
 
 def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, bits=4, Xe=None, v_dbg=None,
@@ -310,18 +332,27 @@ def tac_calibrate(Z_fp, Z_q, g, M, d, workspace=None, rho=3e-4, eps=1e-8, eta=0.
                              _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
-def attention_pv_tac(Q, K, V, H, Mp, d, Z, workspace=None, dbg_codes=None, dbg_l=None, dbg_acc=None, stream=None):
+def attention_pv_tac_workspace_size(L, Hkv):
+    return int(lib.attention_pv_tac_workspace_size(L, Hkv))
+
+
+def attention_pv_tac(Q, K, V, H, Mp, d, Z, workspace=None, dbg_codes=None, dbg_l=None, dbg_acc=None, Hkv=None,
+                     stream=None):
     """Quantised softmax-value product with TAC in its epilogue. Q, K, V are
-    fp16 [L][ld] views (e.g. column slices of the QKV output); Z [L][128 H]."""
+    fp16 or bf16 [L][ld] views (e.g. column slices of the QKV output) with H
+    query heads in Q and Hkv (default H) key/value heads in K and V;
+    Z [L][128 H] of the same type."""
     L = Q.shape[0]
     ld = Q.stride(0)
     assert K.stride(0) == ld and V.stride(0) == ld and Q.stride(1) == K.stride(1) == V.stride(1) == 1
+    assert Q.dtype == K.dtype == V.dtype == Z.dtype
+    Hkv = H if Hkv is None else Hkv
     _contig(Mp, d, Z, workspace, dbg_codes, dbg_l, dbg_acc)
     if workspace is None:
-        workspace = torch.empty(int(lib.attention_pv_tac_workspace_size(L, H)), dtype=torch.uint8, device=Q.device)
-    _check(lib.attention_pv_tac(_p(Q), _p(K), _p(V), ld, L, H, _p(Mp), _p(d), _p(Z), _p(dbg_codes), _p(dbg_l),
-                                _p(dbg_acc), _p(workspace), workspace.numel() * workspace.element_size(),
-                                _stream(stream)))
+        workspace = torch.empty(attention_pv_tac_workspace_size(L, Hkv), dtype=torch.uint8, device=Q.device)
+    _check(lib.attention_pv_tac_gqa(_p(Q), _p(K), _p(V), ld, L, H, Hkv, dtype_code(Q), _p(Mp), _p(d), _p(Z),
+                                    _p(dbg_codes), _p(dbg_l), _p(dbg_acc), _p(workspace),
+                                    workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def sgat_linear_workspace_size(L, K, with_tac, bits=4):
@@ -361,6 +392,22 @@ def sgat_linear_swiglu(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Wq, s_w, H, worksp
                                   d_u, _p(tac_M), _p(tac_d), tac_g, _p(tac_Mp), _p(Wq), _p(We), _p(s_w), _p(bias),
                                   N, bits, _p(H), dtype_code(H), _p(workspace),
                                   workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def add_rmsnorm(X, w, Y, R=None, h_out=None, eps=1e-6, stream=None):
+    """Y = RMSNorm(X + R) * w (R optional); h_out receives X + R."""
+    _contig(X, R, w, h_out, Y)
+    L, K = X.shape
+    _check(lib.glue_add_rmsnorm(_p(X), _p(R), dtype_code(X), L, K, _p(w), float(eps), _p(h_out), _p(Y),
+                                _stream(stream)))
+
+
+def rope(QK, heads, pos, theta, stream=None):
+    """Rotary embedding in place on the first `heads` 128-channel heads of
+    each row of QK (a [L][ld] view with unit column stride)."""
+    assert QK.stride(1) == 1
+    L = QK.shape[0]
+    _check(lib.glue_rope(_p(QK), dtype_code(QK), L, QK.stride(0), heads, _p(pos), float(theta), _stream(stream)))
 
 
 NOALLOC_SCRATCH_BYTES = 32 << 20

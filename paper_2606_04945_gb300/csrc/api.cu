@@ -166,6 +166,11 @@ int check_w8a8(const uint8_t* Xe, const float* s_a, const uint8_t* We, const flo
 
 int report_error(int code, const char* msg) { return fail(code, "%s", msg); }
 
+unsigned* device_status_word() {
+    int rc = STARQ_OK;
+    return status_ptr(&rc);
+}
+
 namespace {
 // Failure-detection self-test: one thread waits on an mbarrier that nothing
 // ever arrives on, through the same bounded wait as every pipeline wait of
@@ -245,6 +250,50 @@ int starq_selftest_wait_timeout(unsigned limit_us, void* stream) {
     selftest_wait_timeout_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(st, 1000ull * limit_us);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "starq_selftest_wait_timeout launch");
+    return STARQ_OK;
+}
+
+int glue_add_rmsnorm(const void* X, const void* R, int dtype, int L, int K, const float* w, float eps, void* h_out,
+                     void* Y, void* stream) {
+    if (dtype != STARQ_F16 && dtype != STARQ_BF16) return fail(STARQ_ERR_ARG, "glue_add_rmsnorm: dtype must be F16 or BF16");
+    if (L < 0 || K < 8 || K % 8 != 0 || K > 20480)
+        return fail(STARQ_ERR_SHAPE, "glue_add_rmsnorm: L=%d, K=%d: need L >= 0, 8 <= K <= 20480, K %% 8 == 0", L, K);
+    if (L == 0) return STARQ_OK;
+    if (!X || (Y && !w) || (!Y && !h_out)) return fail(STARQ_ERR_ARG, "glue_add_rmsnorm: NULL X, w, or no output");
+    if (h_out && !R) return fail(STARQ_ERR_ARG, "glue_add_rmsnorm: h_out needs the residual R");
+    if (!(eps >= 0.f)) return fail(STARQ_ERR_ARG, "glue_add_rmsnorm: eps must be >= 0");
+    if (!aligned(X, 16) || (R && !aligned(R, 16)) || (w && !aligned(w, 16)) || (h_out && !aligned(h_out, 16)) ||
+        (Y && !aligned(Y, 16)))
+        return fail(STARQ_ERR_ALIGN, "glue_add_rmsnorm: X, R, w, h_out, Y must be 16-byte aligned");
+    const cudaError_t e = launch_add_rmsnorm(X, R, dtype, L, K, w, eps, h_out, Y, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "glue_add_rmsnorm launch");
+    return STARQ_OK;
+}
+
+int glue_rope(void* QK, int dtype, int L, int ld, int heads, const int32_t* pos, double theta, void* stream) {
+    if (dtype != STARQ_F16 && dtype != STARQ_BF16) return fail(STARQ_ERR_ARG, "glue_rope: dtype must be F16 or BF16");
+    if (L < 0 || heads < 1 || ld < 128 * heads)
+        return fail(STARQ_ERR_SHAPE, "glue_rope: L=%d, heads=%d, ld=%d: need ld >= 128 heads", L, heads, ld);
+    if (!(theta > 1.0)) return fail(STARQ_ERR_ARG, "glue_rope: theta must be > 1");
+    if (L == 0) return STARQ_OK;
+    if (!QK || !pos) return fail(STARQ_ERR_ARG, "glue_rope: NULL QK or pos");
+    const cudaError_t e = launch_rope(QK, dtype, L, ld, heads, pos, theta, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "glue_rope launch");
+    return STARQ_OK;
+}
+
+int starq_probe_mma(int kind, int iters, unsigned long long* cycles, int* errors, int* ctas, double* macs_per_cta,
+                    void* stream) {
+    if (kind < 0 || kind > 4) return fail(STARQ_ERR_ARG, "starq_probe_mma: kind=%d outside 0..4", kind);
+    if (iters < 1 || iters > 2048) return fail(STARQ_ERR_ARG, "starq_probe_mma: iters=%d outside 1..2048", iters);
+    if (!cycles || !errors || !ctas || !macs_per_cta) return fail(STARQ_ERR_ARG, "starq_probe_mma: NULL pointer");
+    int rc = check_local("starq_probe_mma", static_cast<cudaStream_t>(stream), {cycles, errors});
+    if (rc) return rc;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    const cudaError_t e = launch_probe_mma(kind, iters, cycles, errors, st, ctas, macs_per_cta,
+                                           static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "starq_probe_mma launch");
     return STARQ_OK;
 }
 
@@ -571,21 +620,24 @@ int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, c
     return STARQ_OK;
 }
 
-size_t attention_pv_tac_workspace_size(int L, int H) {
-    if (L <= 0 || H <= 0) return 0;
-    return attn_workspace_bytes(L, H);
+size_t attention_pv_tac_workspace_size(int L, int Hkv) {
+    if (L <= 0 || Hkv <= 0) return 0;
+    return attn_workspace_bytes(L, Hkv);
 }
 
-int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L, int H, const void* Mp,
-                     const float* d, void* Z, uint8_t* dbg_codes, float* dbg_l, int32_t* dbg_acc, void* workspace,
-                     size_t workspace_bytes, void* stream) {
+int attention_pv_tac_gqa(const void* Q, const void* K, const void* V, int ld, int L, int H, int Hkv, int dtype,
+                         const void* Mp, const float* d, void* Z, uint8_t* dbg_codes, float* dbg_l, int32_t* dbg_acc,
+                         void* workspace, size_t workspace_bytes, void* stream) {
     if (!Q || !K || !V || !Mp || !Z || !workspace) return fail(STARQ_ERR_ARG, "attention_pv_tac: NULL pointer");
-    if (H < 1) return fail(STARQ_ERR_SHAPE, "attention_pv_tac: H=%d", H);
+    if (dtype != STARQ_F16 && dtype != STARQ_BF16)
+        return fail(STARQ_ERR_ARG, "attention_pv_tac: dtype must be F16 or BF16");
+    if (H < 1 || Hkv < 1 || H % Hkv != 0)
+        return fail(STARQ_ERR_SHAPE, "attention_pv_tac: H=%d, Hkv=%d: need H a positive multiple of Hkv", H, Hkv);
     if (L < ATTN_TILE || L % ATTN_TILE != 0 || L > 8192)
         return fail(STARQ_ERR_SHAPE, "attention_pv_tac: L=%d: need 128 <= L <= 8192, L %% 128 == 0", L);
     if (ld < ATTN_D * H || ld % 8 != 0)
         return fail(STARQ_ERR_SHAPE, "attention_pv_tac: ld=%d: need ld >= 128 H and ld %% 8 == 0", ld);
-    const size_t need = attention_pv_tac_workspace_size(L, H);
+    const size_t need = attention_pv_tac_workspace_size(L, Hkv);
     if (workspace_bytes < need) return fail(STARQ_ERR_SHAPE, "attention_pv_tac: workspace %zu bytes < %zu", workspace_bytes, need);
     if (!aligned(Q, 16) || !aligned(K, 16) || !aligned(V, 16) || !aligned(Mp, 16) || !aligned(Z, 16) ||
         (d && !aligned(d, 16)) || !aligned(workspace, 256))
@@ -596,11 +648,18 @@ int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L,
     if (!st) return rc;
     uint8_t* ws = static_cast<uint8_t*>(workspace);
     AttnArgs a{Q, K, V, ld, L, H, Mp, d, Z, reinterpret_cast<uint16_t*>(ws),
-               reinterpret_cast<float*>(ws + ((size_t)ATTN_D * H * L * 2 + 255) / 256 * 256),
-               dbg_codes, dbg_l, dbg_acc, st};
+               reinterpret_cast<float*>(ws + ((size_t)ATTN_D * Hkv * L * 2 + 255) / 256 * 256),
+               dbg_codes, dbg_l, dbg_acc, st, Hkv, dtype};
     cudaError_t e = launch_attention_pv_tac(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "attention_pv_tac launch");
     return STARQ_OK;
+}
+
+int attention_pv_tac(const void* Q, const void* K, const void* V, int ld, int L, int H, const void* Mp,
+                     const float* d, void* Z, uint8_t* dbg_codes, float* dbg_l, int32_t* dbg_acc, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+    return attention_pv_tac_gqa(Q, K, V, ld, L, H, H, STARQ_F16, Mp, d, Z, dbg_codes, dbg_l, dbg_acc, workspace,
+                                workspace_bytes, stream);
 }
 
 size_t tac_calibrate_workspace_size(int C, int g) {

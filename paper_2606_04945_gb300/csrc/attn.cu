@@ -15,6 +15,16 @@
 //   acc_ic = sum_j c_ij v_jc exact (|acc| <= 255 * 7 * L < 2^24 in float32).
 //   TAC: Z = Z_hat_h M_h^T + d_h per head (the head's 128 channels are one
 //   block).
+// Grouped-query attention: H query heads share Hkv key/value heads (H a
+// multiple of Hkv); query head h reads key/value head h / (H / Hkv), whose
+// V channels carry one set of codes and scales for the whole group.
+// Element type T of Q, K, V and Z: fp16 or bf16. Q K^T runs in T; the P and
+// V codes are integers held as fp16 (exact either way). The TAC product
+// always runs on fp16 halves (Z_hat and M split into hi + lo, 2^-22
+// relative): before the split Z_hat is scaled by an exact power of two
+// 2^-k chosen per head from its largest V scale, so that its bound
+// 16 * 7 max_c t_c lands in [2^13, 2^14) (inside fp16's range, with its
+// full precision), and the TAC accumulator is scaled back by 2^k.
 //
 // attn_vquant_kernel   V codes per channel, written as fp16 values into
 //                      Vt [128 H][L] (keys contiguous: the K-major B
@@ -55,6 +65,8 @@
 // bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+
+#include <type_traits>
 
 #include "attn.cuh"
 #include "common.cuh"
@@ -140,6 +152,24 @@ __device__ __forceinline__ bool mbar_wait2_bounded_warp(uint32_t b0, uint32_t p0
     return __all_sync(0xffffffffu, ok);
 }
 
+__device__ __forceinline__ float2 to_float2(__half2 h) { return __half22float2(h); }
+__device__ __forceinline__ float2 to_float2(__nv_bfloat162 h) { return __bfloat1622float2(h); }
+
+// Two floats -> T2 bits (round to nearest even), and a float rounded to T
+// and back.
+__device__ __forceinline__ uint32_t pack2(__half, float x, float y) {
+    const __half2 v = __floats2half2_rn(x, y);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+__device__ __forceinline__ uint32_t pack2(__nv_bfloat16, float x, float y) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(x, y);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+__device__ __forceinline__ uint16_t bits_rn(__half, float x) { return __half_as_ushort(__float2half_rn(x)); }
+__device__ __forceinline__ uint16_t bits_rn(__nv_bfloat16, float x) { return __bfloat16_as_ushort(__float2bfloat16_rn(x)); }
+__device__ __forceinline__ float from_bits(__half, uint16_t b) { return __half2float(__ushort_as_half(b)); }
+__device__ __forceinline__ float from_bits(__nv_bfloat16, uint16_t b) { return __bfloat162float(__ushort_as_bfloat16(b)); }
+
 __device__ __forceinline__ void named_sync_softmax() {
     asm volatile("bar.sync 1, %0;" :: "r"(ATT_SOFTMAX_THREADS) : "memory");
 }
@@ -150,13 +180,15 @@ __device__ __forceinline__ void named_sync_softmax() {
 // 512 keys and written as 16-byte rows of Vt.
 constexpr int VQ_CH = 16, VQ_KEYS = 512;
 
+template <typename T>
 __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
+    using T2 = typename std::conditional<std::is_same<T, __half>::value, __half2, __nv_bfloat162>::type;
     __shared__ float red[8][VQ_CH];
     __shared__ float rcp[VQ_CH];
     __shared__ __align__(16) uint16_t tile[VQ_CH][VQ_KEYS + 8];
     const int c0 = blockIdx.x * VQ_CH;
     const int tid = threadIdx.x, hv = tid & 1, rr = tid >> 1, warp = tid >> 5, lane = tid & 31;
-    const __half* col = static_cast<const __half*>(a.V) + c0 + 8 * hv;
+    const T* col = static_cast<const T*>(a.V) + c0 + 8 * hv;
     auto load = [&](int r) {
         return r < a.L ? __ldg(reinterpret_cast<const uint4*>(col + (size_t)r * a.ld)) : make_uint4(0u, 0u, 0u, 0u);
     };
@@ -169,10 +201,10 @@ __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
         for (int u = 0; u < 4; ++u) v[u] = load(r0 + rr + 128 * u);
         #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            const __half2* p = reinterpret_cast<const __half2*>(&v[u]);
+            const T2* p = reinterpret_cast<const T2*>(&v[u]);
             #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                const float2 f = __half22float2(p[k]);
+                const float2 f = to_float2(p[k]);
                 m[2 * k] = fmaxf(m[2 * k], fabsf(f.x));
                 m[2 * k + 1] = fmaxf(m[2 * k + 1], fabsf(f.y));
             }
@@ -206,10 +238,10 @@ __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
         for (int u = 0; u < 4; ++u) v[u] = load(r0 + rr + 128 * u);
         #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            const __half2* p = reinterpret_cast<const __half2*>(&v[u]);
+            const T2* p = reinterpret_cast<const T2*>(&v[u]);
             #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                const float2 f = __half22float2(p[k]);
+                const float2 f = to_float2(p[k]);
                 tile[8 * hv + 2 * k][rr + 128 * u] = __half_as_ushort(__float2half_rn(rintf(__fmul_rn(f.x, rc[2 * k]))));
                 tile[8 * hv + 2 * k + 1][rr + 128 * u] =
                     __half_as_ushort(__float2half_rn(rintf(__fmul_rn(f.y, rc[2 * k + 1]))));
@@ -228,6 +260,7 @@ __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
 
 // A ring slot is refilled once this CTA's MMAs have read it (one commit on
 // its empty barrier).
+template <typename T>
 __global__ void __launch_bounds__(ATT_THREADS, 1)
 attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_z) {
@@ -237,6 +270,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
     AttSm* sh = reinterpret_cast<AttSm*>(smem_raw + (base - raw) + ATT_TILES_BYTES);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int q0 = blockIdx.x * ATTN_TILE, h = blockIdx.y;
+    const int hk = h / (a.H / a.Hkv);                       // key/value head of this query head
     const int nk = a.L / ATTN_TILE;
     volatile int* abort = &sh->abort;
     // (the lambdas capture by value: a local captured by reference lives in
@@ -304,11 +338,11 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 const void* tm = (w < 0 || (w & 1) == 0) ? (const void*)&tm_k : (const void*)&tm_v;
                 int x, y;
                 if (w < 0 || (w & 1) == 0) {                 // K chunk: keys are the rows
-                    x = h * ATTN_D;
+                    x = hk * ATTN_D;
                     y = (w < 0 ? u : w >> 1) * ATTN_TILE;
                 } else {                                     // V chunk: channels are the rows
                     x = (w >> 1) * ATTN_TILE;
-                    y = h * ATTN_D;
+                    y = hk * ATTN_D;
                 }
                 tma_load_2d(dst, tm, x, y, fb);
                 tma_load_2d(dst + ATOM_BYTES, tm, x + 64, y, fb);
@@ -331,14 +365,18 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             if (u >= 0) ok = mbar_wait_bounded_warp(B(sh->empty[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1), abort);
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     } else if (warp == ATT_MMA_WARP) {
-        // f16 A and B, f32 D, N = 128 (bits 17..22), M = 128 (bits 24..28)
-        constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(ATTN_TILE >> 3) << 17) | ((uint32_t)(ATTN_TILE >> 4) << 24);
+        // f32 D, N = 128 (bits 17..22), M = 128 (bits 24..28); A and B fp16
+        // (P V^T: integer codes; TAC: fp16 halves) or of type T (Q K^T; bf16
+        // sets the A and B format fields, bits 7..9 and 10..12)
+        constexpr uint32_t IDESC_F16 = (1u << 4) | ((uint32_t)(ATTN_TILE >> 3) << 17) | ((uint32_t)(ATTN_TILE >> 4) << 24);
+        constexpr uint32_t IDESC_T = IDESC_F16 | (std::is_same<T, __nv_bfloat16>::value ? ((1u << 7) | (1u << 10)) : 0u);
+        (void)IDESC_T;
         bool ok = mbar_wait_bounded_warp(B(sh->q_full), 0, abort);
         // D (+)= A B^T over K = 128: A from TMEM at a_col (8 columns per K
         // step; for P, K steps 2p and 2p + 1 sit at 32 p and 32 p + 8), B
         // the K-major tile at bt
         // (issued by the elected lane)
-        auto mma_tile = [=](uint32_t d, uint32_t a_col, uint32_t bt, bool acc0, bool p_layout) {
+        auto mma_tile = [=](uint32_t d, uint32_t a_col, uint32_t bt, bool acc0, bool p_layout, uint32_t idesc) {
             // K step offsets added to the descriptor's start-address field
             // (addresses below 2^18, so the field never carries)
             const uint64_t bd = smem_desc_sw128(bt);
@@ -347,7 +385,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             for (int ks = 0; ks < ATTN_D / 16; ++ks) {
                 const uint32_t koff = (uint32_t)(ks >> 2) * ATOM_BYTES + (uint32_t)(ks & 3) * 32;
                 const uint32_t ac = p_layout ? 32u * (uint32_t)(ks >> 1) + 8u * (uint32_t)(ks & 1) : 8u * (uint32_t)ks;
-                mma_f16_ts(d, ta + ac, bd + (uint64_t)(koff >> 4), IDESC, (acc0 || ks > 0) ? 1u : 0u);
+                mma_f16_ts(d, ta + ac, bd + (uint64_t)(koff >> 4), idesc, (acc0 || ks > 0) ? 1u : 0u);
             }
         };
         auto release = [=](int u) {           // this CTA's MMAs are done with ring slot u
@@ -368,7 +406,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 return false;
             tc_fence_after();
             if (elect_one()) {
-                mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(u), false, false);
+                mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(u), false, false, IDESC_T);
                 release(u);
                 tc_commit(B(sh->s_full[b]));
             }
@@ -385,7 +423,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 return false;
             tc_fence_after();
             if (elect_one()) {
-                mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(u), j > 0, true);
+                mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(u), j > 0, true, IDESC_F16);
                 release(u);
             }
             __syncwarp();
@@ -404,9 +442,9 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             tc_fence_after();
             if (elect_one()) {
                 if (ok) {
-                    mma_tile(tmem + TM_TAC, TM_ZHI, sMhi, false, false);   // Z_hi M_hi^T
-                    mma_tile(tmem + TM_TAC, TM_ZHI, sMlo, true, false);    // + Z_hi M_lo^T
-                    mma_tile(tmem + TM_TAC, TM_ZLO, sMhi, true, false);    // + Z_lo M_hi^T
+                    mma_tile(tmem + TM_TAC, TM_ZHI, sMhi, false, false, IDESC_F16);   // Z_hi M_hi^T
+                    mma_tile(tmem + TM_TAC, TM_ZHI, sMlo, true, false, IDESC_F16);    // + Z_hi M_lo^T
+                    mma_tile(tmem + TM_TAC, TM_ZLO, sMhi, true, false, IDESC_F16);    // + Z_lo M_hi^T
                 }
                 tc_commit(B(sh->tac_done));
             }
@@ -427,7 +465,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         uint32_t r[32];
         {   // the query row's 32 channels of this part into TMEM (A of Q K^T);
             // the loads of Q, t and d are all in flight together
-            const __half* qp = static_cast<const __half*>(a.Q) + (size_t)(q0 + row) * a.ld + h * ATTN_D + col;
+            const T* qp = static_cast<const T*>(a.Q) + (size_t)(q0 + row) * a.ld + h * ATTN_D + col;
             uint32_t qv[16];
             #pragma unroll
             for (int k = 0; k < 4; ++k) {
@@ -462,7 +500,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             #pragma unroll
             for (int k = 0; k < 32; ++k) mx = fmaxf(mx, __uint_as_float(r[k]));
         }
-        if (threadIdx.x < ATTN_D) sh->tv[threadIdx.x] = a.t[h * ATTN_D + threadIdx.x];   // V channel scales
+        if (threadIdx.x < ATTN_D) sh->tv[threadIdx.x] = a.t[hk * ATTN_D + threadIdx.x];  // V channel scales
         sh->xm[part][row] = mx;
         named_sync_softmax();
         mx = fmaxf(fmaxf(sh->xm[0][row], sh->xm[1][row]), fmaxf(sh->xm[2][row], sh->xm[3][row]));
@@ -513,6 +551,15 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         named_sync_softmax();
         const float l = (sh->xm[0][row] + sh->xm[1][row]) + (sh->xm[2][row] + sh->xm[3][row]);
         const float sp = __fdiv_rn(1.f, __fmul_rn(255.f, l));
+        // the head's power-of-two TAC scale: |Z_hat| <= 16 * 7 max_c t_c (the
+        // codes of a row sum to at most twice 255 l), brought into [2^13, 2^14)
+        float tmax = 0.f;
+        #pragma unroll
+        for (int c = lane; c < ATTN_D; c += 32) tmax = fmaxf(tmax, sh->tv[c]);
+        #pragma unroll
+        for (int m = 16; m > 0; m >>= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, m));
+        const int zk = tmax > 0.f ? ilogbf(112.f * tmax) - 13 : 0;
+        const float zscale = ldexpf(1.f, -zk), zunscale = ldexpf(1.f, zk);
         if (a.dbg_l != nullptr && part == 0) a.dbg_l[(size_t)h * a.L + q0 + row] = l;
         // epilogue 1: Z_hat = (acc sp) t as fp16 hi + lo, the A operands of
         // the TAC product, into TMEM
@@ -531,11 +578,13 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             for (int k = 0; k < 32; k += 2) {
                 float z[2];
                 #pragma unroll
-                for (int u = 0; u < 2; ++u) z[u] = __fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), sh->tv[col + k + u]);
-                const __half h0 = __float2half_rn(z[0]), h1 = __float2half_rn(z[1]);
-                const __half l0 = __float2half_rn(z[0] - __half2float(h0)), l1 = __float2half_rn(z[1] - __half2float(h1));
-                hi[k / 2] = (uint32_t)__half_as_ushort(h0) | ((uint32_t)__half_as_ushort(h1) << 16);
-                lo[k / 2] = (uint32_t)__half_as_ushort(l0) | ((uint32_t)__half_as_ushort(l1) << 16);
+                for (int u = 0; u < 2; ++u)
+                    z[u] = __fmul_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), sh->tv[col + k + u]), zscale);
+                const uint16_t h0 = bits_rn(__half(), z[0]), h1 = bits_rn(__half(), z[1]);
+                const uint16_t l0 = bits_rn(__half(), z[0] - from_bits(__half(), h0)),
+                               l1 = bits_rn(__half(), z[1] - from_bits(__half(), h1));
+                hi[k / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+                lo[k / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
             }
             tmem_st_32x32b_x16(tl + TM_ZHI + part * 16, hi);
             tmem_st_32x32b_x16(tl + TM_ZLO + part * 16, lo);
@@ -558,13 +607,12 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     const int k = 8 * g + 2 * u;
-                    float y0 = __uint_as_float(r[k]), y1 = __uint_as_float(r[k + 1]);
+                    float y0 = __fmul_rn(__uint_as_float(r[k]), zunscale), y1 = __fmul_rn(__uint_as_float(r[k + 1]), zunscale);
                     if (add_d) {
                         y0 = __fadd_rn(y0, sh->dv[col + k]);
                         y1 = __fadd_rn(y1, sh->dv[col + k + 1]);
                     }
-                    const __half2 hv = __floats2half2_rn(y0, y1);
-                    w[u] = *reinterpret_cast<const uint32_t*>(&hv);
+                    w[u] = pack2(T(), y0, y1);
                 }
                 st_shared_v4(box + lane * 64 + 16 * (g ^ ((lane >> 1) & 3)), w[0], w[1], w[2], w[3]);
             }
@@ -586,44 +634,46 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
 }
 
 bool encode_2d(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint64_t row_elems,
-               uint32_t box_rows, uint32_t box_cols, CUtensorMapSwizzle swz) {
+               uint32_t box_rows, uint32_t box_cols, CUtensorMapSwizzle swz,
+               CUtensorMapDataType type = CU_TENSOR_MAP_DATA_TYPE_FLOAT16) {
     const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
     if (fn == nullptr) return false;
     const cuuint64_t dims[2] = {cols, rows};
     const cuuint64_t strides[1] = {row_elems * 2};
     const cuuint32_t box[2] = {box_cols, box_rows};
     const cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+    return fn(m, type, 2, const_cast<void*>(ptr), dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
 
+template <typename T>
 cudaError_t launch_pv_tac(const AttnArgs& a, cudaStream_t stream) {
-    const int C = ATTN_D * a.H;
+    const int C = ATTN_D * a.H, Ckv = ATTN_D * a.Hkv;
+    const CUtensorMapDataType io = std::is_same<T, __half>::value ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                                                   : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     CUtensorMap tk, tv, tz;
-    if (!encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)C, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_2d(&tv, a.Vt, (uint64_t)C, (uint64_t)a.L, (uint64_t)a.L, ATTN_D, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
-        !encode_2d(&tz, a.Z, (uint64_t)a.L, (uint64_t)C, (uint64_t)C, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
+    if (!encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)Ckv, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B, io) ||
+        !encode_2d(&tv, a.Vt, (uint64_t)Ckv, (uint64_t)a.L, (uint64_t)a.L, ATTN_D, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
+        !encode_2d(&tz, a.Z, (uint64_t)a.L, (uint64_t)C, (uint64_t)C, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B, io))
         return cudaErrorInvalidValue;
     static DeviceCache<int> attr;
     int done = 0;
-    const cudaError_t e = attr.get(&done, [](int, int* v) {
+    cudaError_t e = attr.get(&done, [](int, int* v) {
         *v = 1;
-        return cudaFuncSetAttribute(attn_pv_tac_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ATT_SMEM);
+        return cudaFuncSetAttribute(attn_pv_tac_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ATT_SMEM);
     });
     if (e != cudaSuccess) return e;
-    attn_pv_tac_kernel<<<dim3(a.L / ATTN_TILE, a.H), ATT_THREADS, ATT_SMEM, stream>>>(a, tk, tv, tz);
+    attn_vquant_kernel<T><<<Ckv / VQ_CH, 256, 0, stream>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    attn_pv_tac_kernel<T><<<dim3(a.L / ATTN_TILE, a.H), ATT_THREADS, ATT_SMEM, stream>>>(a, tk, tv, tz);
     return cudaGetLastError();
 }
 
 cudaError_t launch_attention_pv_tac(const AttnArgs& a, cudaStream_t stream) {
-    const int C = ATTN_D * a.H;
-    attn_vquant_kernel<<<C / VQ_CH, 256, 0, stream>>>(a);
-    const cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    return launch_pv_tac(a, stream);
+    return a.dtype == STARQ_BF16 ? launch_pv_tac<__nv_bfloat16>(a, stream) : launch_pv_tac<__half>(a, stream);
 }
 
 }  // namespace starq

@@ -7,21 +7,24 @@ start masked and 4 are unmasked per step (seeded random confidence), each
 with a seeded random token, so the trajectory does not depend on the
 outputs. Per block:
 
-    h = RMSNorm(x)
+    h = RMSNorm(x)                          glue_add_rmsnorm
     q, k, v = SGAT-W4A4(h)                  QKV 4096 -> 12288 (Sec. 3.2)
-    a = softmax(RoPE(q) RoPE(k)^T / sqrt(128)) v          (bidirectional)
-    x = x + SGAT-W4A4(TAC(a))               O 4096 -> 4096, TAC 128 x 128 per head (Sec. 3.3)
-    h = RMSNorm(x)
+    q, k = RoPE(q, k)                       glue_rope
+    a = TAC(Q8(softmax(q k^T / sqrt(128))) Q4(v))     attention_pv_tac: the
+                                            quantised softmax-value product with
+                                            TAC, 128 x 128 per head (Sec. 3.3)
+    x = x + SGAT-W4A4(a); h = RMSNorm(x)    O 4096 -> 4096; glue_add_rmsnorm
     g, u = SGAT-W4A4(h)                     gate+up 4096 -> 2 x 12288
     x = x + SGAT-W4A4(silu(g) u)            down 12288 -> 4096
 
-Every linear is one `sgat_linear` call of the C ABI with the token's mask
-bit selecting its transform; the gate+up projection is `sgat_linear_swiglu`,
-which applies silu(g) u in the GEMM epilogue. RMSNorm, RoPE, attention and
-the residuals are glue (torch ops on the GPU), not part of the quantised
-path; the 16-bit baseline applies SwiGLU as glue too.
-The same stack with 16-bit GEMMs (`fp16_gemm_ref`, no quantisation, no
-TAC) is the unquantised baseline for the per-step output drift.
+Every step runs in libstarq kernels: every linear is one `sgat_linear` call
+with the token's mask bit selecting its transform (the gate+up projection
+is `sgat_linear_swiglu`, with silu(g) u in the GEMM epilogue), attention is
+the quantised product whose output TAC compensates, and RMSNorm, RoPE and
+the residuals are the library's glue kernels.
+The same stack with 16-bit GEMMs (`fp16_gemm_ref`), unquantised attention
+(torch's fp16 SDPA) and no TAC is the unquantised baseline for the
+per-step output drift; it applies SwiGLU as glue.
 
 The per-state smoothing of every linear is calibrated on that linear's
 input in one 16-bit pass over the initial state (synthetic calibration).
@@ -50,22 +53,8 @@ class StackConfig:
     seed: int = 0
 
 
-def rms_norm(x, eps=1e-6):
-    xf = x.float()
-    return (xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True) + eps)).to(x.dtype)
-
-
-def rope_tables(L, d, device, base=10000.0):
-    inv = 1.0 / (base ** (torch.arange(0, d, 2, device=device, dtype=torch.float32) / d))
-    ang = torch.arange(L, device=device, dtype=torch.float32)[:, None] * inv[None]
-    return torch.cos(ang), torch.sin(ang)
-
-
-def apply_rope(t, cos, sin):
-    # t [heads, L, d]; rotate the two halves of each head
-    d2 = t.shape[-1] // 2
-    t1, t2 = t[..., :d2].float(), t[..., d2:].float()
-    return torch.cat([t1 * cos - t2 * sin, t1 * sin + t2 * cos], -1).to(t.dtype)
+ROPE_THETA = 10000.0
+EPS = 1e-6
 
 
 class QLinear:
@@ -73,28 +62,15 @@ class QLinear:
     W4A4 form (packed int4 codes, E4M3 copy, per-channel scales), the SGAT
     transforms, optional TAC, and a workspace."""
 
-    def __init__(self, W16, L, tac=None, swiglu=False):
+    def __init__(self, W16, L, swiglu=False):
         self.W16 = W16
         self.N, self.K = W16.shape
         self.L = L
-        self.tac = tac
+        self.tac = None
         # gate+up of the MLP: the W4A4 form keeps the rows in
         # swiglu_row_order and writes silu(gate) * up [L][N / 2]
         self.swiglu = swiglu
         self.sgat = None
-        self.tac_M = self.tac_d = self.tac_Mp = None
-        if tac is not None:
-            dev = W16.device
-            self.tac_M = torch.from_numpy(tac.M).to(dev)
-            self.tac_d = torch.from_numpy(tac.d).to(dev)
-            self.tac_Mp = torch.empty(abi.tac_prepared_bytes(self.K, tac.g), dtype=torch.uint8, device=dev)
-            abi.tac_prepare(self.tac_M, tac.g, W16.dtype, self.tac_Mp)
-
-    def tac_out(self, X):
-        """TAC of the linear's input (float32), as sgat_linear applies it."""
-        Z = torch.empty(X.shape, dtype=torch.float32, device=X.device)
-        abi.tac_apply(X, self.tac_M, self.tac_d, self.tac.g, Z, Mp=self.tac_Mp)
-        return Z
 
     def calibrate(self, X, mask):
         xf = inputs.make_sgat(X.float().cpu().numpy(), mask)
@@ -118,11 +94,35 @@ class QLinear:
                                    Y, self.workspace, We=self.We)
             return
         abi.sgat_linear(X, mask, self.a_m, self.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, self.Wq, self.s_w, Y,
-                        self.workspace, tac_M=self.tac_M, tac_d=self.tac_d,
-                        tac_g=self.tac.g if self.tac is not None else 0, We=self.We, tac_Mp=self.tac_Mp)
+                        self.workspace, We=self.We)
 
     def fp16(self, X, Y):
         abi.fp16_gemm_ref(X, self.W16, Y)
+
+
+class QAttention:
+    """The quantised softmax-value product of one block with TAC in its
+    epilogue (per-head 128 x 128 blocks, prepared once)."""
+
+    def __init__(self, tac, L, heads, device):
+        self.tac = tac
+        self.heads = heads
+        self.M = torch.from_numpy(tac.M).to(device)
+        self.d = torch.from_numpy(tac.d).to(device)
+        self.Mp = torch.empty(abi.tac_prepared_bytes(tac.C, tac.g), dtype=torch.uint8, device=device)
+        abi.tac_prepare(self.M, tac.g, torch.float16, self.Mp)
+        self.workspace = torch.empty(abi.attention_pv_tac_workspace_size(L, heads), dtype=torch.uint8, device=device)
+
+    def run(self, qkv, out, **dbg):
+        C = self.heads * 128
+        abi.attention_pv_tac(qkv[:, :C], qkv[:, C:2 * C], qkv[:, 2 * C:], self.heads, self.Mp, self.d, out,
+                             workspace=self.workspace, **dbg)
+
+    def tac_f32(self, A):
+        """TAC of a 16-bit attention output, in float32 (calibration)."""
+        Z = torch.empty(A.shape, dtype=torch.float32, device=A.device)
+        abi.tac_apply(A, self.M, self.d, self.tac.g, Z, Mp=self.Mp)
+        return Z
 
 
 class DenoiseStack:
@@ -139,10 +139,12 @@ class DenoiseStack:
         for _ in range(c.layers):
             self.blocks.append(dict(
                 qkv=QLinear(w(3 * c.hidden, c.hidden), c.seq),
-                o=QLinear(w(c.hidden, c.hidden), c.seq, tac=inputs.make_tac(rng, c.hidden, c.tac_block)),
+                attn=QAttention(inputs.make_tac(rng, c.hidden, c.tac_block), c.seq, c.heads, device),
+                o=QLinear(w(c.hidden, c.hidden), c.seq),
                 gu=QLinear(w(2 * c.ffn, c.hidden), c.seq, swiglu=True),
                 down=QLinear(w(c.hidden, c.ffn), c.seq)))
-        self.cos, self.sin = rope_tables(c.seq, c.hidden // c.heads, device)
+        self.ones = torch.ones(c.hidden, dtype=torch.float32, device=device)
+        self.pos = torch.arange(c.seq, dtype=torch.int32, device=device)
         # denoising trajectory: prompt tokens, then masked positions unmasked
         # four per step in a seeded order with seeded tokens
         self.prompt = torch.from_numpy(rng.integers(1, c.vocab, c.seq - c.gen)).to(device)
@@ -150,7 +152,8 @@ class DenoiseStack:
         self.new_tokens = rng.integers(1, c.vocab, c.gen)
         L, H, F = c.seq, c.hidden, c.ffn
         t = lambda *s: torch.empty(*s, dtype=torch.float16, device=device)
-        self.buf = dict(qkv=t(L, 3 * H), attn=t(L, H), o=t(L, H), gu=t(L, 2 * F), act=t(L, F), down=t(L, H))
+        self.buf = dict(x=t(L, H), h=t(L, H), qkv=t(L, 3 * H), attn=t(L, H), o=t(L, H), gu=t(L, 2 * F),
+                        act=t(L, F), down=t(L, H))
 
     # -- trajectory -----------------------------------------------------
     def state(self, step):
@@ -167,35 +170,41 @@ class DenoiseStack:
         return tok, mask
 
     # -- one forward pass ------------------------------------------------
-    def _attention(self, qkv):
+    def _sdpa(self, qkv):
+        """Unquantised attention of the 16-bit baseline (on roped q, k)."""
         c = self.cfg
         L, H, nh = c.seq, c.hidden, c.heads
-        d = H // nh
-        q, k, v = qkv.view(L, 3, nh, d).permute(1, 2, 0, 3)          # [3][heads][L][d]
-        q, k = apply_rope(q, self.cos, self.sin), apply_rope(k, self.cos, self.sin)
+        q, k, v = qkv.view(L, 3, nh, H // nh).permute(1, 2, 0, 3)          # [3][heads][L][d]
         a = torch.nn.functional.scaled_dot_product_attention(q[None], k[None], v[None])[0]
-        return a.permute(1, 0, 2).reshape(L, H).contiguous()
+        return a.permute(1, 0, 2).reshape(L, H)
 
     def forward(self, tok, mask, quantised=True, hook=None):
         """One denoising step of the whole stack; returns the final hidden
         state. tok: token ids (device, long), mask: mask bits (numpy or
-        device uint8). `hook(layer, name, linear, X, Y)` runs after each
-        quantised linear (X its input, Y its output) for inspection."""
+        device uint8). `hook(layer, name, module, X, Y)` runs after each
+        quantised linear (X its input, Y its output) and after the quantised
+        attention (X the roped QKV output, Y the TAC-compensated output)."""
         mask_d = mask if torch.is_tensor(mask) else torch.from_numpy(mask).to(self.device)
         return self._forward(tok, mask_d, quantised, hook)
 
     def _forward(self, tok, mask_d, quantised, hook):
         c = self.cfg
         b = self.buf
-        x = self.embed[tok].clone()
+        H, nh = c.hidden, c.heads
+        x, h = b["x"], b["h"]
+        x.copy_(self.embed[tok])
+        abi.add_rmsnorm(x, self.ones, h, eps=EPS)
         for li, blk in enumerate(self.blocks):
-            h = rms_norm(x)
             self._lin(blk["qkv"], h, mask_d, b["qkv"], quantised, hook, li, "qkv")
-            a = self._attention(b["qkv"])
-            b["attn"].copy_(a)
+            abi.rope(b["qkv"], 2 * nh, self.pos, ROPE_THETA)
+            if quantised:
+                blk["attn"].run(b["qkv"], b["attn"])
+                if hook is not None:
+                    hook(li, "attn", blk["attn"], b["qkv"], b["attn"])
+            else:
+                b["attn"].copy_(self._sdpa(b["qkv"]))
             self._lin(blk["o"], b["attn"], mask_d, b["o"], quantised, hook, li, "o")
-            x = x + b["o"]
-            h = rms_norm(x)
+            abi.add_rmsnorm(b["o"], self.ones, h, R=x, h_out=x, eps=EPS)        # x += o; h = norm(x)
             if quantised:                                 # silu(gate) * up in the GEMM epilogue
                 self._lin(blk["gu"], h, mask_d, b["act"], True, hook, li, "gu")
             else:
@@ -203,7 +212,9 @@ class DenoiseStack:
                 gt, up = b["gu"][:, : c.ffn], b["gu"][:, c.ffn:]
                 b["act"].copy_((torch.nn.functional.silu(gt.float()) * up.float()).half())
             self._lin(blk["down"], b["act"], mask_d, b["down"], quantised, hook, li, "down")
-            x = x + b["down"]
+            last = li == len(self.blocks) - 1
+            # x += down; h = norm(x) for the next block
+            abi.add_rmsnorm(b["down"], self.ones, None if last else h, R=x, h_out=x, eps=EPS)
         return x
 
     def capture(self, quantised=True):
@@ -238,27 +249,29 @@ class DenoiseStack:
             lin.fp16(X, Y)
 
     def calibrate(self):
-        """Per-linear smoothing from a 16-bit pass over the initial state."""
+        """Per-linear smoothing from a 16-bit pass over the initial state
+        (the O projection's on the TAC of the unquantised attention)."""
         tok, mask = self.state(0)
         c = self.cfg
         b = self.buf
-        x = self.embed[tok].clone()
+        x, h = b["x"], b["h"]
+        x.copy_(self.embed[tok])
+        abi.add_rmsnorm(x, self.ones, h, eps=EPS)
         for blk in self.blocks:
-            h = rms_norm(x)
             blk["qkv"].fp16(h, b["qkv"])
             blk["qkv"].calibrate(h, mask)
-            b["attn"].copy_(self._attention(b["qkv"]))
-            blk["o"].calibrate(blk["o"].tac_out(b["attn"]), mask)   # its quantiser sees TAC(a)
+            abi.rope(b["qkv"], 2 * c.heads, self.pos, ROPE_THETA)
+            b["attn"].copy_(self._sdpa(b["qkv"]))
+            blk["o"].calibrate(blk["attn"].tac_f32(b["attn"]), mask)
             blk["o"].fp16(b["attn"], b["o"])
-            x = x + b["o"]
-            h = rms_norm(x)
+            abi.add_rmsnorm(b["o"], self.ones, h, R=x, h_out=x, eps=EPS)
             blk["gu"].calibrate(h, mask)
             blk["gu"].fp16(h, b["gu"])
             gt, up = b["gu"][:, : c.ffn], b["gu"][:, c.ffn:]
             b["act"].copy_((torch.nn.functional.silu(gt.float()) * up.float()).half())
             blk["down"].calibrate(b["act"], mask)
             blk["down"].fp16(b["act"], b["down"])
-            x = x + b["down"]
+            abi.add_rmsnorm(b["down"], self.ones, h, R=x, h_out=x, eps=EPS)
 
     def linear_int_ops(self):
         c = self.cfg

@@ -137,3 +137,59 @@ def test_attention_pv_tac_uniform(abi):
         mean = (vq[:, ch] * t[ch][None, :]).astype(np.float64).mean(axis=0)
         ref = np.broadcast_to(mean @ tac.M[h].T + tac.d[h], (L, D))
         H.assert_tac_close(Zg[:, ch], ref, "f16")
+
+
+def run_case_gqa(abi, L, Hh, Hkv, dt, seed, heads=None):
+    """Grouped-query case: Q with Hh heads, K and V with Hkv heads, element
+    type dt ("f16" or "bf16"); the comparisons of run_case, with query head h
+    reading key/value head h // (Hh / Hkv)."""
+    rng = np.random.default_rng(seed)
+    C, Ckv = D * Hh, D * Hkv
+    QKV = rng.standard_normal((L, C + 2 * Ckv)).astype(np.float32)
+    QKV = QKV.astype(np.float16).astype(np.float32) if dt == "f16" else inputs.round_to_bf16(QKV)
+    tdt = H.torch_dtype(dt)
+    Y = H.dev(QKV, tdt)
+    Q, K, V = Y[:, :C], Y[:, C:C + Ckv], Y[:, C + Ckv:]
+    tac = inputs.make_tac(rng, C, D)
+    Mp = torch.empty(abi.tac_prepared_bytes(C, D), dtype=torch.uint8, device="cuda")
+    abi.tac_prepare(H.dev(tac.M), D, torch.float16, Mp)      # fp16 halves for either I/O type
+    Z = torch.full((L, C), float("nan"), dtype=tdt, device="cuda")
+    codes = torch.zeros(Hh, L, L, dtype=torch.uint8, device="cuda")
+    lsum = torch.zeros(Hh, L, dtype=torch.float32, device="cuda")
+    acc = torch.zeros(Hh, L, D, dtype=torch.int32, device="cuda")
+    abi.attention_pv_tac(Q, K, V, Hh, Mp, H.dev(tac.d), Z, dbg_codes=codes, dbg_l=lsum, dbg_acc=acc, Hkv=Hkv)
+    abi.check_status()
+    Zg = H.host(Z)
+    assert not np.isnan(Zg).any()
+    gcodes, gl, gacc = codes.cpu().numpy().astype(np.int32), lsum.cpu().numpy(), acc.cpu().numpy()
+    Qn, Kn, Vn = QKV[:, :C], QKV[:, C:C + Ckv], QKV[:, C + Ckv:]
+    vq, t = oatt.v_codes(Vn)
+    group = Hh // Hkv
+    for h in (range(Hh) if heads is None else heads):
+        ch = slice(h * D, (h + 1) * D)
+        kv = slice((h // group) * D, (h // group + 1) * D)
+        S = oatt.scores(Qn[:, ch], Kn[:, kv], D)
+        oc, ol = oatt.p_codes(S)
+        diff = gcodes[h] != oc
+        if diff.any():
+            e255 = 255.0 * np.exp(S - S.max(axis=1, keepdims=True))
+            near = np.abs(e255 - np.floor(e255) - 0.5) < 1e-3
+            assert np.all(np.abs(gcodes[h] - oc)[diff] == 1) and np.all(near[diff]), f"head {h}: P codes"
+        np.testing.assert_allclose(gl[h], ol, rtol=1e-5, err_msg=f"head {h}: row sums")
+        ref_acc = osg.int_gemm(gcodes[h], vq[:, kv].T)
+        assert np.array_equal(gacc[h], ref_acc), f"head {h}: integer sums"
+        zhat = ref_acc.astype(np.float64) / (255.0 * gl[h].astype(np.float64)[:, None]) * t[kv].astype(np.float64)
+        ref = zhat @ tac.M[h].astype(np.float64).T + tac.d[h].astype(np.float64)[None, :]
+        H.assert_tac_close(Zg[:, ch], ref, dt)
+
+
+@pytest.mark.parametrize("L,Hh,Hkv,dt", [(256, 4, 1, "f16"), (384, 6, 2, "bf16"), (256, 2, 2, "bf16")])
+def test_attention_pv_tac_gqa_and_bf16(abi, L, Hh, Hkv, dt):
+    run_case_gqa(abi, L, Hh, Hkv, dt, seed=L + 10 * Hh + Hkv)
+
+
+def test_attention_pv_tac_dream_shape(abi):
+    """The Dream-7B attention: 2048 tokens (one sequence), 28 query heads
+    over 4 key/value heads, bf16; every seventh head checked (one per
+    group and the group edges)."""
+    run_case_gqa(abi, 2048, 28, 4, "bf16", seed=28, heads=(0, 6, 7, 13, 20, 27))

@@ -125,3 +125,49 @@ def test_sgat_linear_dense(abi, L, K, N, dtype):
     qw_o, sw_o, _ = osg.prepare_weight_dense(case.W, xf.inv_a_w, P)
     Y_o = osg.dequant(osg.int_gemm(codes_o, qw_o), s_o, sw_o, case.bias)
     assert np.linalg.norm(H.host(Y) - Y_o) / np.linalg.norm(Y_o) < 0.02
+
+
+def test_sgat_linear_dense_calibrated_basis(abi):
+    """The dense path on a basis calibrated by App. B's procedure (the
+    oracle's AdamW calibration on the Eq. 15 objective, paper settings, on
+    a synthetic calibration set): the GPU's codes and outputs match the
+    oracle on that basis (teacher-forced, as above), and the calibrated
+    basis gives a smaller error against the full-precision product X W^T
+    than the orthogonalised Gaussian it started from."""
+    from oracle import calibration as oc
+    K = N = 256
+    d_m = d_u = K // 32
+    d_sh = K - 2 * d_m
+    samples, W = inputs.basis_calibration_set(21, K, n_samples=8, tokens=64, N=N)
+    P_cal, hist = oc.calibrate_basis(samples, W, d_sh, d_m, d_u, seed=3)
+    assert hist["objective"][-1] < hist["objective"][0]
+    X, mask = inputs.basis_calibration_set(22, K, n_samples=1, tokens=200, N=N)[0][0]
+    X16 = X.astype(np.float16)
+    ones = np.ones(K, np.float32)
+    errs = []
+    for P in (oc.orthogonal_init(K, 3), P_cal):
+        P16 = P.astype(np.float16)
+        Pt = torch.from_numpy(np.ascontiguousarray(P16.T)).cuda()
+        Wq = torch.empty(N, K // 2, dtype=torch.uint8, device="cuda")
+        s_w = torch.empty(N, dtype=torch.float32, device="cuda")
+        abi.sgat_prepare_weight_dense(H.dev(W, torch.float16), H.dev(ones), Pt, Wq, s_w)
+        We = torch.empty(N, K, dtype=torch.uint8, device="cuda")
+        abi.w4_unpack_e4m3(Wq, We)
+        L = X.shape[0]
+        ws = torch.empty(abi.sgat_linear_dense_workspace_size(L, K), dtype=torch.uint8, device="cuda")
+        Y = torch.empty(L, N, dtype=torch.float16, device="cuda")
+        abi.sgat_linear_dense(H.dev(X16, torch.float16), H.dev(mask), H.dev(ones), H.dev(ones), Pt, d_sh, d_m, d_u,
+                              Wq, s_w, Y, ws, We=We)
+        abi.check_status()
+        a256 = lambda x: (x + 255) // 256 * 256
+        o = 2 * a256(2 * L * K)
+        codes = H.unpack(ws[o: o + L * K // 2].view(L, K // 2))
+        s_a = ws[o + a256(L * K // 2): o + a256(L * K // 2) + 4 * L].view(torch.float32).cpu().numpy()
+        v_gpu = ws[a256(2 * L * K): a256(2 * L * K) + 2 * L * K].view(torch.float16).view(L, K).float().cpu().numpy()
+        q, s = osg.quantize_rows_sym(gated(v_gpu, mask, d_sh, d_m, d_u), 4)
+        assert np.array_equal(codes, q) and np.array_equal(s_a, s), "codes on the GPU's V"
+        ref = osg.dequant(osg.int_gemm(codes, H.unpack(Wq)), s_a, s_w.cpu().numpy(), None)
+        H.assert_output_close(H.host(Y), ref, "f16")
+        exact = X16.astype(np.float64) @ W.astype(np.float64).T
+        errs.append(np.linalg.norm(H.host(Y) - exact) / np.linalg.norm(exact))
+    assert errs[1] < errs[0], errs

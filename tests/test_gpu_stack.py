@@ -1,26 +1,33 @@
 """64-step iterative denoising of a 4-layer LLaDA-8B-shaped stack.
 
 Hidden 4096, FFN 12288, 32 heads; 1024 positions, the last 256 generated,
-4 unmasked per step; every linear is SGAT W4A4 (the O projection with TAC,
-128 x 128 per head; the gate+up projection with silu(gate) * up in its
-epilogue); RMSNorm, RoPE and attention are glue. At steps
-0, 1, 31 and 63 every linear's activation codes, scales and E4M3 bytes are
-compared bit-exactly with the oracle's quantisation of the GPU's own input
-(teacher forcing; TAC within tolerance); at step 0 every linear's outputs
-are compared with the oracle's dequantised integer GEMM on the GPU's weight
-codes. Every step, the stack's output is compared with the same stack on
-16-bit GEMMs. With random-init weights the drift is large (each linear has
-~28% relative error: the gates drop 1/32 of the transformed energy, 4-bit
-codes add ~21%), so the bound only asks that it stays finite and that the
-output stays positively correlated with the 16-bit one (drift < sqrt 2).
+4 unmasked per step; every linear is SGAT W4A4 (the gate+up projection with
+silu(gate) * up in its epilogue), attention is the quantised softmax-value
+product with TAC (128 x 128 per head) in its epilogue, and RMSNorm, RoPE and
+the residuals run in the library's glue kernels. At steps 0, 1, 31 and 63:
+
+- every linear's activation codes, scales and E4M3 bytes are compared
+  bit-exactly with the oracle's quantisation of the GPU's own input (teacher
+  forcing); at step 0 every linear's outputs are compared with the oracle's
+  dequantised integer GEMM on the GPU's weight codes;
+- every layer's attention output equals a standalone call with the debug
+  outputs on the same roped QKV, whose P codes, integer sums and TAC output
+  match the oracle for two heads (teacher-forced on the GPU's codes).
+
+Every step, the stack's output is compared with the same stack on 16-bit
+GEMMs and unquantised attention. With random-init weights the drift is
+large (each linear has ~28% relative error: the gates drop 1/32 of the
+transformed energy, 4-bit codes add ~21%), so the bound only asks that it
+stays finite and that the output stays positively correlated with the
+16-bit one (drift < sqrt 2).
 """
 
 import numpy as np
 import pytest
 import torch
 
+from oracle import attention as oatt
 from oracle import sgat as osg
-from oracle import tac as otac
 from tests import helpers as H
 
 pytestmark = pytest.mark.gpu
@@ -41,16 +48,44 @@ def test_denoise_stack(abi):
     checked = []
     state = {}
 
+    def check_attention(li, att, qkv, Y):
+        L, C, D = cfg.seq, cfg.hidden, 128
+        Z = torch.empty_like(Y)
+        codes = torch.zeros(cfg.heads, L, L, dtype=torch.uint8, device="cuda")
+        lsum = torch.zeros(cfg.heads, L, dtype=torch.float32, device="cuda")
+        acc = torch.zeros(cfg.heads, L, D, dtype=torch.int32, device="cuda")
+        att.run(qkv, Z, dbg_codes=codes, dbg_l=lsum, dbg_acc=acc)
+        torch.cuda.synchronize()
+        assert torch.equal(Z, Y), f"layer {li}: attention output differs from the standalone call"
+        qn = qkv.float().cpu().numpy()
+        vq, t = oatt.v_codes(qn[:, 2 * C:])
+        gc, gl, ga = codes.cpu().numpy().astype(np.int32), lsum.cpu().numpy(), acc.cpu().numpy()
+        for h in (0, cfg.heads - 1):
+            ch = slice(h * D, (h + 1) * D)
+            S = oatt.scores(qn[:, ch], qn[:, C + h * D:C + (h + 1) * D], D)
+            oc, ol = oatt.p_codes(S)
+            diff = gc[h] != oc
+            if diff.any():
+                e255 = 255.0 * np.exp(S - S.max(axis=1, keepdims=True))
+                near = np.abs(e255 - np.floor(e255) - 0.5) < 1e-3
+                assert np.all(np.abs(gc[h] - oc)[diff] == 1) and np.all(near[diff]), f"layer {li} head {h}: P codes"
+            np.testing.assert_allclose(gl[h], ol, rtol=1e-5)
+            ref_acc = osg.int_gemm(gc[h], vq[:, ch].T)
+            assert np.array_equal(ga[h], ref_acc), f"layer {li} head {h}: integer sums"
+            zhat = ref_acc / (255.0 * gl[h].astype(np.float64)[:, None]) * t[ch].astype(np.float64)
+            ref = zhat @ att.tac.M[h].astype(np.float64).T + att.tac.d[h].astype(np.float64)[None, :]
+            H.assert_tac_close(H.host(Y)[:, ch], ref, "f16")
+
     def hook(li, name, lin, X, Y):
         step = state["step"]
+        if name == "attn":
+            check_attention(li, lin, X, Y)
+            checked.append((step, li, name))
+            return
         xf = lin.sgat
-        Xq, s_a, Xe, zt = H.workspace_views(lin.workspace, cfg.seq, lin.K, lin.tac is not None, X.dtype)
+        Xq, s_a, Xe, _ = H.workspace_views(lin.workspace, cfg.seq, lin.K, False, X.dtype)
         mask = state["mask"][rows]
         Xr = X.float().cpu().numpy()[rows]
-        if lin.tac is not None:
-            z = H.host(zt)[rows]
-            H.assert_tac_close(z, otac.tac_apply(Xr, lin.tac.M, lin.tac.d, lin.tac.g), "f16")
-            Xr = z                                       # teacher forcing on the GPU's TAC output
         codes, s = osg.sgat_quantize_act(Xr, mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, 4)
         g_codes = H.unpack(Xq)[rows]
         assert np.array_equal(g_codes, codes), f"step {step} layer {li} {name}: codes"
@@ -76,7 +111,7 @@ def test_denoise_stack(abi):
         out_f = st.forward(tok, mask, quantised=False).float()
         abi.check_status()
         drift.append(float(torch.linalg.norm(out_q - out_f) / torch.linalg.norm(out_f)))
-    assert len(checked) == len(CHECK_STEPS) * cfg.layers * 4
+    assert len(checked) == len(CHECK_STEPS) * cfg.layers * 5
     assert int(st.state(cfg.steps)[1].sum()) == 0                 # every position unmasked at the end
     d = np.array(drift)
     print(f"drift vs 16-bit stack: first {d[0]:.4f} max {d.max():.4f} last {d[-1]:.4f}")
