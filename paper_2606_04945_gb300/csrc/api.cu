@@ -166,11 +166,6 @@ int check_w8a8(const uint8_t* Xe, const float* s_a, const uint8_t* We, const flo
 
 int report_error(int code, const char* msg) { return fail(code, "%s", msg); }
 
-unsigned* device_status_word() {
-    int rc = STARQ_OK;
-    return status_ptr(&rc);
-}
-
 namespace {
 // Failure-detection self-test: one thread waits on an mbarrier that nothing
 // ever arrives on, through the same bounded wait as every pipeline wait of

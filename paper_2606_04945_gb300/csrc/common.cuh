@@ -45,7 +45,6 @@ struct QuantArgs {
     // E4M3 of -z (the zero-point columns of the augmented contraction)
     int asym = 0;
     int32_t* z = nullptr;
-    unsigned* status = nullptr;   // device status word (bounded waits); the launcher fills it
 };
 cudaError_t launch_sgat_quant(const QuantArgs& a, cudaStream_t stream);
 
@@ -100,7 +99,6 @@ cudaError_t launch_tac(const TacArgs& a, cudaStream_t stream);
 cudaError_t launch_tac_prepare(const float* M, int C, int g, int z_dtype, void* Mp, cudaStream_t stream);
 
 int num_sms();  // SM count of the current device (cached per device)
-unsigned* device_status_word();  // status word of the current device, or nullptr
 // Glue (glue.cu): residual add + RMSNorm, rotary position embedding.
 cudaError_t launch_add_rmsnorm(const void* X, const void* R, int dtype, int L, int K, const float* w, float eps,
                                void* h_out, void* Y, cudaStream_t stream);

@@ -410,529 +410,341 @@ template <> struct To<__half> { static __device__ __forceinline__ float f(__half
 template <> struct To<__nv_bfloat16> { static __device__ __forceinline__ float f(__nv_bfloat16 h) { return __bfloat162float(h); } };
 template <> struct To<float> { static __device__ __forceinline__ float f(float h) { return h; } };
 
-__device__ __forceinline__ int swz(int row, int col) {      // float index in a 32 x 32 slice
-    return row * 32 + ((((col >> 2) ^ (row & 7))) << 2) + (col & 3);
-}
-
-// Packed float32 pairs (sm_100 family): each half rounds like the scalar
-// operation (PTX add / sub / mul with the explicit .rn rounding). A packed
-// product that feeds a packed sum can still be fused by the compiler, so no
-// f2mul result is ever added by f2add / f2sub (see quant2).
-__device__ __forceinline__ float2 f2op_add(float2 a, float2 b) {
-    float2 d;
-    asm("{\n\t.reg .b64 A, B, D;\n\tmov.b64 A, {%2, %3};\n\tmov.b64 B, {%4, %5};\n\t"
-        "add.rn.f32x2 D, A, B;\n\tmov.b64 {%0, %1}, D;\n\t}"
-        : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-    return d;
-}
-__device__ __forceinline__ float2 f2op_sub(float2 a, float2 b) {
-    float2 d;
-    asm("{\n\t.reg .b64 A, B, D;\n\tmov.b64 A, {%2, %3};\n\tmov.b64 B, {%4, %5};\n\t"
-        "sub.rn.f32x2 D, A, B;\n\tmov.b64 {%0, %1}, D;\n\t}"
-        : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-    return d;
-}
-__device__ __forceinline__ float2 f2op_mul(float2 a, float2 b) {
-    float2 d;
-    asm("{\n\t.reg .b64 A, B, D;\n\tmov.b64 A, {%2, %3};\n\tmov.b64 B, {%4, %5};\n\t"
-        "mul.rn.f32x2 D, A, B;\n\tmov.b64 {%0, %1}, D;\n\t}"
-        : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-    return d;
-}
-__device__ __forceinline__ float2 f2add(float2 a, float2 b) { return f2op_add(a, b); }
-__device__ __forceinline__ float2 f2sub(float2 a, float2 b) { return f2op_sub(a, b); }
-__device__ __forceinline__ float2 f2mul(float2 a, float2 b) { return f2op_mul(a, b); }
-__device__ __forceinline__ void bfly2(float2& a, float2& b) {
-    const float2 x = a, y = b;
-    a = f2add(x, y);
-    b = f2sub(x, y);
-}
-
-// In-register butterfly stages of 32 values held as 16 pairs (value e in
-// u[e / 2], .x for even e): value distances s = s_lo .. s_end / 2; s = 1
-// pairs the two halves of each float2 (scalar), s >= 2 pairs float2 i with
-// i + s / 2 (packed).
-__device__ __forceinline__ void reg_stages16(float2 (&u)[16], int s_lo, int s_end) {
-    if (s_lo <= 1 && 1 < s_end) {
-        #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            const float a = u[i].x, b = u[i].y;
-            u[i] = make_float2(__fadd_rn(a, b), __fsub_rn(a, b));
-        }
-    }
-    #pragma unroll
-    for (int s = 2; s < 32; s <<= 1) {
-        if (s >= s_lo && s < s_end) {
-            #pragma unroll
-            for (int i = 0; i < 16; ++i)
-                if ((i & (s / 2)) == 0) bfly2(u[i], u[i + s / 2]);
-        }
-    }
-}
-
-// Codes of a pair: q = rne(fl(v * r)). The product rounds once (never a
-// fused multiply-add, which would round the exact product and break ties
-// differently); adding M = 1.5 * 2^23 then rounds it to an integer in one
-// step (the floats of [2^23, 2^24) are the integers, ties to even). t holds
-// M + q, whose low byte is q in two's complement; fl(t - M) is q as a float
-// (+0 for zero).
-// The product is two scalar round-to-nearest multiplies: a packed multiply
-// followed by the packed add is fused into one packed FMA by the compiler
-// even when both are written as .rn PTX, and an FMA rounds the exact product
-// (a value whose product rounds onto a half-integer would then round the
-// other way; on the LLaDA weights 6 of 50 M codes).
-constexpr float ROUND_M = 12582912.0f;
-__device__ __forceinline__ void quant2(float2 v, float2 rr, float2& q, float2& t) {
-    const float2 p = make_float2(__fmul_rn(v.x, rr.x), __fmul_rn(v.y, rr.y));
-    t = f2add(p, make_float2(ROUND_M, ROUND_M));
-    q = f2add(t, make_float2(-ROUND_M, -ROUND_M));
-}
-
-// Eight codes in four pairs (q float values, t biased forms) -> packed
-// nibbles (code k in bits 4k .. 4k + 3) and their eight E4M3 bytes. The
-// nibbles come from the low bytes of the biased forms: the even codes' bytes
-// and the odd codes' bytes are gathered by byte permutes, then the low
-// nibbles of the even ones and the odd ones shifted up are merged.
-__device__ __forceinline__ void pack_codes8(const float2 (&q)[4], const float2 (&t)[4], uint32_t& nib, uint2& e4) {
-    const uint32_t ev = prmt(prmt(__float_as_uint(t[0].x), __float_as_uint(t[1].x), 0x40u),
-                             prmt(__float_as_uint(t[2].x), __float_as_uint(t[3].x), 0x40u), 0x5410u);
-    const uint32_t od = prmt(prmt(__float_as_uint(t[0].y), __float_as_uint(t[1].y), 0x40u),
-                             prmt(__float_as_uint(t[2].y), __float_as_uint(t[3].y), 0x40u), 0x5410u);
-    nib = (ev & 0x0F0F0F0Fu) | ((od << 4) & 0xF0F0F0F0u);
-    uint16_t h[4];
-    #pragma unroll
-    for (int k = 0; k < 4; ++k)          // upper byte from the first operand
-        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(h[k]) : "f"(q[k].y), "f"(q[k].x));
-    e4.x = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
-    e4.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
-}
-__device__ __forceinline__ int code_of(float t) { return (int)(__float_as_uint(t) - 0x4B400000u); }
-
-// Staging of one row's slice of 1024 elements for layout A. The row arrives
-// by TMA in 128-byte lines with the 128-byte swizzle (16-byte unit u of line
-// i at unit u ^ (i & 7)); lane l's 32 elements are 64 bytes (16-bit input,
-// half of line l / 2) or 128 bytes (float, line l), and the swizzle spreads
-// each quarter-warp's 16-byte reads over all banks.
-template <typename Tin> struct Stage;
-__device__ __forceinline__ float2 to_f2(__half2 h) { return __half22float2(h); }
-__device__ __forceinline__ float2 to_f2(__nv_bfloat162 h) { return __bfloat1622float2(h); }
-template <typename T2>
-struct Stage16 {
-    static __device__ __forceinline__ void load(uint32_t chunk, int lane, float2 (&u)[16]) {
-        const uint32_t line = chunk + (uint32_t)(lane >> 1) * 128u;
-        #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const uint32_t unit = (uint32_t)(4 * (lane & 1) + q) ^ (uint32_t)((lane >> 1) & 7);
-            const uint4 w = ld_shared_v4(line + (unit << 4));
-            const T2* h = reinterpret_cast<const T2*>(&w);
-            #pragma unroll
-            for (int k = 0; k < 4; ++k) u[4 * q + k] = to_f2(h[k]);
-        }
-    }
-};
-template <> struct Stage<__half> : Stage16<__half2> {};
-template <> struct Stage<__nv_bfloat16> : Stage16<__nv_bfloat162> {};
-template <> struct Stage<float> {
-    static __device__ __forceinline__ void load(uint32_t chunk, int lane, float2 (&u)[16]) {
-        const uint32_t line = chunk + (uint32_t)lane * 128u;
-        #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            const uint4 w = ld_shared_v4(line + ((uint32_t)(q ^ (lane & 7)) << 4));
-            u[2 * q] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
-            u[2 * q + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
-        }
-    }
-};
-
-namespace rowsk {
-constexpr int G = 2;                          // row groups (four warps each) per CTA
-constexpr int THREADS = 128 * G;
-constexpr int SLICES_BYTES = 4 * 1024 * 4;    // the four warps' transpose slices
-constexpr int SMOOTH_RESIDENT_MAX_K = 8192;   // a_m and a_u stay in shared memory up to here
-constexpr int LINES_PER_COPY = 16;            // 2 KB per TMA copy
-constexpr unsigned STATUS_TIMEOUT_QUANT = 1u << 5;
-
-// Dynamic shared memory: [a_m | a_u, K floats each, swizzled like float
-// staging, when resident][per group: two row buffers of K * esize bytes,
-// then the slices][barriers and reductions]; every region 1024-aligned.
-struct Layout {
-    int smooth_bytes, stage_bytes, group_bytes, total;
-    __host__ __device__ Layout(int K, int esize, bool resident) {
-        smooth_bytes = resident ? 2 * K * 4 : 0;
-        stage_bytes = K * esize;
-        group_bytes = 2 * stage_bytes + SLICES_BYTES;
-        total = 1024 + smooth_bytes + G * group_bytes + 256;
-    }
-};
-struct Ctl {
-    uint64_t full[G][2];
-    float red[G][8];
-    int abort[G];
-};
-}  // namespace rowsk
-
 // ---------------------------------------------------------------------------
 // Rows with Hadamard blocks of 1024 elements or more (hb >= 1024, K a
-// multiple of 1024, K <= 4096 NR). Persistent CTAs of G row groups; a group
-// of four warps transforms and quantises one row at a time, in rounds of
-// 4096 elements (four 1024-element chunks, chunk j of a round in warp j),
-// while the next two rows arrive by TMA into the group's two row buffers.
-// The smoothing vectors are copied into shared memory once per CTA (K <=
-// 8192; larger rows read them from global memory, where they stay cached).
+// multiple of 1024, K <= 4096 NR): one CTA of four warps per row, in rounds
+// of 4096 elements (four 1024-element chunks, chunk j of a round in warp j).
+// A warp reads its chunk of x and of the smoothing vector with coalesced
+// 16-byte loads (lane l at 16 l + 512 q) and passes each through its
+// shared slice to take it back in layout A (16 KB of shared memory per CTA,
+// so registers, not shared memory, bound the CTAs per SM).
 //
 //   layout A  lane l holds elements 32 l .. 32 l + 31 of its warp's chunk:
 //             stages h = 1 .. 16 are between registers;
 //   layout B  lane l holds elements l + 32 i (i = 0 .. 31) of the chunk,
-//             after a transpose through the warp's shared slice: stages
+//             after a transpose through the chunk's shared slice: stages
 //             h = 32 .. 512 are between registers;
 //   layout C  after the round's four chunks are in shared memory, lane l of
 //             warp w holds elements j 1024 + 256 w + 8 l .. + 7 of every
 //             chunk j: stages h = 1024, 2048 are between registers, and the
 //             eight consecutive codes per chunk pack into one 32-bit word.
-// Butterflies, the smoothing multiply and the quantiser's multiply work on
-// register pairs with the packed f32x2 instructions (each half rounds like
-// the scalar operation). A slice holds its 32 x 32 floats with 16-byte
-// column groups XOR-swizzled by the row (row & 7), so the row-wise 16-byte
-// accesses (layouts A and C) and the column-wise 4-byte accesses (layout B)
-// are free of bank conflicts. Every wait is bounded.
+// Butterflies on pairs of registers use the packed f32x2 add and subtract
+// (each half rounds like the scalar operation). The shared slice of a chunk
+// holds its 32 x 32 floats with 16-byte column groups XOR-swizzled by the
+// row (row & 7), so the row-wise 16-byte accesses (layouts A and C) and the
+// column-wise 4-byte accesses (layout B) are all free of bank conflicts.
 // ---------------------------------------------------------------------------
-template <int NR, typename Tin, bool ASYM, bool RESIDENT>
-__global__ void __launch_bounds__(rowsk::THREADS, NR == 1 ? 2 : 1)
-sgat_quant_rows_kernel(QuantArgs a, const __grid_constant__ CUtensorMap tmx) {
-    using namespace rowsk;
-    extern __shared__ uint8_t qrow_smem[];
-    const int K = a.K;
-    const Layout lay(K, (int)sizeof(Tin), RESIDENT);
-    const uint32_t raw = smem_addr(qrow_smem);
-    const uint32_t base = (raw + 1023u) & ~1023u;
-    uint8_t* const gbase = qrow_smem + (base - raw);
-    const int lane = threadIdx.x & 31;
-    const int g = threadIdx.x >> 7;                    // row group
-    const int warp = (threadIdx.x >> 5) & 3;           // warp within the group
-    const int gtid = threadIdx.x & 127;
-    const uint32_t smooth = base;
-    const uint32_t gstage = base + lay.smooth_bytes + g * lay.group_bytes;
-    float* const slices = reinterpret_cast<float*>(gbase + lay.smooth_bytes + g * lay.group_bytes +
-                                                   2 * lay.stage_bytes);
-    float* const slice = slices + warp * 1024;
-    Ctl* const ctl = reinterpret_cast<Ctl*>(gbase + lay.smooth_bytes + G * lay.group_bytes);
-    volatile int* abort = &ctl->abort[g];
-    const int copies = lay.stage_bytes / (LINES_PER_COPY * 128);
-    const long long lines_per_row = (long long)lay.stage_bytes / 128;
-    // rows of group g: first = blockIdx.x * G + g, then + gridDim.x * G
-    const int stride = gridDim.x * G;
-    const int first = blockIdx.x * G + g;
+__device__ __forceinline__ int swz(int row, int col) {      // float index in a 32 x 32 slice
+    return row * 32 + ((((col >> 2) ^ (row & 7))) << 2) + (col & 3);
+}
 
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < G; ++i) {
-            mbar_init(smem_addr(&ctl->full[i][0]), 1);
-            mbar_init(smem_addr(&ctl->full[i][1]), 1);
-            ctl->abort[i] = 0;
-        }
-        mbar_fence_init();
+// Two butterflies (a0, b0) and (a1, b1) with one packed add and one packed
+// subtract: a' = a + b, b' = a - b.
+__device__ __forceinline__ void butterfly2(float& a0, float& a1, float& b0, float& b1) {
+    asm("{\n\t.reg .b64 A, B, S, D;\n\t"
+        "mov.b64 A, {%0, %1};\n\t"
+        "mov.b64 B, {%2, %3};\n\t"
+        "add.rn.f32x2 S, A, B;\n\t"
+        "sub.rn.f32x2 D, A, B;\n\t"
+        "mov.b64 {%0, %1}, S;\n\t"
+        "mov.b64 {%2, %3}, D;\n\t}"
+        : "+f"(a0), "+f"(a1), "+f"(b0), "+f"(b1));
+}
+
+// In-register stages of a 32-value array for register distances
+// s = s_lo .. s_end / 2 (s = 1 scalar, s >= 2 on packed pairs).
+__device__ __forceinline__ void reg_stages32(float (&v)[32], int s_lo, int s_end) {
+    if (s_lo <= 1 && 1 < s_end) {
+        #pragma unroll
+        for (int i = 0; i < 32; i += 2) butterfly(v[i], v[i + 1]);
     }
-    __syncthreads();
+    #pragma unroll
+    for (int s = 2; s < 32; s <<= 1) {
+        if (s >= s_lo && s < s_end) {
+            #pragma unroll
+            for (int i = 0; i < 32; i += 2)
+                if ((i & s) == 0) butterfly2(v[i], v[i + 1], v[i + s], v[i + s + 1]);
+        }
+    }
+}
+
+// Codes of two values: q = rne(fl(v * r)). The product is a scalar
+// round-to-nearest multiply (never contracted: a fused multiply-add would
+// round the exact product and break ties differently). Adding M = 1.5 * 2^23
+// then rounds it to an integer in one step (floats in [2^23, 2^24) are the
+// integers, ties to even), fl(t - M) is that integer as a float (+0 for
+// zero), and the low mantissa bits of t are the integer itself.
+__device__ __forceinline__ void quant_pair(float v0, float v1, float r, float& q0, float& q1, int& i0, int& i1) {
+    const float p0 = __fmul_rn(v0, r), p1 = __fmul_rn(v1, r);
+    asm("{\n\t.reg .b64 V, M, T;\n\t"
+        "mov.b64 V, {%4, %5};\n\t"
+        "mov.b64 M, {%6, %6};\n\t"
+        "add.rn.f32x2 T, V, M;\n\t"
+        "sub.rn.f32x2 V, T, M;\n\t"
+        "mov.b64 {%0, %1}, V;\n\t"
+        "mov.b64 {%2, %3}, T;\n\t}"
+        : "=f"(q0), "=f"(q1), "=r"(i0), "=r"(i1) : "f"(p0), "f"(p1), "f"(12582912.0f));
+    i0 -= 0x4B400000;
+    i1 -= 0x4B400000;
+}
+
+// Eight codes -> packed nibbles (code k in bits 4k .. 4k + 3) and their
+// eight E4M3 bytes (byte k = code k); qf are the codes as floats, qi as ints.
+__device__ __forceinline__ void pack_codes8(const float* qf, const int* qi, uint32_t& nib, uint2& e4) {
+    uint32_t w = 0;
+    #pragma unroll
+    for (int k = 6; k >= 0; k -= 2)      // d = c << 8 | sat4(a) << 4 | sat4(b)
+        asm("cvt.pack.sat.s4.s32.b32 %0, %1, %2, %0;" : "+r"(w) : "r"(qi[k + 1]), "r"(qi[k]));
+    nib = w;
+    uint16_t h[4];
+    #pragma unroll
+    for (int k = 0; k < 4; ++k)          // upper byte from the first operand
+        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(h[k]) : "f"(qf[2 * k + 1]), "f"(qf[2 * k]));
+    e4.x = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
+    e4.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
+}
+
+// ASYM: the asymmetric mode (a compile-time copy, so that the symmetric
+// kernel carries none of its reductions)
+template <int NR, typename Tin, bool ASYM>
+__global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
+sgat_quant_rows_kernel(QuantArgs a) {
+    __shared__ __align__(16) float buf[4096];
+    __shared__ float red[8];              // [0, 4) amax or X_max, [4, 8) -X_min (asym)
     grid_dependency_wait();            // launched with programmatic serialisation
     grid_launch_dependents();
-    auto issue = [&](int row, int buf) {             // one thread of the group
-        const uint32_t bar = smem_addr(&ctl->full[g][buf]);
-        mbar_arrive_expect_tx(bar, (uint32_t)lay.stage_bytes);
-        const uint32_t dst = gstage + (uint32_t)(buf * lay.stage_bytes);
-        for (int c = 0; c < copies; ++c)
-            tma_load_2d(dst + c * LINES_PER_COPY * 128, &tmx, 0,
-                        (int)(row * lines_per_row + c * LINES_PER_COPY), bar);
-    };
-    if (gtid == 0) {
-        if (first < a.L) issue(first, 0);
-        if (first + stride < a.L) issue(first + stride, 1);
-    }
-    if (RESIDENT) {
-        // a_m then a_u (NULL: ones), 4 floats per thread and step, stored in
-        // the swizzled float staging layout of their lines
-        const int n4 = K / 4;
-        for (int f = threadIdx.x; f < 2 * n4; f += THREADS) {
-            const int s = f >= n4, i = f - s * n4;
-            const float* src = s ? a.a_u : a.a_m;
-            const float4 v = src != nullptr ? __ldg(reinterpret_cast<const float4*>(src) + i)
-                                            : make_float4(1.f, 1.f, 1.f, 1.f);
-            const int line = s * (K / 32) + i / 8, unit = (i & 7) ^ (line & 7);
-            st_shared_v4(smooth + line * 128 + unit * 16, __float_as_uint(v.x), __float_as_uint(v.y),
-                         __float_as_uint(v.z), __float_as_uint(v.w));
-        }
-        __syncthreads();
-    }
-    auto group_sync = [&]() { asm volatile("bar.sync %0, 128;" :: "r"(1 + g) : "memory"); };
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int row = blockIdx.x;
+    const int K = a.K;
+    const bool masked = a.mask != nullptr && a.mask[row] != 0;
+    const float* sm = masked ? a.a_m : a.a_u;
+    const int own_lo = masked ? a.d_sh : a.d_sh + a.d_m;
+    const int own_hi = masked ? a.d_sh + a.d_m : K;
+    const Tin* X = static_cast<const Tin*>(a.X) + (size_t)row * K;
+    float* slice = buf + warp * 1024;
 
-    const float qmax = (float)a.qmax;
-    int it = 0;
-    bool ok = true;
-    for (int row = first; row < a.L; row += stride, ++it) {
-        const int buf = it & 1;
-        const uint32_t stage = gstage + (uint32_t)(buf * lay.stage_bytes);
-        // a wait that runs out marks the group; every thread of the group
-        // sees the mark after the round's first group barrier and leaves
-        if (!mbar_wait_bounded(smem_addr(&ctl->full[g][buf]), (uint32_t)((it >> 1) & 1), abort)) *abort = 1;
-        const bool masked = a.mask != nullptr && a.mask[row] != 0;
-        const float* gsm = masked ? a.a_m : a.a_u;             // global copy (RESIDENT = false)
-        const bool smooth_on = RESIDENT ? (masked ? a.a_m : a.a_u) != nullptr : gsm != nullptr;
-        const int own_lo = masked ? a.d_sh : a.d_sh + a.d_m;
-        const int own_hi = masked ? a.d_sh + a.d_m : K;
-
-        float2 v[NR][16];                 // layout C: v[R][4 j + k] = elements e0 + 2k, e0 + 2k + 1 of chunk j
-        float amax = 0.f, nmin = 0.f;     // asym: X_max and -X_min
-        #pragma unroll
-        for (int R = 0; R < NR; ++R) {
-            const int rbase = R * 4096;
-            const int nch = min(4, (K - rbase) >> 10);        // chunks in this round (>= 1)
-            if (warp < nch) {
-                const int c0 = rbase + warp * 1024;             // first element of the chunk
-                float2 u[16];
-                Stage<Tin>::load(stage + (uint32_t)(c0 * (int)sizeof(Tin)), lane, u);
-                if (smooth_on) {
-                    if (RESIDENT) {
-                        const uint32_t sl = smooth + (uint32_t)(((masked ? 0 : K) + c0) * 4 + lane * 128);
-                        #pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            const uint4 w = ld_shared_v4(sl + ((uint32_t)(q ^ (lane & 7)) << 4));
-                            u[2 * q] = f2mul(u[2 * q], make_float2(__uint_as_float(w.x), __uint_as_float(w.y)));
-                            u[2 * q + 1] = f2mul(u[2 * q + 1], make_float2(__uint_as_float(w.z), __uint_as_float(w.w)));
-                        }
-                    } else {
-                        const float4* s4 = reinterpret_cast<const float4*>(gsm + c0 + 32 * lane);
-                        #pragma unroll
-                        for (int q = 0; q < 8; ++q) {
-                            const float4 w = __ldg(s4 + q);
-                            u[2 * q] = f2mul(u[2 * q], make_float2(w.x, w.y));
-                            u[2 * q + 1] = f2mul(u[2 * q + 1], make_float2(w.z, w.w));
-                        }
-                    }
-                }
-                reg_stages16(u, 1, 32);                          // h = 1 .. 16
+    float v[NR][32];                      // layout C: v[R][8 j + k]
+    float amax = 0.f, nmin = 0.f;         // asym: X_max and -X_min
+    #pragma unroll
+    for (int R = 0; R < NR; ++R) {
+        const int base = R * 4096;
+        const int nch = min(4, (K - base) >> 10);        // chunks in this round (>= 1)
+        float u[32];
+        if (warp < nch) {
+            // coalesced loads (lane l: 16 bytes at 16 l + 512 q); x and then
+            // the smoothing vector pass through the warp's slice and come
+            // back in layout A
+            const int c0 = base + warp * 1024;                   // first element of the chunk
+            float4 sr[8];
+            if (sizeof(Tin) == 2) {
+                uint4 xr[4];
                 #pragma unroll
-                for (int q = 0; q < 8; ++q)                      // layout A -> slice
-                    *reinterpret_cast<float4*>(slice + swz(lane, 4 * q)) =
-                        make_float4(u[2 * q].x, u[2 * q].y, u[2 * q + 1].x, u[2 * q + 1].y);
+                for (int q = 0; q < 4; ++q) xr[q] = __ldg(reinterpret_cast<const uint4*>(X + c0) + lane + 32 * q);
+                // 16-bit staging: 32 rows of 64 bytes, 16-byte group g of row R at g ^ ((R >> 1) & 3)
+                uint8_t* st8 = reinterpret_cast<uint8_t*>(slice);
+                #pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int R = (lane >> 2) + 8 * q, g = lane & 3;
+                    *reinterpret_cast<uint4*>(st8 + R * 64 + 16 * (g ^ ((R >> 1) & 3))) = xr[q];
+                }
+                if (sm != nullptr) {
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
+                }
                 __syncwarp();
                 #pragma unroll
-                for (int i = 0; i < 16; ++i)                     // layout B: u[i] = rows 2i, 2i + 1
-                    u[i] = make_float2(slice[swz(2 * i, lane)], slice[swz(2 * i + 1, lane)]);
-                reg_stages16(u, 1, a.hb / 32);                   // h = 32 .. min(hb, 1024) / 2
+                for (int g = 0; g < 4; ++g) {
+                    const uint4 w = *reinterpret_cast<const uint4*>(st8 + lane * 64 + 16 * (g ^ ((lane >> 1) & 3)));
+                    const Tin* h = reinterpret_cast<const Tin*>(&w);
+                    #pragma unroll
+                    for (int k = 0; k < 8; ++k) u[8 * g + k] = To<Tin>::f(h[k]);
+                }
+            } else {
+                float4 xr[8];
                 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    slice[swz(2 * i, lane)] = u[i].x;
-                    slice[swz(2 * i + 1, lane)] = u[i].y;
+                for (int q = 0; q < 8; ++q) xr[q] = __ldg(reinterpret_cast<const float4*>(X + c0) + lane + 32 * q);
+                #pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = xr[q];
+                if (sm != nullptr) {
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
+                }
+                __syncwarp();
+                #pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float4 w = *reinterpret_cast<const float4*>(slice + swz(lane, 4 * q));
+                    u[4 * q] = w.x; u[4 * q + 1] = w.y; u[4 * q + 2] = w.z; u[4 * q + 3] = w.w;
                 }
             }
-            group_sync();
-            if (*abort) { ok = false; break; }
-            // the row buffer has been read in full: it takes the row after next
-            if (R == NR - 1 && gtid == 0 && row + 2 * stride < a.L) {
-                fence_proxy_async_smem();
-                issue(row + 2 * stride, buf);
+            if (sm != nullptr) {
+                __syncwarp();                                    // x has left the slice
+                #pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
+                __syncwarp();
+                #pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float4 w = *reinterpret_cast<const float4*>(slice + swz(lane, 4 * q));
+                    u[4 * q] = __fmul_rn(u[4 * q], w.x);
+                    u[4 * q + 1] = __fmul_rn(u[4 * q + 1], w.y);
+                    u[4 * q + 2] = __fmul_rn(u[4 * q + 2], w.z);
+                    u[4 * q + 3] = __fmul_rn(u[4 * q + 3], w.w);
+                }
             }
+            __syncwarp();
+            reg_stages32(u, 1, 32);                              // h = 1 .. 16
             #pragma unroll
-            for (int j = 0; j < 4; ++j) {                        // layout C
-                if (j < nch) {
-                    const int r = warp * 8 + (lane >> 2), c = (lane & 3) * 8;
-                    const float4 p0 = *reinterpret_cast<const float4*>(slices + j * 1024 + swz(r, c));
-                    const float4 p1 = *reinterpret_cast<const float4*>(slices + j * 1024 + swz(r, c + 4));
-                    v[R][4 * j] = make_float2(p0.x, p0.y);
-                    v[R][4 * j + 1] = make_float2(p0.z, p0.w);
-                    v[R][4 * j + 2] = make_float2(p1.x, p1.y);
-                    v[R][4 * j + 3] = make_float2(p1.z, p1.w);
-                } else {
-                    #pragma unroll
-                    for (int k = 0; k < 4; ++k) v[R][4 * j + k] = make_float2(0.f, 0.f);
-                }
-            }
-            if (NR > 1) group_sync();                            // the next round reuses the slices
-            if (a.hb > 1024) {                                   // h = 1024: chunks j, j ^ 1
-                #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    bfly2(v[R][k], v[R][4 + k]);
-                    bfly2(v[R][8 + k], v[R][12 + k]);
-                }
-            }
-            if (a.hb > 2048) {                                   // h = 2048: chunks j, j ^ 2
-                #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    bfly2(v[R][k], v[R][8 + k]);
-                    bfly2(v[R][4 + k], v[R][12 + k]);
-                }
-            }
+            for (int q = 0; q < 8; ++q)                          // layout A -> slice
+                *reinterpret_cast<float4*>(slice + swz(lane, 4 * q)) =
+                    make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
+            __syncwarp();
             #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int e0 = rbase + j * 1024 + warp * 256 + 8 * lane;    // first element of the group
-                if (j >= nch) continue;
-                const bool all_keep = (e0 + 8 <= a.d_sh) || (e0 >= own_lo && e0 + 8 <= own_hi);
-                if (!all_keep) {
-                    #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        const int e = e0 + k;
-                        if (!(e < a.d_sh || (e >= own_lo && e < own_hi))) {
-                            if (k & 1) v[R][4 * j + k / 2].y = 0.f;
-                            else v[R][4 * j + k / 2].x = 0.f;
-                        }
-                    }
-                }
-                if (a.post_scale != 1.f) {
-                    #pragma unroll
-                    for (int k = 0; k < 4; ++k) v[R][4 * j + k] = f2mul(v[R][4 * j + k], make_float2(a.post_scale, a.post_scale));
-                }
-                if (ASYM) {
-                    #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const float2 w = v[R][4 * j + k];
-                        amax = fmaxf(amax, fmaxf(w.x, w.y));
-                        nmin = fmaxf(nmin, fmaxf(-w.x, -w.y));
-                    }
-                } else {
-                    #pragma unroll
-                    for (int k = 0; k < 4; ++k)
-                        amax = fmaxf(amax, fmaxf(fabsf(v[R][4 * j + k].x), fabsf(v[R][4 * j + k].y)));
-                }
-                if (a.v_dbg != nullptr) {
-                    float4* d4 = reinterpret_cast<float4*>(a.v_dbg + (size_t)row * K + e0);
-                    d4[0] = make_float4(v[R][4 * j].x, v[R][4 * j].y, v[R][4 * j + 1].x, v[R][4 * j + 1].y);
-                    d4[1] = make_float4(v[R][4 * j + 2].x, v[R][4 * j + 2].y, v[R][4 * j + 3].x, v[R][4 * j + 3].y);
-                }
-            }
+            for (int i = 0; i < 32; ++i) u[i] = slice[swz(i, lane)];   // layout B
+            reg_stages32(u, 1, a.hb / 32);                       // h = 32 .. min(hb, 1024) / 2
+            #pragma unroll
+            for (int i = 0; i < 32; ++i) slice[swz(i, lane)] = u[i];
         }
-        if (!ok) break;
+        __syncthreads();
         #pragma unroll
-        for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
-        if (ASYM) {
-            #pragma unroll
-            for (int m = 16; m > 0; m >>= 1) nmin = fmaxf(nmin, __shfl_xor_sync(0xffffffffu, nmin, m));
-        }
-        if (lane == 0) {
-            ctl->red[g][warp] = amax;
-            if (ASYM) ctl->red[g][4 + warp] = nmin;
-        }
-        group_sync();
-        amax = fmaxf(fmaxf(ctl->red[g][0], ctl->red[g][1]), fmaxf(ctl->red[g][2], ctl->red[g][3]));
-        if (ASYM) nmin = fmaxf(fmaxf(ctl->red[g][4], ctl->red[g][5]), fmaxf(ctl->red[g][6], ctl->red[g][7]));
-
-        const float range = ASYM ? __fadd_rn(amax, nmin) : amax;     // X_max - X_min, or amax
-        const bool nz = range > 0.f;
-        const float s = nz ? __fdiv_rn(range, qmax) : 0.f;
-        const float r = nz ? __fdiv_rn(qmax, range) : 0.f;
-        const float2 rr = make_float2(r, r);
-        const int zp = ASYM ? min(max(__float2int_rn(__fmul_rn(nmin, r)), 0), a.qmax) : 0;
-        if (gtid == 0) {
-            a.s[row] = s;
-            if (ASYM) a.z[row] = zp;
-        }
-        if (ASYM && a.Xe != nullptr && gtid < 8)
-            store_zero_point_columns(a.Xe + (size_t)row * (K + 128) + K, zp, gtid);
-        #pragma unroll
-        for (int R = 0; R < NR; ++R) {
-            const int rbase = R * 4096;
-            const int nch = min(4, (K - rbase) >> 10);
-            #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                if (j >= nch) continue;
-                const int e0 = rbase + j * 1024 + warp * 256 + 8 * lane;
-                float2 qf[4], qt[4];
+        for (int j = 0; j < 4; ++j) {                            // layout C
+            if (j < nch) {
+                const int r = warp * 8 + (lane >> 2), c = (lane & 3) * 8;
+                const float4 p0 = *reinterpret_cast<const float4*>(buf + j * 1024 + swz(r, c));
+                const float4 p1 = *reinterpret_cast<const float4*>(buf + j * 1024 + swz(r, c + 4));
+                v[R][8 * j] = p0.x; v[R][8 * j + 1] = p0.y; v[R][8 * j + 2] = p0.z; v[R][8 * j + 3] = p0.w;
+                v[R][8 * j + 4] = p1.x; v[R][8 * j + 5] = p1.y; v[R][8 * j + 6] = p1.z; v[R][8 * j + 7] = p1.w;
+            } else {
                 #pragma unroll
-                for (int k = 0; k < 4; ++k) quant2(v[R][4 * j + k], rr, qf[k], qt[k]);
-                if (ASYM || a.qmax > 15) {
-                    int qi[8];
-                    #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        qi[2 * k] = code_of(qt[k].x);
-                        qi[2 * k + 1] = code_of(qt[k].y);
-                    }
-                    if (ASYM) {          // codes in [0, qmax]: unsigned nibbles and E4M3 bytes
-                        int q[8];
-                        #pragma unroll
-                        for (int k = 0; k < 8; ++k) q[k] = min(max(qi[k] + zp, 0), a.qmax);
-                        *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = pack8(q);
-                        if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * (K + 128) + e0) = e4m3_of8(q);
-                    } else {             // 8-bit codes: bytes and their E4M3 split
-                        uint2 bytes, eh, el;
-                        split_codes8(qi, bytes, eh, el);
-                        *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + e0) = bytes;
-                        if (a.Xe != nullptr) {
-                            *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + e0) = eh;
-                            *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + e0) = el;
-                        }
-                    }
-                    continue;
+                for (int k = 0; k < 8; ++k) v[R][8 * j + k] = 0.f;
+            }
+        }
+        if (NR > 1) __syncthreads();                             // the next round reuses buf
+        if (a.hb > 1024) {                                       // h = 1024: chunks j, j ^ 1
+            #pragma unroll
+            for (int k = 0; k < 8; k += 2) {
+                butterfly2(v[R][k], v[R][k + 1], v[R][8 + k], v[R][9 + k]);
+                butterfly2(v[R][16 + k], v[R][17 + k], v[R][24 + k], v[R][25 + k]);
+            }
+        }
+        if (a.hb > 2048) {                                       // h = 2048: chunks j, j ^ 2
+            #pragma unroll
+            for (int k = 0; k < 8; k += 2) {
+                butterfly2(v[R][k], v[R][k + 1], v[R][16 + k], v[R][17 + k]);
+                butterfly2(v[R][8 + k], v[R][9 + k], v[R][24 + k], v[R][25 + k]);
+            }
+        }
+        #pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int e0 = base + j * 1024 + warp * 256 + 8 * lane;    // first element of the group
+            if (j >= nch) continue;
+            const bool all_keep = (e0 + 8 <= a.d_sh) || (e0 >= own_lo && e0 + 8 <= own_hi);
+            if (!all_keep) {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const int e = e0 + k;
+                    if (!(e < a.d_sh || (e >= own_lo && e < own_hi))) v[R][8 * j + k] = 0.f;
                 }
-                uint32_t nib;
-                uint2 e4;
-                pack_codes8(qf, qt, nib, e4);
-                if (a.Xq != nullptr) *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = nib;
-                if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * K + e0) = e4;
+            }
+            if (a.post_scale != 1.f) {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) v[R][8 * j + k] = __fmul_rn(v[R][8 * j + k], a.post_scale);
+            }
+            if (ASYM) {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    amax = fmaxf(amax, v[R][8 * j + k]);
+                    nmin = fmaxf(nmin, -v[R][8 * j + k]);
+                }
+            } else {
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) amax = fmaxf(amax, fabsf(v[R][8 * j + k]));
+            }
+            if (a.v_dbg != nullptr) {
+                float4* d4 = reinterpret_cast<float4*>(a.v_dbg + (size_t)row * K + e0);
+                d4[0] = make_float4(v[R][8 * j], v[R][8 * j + 1], v[R][8 * j + 2], v[R][8 * j + 3]);
+                d4[1] = make_float4(v[R][8 * j + 4], v[R][8 * j + 5], v[R][8 * j + 6], v[R][8 * j + 7]);
             }
         }
     }
-    if (!ok && gtid == 0) {
-        // record the timeout, then give the copies this group issued (the
-        // row that did not arrive, and the one after it) a bounded chance to
-        // land before the CTA's shared memory is released
-        if (a.status != nullptr) atomicOr(a.status, STATUS_TIMEOUT_QUANT);
-        volatile int never = 0;
-        for (int k = it; k < it + 2; ++k)
-            if (first + k * stride < a.L)
-                mbar_wait_bounded(smem_addr(&ctl->full[g][k & 1]), (uint32_t)((k >> 1) & 1), &never);
+    #pragma unroll
+    for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
+    if (ASYM) {
+        #pragma unroll
+        for (int m = 16; m > 0; m >>= 1) nmin = fmaxf(nmin, __shfl_xor_sync(0xffffffffu, nmin, m));
     }
-}
+    if (lane == 0) {
+        red[warp] = amax;
+        if (ASYM) red[4 + warp] = nmin;
+    }
+    __syncthreads();
+    amax = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+    if (ASYM) nmin = fmaxf(fmaxf(red[4], red[5]), fmaxf(red[6], red[7]));
 
-// Tensor map of the rows of X as 128-byte lines ([L * K * esize / 128][128]
-// bytes), boxes of LINES_PER_COPY lines with the 128-byte swizzle.
-bool encode_rows_tmap(CUtensorMap* m, const void* X, size_t bytes) {
-    const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
-    if (fn == nullptr) return false;
-    const cuuint64_t dims[2] = {128, bytes / 128};
-    const cuuint64_t strides[1] = {128};
-    const cuuint32_t box[2] = {128, rowsk::LINES_PER_COPY};
-    const cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(X), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-template <int NR, typename Tin, bool ASYM, bool RES>
-cudaError_t launch_rows_inst(const QuantArgs& a, const CUtensorMap& tm, cudaStream_t stream) {
-    const rowsk::Layout lay(a.K, (int)sizeof(Tin), RES);
-    auto kernel = sgat_quant_rows_kernel<NR, Tin, ASYM, RES>;
-    // CTAs resident per SM at this size (once per device and size)
-    static DeviceCache<int> attr;
-    int done = 0;
-    cudaError_t e = attr.get(&done, [&](int, int* v) {
-        *v = 1;
-        return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-    });
-    if (e != cudaSuccess) return e;
-    int per_sm = 0;
-    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, rowsk::THREADS, lay.total)) != cudaSuccess)
-        return e;
-    if (per_sm < 1) return cudaErrorInvalidConfiguration;
-    const long long groups = ((long long)a.L + rowsk::G - 1) / rowsk::G;
-    const long long slots = (long long)num_sms() * per_sm;
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute at[1] = {pdl_attribute()};
-    cfg.gridDim = dim3((unsigned)(groups < slots ? groups : slots));
-    cfg.blockDim = dim3(rowsk::THREADS);
-    cfg.dynamicSmemBytes = lay.total;
-    cfg.stream = stream;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, a, tm);
+    const float qmax = (float)a.qmax;
+    const float range = ASYM ? __fadd_rn(amax, nmin) : amax;     // X_max - X_min, or amax
+    const bool nz = range > 0.f;
+    const float s = nz ? __fdiv_rn(range, qmax) : 0.f;
+    const float r = nz ? __fdiv_rn(qmax, range) : 0.f;
+    const int zp = ASYM ? min(max(__float2int_rn(__fmul_rn(nmin, r)), 0), a.qmax) : 0;
+    if (threadIdx.x == 0) {
+        a.s[row] = s;
+        if (ASYM) a.z[row] = zp;
+    }
+    if (ASYM && a.Xe != nullptr && threadIdx.x < 8)
+        store_zero_point_columns(a.Xe + (size_t)row * (K + 128) + K, zp, threadIdx.x);
+    #pragma unroll
+    for (int R = 0; R < NR; ++R) {
+        const int base = R * 4096;
+        const int nch = min(4, (K - base) >> 10);
+        #pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            if (j >= nch) continue;
+            const int e0 = base + j * 1024 + warp * 256 + 8 * lane;
+            float qf[8];
+            int qi[8];
+            #pragma unroll
+            for (int k = 0; k < 8; k += 2)
+                quant_pair(v[R][8 * j + k], v[R][8 * j + k + 1], r, qf[k], qf[k + 1], qi[k], qi[k + 1]);
+            if (ASYM) {                  // codes in [0, qmax]: unsigned nibbles and E4M3 bytes
+                int q[8];
+                #pragma unroll
+                for (int k = 0; k < 8; ++k) q[k] = min(max(qi[k] + zp, 0), a.qmax);
+                *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = pack8(q);
+                if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * (K + 128) + e0) = e4m3_of8(q);
+                continue;
+            }
+            if (a.qmax > 15) {           // 8-bit codes: bytes and their E4M3 split
+                uint2 bytes, eh, el;
+                split_codes8(qi, bytes, eh, el);
+                *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + e0) = bytes;
+                if (a.Xe != nullptr) {
+                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + e0) = eh;
+                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + e0) = el;
+                }
+                continue;
+            }
+            uint32_t nib;
+            uint2 e4;
+            pack_codes8(qf, qi, nib, e4);
+            *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = nib;
+            if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * K + e0) = e4;
+        }
+    }
 }
 
 template <int NR, typename Tin>
 cudaError_t launch_rows_nr(const QuantArgs& a, cudaStream_t stream) {
-    CUtensorMap tm;
-    if (!encode_rows_tmap(&tm, a.X, (size_t)a.L * a.K * sizeof(Tin))) return cudaErrorInvalidValue;
-    const bool res = a.K <= rowsk::SMOOTH_RESIDENT_MAX_K;
-    if (a.asym)
-        return res ? launch_rows_inst<NR, Tin, true, true>(a, tm, stream)
-                   : launch_rows_inst<NR, Tin, true, false>(a, tm, stream);
-    return res ? launch_rows_inst<NR, Tin, false, true>(a, tm, stream)
-               : launch_rows_inst<NR, Tin, false, false>(a, tm, stream);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1] = {pdl_attribute()};
+    cfg.gridDim = dim3(a.L);
+    cfg.blockDim = dim3(128);
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return a.asym ? cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, true>, a)
+                  : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, false>, a);
 }
 
 template <typename Tin>
@@ -982,22 +794,17 @@ cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
 
 template <typename Tin>
 cudaError_t launch_typed(const QuantArgs& a, cudaStream_t stream) {
-    // hb >= 1024 and up to 16384 features: the persistent row kernel (when
-    // its shared memory fits); otherwise a warp's chunk is 1024 elements
-    // (hb >= 1024, blocks finish across warps) or 512 elements holding
-    // 512 / hb blocks
-    if (a.hb >= 1024 && a.K % 1024 == 0 && a.K <= 16384 &&
-        rowsk::Layout(a.K, (int)sizeof(Tin), a.K <= rowsk::SMOOTH_RESIDENT_MAX_K).total <= 227 * 1024)
-        return launch_rows<Tin>(a, stream);
+    // hb >= 1024 and up to 16384 features: a CTA per row; otherwise a warp's
+    // chunk is 1024 elements (hb >= 1024, blocks finish across warps) or 512
+    // elements holding 512 / hb blocks
+    if (a.hb >= 1024 && a.K % 1024 == 0 && a.K <= 16384) return launch_rows<Tin>(a, stream);
     return a.hb >= 1024 ? launch_e<32, Tin>(a, stream) : launch_e<16, Tin>(a, stream);
 }
 
 }  // namespace
 
-cudaError_t launch_sgat_quant(const QuantArgs& args, cudaStream_t stream) {
-    if (args.L == 0) return cudaSuccess;
-    QuantArgs a = args;
-    if (a.status == nullptr) a.status = device_status_word();
+cudaError_t launch_sgat_quant(const QuantArgs& a, cudaStream_t stream) {
+    if (a.L == 0) return cudaSuccess;
     switch (a.x_dtype) {
         case STARQ_F16: return launch_typed<__half>(a, stream);
         case STARQ_BF16: return launch_typed<__nv_bfloat16>(a, stream);
