@@ -6,8 +6,9 @@ step -- 1024 tokens (prompt 512 unmasked, 512 generated with a 75% masked
 suffix), hidden 4096, fused QKV 4096 -> 12288 and O 4096 -> 4096, TAC with
 128 x 128 per-head blocks on the attention output, FP16 activations with
 0.5% Student-t(3) channels, random N(0, 0.02) weights prepared once
-(untimed) into folded int4 codes. A step is five kernels: quantise X, QKV
-GEMM, TAC on Z, quantise, O GEMM.
+(untimed) into folded int4 codes. A step is five kernels in two branches
+of one CUDA graph: quantise X -> QKV GEMM, and TAC on Z -> quantise -> O
+GEMM (the projections are independent; the O branch is issued first).
 
 Prints one JSON line (rank 0). Value = SGAT W4A4 linear throughput in TOPS
 (2 L N K integer ops of both GEMMs per step / step time), summed over ranks
@@ -79,7 +80,8 @@ def config_dict(graph):
     return {"workload": "llada8b_attention_projections_step", "tokens": 1024, "hidden": 4096,
             "qkv": "4096->12288", "o": "4096->4096", "tac_block": 128, "hadamard_block": 4096,
             "gates": "d_m = d_u = 128", "mask": "0..639 unmasked, 640..1023 masked",
-            "l2": "flushed between timed steps (256 MiB write)", "cuda_graph": bool(graph)}
+            "l2": "flushed between timed steps (256 MiB write)", "cuda_graph": bool(graph),
+            "streams": "QKV and TAC + O branches forked and joined within the step"}
 
 
 # ---------------------------------------------------------------------------

@@ -10,7 +10,8 @@ two state transforms, optional TAC parameters and a workspace. ``run`` is one ca
 step of a LLaDA-shaped layer: the fused QKV projection of the layer input,
 then TAC on the attention output followed by the O projection (Sec. 3.3: TAC
 sits between the softmax-value product and W_o). ``capture`` records the step
-in a CUDA graph so a replay issues all five kernels with one launch.
+in a CUDA graph so a replay issues all five kernels with one launch; the
+two projections run as two branches of the graph.
 """
 
 import numpy as np
@@ -86,11 +87,22 @@ class AttentionProjections:
         self.mask = _dev(qkv_case.mask, device=device)
         self.Y_qkv = torch.empty(self.L, self.qkv.N, dtype=self.qkv.out_dtype, device=device)
         self.Y_o = torch.empty(self.L, self.o.N, dtype=self.o.out_dtype, device=device)
+        self.side = torch.cuda.Stream(device=device)
         self.graph = None
 
     def step(self, stream=None):
-        self.qkv.run(self.X, self.mask, self.Y_qkv, stream)
-        self.o.run(self.Z, self.mask, self.Y_o, stream)
+        """The two projections are independent, so the O chain (TAC,
+        quantiser, GEMM) runs on a side stream forked from `stream` and
+        joined back at the end: its CUDA-core kernels overlap the QKV
+        quantiser and the gaps between launches. The O chain is issued
+        first, so that TAC starts beside the QKV quantiser. Outputs are
+        identical to running the two projections one after the other."""
+        main = stream if stream is not None else torch.cuda.current_stream()
+        self.side.wait_stream(main)
+        with torch.cuda.stream(self.side):
+            self.o.run(self.Z, self.mask, self.Y_o, self.side)
+        self.qkv.run(self.X, self.mask, self.Y_qkv, main)
+        main.wait_stream(self.side)
 
     def capture(self):
         """Record one step in a CUDA graph (call after a warm-up step)."""
