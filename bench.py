@@ -54,7 +54,8 @@ def parse():
     p.add_argument("--skip-stack", action="store_true", help="leave out the short denoising-stack run")
     p.add_argument("--workload", default="attention_step",
                    choices=["attention_step", "denoise_stack", "tac_calibration", "attention_pv_tac", "w8a8_linear",
-                            "asym_linear", "dense_linear", "dream_block"],
+                            "asym_linear", "dense_linear", "dream_block", "hbm_passes", "llada_mlp",
+                            "single_linear"],
                    help="attention_step: the LLaDA attention projections (default); denoise_stack: the "
                         "64-step 4-layer LLaDA-shaped stack (per-step tokens/s, latency, drift vs fp16); "
                         "tac_calibration: App. C's closed-form TAC calibration on the GPU vs the oracle; "
@@ -62,7 +63,11 @@ def parse():
                         "w8a8_linear: the attention projections at 8 bits (Tab. 5); "
                         "asym_linear: the attention projections with asymmetric A4 activations (Eq. 2-4); "
                         "dense_linear: the attention projections with a dense orthogonal basis (App. B); "
-                        "dream_block: the full Dream-7B-shaped block (GQA 28/4 heads, bf16, 4 x 2048 tokens)")
+                        "dream_block: the full Dream-7B-shaped block (GQA 28/4 heads, bf16, 4 x 2048 tokens); "
+                        "hbm_passes: the quantiser and TAC alone at 8192 tokens (the default line's "
+                        "roofline_hbm_kernels.large, without the rest of the run); "
+                        "llada_mlp: the LLaDA-8B MLP step (gate+up with SwiGLU, down) at mask ratios "
+                        "0.1 / 0.5 / 0.9; single_linear: the 256 x 512 -> 512 linear with TAC (latency)")
     return p.parse_args()
 
 
@@ -320,6 +325,220 @@ def hbm_passes_large(abi, o, flush, torch, L=8192):
                                            "bytes_algorithmic": alg, "gbs": round(alg / ms / 1e6, 1)}
     del Zs
     return out
+
+
+def _dev_np(torch, x, dtype=None):
+    t = torch.from_numpy(__import__("numpy").ascontiguousarray(x))
+    return (t.to(dtype) if dtype is not None else t).cuda()
+
+
+def _graph(torch, body):
+    """Capture body() in a CUDA graph after one eager call on a side stream."""
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        body()
+    torch.cuda.current_stream().wait_stream(s)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        body()
+    return g
+
+
+def run_llada_mlp(args):
+    """The LLaDA-8B MLP at one denoising step (1024 tokens): gate+up 4096 ->
+    2 x 12288 with silu(gate) * up in the GEMM epilogue, then down 12288 ->
+    4096, both SGAT W4A4 with their quantisers, for the mask ratios 0.1, 0.5
+    and 0.9 (semi-autoregressive blocks of 32). The down projection's
+    smoothing comes from the GPU's own SwiGLU output of the same inputs. Each
+    step is one CUDA graph replay after an L2 flush; the fp16 GEMMs of the
+    same shapes (SwiGLU left out) are timed beside it."""
+    import numpy as np
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi, inputs
+    from oracle import sgat as osg
+    torch.cuda.set_device(0)
+    L, Hd, F = 1024, 4096, 12288
+    f16 = torch.float16
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    flush = lambda: flush_buf.zero_()
+    ops = 2 * L * (2 * F) * Hd + 2 * L * Hd * F
+    out = {}
+    t_orc = None
+    for ratio in (0.1, 0.5, 0.9):
+        gu, W_down, mask_np = inputs.llada_mlp(0, ratio)
+        xf = gu.xf
+        X = _dev_np(torch, gu.X, f16)
+        mask = _dev_np(torch, mask_np)
+        perm = abi.swiglu_row_order(F, "cuda")
+        W16 = _dev_np(torch, gu.W, f16)[perm].contiguous()
+        Wq_gu = torch.empty(2 * F, Hd // 2, dtype=torch.uint8, device="cuda")
+        s_gu = torch.empty(2 * F, dtype=torch.float32, device="cuda")
+        abi.sgat_prepare_weight(W16, _dev_np(torch, xf.inv_a_w), xf.hb, Wq_gu, s_gu)
+        We_gu = torch.empty(2 * F, Hd, dtype=torch.uint8, device="cuda")
+        abi.w4_unpack_e4m3(Wq_gu, We_gu)
+        del W16
+        a_m, a_u = _dev_np(torch, xf.a_m), _dev_np(torch, xf.a_u)
+        ws_gu = torch.empty(abi.sgat_linear_workspace_size(L, Hd, False), dtype=torch.uint8, device="cuda")
+        Hbuf = torch.empty(L, F, dtype=f16, device="cuda")
+        abi.sgat_linear_swiglu(X, mask, a_m, a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, Wq_gu, s_gu, Hbuf, ws_gu,
+                               We=We_gu)
+        torch.cuda.synchronize()
+        xd = inputs.make_sgat(Hbuf.float().cpu().numpy(), mask_np)
+        Wq_d = torch.empty(Hd, F // 2, dtype=torch.uint8, device="cuda")
+        s_d = torch.empty(Hd, dtype=torch.float32, device="cuda")
+        abi.sgat_prepare_weight(_dev_np(torch, W_down, f16), _dev_np(torch, xd.inv_a_w), xd.hb, Wq_d, s_d)
+        We_d = torch.empty(Hd, F, dtype=torch.uint8, device="cuda")
+        abi.w4_unpack_e4m3(Wq_d, We_d)
+        am_d, au_d = _dev_np(torch, xd.a_m), _dev_np(torch, xd.a_u)
+        ws_d = torch.empty(abi.sgat_linear_workspace_size(L, F, False), dtype=torch.uint8, device="cuda")
+        Y = torch.empty(L, Hd, dtype=f16, device="cuda")
+
+        def step():
+            abi.sgat_linear_swiglu(X, mask, a_m, a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, Wq_gu, s_gu, Hbuf, ws_gu,
+                                   We=We_gu)
+            abi.sgat_linear(Hbuf, mask, am_d, au_d, xd.hb, xd.d_sh, xd.d_m, xd.d_u, Wq_d, s_d, Y, ws_d, We=We_d)
+
+        for _ in range(max(args.warmup, 3)):
+            step()
+        abi.check_status()
+        g = _graph(torch, step)
+        t = time_kernel(g.replay, flush, max(args.steps, 20), torch)
+        abi.check_status()
+        out[str(ratio)] = {"ms": round(t, 4), "tops": round(ops / (t * 1e-3) / 1e12, 1),
+                           "tokens_per_s": round(L / (t * 1e-3), 1), "masked_tokens": int(mask_np.sum()),
+                           "down_hadamard_block": int(xd.hb)}
+        if t_orc is None:
+            rows = np.arange(0, L, 64)
+            qw, sw = osg.prepare_weight(gu.W, xf.inv_a_w, xf.hb, 4)
+            t0 = time.perf_counter()
+            osg.sgat_linear(gu.X[rows].astype(np.float32), mask_np[rows], xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m,
+                            xf.d_u, qw, sw, None, 4)
+            t_orc = (time.perf_counter() - t0, len(rows))
+        del Wq_gu, We_gu, Wq_d, We_d, ws_gu, ws_d
+    # the unquantised GEMMs of the same shapes
+    Xh = torch.randn(L, Hd, device="cuda").to(f16)
+    Hh = torch.randn(L, F, device="cuda").to(f16)
+    Wg = (0.02 * torch.randn(2 * F, Hd, device="cuda")).to(f16)
+    Wd = (0.02 * torch.randn(Hd, F, device="cuda")).to(f16)
+    Yg = torch.empty(L, 2 * F, dtype=f16, device="cuda")
+    Yd = torch.empty(L, Hd, dtype=f16, device="cuda")
+
+    def fp16_step():
+        abi.fp16_gemm_ref(Xh, Wg, Yg)
+        abi.fp16_gemm_ref(Hh, Wd, Yd)
+
+    for _ in range(3):
+        fp16_step()
+    g16 = _graph(torch, fp16_step)
+    t16 = time_kernel(g16.replay, flush, max(args.steps, 20), torch)
+    abi.check_status()
+    mid = out["0.5"]
+    peaks, peak_src = load_peaks()
+    return {"metric": "LLaDA-8B MLP step (SGAT W4A4 gate+up with SwiGLU, down): integer TOPS, quantisers included",
+            "value": mid["tops"], "unit": "TOPS", "higher_is_better": True, "n_gpus": 1,
+            "ms_per_step": mid["ms"], "tokens_per_s": mid["tokens_per_s"],
+            "data": "synthetic (seeded; heavy-tailed fp16 activations, N(0, 0.02) weights)",
+            "dtype": "int4 codes (E4M3 on the tensor cores), exact integer sums, fp16 out",
+            "config": {"workload": "llada8b_mlp_step", "tokens": L, "hidden": Hd, "ffn": F,
+                       "gate_up": "4096->2x12288 (SwiGLU in the epilogue)", "down": "12288->4096",
+                       "mask": "semi-autoregressive blocks of 32; value at ratio 0.5",
+                       "l2": "flushed before each timed step", "cuda_graph": True},
+            "by_mask_ratio": out,
+            "fp16_gemms": {"ms": round(t16, 4), "tflops": round(ops / (t16 * 1e-3) / 1e12, 1),
+                           "speedup": round(t16 / mid["ms"], 3),
+                           "note": "fp16_gemm_ref on the same shapes, SwiGLU not included"},
+            "gpu_launches": 4 * max(args.steps, 20),
+            "cpu_baseline": {"kind": "oracle", "unit": "TOPS", "cores": cpu_cores(),
+                             "value": round(2 * t_orc[1] * 2 * F * Hd / t_orc[0] / 1e12, 6),
+                             "sample": f"gate+up linear on {t_orc[1]} of {L} tokens at ratio 0.1"}}
+
+
+def run_single_linear(args):
+    """The CPU-oracle-scale linear: 256 tokens x 512 -> 512 with TAC (block
+    64) on its input, one sgat_linear call (TAC, quantiser, GEMM) per step,
+    replayed as a CUDA graph after an L2 flush. At this size the call is
+    launch- and latency-bound; the line reports its latency."""
+    import numpy as np
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi, inputs
+    from oracle import sgat as osg
+    from oracle import tac as otac
+    torch.cuda.set_device(0)
+    case = inputs.single_linear(0)
+    xf = case.xf
+    L, K, N = case.L, case.K, case.N
+    f16 = torch.float16
+    X = _dev_np(torch, case.X, f16)
+    mask = _dev_np(torch, case.mask)
+    Wq = torch.empty(N, K // 2, dtype=torch.uint8, device="cuda")
+    s_w = torch.empty(N, dtype=torch.float32, device="cuda")
+    abi.sgat_prepare_weight(_dev_np(torch, case.W, f16), _dev_np(torch, xf.inv_a_w), xf.hb, Wq, s_w)
+    We = torch.empty(N, K, dtype=torch.uint8, device="cuda")
+    abi.w4_unpack_e4m3(Wq, We)
+    a_m, a_u = _dev_np(torch, xf.a_m), _dev_np(torch, xf.a_u)
+    M, d = _dev_np(torch, case.tac.M), _dev_np(torch, case.tac.d)
+    ws = torch.empty(abi.sgat_linear_workspace_size(L, K, True), dtype=torch.uint8, device="cuda")
+    Y = torch.empty(L, N, dtype=f16, device="cuda")
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    flush = lambda: flush_buf.zero_()
+
+    def step():
+        abi.sgat_linear(X, mask, a_m, a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, Wq, s_w, Y, ws, tac_M=M, tac_d=d,
+                        tac_g=case.tac.g, We=We)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    abi.check_status()
+    g = _graph(torch, step)
+    t = time_kernel(g.replay, flush, max(args.steps, 50), torch)
+    abi.check_status()
+    ops = 2 * L * N * K
+    qw, sw = osg.prepare_weight(case.W, xf.inv_a_w, xf.hb, 4)
+    reps = 0
+    t0 = time.perf_counter()
+    while time.perf_counter() - t0 < 2.0:
+        z = otac.tac_apply(case.X, case.tac.M, case.tac.d, case.tac.g)
+        osg.sgat_linear(z, case.mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, qw, sw, None, 4)
+        reps += 1
+    t_orc = (time.perf_counter() - t0) / reps
+    return {"metric": "single SGAT linear with TAC (256 x 512 -> 512): latency per call",
+            "value": round(t * 1e3, 2), "unit": "us", "higher_is_better": False, "n_gpus": 1,
+            "tops": round(ops / (t * 1e-3) / 1e12, 3),
+            "data": "synthetic (seeded; 8 outlier channels, N(0, 0.02) weights, TAC blocks I + N(0, 0.01))",
+            "dtype": "int4 codes (E4M3 on the tensor cores), exact integer sums, fp16 out",
+            "config": {"workload": "single_linear_256x512x512", "tokens": L, "K": K, "N": N, "tac_block": 64,
+                       "hadamard_block": xf.hb, "l2": "flushed before each timed call", "cuda_graph": True},
+            "gpu_launches": 3 * max(args.steps, 50),
+            "cpu_baseline": {"kind": "oracle", "value": round(t_orc * 1e6, 1), "unit": "us", "cores": cpu_cores(),
+                             "sample": f"the whole call (TAC, quantiser, integer GEMM), {reps} repetitions"}}
+
+
+def run_hbm_passes(args):
+    """The quantiser and TAC of the O projection at 8192 tokens, each timed
+    back to back (hbm_passes_large), without the step, probes or baselines:
+    the small program the quantiser's ncu capture runs. Launch order: the
+    weight preparation's quantiser launch, then per entry three warm-up and
+    twelve timed launches."""
+    import torch
+    torch.cuda.set_device(0)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi, inputs
+    from paper_2606_04945_gb300.pipeline import SgatLinear
+    _, o_case = inputs.llada_attention(seed=0)
+    o = SgatLinear(o_case)
+    flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    large = hbm_passes_large(abi, o, lambda: flush_buf.zero_(), torch)
+    abi.check_status()
+    peaks, src = load_peaks()
+    for v in large.values():
+        v["frac"] = round(v["gbs"] / peaks["hbm_gbs"], 4)
+    return {"workload": "hbm_passes", "peak_gbs": peaks["hbm_gbs"], "peak_source": src, "passes": large}
 
 
 def run_ours(args):
@@ -1342,6 +1561,17 @@ def main():
             return
         out = run_dream_block(args)
         print(json.dumps(out))
+        return
+    if args.workload in ("llada_mlp", "single_linear"):
+        fn = run_llada_mlp if args.workload == "llada_mlp" else run_single_linear
+        out = fn(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
+                                                    "the oracle arm times the attention-step workload"}
+        print(json.dumps(out), flush=True)
+        return
+    if args.workload == "hbm_passes":
+        out = run_hbm_passes(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
+                                                                "the oracle arm times the attention-step workload"}
+        print(json.dumps(out), flush=True)
         return
     if args.workload == "denoise_stack":
         out = run_stack(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
