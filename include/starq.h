@@ -41,6 +41,31 @@ extern "C" {
 /* Element types of activations, weights and outputs. */
 enum starq_dtype { STARQ_F16 = 0, STARQ_BF16 = 1, STARQ_F32 = 2 };
 
+/*
+ * TAC parameters for the tac option of sgat_quantize_act and w4a4_gemm
+ * (Sec. 3.3 Eq. 17: z_b <- M_b z_b + d_b on every block of g channels; the
+ * same arithmetic as tac_apply). All pointers are device memory the caller
+ * owns.
+ *   g        block size: 4, 8, 16, 32, 64 or 128; the channel count is a
+ *            multiple of g.
+ *   M, d     [C/g][g][g] and [C/g][g] float32, 16-byte aligned (d NULL =
+ *            zeros).
+ *   Mp       tac_prepare output for the tensor being compensated (its
+ *            element type, this C and g), or NULL (see tac_apply).
+ *   scratch  [L][C] buffer, 16-byte aligned, of the compensated tensor's
+ *            element type: sgat_quantize_act writes the compensated input
+ *            there and quantises it; w4a4_gemm writes the uncompensated
+ *            output there and compensates it into Y. It must not overlap
+ *            the call's other buffers.
+ */
+typedef struct {
+    int g;
+    const float* M;
+    const float* d;
+    const void* Mp;
+    void* scratch;
+} starq_tac;
+
 /* Return codes. */
 enum starq_status {
     STARQ_OK = 0,
@@ -156,11 +181,19 @@ int starq_probe_mma(int kind, int iters, unsigned long long* cycles, int* errors
  *           operand of w8a8_gemm).
  *   v_dbg   [L][K] float32 transformed activations out (before rounding),
  *           16-byte aligned, or NULL.
+ *   tac     NULL, or TAC on the input first (the attention output before
+ *           the output projection, Sec. 3.3): tac->scratch [L][K] of x_dtype
+ *           receives TAC(X), and the transform and quantisation above read
+ *           it in place of X. Two kernels (TAC on the tensor cores for
+ *           16-bit X and g = 64 or 128, then the quantiser): a token's
+ *           transform needs all K compensated channels, every one of the
+ *           K / g blocks of M.
  * Shapes: L >= 0, 16 <= K <= 20480, K % 16 == 0.
  */
 int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                      int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg, void* stream);
+                      const starq_tac* tac, int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg,
+                      void* stream);
 
 /*
  * sgat_prepare_weight -- the unified static weight transform, quantised once
@@ -324,12 +357,16 @@ int sgat_linear_asym(const void* X, int x_dtype, int L, int K, const uint8_t* ma
  *   s_a [L], s_w [N] float32; bias [N] float32 or NULL.
  *   Y  [L][N] out, y_dtype F16, BF16 or F32, 16-byte aligned.
  *   acc_dbg [L][N] int32 out (the exact accumulators) or NULL.
+ *   out_tac NULL, or TAC on the output (C = N): the dequantised output goes
+ *      to out_tac->scratch [L][N] of y_dtype, and Y = TAC(scratch) (a
+ *      second kernel; the quantised softmax-value product has its TAC
+ *      fused into its epilogue, attention_pv_tac).
  * Shapes: L >= 0, N >= 32 with N % 32 == 0, K >= 128 with K % 128 == 0,
  * K <= 65536 (so |acc| <= 49 K < 2^22).
  */
 int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq,
               const uint8_t* We, const float* s_w, const float* bias, int L, int N, int K, void* Y,
-              int y_dtype, int32_t* acc_dbg, void* stream);
+              int y_dtype, const starq_tac* out_tac, int32_t* acc_dbg, void* stream);
 
 /*
  * Tile of the last Xe + We (or fp16_gemm_ref) launch on the calling thread,

@@ -30,6 +30,26 @@ EXPORTED = (
 )
 
 
+class StarqTac(ctypes.Structure):
+    """starq_tac: TAC parameters of the tac option of sgat_quantize_act and
+    w4a4_gemm."""
+    _fields_ = [("g", ctypes.c_int), ("M", ctypes.c_void_p), ("d", ctypes.c_void_p), ("Mp", ctypes.c_void_p),
+                ("scratch", ctypes.c_void_p)]
+
+
+def _tac_struct(M, d, g, Mp, scratch):
+    """A StarqTac for the given tensors, or None when M is None."""
+    if M is None:
+        return None
+    _contig(M, d, Mp, scratch)
+    ptr = lambda t: None if t is None else t.data_ptr()
+    return StarqTac(int(g), ptr(M), ptr(d), ptr(Mp), ptr(scratch))
+
+
+def _ref(struct):
+    return None if struct is None else ctypes.byref(struct)
+
+
 class StarqError(RuntimeError):
     def __init__(self, code, msg):
         super().__init__(f"starq error {code}: {msg}")
@@ -49,10 +69,10 @@ def _load():
     lib.glue_add_rmsnorm.argtypes = [vp, vp, i, i, i, f_p, ctypes.c_float, vp, vp, vp]
     lib.glue_rope.argtypes = [vp, i, i, i, i, vp, ctypes.c_double, vp]
     lib.starq_probe_mma.argtypes = [i, i, vp, vp, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double), vp]
-    lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, i, u8p, f_p, u8p, f_p, vp]
+    lib.sgat_quantize_act.argtypes = [vp, i, i, i, u8p, f_p, f_p, i, i, i, i, vp, i, u8p, f_p, u8p, f_p, vp]
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
-    lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp, vp]
     lib.w8_split_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w8a8_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.sgat_linear_workspace_size_bits.argtypes = [i, i, i, i]
@@ -152,11 +172,14 @@ def probe_mma(kind, iters, cycles, errors, stream=None):
 
 
 def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, bits=4, Xe=None, v_dbg=None,
-                      stream=None):
+                      stream=None, tac_M=None, tac_d=None, tac_g=0, tac_Mp=None, tac_scratch=None):
+    """With tac_M: TAC on X first (into tac_scratch [L][K], X's type), then
+    the quantiser on the compensated rows."""
     _contig(X, mask, a_m, a_u, Xq, s_a, Xe, v_dbg)
     L, K = X.shape
+    tac = _tac_struct(tac_M, tac_d, tac_g, tac_Mp, tac_scratch)
     _check(lib.sgat_quantize_act(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb,
-                                 d_sh, d_m, d_u, bits, _p(Xq), _p(s_a), _p(Xe), _p(v_dbg),
+                                 d_sh, d_m, d_u, _ref(tac), bits, _p(Xq), _p(s_a), _p(Xe), _p(v_dbg),
                                  _stream(stream)))
 
 
@@ -270,15 +293,19 @@ def w8a8_gemm(Xe, s_a, We, s_w, Y, bias=None, acc_dbg=None, stream=None):
                          _stream(stream)))
 
 
-def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, stream=None):
+def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, stream=None, tac_M=None,
+              tac_d=None, tac_g=0, tac_Mp=None, tac_scratch=None):
     """Xq: packed int4 codes [L][K/2] (may be None when Xe is given);
     Xe: the same codes as E4M3 bytes [L][K] (selects a TMA CTA-pair kernel);
-    We: the weight codes as E4M3 bytes [N][K] (with Xe: both operands by TMA)."""
+    We: the weight codes as E4M3 bytes [N][K] (with Xe: both operands by TMA).
+    With tac_M: the dequantised output goes to tac_scratch [L][N] (Y's type)
+    and Y receives its TAC."""
     _contig(Xq, Xe, s_a, Wq, We, s_w, Y, bias, acc_dbg)
     L = Y.shape[0]
     N, K = _weight_shape(Wq, We)
+    tac = _tac_struct(tac_M, tac_d, tac_g, tac_Mp, tac_scratch)
     _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y),
-                         dtype_code(Y), _p(acc_dbg), _stream(stream)))
+                         dtype_code(Y), _ref(tac), _p(acc_dbg), _stream(stream)))
 
 
 def last_gemm_tile():

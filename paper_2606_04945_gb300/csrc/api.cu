@@ -77,6 +77,25 @@ int check_tac(int L, int C, int g, const float* M, const float* d) {
     return STARQ_OK;
 }
 
+int check_tac_prepared(const void* Mp, int z_dtype, int g) {
+    if (!Mp) return STARQ_OK;
+    if ((z_dtype != STARQ_F16 && z_dtype != STARQ_BF16) || (g != 64 && g != 128))
+        return fail(STARQ_ERR_ARG, "prepared TAC matrix: 16-bit Z and g = 64 or 128 only");
+    if (!aligned(Mp, 16)) return fail(STARQ_ERR_ALIGN, "prepared TAC matrix must be 16-byte aligned");
+    return STARQ_OK;
+}
+
+// The tac option of sgat_quantize_act and w4a4_gemm: parameters for a
+// [L][C] tensor of element type dtype (its scratch buffer included).
+int check_tac_option(const char* who, const starq_tac* t, int L, int C, int dtype) {
+    int rc = check_tac(L, C, t->g, t->M, t->d);
+    if (rc) return rc;
+    if ((rc = check_tac_prepared(t->Mp, dtype, t->g))) return rc;
+    if (L > 0 && !t->scratch) return fail(STARQ_ERR_ARG, "%s: tac->scratch is NULL", who);
+    if (L > 0 && !aligned(t->scratch, 16)) return fail(STARQ_ERR_ALIGN, "%s: tac->scratch must be 16-byte aligned", who);
+    return STARQ_OK;
+}
+
 int check_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq, const uint8_t* We,
                const float* s_w, const float* bias, int L, int N, int K, void* Y, int y_dtype) {
     if ((!Wq && !We) || !s_w) return fail(STARQ_ERR_ARG, "w4a4_gemm: NULL Wq/We or s_w");
@@ -294,7 +313,8 @@ int starq_probe_mma(int kind, int iters, unsigned long long* cycles, int* errors
 
 int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* mask,
                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
-                      int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg, void* stream) {
+                      const starq_tac* tac, int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg,
+                      void* stream) {
     if (L > 0 && (!X || !Xq || !s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, Xq or s_a");
     if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: unknown dtype %d", x_dtype);
     if (bits != 4 && bits != 8) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4- and 8-bit codes", bits);
@@ -304,8 +324,20 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
     if (L == 0) return STARQ_OK;
     if (!aligned(X, 16) || !aligned(Xq, 8) || (v_dbg && !aligned(v_dbg, 16)) || (Xe && !aligned(Xe, 16)))
         return fail(STARQ_ERR_ALIGN, "sgat_quantize_act: X (16 B), Xq (8 B), Xe (16 B), v_dbg (16 B) alignment");
-    QuantArgs a{X, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits == 8 ? 127 : 7, 1.f, Xq, s_a, v_dbg, Xe};
-    cudaError_t e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
+    const void* src = X;
+    cudaError_t e;
+    if (tac) {                       // TAC(X) into the scratch buffer, then quantise that
+        if ((rc = check_tac_option("sgat_quantize_act", tac, L, K, x_dtype))) return rc;
+        if ((rc = check_local("sgat_quantize_act", static_cast<cudaStream_t>(stream), {X, tac->scratch}))) return rc;
+        unsigned* st = status_ptr(&rc);
+        if (!st) return rc;
+        TacArgs t{X, x_dtype, L, K, tac->g, tac->M, tac->d, tac->scratch, x_dtype, st, tac->Mp};
+        if ((e = launch_tac(t, static_cast<cudaStream_t>(stream))) != cudaSuccess)
+            return cuda_fail(e, "sgat_quantize_act: TAC launch");
+        src = tac->scratch;
+    }
+    QuantArgs a{src, x_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits == 8 ? 127 : 7, 1.f, Xq, s_a, v_dbg, Xe};
+    e = launch_sgat_quant(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "sgat_quantize_act launch");
     return STARQ_OK;
 }
@@ -340,17 +372,25 @@ int w4_unpack_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream) {
 
 int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint8_t* Wq, const uint8_t* We,
               const float* s_w, const float* bias, int L, int N, int K, void* Y, int y_dtype,
-              int32_t* acc_dbg, void* stream) {
+              const starq_tac* out_tac, int32_t* acc_dbg, void* stream) {
     int rc = check_gemm(Xq, Xe, s_a, Wq, We, s_w, bias, L, N, K, Y, y_dtype);
     if (rc) return rc;
     if (acc_dbg && !aligned(acc_dbg, 16)) return fail(STARQ_ERR_ALIGN, "acc_dbg must be 16-byte aligned");
-    if (L > 0 && (rc = check_local("w4a4_gemm", static_cast<cudaStream_t>(stream), {Xe, Xe ? We : nullptr, Xe ? Wq : nullptr, Y})))
+    if (out_tac && (rc = check_tac_option("w4a4_gemm", out_tac, L, N, y_dtype))) return rc;
+    void* dst = out_tac ? out_tac->scratch : Y;    // the dequantised output before TAC
+    if (L > 0 && (rc = check_local("w4a4_gemm", static_cast<cudaStream_t>(stream),
+                                   {Xe, Xe ? We : nullptr, Xe ? Wq : nullptr, Y, dst})))
         return rc;
     unsigned* st = status_ptr(&rc);
     if (!st) return rc;
-    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, st, Xe, Xe ? We : nullptr};
+    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, dst, y_dtype, acc_dbg, st, Xe, Xe ? We : nullptr};
     cudaError_t e = launch_w4a4_gemm(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm launch");
+    if (out_tac && L > 0) {
+        TacArgs t{dst, y_dtype, L, N, out_tac->g, out_tac->M, out_tac->d, Y, y_dtype, st, out_tac->Mp};
+        if ((e = launch_tac(t, static_cast<cudaStream_t>(stream))) != cudaSuccess)
+            return cuda_fail(e, "w4a4_gemm: TAC launch");
+    }
     return STARQ_OK;
 }
 
@@ -587,15 +627,6 @@ int tac_prepare(const float* M, int C, int g, int z_dtype, void* Mp, void* strea
     return STARQ_OK;
 }
 
-namespace {
-int check_tac_prepared(const void* Mp, int z_dtype, int g) {
-    if (!Mp) return STARQ_OK;
-    if ((z_dtype != STARQ_F16 && z_dtype != STARQ_BF16) || (g != 64 && g != 128))
-        return fail(STARQ_ERR_ARG, "prepared TAC matrix: 16-bit Z and g = 64 or 128 only");
-    if (!aligned(Mp, 16)) return fail(STARQ_ERR_ALIGN, "prepared TAC matrix must be 16-byte aligned");
-    return STARQ_OK;
-}
-}  // namespace
 
 int tac_apply(const void* Z, int z_dtype, int L, int C, int g, const float* M, const float* d, const void* Mp,
               void* out, int out_dtype, void* stream) {

@@ -29,8 +29,9 @@
 // attn_vquant_kernel   V codes per channel, written as fp16 values into
 //                      Vt [128 H][L] (keys contiguous: the K-major B
 //                      operand of P V^T), and the channel scales t.
-// attn_pv_tac_kernel   one CTA per (128-query tile, head), each loading its
-//                      own K / V tiles by TMA. 16 softmax / epilogue warps (a
+// attn_pv_tac_kernel   persistent CTAs (at most one per SM) looping over the
+//                      (128-query tile, head) items, each loading its own
+//                      K / V tiles by TMA. 16 softmax / epilogue warps (a
 //                      TMEM lane quarter times 32 of the 128 columns each),
 //                      a TMA warp and one MMA warp, which issues every MMA
 //                      (tcgen05 kind::f16 on one CTA, M = N = 128, K = 16)
@@ -55,8 +56,9 @@
 //           prepared halves (tac_prepare); + d; rounded to fp16 and stored
 //           by TMA.
 // Shared memory holds only B operands: a ring of six 32 KB tiles streams
-// pass 1's K chunks and pass 2's K and V chunks in the order the MMAs read
-// them; two of its slots then take M's halves and one the output boxes.
+// each item's pass-1 K chunks, pass-2 K and V chunks, M's two halves and
+// then the slot of its output boxes, in the order they are used, running
+// on into the next item.
 // TMEM (512 columns): two S / P buffers, the P V^T accumulator and Q; the
 // TAC accumulator and Z_hat reuse the S buffers. The MMA warp queries its
 // two barriers per MMA group back to back, so their latencies overlap: with
@@ -93,7 +95,7 @@ constexpr uint32_t TM_TAC = 0, TM_ZHI = 128, TM_ZLO = 192;
 
 struct AttSm {
     uint64_t q_full, full[ATT_SLOTS], empty[ATT_SLOTS], s_full[3], s_empty[3];
-    uint64_t pv_done, z_full, m_full, tac_done;
+    uint64_t pv_done, z_full, tac_done, tac_read;
     uint32_t tmem_base;
     int abort;
     float xm[4][ATTN_TILE];            // row maxima / sums of the four column parts
@@ -258,8 +260,25 @@ __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
     }
 }
 
-// A ring slot is refilled once this CTA's MMAs have read it (one commit on
-// its empty barrier).
+// Persistent: a CTA takes the work items w = blockIdx.x + i gridDim.x (i =
+// 0, 1, ...) of the nq H items (query tile w mod nq of head w / nq), so the
+// CTAs running at one time share heads and their K / V tiles in L2. Every
+// role loops over the same items, and every barrier's phase runs on across
+// items.
+//
+// The ring's entries of item i are E = 3 nk + 3 in number, global index
+// G = i E + u: u = 0 .. nk-1 the K chunks of pass 1, u = nk + 2j, nk + 2j + 1
+// chunk j's K and V for pass 2, u = 3 nk and 3 nk + 1 M's halves (one bulk
+// copy each), u = 3 nk + 2 the output boxes (the TMA warp hands the free
+// slot to the softmax warps with a plain arrive on its full barrier; they
+// give it back after their stores have read it). Entry G uses slot G mod 6
+// for the (G / 6)-th time. So the next item's K chunks stream in while this
+// item's epilogue runs.
+//
+// TMEM across items: the next item's Q is written as soon as this item's
+// P V^T has completed (its columns are then dead), and its first Q K^T
+// waits until the epilogue has read this item's TAC accumulator (tac_read),
+// which sits in the first S buffer.
 template <typename T>
 __global__ void __launch_bounds__(ATT_THREADS, 1)
 attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
@@ -269,33 +288,35 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
     const uint32_t base = (raw + 1023u) & ~1023u;
     AttSm* sh = reinterpret_cast<AttSm*>(smem_raw + (base - raw) + ATT_TILES_BYTES);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int q0 = blockIdx.x * ATTN_TILE, h = blockIdx.y;
-    const int hk = h / (a.H / a.Hkv);                       // key/value head of this query head
-    const int nk = a.L / ATTN_TILE;
+    const int nk = a.L / ATTN_TILE;                          // key chunks = query tiles of a head
+    const int items = nk * a.H;
+    const int my_items = blockIdx.x < (unsigned)items ? (items - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    const int group = a.H / a.Hkv;
     volatile int* abort = &sh->abort;
     // (the lambdas capture by value: a local captured by reference lives in
     // memory and is reloaded after every asm with a memory clobber)
     auto B = [](const uint64_t& bar) { return smem_addr(&bar); };
-    // The ring's loads in order: u = 0 .. nk-1 the K chunks of pass 1, then
-    // u = nk + 2j, nk + 2j + 1 chunk j's K and V tiles for pass 2. Load u
-    // goes to slot u mod 6 (its (u / 6)-th use). M's halves take the slots
-    // of u = U - 6 and U - 5 once those loads are consumed (a negative u
-    // names a slot no load uses), the output boxes the slot of U - 1.
-    const int U = 3 * nk;
-    auto slot_idx = [](int u) { return ((u % ATT_SLOTS) + ATT_SLOTS) % ATT_SLOTS; };
-    auto slot = [=](int u) { return base + (uint32_t)slot_idx(u) * TILE_BYTES; };
-    const uint32_t sMhi = slot(U - 6), sMlo = slot(U - 5), sOut = slot(U - 1);
-    // S buffer of Q K^T number it (pass 1: it = 0 .. nk-1, three buffers,
-    // the third in O's columns, which pass 1 leaves unused; pass 2: it =
-    // nk + j, two buffers) and the number of that buffer's earlier uses
-    auto sbuf = [nk](int it, int& b, int& n) {
+    const int E = 3 * nk + 3;                                // ring entries per item
+    auto slot = [=](long long g) { return base + (uint32_t)(g % ATT_SLOTS) * TILE_BYTES; };
+    auto full_bar = [=](long long g) { return B(sh->full[g % ATT_SLOTS]); };
+    auto empty_bar = [=](long long g) { return B(sh->empty[g % ATT_SLOTS]); };
+    auto use_parity = [](long long g) { return (uint32_t)((g / ATT_SLOTS) & 1); };
+    auto item_q0 = [=](int i) { return ((int)blockIdx.x + i * (int)gridDim.x) % nk * ATTN_TILE; };
+    auto item_h = [=](int i) { return ((int)blockIdx.x + i * (int)gridDim.x) / nk; };
+    // S buffer of Q K^T number it of item i (pass 1: it = 0 .. nk-1, three
+    // buffers, the third in the columns of the P V^T accumulator, which pass
+    // 1 leaves unused; pass 2: it = nk + j, two buffers) and the number of
+    // that buffer's earlier uses, counted over all items
+    const int p1_0 = (nk + 2) / 3, p1_1 = (nk + 1) / 3, p1_2 = nk / 3;   // pass-1 uses per item
+    const int p2_0 = (nk + 1) / 2, p2_1 = nk / 2;                       // pass-2 uses per item
+    auto sbuf = [=](int i, int it, int& b, int& n) {
         if (it < nk) {
             b = it % 3;
-            n = it / 3;
+            n = it / 3 + i * (b == 0 ? p1_0 + p2_0 : b == 1 ? p1_1 + p2_1 : p1_2);
         } else {
             const int j = it - nk;
             b = j & 1;
-            n = (nk - b + 2) / 3 + (j >> 1);
+            n = (b == 0 ? p1_0 : p1_1) + (j >> 1) + i * (b == 0 ? p1_0 + p2_0 : p1_1 + p2_1);
         }
     };
 
@@ -311,8 +332,8 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         }
         mbar_init(B(sh->pv_done), 1);
         mbar_init(B(sh->z_full), ATT_SOFTMAX_WARPS);
-        mbar_init(B(sh->m_full), 1);
         mbar_init(B(sh->tac_done), 1);
+        mbar_init(B(sh->tac_read), ATT_SOFTMAX_WARPS);
         sh->abort = 0;
         mbar_fence_init();
     }
@@ -327,42 +348,44 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
 
     if (warp == ATT_TMA_WARP) {
         bool ok = true;
-        for (int u = 0; u < U && ok; ++u) {
-            const int k = u % ATT_SLOTS, n = u / ATT_SLOTS;
-            if (!mbar_wait_bounded_warp(B(sh->empty[k]), (uint32_t)(n & 1) ^ 1u, abort)) { ok = false; break; }
-            const uint32_t dst = slot(u);
-            if (elect_one()) {
-                mbar_arrive_expect_tx(B(sh->full[k]), TILE_BYTES);
-                const int w = u - nk;
-                const uint32_t fb = B(sh->full[k]);
-                const void* tm = (w < 0 || (w & 1) == 0) ? (const void*)&tm_k : (const void*)&tm_v;
-                int x, y;
-                if (w < 0 || (w & 1) == 0) {                 // K chunk: keys are the rows
-                    x = hk * ATTN_D;
-                    y = (w < 0 ? u : w >> 1) * ATTN_TILE;
-                } else {                                     // V chunk: channels are the rows
-                    x = (w >> 1) * ATTN_TILE;
-                    y = hk * ATTN_D;
+        for (int i = 0; i < my_items && ok; ++i) {
+            const int h = item_h(i), hk = h / group;
+            for (int u = 0; u < E && ok; ++u) {
+                const long long g = (long long)i * E + u;
+                if (!mbar_wait_bounded_warp(empty_bar(g), use_parity(g) ^ 1u, abort)) { ok = false; break; }
+                const uint32_t dst = slot(g), fb = full_bar(g);
+                if (elect_one()) {
+                    if (u < 3 * nk) {
+                        mbar_arrive_expect_tx(fb, TILE_BYTES);
+                        const int w = u - nk;
+                        const void* tm = (w < 0 || (w & 1) == 0) ? (const void*)&tm_k : (const void*)&tm_v;
+                        int x, y;
+                        if (w < 0 || (w & 1) == 0) {             // K chunk: keys are the rows
+                            x = hk * ATTN_D;
+                            y = (w < 0 ? u : w >> 1) * ATTN_TILE;
+                        } else {                                 // V chunk: channels are the rows
+                            x = (w >> 1) * ATTN_TILE;
+                            y = hk * ATTN_D;
+                        }
+                        tma_load_2d(dst, tm, x, y, fb);
+                        tma_load_2d(dst + ATOM_BYTES, tm, x + 64, y, fb);
+                    } else if (u < 3 * nk + 2) {                 // M_hi, M_lo of head h
+                        const uint8_t* mp = static_cast<const uint8_t*>(a.Mp) +
+                                            ((size_t)h * 2 + (size_t)(u - 3 * nk)) * TILE_BYTES;
+                        mbar_arrive_expect_tx(fb, TILE_BYTES);
+                        bulk_load(dst, mp, TILE_BYTES, fb);
+                    } else {                                     // the output boxes' slot
+                        mbar_arrive(fb);
+                    }
                 }
-                tma_load_2d(dst, tm, x, y, fb);
-                tma_load_2d(dst + ATOM_BYTES, tm, x + 64, y, fb);
+                __syncwarp();
             }
-            __syncwarp();
         }
-        // M's halves once their slots' last loads have been consumed
-        for (int u = U - 6; u < U - 4 && ok; ++u)
-            if (u >= 0) ok = mbar_wait_bounded_warp(B(sh->empty[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1), abort);
-        if (ok && elect_one()) {
-            const uint8_t* mp = static_cast<const uint8_t*>(a.Mp) + (size_t)h * 2 * TILE_BYTES;
-            mbar_arrive_expect_tx(B(sh->m_full), 2 * TILE_BYTES);
-            bulk_load(sMhi, mp, TILE_BYTES, B(sh->m_full));
-            bulk_load(sMlo, mp + TILE_BYTES, TILE_BYTES, B(sh->m_full));
-        }
-        __syncwarp();
-        // the commits for the last use of each slot have arrived, so none
+        // every slot's last use has been given back, so no commit or arrive
         // lands after this CTA has exited
-        for (int u = U - ATT_SLOTS; u < U && ok; ++u)
-            if (u >= 0) ok = mbar_wait_bounded_warp(B(sh->empty[u % ATT_SLOTS]), (uint32_t)((u / ATT_SLOTS) & 1), abort);
+        const long long G = (long long)my_items * E;
+        for (long long g = G - ATT_SLOTS; g < G && ok; ++g)
+            if (g >= 0) ok = mbar_wait_bounded_warp(empty_bar(g), use_parity(g), abort);
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     } else if (warp == ATT_MMA_WARP) {
         // f32 D, N = 128 (bits 17..22), M = 128 (bits 24..28); A and B fp16
@@ -370,8 +393,6 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         // sets the A and B format fields, bits 7..9 and 10..12)
         constexpr uint32_t IDESC_F16 = (1u << 4) | ((uint32_t)(ATTN_TILE >> 3) << 17) | ((uint32_t)(ATTN_TILE >> 4) << 24);
         constexpr uint32_t IDESC_T = IDESC_F16 | (std::is_same<T, __nv_bfloat16>::value ? ((1u << 7) | (1u << 10)) : 0u);
-        (void)IDESC_T;
-        bool ok = mbar_wait_bounded_warp(B(sh->q_full), 0, abort);
         // D (+)= A B^T over K = 128: A from TMEM at a_col (8 columns per K
         // step; for P, K steps 2p and 2p + 1 sit at 32 p and 32 p + 8), B
         // the K-major tile at bt
@@ -388,49 +409,53 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 mma_f16_ts(d, ta + ac, bd + (uint64_t)(koff >> 4), idesc, (acc0 || ks > 0) ? 1u : 0u);
             }
         };
-        auto release = [=](int u) {           // this CTA's MMAs are done with ring slot u
-            tc_commit(B(sh->empty[u % ATT_SLOTS]));
-        };
-        // Q K^T number it, once its K tile has landed and its S buffer's
-        // previous use is consumed: S read by the softmax warps, or P
-        // written by them and read by the P V^T issued before this MMA (the
-        // MMAs of one thread run in issue order). For pass-2 chunks from 2
-        // on, that P V^T's own wait has already seen the P written.
-        auto qk = [=](int it) -> bool {
-            const int u = it < nk ? it : nk + 2 * (it - nk);
-            int b, n;
-            sbuf(it, b, n);
-            const uint32_t fb = B(sh->full[u % ATT_SLOTS]), fp = (uint32_t)((u / ATT_SLOTS) & 1);
-            if (!(it >= nk + 2 ? mbar_wait_bounded_warp(fb, fp, abort)
-                               : mbar_wait2_bounded_warp(fb, fp, B(sh->s_empty[b]), (uint32_t)(n & 1) ^ 1u, abort)))
-                return false;
-            tc_fence_after();
-            if (elect_one()) {
-                mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(u), false, false, IDESC_T);
-                release(u);
-                tc_commit(B(sh->s_full[b]));
-            }
-            __syncwarp();
-            return true;
-        };
-        // P V^T of pass-2 chunk j, once its P is in its S buffer
-        auto pv = [=](int j) -> bool {
-            const int u = nk + 2 * j + 1;
-            int b, n;
-            sbuf(nk + j, b, n);
-            if (!mbar_wait2_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1), B(sh->full[u % ATT_SLOTS]),
-                                         (uint32_t)((u / ATT_SLOTS) & 1), abort))
-                return false;
-            tc_fence_after();
-            if (elect_one()) {
-                mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(u), j > 0, true, IDESC_F16);
-                release(u);
-            }
-            __syncwarp();
-            return true;
-        };
+        bool ok = true;
+        int tac_commits = 0;
         tc_fence_after();
-        {
+        for (int i = 0; i < my_items && ok; ++i) {
+            const long long g0 = (long long)i * E;
+            // Q in TMEM; for i > 0 the previous TAC accumulator read out
+            ok = i == 0 ? mbar_wait_bounded_warp(B(sh->q_full), 0, abort)
+                        : mbar_wait2_bounded_warp(B(sh->q_full), (uint32_t)(i & 1), B(sh->tac_read),
+                                                  (uint32_t)((i - 1) & 1), abort);
+            // Q K^T number it, once its K tile has landed and its S buffer's
+            // previous use is consumed: S read by the softmax warps, or P
+            // written by them and read by the P V^T issued before this MMA
+            // (the MMAs of one thread run in issue order). For pass-2 chunks
+            // from 2 on, that P V^T's own wait has already seen the P written.
+            auto qk = [=](int it) -> bool {
+                const long long g = g0 + (it < nk ? it : nk + 2 * (it - nk));
+                int b, n;
+                sbuf(i, it, b, n);
+                if (!(it >= nk + 2 ? mbar_wait_bounded_warp(full_bar(g), use_parity(g), abort)
+                                   : mbar_wait2_bounded_warp(full_bar(g), use_parity(g), B(sh->s_empty[b]),
+                                                             (uint32_t)(n & 1) ^ 1u, abort)))
+                    return false;
+                tc_fence_after();
+                if (elect_one()) {
+                    mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(g), false, false, IDESC_T);
+                    tc_commit(empty_bar(g));
+                    tc_commit(B(sh->s_full[b]));
+                }
+                __syncwarp();
+                return true;
+            };
+            // P V^T of pass-2 chunk j, once its P is in its S buffer
+            auto pv = [=](int j) -> bool {
+                const long long g = g0 + nk + 2 * j + 1;
+                int b, n;
+                sbuf(i, nk + j, b, n);
+                if (!mbar_wait2_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1), full_bar(g), use_parity(g), abort))
+                    return false;
+                tc_fence_after();
+                if (elect_one()) {
+                    mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(g), j > 0, true, IDESC_F16);
+                    tc_commit(empty_bar(g));
+                }
+                __syncwarp();
+                return true;
+            };
+            tc_fence_after();
             for (int it = 0; it < 2 * nk && ok; ++it) {
                 ok = qk(it);
                 if (ok && it > nk) ok = pv(it - 1 - nk);   // one chunk behind the scores
@@ -438,24 +463,29 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             if (ok) ok = pv(nk - 1);
             if (elect_one()) tc_commit(B(sh->pv_done));
             __syncwarp();
-            ok = ok && mbar_wait2_bounded_warp(B(sh->z_full), 0, B(sh->m_full), 0, abort);
+            const long long gm = g0 + 3 * nk;               // M_hi; M_lo at gm + 1
+            ok = ok && mbar_wait2_bounded_warp(B(sh->z_full), (uint32_t)(i & 1), full_bar(gm), use_parity(gm), abort) &&
+                 mbar_wait_bounded_warp(full_bar(gm + 1), use_parity(gm + 1), abort);
             tc_fence_after();
             if (elect_one()) {
                 if (ok) {
-                    mma_tile(tmem + TM_TAC, TM_ZHI, sMhi, false, false, IDESC_F16);   // Z_hi M_hi^T
-                    mma_tile(tmem + TM_TAC, TM_ZHI, sMlo, true, false, IDESC_F16);    // + Z_hi M_lo^T
-                    mma_tile(tmem + TM_TAC, TM_ZLO, sMhi, true, false, IDESC_F16);    // + Z_lo M_hi^T
+                    mma_tile(tmem + TM_TAC, TM_ZHI, slot(gm), false, false, IDESC_F16);       // Z_hi M_hi^T
+                    mma_tile(tmem + TM_TAC, TM_ZHI, slot(gm + 1), true, false, IDESC_F16);    // + Z_hi M_lo^T
+                    mma_tile(tmem + TM_TAC, TM_ZLO, slot(gm), true, false, IDESC_F16);        // + Z_lo M_hi^T
+                    tc_commit(empty_bar(gm));
+                    tc_commit(empty_bar(gm + 1));
                 }
                 tc_commit(B(sh->tac_done));
             }
             __syncwarp();
-            if (lane == 0) {
-                // every MMA of this thread has completed before TMEM is released
-                volatile int never = 0;
-                if (!mbar_wait_bounded(B(sh->tac_done), 0, &never)) ok = false;
-            }
-            __syncwarp();
+            ++tac_commits;
         }
+        if (tac_commits > 0 && lane == 0) {
+            // every MMA of this thread has completed before TMEM is released
+            volatile int never = 0;
+            if (!mbar_wait_bounded(B(sh->tac_done), (uint32_t)((tac_commits - 1) & 1), &never)) ok = false;
+        }
+        __syncwarp();
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     } else {
         const int quarter = warp & 3, part = warp >> 2, col = part * 32;
@@ -463,9 +493,9 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
         bool ok = true;
         uint32_t r[32];
-        {   // the query row's 32 channels of this part into TMEM (A of Q K^T);
-            // the loads of Q, t and d are all in flight together
-            const T* qp = static_cast<const T*>(a.Q) + (size_t)(q0 + row) * a.ld + h * ATTN_D + col;
+        // the query row's 32 channels of this part into TMEM (A of Q K^T)
+        auto put_q = [=](int i) {
+            const T* qp = static_cast<const T*>(a.Q) + (size_t)(item_q0(i) + row) * a.ld + item_h(i) * ATTN_D + col;
             uint32_t qv[16];
             #pragma unroll
             for (int k = 0; k < 4; ++k) {
@@ -475,155 +505,175 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 qv[4 * k + 2] = w.z;
                 qv[4 * k + 3] = w.w;
             }
-            if (threadIdx.x >= ATTN_D && threadIdx.x < 2 * ATTN_D) {
-                const int c = threadIdx.x - ATTN_D;
-                sh->dv[c] = a.d != nullptr ? a.d[h * ATTN_D + c] : 0.f;
-            }
             tmem_st_32x32b_x16(tl + TM_Q + part * 16, qv);
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(B(sh->q_full));
-        }
-        // pass 1: row maxima
-        float mx = -INFINITY;
-        for (int it = 0; it < nk && ok; ++it) {
-            int b, n;
-            sbuf(it, b, n);
-            if (!mbar_wait_bounded_warp(B(sh->s_full[b]), (uint32_t)(n & 1), abort)) { ok = false; break; }
-            tc_fence_after();
-            tmem_ld_32x32b_x32(tl + TM_S + b * ATTN_TILE + col, r);
-            tmem_ld_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
-            #pragma unroll
-            for (int k = 0; k < 32; ++k) mx = fmaxf(mx, __uint_as_float(r[k]));
-        }
-        if (threadIdx.x < ATTN_D) sh->tv[threadIdx.x] = a.t[hk * ATTN_D + threadIdx.x];  // V channel scales
-        sh->xm[part][row] = mx;
-        named_sync_softmax();
-        mx = fmaxf(fmaxf(sh->xm[0][row], sh->xm[1][row]), fmaxf(sh->xm[2][row], sh->xm[3][row]));
-        named_sync_softmax();
-        // pass 2: probabilities, their codes and the row sums
-        float lp[4] = {0.f, 0.f, 0.f, 0.f};      // partial row sums (independent chains)
-        for (int j = 0; j < nk && ok; ++j) {
-            int b, n;
-            sbuf(nk + j, b, n);
-            if (!mbar_wait_bounded_warp(B(sh->s_full[b]), (uint32_t)(n & 1), abort)) { ok = false; break; }
-            tc_fence_after();
-            tmem_ld_32x32b_x32(tl + TM_S + b * ATTN_TILE + col, r);
-            tmem_ld_wait();
-            // e = 2^((s - m) log2(e) / sqrt(d)); the code n = rne(255 e) in
-            // one rounding: the low halves of fma(255, e, ROUND_BIAS) are the
-            // fp16 values 1024 + n of two codes, and 1024 is subtracted
-            // exactly in fp16
-            uint32_t packed[16];
-            const __half2 minus1024 = __float2half2_rn(-1024.f);
-            #pragma unroll
-            for (int k = 0; k < 32; k += 2) {
-                const float e0 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k]), mx), EXP_SCALE));
-                const float e1 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k + 1]), mx), EXP_SCALE));
-                lp[(k >> 1) & 1] += e0;
-                lp[2 + ((k >> 1) & 1)] += e1;
-                const uint32_t t0 = __float_as_uint(fmaf(255.f, e0, ROUND_BIAS));
-                const uint32_t t1 = __float_as_uint(fmaf(255.f, e1, ROUND_BIAS));
-                const uint32_t biased = prmt(t0, t1, 0x5410u);           // {1024 + n0, 1024 + n1}
-                const __half2 hc = __hadd2(*reinterpret_cast<const __half2*>(&biased), minus1024);
-                packed[k / 2] = *reinterpret_cast<const uint32_t*>(&hc);
+        };
+        if (my_items > 0) put_q(0);
+        // Every softmax warp runs every item and every named barrier; after a
+        // failed wait it only skips the work.
+        for (int i = 0; i < my_items; ++i) {
+            const int q0 = item_q0(i), h = item_h(i), hk = h / group;
+            const long long g0 = (long long)i * E;
+            const uint32_t ip = (uint32_t)(i & 1);
+            if (threadIdx.x >= ATTN_D && threadIdx.x < 2 * ATTN_D) {
+                const int c = threadIdx.x - ATTN_D;
+                sh->dv[c] = a.d != nullptr ? a.d[h * ATTN_D + c] : 0.f;
             }
-            if (a.dbg_codes != nullptr) {
-                uint8_t* dc = a.dbg_codes + ((size_t)h * a.L + q0 + row) * a.L + j * ATTN_TILE + col;
+            // pass 1: row maxima
+            float mx = -INFINITY;
+            for (int it = 0; it < nk && ok; ++it) {
+                int b, n;
+                sbuf(i, it, b, n);
+                if (!mbar_wait_bounded_warp(B(sh->s_full[b]), (uint32_t)(n & 1), abort)) { ok = false; break; }
+                tc_fence_after();
+                tmem_ld_32x32b_x32(tl + TM_S + b * ATTN_TILE + col, r);
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
                 #pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    dc[2 * k] = (uint8_t)__half2float(__ushort_as_half((uint16_t)(packed[k] & 0xFFFFu)));
-                    dc[2 * k + 1] = (uint8_t)__half2float(__ushort_as_half((uint16_t)(packed[k] >> 16)));
+                for (int k = 0; k < 32; ++k) mx = fmaxf(mx, __uint_as_float(r[k]));
+            }
+            if (threadIdx.x < ATTN_D) sh->tv[threadIdx.x] = a.t[hk * ATTN_D + threadIdx.x];  // V channel scales
+            sh->xm[part][row] = mx;
+            named_sync_softmax();
+            mx = fmaxf(fmaxf(sh->xm[0][row], sh->xm[1][row]), fmaxf(sh->xm[2][row], sh->xm[3][row]));
+            named_sync_softmax();
+            // pass 2: probabilities, their codes and the row sums
+            float lp[4] = {0.f, 0.f, 0.f, 0.f};      // partial row sums (independent chains)
+            for (int j = 0; j < nk && ok; ++j) {
+                int b, n;
+                sbuf(i, nk + j, b, n);
+                if (!mbar_wait_bounded_warp(B(sh->s_full[b]), (uint32_t)(n & 1), abort)) { ok = false; break; }
+                tc_fence_after();
+                tmem_ld_32x32b_x32(tl + TM_S + b * ATTN_TILE + col, r);
+                tmem_ld_wait();
+                // e = 2^((s - m) log2(e) / sqrt(d)); the code n = rne(255 e) in
+                // one rounding: the low halves of fma(255, e, ROUND_BIAS) are the
+                // fp16 values 1024 + n of two codes, and 1024 is subtracted
+                // exactly in fp16
+                uint32_t packed[16];
+                const __half2 minus1024 = __float2half2_rn(-1024.f);
+                #pragma unroll
+                for (int k = 0; k < 32; k += 2) {
+                    const float e0 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k]), mx), EXP_SCALE));
+                    const float e1 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k + 1]), mx), EXP_SCALE));
+                    lp[(k >> 1) & 1] += e0;
+                    lp[2 + ((k >> 1) & 1)] += e1;
+                    const uint32_t t0 = __float_as_uint(fmaf(255.f, e0, ROUND_BIAS));
+                    const uint32_t t1 = __float_as_uint(fmaf(255.f, e1, ROUND_BIAS));
+                    const uint32_t biased = prmt(t0, t1, 0x5410u);           // {1024 + n0, 1024 + n1}
+                    const __half2 hc = __hadd2(*reinterpret_cast<const __half2*>(&biased), minus1024);
+                    packed[k / 2] = *reinterpret_cast<const uint32_t*>(&hc);
                 }
-            }
-            // P over the S columns this warp has read
-            tmem_st_32x32b_x16(tl + TM_S + b * ATTN_TILE + col, packed);
-            tmem_st_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
-        }
-        sh->xm[part][row] = (lp[0] + lp[1]) + (lp[2] + lp[3]);
-        named_sync_softmax();
-        const float l = (sh->xm[0][row] + sh->xm[1][row]) + (sh->xm[2][row] + sh->xm[3][row]);
-        const float sp = __fdiv_rn(1.f, __fmul_rn(255.f, l));
-        // the head's power-of-two TAC scale: |Z_hat| <= 16 * 7 max_c t_c (the
-        // codes of a row sum to at most twice 255 l), brought into [2^13, 2^14)
-        float tmax = 0.f;
-        #pragma unroll
-        for (int c = lane; c < ATTN_D; c += 32) tmax = fmaxf(tmax, sh->tv[c]);
-        #pragma unroll
-        for (int m = 16; m > 0; m >>= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, m));
-        const int zk = tmax > 0.f ? ilogbf(112.f * tmax) - 13 : 0;
-        const float zscale = ldexpf(1.f, -zk), zunscale = ldexpf(1.f, zk);
-        if (a.dbg_l != nullptr && part == 0) a.dbg_l[(size_t)h * a.L + q0 + row] = l;
-        // epilogue 1: Z_hat = (acc sp) t as fp16 hi + lo, the A operands of
-        // the TAC product, into TMEM
-        ok = ok && mbar_wait_bounded_warp(B(sh->pv_done), 0, abort);
-        if (ok) {
-            tc_fence_after();
-            tmem_ld_32x32b_x32(tl + TM_O + col, r);
-            tmem_ld_wait();
-            if (a.dbg_acc != nullptr) {
-                int32_t* da = a.dbg_acc + ((size_t)h * a.L + q0 + row) * ATTN_D + col;
-                #pragma unroll
-                for (int k = 0; k < 32; ++k) da[k] = __float2int_rn(__uint_as_float(r[k]));
-            }
-            uint32_t hi[16], lo[16];
-            #pragma unroll
-            for (int k = 0; k < 32; k += 2) {
-                float z[2];
-                #pragma unroll
-                for (int u = 0; u < 2; ++u)
-                    z[u] = __fmul_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), sh->tv[col + k + u]), zscale);
-                const uint16_t h0 = bits_rn(__half(), z[0]), h1 = bits_rn(__half(), z[1]);
-                const uint16_t l0 = bits_rn(__half(), z[0] - from_bits(__half(), h0)),
-                               l1 = bits_rn(__half(), z[1] - from_bits(__half(), h1));
-                hi[k / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-                lo[k / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
-            }
-            tmem_st_32x32b_x16(tl + TM_ZHI + part * 16, hi);
-            tmem_st_32x32b_x16(tl + TM_ZLO + part * 16, lo);
-            tmem_st_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(B(sh->z_full));
-        }
-        // epilogue 2: + d, fp16, TMA store
-        ok = ok && mbar_wait_bounded_warp(B(sh->tac_done), 0, abort);
-        if (ok) {
-            tc_fence_after();
-            tmem_ld_32x32b_x32(tl + TM_TAC + col, r);
-            tmem_ld_wait();
-            const uint32_t box = sOut + (uint32_t)warp * 2048;
-            const bool add_d = a.d != nullptr;
-            #pragma unroll
-            for (int g = 0; g < 4; ++g) {
-                uint32_t w[4];
-                #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int k = 8 * g + 2 * u;
-                    float y0 = __fmul_rn(__uint_as_float(r[k]), zunscale), y1 = __fmul_rn(__uint_as_float(r[k + 1]), zunscale);
-                    if (add_d) {
-                        y0 = __fadd_rn(y0, sh->dv[col + k]);
-                        y1 = __fadd_rn(y1, sh->dv[col + k + 1]);
+                if (a.dbg_codes != nullptr) {
+                    uint8_t* dc = a.dbg_codes + ((size_t)h * a.L + q0 + row) * a.L + j * ATTN_TILE + col;
+                    #pragma unroll
+                    for (int k = 0; k < 16; ++k) {
+                        dc[2 * k] = (uint8_t)__half2float(__ushort_as_half((uint16_t)(packed[k] & 0xFFFFu)));
+                        dc[2 * k + 1] = (uint8_t)__half2float(__ushort_as_half((uint16_t)(packed[k] >> 16)));
                     }
-                    w[u] = pack2(T(), y0, y1);
                 }
-                st_shared_v4(box + lane * 64 + 16 * (g ^ ((lane >> 1) & 3)), w[0], w[1], w[2], w[3]);
+                // P over the S columns this warp has read
+                tmem_st_32x32b_x16(tl + TM_S + b * ATTN_TILE + col, packed);
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
             }
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                tma_store_2d(&tm_z, h * ATTN_D + col, q0 + quarter * 32, box);
-                bulk_commit();
-                bulk_wait_read0();           // the box has been read; the write completes with the grid
+            sh->xm[part][row] = (lp[0] + lp[1]) + (lp[2] + lp[3]);
+            named_sync_softmax();
+            const float l = (sh->xm[0][row] + sh->xm[1][row]) + (sh->xm[2][row] + sh->xm[3][row]);
+            const float sp = __fdiv_rn(1.f, __fmul_rn(255.f, l));
+            // the head's power-of-two TAC scale: |Z_hat| <= 16 * 7 max_c t_c (the
+            // codes of a row sum to at most twice 255 l), brought into [2^13, 2^14)
+            float tmax = 0.f;
+            #pragma unroll
+            for (int c = lane; c < ATTN_D; c += 32) tmax = fmaxf(tmax, sh->tv[c]);
+            #pragma unroll
+            for (int m = 16; m > 0; m >>= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, m));
+            const int zk = tmax > 0.f ? ilogbf(112.f * tmax) - 13 : 0;
+            const float zscale = ldexpf(1.f, -zk), zunscale = ldexpf(1.f, zk);
+            if (a.dbg_l != nullptr && part == 0) a.dbg_l[(size_t)h * a.L + q0 + row] = l;
+            // epilogue 1: Z_hat = (acc sp) t as fp16 hi + lo, the A operands of
+            // the TAC product, into TMEM
+            ok = ok && mbar_wait_bounded_warp(B(sh->pv_done), ip, abort);
+            if (ok) {
+                tc_fence_after();
+                tmem_ld_32x32b_x32(tl + TM_O + col, r);
+                tmem_ld_wait();
+                if (a.dbg_acc != nullptr) {
+                    int32_t* da = a.dbg_acc + ((size_t)h * a.L + q0 + row) * ATTN_D + col;
+                    #pragma unroll
+                    for (int k = 0; k < 32; ++k) da[k] = __float2int_rn(__uint_as_float(r[k]));
+                }
+                uint32_t hi[16], lo[16];
+                #pragma unroll
+                for (int k = 0; k < 32; k += 2) {
+                    float z[2];
+                    #pragma unroll
+                    for (int u = 0; u < 2; ++u)
+                        z[u] = __fmul_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), sh->tv[col + k + u]), zscale);
+                    const uint16_t h0 = bits_rn(__half(), z[0]), h1 = bits_rn(__half(), z[1]);
+                    const uint16_t l0 = bits_rn(__half(), z[0] - from_bits(__half(), h0)),
+                                   l1 = bits_rn(__half(), z[1] - from_bits(__half(), h1));
+                    hi[k / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+                    lo[k / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+                }
+                tmem_st_32x32b_x16(tl + TM_ZHI + part * 16, hi);
+                tmem_st_32x32b_x16(tl + TM_ZLO + part * 16, lo);
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(B(sh->z_full));
+                // every MMA reading Q has completed (pv_done), so the next
+                // item's Q goes in now, beside this item's TAC product
+                if (i + 1 < my_items) put_q(i + 1);
             }
-            __syncwarp();
+            // epilogue 2: + d, rounded to T, TMA store from the ring slot of
+            // entry 3 nk + 2
+            const long long go = g0 + 3 * nk + 2;
+            ok = ok && mbar_wait2_bounded_warp(B(sh->tac_done), ip, full_bar(go), use_parity(go), abort);
+            if (ok) {
+                tc_fence_after();
+                tmem_ld_32x32b_x32(tl + TM_TAC + col, r);
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(B(sh->tac_read));     // the TAC columns may be reused
+                const uint32_t box = slot(go) + (uint32_t)warp * 2048;
+                const bool add_d = a.d != nullptr;
+                #pragma unroll
+                for (int g = 0; g < 4; ++g) {
+                    uint32_t w[4];
+                    #pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int k = 8 * g + 2 * u;
+                        float y0 = __fmul_rn(__uint_as_float(r[k]), zunscale), y1 = __fmul_rn(__uint_as_float(r[k + 1]), zunscale);
+                        if (add_d) {
+                            y0 = __fadd_rn(y0, sh->dv[col + k]);
+                            y1 = __fadd_rn(y1, sh->dv[col + k + 1]);
+                        }
+                        w[u] = pack2(T(), y0, y1);
+                    }
+                    st_shared_v4(box + lane * 64 + 16 * (g ^ ((lane >> 1) & 3)), w[0], w[1], w[2], w[3]);
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&tm_z, h * ATTN_D + col, q0 + quarter * 32, box);
+                    bulk_commit();
+                    bulk_wait_read0();           // the box has been read; the write completes with the grid
+                }
+                __syncwarp();
+            }
+            // item boundary: every box of this slot has been read, and dv, tv
+            // and xm are free for the next item
+            named_sync_softmax();
+            if (ok && threadIdx.x == 0) mbar_arrive(empty_bar(go));
         }
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     }
@@ -668,7 +718,12 @@ cudaError_t launch_pv_tac(const AttnArgs& a, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     attn_vquant_kernel<T><<<Ckv / VQ_CH, 256, 0, stream>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    attn_pv_tac_kernel<T><<<dim3(a.L / ATTN_TILE, a.H), ATT_THREADS, ATT_SMEM, stream>>>(a, tk, tv, tz);
+    // persistent CTAs, one per SM at most, each with the same number of
+    // items (the last CTAs one fewer)
+    const int items = a.L / ATTN_TILE * a.H;
+    const int per_cta = (items + num_sms() - 1) / num_sms();
+    const int grid = (items + per_cta - 1) / per_cta;
+    attn_pv_tac_kernel<T><<<grid, ATT_THREADS, ATT_SMEM, stream>>>(a, tk, tv, tz);
     return cudaGetLastError();
 }
 

@@ -53,15 +53,15 @@ P = ctypes.c_void_p(4096)  # a non-null, 16-byte-aligned stand-in; never derefer
 
 
 @pytest.mark.parametrize("args,code", [
-    ((None, 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -1),   # NULL X
-    ((P, 9, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -1),      # dtype
-    ((P, 0, 4, 512, None, None, None, 512, 512, 0, 0, 6, P, P, None, None, None), -4),      # bits (4 or 8)
-    ((P, 0, 4, 100, None, None, None, 4, 100, 0, 0, 4, P, P, None, None, None), -2),        # K % 16
-    ((P, 0, 4, 512, None, None, None, 384, 512, 0, 0, 4, P, P, None, None, None), -2),      # hb not pow2
-    ((P, 0, 4, 512, None, None, None, 8192, 512, 0, 0, 4, P, P, None, None, None), -2),     # hb > K
-    ((P, 0, 4, 512, None, None, None, 512, 500, 6, 0, 4, P, P, None, None, None), -2),      # gate sum
-    ((P, 0, -1, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -2),     # L < 0
-    ((ctypes.c_void_p(4100), 0, 4, 512, None, None, None, 512, 512, 0, 0, 4, P, P, None, None, None), -3),
+    ((None, 0, 4, 512, None, None, None, 512, 512, 0, 0, None, 4, P, P, None, None, None), -1),   # NULL X
+    ((P, 9, 4, 512, None, None, None, 512, 512, 0, 0, None, 4, P, P, None, None, None), -1),      # dtype
+    ((P, 0, 4, 512, None, None, None, 512, 512, 0, 0, None, 6, P, P, None, None, None), -4),      # bits (4 or 8)
+    ((P, 0, 4, 100, None, None, None, 4, 100, 0, 0, None, 4, P, P, None, None, None), -2),        # K % 16
+    ((P, 0, 4, 512, None, None, None, 384, 512, 0, 0, None, 4, P, P, None, None, None), -2),      # hb not pow2
+    ((P, 0, 4, 512, None, None, None, 8192, 512, 0, 0, None, 4, P, P, None, None, None), -2),     # hb > K
+    ((P, 0, 4, 512, None, None, None, 512, 500, 6, 0, None, 4, P, P, None, None, None), -2),      # gate sum
+    ((P, 0, -1, 512, None, None, None, 512, 512, 0, 0, None, 4, P, P, None, None, None), -2),     # L < 0
+    ((ctypes.c_void_p(4100), 0, 4, 512, None, None, None, 512, 512, 0, 0, None, 4, P, P, None, None, None), -3),
 ])
 def test_quantize_act_validation(lib, args, code):
     assert lib.lib.sgat_quantize_act(*args) == code
@@ -95,21 +95,26 @@ def test_linear_workspace_by_bits(lib):
     assert lib.lib.sgat_linear_workspace_size_bits(L, K, 0, 6) == 0
 
 
+def W4(lib, *args):
+    """w4a4_gemm with out_tac = NULL (the argument before acc_dbg)."""
+    return lib.lib.w4a4_gemm(*args[:12], None, *args[12:])
+
+
 @pytest.mark.parametrize("L,N,K,code", [(4, 100, 512, -2), (4, 256, 200, -2), (4, 256, 131072, -2),
                                         (-1, 256, 512, -2)])
 def test_gemm_validation(lib, L, N, K, code):
-    assert lib.lib.w4a4_gemm(P, None, P, P, None, P, None, L, N, K, P, 0, None, None) == code
+    assert W4(lib, P, None, P, P, None, P, None, L, N, K, P, 0, None, None) == code
 
 
 def test_gemm_null_and_alignment(lib):
-    assert lib.lib.w4a4_gemm(None, None, P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -1
-    assert lib.lib.w4a4_gemm(P, None, P, None, None, P, None, 4, 256, 512, P, 0, None, None) == -1
+    assert W4(lib, None, None, P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -1
+    assert W4(lib, P, None, P, None, None, P, None, 4, 256, 512, P, 0, None, None) == -1
     # E4M3 weights need E4M3 activations when there are no packed weights
-    assert lib.lib.w4a4_gemm(P, None, P, None, P, P, None, 4, 256, 512, P, 0, None, None) == -1
-    assert lib.lib.w4a4_gemm(ctypes.c_void_p(4104), None, P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -3
-    assert lib.lib.w4a4_gemm(None, ctypes.c_void_p(4104), P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -3
-    assert lib.lib.w4a4_gemm(None, P, P, None, ctypes.c_void_p(4104), P, None, 4, 256, 512, P, 0, None, None) == -3
-    assert lib.lib.w4a4_gemm(P, None, P, P, None, P, None, 4, 256, 512, P, 7, None, None) == -1
+    assert W4(lib, P, None, P, None, P, P, None, 4, 256, 512, P, 0, None, None) == -1
+    assert W4(lib, ctypes.c_void_p(4104), None, P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert W4(lib, None, ctypes.c_void_p(4104), P, P, None, P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert W4(lib, None, P, P, None, ctypes.c_void_p(4104), P, None, 4, 256, 512, P, 0, None, None) == -3
+    assert W4(lib, P, None, P, P, None, P, None, 4, 256, 512, P, 7, None, None) == -1
 
 
 @pytest.mark.parametrize("N,K,code", [(-1, 512, -2), (4, 48, -2), (4, 16, -2)])
@@ -285,7 +290,7 @@ def test_validation_from_eight_threads(lib):
             barrier.wait()
             for it in range(200):
                 K = 100 + 16 * t                     # K % 16 != 0 for every t: a shape error
-                rc = lib_.sgat_quantize_act(P, 0, 4, K, None, None, None, 4, K, 0, 0, 4, P, P, None, None, None)
+                rc = lib_.sgat_quantize_act(P, 0, 4, K, None, None, None, 4, K, 0, 0, None, 4, P, P, None, None, None)
                 msg = lib_.starq_last_error().decode()
                 if rc != -2 or f"K={K}" not in msg:
                     errors.append((t, it, rc, msg))
@@ -307,3 +312,24 @@ def test_validation_from_eight_threads(lib):
     for th in threads:
         th.join()
     assert not errors, errors[:5]
+
+
+@pytest.mark.parametrize("g,M,Mp,scratch,dtype,code", [
+    (5, P, None, P, 0, -2),                          # block size
+    (64, None, None, P, 0, -1),                      # no M
+    (64, P, None, None, 0, -1),                      # no scratch buffer
+    (64, P, None, ctypes.c_void_p(4104), 0, -3),     # scratch alignment
+    (16, P, P, P, 0, -1),                            # prepared M only for g = 64 / 128
+    (64, P, P, P, 2, -1),                            # prepared M only for 16-bit tensors
+])
+def test_tac_option_validation(lib, g, M, Mp, scratch, dtype, code):
+    """The tac option of sgat_quantize_act (TAC on the input) and the out_tac
+    option of w4a4_gemm (TAC on the output) are validated before any launch."""
+    from paper_2606_04945_gb300.abi import StarqTac
+    v = lambda p: None if p is None else p.value
+    t = StarqTac(g, v(M), None, v(Mp), v(scratch))
+    assert lib.lib.sgat_quantize_act(P, dtype, 4, 512, None, None, None, 512, 512, 0, 0, ctypes.byref(t), 4, P, P,
+                                     None, None, None) == code
+    assert lib.lib.starq_last_error()
+    assert lib.lib.w4a4_gemm(P, None, P, P, None, P, None, 4, 256, 512, P, dtype, ctypes.byref(t), None,
+                             None) == (code if g != 5 else -2)

@@ -471,3 +471,61 @@ def test_empty_batch(abi):
     abi.w4_unpack_e4m3(torch.empty(0, K // 2, dtype=torch.uint8, device="cuda"),
                        torch.empty(0, K, dtype=torch.uint8, device="cuda"))
     abi.check_status()
+
+
+@pytest.mark.parametrize("L,K,g,dtype,prepared", [(300, 1024, 64, "f16", True), (129, 4096, 128, "bf16", False),
+                                                   (77, 512, 16, "f32", False)])
+def test_quantize_act_tac_option(abi, L, K, g, dtype, prepared):
+    """sgat_quantize_act with its tac option (Sec. 3.3: TAC on the attention
+    output before the output projection's quantiser): the compensated rows in
+    the scratch buffer within the TAC tolerance of the oracle's TAC, and the
+    codes, scales and E4M3 bytes bit-exact with the oracle's quantiser on
+    those rows (teacher-forced)."""
+    case = inputs.random_linear(L * 3 + g, L, K, 128, dtype=dtype, tac_g=g)
+    xf, tp = case.xf, case.tac
+    dt = H.torch_dtype(dtype)
+    X = H.dev(case.X, dt)
+    Md = H.dev(tp.M)
+    Mp = None
+    if prepared:
+        Mp = torch.empty(abi.tac_prepared_bytes(K, g), dtype=torch.uint8, device="cuda")
+        abi.tac_prepare(Md, g, dt, Mp)
+    scratch = torch.empty(L, K, dtype=dt, device="cuda")
+    Xq = torch.empty(L, K // 2, dtype=torch.uint8, device="cuda")
+    Xe = torch.empty(L, K, dtype=torch.uint8, device="cuda")
+    s_a = torch.empty(L, dtype=torch.float32, device="cuda")
+    abi.sgat_quantize_act(X, H.dev(case.mask), H.dev(xf.a_m), H.dev(xf.a_u), xf.hb, xf.d_sh, xf.d_m, xf.d_u, Xq, s_a,
+                          Xe=Xe, tac_M=Md, tac_d=H.dev(tp.d), tac_g=g, tac_Mp=Mp, tac_scratch=scratch)
+    abi.check_status()
+    z = H.host(scratch)
+    H.assert_tac_close(z, otac.tac_apply(case.X, tp.M, tp.d, g), dtype)
+    codes, s = osg.sgat_quantize_act(z, case.mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, 4)
+    assert np.array_equal(H.unpack(Xq), codes)
+    assert np.array_equal(H.host(s_a), s)
+    assert np.array_equal(H.host(Xe), H.e4m3_bytes(codes))
+
+
+@pytest.mark.parametrize("L,N,K,g,dtype", [(256, 512, 512, 128, "f16"), (100, 384, 1024, 32, "bf16")])
+def test_gemm_out_tac_option(abi, L, N, K, g, dtype):
+    """w4a4_gemm with its out_tac option: the dequantised output in the
+    scratch buffer within the output tolerance of the oracle, Y within the
+    TAC tolerance of the oracle's TAC of that scratch output
+    (teacher-forced), and the integer accumulators exact."""
+    qa, qw, s_a, s_w = H.gemm_codes(L + N + K, L, N, K)
+    rng = np.random.default_rng(g + L)
+    tp = inputs.make_tac(rng, N, g, noise=0.05)
+    dt = H.torch_dtype(dtype)
+    Xe = H.dev(H.e4m3_bytes(qa))
+    We = H.dev(H.e4m3_bytes(qw))
+    Wq = H.dev(osg.pack_int4(qw))
+    Y = torch.empty(L, N, dtype=dt, device="cuda")
+    scratch = torch.empty(L, N, dtype=dt, device="cuda")
+    acc = torch.empty(L, N, dtype=torch.int32, device="cuda")
+    abi.w4a4_gemm(None, H.dev(s_a), Wq, H.dev(s_w), Y, acc_dbg=acc, Xe=Xe, We=We, tac_M=H.dev(tp.M),
+                  tac_d=H.dev(tp.d), tac_g=g, tac_scratch=scratch)
+    abi.check_status()
+    ref_acc = osg.int_gemm(qa, qw)
+    assert np.array_equal(H.host(acc), ref_acc)
+    pre = H.host(scratch)
+    H.assert_output_close(pre, osg.dequant(ref_acc, s_a, s_w, None), dtype, what="pre-TAC output")
+    H.assert_tac_close(H.host(Y), otac.tac_apply(pre, tp.M, tp.d, g), dtype)
