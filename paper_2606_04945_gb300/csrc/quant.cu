@@ -211,8 +211,10 @@ __device__ __forceinline__ uint32_t pack8(const int* q) {
     return w;
 }
 
+// Up to 8 warps per row, or up to 20 when hb <= C (E = 16, at most two
+// chunks per warp; no stage crosses warps then).
 template <int E, int NC, typename Tin>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(E == 16 && NC <= 2 ? 640 : 256)
 sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
     extern __shared__ float qsm[];
     constexpr int C = 32 * E;
@@ -221,7 +223,7 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
     const int wr = warp % warps_per_row;                 // warp index within its row
     const int row = blockIdx.x * rows_per_cta + warp / warps_per_row;
     float* buf = qsm + warp * (C + 32);
-    float* red = qsm + (blockDim.x >> 5) * (C + 32);     // [warps] partial amax
+    float* red = qsm + (blockDim.x >> 5) * (C + 32);     // [32] partial amax, [32] partial -min
     const bool row_ok = row < a.L;
     const int K = a.K;
     const int nchunks = (K + C - 1) / C;   // a partial last chunk only when hb < 512
@@ -317,7 +319,7 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
     if (warps_per_row > 1) {
         if (lane == 0) {
             red[warp] = amax;
-            red[8 + warp] = nmin;
+            red[32 + warp] = nmin;
         }
         __syncthreads();
         amax = 0.f;
@@ -325,7 +327,7 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
         const int first = warp - wr;                     // first warp of this row
         for (int w = 0; w < warps_per_row; ++w) {
             amax = fmaxf(amax, red[first + w]);
-            nmin = fmaxf(nmin, red[8 + first + w]);
+            nmin = fmaxf(nmin, red[32 + first + w]);
         }
     }
     if (!row_ok) return;
@@ -416,7 +418,7 @@ template <> struct To<float> { static __device__ __forceinline__ float f(float h
 // of 4096 elements (four 1024-element chunks, chunk j of a round in warp j).
 // A warp reads its chunk of x and of the smoothing vector with coalesced
 // 16-byte loads (lane l at 16 l + 512 q) and passes each through its
-// shared slice to take it back in layout A (16 KB of shared memory per CTA,
+// shared slice to take it back in layout A (18 KB of shared memory per CTA,
 // so registers, not shared memory, bound the CTAs per SM).
 //
 //   layout A  lane l holds elements 32 l .. 32 l + 31 of its warp's chunk:
@@ -430,12 +432,16 @@ template <> struct To<float> { static __device__ __forceinline__ float f(float h
 //             eight consecutive codes per chunk pack into one 32-bit word.
 // Butterflies on pairs of registers use the packed f32x2 add and subtract
 // (each half rounds like the scalar operation). The shared slice of a chunk
-// holds its 32 x 32 floats with 16-byte column groups XOR-swizzled by the
-// row (row & 7), so the row-wise 16-byte accesses (layouts A and C) and the
-// column-wise 4-byte accesses (layout B) are all free of bank conflicts.
+// holds its 32 x 32 floats in rows of 36 (four floats of padding): row r
+// starts 4 r banks further on, so the row-wise 16-byte accesses (layouts A
+// and C, eight lanes per phase) and the column-wise 4-byte accesses (layout
+// B) are all free of bank conflicts, and every address is a per-thread base
+// plus a constant.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ int swz(int row, int col) {      // float index in a 32 x 32 slice
-    return row * 32 + ((((col >> 2) ^ (row & 7))) << 2) + (col & 3);
+constexpr int SROW = 36;                                   // floats per row of a 32 x 32 slice
+constexpr int SLICE = 32 * SROW;                           // floats per slice
+__device__ __forceinline__ int pad(int row, int col) {     // float index in a padded slice
+    return row * SROW + col;
 }
 
 // Two butterflies (a0, b0) and (a1, b1) with one packed add and one packed
@@ -509,7 +515,7 @@ __device__ __forceinline__ void pack_codes8(const float* qf, const int* qi, uint
 template <int NR, typename Tin, bool ASYM>
 __global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
 sgat_quant_rows_kernel(QuantArgs a) {
-    __shared__ __align__(16) float buf[4096];
+    __shared__ __align__(16) float buf[4 * SLICE];
     __shared__ float red[8];              // [0, 4) amax or X_max, [4, 8) -X_min (asym)
     grid_dependency_wait();            // launched with programmatic serialisation
     grid_launch_dependents();
@@ -522,7 +528,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
     const int own_lo = masked ? a.d_sh : a.d_sh + a.d_m;
     const int own_hi = masked ? a.d_sh + a.d_m : K;
     const Tin* X = static_cast<const Tin*>(a.X) + (size_t)row * K;
-    float* slice = buf + warp * 1024;
+    float* slice = buf + warp * SLICE;
 
     float v[NR][32];                      // layout C: v[R][8 j + k]
     float amax = 0.f, nmin = 0.f;         // asym: X_max and -X_min
@@ -566,7 +572,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 for (int q = 0; q < 8; ++q) xr[q] = __ldg(reinterpret_cast<const float4*>(X + c0) + lane + 32 * q);
                 #pragma unroll
                 for (int q = 0; q < 8; ++q)
-                    *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = xr[q];
+                    *reinterpret_cast<float4*>(slice + pad((lane >> 3) + 4 * q, 4 * (lane & 7))) = xr[q];
                 if (sm != nullptr) {
                     #pragma unroll
                     for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
@@ -574,7 +580,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 __syncwarp();
                 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
-                    const float4 w = *reinterpret_cast<const float4*>(slice + swz(lane, 4 * q));
+                    const float4 w = *reinterpret_cast<const float4*>(slice + pad(lane, 4 * q));
                     u[4 * q] = w.x; u[4 * q + 1] = w.y; u[4 * q + 2] = w.z; u[4 * q + 3] = w.w;
                 }
             }
@@ -582,11 +588,11 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 __syncwarp();                                    // x has left the slice
                 #pragma unroll
                 for (int q = 0; q < 8; ++q)
-                    *reinterpret_cast<float4*>(slice + swz((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
+                    *reinterpret_cast<float4*>(slice + pad((lane >> 3) + 4 * q, 4 * (lane & 7))) = sr[q];
                 __syncwarp();
                 #pragma unroll
                 for (int q = 0; q < 8; ++q) {
-                    const float4 w = *reinterpret_cast<const float4*>(slice + swz(lane, 4 * q));
+                    const float4 w = *reinterpret_cast<const float4*>(slice + pad(lane, 4 * q));
                     u[4 * q] = __fmul_rn(u[4 * q], w.x);
                     u[4 * q + 1] = __fmul_rn(u[4 * q + 1], w.y);
                     u[4 * q + 2] = __fmul_rn(u[4 * q + 2], w.z);
@@ -597,22 +603,22 @@ sgat_quant_rows_kernel(QuantArgs a) {
             reg_stages32(u, 1, 32);                              // h = 1 .. 16
             #pragma unroll
             for (int q = 0; q < 8; ++q)                          // layout A -> slice
-                *reinterpret_cast<float4*>(slice + swz(lane, 4 * q)) =
+                *reinterpret_cast<float4*>(slice + pad(lane, 4 * q)) =
                     make_float4(u[4 * q], u[4 * q + 1], u[4 * q + 2], u[4 * q + 3]);
             __syncwarp();
             #pragma unroll
-            for (int i = 0; i < 32; ++i) u[i] = slice[swz(i, lane)];   // layout B
+            for (int i = 0; i < 32; ++i) u[i] = slice[pad(i, lane)];   // layout B
             reg_stages32(u, 1, a.hb / 32);                       // h = 32 .. min(hb, 1024) / 2
             #pragma unroll
-            for (int i = 0; i < 32; ++i) slice[swz(i, lane)] = u[i];
+            for (int i = 0; i < 32; ++i) slice[pad(i, lane)] = u[i];
         }
         __syncthreads();
         #pragma unroll
         for (int j = 0; j < 4; ++j) {                            // layout C
             if (j < nch) {
                 const int r = warp * 8 + (lane >> 2), c = (lane & 3) * 8;
-                const float4 p0 = *reinterpret_cast<const float4*>(buf + j * 1024 + swz(r, c));
-                const float4 p1 = *reinterpret_cast<const float4*>(buf + j * 1024 + swz(r, c + 4));
+                const float4 p0 = *reinterpret_cast<const float4*>(buf + j * SLICE + pad(r, c));
+                const float4 p1 = *reinterpret_cast<const float4*>(buf + j * SLICE + pad(r, c + 4));
                 v[R][8 * j] = p0.x; v[R][8 * j + 1] = p0.y; v[R][8 * j + 2] = p0.z; v[R][8 * j + 3] = p0.w;
                 v[R][8 * j + 4] = p1.x; v[R][8 * j + 5] = p1.y; v[R][8 * j + 6] = p1.z; v[R][8 * j + 7] = p1.w;
             } else {
@@ -762,11 +768,17 @@ template <int E, typename Tin>
 cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
     constexpr int C = 32 * E;
     const int n = (a.K + C - 1) / C;                 // chunks per row
-    const int wpr = n < 8 ? n : 8;                   // warps per row (a multiple of hb / C)
+    int wpr, nc;                                     // warps per row, rounds
+    if (E == 16 && a.hb <= C && n > 8) {             // no stage crosses warps: up to 20 warps, 2 rounds
+        nc = (n + 19) / 20;
+        wpr = (n + nc - 1) / nc;
+    } else {
+        wpr = n < 8 ? n : 8;                         // a multiple of hb / C
+        nc = (n + wpr - 1) / wpr;
+    }
     const int rpc = wpr <= 4 ? 8 / wpr : 1;          // rows per CTA
-    const int nc = (n + wpr - 1) / wpr;              // rounds
     const int warps = wpr * rpc;
-    const size_t smem = (size_t)warps * (C + 32) * 4 + 16 * 4;
+    const size_t smem = (size_t)warps * (C + 32) * 4 + 64 * 4;
     dim3 grid((a.L + rpc - 1) / rpc), block(32 * warps);
     #define STARQ_QUANT_LAUNCH(NCV)                                                            \
         {                                                                                      \

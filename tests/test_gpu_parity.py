@@ -54,6 +54,10 @@ QUANT_CASES = [
     (11, 5120, 1024, "f32", True),        # last round holds one chunk
     (4, 6144, 2048, "f16", False),        # last round holds one 2048 block
     (3, 20480, 4096, "f16", True),        # beyond 16384 features: warp-per-chunk kernel
+    # warp-per-chunk rows: a half last 1024-chunk, small blocks, 20 warps per row
+    (20, 1536, 64, "f32", True),
+    (13, 2560, 1, "f16", False),
+    (7, 20480, 512, "bf16", True),
 ]
 
 
