@@ -421,6 +421,233 @@ tac_tc_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __gri
     if (warp == 0) tmem_dealloc(tmem, P::TMEM_COLS);
 }
 
+// ---------------------------------------------------------------------------
+// Streaming tensor-core TAC (prepared M, 16-bit Z, g = 64 or 128): the same
+// products as tac_tc_kernel, in the same order, so the same bits. Persistent
+// CTAs each take a contiguous run of the (block b, 128-token tile) jobs in
+// block-major order, at most two blocks per run:
+//   TMA warp   M_b's halves once per block (one bulk copy; the second block's
+//              after the MMAs of the first have completed), then the Z tiles
+//              through a ring of ZS stages;
+//   MMA warp   per tile 2 g / 16 MMAs (Z M_hi^T, Z M_lo^T per K step) into one
+//              of two TMEM accumulators;
+//   8 warps    read the accumulator (a TMEM lane quarter, half the columns),
+//              free it, add d_b, round to the output type and store 32 x 32
+//              boxes by TMA from two staging boxes per warp.
+// Loads, products and stores of consecutive tiles overlap.
+// ---------------------------------------------------------------------------
+constexpr int TS_EPI_WARPS = 8;
+constexpr int TS_TMA_WARP = TS_EPI_WARPS, TS_MMA_WARP = TS_EPI_WARPS + 1;
+constexpr int TS_THREADS = (TS_EPI_WARPS + 2) * 32;
+
+template <int G, typename TOut>
+struct TacStream {
+    static constexpr int ATOMS = G / 64;
+    static constexpr int Z_BYTES = TC_TM * G * 2;
+    static constexpr int M_BYTES = G * G * 2;                          // one half
+    static constexpr int BOX_BYTES = 32 * 32 * (int)sizeof(TOut);
+    static constexpr int ZS = sizeof(TOut) == 4 ? 2 : 3;               // Z ring stages
+    static constexpr int OFF_Z = 2 * M_BYTES;
+    static constexpr int OFF_BOX = OFF_Z + ZS * Z_BYTES;
+    static constexpr size_t SMEM = (size_t)OFF_BOX + (size_t)TS_EPI_WARPS * 2 * BOX_BYTES + 1024;
+    static constexpr int TMEM_COLS = 2 * G;
+    static_assert(SMEM <= 227 * 1024, "shared memory");
+};
+
+template <int G, typename TIn, typename TOut>
+__global__ void __launch_bounds__(TS_THREADS, 1)
+tac_stream_kernel(TacArgs a, const __grid_constant__ CUtensorMap tmap_z, const __grid_constant__ CUtensorMap tmap_out,
+                  unsigned* status, int nt, long long jobs) {
+    using P = TacStream<G, TOut>;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t zfull[P::ZS], zempty[P::ZS], accfull[2], accempty[2], mfull, mempty;
+    __shared__ __align__(16) float dsm[2][G];
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_flag;
+    const uint32_t raw = smem_addr(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    const uint32_t sMh = base, sMl = base + P::M_BYTES;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    volatile int* abort = &abort_flag;
+    auto B = [](const uint64_t& bar) { return smem_addr(&bar); };
+    // this CTA's jobs [j0, j1): block j / nt, tile j mod nt
+    const long long j0 = jobs * blockIdx.x / gridDim.x, j1 = jobs * (blockIdx.x + 1) / gridDim.x;
+    const int n = (int)(j1 - j0);
+    const int b0 = (int)(j0 / nt);
+
+    if (threadIdx.x == 0) {
+        for (int k = 0; k < P::ZS; ++k) {
+            mbar_init(B(zfull[k]), 1);
+            mbar_init(B(zempty[k]), 1);
+        }
+        for (int k = 0; k < 2; ++k) {
+            mbar_init(B(accfull[k]), 1);
+            mbar_init(B(accempty[k]), TS_EPI_WARPS);
+        }
+        mbar_init(B(mfull), 1);
+        mbar_init(B(mempty), 1);
+        abort_flag = 0;
+        mbar_fence_init();
+    }
+    if (warp == TS_MMA_WARP) {
+        tmem_alloc(smem_addr(&tmem_slot), P::TMEM_COLS);
+        tmem_relinquish();
+    }
+    grid_dependency_wait();            // launched with programmatic serialisation
+    grid_launch_dependents();
+    // d of the run's (at most two) blocks
+    for (int i = threadIdx.x; i < 2 * G; i += blockDim.x) {
+        const int bb = b0 + i / G;
+        dsm[i / G][i % G] = (a.d != nullptr && bb < a.C / G) ? a.d[(size_t)bb * G + i % G] : 0.f;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == TS_TMA_WARP) {
+        bool ok = true;
+        if (elect_one()) {
+            int mb = -1, mloads = 0;
+            for (int i = 0; i < n && ok; ++i) {
+                const long long j = j0 + i;
+                const int b = (int)(j / nt), t = (int)(j % nt);
+                if (b != mb) {                               // the block's M halves (after the previous block's MMAs)
+                    if (mloads > 0 && !mbar_wait_bounded(B(mempty), (uint32_t)((mloads - 1) & 1), abort)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(B(mfull), 2 * P::M_BYTES);
+                    bulk_load(sMh, static_cast<const uint8_t*>(a.Mp) + (size_t)b * 2 * P::M_BYTES, 2 * P::M_BYTES,
+                              B(mfull));
+                    mb = b;
+                    ++mloads;
+                }
+                const int k = i % P::ZS;
+                if (!mbar_wait_bounded(B(zempty[k]), (uint32_t)(((i / P::ZS) & 1) ^ 1), abort)) { ok = false; break; }
+                const uint32_t sZ = base + P::OFF_Z + (uint32_t)k * P::Z_BYTES;
+                mbar_arrive_expect_tx(B(zfull[k]), P::Z_BYTES);
+                for (int at = 0; at < P::ATOMS; ++at)
+                    tma_load_2d(sZ + at * (TC_TM * 128), &tmap_z, b * G + at * 64, t * TC_TM, B(zfull[k]));
+            }
+            // the last commits on the Z ring have arrived before the CTA exits
+            for (int i = n - P::ZS; i < n && ok; ++i)
+                if (i >= 0) ok = mbar_wait_bounded(B(zempty[i % P::ZS]), (uint32_t)((i / P::ZS) & 1), abort);
+            if (!ok) { *abort = 1; atomicOr(status, STATUS_TIMEOUT_TAC); }
+        }
+        __syncwarp();
+    } else if (warp == TS_MMA_WARP) {
+        if (elect_one()) {
+            constexpr uint32_t IDESC = (1u << 4) | (Split16<TIn>::KIND << 7) | (Split16<TIn>::KIND << 10) |
+                                       ((uint32_t)(G >> 3) << 17) | ((uint32_t)(TC_TM >> 4) << 24);
+            bool ok = true;
+            int mb = -1, mloads = 0, issued = 0;
+            for (int i = 0; i < n && ok; ++i) {
+                const int b = (int)((j0 + i) / nt);
+                if (b != mb) {
+                    if (mloads > 0) tc_commit(B(mempty));      // the previous block's MMAs done with M
+                    if (!mbar_wait_bounded(B(mfull), (uint32_t)(mloads & 1), abort)) { ok = false; break; }
+                    mb = b;
+                    ++mloads;
+                }
+                const int k = i % P::ZS, acc = i & 1;
+                if (!mbar_wait_bounded(B(zfull[k]), (uint32_t)((i / P::ZS) & 1), abort) ||
+                    !mbar_wait_bounded(B(accempty[acc]), (uint32_t)(((i >> 1) & 1) ^ 1), abort)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sZ = base + P::OFF_Z + (uint32_t)k * P::Z_BYTES;
+                #pragma unroll
+                for (int ks = 0; ks < G / 16; ++ks) {
+                    const uint32_t koff = (ks / 4) * (TC_TM * 128) + (ks % 4) * 32;
+                    const uint32_t moff = (ks / 4) * (G * 128) + (ks % 4) * 32;
+                    const uint64_t ad = smem_desc_sw128(sZ + koff);
+                    mma_f16(tmem + (uint32_t)(acc * G), ad, smem_desc_sw128(sMh + moff), IDESC, ks > 0 ? 1u : 0u);
+                    mma_f16(tmem + (uint32_t)(acc * G), ad, smem_desc_sw128(sMl + moff), IDESC, 1u);
+                }
+                tc_commit(B(zempty[k]));
+                tc_commit(B(accfull[acc]));
+                ++issued;
+            }
+            if (issued > 0) {                 // every MMA has completed before TMEM is released
+                volatile int never = 0;
+                if (!mbar_wait_bounded(B(accfull[(issued - 1) & 1]), (uint32_t)(((issued - 1) >> 1) & 1), &never))
+                    ok = false;
+            }
+            if (!ok) { *abort = 1; atomicOr(status, STATUS_TIMEOUT_TAC); }
+        }
+        __syncwarp();
+    } else {
+        const int quarter = warp & 3, chalf = warp >> 2;
+        const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+        const uint32_t boxes = base + P::OFF_BOX + (uint32_t)warp * 2 * P::BOX_BYTES;
+        int stores = 0;
+        bool ok = true;
+        for (int i = 0; i < n && ok; ++i) {
+            const long long j = j0 + i;
+            const int b = (int)(j / nt), t = (int)(j % nt);
+            const int acc = i & 1;
+            if (!mbar_wait_bounded_warp(B(accfull[acc]), (uint32_t)((i >> 1) & 1), abort)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t r[G / 64][32];
+            #pragma unroll
+            for (int c = 0; c < G / 64; ++c)
+                tmem_ld_32x32b_x32(trow + (uint32_t)(acc * G + chalf * (G / 2) + c * 32), r[c]);
+            tmem_ld_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(B(accempty[acc]));      // the accumulator may take the next tile
+            const float* dd = dsm[b - b0];
+            #pragma unroll
+            for (int c = 0; c < G / 64; ++c) {
+                const int col = chalf * (G / 2) + c * 32;
+                float v[32];
+                #pragma unroll
+                for (int q = 0; q < 32; ++q) v[q] = __uint_as_float(r[c][q]) + dd[col + q];
+                const uint32_t box = boxes + (uint32_t)(stores & 1) * P::BOX_BYTES;
+                if (stores >= 2) {                               // the store from this box two boxes ago has read it
+                    if (lane == 0) bulk_wait_read1();
+                    __syncwarp();
+                }
+                if (sizeof(TOut) == 4) {                         // 128-byte rows: group q at q ^ (row & 7)
+                    #pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        st_shared_v4(box + lane * 128 + ((q ^ (lane & 7)) << 4), __float_as_uint(v[4 * q]),
+                                     __float_as_uint(v[4 * q + 1]), __float_as_uint(v[4 * q + 2]),
+                                     __float_as_uint(v[4 * q + 3]));
+                } else {                                         // 64-byte rows: group q at q ^ ((row >> 1) & 3)
+                    #pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint32_t w[4];
+                        #pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            TOut x0 = from_f<TOut>(v[8 * q + 2 * e]), x1 = from_f<TOut>(v[8 * q + 2 * e + 1]);
+                            w[e] = (uint32_t)(*reinterpret_cast<uint16_t*>(&x0)) |
+                                   ((uint32_t)(*reinterpret_cast<uint16_t*>(&x1)) << 16);
+                        }
+                        st_shared_v4(box + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4), w[0], w[1], w[2], w[3]);
+                    }
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&tmap_out, b * G + col, t * TC_TM + quarter * 32, box);
+                    bulk_commit();
+                }
+                ++stores;
+            }
+        }
+        if (lane == 0) bulk_wait0();
+        __syncwarp();
+        if (!ok && lane == 0) { *abort = 1; atomicOr(status, STATUS_TIMEOUT_TAC); }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == TS_MMA_WARP) tmem_dealloc(tmem, P::TMEM_COLS);
+}
+
 bool encode_u16_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
                      uint32_t box_cols) {
     const PFN_cuTensorMapEncodeTiled_v12000 fn = tensor_map_encoder();
@@ -477,10 +704,48 @@ cudaError_t launch_tc(const TacArgs& a, cudaStream_t stream) {
     return cudaLaunchKernelEx(&cfg, tac_tc_kernel<G, TIn, TOut>, a, tz, to, a.status);
 }
 
+template <int G, typename TIn, typename TOut>
+cudaError_t launch_stream(const TacArgs& a, cudaStream_t stream) {
+    using P = TacStream<G, TOut>;
+    static DeviceCache<int> attr;
+    int done = 0;
+    const cudaError_t e = attr.get(&done, [](int, int* v) {
+        *v = 1;
+        return cudaFuncSetAttribute(tac_stream_kernel<G, TIn, TOut>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)P::SMEM);
+    });
+    if (e != cudaSuccess) return e;
+    CUtensorMap tz, to;
+    if (!encode_u16_tmap(&tz, a.Z, (uint64_t)a.L, (uint64_t)a.C, TC_TM, 64)) return cudaErrorInvalidValue;
+    if (!encode_out_tmap16or32(&to, a.out, sizeof(TOut), std::is_same<TOut, __half>::value, (uint64_t)a.L,
+                               (uint64_t)a.C))
+        return cudaErrorInvalidValue;
+    // at least one CTA per block, so that a CTA's run of jobs (at most nt
+    // long) spans at most two blocks
+    const int nb = a.C / G, nt = (a.L + TC_TM - 1) / TC_TM;
+    const long long jobs = (long long)nb * nt;
+    long long ctas = jobs < num_sms() ? jobs : num_sms();
+    if (ctas < nb) ctas = nb;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1] = {pdl_attribute()};
+    cfg.gridDim = dim3((unsigned)ctas);
+    cfg.blockDim = dim3(TS_THREADS);
+    cfg.dynamicSmemBytes = P::SMEM;
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, tac_stream_kernel<G, TIn, TOut>, a, tz, to, a.status, nt, jobs);
+}
+
 template <typename TIn, typename TOut>
 cudaError_t launch_io(const TacArgs& a, cudaStream_t stream) {
     if constexpr (!std::is_same<TIn, float>::value) {
         if (a.status != nullptr && (a.g == 64 || a.g == 128)) {
+            // prepared halves and more jobs than one wave of the per-tile
+            // kernel (two CTAs per SM) holds: the streaming kernel
+            const long long jobs = (long long)(a.C / a.g) * ((a.L + TC_TM - 1) / TC_TM);
+            if (a.Mp != nullptr && jobs > 2LL * num_sms())
+                return a.g == 64 ? launch_stream<64, TIn, TOut>(a, stream) : launch_stream<128, TIn, TOut>(a, stream);
             return a.g == 64 ? launch_tc<64, TIn, TOut>(a, stream) : launch_tc<128, TIn, TOut>(a, stream);
         }
     }

@@ -281,7 +281,11 @@ def test_w4a4_gemm_adversarial_exactness(abi, K, path):
 @pytest.mark.parametrize("g,L,C,zin,zout", [(4, 33, 64, "f16", "f32"), (8, 100, 256, "f16", "f16"),
                                             (16, 1025, 512, "bf16", "f32"), (32, 7, 96, "f32", "f32"),
                                             (64, 256, 512, "f16", "f32"), (128, 130, 4096, "f16", "f32"),
-                                            (128, 64, 4096, "bf16", "bf16")])
+                                            (128, 64, 4096, "bf16", "bf16"),
+                                            # more jobs than one wave: the streaming kernel with prepared
+                                            # halves (runs crossing block boundaries, a ragged last tile)
+                                            (128, 1407, 4096, "f16", "f16"), (64, 1201, 2048, "bf16", "f32"),
+                                            (128, 8192, 3584, "bf16", "bf16")])
 def test_tac_apply(abi, g, L, C, zin, zout):
     rng = np.random.default_rng(g * 1000 + L)
     Z = rng.standard_normal((L, C)).astype(np.float32)
