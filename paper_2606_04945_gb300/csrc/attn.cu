@@ -297,10 +297,12 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
     // memory and is reloaded after every asm with a memory clobber)
     auto B = [](const uint64_t& bar) { return smem_addr(&bar); };
     const int E = 3 * nk + 3;                                // ring entries per item
-    auto slot = [=](long long g) { return base + (uint32_t)(g % ATT_SLOTS) * TILE_BYTES; };
-    auto full_bar = [=](long long g) { return B(sh->full[g % ATT_SLOTS]); };
-    auto empty_bar = [=](long long g) { return B(sh->empty[g % ATT_SLOTS]); };
-    auto use_parity = [](long long g) { return (uint32_t)((g / ATT_SLOTS) & 1); };
+    // (entry indices stay below 2^31: at most 64 key chunks per head and
+    // a few thousand items per CTA; 32-bit division by a constant is cheap)
+    auto slot = [=](int g) { return base + ((uint32_t)g % ATT_SLOTS) * TILE_BYTES; };
+    auto full_bar = [=](int g) { return B(sh->full[(uint32_t)g % ATT_SLOTS]); };
+    auto empty_bar = [=](int g) { return B(sh->empty[(uint32_t)g % ATT_SLOTS]); };
+    auto use_parity = [](int g) { return ((uint32_t)g / ATT_SLOTS) & 1u; };
     auto item_q0 = [=](int i) { return ((int)blockIdx.x + i * (int)gridDim.x) % nk * ATTN_TILE; };
     auto item_h = [=](int i) { return ((int)blockIdx.x + i * (int)gridDim.x) / nk; };
     // S buffer of Q K^T number it of item i (pass 1: it = 0 .. nk-1, three
@@ -351,7 +353,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         for (int i = 0; i < my_items && ok; ++i) {
             const int h = item_h(i), hk = h / group;
             for (int u = 0; u < E && ok; ++u) {
-                const long long g = (long long)i * E + u;
+                const int g = i * E + u;
                 if (!mbar_wait_bounded_warp(empty_bar(g), use_parity(g) ^ 1u, abort)) { ok = false; break; }
                 const uint32_t dst = slot(g), fb = full_bar(g);
                 if (elect_one()) {
@@ -383,8 +385,8 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         }
         // every slot's last use has been given back, so no commit or arrive
         // lands after this CTA has exited
-        const long long G = (long long)my_items * E;
-        for (long long g = G - ATT_SLOTS; g < G && ok; ++g)
+        const int G = my_items * E;
+        for (int g = G - ATT_SLOTS; g < G && ok; ++g)
             if (g >= 0) ok = mbar_wait_bounded_warp(empty_bar(g), use_parity(g), abort);
         if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_ATTN); }
     } else if (warp == ATT_MMA_WARP) {
@@ -413,7 +415,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         int tac_commits = 0;
         tc_fence_after();
         for (int i = 0; i < my_items && ok; ++i) {
-            const long long g0 = (long long)i * E;
+            const int g0 = i * E;
             // Q in TMEM; for i > 0 the previous TAC accumulator read out
             ok = i == 0 ? mbar_wait_bounded_warp(B(sh->q_full), 0, abort)
                         : mbar_wait2_bounded_warp(B(sh->q_full), (uint32_t)(i & 1), B(sh->tac_read),
@@ -424,7 +426,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             // (the MMAs of one thread run in issue order). For pass-2 chunks
             // from 2 on, that P V^T's own wait has already seen the P written.
             auto qk = [=](int it) -> bool {
-                const long long g = g0 + (it < nk ? it : nk + 2 * (it - nk));
+                const int g = g0 + (it < nk ? it : nk + 2 * (it - nk));
                 int b, n;
                 sbuf(i, it, b, n);
                 if (!(it >= nk + 2 ? mbar_wait_bounded_warp(full_bar(g), use_parity(g), abort)
@@ -442,7 +444,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             };
             // P V^T of pass-2 chunk j, once its P is in its S buffer
             auto pv = [=](int j) -> bool {
-                const long long g = g0 + nk + 2 * j + 1;
+                const int g = g0 + nk + 2 * j + 1;
                 int b, n;
                 sbuf(i, nk + j, b, n);
                 if (!mbar_wait2_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1), full_bar(g), use_parity(g), abort))
@@ -463,7 +465,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             if (ok) ok = pv(nk - 1);
             if (elect_one()) tc_commit(B(sh->pv_done));
             __syncwarp();
-            const long long gm = g0 + 3 * nk;               // M_hi; M_lo at gm + 1
+            const int gm = g0 + 3 * nk;               // M_hi; M_lo at gm + 1
             ok = ok && mbar_wait2_bounded_warp(B(sh->z_full), (uint32_t)(i & 1), full_bar(gm), use_parity(gm), abort) &&
                  mbar_wait_bounded_warp(full_bar(gm + 1), use_parity(gm + 1), abort);
             tc_fence_after();
@@ -516,7 +518,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         // failed wait it only skips the work.
         for (int i = 0; i < my_items; ++i) {
             const int q0 = item_q0(i), h = item_h(i), hk = h / group;
-            const long long g0 = (long long)i * E;
+            const int g0 = i * E;
             const uint32_t ip = (uint32_t)(i & 1);
             if (threadIdx.x >= ATTN_D && threadIdx.x < 2 * ATTN_D) {
                 const int c = threadIdx.x - ATTN_D;
@@ -635,7 +637,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             }
             // epilogue 2: + d, rounded to T, TMA store from the ring slot of
             // entry 3 nk + 2
-            const long long go = g0 + 3 * nk + 2;
+            const int go = g0 + 3 * nk + 2;
             ok = ok && mbar_wait2_bounded_warp(B(sh->tac_done), ip, full_bar(go), use_parity(go), abort);
             if (ok) {
                 tc_fence_after();
