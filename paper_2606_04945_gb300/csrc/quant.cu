@@ -414,8 +414,10 @@ template <> struct To<float> { static __device__ __forceinline__ float f(float h
 
 // ---------------------------------------------------------------------------
 // Rows with Hadamard blocks of 1024 elements or more (hb >= 1024, K a
-// multiple of 1024, K <= 4096 NR): one CTA of four warps per row, in rounds
-// of 4096 elements (four 1024-element chunks, chunk j of a round in warp j).
+// multiple of 1024, K <= 4096 NR), or of at most 512 (1024 <= K <= 4096,
+// K % 512 == 0, a last chunk of 512 allowed): one CTA of four warps per
+// row, in rounds of 4096 elements (four 1024-element chunks, chunk j of a
+// round in warp j).
 // A warp reads its chunk of x and of the smoothing vector with coalesced
 // 16-byte loads (lane l at 16 l + 512 q) and passes each through its
 // shared slice to take it back in layout A (18 KB of shared memory per CTA,
@@ -535,18 +537,23 @@ sgat_quant_rows_kernel(QuantArgs a) {
     #pragma unroll
     for (int R = 0; R < NR; ++R) {
         const int base = R * 4096;
-        const int nch = min(4, (K - base) >> 10);        // chunks in this round (>= 1)
+        const int nch = min(4, (K - base + 1023) >> 10); // chunks in this round (>= 1)
         float u[32];
         if (warp < nch) {
             // coalesced loads (lane l: 16 bytes at 16 l + 512 q); x and then
             // the smoothing vector pass through the warp's slice and come
             // back in layout A
             const int c0 = base + warp * 1024;                   // first element of the chunk
+            // a last chunk of 512 (hb <= 512 only): the upper half is zeros,
+            // its own Hadamard blocks, never stored
+            const bool half = K - c0 < 1024;
             float4 sr[8];
             if (sizeof(Tin) == 2) {
                 uint4 xr[4];
                 #pragma unroll
-                for (int q = 0; q < 4; ++q) xr[q] = __ldg(reinterpret_cast<const uint4*>(X + c0) + lane + 32 * q);
+                for (int q = 0; q < 4; ++q)
+                    xr[q] = (!half || q < 2) ? __ldg(reinterpret_cast<const uint4*>(X + c0) + lane + 32 * q)
+                                             : make_uint4(0u, 0u, 0u, 0u);
                 // 16-bit staging: 32 rows of 64 bytes, 16-byte group g of row R at g ^ ((R >> 1) & 3)
                 uint8_t* st8 = reinterpret_cast<uint8_t*>(slice);
                 #pragma unroll
@@ -556,7 +563,9 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 }
                 if (sm != nullptr) {
                     #pragma unroll
-                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
+                    for (int q = 0; q < 8; ++q)
+                        sr[q] = (!half || q < 4) ? __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q)
+                                                 : make_float4(0.f, 0.f, 0.f, 0.f);
                 }
                 __syncwarp();
                 #pragma unroll
@@ -569,13 +578,17 @@ sgat_quant_rows_kernel(QuantArgs a) {
             } else {
                 float4 xr[8];
                 #pragma unroll
-                for (int q = 0; q < 8; ++q) xr[q] = __ldg(reinterpret_cast<const float4*>(X + c0) + lane + 32 * q);
+                for (int q = 0; q < 8; ++q)
+                    xr[q] = (!half || q < 4) ? __ldg(reinterpret_cast<const float4*>(X + c0) + lane + 32 * q)
+                                             : make_float4(0.f, 0.f, 0.f, 0.f);
                 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     *reinterpret_cast<float4*>(slice + pad((lane >> 3) + 4 * q, 4 * (lane & 7))) = xr[q];
                 if (sm != nullptr) {
                     #pragma unroll
-                    for (int q = 0; q < 8; ++q) sr[q] = __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q);
+                    for (int q = 0; q < 8; ++q)
+                        sr[q] = (!half || q < 4) ? __ldg(reinterpret_cast<const float4*>(sm + c0) + lane + 32 * q)
+                                                 : make_float4(0.f, 0.f, 0.f, 0.f);
                 }
                 __syncwarp();
                 #pragma unroll
@@ -600,7 +613,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
                 }
             }
             __syncwarp();
-            reg_stages32(u, 1, 32);                              // h = 1 .. 16
+            reg_stages32(u, 1, a.hb < 32 ? a.hb : 32);          // h = 1 .. min(hb, 32) / 2
             #pragma unroll
             for (int q = 0; q < 8; ++q)                          // layout A -> slice
                 *reinterpret_cast<float4*>(slice + pad(lane, 4 * q)) =
@@ -644,7 +657,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
         #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int e0 = base + j * 1024 + warp * 256 + 8 * lane;    // first element of the group
-            if (j >= nch) continue;
+            if (j >= nch || e0 >= K) continue;
             const bool all_keep = (e0 + 8 <= a.d_sh) || (e0 >= own_lo && e0 + 8 <= own_hi);
             if (!all_keep) {
                 #pragma unroll
@@ -703,11 +716,11 @@ sgat_quant_rows_kernel(QuantArgs a) {
     #pragma unroll
     for (int R = 0; R < NR; ++R) {
         const int base = R * 4096;
-        const int nch = min(4, (K - base) >> 10);
+        const int nch = min(4, (K - base + 1023) >> 10);
         #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            if (j >= nch) continue;
             const int e0 = base + j * 1024 + warp * 256 + 8 * lane;
+            if (j >= nch || e0 >= K) continue;
             float qf[8];
             int qi[8];
             #pragma unroll
@@ -810,6 +823,9 @@ cudaError_t launch_typed(const QuantArgs& a, cudaStream_t stream) {
     // chunk is 1024 elements (hb >= 1024, blocks finish across warps) or 512
     // elements holding 512 / hb blocks
     if (a.hb >= 1024 && a.K % 1024 == 0 && a.K <= 16384) return launch_rows<Tin>(a, stream);
+    // blocks of up to 512 in rows of 1024 to 4096 features, K % 512 == 0:
+    // the same kernel, a last chunk of 512 allowed
+    if (a.hb <= 512 && a.K >= 1024 && a.K <= 4096 && a.K % 512 == 0) return launch_rows_nr<1, Tin>(a, stream);
     return a.hb >= 1024 ? launch_e<32, Tin>(a, stream) : launch_e<16, Tin>(a, stream);
 }
 
