@@ -512,18 +512,30 @@ __device__ __forceinline__ void pack_codes8(const float* qf, const int* qi, uint
     e4.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
 }
 
+__device__ __forceinline__ float ld_shared_cluster_f32(uint32_t cluster_addr) {
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(cluster_addr) : "memory");
+    return v;
+}
+
 // ASYM: the asymmetric mode (a compile-time copy, so that the symmetric
-// kernel carries none of its reductions)
-template <int NR, typename Tin, bool ASYM>
+// kernel carries none of its reductions). CL > 1 (with NR = 1): a cluster
+// of CL CTAs per row, CTA r taking the row's features 4096 r .. 4096 r +
+// 4095; the CTAs exchange their maxima through distributed shared memory,
+// so no thread holds more than one 4096-feature slice.
+template <int NR, typename Tin, bool ASYM, int CL = 1>
 __global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
 sgat_quant_rows_kernel(QuantArgs a) {
+    static_assert(CL == 1 || NR == 1, "one slice per CTA of a cluster");
     __shared__ __align__(16) float buf[4 * SLICE];
     __shared__ float red[8];              // [0, 4) amax or X_max, [4, 8) -X_min (asym)
+    __shared__ float cl_red[2];           // this CTA's maximum (and -minimum) for its cluster
     grid_dependency_wait();            // launched with programmatic serialisation
     grid_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
-    const int row = blockIdx.x;
+    const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
+    const int row = CL > 1 ? (int)blockIdx.x / CL : (int)blockIdx.x;
     const int K = a.K;
     const bool masked = a.mask != nullptr && a.mask[row] != 0;
     const float* sm = masked ? a.a_m : a.a_u;
@@ -536,7 +548,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
     float amax = 0.f, nmin = 0.f;         // asym: X_max and -X_min
     #pragma unroll
     for (int R = 0; R < NR; ++R) {
-        const int base = R * 4096;
+        const int base = (rank + R) * 4096;
         const int nch = min(4, (K - base + 1023) >> 10); // chunks in this round (>= 1)
         float u[32];
         if (warp < nch) {
@@ -700,6 +712,18 @@ sgat_quant_rows_kernel(QuantArgs a) {
     __syncthreads();
     amax = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
     if (ASYM) nmin = fmaxf(fmaxf(red[4], red[5]), fmaxf(red[6], red[7]));
+    if (CL > 1) {                      // the row's maximum over the cluster's slices
+        if (threadIdx.x == 0) {
+            cl_red[0] = amax;
+            cl_red[1] = nmin;
+        }
+        cluster_sync();
+        #pragma unroll
+        for (int c = 0; c < CL; ++c) {
+            amax = fmaxf(amax, ld_shared_cluster_f32(mapa_shared(smem_addr(&cl_red[0]), (uint32_t)c)));
+            if (ASYM) nmin = fmaxf(nmin, ld_shared_cluster_f32(mapa_shared(smem_addr(&cl_red[1]), (uint32_t)c)));
+        }
+    }
 
     const float qmax = (float)a.qmax;
     const float range = ASYM ? __fadd_rn(amax, nmin) : amax;     // X_max - X_min, or amax
@@ -707,15 +731,15 @@ sgat_quant_rows_kernel(QuantArgs a) {
     const float s = nz ? __fdiv_rn(range, qmax) : 0.f;
     const float r = nz ? __fdiv_rn(qmax, range) : 0.f;
     const int zp = ASYM ? min(max(__float2int_rn(__fmul_rn(nmin, r)), 0), a.qmax) : 0;
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0 && rank == 0) {
         a.s[row] = s;
         if (ASYM) a.z[row] = zp;
     }
-    if (ASYM && a.Xe != nullptr && threadIdx.x < 8)
+    if (ASYM && a.Xe != nullptr && threadIdx.x < 8 && rank == 0)
         store_zero_point_columns(a.Xe + (size_t)row * (K + 128) + K, zp, threadIdx.x);
     #pragma unroll
     for (int R = 0; R < NR; ++R) {
-        const int base = R * 4096;
+        const int base = (rank + R) * 4096;
         const int nch = min(4, (K - base + 1023) >> 10);
         #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -751,6 +775,7 @@ sgat_quant_rows_kernel(QuantArgs a) {
             if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * K + e0) = e4;
         }
     }
+    if (CL > 1) cluster_sync();        // no CTA leaves while its maximum may still be read
 }
 
 template <int NR, typename Tin>
@@ -766,13 +791,34 @@ cudaError_t launch_rows_nr(const QuantArgs& a, cudaStream_t stream) {
                   : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, false>, a);
 }
 
+// Rows longer than 4096: a cluster of CL CTAs per row, one 4096-feature
+// slice each.
+template <int CL, typename Tin>
+cudaError_t launch_rows_cl(const QuantArgs& a, cudaStream_t stream) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[2];
+    at[0] = pdl_attribute();
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = CL;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.gridDim = dim3((unsigned)a.L * CL);
+    cfg.blockDim = dim3(128);
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    return a.asym ? cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<1, Tin, true, CL>, a)
+                  : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<1, Tin, false, CL>, a);
+}
+
 template <typename Tin>
 cudaError_t launch_rows(const QuantArgs& a, cudaStream_t stream) {
     switch ((a.K + 4095) / 4096) {
         case 1: return launch_rows_nr<1, Tin>(a, stream);
-        case 2: return launch_rows_nr<2, Tin>(a, stream);
-        case 3: return launch_rows_nr<3, Tin>(a, stream);
-        case 4: return launch_rows_nr<4, Tin>(a, stream);
+        case 2: return launch_rows_cl<2, Tin>(a, stream);
+        case 3: return launch_rows_cl<3, Tin>(a, stream);
+        case 4: return launch_rows_cl<4, Tin>(a, stream);
+        case 5: return launch_rows_cl<5, Tin>(a, stream);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -819,13 +865,13 @@ cudaError_t launch_e(const QuantArgs& a, cudaStream_t stream) {
 
 template <typename Tin>
 cudaError_t launch_typed(const QuantArgs& a, cudaStream_t stream) {
-    // hb >= 1024 and up to 16384 features: a CTA per row; otherwise a warp's
-    // chunk is 1024 elements (hb >= 1024, blocks finish across warps) or 512
-    // elements holding 512 / hb blocks
-    if (a.hb >= 1024 && a.K % 1024 == 0 && a.K <= 16384) return launch_rows<Tin>(a, stream);
-    // blocks of up to 512 in rows of 1024 to 4096 features, K % 512 == 0:
-    // the same kernel, a last chunk of 512 allowed
-    if (a.hb <= 512 && a.K >= 1024 && a.K <= 4096 && a.K % 512 == 0) return launch_rows_nr<1, Tin>(a, stream);
+    // otherwise a warp's chunk is 1024 elements (hb >= 1024, blocks finish
+    // across warps) or 512 elements holding 512 / hb blocks
+    // up to 20480 features in 4096-feature slices (a cluster of CTAs per row
+    // beyond 4096): blocks of 1024 or more with K % 1024 == 0, or of up to
+    // 512 with K % 512 == 0 (a last chunk of 512 allowed)
+    if (a.K <= 20480 && ((a.hb >= 1024 && a.K % 1024 == 0) || (a.hb <= 512 && a.K >= 1024 && a.K % 512 == 0)))
+        return launch_rows<Tin>(a, stream);
     return a.hb >= 1024 ? launch_e<32, Tin>(a, stream) : launch_e<16, Tin>(a, stream);
 }
 
