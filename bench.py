@@ -55,7 +55,7 @@ def parse():
     p.add_argument("--workload", default="attention_step",
                    choices=["attention_step", "denoise_stack", "tac_calibration", "attention_pv_tac", "w8a8_linear",
                             "asym_linear", "dense_linear", "dream_block", "hbm_passes", "llada_mlp",
-                            "single_linear"],
+                            "single_linear", "mma_sync_gemm"],
                    help="attention_step: the LLaDA attention projections (default); denoise_stack: the "
                         "64-step 4-layer LLaDA-shaped stack (per-step tokens/s, latency, drift vs fp16); "
                         "tac_calibration: App. C's closed-form TAC calibration on the GPU vs the oracle; "
@@ -67,7 +67,8 @@ def parse():
                         "hbm_passes: the quantiser and TAC alone at 8192 tokens (the default line's "
                         "roofline_hbm_kernels.large, without the rest of the run); "
                         "llada_mlp: the LLaDA-8B MLP step (gate+up with SwiGLU, down) at mask ratios "
-                        "0.1 / 0.5 / 0.9; single_linear: the 256 x 512 -> 512 linear with TAC (latency)")
+                        "0.1 / 0.5 / 0.9; single_linear: the 256 x 512 -> 512 linear with TAC (latency); "
+                        "mma_sync_gemm: the projections' GEMMs on mma.sync s4 against the FP8-kind GEMM")
     return p.parse_args()
 
 
@@ -454,6 +455,57 @@ def run_llada_mlp(args):
             "cpu_baseline": {"kind": "oracle", "unit": "TOPS", "cores": cpu_cores(),
                              "value": round(2 * t_orc[1] * 2 * F * Hd / t_orc[0] / 1e12, 6),
                              "sample": f"gate+up linear on {t_orc[1]} of {L} tokens at ratio 0.1"}}
+
+
+def run_mma_sync_gemm(args):
+    """The LLaDA attention projections' two GEMMs (1024 tokens, QKV 4096 ->
+    12288, O 4096 -> 4096) on the warp-level int4 MMA (w4a4_gemm_mma_sync)
+    against the FP8-kind CTA-pair GEMM (w4a4_gemm with E4M3 operands), each
+    timed back to back over operand sets larger than L2: the measured side of
+    the integer-path choice."""
+    import numpy as np
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_04945_gb300 import abi
+    torch.cuda.set_device(0)
+    L, K = 1024, 4096
+    rng = np.random.default_rng(0)
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    flush = lambda: flush_buf.zero_()
+    out = {}
+    for name, N in (("qkv", 12288), ("o", 4096)):
+        sets = []
+        for _ in range(3):
+            Xq = torch.from_numpy(rng.integers(0, 256, (L, K // 2), dtype=np.uint8)).cuda()
+            Wq = torch.from_numpy(rng.integers(0, 256, (N, K // 2), dtype=np.uint8)).cuda()
+            Xe = torch.empty(L, K, dtype=torch.uint8, device="cuda")
+            We = torch.empty(N, K, dtype=torch.uint8, device="cuda")
+            abi.w4_unpack_e4m3(Xq, Xe)
+            abi.w4_unpack_e4m3(Wq, We)
+            sets.append((Xq, Wq, Xe, We))
+        s_a = torch.rand(L, device="cuda") + 0.5
+        s_w = torch.rand(N, device="cuda") * 0.01
+        Y = torch.empty(L, N, dtype=torch.float16, device="cuda")
+        t_sync = time_stream([lambda i=i: abi.w4a4_gemm_mma_sync(sets[i][0], s_a, sets[i][1], s_w, Y)
+                              for i in range(3)], flush, torch, rounds=4)
+        t_fp8 = time_stream([lambda i=i: abi.w4a4_gemm(None, s_a, None, s_w, Y, Xe=sets[i][2], We=sets[i][3])
+                             for i in range(3)], flush, torch, rounds=4)
+        abi.check_status()
+        ops = 2 * L * N * K
+        out[name] = {"mma_sync_ms": round(t_sync, 4), "mma_sync_tops": round(ops / (t_sync * 1e-3) / 1e12, 1),
+                     "fp8_kind_ms": round(t_fp8, 4), "fp8_kind_tops": round(ops / (t_fp8 * 1e-3) / 1e12, 1),
+                     "fp8_kind_speedup": round(t_sync / t_fp8, 2)}
+        del sets
+    ops = 2 * L * (12288 + 4096) * K
+    t = out["qkv"]["mma_sync_ms"] + out["o"]["mma_sync_ms"]
+    return {"metric": "W4A4 GEMMs of the LLaDA attention projections on mma.sync s4 (int32 accumulators), TOPS",
+            "value": round(ops / (t * 1e-3) / 1e12, 1), "unit": "TOPS", "higher_is_better": True, "n_gpus": 1,
+            "data": "synthetic (seeded uniform int4 codes)", "dtype": "int4 codes, int32 accumulators, fp16 out",
+            "config": {"workload": "mma_sync_gemm", "tokens": L, "hidden": K, "qkv": "4096->12288", "o": "4096->4096",
+                       "l2": "operand sets larger than L2, back to back"},
+            "by_projection": out,
+            "note": "the comparison point of the integer-path choice; the hot path runs the FP8-kind GEMM"}
 
 
 def run_single_linear(args):
@@ -1562,8 +1614,9 @@ def main():
         out = run_dream_block(args)
         print(json.dumps(out))
         return
-    if args.workload in ("llada_mlp", "single_linear"):
-        fn = run_llada_mlp if args.workload == "llada_mlp" else run_single_linear
+    if args.workload in ("llada_mlp", "single_linear", "mma_sync_gemm"):
+        fn = {"llada_mlp": run_llada_mlp, "single_linear": run_single_linear,
+              "mma_sync_gemm": run_mma_sync_gemm}[args.workload]
         out = fn(args) if args.impl == "ours" else {"impl": "reference", "unavailable":
                                                     "the oracle arm times the attention-step workload"}
         print(json.dumps(out), flush=True)

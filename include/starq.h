@@ -369,6 +369,25 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
               int y_dtype, const starq_tac* out_tac, int32_t* acc_dbg, void* stream);
 
 /*
+ * w4a4_gemm_mma_sync -- the same integer projection and dequantisation as
+ * w4a4_gemm (Sec. 3.2 Eq. 13, Eq. 5, Eq. 3) on the warp-level integer MMA
+ * (mma.sync m16n8k64 s4.s4.s32, the only int4 tensor-core instruction of
+ * sm_103a), with native int32 accumulators: the comparison point for the
+ * FP8-kind path that w4a4_gemm takes (starq_probe_mma kinds 1 and 4 give
+ * the two instructions' rates).
+ *
+ *   Xq [L][K/2], Wq [N][K/2] packed int4 (low nibble = even k), 16-byte
+ *   aligned; s_a [L], s_w [N] float32; bias [N] float32 or NULL; Y [L][N]
+ *   out, y_dtype F16, BF16 or F32; acc_dbg [L][N] int32 out or NULL.
+ *   Y[i][n] = fl(fl((float)acc s_a[i]) s_w[n]) (+ bias[n]), one rounding to
+ *   y_dtype, as w4a4_gemm.
+ * Shapes: L >= 0, N >= 1, K >= 128 with K % 128 == 0, K <= 65536.
+ */
+int w4a4_gemm_mma_sync(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
+                       const float* bias, int L, int N, int K, void* Y, int y_dtype, int32_t* acc_dbg,
+                       void* stream);
+
+/*
  * Tile of the last Xe + We (or fp16_gemm_ref) launch on the calling thread,
  * as BN * 10 + cluster size: 2562 (256-channel pair tiles) or 2242
  * (224-channel pair tiles); a cluster is one CTA pair, and each CTA loads

@@ -27,6 +27,7 @@ EXPORTED = (
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
     "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
     "starq_selftest_wait_timeout", "starq_probe_mma", "attention_pv_tac_gqa", "glue_add_rmsnorm", "glue_rope",
+    "w4a4_gemm_mma_sync",
 )
 
 
@@ -74,6 +75,7 @@ def _load():
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp, vp]
     lib.w8_split_e4m3.argtypes = [u8p, i, i, u8p, vp]
+    lib.w4a4_gemm_mma_sync.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.w8a8_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.sgat_linear_workspace_size_bits.argtypes = [i, i, i, i]
     lib.sgat_linear_workspace_size_bits.restype = ctypes.c_size_t
@@ -306,6 +308,16 @@ def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, st
     tac = _tac_struct(tac_M, tac_d, tac_g, tac_Mp, tac_scratch)
     _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y),
                          dtype_code(Y), _ref(tac), _p(acc_dbg), _stream(stream)))
+
+
+def w4a4_gemm_mma_sync(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, stream=None):
+    """The same product on the warp-level int4 MMA (mma.sync s4), packed
+    operands Xq [L][K/2], Wq [N][K/2]."""
+    _contig(Xq, s_a, Wq, s_w, Y, bias, acc_dbg)
+    L, N = Y.shape
+    K = Wq.shape[1] * 2
+    _check(lib.w4a4_gemm_mma_sync(_p(Xq), _p(s_a), _p(Wq), _p(s_w), _p(bias), L, N, K, _p(Y), dtype_code(Y),
+                                  _p(acc_dbg), _stream(stream)))
 
 
 def last_gemm_tile():

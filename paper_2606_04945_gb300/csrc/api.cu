@@ -394,6 +394,26 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
     return STARQ_OK;
 }
 
+int w4a4_gemm_mma_sync(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
+                       const float* bias, int L, int N, int K, void* Y, int y_dtype, int32_t* acc_dbg,
+                       void* stream) {
+    if (L > 0 && (!Xq || !s_a || !Y)) return fail(STARQ_ERR_ARG, "w4a4_gemm_mma_sync: NULL Xq, s_a or Y");
+    if (!Wq || !s_w) return fail(STARQ_ERR_ARG, "w4a4_gemm_mma_sync: NULL Wq or s_w");
+    if (!dtype_ok(y_dtype)) return fail(STARQ_ERR_ARG, "w4a4_gemm_mma_sync: unknown output dtype %d", y_dtype);
+    if (L < 0 || N < 1 || K < 128 || K % 128 != 0 || K > 65536)
+        return fail(STARQ_ERR_SHAPE, "w4a4_gemm_mma_sync: L=%d N=%d K=%d (N >= 1, K %% 128 == 0, 128 <= K <= 65536)",
+                    L, N, K);
+    if (L == 0) return STARQ_OK;
+    if (!aligned(Xq, 16) || !aligned(Wq, 16))
+        return fail(STARQ_ERR_ALIGN, "w4a4_gemm_mma_sync: Xq and Wq must be 16-byte aligned");
+    int rc = check_local("w4a4_gemm_mma_sync", static_cast<cudaStream_t>(stream), {Xq, Wq, Y});
+    if (rc) return rc;
+    GemmArgs a{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, acc_dbg, nullptr};
+    cudaError_t e = launch_w4a4_gemm_mmasync(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm_mma_sync launch");
+    return STARQ_OK;
+}
+
 int sgat_quantize_act_asym(const void* X, int x_dtype, int L, int K, const uint8_t* mask, const float* a_m,
                            const float* a_u, int hb, int d_sh, int d_m, int d_u, uint8_t* Xq, float* s_a,
                            int32_t* z_a, uint8_t* Xe, void* stream) {

@@ -64,6 +64,8 @@ struct GemmArgs {
     int swiglu = 0;
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+// The same product on the warp-level int4 MMA (mma.sync s4), packed operands.
+cudaError_t launch_w4a4_gemm_mmasync(const GemmArgs& a, cudaStream_t stream);
 // Tile of the calling thread's last TMA pair GEMM launch (BN * 10 + cluster
 // size; 0 before the first).
 int last_gemm_tile();

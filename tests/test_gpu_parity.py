@@ -537,3 +537,33 @@ def test_gemm_out_tac_option(abi, L, N, K, g, dtype):
     pre = H.host(scratch)
     H.assert_output_close(pre, osg.dequant(ref_acc, s_a, s_w, None), dtype, what="pre-TAC output")
     H.assert_tac_close(H.host(Y), otac.tac_apply(pre, tp.M, tp.d, g), dtype)
+
+
+@pytest.mark.parametrize("L,N,K,out", [(1, 8, 128, "f32"), (200, 136, 512, "f16"), (129, 300, 1024, "bf16"),
+                                       (1024, 4096, 4096, "f16")])
+def test_gemm_mma_sync(abi, L, N, K, out):
+    """The W4A4 GEMM on the warp-level int4 MMA (mma.sync m16n8k64 s4):
+    int32 accumulators bit-exact with the oracle's integer product (ragged
+    tiles, all-(-7) and all-(+7) rows for the extreme sums), outputs within
+    the output tolerance, and the same outputs as w4a4_gemm's FP8-kind path
+    bit for bit (the same float32 epilogue on the same exact sums)."""
+    qa, qw, s_a, s_w = H.gemm_codes(L * 7 + N + K, L, N, K)
+    qa[0] = -7
+    qw[0] = -7
+    if L > 1:
+        qa[1] = 7
+    Xq, Wq = H.dev(osg.pack_int4(qa)), H.dev(osg.pack_int4(qw))
+    dt = H.torch_dtype(out)
+    Y = torch.empty(L, N, dtype=dt, device="cuda")
+    acc = torch.empty(L, N, dtype=torch.int32, device="cuda")
+    abi.w4a4_gemm_mma_sync(Xq, H.dev(s_a), Wq, H.dev(s_w), Y, acc_dbg=acc)
+    abi.check_status()
+    ref = osg.int_gemm(qa, qw)
+    assert np.array_equal(acc.cpu().numpy(), ref)
+    assert ref[0, 0] == 49 * K
+    H.assert_output_close(H.host(Y), osg.dequant(ref, s_a, s_w, None), out)
+    if N % 32 == 0:
+        Y2 = torch.empty_like(Y)
+        abi.w4a4_gemm(Xq, H.dev(s_a), Wq, H.dev(s_w), Y2)
+        abi.check_status()
+        assert torch.equal(Y, Y2)
