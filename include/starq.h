@@ -369,6 +369,17 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
               int y_dtype, const starq_tac* out_tac, int32_t* acc_dbg, void* stream);
 
 /*
+ * starq_set_gemm_pair_limit -- at most `pairs` CTA pairs (two SMs each) for
+ * the W4A4 and 16-bit TMA pair GEMMs launched afterwards from the calling
+ * thread (w4a4_gemm with Xe and We, the sgat_linear family, fp16_gemm_ref);
+ * 0 removes the cap. Returns the previous cap (>= 0), or STARQ_ERR_ARG for
+ * pairs < 0. The cap is part of the launch, so a CUDA graph captured under
+ * it keeps it. Use: a GEMM that runs beside other kernels (two branches of
+ * one step) leaves them the remaining SMs; the results do not depend on it.
+ */
+int starq_set_gemm_pair_limit(int pairs);
+
+/*
  * w4a4_gemm_mma_sync -- the same integer projection and dequantisation as
  * w4a4_gemm (Sec. 3.2 Eq. 13, Eq. 5, Eq. 3) on the warp-level integer MMA
  * (mma.sync m16n8k64 s4.s4.s32, the only int4 tensor-core instruction of

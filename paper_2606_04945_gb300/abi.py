@@ -27,7 +27,7 @@ EXPORTED = (
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
     "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
     "starq_selftest_wait_timeout", "starq_probe_mma", "attention_pv_tac_gqa", "glue_add_rmsnorm", "glue_rope",
-    "w4a4_gemm_mma_sync",
+    "w4a4_gemm_mma_sync", "starq_set_gemm_pair_limit",
 )
 
 
@@ -76,6 +76,8 @@ def _load():
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp, vp]
     lib.w8_split_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm_mma_sync.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.starq_set_gemm_pair_limit.argtypes = [i]
+    lib.starq_set_gemm_pair_limit.restype = i
     lib.w8a8_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.sgat_linear_workspace_size_bits.argtypes = [i, i, i, i]
     lib.sgat_linear_workspace_size_bits.restype = ctypes.c_size_t
@@ -318,6 +320,15 @@ def w4a4_gemm_mma_sync(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, stream=None
     K = Wq.shape[1] * 2
     _check(lib.w4a4_gemm_mma_sync(_p(Xq), _p(s_a), _p(Wq), _p(s_w), _p(bias), L, N, K, _p(Y), dtype_code(Y),
                                   _p(acc_dbg), _stream(stream)))
+
+
+def set_gemm_pair_limit(pairs):
+    """Cap the CTA pairs of the pair GEMMs launched afterwards from this
+    thread (0 = no cap); returns the previous cap."""
+    rc = int(lib.starq_set_gemm_pair_limit(int(pairs)))
+    if rc < 0:
+        raise StarqError(rc, lib.starq_last_error().decode())
+    return rc
 
 
 def last_gemm_tile():

@@ -394,6 +394,11 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
     return STARQ_OK;
 }
 
+int starq_set_gemm_pair_limit(int pairs) {
+    if (pairs < 0) return fail(STARQ_ERR_ARG, "starq_set_gemm_pair_limit: pairs=%d < 0", pairs);
+    return set_gemm_pair_limit(pairs);
+}
+
 int w4a4_gemm_mma_sync(const uint8_t* Xq, const float* s_a, const uint8_t* Wq, const float* s_w,
                        const float* bias, int L, int N, int K, void* Y, int y_dtype, int32_t* acc_dbg,
                        void* stream) {

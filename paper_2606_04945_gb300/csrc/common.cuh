@@ -64,6 +64,9 @@ struct GemmArgs {
     int swiglu = 0;
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+// Thread-local cap on the CTA pairs of the TMA pair GEMMs launched from the
+// calling thread (0 = none); returns the previous cap.
+int set_gemm_pair_limit(int pairs);
 // The same product on the warp-level int4 MMA (mma.sync s4), packed operands.
 cudaError_t launch_w4a4_gemm_mmasync(const GemmArgs& a, cudaStream_t stream);
 // Tile of the calling thread's last TMA pair GEMM launch (BN * 10 + cluster

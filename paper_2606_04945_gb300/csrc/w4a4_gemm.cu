@@ -832,6 +832,9 @@ struct Cfg {
 // Tile of the calling thread's last TMA pair GEMM launch: BN * 10 + 2 (CTAs
 // per cluster).
 thread_local int g_last_tile = 0;
+// Most CTA pairs a TMA pair GEMM launched from this thread may use (0 = as
+// many as are resident).
+thread_local int g_pair_limit = 0;
 
 // Output tiles of the pair GEMM: 256-token rows x BN-channel pair tiles.
 int tma_tiles(int L, int N, int BN) {
@@ -1214,6 +1217,10 @@ cudaError_t launch_tma_shape(const GemmArgs& a, cudaStream_t stream) {
     cudaError_t e = tma_max_clusters<TOut, OPK, 256, SW>(&c256);
     if (e != cudaSuccess) return e;
     if ((e = tma_max_clusters<TOut, OPK, 224, SW>(&c224)) != cudaSuccess) return e;
+    if (g_pair_limit > 0) {
+        if (c256 > g_pair_limit) c256 = g_pair_limit;
+        if (c224 > g_pair_limit) c224 = g_pair_limit;
+    }
     const long long t256 = tma_round_cost(a.L, a.N, 256, c256);
     const long long t224 = tma_round_cost(a.L, a.N, 224, c224);
     if (t224 < t256) {
@@ -1329,6 +1336,12 @@ cudaError_t launch_fp16_gemm(const GemmArgs& a, cudaStream_t stream) {
         case STARQ_BF16: return launch_tma_typed<__nv_bfloat16, 2>(a, stream);
         default: return cudaErrorInvalidValue;
     }
+}
+
+int set_gemm_pair_limit(int pairs) {
+    const int prev = g_pair_limit;
+    g_pair_limit = pairs;
+    return prev;
 }
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {

@@ -76,9 +76,16 @@ class SgatLinear:
 
 
 class AttentionProjections:
-    """QKV projection of X and TAC + O projection of Z for one step."""
+    """QKV projection of X and TAC + O projection of Z for one step.
 
-    def __init__(self, qkv_case, o_case, device="cuda", e4m3_weights=True):
+    qkv_pair_limit caps the CTA pairs of the QKV GEMM so that the O branch's
+    TAC and quantiser can run beside it on the remaining SMs (0 = no cap,
+    the default). On GB300 with the LLaDA shapes a cap of 48 pairs gave
+    either 67-69 us or 82 us per replay, depending on which branch's CTAs
+    the hardware placed first (against a steady 71-73 us uncapped), so it
+    is off by default. Results do not depend on it."""
+
+    def __init__(self, qkv_case, o_case, device="cuda", e4m3_weights=True, qkv_pair_limit=0):
         self.qkv = SgatLinear(qkv_case, device, e4m3_weights=e4m3_weights)
         self.o = SgatLinear(o_case, device, e4m3_weights=e4m3_weights)
         self.L = qkv_case.L
@@ -88,6 +95,7 @@ class AttentionProjections:
         self.Y_qkv = torch.empty(self.L, self.qkv.N, dtype=self.qkv.out_dtype, device=device)
         self.Y_o = torch.empty(self.L, self.o.N, dtype=self.o.out_dtype, device=device)
         self.side = torch.cuda.Stream(device=device)
+        self.qkv_pair_limit = qkv_pair_limit
         self.graph = None
 
     def step(self, stream=None):
@@ -101,7 +109,11 @@ class AttentionProjections:
         self.side.wait_stream(main)
         with torch.cuda.stream(self.side):
             self.o.run(self.Z, self.mask, self.Y_o, self.side)
-        self.qkv.run(self.X, self.mask, self.Y_qkv, main)
+        prev = abi.set_gemm_pair_limit(self.qkv_pair_limit)
+        try:
+            self.qkv.run(self.X, self.mask, self.Y_qkv, main)
+        finally:
+            abi.set_gemm_pair_limit(prev)
         main.wait_stream(self.side)
 
     def capture(self):

@@ -333,3 +333,16 @@ def test_tac_option_validation(lib, g, M, Mp, scratch, dtype, code):
     assert lib.lib.starq_last_error()
     assert lib.lib.w4a4_gemm(P, None, P, P, None, P, None, 4, 256, 512, P, dtype, ctypes.byref(t), None,
                              None) == (code if g != 5 else -2)
+
+
+def test_gemm_pair_limit(lib):
+    """The pair cap is thread-local state: it returns the previous cap and
+    rejects negative values without touching it."""
+    prev = lib.set_gemm_pair_limit(48)
+    try:
+        assert lib.set_gemm_pair_limit(12) == 48
+        with pytest.raises(lib.StarqError):
+            lib.set_gemm_pair_limit(-1)
+        assert lib.set_gemm_pair_limit(0) == 12
+    finally:
+        lib.set_gemm_pair_limit(prev)
