@@ -59,12 +59,14 @@
 // each item's pass-1 K chunks, pass-2 K and V chunks, M's two halves and
 // then the slot of its output boxes, in the order they are used, running
 // on into the next item.
-// TMEM (512 columns): two S / P buffers, the P V^T accumulator and Q; the
-// TAC accumulator and Z_hat reuse the S buffers. The MMA warp queries its
-// two barriers per MMA group back to back, so their latencies overlap: with
-// about 50 cycles per issued MMA and ~160 per barrier query, a single
-// issuing thread is what bounds the tensor pipe here. Every wait is
-// bounded.
+// TMEM (512 columns): two S / P buffers (pass 1 also uses the P V^T
+// accumulator's columns as a third), the P V^T accumulator and Q; the TAC
+// accumulator and Z_hat reuse the S buffers. The tensor pipe keeps almost
+// no queue of issued MMAs, so it runs dry whenever the issuing thread
+// waits, and a barrier query costs ~160-380 cycles even on a completed
+// phase: the MMA warp therefore waits once per pass-2 chunk, on all of the
+// chunk's barriers at once, and then issues its P V^T and the Q K^T two
+// chunks ahead back to back. Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -88,8 +90,11 @@ constexpr int ATT_TILES_BYTES = ATT_SLOTS * TILE_BYTES;
 // TMEM columns: S in two buffers of 128, the P V^T accumulator O and Q
 // (16-bit, two per column). P overwrites the S it came from: the warp that
 // read S columns [32 p, 32 p + 32) writes their 32 codes to columns
-// [32 p, 32 p + 16). After the passes the TAC accumulator takes the first S
-// buffer and Z_hat's halves the second.
+// [32 p, 32 p + 16), so no other warp's scores are touched and no wait is
+// needed; the next Q K^T into that buffer is issued after the P V^T that
+// reads P, and the MMAs of one thread run in issue order. After the passes
+// the TAC accumulator takes the first S buffer and Z_hat's halves the
+// second.
 constexpr uint32_t TM_S = 0, TM_O = 256, TM_Q = 384;
 constexpr uint32_t TM_TAC = 0, TM_ZHI = 128, TM_ZLO = 192;
 
@@ -151,6 +156,19 @@ __device__ __forceinline__ bool mbar_wait2_bounded_warp(uint32_t b0, uint32_t p0
     const bool d1 = mbar_try_wait(b1, p1);
     bool ok = true;
     if (!(d0 && d1)) ok = (d0 || mbar_wait_bounded(b0, p0, abort)) && (d1 || mbar_wait_bounded(b1, p1, abort));
+    return __all_sync(0xffffffffu, ok);
+}
+
+// Three phases complete, the first queries back to back as above.
+__device__ __forceinline__ bool mbar_wait3_bounded_warp(uint32_t b0, uint32_t p0, uint32_t b1, uint32_t p1, uint32_t b2,
+                                                        uint32_t p2, volatile int* abort) {
+    const bool d0 = mbar_try_wait(b0, p0);
+    const bool d1 = mbar_try_wait(b1, p1);
+    const bool d2 = mbar_try_wait(b2, p2);
+    bool ok = true;
+    if (!(d0 && d1 && d2))
+        ok = (d0 || mbar_wait_bounded(b0, p0, abort)) && (d1 || mbar_wait_bounded(b1, p1, abort)) &&
+             (d2 || mbar_wait_bounded(b2, p2, abort));
     return __all_sync(0xffffffffu, ok);
 }
 
@@ -397,8 +415,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         constexpr uint32_t IDESC_T = IDESC_F16 | (std::is_same<T, __nv_bfloat16>::value ? ((1u << 7) | (1u << 10)) : 0u);
         // D (+)= A B^T over K = 128: A from TMEM at a_col (8 columns per K
         // step; for P, K steps 2p and 2p + 1 sit at 32 p and 32 p + 8), B
-        // the K-major tile at bt
-        // (issued by the elected lane)
+        // the K-major tile at bt (issued by the elected lane)
         auto mma_tile = [=](uint32_t d, uint32_t a_col, uint32_t bt, bool acc0, bool p_layout, uint32_t idesc) {
             // K step offsets added to the descriptor's start-address field
             // (addresses below 2^18, so the field never carries)
@@ -420,18 +437,14 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             ok = i == 0 ? mbar_wait_bounded_warp(B(sh->q_full), 0, abort)
                         : mbar_wait2_bounded_warp(B(sh->q_full), (uint32_t)(i & 1), B(sh->tac_read),
                                                   (uint32_t)((i - 1) & 1), abort);
-            // Q K^T number it, once its K tile has landed and its S buffer's
-            // previous use is consumed: S read by the softmax warps, or P
-            // written by them and read by the P V^T issued before this MMA
-            // (the MMAs of one thread run in issue order). For pass-2 chunks
-            // from 2 on, that P V^T's own wait has already seen the P written.
+            // Q K^T number it, once its K tile has landed and the softmax
+            // warps have read the S buffer's previous scores (s_empty)
             auto qk = [=](int it) -> bool {
                 const int g = g0 + (it < nk ? it : nk + 2 * (it - nk));
                 int b, n;
                 sbuf(i, it, b, n);
-                if (!(it >= nk + 2 ? mbar_wait_bounded_warp(full_bar(g), use_parity(g), abort)
-                                   : mbar_wait2_bounded_warp(full_bar(g), use_parity(g), B(sh->s_empty[b]),
-                                                             (uint32_t)(n & 1) ^ 1u, abort)))
+                if (!mbar_wait2_bounded_warp(full_bar(g), use_parity(g), B(sh->s_empty[b]), (uint32_t)(n & 1) ^ 1u,
+                                             abort))
                     return false;
                 tc_fence_after();
                 if (elect_one()) {
@@ -442,27 +455,39 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 __syncwarp();
                 return true;
             };
-            // P V^T of pass-2 chunk j, once its P is in its S buffer
-            auto pv = [=](int j) -> bool {
-                const int g = g0 + nk + 2 * j + 1;
+            // Pass 2, one wait per chunk: P V^T of chunk j once its P is in
+            // place over S(j) (the softmax warps arrive on the buffer's
+            // s_empty after writing it) and its V tile has landed, then
+            // Q K^T of chunk j + 2 into the same buffer once its K tile has
+            // landed. Every wait of the issuing thread lets the tensor pipe
+            // run dry, so the two products go out back to back behind a
+            // single wait.
+            auto step2 = [=](int j) -> bool {
+                const int gv = g0 + nk + 2 * j + 1, gk = gv + 3;
+                const bool more = j + 2 < nk;
                 int b, n;
                 sbuf(i, nk + j, b, n);
-                if (!mbar_wait2_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1), full_bar(g), use_parity(g), abort))
+                if (!(more ? mbar_wait3_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1), full_bar(gv), use_parity(gv),
+                                                     full_bar(gk), use_parity(gk), abort)
+                           : mbar_wait2_bounded_warp(B(sh->s_empty[b]), (uint32_t)(n & 1), full_bar(gv), use_parity(gv),
+                                                     abort)))
                     return false;
                 tc_fence_after();
                 if (elect_one()) {
-                    mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(g), j > 0, true, IDESC_F16);
-                    tc_commit(empty_bar(g));
+                    mma_tile(tmem + TM_O, TM_S + b * ATTN_TILE, slot(gv), j > 0, true, IDESC_F16);
+                    tc_commit(empty_bar(gv));
+                    if (more) {
+                        mma_tile(tmem + TM_S + b * ATTN_TILE, TM_Q, slot(gk), false, false, IDESC_T);
+                        tc_commit(empty_bar(gk));
+                        tc_commit(B(sh->s_full[b]));
+                    }
                 }
                 __syncwarp();
                 return true;
             };
             tc_fence_after();
-            for (int it = 0; it < 2 * nk && ok; ++it) {
-                ok = qk(it);
-                if (ok && it > nk) ok = pv(it - 1 - nk);   // one chunk behind the scores
-            }
-            if (ok) ok = pv(nk - 1);
+            for (int it = 0; it < nk + 2 && it < 2 * nk && ok; ++it) ok = qk(it);   // pass 1, then two chunks ahead
+            for (int j = 0; j < nk && ok; ++j) ok = step2(j);
             if (elect_one()) tc_commit(B(sh->pv_done));
             __syncwarp();
             const int gm = g0 + 3 * nk;               // M_hi; M_lo at gm + 1
