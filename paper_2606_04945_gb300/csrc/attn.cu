@@ -93,18 +93,22 @@ constexpr int ATT_TILES_BYTES = ATT_SLOTS * TILE_BYTES;
 // [32 p, 32 p + 16), so no other warp's scores are touched and no wait is
 // needed; the next Q K^T into that buffer is issued after the P V^T that
 // reads P, and the MMAs of one thread run in issue order. After the passes
-// the TAC accumulator takes the first S buffer and Z_hat's halves the
-// second.
+// the TAC accumulator takes the P V^T accumulator's columns (read out by
+// then), Z_hat's high half the last 64 columns and its low half the upper
+// half of the second S buffer. The first S buffer and the lower half of the
+// second stay free, so the next item's Q K^T can follow the TAC product at
+// once (the MMAs of one thread run in issue order, so it cannot overwrite
+// Z_lo before the TAC product has read it).
 constexpr uint32_t TM_S = 0, TM_O = 256, TM_Q = 384;
-constexpr uint32_t TM_TAC = 0, TM_ZHI = 128, TM_ZLO = 192;
+constexpr uint32_t TM_TAC = TM_O, TM_ZHI = 448, TM_ZLO = 192;
 
 struct AttSm {
-    uint64_t q_full, full[ATT_SLOTS], empty[ATT_SLOTS], s_full[3], s_empty[3];
-    uint64_t pv_done, z_full, tac_done, tac_read;
+    uint64_t q_full, full[ATT_SLOTS], empty[ATT_SLOTS], s_full[2], s_empty[2];
+    uint64_t pv_done, z_full, tac_done;
     uint32_t tmem_base;
     int abort;
-    float xm[4][ATTN_TILE];            // row maxima / sums of the four column parts
-    float tv[ATTN_D], dv[ATTN_D];      // the head's V channel scales and TAC offsets
+    alignas(16) float xm[4][ATTN_TILE];            // row maxima / sums of the four column parts
+    alignas(16) float tv[ATTN_D], dv[ATTN_D];      // the head's V channel scales and TAC offsets
 };
 constexpr size_t ATT_SMEM = ATT_TILES_BYTES + 1024 + sizeof(AttSm);
 
@@ -284,23 +288,24 @@ __global__ void __launch_bounds__(256) attn_vquant_kernel(AttnArgs a) {
 // role loops over the same items, and every barrier's phase runs on across
 // items.
 //
-// The ring's entries of item i are E = 3 nk + 3 in number, global index
-// G = i E + u: u = 0 .. nk-1 the K chunks of pass 1, u = nk + 2j, nk + 2j + 1
-// chunk j's K and V for pass 2, u = 3 nk and 3 nk + 1 M's halves (one bulk
-// copy each), u = 3 nk + 2 the output boxes (the TMA warp hands the free
-// slot to the softmax warps with a plain arrive on its full barrier; they
-// give it back after their stores have read it). Entry G uses slot G mod 6
-// for the (G / 6)-th time. So the next item's K chunks stream in while this
-// item's epilogue runs.
+// The ring's entries of item i are E = 3 nk + 4 in number, global index
+// G = i E + 1 + u: u = -1 the item's Q tile (the softmax warps copy it into
+// TMEM; the MMA warp gives the slot back once they have), u = 0 .. nk-1 the
+// K chunks of pass 1, u = nk + 2j, nk + 2j + 1 chunk j's K and V for pass 2,
+// u = 3 nk and 3 nk + 1 M's halves (one bulk copy each), u = 3 nk + 2 the
+// output boxes (the TMA warp hands the free slot to the softmax warps with
+// a plain arrive on its full barrier; they give it back after their stores
+// have read it). Entry G uses slot G mod 6 for the (G / 6)-th time. So the
+// next item's Q and K chunks stream in while this item's epilogue runs.
 //
 // TMEM across items: the next item's Q is written as soon as this item's
-// P V^T has completed (its columns are then dead), and its first Q K^T
-// waits until the epilogue has read this item's TAC accumulator (tac_read),
-// which sits in the first S buffer.
+// P V^T has completed (its columns are then dead), before Z_hat, and the
+// MMA warp issues the next item's first Q K^T right after this item's TAC
+// product (see the column map above).
 template <typename T>
 __global__ void __launch_bounds__(ATT_THREADS, 1)
-attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                   const __grid_constant__ CUtensorMap tm_z) {
+attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                   const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_z) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -314,7 +319,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
     // (the lambdas capture by value: a local captured by reference lives in
     // memory and is reloaded after every asm with a memory clobber)
     auto B = [](const uint64_t& bar) { return smem_addr(&bar); };
-    const int E = 3 * nk + 3;                                // ring entries per item
+    const int E = 3 * nk + 4;                                // ring entries per item
     // (entry indices stay below 2^31: at most 64 key chunks per head and
     // a few thousand items per CTA; 32-bit division by a constant is cheap)
     auto slot = [=](int g) { return base + ((uint32_t)g % ATT_SLOTS) * TILE_BYTES; };
@@ -323,21 +328,15 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
     auto use_parity = [](int g) { return ((uint32_t)g / ATT_SLOTS) & 1u; };
     auto item_q0 = [=](int i) { return ((int)blockIdx.x + i * (int)gridDim.x) % nk * ATTN_TILE; };
     auto item_h = [=](int i) { return ((int)blockIdx.x + i * (int)gridDim.x) / nk; };
-    // S buffer of Q K^T number it of item i (pass 1: it = 0 .. nk-1, three
-    // buffers, the third in the columns of the P V^T accumulator, which pass
-    // 1 leaves unused; pass 2: it = nk + j, two buffers) and the number of
-    // that buffer's earlier uses, counted over all items
-    const int p1_0 = (nk + 2) / 3, p1_1 = (nk + 1) / 3, p1_2 = nk / 3;   // pass-1 uses per item
-    const int p2_0 = (nk + 1) / 2, p2_1 = nk / 2;                       // pass-2 uses per item
+    // S buffer of Q K^T number it of item i (pass 1: it = 0 .. nk-1; pass
+    // 2: it = nk + j; the two buffers alternate within each pass) and the
+    // number of that buffer's earlier uses, counted over all items
+    const int u0 = (nk + 1) / 2, u1 = nk / 2;                // uses of buffer 0 / 1 per pass
     auto sbuf = [=](int i, int it, int& b, int& n) {
-        if (it < nk) {
-            b = it % 3;
-            n = it / 3 + i * (b == 0 ? p1_0 + p2_0 : b == 1 ? p1_1 + p2_1 : p1_2);
-        } else {
-            const int j = it - nk;
-            b = j & 1;
-            n = (b == 0 ? p1_0 : p1_1) + (j >> 1) + i * (b == 0 ? p1_0 + p2_0 : p1_1 + p2_1);
-        }
+        const int j = it < nk ? it : it - nk;
+        b = j & 1;
+        const int per = b == 0 ? u0 : u1;
+        n = (j >> 1) + (it < nk ? 0 : per) + i * 2 * per;
     };
 
     if (threadIdx.x == 0) {
@@ -346,14 +345,13 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             mbar_init(B(sh->full[k]), 1);
             mbar_init(B(sh->empty[k]), 1);
         }
-        for (int b = 0; b < 3; ++b) {
+        for (int b = 0; b < 2; ++b) {
             mbar_init(B(sh->s_full[b]), 1);
             mbar_init(B(sh->s_empty[b]), ATT_SOFTMAX_WARPS);
         }
         mbar_init(B(sh->pv_done), 1);
         mbar_init(B(sh->z_full), ATT_SOFTMAX_WARPS);
         mbar_init(B(sh->tac_done), 1);
-        mbar_init(B(sh->tac_read), ATT_SOFTMAX_WARPS);
         sh->abort = 0;
         mbar_fence_init();
     }
@@ -370,12 +368,17 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         bool ok = true;
         for (int i = 0; i < my_items && ok; ++i) {
             const int h = item_h(i), hk = h / group;
-            for (int u = 0; u < E && ok; ++u) {
-                const int g = i * E + u;
+            for (int ue = 0; ue < E && ok; ++ue) {
+                const int g = i * E + ue;
+                const int u = ue - 1;                            // -1: Q; from 0 the entries below
                 if (!mbar_wait_bounded_warp(empty_bar(g), use_parity(g) ^ 1u, abort)) { ok = false; break; }
                 const uint32_t dst = slot(g), fb = full_bar(g);
                 if (elect_one()) {
-                    if (u < 3 * nk) {
+                    if (u < 0) {                                 // the item's Q tile, as A of Q K^T
+                        mbar_arrive_expect_tx(fb, TILE_BYTES);
+                        tma_load_2d(dst, &tm_q, h * ATTN_D, item_q0(i), fb);
+                        tma_load_2d(dst + ATOM_BYTES, &tm_q, h * ATTN_D + 64, item_q0(i), fb);
+                    } else if (u < 3 * nk) {
                         mbar_arrive_expect_tx(fb, TILE_BYTES);
                         const int w = u - nk;
                         const void* tm = (w < 0 || (w & 1) == 0) ? (const void*)&tm_k : (const void*)&tm_v;
@@ -432,11 +435,11 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         int tac_commits = 0;
         tc_fence_after();
         for (int i = 0; i < my_items && ok; ++i) {
-            const int g0 = i * E;
-            // Q in TMEM; for i > 0 the previous TAC accumulator read out
-            ok = i == 0 ? mbar_wait_bounded_warp(B(sh->q_full), 0, abort)
-                        : mbar_wait2_bounded_warp(B(sh->q_full), (uint32_t)(i & 1), B(sh->tac_read),
-                                                  (uint32_t)((i - 1) & 1), abort);
+            const int gq = i * E, g0 = gq + 1;
+            // Q in TMEM: its ring slot is free again
+            ok = mbar_wait_bounded_warp(B(sh->q_full), (uint32_t)(i & 1), abort);
+            if (ok && elect_one()) mbar_arrive(empty_bar(gq));
+            __syncwarp();
             // Q K^T number it, once its K tile has landed and the softmax
             // warps have read the S buffer's previous scores (s_empty)
             auto qk = [=](int it) -> bool {
@@ -520,13 +523,17 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
         const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
         bool ok = true;
         uint32_t r[32];
-        // the query row's 32 channels of this part into TMEM (A of Q K^T)
-        auto put_q = [=](int i) {
-            const T* qp = static_cast<const T*>(a.Q) + (size_t)(item_q0(i) + row) * a.ld + item_h(i) * ATTN_D + col;
+        // the query row's 32 channels of this part, from item i's Q tile in
+        // its ring slot (two 64-channel halves of 128-byte rows, the 16-byte
+        // chunks of row r XOR-ed with r mod 8), into TMEM (A of Q K^T)
+        auto put_q = [=](int i) -> bool {
+            const int gq = i * E;
+            if (!mbar_wait_bounded_warp(full_bar(gq), use_parity(gq), abort)) return false;
+            const uint32_t src = slot(gq) + (uint32_t)(part >> 1) * ATOM_BYTES + (uint32_t)row * 128u;
             uint32_t qv[16];
             #pragma unroll
             for (int k = 0; k < 4; ++k) {
-                const uint4 w = ld_global_nc_v4(qp + 8 * k);
+                const uint4 w = ld_shared_v4(src + ((uint32_t)(((part & 1) * 4 + k) ^ (row & 7)) << 4));
                 qv[4 * k] = w.x;
                 qv[4 * k + 1] = w.y;
                 qv[4 * k + 2] = w.z;
@@ -537,13 +544,14 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(B(sh->q_full));
+            return true;
         };
-        if (my_items > 0) put_q(0);
+        if (my_items > 0) ok = put_q(0);
         // Every softmax warp runs every item and every named barrier; after a
         // failed wait it only skips the work.
         for (int i = 0; i < my_items; ++i) {
             const int q0 = item_q0(i), h = item_h(i), hk = h / group;
-            const int g0 = i * E;
+            const int g0 = i * E + 1;
             const uint32_t ip = (uint32_t)(i & 1);
             if (threadIdx.x >= ATTN_D && threadIdx.x < 2 * ATTN_D) {
                 const int c = threadIdx.x - ATTN_D;
@@ -625,9 +633,13 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
             const int zk = tmax > 0.f ? ilogbf(112.f * tmax) - 13 : 0;
             const float zscale = ldexpf(1.f, -zk), zunscale = ldexpf(1.f, zk);
             if (a.dbg_l != nullptr && part == 0) a.dbg_l[(size_t)h * a.L + q0 + row] = l;
+            // every MMA reading Q has completed (pv_done), so the next item's
+            // Q goes in first, for its Q K^T right after this item's TAC
+            // product
+            ok = ok && mbar_wait_bounded_warp(B(sh->pv_done), ip, abort);
+            if (ok && i + 1 < my_items) ok = put_q(i + 1);
             // epilogue 1: Z_hat = (acc sp) t as fp16 hi + lo, the A operands of
             // the TAC product, into TMEM
-            ok = ok && mbar_wait_bounded_warp(B(sh->pv_done), ip, abort);
             if (ok) {
                 tc_fence_after();
                 tmem_ld_32x32b_x32(tl + TM_O + col, r);
@@ -639,16 +651,19 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 }
                 uint32_t hi[16], lo[16];
                 #pragma unroll
-                for (int k = 0; k < 32; k += 2) {
-                    float z[2];
+                for (int k = 0; k < 32; k += 4) {
+                    const float4 t4 = *reinterpret_cast<const float4*>(&sh->tv[col + k]);
+                    const float tk[4] = {t4.x, t4.y, t4.z, t4.w};
                     #pragma unroll
-                    for (int u = 0; u < 2; ++u)
-                        z[u] = __fmul_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), sh->tv[col + k + u]), zscale);
-                    const uint16_t h0 = bits_rn(__half(), z[0]), h1 = bits_rn(__half(), z[1]);
-                    const uint16_t l0 = bits_rn(__half(), z[0] - from_bits(__half(), h0)),
-                                   l1 = bits_rn(__half(), z[1] - from_bits(__half(), h1));
-                    hi[k / 2] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-                    lo[k / 2] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+                    for (int u = 0; u < 4; u += 2) {
+                        const float z0 = __fmul_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[k + u]), sp), tk[u]), zscale);
+                        const float z1 = __fmul_rn(__fmul_rn(__fmul_rn(__uint_as_float(r[k + u + 1]), sp), tk[u + 1]), zscale);
+                        const __half2 zh = __floats2half2_rn(z0, z1);
+                        const float2 zb = __half22float2(zh);
+                        const __half2 zl = __floats2half2_rn(__fsub_rn(z0, zb.x), __fsub_rn(z1, zb.y));
+                        hi[(k + u) / 2] = *reinterpret_cast<const uint32_t*>(&zh);
+                        lo[(k + u) / 2] = *reinterpret_cast<const uint32_t*>(&zl);
+                    }
                 }
                 tmem_st_32x32b_x16(tl + TM_ZHI + part * 16, hi);
                 tmem_st_32x32b_x16(tl + TM_ZLO + part * 16, lo);
@@ -656,9 +671,6 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(B(sh->z_full));
-                // every MMA reading Q has completed (pv_done), so the next
-                // item's Q goes in now, beside this item's TAC product
-                if (i + 1 < my_items) put_q(i + 1);
             }
             // epilogue 2: + d, rounded to T, TMA store from the ring slot of
             // entry 3 nk + 2
@@ -668,9 +680,6 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_k, const _
                 tc_fence_after();
                 tmem_ld_32x32b_x32(tl + TM_TAC + col, r);
                 tmem_ld_wait();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(B(sh->tac_read));     // the TAC columns may be reused
                 const uint32_t box = slot(go) + (uint32_t)warp * 2048;
                 const bool add_d = a.d != nullptr;
                 #pragma unroll
@@ -731,8 +740,9 @@ cudaError_t launch_pv_tac(const AttnArgs& a, cudaStream_t stream) {
     const int C = ATTN_D * a.H, Ckv = ATTN_D * a.Hkv;
     const CUtensorMapDataType io = std::is_same<T, __half>::value ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
                                                                    : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
-    CUtensorMap tk, tv, tz;
-    if (!encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)Ckv, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B, io) ||
+    CUtensorMap tq, tk, tv, tz;
+    if (!encode_2d(&tq, a.Q, (uint64_t)a.L, (uint64_t)C, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B, io) ||
+        !encode_2d(&tk, a.K, (uint64_t)a.L, (uint64_t)Ckv, (uint64_t)a.ld, ATTN_TILE, 64, CU_TENSOR_MAP_SWIZZLE_128B, io) ||
         !encode_2d(&tv, a.Vt, (uint64_t)Ckv, (uint64_t)a.L, (uint64_t)a.L, ATTN_D, 64, CU_TENSOR_MAP_SWIZZLE_128B) ||
         !encode_2d(&tz, a.Z, (uint64_t)a.L, (uint64_t)C, (uint64_t)C, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B, io))
         return cudaErrorInvalidValue;
@@ -750,7 +760,7 @@ cudaError_t launch_pv_tac(const AttnArgs& a, cudaStream_t stream) {
     const int items = a.L / ATTN_TILE * a.H;
     const int per_cta = (items + num_sms() - 1) / num_sms();
     const int grid = (items + per_cta - 1) / per_cta;
-    attn_pv_tac_kernel<T><<<grid, ATT_THREADS, ATT_SMEM, stream>>>(a, tk, tv, tz);
+    attn_pv_tac_kernel<T><<<grid, ATT_THREADS, ATT_SMEM, stream>>>(a, tq, tk, tv, tz);
     return cudaGetLastError();
 }
 
