@@ -37,28 +37,26 @@
 //                      (tcgen05 kind::f16 on one CTA, M = N = 128, K = 16)
 //                      with the A operand (Q, P, Z_hat) in tensor memory and
 //                      B (K, V, M) in shared memory.
-//   prologue  the softmax warps write the Q tile into TMEM.
-//   pass 1  S = Q K^T chunk by chunk (128 keys; three TMEM buffers, the
-//           third in the columns of the P V^T accumulator, which pass 1
-//           does not use); each thread keeps the running maximum of its
-//           row's part of S.
-//   pass 2  S again (two buffers); each thread turns its 32 scores into
-//           e = exp2((s - m) log2(e) / sqrt(d)) (ex2.approx), adds them to l
-//           (four partial sums) and writes the codes rne(255 e), rounded
-//           exactly by a float32 bias whose low bits are fp16 1024 + code,
-//           as fp16 over the S columns it has read. P is thus double-
-//           buffered with S, and the next chunk's probabilities need not
-//           wait for this P V^T. The MMA warp accumulates P V^T one chunk
-//           behind the scores (exact integers).
+//   prologue  the softmax warps copy the Q tile (loaded by TMA) into TMEM.
+//   pass 1  S = Q K^T chunk by chunk (128 keys, two TMEM buffers); each
+//           thread keeps the running maximum of its row's part of S.
+//   pass 2  S again; each thread turns its 32 scores into
+//           e = exp2(s c - m c), c = log2(e) / sqrt(d) (one fma, ex2.approx),
+//           adds them to l (four partial sums) and writes the codes
+//           rne(255 e), rounded exactly by a float32 bias whose low bits
+//           are fp16 1024 + code, as fp16 over the S columns it has read.
+//           The MMA warp then accumulates P V^T (exact integers) and
+//           computes the scores two chunks ahead into the same buffer.
 //   epilogue  Z_hat from the accumulator, split into fp16 hi + lo (Z_hat =
 //           hi + lo to ~2^-22), written to TMEM as the A operands of the
 //           TAC product Z_hi M_hi^T + Z_hi M_lo^T + Z_lo M_hi^T with M's
-//           prepared halves (tac_prepare); + d; rounded to fp16 and stored
-//           by TMA.
-// Shared memory holds only B operands: a ring of six 32 KB tiles streams
-// each item's pass-1 K chunks, pass-2 K and V chunks, M's two halves and
-// then the slot of its output boxes, in the order they are used, running
-// on into the next item.
+//           prepared halves (tac_prepare); + d; rounded to the I/O type and
+//           stored by TMA (stores straight from registers, 64 bytes per
+//           thread and row, measured slower).
+// Shared memory holds only operand tiles and the output boxes: a ring of
+// six 32 KB tiles streams each item's Q tile, pass-1 K chunks, pass-2 K and
+// V chunks, M's two halves and then the slot of its output boxes, in the
+// order they are used, running on into the next item.
 // TMEM (512 columns): two S / P buffers (pass 1 also uses the P V^T
 // accumulator's columns as a third), the P V^T accumulator and Q; the TAC
 // accumulator and Z_hat reuse the S buffers. The tensor pipe keeps almost
@@ -579,6 +577,10 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
             named_sync_softmax();
             // pass 2: probabilities, their codes and the row sums
             float lp[4] = {0.f, 0.f, 0.f, 0.f};      // partial row sums (independent chains)
+            // the exponent as one fma: s c - m c differs from (s - m) c by an
+            // ulp of m c at most, ~1e-6 in e at |m| <= 100 (the codes' rounding
+            // decisions move only within 3e-4 of a half-integer)
+            const float mxc = __fmul_rn(mx, EXP_SCALE);
             for (int j = 0; j < nk && ok; ++j) {
                 int b, n;
                 sbuf(i, nk + j, b, n);
@@ -594,8 +596,8 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
                 const __half2 minus1024 = __float2half2_rn(-1024.f);
                 #pragma unroll
                 for (int k = 0; k < 32; k += 2) {
-                    const float e0 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k]), mx), EXP_SCALE));
-                    const float e1 = ex2_approx(__fmul_rn(__fsub_rn(__uint_as_float(r[k + 1]), mx), EXP_SCALE));
+                    const float e0 = ex2_approx(__fmaf_rn(__uint_as_float(r[k]), EXP_SCALE, -mxc));
+                    const float e1 = ex2_approx(__fmaf_rn(__uint_as_float(r[k + 1]), EXP_SCALE, -mxc));
                     lp[(k >> 1) & 1] += e0;
                     lp[2 + ((k >> 1) & 1)] += e1;
                     const uint32_t t0 = __float_as_uint(fmaf(255.f, e0, ROUND_BIAS));
@@ -684,14 +686,17 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
                 const bool add_d = a.d != nullptr;
                 #pragma unroll
                 for (int g = 0; g < 4; ++g) {
+                    const float4 d0 = *reinterpret_cast<const float4*>(&sh->dv[col + 8 * g]);
+                    const float4 d1 = *reinterpret_cast<const float4*>(&sh->dv[col + 8 * g + 4]);
+                    const float dk[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
                     uint32_t w[4];
                     #pragma unroll
                     for (int u = 0; u < 4; ++u) {
                         const int k = 8 * g + 2 * u;
                         float y0 = __fmul_rn(__uint_as_float(r[k]), zunscale), y1 = __fmul_rn(__uint_as_float(r[k + 1]), zunscale);
                         if (add_d) {
-                            y0 = __fadd_rn(y0, sh->dv[col + k]);
-                            y1 = __fadd_rn(y1, sh->dv[col + k + 1]);
+                            y0 = __fadd_rn(y0, dk[2 * u]);
+                            y1 = __fadd_rn(y1, dk[2 * u + 1]);
                         }
                         w[u] = pack2(T(), y0, y1);
                     }
