@@ -52,6 +52,9 @@ def parse():
     p.add_argument("--ref-sample-tokens", type=int, default=128)
     p.add_argument("--skip-cpu-baseline", action="store_true")
     p.add_argument("--skip-stack", action="store_true", help="leave out the short denoising-stack run")
+    p.add_argument("--forked-step", action="store_true",
+                   help="attention_step: run the two projections as forked branches with a GEMM launch each "
+                        "(the default groups both GEMMs into one launch)")
     p.add_argument("--workload", default="attention_step",
                    choices=["attention_step", "denoise_stack", "tac_calibration", "attention_pv_tac", "w8a8_linear",
                             "asym_linear", "dense_linear", "dream_block", "hbm_passes", "llada_mlp",
@@ -82,12 +85,14 @@ def load_peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
-def config_dict(graph):
+def config_dict(graph, grouped=True):
     return {"workload": "llada8b_attention_projections_step", "tokens": 1024, "hidden": 4096,
             "qkv": "4096->12288", "o": "4096->4096", "tac_block": 128, "hadamard_block": 4096,
             "gates": "d_m = d_u = 128", "mask": "0..639 unmasked, 640..1023 masked",
             "l2": "flushed between timed steps (256 MiB write)", "cuda_graph": bool(graph),
-            "streams": "QKV and TAC + O branches forked and joined within the step"}
+            "streams": ("the QKV quantiser beside TAC + the O quantiser (two streams), then both GEMMs in one "
+                        "grouped launch" if grouped else
+                        "QKV and TAC + O branches forked and joined within the step")}
 
 
 # ---------------------------------------------------------------------------
@@ -169,8 +174,9 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
-    """DRAM bytes per launch of the GEMM from the committed ncu summary, if it
+def profiled_traffic(grouped=True):
+    """DRAM bytes per launch of the GEMM from the committed ncu summary (the
+    grouped QKV + O launch, or the mean of the two single launches), if it
     was taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", "w4a4_gemm_llada_qkv_traffic.txt")
     try:
@@ -182,7 +188,7 @@ def profiled_traffic():
                     kv[k.strip()] = v.strip()
         if kv.get("kernel_source_sha256_16") != kernel_source_hash():
             return None
-        return float(kv["dram_bytes_per_launch_avg"])
+        return float(kv["dram_bytes_per_launch_grouped" if grouped else "dram_bytes_per_launch_avg"])
     except Exception:
         return None
 
@@ -613,7 +619,8 @@ def run_ours(args):
     from paper_2606_04945_gb300.pipeline import AttentionProjections
 
     qkv_case, o_case = inputs.llada_attention(seed=rank_seed(rank))
-    step = AttentionProjections(qkv_case, o_case)
+    grouped = not args.forked_step
+    step = AttentionProjections(qkv_case, o_case, grouped=grouped)
     L, K = step.L, step.qkv.K
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
     flush = lambda: flush_buf.zero_()
@@ -672,6 +679,12 @@ def run_ours(args):
                             flush, torch)
     s_gemm_o = time_stream([lambda i=i: abi.w4a4_gemm(None, s_a, o.Wq, o.s_w, step.Y_o, Xe=Xer[i % 3], We=Wr_o[i])
                             for i in range(8)], flush, torch, rounds=3)
+    # both GEMMs in one grouped launch, as the default step runs them
+    s_gemm_grp = time_stream([lambda i=i: abi.w4a4_gemm_grouped(Xer[i % 3], s_a, Wr_q[i % 3], q.s_w, step.Y_qkv,
+                                                                Xer[(i + 1) % 3], s_a, Wr_o[i], o.s_w, step.Y_o)
+                              for i in range(8)], flush, torch, rounds=3)
+    t_gemm_grp = time_kernel(lambda: abi.w4a4_gemm_grouped(Xe, s_a, q.We, q.s_w, step.Y_qkv, Xe, s_a, o.We, o.s_w,
+                                                           step.Y_o), flush, reps, torch)
     abi.check_status()
     del Xr, Zr, Zf, Wr_q, Wr_o, Xer
     large = hbm_passes_large(abi, o, flush, torch)
@@ -791,7 +804,7 @@ def run_ours(args):
     tokens_s = world * L / (ms * 1e-3)
     peaks, peak_src = load_peaks()
     gemm_ops = q.int_ops() + o.int_ops()
-    gemm_ms = s_gemm_qkv + s_gemm_o
+    gemm_ms = s_gemm_grp if grouped else s_gemm_qkv + s_gemm_o
     achieved = gemm_ops / (gemm_ms * 1e-3) / 1e12
     peak_bf16x2 = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]) * FP8_PER_BF16
     pair_probe = probes[abi.PROBE_KINDS[1]]
@@ -800,7 +813,7 @@ def run_ours(args):
     quant_x_bytes = L * K * 2 + L * K // 2 + L * K + 4 * L     # X in; packed + E4M3 codes, scales out
     quant_z_bytes = L * K * 2 + L * K // 2 + L * K + 4 * L             # the TAC output (16-bit) in
     tac_bytes = L * K * 2 + L * K * 2 + K * o.tac_g * 4 + K * 4      # Z in, 16-bit out, M (prepared: 4 C g B), d
-    traffic = profiled_traffic()
+    traffic = profiled_traffic(grouped)
     wbytes = lambda lin: lin.N * K if lin.We is not None else lin.N * K // 2
     gemm_bytes = [L * K + wbytes(q) + 2 * L * q.N + 4 * (L + q.N),    # E4M3 codes, weights, fp16 out
                   L * K + wbytes(o) + 2 * L * o.N + 4 * (L + o.N)]
@@ -816,10 +829,12 @@ def run_ours(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "int4 (W4A4 codes, exact integer accumulation; fp32 transform and dequant; fp16 I/O)",
         "data": "synthetic (seeded; LLaDA-8B-shaped activations and random-init weights)",
-        "config": config_dict(graph),
+        "config": config_dict(graph, grouped),
         "tokens_per_s": round(tokens_s, 1),
         "roofline": {
-            "bound": "tensor", "kernel": "w4a4_gemm_tma_pair_kernel (QKV + O launches)",
+            "bound": "tensor",
+            "kernel": ("w4a4_gemm_tma_pair_kernel (QKV and O tiles in one grouped launch)" if grouped
+                       else "w4a4_gemm_tma_pair_kernel (QKV + O launches)"),
             "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
             "frac": round(achieved / peak, 4), "traffic": traffic,
             "peak_source": "starq_probe_mma kind 1 (tcgen05 kind::f8f6f4 cta_group::2 back-to-back MMAs on "
@@ -827,12 +842,13 @@ def run_ours(args):
                            "issues; sm_103a has no integer tcgen05 MMA",
             "peak_bf16x2": round(peak_bf16x2, 1), "frac_bf16x2": round(achieved / peak_bf16x2, 4),
             "peak_bf16x2_source": f"{peak_src} bf16 dense burst x {FP8_PER_BF16} (nominal fp8 / bf16 ratio)",
-            "per_launch_frac": {"qkv": round(q.int_ops() / (s_gemm_qkv * 1e-3) / 1e12 / peak, 4),
+            "per_launch_frac": {"grouped": round(gemm_ops / (s_gemm_grp * 1e-3) / 1e12 / peak, 4),
+                                "qkv": round(q.int_ops() / (s_gemm_qkv * 1e-3) / 1e12 / peak, 4),
                                 "o": round(o.int_ops() / (s_gemm_o * 1e-3) / 1e12 / peak, 4)},
-            "algorithmic": f"{gemm_ops} int ops per step over 2 launches; "
+            "algorithmic": f"{gemm_ops} int ops per step over {1 if grouped else 2} launch(es); "
                            f"{sum(gemm_bytes)} algorithmic bytes per step",
-            "stream_ms": {"qkv": round(s_gemm_qkv, 5), "o": round(s_gemm_o, 5)},
-            "launch_ms": {"qkv": round(t_gemm_qkv, 5), "o": round(t_gemm_o, 5)},
+            "stream_ms": {"grouped": round(s_gemm_grp, 5), "qkv": round(s_gemm_qkv, 5), "o": round(s_gemm_o, 5)},
+            "launch_ms": {"grouped": round(t_gemm_grp, 5), "qkv": round(t_gemm_qkv, 5), "o": round(t_gemm_o, 5)},
             "timing": "stream_ms: back-to-back launches over rotating operand sets larger than L2 (the "
                       "roofline's duration); launch_ms: one launch after an L2 flush, launch latency included",
         },

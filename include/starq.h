@@ -369,6 +369,31 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
               int y_dtype, const starq_tac* out_tac, int32_t* acc_dbg, void* stream);
 
 /*
+ * w4a4_gemm_grouped -- two independent W4A4 products of w4a4_gemm's
+ * definition (Sec. 3.2 Eq. 13, Sec. 3.1 Eq. 3 and Eq. 5) in one launch:
+ * Y0 = dequant(Xe0 We0^T) and Y1 = dequant(Xe1 We1^T), with the same L, K
+ * and output type (e.g. the QKV projection of X and the O projection of the
+ * compensated attention output, which share their token count and width).
+ * The output tiles of problem 1 follow those of problem 0 in one persistent
+ * stream of CTA-pair tiles, so a short problem's pipeline fill and drain
+ * hide behind the other's tiles. Each output is bit-identical to a
+ * w4a4_gemm call with Xe and We.
+ *
+ *   Xe0 [L][K], Xe1 [L][K]: E4M3 activation codes; We0 [N0][K], We1 [N1][K]:
+ *      E4M3 weight codes (w4_unpack_e4m3); all 16-byte aligned, device
+ *      memory of the current device (the caller owns every buffer).
+ *   s_a0, s_a1 [L], s_w0 [N0], s_w1 [N1] float32; bias0, bias1 or NULL.
+ *   Y0 [L][N0], Y1 [L][N1] of y_dtype (F16, BF16 or F32), 16-byte aligned.
+ *   acc_dbg0, acc_dbg1: the exact int32 accumulators, or NULL.
+ * Shapes and errors as w4a4_gemm for each problem (N0, N1 >= 32 and
+ * multiples of 32; 128 <= K <= 65536, K % 128 == 0); L == 0 does nothing.
+ */
+int w4a4_gemm_grouped(const uint8_t* Xe0, const float* s_a0, const uint8_t* We0, const float* s_w0,
+                      const float* bias0, int N0, void* Y0, const uint8_t* Xe1, const float* s_a1,
+                      const uint8_t* We1, const float* s_w1, const float* bias1, int N1, void* Y1, int L, int K,
+                      int y_dtype, int32_t* acc_dbg0, int32_t* acc_dbg1, void* stream);
+
+/*
  * starq_set_gemm_pair_limit -- at most `pairs` CTA pairs (two SMs each) for
  * the W4A4 and 16-bit TMA pair GEMMs launched afterwards from the calling
  * thread (w4a4_gemm with Xe and We, the sgat_linear family, fp16_gemm_ref);

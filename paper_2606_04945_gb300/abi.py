@@ -27,7 +27,7 @@ EXPORTED = (
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
     "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
     "starq_selftest_wait_timeout", "starq_probe_mma", "attention_pv_tac_gqa", "glue_add_rmsnorm", "glue_rope",
-    "w4a4_gemm_mma_sync", "starq_set_gemm_pair_limit",
+    "w4a4_gemm_mma_sync", "starq_set_gemm_pair_limit", "w4a4_gemm_grouped",
 )
 
 
@@ -76,6 +76,8 @@ def _load():
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp, vp]
     lib.w8_split_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm_mma_sync.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.w4a4_gemm_grouped.argtypes = [u8p, f_p, u8p, f_p, f_p, i, vp, u8p, f_p, u8p, f_p, f_p, i, vp, i, i, i, vp,
+                                      vp, vp]
     lib.starq_set_gemm_pair_limit.argtypes = [i]
     lib.starq_set_gemm_pair_limit.restype = i
     lib.w8a8_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
@@ -310,6 +312,20 @@ def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, st
     tac = _tac_struct(tac_M, tac_d, tac_g, tac_Mp, tac_scratch)
     _check(lib.w4a4_gemm(_p(Xq), _p(Xe), _p(s_a), _p(Wq), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y),
                          dtype_code(Y), _ref(tac), _p(acc_dbg), _stream(stream)))
+
+
+def w4a4_gemm_grouped(Xe0, s_a0, We0, s_w0, Y0, Xe1, s_a1, We1, s_w1, Y1, bias0=None, bias1=None,
+                      acc_dbg0=None, acc_dbg1=None, stream=None):
+    """Two independent W4A4 products (same L, K and output type) in one
+    launch: Y0 from Xe0 [L][K] and We0 [N0][K], Y1 from Xe1 and We1 (E4M3
+    codes)."""
+    _contig(Xe0, s_a0, We0, s_w0, Y0, bias0, acc_dbg0, Xe1, s_a1, We1, s_w1, Y1, bias1, acc_dbg1)
+    L, K = Xe0.shape
+    if tuple(Xe1.shape) != (L, K) or Y0.dtype != Y1.dtype:
+        raise StarqError(-2, "w4a4_gemm_grouped: the problems need the same L, K and output type")
+    _check(lib.w4a4_gemm_grouped(_p(Xe0), _p(s_a0), _p(We0), _p(s_w0), _p(bias0), We0.shape[0], _p(Y0),
+                                 _p(Xe1), _p(s_a1), _p(We1), _p(s_w1), _p(bias1), We1.shape[0], _p(Y1), L, K,
+                                 dtype_code(Y0), _p(acc_dbg0), _p(acc_dbg1), _stream(stream)))
 
 
 def w4a4_gemm_mma_sync(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, stream=None):

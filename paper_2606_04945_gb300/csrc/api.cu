@@ -394,6 +394,29 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
     return STARQ_OK;
 }
 
+int w4a4_gemm_grouped(const uint8_t* Xe0, const float* s_a0, const uint8_t* We0, const float* s_w0,
+                      const float* bias0, int N0, void* Y0, const uint8_t* Xe1, const float* s_a1,
+                      const uint8_t* We1, const float* s_w1, const float* bias1, int N1, void* Y1, int L, int K,
+                      int y_dtype, int32_t* acc_dbg0, int32_t* acc_dbg1, void* stream) {
+    if (!We0 || !We1) return fail(STARQ_ERR_ARG, "w4a4_gemm_grouped: NULL We0 or We1");
+    if (L > 0 && (!Xe0 || !Xe1)) return fail(STARQ_ERR_ARG, "w4a4_gemm_grouped: NULL Xe0 or Xe1");
+    int rc = check_gemm(nullptr, Xe0, s_a0, nullptr, We0, s_w0, bias0, L, N0, K, Y0, y_dtype);
+    if (rc) return rc;
+    if ((rc = check_gemm(nullptr, Xe1, s_a1, nullptr, We1, s_w1, bias1, L, N1, K, Y1, y_dtype))) return rc;
+    if ((acc_dbg0 && !aligned(acc_dbg0, 16)) || (acc_dbg1 && !aligned(acc_dbg1, 16)))
+        return fail(STARQ_ERR_ALIGN, "w4a4_gemm_grouped: acc_dbg must be 16-byte aligned");
+    if (L == 0) return STARQ_OK;
+    if ((rc = check_local("w4a4_gemm_grouped", static_cast<cudaStream_t>(stream), {Xe0, We0, Y0, Xe1, We1, Y1})))
+        return rc;
+    unsigned* st = status_ptr(&rc);
+    if (!st) return rc;
+    GemmArgs a{nullptr, s_a0, nullptr, s_w0, bias0, L, N0, K, Y0, y_dtype, acc_dbg0, st, Xe0, We0};
+    GemmArgs b{nullptr, s_a1, nullptr, s_w1, bias1, L, N1, K, Y1, y_dtype, acc_dbg1, st, Xe1, We1};
+    cudaError_t e = launch_w4a4_gemm_grouped(a, b, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm_grouped launch");
+    return STARQ_OK;
+}
+
 int starq_set_gemm_pair_limit(int pairs) {
     if (pairs < 0) return fail(STARQ_ERR_ARG, "starq_set_gemm_pair_limit: pairs=%d < 0", pairs);
     return set_gemm_pair_limit(pairs);

@@ -64,6 +64,9 @@ struct GemmArgs {
     int swiglu = 0;
 };
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream);
+// Two independent products in one persistent TMA pair launch (the same L,
+// K and output type; Xe and We given for both; no SwiGLU).
+cudaError_t launch_w4a4_gemm_grouped(const GemmArgs& a, const GemmArgs& b, cudaStream_t stream);
 // Thread-local cap on the CTA pairs of the TMA pair GEMMs launched from the
 // calling thread (0 = none); returns the previous cap.
 int set_gemm_pair_limit(int pairs);

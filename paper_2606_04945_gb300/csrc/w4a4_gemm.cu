@@ -854,10 +854,15 @@ long long tma_round_cost(int L, int N, int BN, int clusters) {
 // 16 k .. 16 k + 15, then the matching up rows), so every 32-column chunk
 // of the accumulator holds 16 gate and 16 up channels; the epilogue writes
 // silu(gate) * up, rounded once, to column nc / 2 of an [L][N / 2] output.
-template <typename TOut, int OPK, int BN, bool SWIGLU = false>
+// G2: a second, independent problem b (the same L, K and output type) whose
+// tiles follow a's in the one persistent tile stream, so that a short
+// problem's pipeline fill and drain hide behind the other's tiles.
+template <typename TOut, int OPK, int BN, bool SWIGLU = false, bool G2 = false>
 __global__ void __launch_bounds__(tmak::THREADS, 1)
 w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a,
-                          const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y) {
+                          const __grid_constant__ CUtensorMap tmap_b, const __grid_constant__ CUtensorMap tmap_y,
+                          GemmArgs b, const __grid_constant__ CUtensorMap tmap_a2,
+                          const __grid_constant__ CUtensorMap tmap_b2, const __grid_constant__ CUtensorMap tmap_y2) {
     using Tile = tmak::Tile<BN>;
     using Cfg = tmak::Cfg<sizeof(TOut), BN>;
     constexpr int BM = tmak::BM, BN_CTA = Tile::BN_CTA, BK = tmak::BK;
@@ -885,8 +890,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     const uint32_t half = cluster_ctarank(), leader = 0;
     const int L = a.L, N = a.N, K = a.K;
     const int num_m = (L + 2 * BM - 1) / (2 * BM);
-    const int num_n = (N + BN - 1) / BN;
-    const int num_tiles = num_m * num_n;
+    const int num_tiles0 = num_m * ((N + BN - 1) / BN);  // problem a's tiles, then problem b's
+    const int num_tiles = num_tiles0 + (G2 ? num_m * ((b.N + BN - 1) / BN) : 0);
     const int num_k = K / BKE;
     const int cluster = blockIdx.x / 2, num_clusters = gridDim.x / 2;
 
@@ -926,11 +931,14 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         int pre = 0;
         if (a.weights_ready && cluster < num_tiles) {
             pre = num_k < STAGES ? num_k : STAGES;
-            const int n_rows = (cluster / num_m) * BN + (int)half * BN_CTA;
+            const bool p1 = G2 && cluster >= num_tiles0;
+            const int lt = p1 ? cluster - num_tiles0 : cluster;
+            const void* mb = p1 ? (const void*)&tmap_b2 : (const void*)&tmap_b;
+            const int n_rows = (lt / num_m) * BN + (int)half * BN_CTA;
             for (int kc = 0; kc < pre; ++kc) {
                 if (elect_one()) {
                     if (half == 0) mbar_arrive_expect_tx(smem_addr(&sh->full[kc]), 2 * (A_BYTES + B_BYTES));
-                    tma_load_2d_pair(base + kc * STAGE_BYTES + A_BYTES, &tmap_b, kc * BKE, n_rows,
+                    tma_load_2d_pair(base + kc * STAGE_BYTES + A_BYTES, mb, kc * BKE, n_rows,
                                      leader_full0 + kc * 8);
                 }
                 __syncwarp();
@@ -941,8 +949,12 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         uint32_t phase = 0;
         bool ok = true;
         for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters) {
-            const int m_rows = (tile % num_m) * 2 * BM + (int)half * BM;
-            const int n_rows = (tile / num_m) * BN + (int)half * BN_CTA;
+            const bool p1 = G2 && tile >= num_tiles0;
+            const int lt = p1 ? tile - num_tiles0 : tile;
+            const void* ma = p1 ? (const void*)&tmap_a2 : (const void*)&tmap_a;
+            const void* mb = p1 ? (const void*)&tmap_b2 : (const void*)&tmap_b;
+            const int m_rows = (lt % num_m) * 2 * BM + (int)half * BM;
+            const int n_rows = (lt / num_m) * BN + (int)half * BN_CTA;
             for (int kc = 0; kc < num_k; ++kc) {
                 const bool early = tile == cluster && kc < pre;  // weights already in flight
                 if (!early && !mbar_wait_bounded_warp(smem_addr(&sh->empty[stage]), phase ^ 1u, abort)) { ok = false; break; }
@@ -950,8 +962,8 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 const uint32_t bar = leader_full0 + stage * 8;
                 if (elect_one()) {
                     if (half == 0 && !early) mbar_arrive_expect_tx(smem_addr(&sh->full[stage]), 2 * (A_BYTES + B_BYTES));
-                    tma_load_2d_pair(st, &tmap_a, kc * BKE, m_rows, bar);
-                    if (!early) tma_load_2d_pair(st + A_BYTES, &tmap_b, kc * BKE, n_rows, bar);
+                    tma_load_2d_pair(st, ma, kc * BKE, m_rows, bar);
+                    if (!early) tma_load_2d_pair(st + A_BYTES, mb, kc * BKE, n_rows, bar);
                 }
                 __syncwarp();
                 if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -1018,19 +1030,24 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
         int it = 0;
         int nbox = 0;
         for (int tile = cluster; tile < num_tiles; tile += num_clusters, ++it) {
-            const int m0 = (tile % num_m) * 2 * BM + (int)half * BM;
-            const int n0 = (tile / num_m) * BN;
+            const bool p1 = G2 && tile >= num_tiles0;
+            const int lt = p1 ? tile - num_tiles0 : tile;
+            const GemmArgs& P = p1 ? b : a;
+            const void* my = p1 ? (const void*)&tmap_y2 : (const void*)&tmap_y;
+            const int N = P.N;
+            const int m0 = (lt % num_m) * 2 * BM + (int)half * BM;
+            const int n0 = (lt / num_m) * BN;
             const int acc = it & 1;
             const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
             const int row = m0 + quarter * 32 + lane;
             const bool valid = row < L;
-            const float sa = (DEQUANT && valid) ? __ldg(a.s_a + row) : 0.f;
+            const float sa = (DEQUANT && valid) ? __ldg(P.s_a + row) : 0.f;
             if (DEQUANT) {
                 const int ncol = n0 + chalf * (EPI_CHUNKS * 32) + 4 * lane;
                 float4 w = make_float4(0.f, 0.f, 0.f, 0.f), bb = w;
                 if (ncol < N) {
-                    w = __ldg(reinterpret_cast<const float4*>(a.s_w + ncol));
-                    if (a.bias != nullptr) bb = __ldg(reinterpret_cast<const float4*>(a.bias + ncol));
+                    w = __ldg(reinterpret_cast<const float4*>(P.s_w + ncol));
+                    if (P.bias != nullptr) bb = __ldg(reinterpret_cast<const float4*>(P.bias + ncol));
                 }
                 __syncwarp();
                 reinterpret_cast<float4*>(epi_sw)[lane] = w;
@@ -1059,7 +1076,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                     y[4 * u + 2] = __uint_as_float(r[4 * u + 2]);
                     y[4 * u + 3] = __uint_as_float(r[4 * u + 3]);
                 }
-                if (DEQUANT && a.bias == nullptr) {
+                if (DEQUANT && P.bias == nullptr) {
                     // fl(fl(acc s_a) s_w) on packed pairs (two multiplies: nothing to contract)
                     #pragma unroll
                     for (int u = 0; u < 8; ++u) {
@@ -1079,7 +1096,7 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                         y[4 * u + 3] = __fmul_rn(__fmul_rn(__uint_as_float(r[4 * u + 3]), sa), sw.w);
                     }
                 }
-                if (DEQUANT && a.bias != nullptr) {
+                if (DEQUANT && P.bias != nullptr) {
                     #pragma unroll
                     for (int u = 0; u < 8; ++u) {
                         const float4 bq = b4[u];
@@ -1108,12 +1125,12 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) {
-                    tma_store_2d(&tmap_y, SWIGLU ? nc / 2 : nc, m0 + quarter * 32, box);
+                    tma_store_2d(my, SWIGLU ? nc / 2 : nc, m0 + quarter * 32, box);
                     bulk_commit();
                 }
                 ++nbox;
-                if (a.acc_dbg != nullptr && valid) {
-                    int4* d4 = reinterpret_cast<int4*>(a.acc_dbg + (size_t)row * N + nc);
+                if (P.acc_dbg != nullptr && valid) {
+                    int4* d4 = reinterpret_cast<int4*>(P.acc_dbg + (size_t)row * N + nc);
                     #pragma unroll
                     for (int u = 0; u < 8; ++u)
                         d4[u] = make_int4(__float2int_rn(__uint_as_float(r[4 * u])),
@@ -1146,12 +1163,12 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
 // Clusters (CTA pairs) of this instantiation resident at once on the current
 // device (queried once per device; also sets the kernel's shared-memory
 // limit).
-template <typename TOut, int OPK, int BN, bool SW>
+template <typename TOut, int OPK, int BN, bool SW, bool G2 = false>
 cudaError_t tma_max_clusters(int* clusters) {
     constexpr size_t SMEM_BYTES = tmak::Cfg<sizeof(TOut), BN>::SMEM_BYTES;
     static DeviceCache<int> cache;
     return cache.get(clusters, [](int, int* v) {
-        auto kernel = w4a4_gemm_tma_pair_kernel<TOut, OPK, BN, SW>;
+        auto kernel = w4a4_gemm_tma_pair_kernel<TOut, OPK, BN, SW, G2>;
         cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
         if (e != cudaSuccess) return e;
         cudaLaunchConfig_t cfg = {};
@@ -1173,8 +1190,9 @@ cudaError_t tma_max_clusters(int* clusters) {
     });
 }
 
-template <typename TOut, int OPK, int BN, bool SW>
-cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) {
+// b: the second problem of a grouped launch (G2), else unused.
+template <typename TOut, int OPK, int BN, bool SW, bool G2 = false>
+cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters, const GemmArgs* b = nullptr) {
     constexpr int BM = tmak::BM, BN_CTA = tmak::Tile<BN>::BN_CTA, BK = tmak::BK;
     constexpr int ELEM = OPK == 0 ? 1 : 2;
     cudaLaunchConfig_t cfg = {};
@@ -1189,19 +1207,30 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters) 
     cfg.stream = stream;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    CUtensorMap ta, tb, ty;
+    CUtensorMap ta, tb, ty, ta2, tb2, ty2;
     const CUtensorMapDataType opt = OPK == 0 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16;
-    if (!encode_operand_tmap(&ta, a.Xe, opt, ELEM, (uint64_t)a.L, (uint64_t)a.K, BM, BK / ELEM) ||
-        !encode_operand_tmap(&tb, a.We, opt, ELEM, (uint64_t)a.N, (uint64_t)a.K, BN_CTA, BK / ELEM) ||
-        !(SW ? encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N / 2,
-                               CU_TENSOR_MAP_SWIZZLE_32B, 16)
-             : encode_out_tmap(&ty, a.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)a.L, (uint64_t)a.N,
-                               Out<TOut>::TMAP_SWIZZLE)))
-        return cudaErrorInvalidValue;
-    const int num_tiles = tma_tiles(a.L, a.N, BN);
+    auto maps = [&](const GemmArgs& p, CUtensorMap* xa, CUtensorMap* xb, CUtensorMap* xy) {
+        return encode_operand_tmap(xa, p.Xe, opt, ELEM, (uint64_t)p.L, (uint64_t)p.K, BM, BK / ELEM) &&
+               encode_operand_tmap(xb, p.We, opt, ELEM, (uint64_t)p.N, (uint64_t)p.K, BN_CTA, BK / ELEM) &&
+               (SW ? encode_out_tmap(xy, p.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)p.L, (uint64_t)p.N / 2,
+                                     CU_TENSOR_MAP_SWIZZLE_32B, 16)
+                   : encode_out_tmap(xy, p.Y, Out<TOut>::TMAP_TYPE, sizeof(TOut), (uint64_t)p.L, (uint64_t)p.N,
+                                     Out<TOut>::TMAP_SWIZZLE));
+    };
+    if (!maps(a, &ta, &tb, &ty)) return cudaErrorInvalidValue;
+    int num_tiles = tma_tiles(a.L, a.N, BN);
+    if (G2) {
+        if (b == nullptr || !maps(*b, &ta2, &tb2, &ty2)) return cudaErrorInvalidValue;
+        num_tiles += tma_tiles(b->L, b->N, BN);
+    } else {
+        ta2 = ta;
+        tb2 = tb;
+        ty2 = ty;
+    }
     if (num_tiles < clusters) clusters = num_tiles;
     cfg.gridDim = dim3(2 * clusters);
-    return cudaLaunchKernelEx(&cfg, w4a4_gemm_tma_pair_kernel<TOut, OPK, BN, SW>, a, ta, tb, ty);
+    return cudaLaunchKernelEx(&cfg, w4a4_gemm_tma_pair_kernel<TOut, OPK, BN, SW, G2>, a, ta, tb, ty,
+                              G2 ? *b : a, ta2, tb2, ty2);
 }
 
 // Tile shape per problem. A stage's steady state is bound by shared memory:
@@ -1229,6 +1258,33 @@ cudaError_t launch_tma_shape(const GemmArgs& a, cudaStream_t stream) {
     }
     g_last_tile = 256 * 10 + 2;
     return launch_tma_cl<TOut, OPK, 256, SW>(a, stream, c256);
+}
+
+// Two independent problems (same L, K and output type, E4M3 operands, no
+// SwiGLU) in one persistent launch: the tile width is chosen for the two
+// together.
+template <typename TOut>
+cudaError_t launch_tma_grouped(const GemmArgs& a, const GemmArgs& b, cudaStream_t stream) {
+    int c256 = 0, c224 = 0;
+    cudaError_t e = tma_max_clusters<TOut, 0, 256, false, true>(&c256);
+    if (e != cudaSuccess) return e;
+    if ((e = tma_max_clusters<TOut, 0, 224, false, true>(&c224)) != cudaSuccess) return e;
+    if (g_pair_limit > 0) {
+        if (c256 > g_pair_limit) c256 = g_pair_limit;
+        if (c224 > g_pair_limit) c224 = g_pair_limit;
+    }
+    auto cost = [&](int bn, int cl) {
+        const long long tiles = tma_tiles(a.L, a.N, bn) + tma_tiles(b.L, b.N, bn);
+        const long long used = cl < 1 ? 1 : cl;
+        const long long stage2 = 4LL * bn > 512LL + 3LL * bn ? 4LL * bn : 512LL + 3LL * bn;
+        return (tiles + used - 1) / used * stage2;
+    };
+    if (cost(224, c224) < cost(256, c256)) {
+        g_last_tile = 224 * 10 + 2;
+        return launch_tma_cl<TOut, 0, 224, false, true>(a, stream, c224, &b);
+    }
+    g_last_tile = 256 * 10 + 2;
+    return launch_tma_cl<TOut, 0, 256, false, true>(a, stream, c256, &b);
 }
 
 template <typename TOut, int OPK = 0>
@@ -1342,6 +1398,19 @@ int set_gemm_pair_limit(int pairs) {
     const int prev = g_pair_limit;
     g_pair_limit = pairs;
     return prev;
+}
+
+cudaError_t launch_w4a4_gemm_grouped(const GemmArgs& a, const GemmArgs& b, cudaStream_t stream) {
+    if (a.L != b.L || a.K != b.K || a.y_dtype != b.y_dtype || !a.Xe || !a.We || !b.Xe || !b.We || a.swiglu ||
+        b.swiglu)
+        return cudaErrorInvalidValue;
+    if (a.L == 0) return cudaSuccess;
+    switch (a.y_dtype) {
+        case STARQ_F16: return launch_tma_grouped<__half>(a, b, stream);
+        case STARQ_BF16: return launch_tma_grouped<__nv_bfloat16>(a, b, stream);
+        case STARQ_F32: return launch_tma_grouped<float>(a, b, stream);
+        default: return cudaErrorInvalidValue;
+    }
 }
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& a, cudaStream_t stream) {

@@ -71,6 +71,21 @@ class SgatLinear:
                         self.Wq, self.s_w, Y, self.workspace, bias=self.bias, tac_M=self.tac_M,
                         tac_d=self.tac_d, tac_g=self.tac_g, We=self.We, tac_Mp=self.tac_Mp, stream=stream)
 
+    def quantize(self, X, mask, stream=None):
+        """TAC (when the layer has it) and the state-guided quantisation of X
+        into the layer's own code buffers (Xq, s_a, Xe), without the GEMM:
+        for a grouped launch of several layers' GEMMs."""
+        if not hasattr(self, "Xq"):
+            dev = self.s_w.device
+            self.Xq = torch.empty(self.L, self.K // 2, dtype=torch.uint8, device=dev)
+            self.s_a = torch.empty(self.L, dtype=torch.float32, device=dev)
+            self.Xe = torch.empty(self.L, self.K, dtype=torch.uint8, device=dev)
+            self.tac_scratch = (torch.empty(self.L, self.K, dtype=self.dtype, device=dev)
+                                if self.tac is not None else None)
+        abi.sgat_quantize_act(X, mask, self.a_m, self.a_u, self.hb, self.d_sh, self.d_m, self.d_u, self.Xq,
+                              self.s_a, Xe=self.Xe, stream=stream, tac_M=self.tac_M, tac_d=self.tac_d,
+                              tac_g=self.tac_g, tac_Mp=self.tac_Mp, tac_scratch=self.tac_scratch)
+
     def int_ops(self, L=None):
         return 2 * (L or self.L) * self.N * self.K
 
@@ -85,7 +100,7 @@ class AttentionProjections:
     the hardware placed first (against a steady 71-73 us uncapped), so it
     is off by default. Results do not depend on it."""
 
-    def __init__(self, qkv_case, o_case, device="cuda", e4m3_weights=True, qkv_pair_limit=0):
+    def __init__(self, qkv_case, o_case, device="cuda", e4m3_weights=True, qkv_pair_limit=0, grouped=False):
         self.qkv = SgatLinear(qkv_case, device, e4m3_weights=e4m3_weights)
         self.o = SgatLinear(o_case, device, e4m3_weights=e4m3_weights)
         self.L = qkv_case.L
@@ -96,6 +111,8 @@ class AttentionProjections:
         self.Y_o = torch.empty(self.L, self.o.N, dtype=self.o.out_dtype, device=device)
         self.side = torch.cuda.Stream(device=device)
         self.qkv_pair_limit = qkv_pair_limit
+        self.grouped = grouped and e4m3_weights
+        self.KERNELS_PER_STEP = 4 if self.grouped else 5
         self.graph = None
 
     def step(self, stream=None):
@@ -104,8 +121,22 @@ class AttentionProjections:
         joined back at the end: its CUDA-core kernels overlap the QKV
         quantiser and the gaps between launches. The O chain is issued
         first, so that TAC starts beside the QKV quantiser. Outputs are
-        identical to running the two projections one after the other."""
+        identical to running the two projections one after the other.
+
+        grouped: the O chain's TAC and quantiser run on the side stream
+        beside the QKV quantiser, and both GEMMs then go out as one
+        launch (w4a4_gemm_grouped), the O tiles after the QKV tiles."""
         main = stream if stream is not None else torch.cuda.current_stream()
+        if self.grouped:
+            self.side.wait_stream(main)
+            with torch.cuda.stream(self.side):
+                self.o.quantize(self.Z, self.mask, self.side)
+            self.qkv.quantize(self.X, self.mask, main)
+            main.wait_stream(self.side)
+            q, o = self.qkv, self.o
+            abi.w4a4_gemm_grouped(q.Xe, q.s_a, q.We, q.s_w, self.Y_qkv, o.Xe, o.s_a, o.We, o.s_w, self.Y_o,
+                                  bias0=q.bias, bias1=o.bias, stream=main)
+            return
         self.side.wait_stream(main)
         with torch.cuda.stream(self.side):
             self.o.run(self.Z, self.mask, self.Y_o, self.side)
@@ -135,4 +166,4 @@ class AttentionProjections:
     def int_ops(self):
         return self.qkv.int_ops() + self.o.int_ops()
 
-    KERNELS_PER_STEP = 5   # quant + GEMM (QKV); TAC + quant + GEMM (O)
+    KERNELS_PER_STEP = 5   # quant + GEMM (QKV); TAC + quant + GEMM (O); 4 when grouped (one GEMM launch)

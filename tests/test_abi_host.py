@@ -117,6 +117,31 @@ def test_gemm_null_and_alignment(lib):
     assert W4(lib, P, None, P, P, None, P, None, 4, 256, 512, P, 7, None, None) == -1
 
 
+def G2(lib, Xe0=P, We0=P, N0=256, Y0=P, Xe1=P, We1=P, N1=128, L=4, K=512, dt=0, acc0=None):
+    """w4a4_gemm_grouped with valid placeholders except where overridden
+    (validation returns before any device access)."""
+    return lib.lib.w4a4_gemm_grouped(Xe0, P, We0, P, None, N0, Y0, Xe1, P, We1, P, None, N1, P, L, K, dt, acc0,
+                                     None, None)
+
+
+@pytest.mark.parametrize("N0,N1,K,L,code", [(100, 256, 512, 4, -2), (256, 31, 512, 4, -2), (256, 256, 200, 4, -2),
+                                            (256, 256, 131072, 4, -2), (256, 256, 512, -1, -2)])
+def test_gemm_grouped_validation(lib, N0, N1, K, L, code):
+    assert G2(lib, N0=N0, N1=N1, K=K, L=L) == code
+
+
+def test_gemm_grouped_null_and_alignment(lib):
+    assert G2(lib, We0=None) == -1
+    assert G2(lib, We1=None) == -1
+    assert G2(lib, Xe1=None) == -1
+    assert G2(lib, Xe0=ctypes.c_void_p(4104)) == -3
+    assert G2(lib, We1=ctypes.c_void_p(4104)) == -3
+    assert G2(lib, Y0=ctypes.c_void_p(4104)) == -3
+    assert G2(lib, acc0=ctypes.c_void_p(4100)) == -3
+    assert G2(lib, dt=7) == -1
+    assert G2(lib, L=0, Xe0=None, Xe1=None) == 0
+
+
 @pytest.mark.parametrize("N,K,code", [(-1, 512, -2), (4, 48, -2), (4, 16, -2)])
 def test_unpack_validation(lib, N, K, code):
     assert lib.lib.w4_unpack_e4m3(P, N, K, P, None) == code

@@ -220,6 +220,49 @@ def test_w4a4_gemm_tile_widths(abi, out):
     assert seen == {224, 256}, seen
 
 
+@pytest.mark.parametrize("L,N0,N1,K,out", [(300, 768, 288, 512, "f16"), (1, 256, 32, 128, "bf16"),
+                                            (513, 160, 4096, 256, "f32"), (257, 4096, 12288, 128, "f16")])
+def test_w4a4_gemm_grouped(abi, L, N0, N1, K, out):
+    """Two products in one launch (problem 1's tiles follow problem 0's):
+    the exact integer sums of both against the oracle, outputs within the
+    dequantisation bound, and each bit-identical to a w4a4_gemm call of its
+    own. Ragged L, widths that are not multiples of the pair tile, a bias
+    on one problem only, and more tiles than CTA pairs (257 x 16384)."""
+    qa0, qw0, s_a0, s_w0 = H.gemm_codes(L + N0 + K, L, N0, K)
+    qa1, qw1, s_a1, s_w1 = H.gemm_codes(L + N1 + 2 * K + 1, L, N1, K)
+    bias1 = np.random.default_rng(L + 5).normal(0, 0.1, N1).astype(np.float32)
+    Xe0, Xe1 = H.dev(H.e4m3_bytes(qa0)), H.dev(H.e4m3_bytes(qa1))
+    We0, We1 = H.dev(H.e4m3_bytes(qw0)), H.dev(H.e4m3_bytes(qw1))
+    sa0, sa1, sw0, sw1, b1 = H.dev(s_a0), H.dev(s_a1), H.dev(s_w0), H.dev(s_w1), H.dev(bias1)
+    td = H.torch_dtype(out)
+    Y0 = torch.empty(L, N0, dtype=td, device="cuda")
+    Y1 = torch.empty(L, N1, dtype=td, device="cuda")
+    acc0 = torch.empty(L, N0, dtype=torch.int32, device="cuda")
+    acc1 = torch.empty(L, N1, dtype=torch.int32, device="cuda")
+    abi.w4a4_gemm_grouped(Xe0, sa0, We0, sw0, Y0, Xe1, sa1, We1, sw1, Y1, bias1=b1, acc_dbg0=acc0, acc_dbg1=acc1)
+    abi.check_status()
+    ref0, ref1 = osg.int_gemm(qa0, qw0), osg.int_gemm(qa1, qw1)
+    assert np.array_equal(acc0.cpu().numpy(), ref0), "integer accumulators differ (problem 0)"
+    assert np.array_equal(acc1.cpu().numpy(), ref1), "integer accumulators differ (problem 1)"
+    if out == "f32":
+        # float32 output: Eq. 3's float32 steps, each rounded (a bias can
+        # cancel most of the product, so a float64 reference with a relative
+        # bound would not fit): bit for bit
+        def deq32(acc, sa, sw, b):
+            y = (acc.astype(np.float32) * sa.astype(np.float32)[:, None]) * sw.astype(np.float32)[None, :]
+            return y if b is None else y + b.astype(np.float32)[None, :]
+        assert np.array_equal(H.host(Y0), deq32(ref0, s_a0, s_w0, None)), "outputs differ (problem 0)"
+        assert np.array_equal(H.host(Y1), deq32(ref1, s_a1, s_w1, bias1)), "outputs differ (problem 1)"
+    else:
+        H.assert_output_close(H.host(Y0), osg.dequant(ref0, s_a0, s_w0, None), out)
+        H.assert_output_close(H.host(Y1), osg.dequant(ref1, s_a1, s_w1, bias1), out)
+    Z0, Z1 = torch.empty_like(Y0), torch.empty_like(Y1)
+    abi.w4a4_gemm(None, sa0, None, sw0, Z0, Xe=Xe0, We=We0)
+    abi.w4a4_gemm(None, sa1, None, sw1, Z1, bias=b1, Xe=Xe1, We=We1)
+    abi.check_status()
+    assert torch.equal(Z0, Y0) and torch.equal(Z1, Y1), "grouped launch differs from single launches"
+
+
 @pytest.mark.parametrize("M,N,K,dt", [(1, 32, 64, "f16"), (129, 288, 640, "f16"), (300, 512, 1024, "bf16"), (4608, 1024, 128, "bf16"),
                                       (1024, 4096, 4096, "f16"), (77, 768, 4096, "bf16")])
 def test_fp16_gemm_ref(abi, M, N, K, dt):

@@ -1,9 +1,11 @@
-"""The LLaDA attention-projection step as the bench runs it: the QKV
-projection on the calling stream and TAC + O projection on a side stream,
-forked and joined inside one CUDA graph. Its outputs must equal those of the
-two projections run one after the other on one stream (which the parity
-tests check against the oracle), eagerly and on graph replay, and the
-step's buffers must not be touched by a replay of the other branch.
+"""The LLaDA attention-projection step as the bench runs it, in both of its
+forms: forked (the QKV projection on the calling stream, TAC + O projection
+on a side stream, joined inside one CUDA graph) and grouped (the two
+quantisations on two streams, then both GEMMs in one w4a4_gemm_grouped
+launch). Its outputs must equal those of the two projections run one after
+the other on one stream (which the parity tests check against the oracle),
+eagerly and on graph replay, and the step's buffers must not be touched by a
+replay of the other branch.
 """
 
 import pytest
@@ -14,10 +16,12 @@ from paper_2606_04945_gb300 import inputs
 pytestmark = pytest.mark.gpu
 
 
-def test_forked_step_equals_sequential(abi):
+@pytest.mark.parametrize("grouped", [False, True])
+def test_step_equals_sequential(abi, grouped):
     from paper_2606_04945_gb300.pipeline import AttentionProjections
     qkv_case, o_case = inputs.llada_attention(seed=3)
-    st = AttentionProjections(qkv_case, o_case)
+    st = AttentionProjections(qkv_case, o_case, grouped=grouped)
+    assert st.KERNELS_PER_STEP == (4 if grouped else 5)
     st.qkv.run(st.X, st.mask, st.Y_qkv)
     st.o.run(st.Z, st.mask, st.Y_o)
     torch.cuda.synchronize()
