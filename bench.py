@@ -52,9 +52,11 @@ def parse():
     p.add_argument("--ref-sample-tokens", type=int, default=128)
     p.add_argument("--skip-cpu-baseline", action="store_true")
     p.add_argument("--skip-stack", action="store_true", help="leave out the short denoising-stack run")
-    p.add_argument("--forked-step", action="store_true",
-                   help="attention_step: run the two projections as forked branches with a GEMM launch each "
-                        "(the default groups both GEMMs into one launch)")
+    p.add_argument("--step-form", default="grouped", choices=["grouped", "grouped-gemm", "forked"],
+                   help="attention_step: grouped (default): TAC, then both quantisations in one launch, then "
+                        "both GEMMs in one launch; grouped-gemm: the two quantisation chains on two streams, "
+                        "then one GEMM launch; forked: the two projections as forked branches with a GEMM "
+                        "launch each")
     p.add_argument("--workload", default="attention_step",
                    choices=["attention_step", "denoise_stack", "tac_calibration", "attention_pv_tac", "w8a8_linear",
                             "asym_linear", "dense_linear", "dream_block", "hbm_passes", "llada_mlp",
@@ -86,13 +88,16 @@ def load_peaks():
 
 
 def config_dict(graph, grouped=True):
+    forms = {True: "TAC on Z, then the QKV and O quantisations in one launch (the QKV rows start during TAC), "
+                   "then both GEMMs in one grouped launch",
+             "gemm": "the QKV quantiser beside TAC + the O quantiser (two streams), then both GEMMs in one "
+                     "grouped launch",
+             False: "QKV and TAC + O branches forked and joined within the step"}
     return {"workload": "llada8b_attention_projections_step", "tokens": 1024, "hidden": 4096,
             "qkv": "4096->12288", "o": "4096->4096", "tac_block": 128, "hadamard_block": 4096,
             "gates": "d_m = d_u = 128", "mask": "0..639 unmasked, 640..1023 masked",
             "l2": "flushed between timed steps (256 MiB write)", "cuda_graph": bool(graph),
-            "streams": ("the QKV quantiser beside TAC + the O quantiser (two streams), then both GEMMs in one "
-                        "grouped launch" if grouped else
-                        "QKV and TAC + O branches forked and joined within the step")}
+            "streams": forms[grouped]}
 
 
 # ---------------------------------------------------------------------------
@@ -619,7 +624,7 @@ def run_ours(args):
     from paper_2606_04945_gb300.pipeline import AttentionProjections
 
     qkv_case, o_case = inputs.llada_attention(seed=rank_seed(rank))
-    grouped = not args.forked_step
+    grouped = {"grouped": True, "grouped-gemm": "gemm", "forked": False}[args.step_form]
     step = AttentionProjections(qkv_case, o_case, grouped=grouped)
     L, K = step.L, step.qkv.K
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
@@ -685,6 +690,13 @@ def run_ours(args):
                               for i in range(8)], flush, torch, rounds=3)
     t_gemm_grp = time_kernel(lambda: abi.w4a4_gemm_grouped(Xe, s_a, q.We, q.s_w, step.Y_qkv, Xe, s_a, o.We, o.s_w,
                                                            step.Y_o), flush, reps, torch)
+    # both quantisations in one launch, as the default step runs them
+    Xq2, s_a2, Xe2 = torch.empty_like(Xq), torch.empty_like(s_a), torch.empty_like(Xe)
+    qio = lambda lin, X, xq, sa, xe: dict(X=X, mask=step.mask, a_m=lin.a_m, a_u=lin.a_u, d_sh=lin.d_sh,
+                                          d_m=lin.d_m, d_u=lin.d_u, Xq=xq, s_a=sa, Xe=xe)
+    s_quant_grp = time_stream([lambda i=i: abi.sgat_quantize_act_grouped(qio(q, Xr[i], Xq, s_a, Xe),
+                                                                         qio(o, Zf[i], Xq2, s_a2, Xe2), q.hb)
+                               for i in range(R)], flush, torch)
     abi.check_status()
     del Xr, Zr, Zf, Wr_q, Wr_o, Xer
     large = hbm_passes_large(abi, o, flush, torch)
@@ -866,6 +878,12 @@ def run_ours(args):
             "sgat_quantize_act_tac_out": {"ms": round(s_quant_z, 5), "launch_ms": round(t_quant_z, 5), "bytes": quant_z_bytes,
                                       "gbs": round(quant_z_bytes / s_quant_z / 1e6, 1),
                                       "frac": round(quant_z_bytes / s_quant_z / 1e6 / hbm, 4)},
+            "sgat_quantize_act_grouped_f16": {"ms": round(s_quant_grp, 5), "bytes": quant_x_bytes + quant_z_bytes,
+                                              "gbs": round((quant_x_bytes + quant_z_bytes) / s_quant_grp / 1e6, 1),
+                                              "frac": round((quant_x_bytes + quant_z_bytes) / s_quant_grp / 1e6 / hbm,
+                                                            4),
+                                              "note": "the X and TAC-output quantisations in one launch (2 x 1024 "
+                                                      "rows), as the default step runs them"},
         },
         "tensor_probes": probes,
         "denoise_step": denoise,

@@ -196,6 +196,35 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
                       void* stream);
 
 /*
+ * sgat_quantize_act_grouped -- two independent state-guided quantisations
+ * of sgat_quantize_act's definition (Sec. 3.2 Eq. 7-11 and Eq. 2) in one
+ * launch, e.g. the QKV projection's input and the O projection's
+ * TAC-compensated input of one step. p0 and p1 each name an input X
+ * [L][K] of x_dtype, its mask, smoothing vectors, gate layout and outputs
+ * (Xq, s_a and optionally Xe), with the meanings of sgat_quantize_act; K,
+ * hb, L, x_dtype and bits are shared. The results are bit-identical to two
+ * sgat_quantize_act calls (no TAC option: apply tac_apply first). Symmetric
+ * codes with K <= 4096 run as one kernel with one CTA per row of either
+ * problem; other shapes run as two launches. Errors as sgat_quantize_act.
+ */
+typedef struct {
+    const void* X;
+    const uint8_t* mask;
+    const float* a_m;
+    const float* a_u;
+    int d_sh, d_m, d_u;
+    uint8_t* Xq;
+    float* s_a;
+    uint8_t* Xe;
+    int independent;   /* 1: the caller guarantees that the launch just before this
+                          call on the stream neither writes X, mask, a_m, a_u nor reads
+                          or writes Xq, s_a, Xe; this problem's rows may then start
+                          while that launch finishes (programmatic launch). 0: wait. */
+} starq_quant_io;
+int sgat_quantize_act_grouped(const starq_quant_io* p0, const starq_quant_io* p1, int x_dtype, int L, int K,
+                              int hb, int bits, void* stream);
+
+/*
  * sgat_prepare_weight -- the unified static weight transform, quantised once
  * (Sec. 3.2 Eq. 12; App. B W_f = Q_w(P^T W^T)), per-output-channel symmetric.
  *
@@ -385,13 +414,18 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
  *   s_a0, s_a1 [L], s_w0 [N0], s_w1 [N1] float32; bias0, bias1 or NULL.
  *   Y0 [L][N0], Y1 [L][N1] of y_dtype (F16, BF16 or F32), 16-byte aligned.
  *   acc_dbg0, acc_dbg1: the exact int32 accumulators, or NULL.
+ *   flags: 0, or STARQ_GEMM_WEIGHTS_READY: the caller guarantees that the
+ *      launch just before this call on the stream does not write We0 or
+ *      We1, so the first weight tiles are fetched while it finishes
+ *      (programmatic launch); other bits are an error (STARQ_ERR_ARG).
  * Shapes and errors as w4a4_gemm for each problem (N0, N1 >= 32 and
  * multiples of 32; 128 <= K <= 65536, K % 128 == 0); L == 0 does nothing.
  */
+#define STARQ_GEMM_WEIGHTS_READY 1
 int w4a4_gemm_grouped(const uint8_t* Xe0, const float* s_a0, const uint8_t* We0, const float* s_w0,
                       const float* bias0, int N0, void* Y0, const uint8_t* Xe1, const float* s_a1,
                       const uint8_t* We1, const float* s_w1, const float* bias1, int N1, void* Y1, int L, int K,
-                      int y_dtype, int32_t* acc_dbg0, int32_t* acc_dbg1, void* stream);
+                      int y_dtype, int32_t* acc_dbg0, int32_t* acc_dbg1, int flags, void* stream);
 
 /*
  * starq_set_gemm_pair_limit -- at most `pairs` CTA pairs (two SMs each) for

@@ -27,8 +27,16 @@ EXPORTED = (
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
     "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
     "starq_selftest_wait_timeout", "starq_probe_mma", "attention_pv_tac_gqa", "glue_add_rmsnorm", "glue_rope",
-    "w4a4_gemm_mma_sync", "starq_set_gemm_pair_limit", "w4a4_gemm_grouped",
+    "w4a4_gemm_mma_sync", "starq_set_gemm_pair_limit", "w4a4_gemm_grouped", "sgat_quantize_act_grouped",
 )
+
+
+class StarqQuantIo(ctypes.Structure):
+    """starq_quant_io: one problem of sgat_quantize_act_grouped."""
+    _fields_ = [("X", ctypes.c_void_p), ("mask", ctypes.c_void_p), ("a_m", ctypes.c_void_p),
+                ("a_u", ctypes.c_void_p), ("d_sh", ctypes.c_int), ("d_m", ctypes.c_int), ("d_u", ctypes.c_int),
+                ("Xq", ctypes.c_void_p), ("s_a", ctypes.c_void_p), ("Xe", ctypes.c_void_p),
+                ("independent", ctypes.c_int)]
 
 
 class StarqTac(ctypes.Structure):
@@ -76,8 +84,9 @@ def _load():
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp, vp]
     lib.w8_split_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm_mma_sync.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
+    lib.sgat_quantize_act_grouped.argtypes = [vp, vp, i, i, i, i, i, vp]
     lib.w4a4_gemm_grouped.argtypes = [u8p, f_p, u8p, f_p, f_p, i, vp, u8p, f_p, u8p, f_p, f_p, i, vp, i, i, i, vp,
-                                      vp, vp]
+                                      vp, i, vp]
     lib.starq_set_gemm_pair_limit.argtypes = [i]
     lib.starq_set_gemm_pair_limit.restype = i
     lib.w8a8_gemm.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
@@ -187,6 +196,25 @@ def sgat_quantize_act(X, mask, a_m, a_u, hb, d_sh, d_m, d_u, Xq, s_a, bits=4, Xe
     _check(lib.sgat_quantize_act(_p(X), dtype_code(X), L, K, _p(mask), _p(a_m), _p(a_u), hb,
                                  d_sh, d_m, d_u, _ref(tac), bits, _p(Xq), _p(s_a), _p(Xe), _p(v_dbg),
                                  _stream(stream)))
+
+
+def sgat_quantize_act_grouped(p0, p1, hb, bits=4, stream=None):
+    """Two quantisations in one launch. p0, p1: dicts with X [L][K], mask,
+    a_m, a_u, d_sh, d_m, d_u, Xq, s_a and optionally Xe (the meanings of
+    sgat_quantize_act) and independent (see starq_quant_io); the two X share
+    shape and dtype."""
+    X0, X1 = p0["X"], p1["X"]
+    if tuple(X0.shape) != tuple(X1.shape) or X0.dtype != X1.dtype:
+        raise StarqError(-2, "sgat_quantize_act_grouped: the inputs need the same shape and dtype")
+    ios = []
+    for p in (p0, p1):
+        _contig(p["X"], p.get("mask"), p.get("a_m"), p.get("a_u"), p["Xq"], p["s_a"], p.get("Xe"))
+        ios.append(StarqQuantIo(_p(p["X"]), _p(p.get("mask")), _p(p.get("a_m")), _p(p.get("a_u")), p["d_sh"],
+                                p["d_m"], p["d_u"], _p(p["Xq"]), _p(p["s_a"]), _p(p.get("Xe")),
+                                int(bool(p.get("independent", False)))))
+    L, K = X0.shape
+    _check(lib.sgat_quantize_act_grouped(ctypes.byref(ios[0]), ctypes.byref(ios[1]), dtype_code(X0), L, K, hb,
+                                         bits, _stream(stream)))
 
 
 def sgat_prepare_weight(W, inv_a_w, hb, Wq, s_w, bits=4, stream=None):
@@ -314,18 +342,23 @@ def w4a4_gemm(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, Xe=None, We=None, st
                          dtype_code(Y), _ref(tac), _p(acc_dbg), _stream(stream)))
 
 
+GEMM_WEIGHTS_READY = 1
+
+
 def w4a4_gemm_grouped(Xe0, s_a0, We0, s_w0, Y0, Xe1, s_a1, We1, s_w1, Y1, bias0=None, bias1=None,
-                      acc_dbg0=None, acc_dbg1=None, stream=None):
+                      acc_dbg0=None, acc_dbg1=None, weights_ready=False, stream=None):
     """Two independent W4A4 products (same L, K and output type) in one
     launch: Y0 from Xe0 [L][K] and We0 [N0][K], Y1 from Xe1 and We1 (E4M3
-    codes)."""
+    codes). weights_ready: the launch just before this one does not write
+    We0 or We1 (their first tiles are fetched while it finishes)."""
     _contig(Xe0, s_a0, We0, s_w0, Y0, bias0, acc_dbg0, Xe1, s_a1, We1, s_w1, Y1, bias1, acc_dbg1)
     L, K = Xe0.shape
     if tuple(Xe1.shape) != (L, K) or Y0.dtype != Y1.dtype:
         raise StarqError(-2, "w4a4_gemm_grouped: the problems need the same L, K and output type")
     _check(lib.w4a4_gemm_grouped(_p(Xe0), _p(s_a0), _p(We0), _p(s_w0), _p(bias0), We0.shape[0], _p(Y0),
                                  _p(Xe1), _p(s_a1), _p(We1), _p(s_w1), _p(bias1), We1.shape[0], _p(Y1), L, K,
-                                 dtype_code(Y0), _p(acc_dbg0), _p(acc_dbg1), _stream(stream)))
+                                 dtype_code(Y0), _p(acc_dbg0), _p(acc_dbg1),
+                                 GEMM_WEIGHTS_READY if weights_ready else 0, _stream(stream)))
 
 
 def w4a4_gemm_mma_sync(Xq, s_a, Wq, s_w, Y, bias=None, acc_dbg=None, stream=None):

@@ -342,6 +342,32 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
     return STARQ_OK;
 }
 
+int sgat_quantize_act_grouped(const starq_quant_io* p0, const starq_quant_io* p1, int x_dtype, int L, int K,
+                              int hb, int bits, void* stream) {
+    if (!p0 || !p1) return fail(STARQ_ERR_ARG, "sgat_quantize_act_grouped: NULL problem");
+    if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act_grouped: unknown dtype %d", x_dtype);
+    if (bits != 4 && bits != 8) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4- and 8-bit codes", bits);
+    if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
+    for (const starq_quant_io* p : {p0, p1}) {
+        if (L > 0 && (!p->X || !p->Xq || !p->s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act_grouped: NULL X, Xq or s_a");
+        int rc = check_transform(K, hb, p->d_sh, p->d_m, p->d_u, p->a_m, p->a_u);
+        if (rc) return rc;
+        if (L > 0 && (!aligned(p->X, 16) || !aligned(p->Xq, 8) || (p->Xe && !aligned(p->Xe, 16))))
+            return fail(STARQ_ERR_ALIGN, "sgat_quantize_act_grouped: X (16 B), Xq (8 B), Xe (16 B) alignment");
+    }
+    if (L == 0) return STARQ_OK;
+    const int qmax = bits == 8 ? 127 : 7;
+    QuantArgs a{p0->X, x_dtype, L, K, p0->mask, p0->a_m, p0->a_u, hb, p0->d_sh, p0->d_m, p0->d_u, qmax, 1.f,
+                p0->Xq, p0->s_a, nullptr, p0->Xe};
+    QuantArgs b{p1->X, x_dtype, L, K, p1->mask, p1->a_m, p1->a_u, hb, p1->d_sh, p1->d_m, p1->d_u, qmax, 1.f,
+                p1->Xq, p1->s_a, nullptr, p1->Xe};
+    a.independent = p0->independent != 0;
+    b.independent = p1->independent != 0;
+    const cudaError_t e = launch_sgat_quant_grouped(a, b, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "sgat_quantize_act_grouped launch");
+    return STARQ_OK;
+}
+
 int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* inv_a_w, int hb,
                         int bits, uint8_t* Wq, float* s_w, void* stream) {
     if (N > 0 && (!W || !Wq || !s_w)) return fail(STARQ_ERR_ARG, "sgat_prepare_weight: NULL W, Wq or s_w");
@@ -397,8 +423,9 @@ int w4a4_gemm(const uint8_t* Xq, const uint8_t* Xe, const float* s_a, const uint
 int w4a4_gemm_grouped(const uint8_t* Xe0, const float* s_a0, const uint8_t* We0, const float* s_w0,
                       const float* bias0, int N0, void* Y0, const uint8_t* Xe1, const float* s_a1,
                       const uint8_t* We1, const float* s_w1, const float* bias1, int N1, void* Y1, int L, int K,
-                      int y_dtype, int32_t* acc_dbg0, int32_t* acc_dbg1, void* stream) {
+                      int y_dtype, int32_t* acc_dbg0, int32_t* acc_dbg1, int flags, void* stream) {
     if (!We0 || !We1) return fail(STARQ_ERR_ARG, "w4a4_gemm_grouped: NULL We0 or We1");
+    if (flags & ~STARQ_GEMM_WEIGHTS_READY) return fail(STARQ_ERR_ARG, "w4a4_gemm_grouped: unknown flags %d", flags);
     if (L > 0 && (!Xe0 || !Xe1)) return fail(STARQ_ERR_ARG, "w4a4_gemm_grouped: NULL Xe0 or Xe1");
     int rc = check_gemm(nullptr, Xe0, s_a0, nullptr, We0, s_w0, bias0, L, N0, K, Y0, y_dtype);
     if (rc) return rc;
@@ -412,6 +439,7 @@ int w4a4_gemm_grouped(const uint8_t* Xe0, const float* s_a0, const uint8_t* We0,
     if (!st) return rc;
     GemmArgs a{nullptr, s_a0, nullptr, s_w0, bias0, L, N0, K, Y0, y_dtype, acc_dbg0, st, Xe0, We0};
     GemmArgs b{nullptr, s_a1, nullptr, s_w1, bias1, L, N1, K, Y1, y_dtype, acc_dbg1, st, Xe1, We1};
+    a.weights_ready = b.weights_ready = (flags & STARQ_GEMM_WEIGHTS_READY) ? 1 : 0;
     cudaError_t e = launch_w4a4_gemm_grouped(a, b, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "w4a4_gemm_grouped launch");
     return STARQ_OK;

@@ -45,8 +45,17 @@ struct QuantArgs {
     // E4M3 of -z (the zero-point columns of the augmented contraction)
     int asym = 0;
     int32_t* z = nullptr;
+    // the caller guarantees that the launch just before this one on the
+    // stream neither writes X, mask, a_m, a_u nor reads or writes the
+    // outputs, so the rows may start before it completes (programmatic
+    // launch; everything earlier has completed by then)
+    int independent = 0;
 };
 cudaError_t launch_sgat_quant(const QuantArgs& a, cudaStream_t stream);
+// Two quantisations in one launch when both run the row kernel with one CTA
+// per row (the same input type, K <= 4096, hb and code width, symmetric);
+// otherwise two launches.
+cudaError_t launch_sgat_quant_grouped(const QuantArgs& a, const QuantArgs& b, cudaStream_t stream);
 
 struct GemmArgs {
     const uint8_t* Xq; const float* s_a; const uint8_t* Wq; const float* s_w;

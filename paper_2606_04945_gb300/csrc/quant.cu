@@ -523,19 +523,28 @@ __device__ __forceinline__ float ld_shared_cluster_f32(uint32_t cluster_addr) {
 // of CL CTAs per row, CTA r taking the row's features 4096 r .. 4096 r +
 // 4095; the CTAs exchange their maxima through distributed shared memory,
 // so no thread holds more than one 4096-feature slice.
-template <int NR, typename Tin, bool ASYM, int CL = 1>
+// G2: rows a0.L .. a0.L + b.L - 1 of the grid quantise problem b (the same
+// K, hb, input type and code width; its own X, mask, transform and outputs):
+// two quantisations in one launch.
+template <int NR, typename Tin, bool ASYM, int CL = 1, bool G2 = false>
 __global__ void __launch_bounds__(128, NR == 1 ? 7 : 1)
-sgat_quant_rows_kernel(QuantArgs a) {
+sgat_quant_rows_kernel(QuantArgs a0, QuantArgs b) {
     static_assert(CL == 1 || NR == 1, "one slice per CTA of a cluster");
+    static_assert(!G2 || CL == 1, "grouped launches run one CTA per row");
+    const bool p1 = G2 && (int)blockIdx.x >= a0.L;
+    const QuantArgs& a = p1 ? b : a0;
     __shared__ __align__(16) float buf[4 * SLICE];
     __shared__ float red[8];              // [0, 4) amax or X_max, [4, 8) -X_min (asym)
     __shared__ float cl_red[2];           // this CTA's maximum (and -minimum) for its cluster
-    grid_dependency_wait();            // launched with programmatic serialisation
+    // launched with programmatic serialisation: the rows of a problem whose
+    // caller vouches that the preceding launch neither writes its inputs
+    // nor touches its outputs start without waiting for that launch
+    if (!a.independent) grid_dependency_wait();
     grid_launch_dependents();
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int rank = CL > 1 ? (int)cluster_ctarank() : 0;
-    const int row = CL > 1 ? (int)blockIdx.x / CL : (int)blockIdx.x;
+    const int row = CL > 1 ? (int)blockIdx.x / CL : (int)blockIdx.x - (p1 ? a0.L : 0);
     const int K = a.K;
     const bool masked = a.mask != nullptr && a.mask[row] != 0;
     const float* sm = masked ? a.a_m : a.a_u;
@@ -787,8 +796,8 @@ cudaError_t launch_rows_nr(const QuantArgs& a, cudaStream_t stream) {
     cfg.stream = stream;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    return a.asym ? cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, true>, a)
-                  : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, false>, a);
+    return a.asym ? cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, true>, a, a)
+                  : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<NR, Tin, false>, a, a);
 }
 
 // Rows longer than 4096: a cluster of CL CTAs per row, one 4096-feature
@@ -807,8 +816,22 @@ cudaError_t launch_rows_cl(const QuantArgs& a, cudaStream_t stream) {
     cfg.stream = stream;
     cfg.attrs = at;
     cfg.numAttrs = 2;
-    return a.asym ? cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<1, Tin, true, CL>, a)
-                  : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<1, Tin, false, CL>, a);
+    return a.asym ? cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<1, Tin, true, CL>, a, a)
+                  : cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<1, Tin, false, CL>, a, a);
+}
+
+// Two symmetric quantisations of rows up to 4096 features in one launch
+// (one CTA per row of either problem).
+template <typename Tin>
+cudaError_t launch_rows_grouped(const QuantArgs& a, const QuantArgs& b, cudaStream_t stream) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1] = {pdl_attribute()};
+    cfg.gridDim = dim3((unsigned)(a.L + b.L));
+    cfg.blockDim = dim3(128);
+    cfg.stream = stream;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, sgat_quant_rows_kernel<1, Tin, false, 1, true>, a, b);
 }
 
 template <typename Tin>
@@ -883,6 +906,27 @@ cudaError_t launch_sgat_quant(const QuantArgs& a, cudaStream_t stream) {
         case STARQ_F16: return launch_typed<__half>(a, stream);
         case STARQ_BF16: return launch_typed<__nv_bfloat16>(a, stream);
         case STARQ_F32: return launch_typed<float>(a, stream);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+// Whether the row kernel with one CTA per row takes this problem.
+static bool rows_one_cta(const QuantArgs& a) {
+    return !a.asym && a.K <= 4096 &&
+           ((a.hb >= 1024 && a.K % 1024 == 0) || (a.hb <= 512 && a.K >= 1024 && a.K % 512 == 0));
+}
+
+cudaError_t launch_sgat_quant_grouped(const QuantArgs& a, const QuantArgs& b, cudaStream_t stream) {
+    const bool same = a.x_dtype == b.x_dtype && a.K == b.K && a.hb == b.hb && a.qmax == b.qmax &&
+                      a.post_scale == b.post_scale && rows_one_cta(a) && rows_one_cta(b);
+    if (!same || a.L == 0 || b.L == 0) {             // two launches
+        cudaError_t e = launch_sgat_quant(a, stream);
+        return e != cudaSuccess ? e : launch_sgat_quant(b, stream);
+    }
+    switch (a.x_dtype) {
+        case STARQ_F16: return launch_rows_grouped<__half>(a, b, stream);
+        case STARQ_BF16: return launch_rows_grouped<__nv_bfloat16>(a, b, stream);
+        case STARQ_F32: return launch_rows_grouped<float>(a, b, stream);
         default: return cudaErrorInvalidValue;
     }
 }

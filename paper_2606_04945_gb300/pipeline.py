@@ -71,10 +71,9 @@ class SgatLinear:
                         self.Wq, self.s_w, Y, self.workspace, bias=self.bias, tac_M=self.tac_M,
                         tac_d=self.tac_d, tac_g=self.tac_g, We=self.We, tac_Mp=self.tac_Mp, stream=stream)
 
-    def quantize(self, X, mask, stream=None):
-        """TAC (when the layer has it) and the state-guided quantisation of X
-        into the layer's own code buffers (Xq, s_a, Xe), without the GEMM:
-        for a grouped launch of several layers' GEMMs."""
+    def buffers(self):
+        """The layer's own code buffers (Xq, s_a, Xe) and TAC scratch, for
+        launches that group several layers' quantisations or GEMMs."""
         if not hasattr(self, "Xq"):
             dev = self.s_w.device
             self.Xq = torch.empty(self.L, self.K // 2, dtype=torch.uint8, device=dev)
@@ -82,6 +81,12 @@ class SgatLinear:
             self.Xe = torch.empty(self.L, self.K, dtype=torch.uint8, device=dev)
             self.tac_scratch = (torch.empty(self.L, self.K, dtype=self.dtype, device=dev)
                                 if self.tac is not None else None)
+
+    def quantize(self, X, mask, stream=None):
+        """TAC (when the layer has it) and the state-guided quantisation of X
+        into the layer's own code buffers (Xq, s_a, Xe), without the GEMM:
+        for a grouped launch of several layers' GEMMs."""
+        self.buffers()
         abi.sgat_quantize_act(X, mask, self.a_m, self.a_u, self.hb, self.d_sh, self.d_m, self.d_u, self.Xq,
                               self.s_a, Xe=self.Xe, stream=stream, tac_M=self.tac_M, tac_d=self.tac_d,
                               tac_g=self.tac_g, tac_Mp=self.tac_Mp, tac_scratch=self.tac_scratch)
@@ -111,8 +116,8 @@ class AttentionProjections:
         self.Y_o = torch.empty(self.L, self.o.N, dtype=self.o.out_dtype, device=device)
         self.side = torch.cuda.Stream(device=device)
         self.qkv_pair_limit = qkv_pair_limit
-        self.grouped = grouped and e4m3_weights
-        self.KERNELS_PER_STEP = 4 if self.grouped else 5
+        self.grouped = grouped if e4m3_weights else False
+        self.KERNELS_PER_STEP = 3 if self.grouped is True else 4 if self.grouped else 5
         self.graph = None
 
     def step(self, stream=None):
@@ -123,10 +128,25 @@ class AttentionProjections:
         first, so that TAC starts beside the QKV quantiser. Outputs are
         identical to running the two projections one after the other.
 
-        grouped: the O chain's TAC and quantiser run on the side stream
-        beside the QKV quantiser, and both GEMMs then go out as one
-        launch (w4a4_gemm_grouped), the O tiles after the QKV tiles."""
+        grouped=True: TAC on Z, then both quantisations in one launch
+        (sgat_quantize_act_grouped) and both GEMMs in one launch
+        (w4a4_gemm_grouped, the O tiles after the QKV tiles): three kernels
+        on one stream. grouped="gemm": the O chain's TAC and quantiser run
+        on the side stream beside the QKV quantiser, then the grouped GEMM."""
         main = stream if stream is not None else torch.cuda.current_stream()
+        if self.grouped is True:
+            q, o = self.qkv, self.o
+            for lin in (q, o):
+                lin.buffers()
+            abi.tac_apply(self.Z, o.tac_M, o.tac_d, o.tac_g, o.tac_scratch, Mp=o.tac_Mp, stream=main)
+            io = lambda lin, X: dict(X=X, mask=self.mask, a_m=lin.a_m, a_u=lin.a_u, d_sh=lin.d_sh, d_m=lin.d_m,
+                                     d_u=lin.d_u, Xq=lin.Xq, s_a=lin.s_a, Xe=lin.Xe)
+            # the QKV rows do not depend on the TAC launch just before them
+            abi.sgat_quantize_act_grouped(dict(io(q, self.X), independent=True), io(o, o.tac_scratch), q.hb,
+                                          stream=main)
+            abi.w4a4_gemm_grouped(q.Xe, q.s_a, q.We, q.s_w, self.Y_qkv, o.Xe, o.s_a, o.We, o.s_w, self.Y_o,
+                                  bias0=q.bias, bias1=o.bias, weights_ready=True, stream=main)
+            return
         if self.grouped:
             self.side.wait_stream(main)
             with torch.cuda.stream(self.side):

@@ -117,11 +117,35 @@ def test_gemm_null_and_alignment(lib):
     assert W4(lib, P, None, P, P, None, P, None, 4, 256, 512, P, 7, None, None) == -1
 
 
-def G2(lib, Xe0=P, We0=P, N0=256, Y0=P, Xe1=P, We1=P, N1=128, L=4, K=512, dt=0, acc0=None):
+def Q2(lib, X0=P, Xq1=P, d_m=0, hb=512, bits=4, L=4, K=512, dt=0, none=None):
+    """sgat_quantize_act_grouped with valid placeholder problems except
+    where overridden (validation returns before any device access)."""
+    io = lambda X, Xq: lib.StarqQuantIo(X, None, None, None, K, d_m, 0, Xq, P, None)
+    p0, p1 = io(X0, P), io(P, Xq1)
+    args = [ctypes.byref(p0), ctypes.byref(p1)]
+    if none is not None:
+        args[none] = None
+    return lib.lib.sgat_quantize_act_grouped(*args, dt, L, K, hb, bits, None)
+
+
+def test_quantize_grouped_validation(lib):
+    assert Q2(lib, none=0) == -1
+    assert Q2(lib, none=1) == -1
+    assert Q2(lib, Xq1=None) == -1
+    assert Q2(lib, dt=7) == -1
+    assert Q2(lib, bits=6) == -4
+    assert Q2(lib, hb=3) == -2
+    assert Q2(lib, d_m=5) == -2                       # d_sh + d_m + d_u != K
+    assert Q2(lib, L=-1) == -2
+    assert Q2(lib, X0=ctypes.c_void_p(4104)) == -3
+    assert Q2(lib, L=0, X0=None, Xq1=None) == 0
+
+
+def G2(lib, Xe0=P, We0=P, N0=256, Y0=P, Xe1=P, We1=P, N1=128, L=4, K=512, dt=0, acc0=None, flags=0):
     """w4a4_gemm_grouped with valid placeholders except where overridden
     (validation returns before any device access)."""
     return lib.lib.w4a4_gemm_grouped(Xe0, P, We0, P, None, N0, Y0, Xe1, P, We1, P, None, N1, P, L, K, dt, acc0,
-                                     None, None)
+                                     None, flags, None)
 
 
 @pytest.mark.parametrize("N0,N1,K,L,code", [(100, 256, 512, 4, -2), (256, 31, 512, 4, -2), (256, 256, 200, 4, -2),
@@ -139,7 +163,9 @@ def test_gemm_grouped_null_and_alignment(lib):
     assert G2(lib, Y0=ctypes.c_void_p(4104)) == -3
     assert G2(lib, acc0=ctypes.c_void_p(4100)) == -3
     assert G2(lib, dt=7) == -1
+    assert G2(lib, flags=2) == -1
     assert G2(lib, L=0, Xe0=None, Xe1=None) == 0
+    assert G2(lib, L=0, Xe0=None, Xe1=None, flags=1) == 0
 
 
 @pytest.mark.parametrize("N,K,code", [(-1, 512, -2), (4, 48, -2), (4, 16, -2)])

@@ -73,6 +73,40 @@ def test_quantize_act_bitexact(abi, L, K, hb, dtype, gates):
     assert np.array_equal(s_a.cpu().numpy(), s), "scales differ"
 
 
+@pytest.mark.parametrize("L,K,hb,dtype", [(300, 4096, 4096, "f16"), (77, 1024, 512, "bf16"), (5, 2048, 2048, "f32"),
+                                           (1, 3584, 512, "bf16"), (9, 12288, 4096, "f16"), (4, 256, 16, "f16")])
+def test_quantize_act_grouped(abi, L, K, hb, dtype):
+    """Two quantisations in one launch (each problem with its own input,
+    mask, smoothing vectors and gate layout): both against the oracle (codes
+    and scales bit for bit), and bit-identical to two single calls. The
+    last two shapes (rows beyond 4096 features, blocks of 16) fall back to
+    two launches."""
+    cases = [inputs.random_linear(L + K + hb + 11 * t, L, K, 128, dtype=dtype, gates_on=(t == 0), hb=hb)
+             for t in range(2)]
+    td = H.torch_dtype(dtype)
+    ios, outs = [], []
+    for c in cases:
+        xf = c.xf
+        io = dict(X=H.dev(c.X, td), mask=H.dev(c.mask), a_m=H.dev(xf.a_m), a_u=H.dev(xf.a_u), d_sh=xf.d_sh,
+                  d_m=xf.d_m, d_u=xf.d_u, Xq=torch.empty(L, K // 2, dtype=torch.uint8, device="cuda"),
+                  s_a=torch.empty(L, dtype=torch.float32, device="cuda"),
+                  Xe=torch.empty(L, K, dtype=torch.uint8, device="cuda"))
+        ios.append(io)
+    abi.sgat_quantize_act_grouped(ios[0], ios[1], hb)
+    abi.check_status()
+    for c, io in zip(cases, ios):
+        xf = c.xf
+        codes, sc = osg.sgat_quantize_act(c.X, c.mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, 4)
+        assert np.array_equal(H.unpack(io["Xq"]), codes), "int4 codes differ"
+        assert np.array_equal(io["s_a"].cpu().numpy(), sc), "scales differ"
+        assert np.array_equal(io["Xe"].cpu().numpy(), H.e4m3_bytes(codes)), "E4M3 codes differ"
+        Xq1, s1, Xe1 = torch.empty_like(io["Xq"]), torch.empty_like(io["s_a"]), torch.empty_like(io["Xe"])
+        abi.sgat_quantize_act(io["X"], io["mask"], io["a_m"], io["a_u"], hb, io["d_sh"], io["d_m"], io["d_u"], Xq1,
+                              s1, Xe=Xe1)
+        abi.check_status()
+        assert torch.equal(Xq1, io["Xq"]) and torch.equal(s1, io["s_a"]) and torch.equal(Xe1, io["Xe"])
+
+
 @pytest.mark.parametrize("K,hb", [(4096, 4096), (2048, 1024), (1024, 512), (256, 16)])
 def test_quantize_act_exact_ties(abi, K, hb):
     """Transformed values that sit exactly on a rounding tie (x.5 after the
@@ -239,7 +273,8 @@ def test_w4a4_gemm_grouped(abi, L, N0, N1, K, out):
     Y1 = torch.empty(L, N1, dtype=td, device="cuda")
     acc0 = torch.empty(L, N0, dtype=torch.int32, device="cuda")
     acc1 = torch.empty(L, N1, dtype=torch.int32, device="cuda")
-    abi.w4a4_gemm_grouped(Xe0, sa0, We0, sw0, Y0, Xe1, sa1, We1, sw1, Y1, bias1=b1, acc_dbg0=acc0, acc_dbg1=acc1)
+    abi.w4a4_gemm_grouped(Xe0, sa0, We0, sw0, Y0, Xe1, sa1, We1, sw1, Y1, bias1=b1, acc_dbg0=acc0, acc_dbg1=acc1,
+                          weights_ready=(L == 300))
     abi.check_status()
     ref0, ref1 = osg.int_gemm(qa0, qw0), osg.int_gemm(qa1, qw1)
     assert np.array_equal(acc0.cpu().numpy(), ref0), "integer accumulators differ (problem 0)"

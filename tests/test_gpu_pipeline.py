@@ -16,12 +16,12 @@ from paper_2606_04945_gb300 import inputs
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("grouped", [False, True])
+@pytest.mark.parametrize("grouped", [False, "gemm", True])
 def test_step_equals_sequential(abi, grouped):
     from paper_2606_04945_gb300.pipeline import AttentionProjections
     qkv_case, o_case = inputs.llada_attention(seed=3)
     st = AttentionProjections(qkv_case, o_case, grouped=grouped)
-    assert st.KERNELS_PER_STEP == (4 if grouped else 5)
+    assert st.KERNELS_PER_STEP == {False: 5, "gemm": 4, True: 3}[grouped]
     st.qkv.run(st.X, st.mask, st.Y_qkv)
     st.o.run(st.Z, st.mask, st.Y_o)
     torch.cuda.synchronize()
