@@ -120,6 +120,26 @@ constexpr float ROUND_BIAS = 12608512.f;
 
 // 2^x by the PTX approximation (relative error about 2^-22; subnormal
 // results flush to zero, where the code is 0 anyway)
+// Two independent IEEE float32 operations on a register pair (the f32x2
+// forms): each lane rounds exactly as the scalar fma / add would, with half
+// the issue slots.
+__device__ __forceinline__ float2 fma2_rn(float2 a, float2 b, float2 c) {
+    float2 d;
+    asm("{\n\t.reg .b64 A, B, C, D;\n\t"
+        "mov.b64 A, {%2, %3};\n\tmov.b64 B, {%4, %5};\n\tmov.b64 C, {%6, %7};\n\t"
+        "fma.rn.f32x2 D, A, B, C;\n\tmov.b64 {%0, %1}, D;\n\t}"
+        : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+__device__ __forceinline__ float2 add2_rn(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 A, B, D;\n\t"
+        "mov.b64 A, {%2, %3};\n\tmov.b64 B, {%4, %5};\n\t"
+        "add.rn.f32x2 D, A, B;\n\tmov.b64 {%0, %1}, D;\n\t}"
+        : "=f"(d.x), "=f"(d.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
 __device__ __forceinline__ float ex2_approx(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -576,7 +596,9 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
             mx = fmaxf(fmaxf(sh->xm[0][row], sh->xm[1][row]), fmaxf(sh->xm[2][row], sh->xm[3][row]));
             named_sync_softmax();
             // pass 2: probabilities, their codes and the row sums
-            float lp[4] = {0.f, 0.f, 0.f, 0.f};      // partial row sums (independent chains)
+            // partial row sums, four independent chains held as two pairs:
+            // (l0, l2) and (l1, l3), l0 + l1 over even-k scores, l2 + l3 odd
+            float2 lpa = make_float2(0.f, 0.f), lpb = make_float2(0.f, 0.f);
             // the exponent as one fma: s c - m c differs from (s - m) c by an
             // ulp of m c at most, ~1e-6 in e at |m| <= 100 (the codes' rounding
             // decisions move only within 3e-4 of a half-integer)
@@ -594,15 +616,16 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
                 // exactly in fp16
                 uint32_t packed[16];
                 const __half2 minus1024 = __float2half2_rn(-1024.f);
+                const float2 c2 = make_float2(EXP_SCALE, EXP_SCALE), nm2 = make_float2(-mxc, -mxc);
+                const float2 q2 = make_float2(255.f, 255.f), bias2 = make_float2(ROUND_BIAS, ROUND_BIAS);
                 #pragma unroll
                 for (int k = 0; k < 32; k += 2) {
-                    const float e0 = ex2_approx(__fmaf_rn(__uint_as_float(r[k]), EXP_SCALE, -mxc));
-                    const float e1 = ex2_approx(__fmaf_rn(__uint_as_float(r[k + 1]), EXP_SCALE, -mxc));
-                    lp[(k >> 1) & 1] += e0;
-                    lp[2 + ((k >> 1) & 1)] += e1;
-                    const uint32_t t0 = __float_as_uint(fmaf(255.f, e0, ROUND_BIAS));
-                    const uint32_t t1 = __float_as_uint(fmaf(255.f, e1, ROUND_BIAS));
-                    const uint32_t biased = prmt(t0, t1, 0x5410u);           // {1024 + n0, 1024 + n1}
+                    const float2 t = fma2_rn(make_float2(__uint_as_float(r[k]), __uint_as_float(r[k + 1])), c2, nm2);
+                    const float2 e = make_float2(ex2_approx(t.x), ex2_approx(t.y));
+                    if ((k >> 1) & 1) lpb = add2_rn(lpb, e);
+                    else lpa = add2_rn(lpa, e);
+                    const float2 u = fma2_rn(e, q2, bias2);
+                    const uint32_t biased = prmt(__float_as_uint(u.x), __float_as_uint(u.y), 0x5410u);   // {1024 + n0, 1024 + n1}
                     const __half2 hc = __hadd2(*reinterpret_cast<const __half2*>(&biased), minus1024);
                     packed[k / 2] = *reinterpret_cast<const uint32_t*>(&hc);
                 }
@@ -621,7 +644,7 @@ attn_pv_tac_kernel(AttnArgs a, const __grid_constant__ CUtensorMap tm_q, const _
                 __syncwarp();
                 if (lane == 0) mbar_arrive(B(sh->s_empty[b]));
             }
-            sh->xm[part][row] = (lp[0] + lp[1]) + (lp[2] + lp[3]);
+            sh->xm[part][row] = (lpa.x + lpb.x) + (lpa.y + lpb.y);
             named_sync_softmax();
             const float l = (sh->xm[0][row] + sh->xm[1][row]) + (sh->xm[2][row] + sh->xm[3][row]);
             const float sp = __fdiv_rn(1.f, __fmul_rn(255.f, l));
