@@ -171,7 +171,8 @@ int starq_probe_mma(int kind, int iters, unsigned long long* cycles, int* errors
  *   bits    4, or 8 for the W8A8 setting (Tab. 5): the same quantiser with
  *           127 in place of 7.
  *   Xq      codes out, 8-byte aligned: bits 4: [L][K/2] packed int4 (low
- *           nibble = even k); bits 8: [L][K] int8.
+ *           nibble = even k); bits 8: [L][K] int8. May be NULL when Xe is
+ *           given (then only the GEMM operand form is written).
  *   s_a     [L] float32 per-token scales out (0 for an all-zero row).
  *   Xe      the GEMM operand out, 16-byte aligned, or NULL. bits 4: [L][K]
  *           the codes as E4M3 bytes (the form w4a4_gemm streams by TMA).
@@ -628,12 +629,13 @@ int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, 
  *   workspace: device buffer of at least sgat_linear_workspace_size(L, K,
  *   tac_M != NULL) bytes (bits 4) or sgat_linear_workspace_size_bits(L, K,
  *   tac_M != NULL, bits), 256-byte aligned, owned by the caller. On return
- *   it holds the intermediates, laid out as [codes Xq: L*K/2 bytes (bits 4)
- *   or L*K (bits 8), padded to 256][s_a: 4*L bytes, padded to 256][GEMM
- *   operand Xe: L*K bytes (bits 4) or 2*L*K (bits 8), padded to 256][TAC
- *   output: L*K values of x_dtype (room for float32), only with TAC]. The
- *   TAC output is rounded to x_dtype once, as the unquantised model stores
- *   attention outputs, and the quantiser reads it.
+ *   it holds the intermediates, laid out as [a region of L*K/2 bytes (bits
+ *   4) or L*K (bits 8), padded to 256, left unwritten: the GEMM reads the
+ *   codes in their operand form only][s_a: 4*L bytes, padded to 256][GEMM
+ *   operand Xe, the codes: L*K E4M3 bytes (bits 4) or 2*L*K (bits 8),
+ *   padded to 256][TAC output: L*K values of x_dtype (room for float32),
+ *   only with TAC]. The TAC output is rounded to x_dtype once, as the
+ *   unquantised model stores attention outputs, and the quantiser reads it.
  *   bits 8 (the W8A8 setting): Wq may be NULL; We is the w8_split_e4m3
  *   output and the GEMM is w8a8_gemm's; N % 128 == 0.
  *

@@ -315,7 +315,7 @@ int sgat_quantize_act(const void* X, int x_dtype, int L, int K, const uint8_t* m
                       const float* a_m, const float* a_u, int hb, int d_sh, int d_m, int d_u,
                       const starq_tac* tac, int bits, uint8_t* Xq, float* s_a, uint8_t* Xe, float* v_dbg,
                       void* stream) {
-    if (L > 0 && (!X || !Xq || !s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, Xq or s_a");
+    if (L > 0 && (!X || (!Xq && !Xe) || !s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: NULL X, s_a, or both Xq and Xe");
     if (!dtype_ok(x_dtype)) return fail(STARQ_ERR_ARG, "sgat_quantize_act: unknown dtype %d", x_dtype);
     if (bits != 4 && bits != 8) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4- and 8-bit codes", bits);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
@@ -349,7 +349,8 @@ int sgat_quantize_act_grouped(const starq_quant_io* p0, const starq_quant_io* p1
     if (bits != 4 && bits != 8) return fail(STARQ_ERR_BITS, "bits=%d: the GPU path implements 4- and 8-bit codes", bits);
     if (L < 0) return fail(STARQ_ERR_SHAPE, "L=%d < 0", L);
     for (const starq_quant_io* p : {p0, p1}) {
-        if (L > 0 && (!p->X || !p->Xq || !p->s_a)) return fail(STARQ_ERR_ARG, "sgat_quantize_act_grouped: NULL X, Xq or s_a");
+        if (L > 0 && (!p->X || (!p->Xq && !p->Xe) || !p->s_a))
+            return fail(STARQ_ERR_ARG, "sgat_quantize_act_grouped: NULL X, s_a, or both Xq and Xe");
         int rc = check_transform(K, hb, p->d_sh, p->d_m, p->d_u, p->a_m, p->a_u);
         if (rc) return rc;
         if (L > 0 && (!aligned(p->X, 16) || !aligned(p->Xq, 8) || (p->Xe && !aligned(p->Xe, 16))))
@@ -637,9 +638,9 @@ int sgat_linear_dense(const void* X, int x_dtype, int L, int K, const uint8_t* m
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = dense_transform(X, x_dtype, L, K, mask, a_m, a_u, Pt, Xs, V, st, s);
     if (e != cudaSuccess) return cuda_fail(e, "sgat_linear_dense: transform launch");
-    QuantArgs q{V, STARQ_F16, L, K, mask, nullptr, nullptr, 1, d_sh, d_m, d_u, 7, 1.f, Xq, s_a, nullptr, Xe};
+    QuantArgs q{V, STARQ_F16, L, K, mask, nullptr, nullptr, 1, d_sh, d_m, d_u, 7, 1.f, nullptr, s_a, nullptr, Xe};
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear_dense: quant launch");
-    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
+    GemmArgs g{nullptr, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};   // Xe: no packed codes read
     g.weights_ready = 1;
     if ((e = launch_w4a4_gemm(g, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear_dense: gemm launch");
     return STARQ_OK;
@@ -860,14 +861,15 @@ int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* ma
         qin = zt;
         qin_dtype = x_dtype;
     }
-    QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits == 8 ? 127 : 7, 1.f, Xq, s_a, nullptr, Xe};
+    // every GEMM path below reads the E4M3 form, so the packed codes are not written
+    QuantArgs q{qin, qin_dtype, L, K, mask, a_m, a_u, hb, d_sh, d_m, d_u, bits == 8 ? 127 : 7, 1.f, nullptr, s_a, nullptr, Xe};
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");
     if (bits == 8) {
         GemmArgs g8{nullptr, s_a, nullptr, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
         if ((e = launch_w8a8_gemm(g8, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: w8a8 gemm launch");
         return STARQ_OK;
     }
-    GemmArgs g{Xq, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
+    GemmArgs g{nullptr, s_a, Wq, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};   // Xe: no packed codes read
     // the GEMM's predecessor is the quantiser launched above, which waits for
     // everything before it and does not write the weights
     g.weights_ready = 1;

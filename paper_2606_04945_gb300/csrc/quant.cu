@@ -356,7 +356,7 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
                 #pragma unroll
                 for (int k = 0; k < 8; ++k)
                     q[k] = min(max(__float2int_rn(__fmul_rn(v[j][8 * u + k], r)) + zp, 0), a.qmax);
-                *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + lo / 2 + 4 * u) = pack8(q);
+                if (a.Xq != nullptr) *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + lo / 2 + 4 * u) = pack8(q);
                 if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * (K + 128) + lo + 8 * u) = e4m3_of8(q);
             }
             continue;
@@ -369,7 +369,7 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
                 for (int k = 0; k < 8; ++k) q[k] = __float2int_rn(__fmul_rn(v[j][8 * u + k], r));
                 uint2 bytes, eh, el;
                 split_codes8(q, bytes, eh, el);
-                *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + lo + 8 * u) = bytes;
+                if (a.Xq != nullptr) *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + lo + 8 * u) = bytes;
                 if (a.Xe != nullptr) {
                     *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + lo + 8 * u) = eh;
                     *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + lo + 8 * u) = el;
@@ -386,7 +386,8 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
             packed[u] = pack8(q);
         }
         uint8_t* dst = a.Xq + (size_t)row * (K / 2) + lo / 2;
-        if (E == 16) {
+        if (a.Xq == nullptr) {
+        } else if (E == 16) {
             *reinterpret_cast<uint2*>(dst) = make_uint2(packed[0], packed[1]);
         } else {
             #pragma unroll
@@ -496,20 +497,21 @@ __device__ __forceinline__ void quant_pair(float v0, float v1, float r, float& q
     i1 -= 0x4B400000;
 }
 
-// Eight codes -> packed nibbles (code k in bits 4k .. 4k + 3) and their
-// eight E4M3 bytes (byte k = code k); qf are the codes as floats, qi as ints.
-__device__ __forceinline__ void pack_codes8(const float* qf, const int* qi, uint32_t& nib, uint2& e4) {
+// Eight codes (ints) -> packed nibbles, code k in bits 4k .. 4k + 3.
+__device__ __forceinline__ uint32_t pack_nibbles8(const int* qi) {
     uint32_t w = 0;
     #pragma unroll
     for (int k = 6; k >= 0; k -= 2)      // d = c << 8 | sat4(a) << 4 | sat4(b)
         asm("cvt.pack.sat.s4.s32.b32 %0, %1, %2, %0;" : "+r"(w) : "r"(qi[k + 1]), "r"(qi[k]));
-    nib = w;
+    return w;
+}
+// Eight codes (floats) -> their eight E4M3 bytes (byte k = code k).
+__device__ __forceinline__ uint2 e4m3_bytes8(const float* qf) {
     uint16_t h[4];
     #pragma unroll
     for (int k = 0; k < 4; ++k)          // upper byte from the first operand
         asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(h[k]) : "f"(qf[2 * k + 1]), "f"(qf[2 * k]));
-    e4.x = (uint32_t)h[0] | ((uint32_t)h[1] << 16);
-    e4.y = (uint32_t)h[2] | ((uint32_t)h[3] << 16);
+    return make_uint2((uint32_t)h[0] | ((uint32_t)h[1] << 16), (uint32_t)h[2] | ((uint32_t)h[3] << 16));
 }
 
 __device__ __forceinline__ float ld_shared_cluster_f32(uint32_t cluster_addr) {
@@ -763,25 +765,23 @@ sgat_quant_rows_kernel(QuantArgs a0, QuantArgs b) {
                 int q[8];
                 #pragma unroll
                 for (int k = 0; k < 8; ++k) q[k] = min(max(qi[k] + zp, 0), a.qmax);
-                *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = pack8(q);
+                if (a.Xq != nullptr) *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = pack8(q);
                 if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * (K + 128) + e0) = e4m3_of8(q);
                 continue;
             }
             if (a.qmax > 15) {           // 8-bit codes: bytes and their E4M3 split
                 uint2 bytes, eh, el;
                 split_codes8(qi, bytes, eh, el);
-                *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + e0) = bytes;
+                if (a.Xq != nullptr) *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + e0) = bytes;
                 if (a.Xe != nullptr) {
                     *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + e0) = eh;
                     *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + e0) = el;
                 }
                 continue;
             }
-            uint32_t nib;
-            uint2 e4;
-            pack_codes8(qf, qi, nib, e4);
-            *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = nib;
-            if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * K + e0) = e4;
+            if (a.Xq != nullptr)
+                *reinterpret_cast<uint32_t*>(a.Xq + (size_t)row * (K / 2) + e0 / 2) = pack_nibbles8(qi);
+            if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * K + e0) = e4m3_bytes8(qf);
         }
     }
     if (CL > 1) cluster_sync();        // no CTA leaves while its maximum may still be read

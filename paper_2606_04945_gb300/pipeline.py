@@ -72,11 +72,11 @@ class SgatLinear:
                         tac_d=self.tac_d, tac_g=self.tac_g, We=self.We, tac_Mp=self.tac_Mp, stream=stream)
 
     def buffers(self):
-        """The layer's own code buffers (Xq, s_a, Xe) and TAC scratch, for
+        """The layer's own code buffers (s_a and the E4M3 codes Xe; the packed
+        codes are not needed, as the GEMM reads Xe) and TAC scratch, for
         launches that group several layers' quantisations or GEMMs."""
-        if not hasattr(self, "Xq"):
+        if not hasattr(self, "Xe"):
             dev = self.s_w.device
-            self.Xq = torch.empty(self.L, self.K // 2, dtype=torch.uint8, device=dev)
             self.s_a = torch.empty(self.L, dtype=torch.float32, device=dev)
             self.Xe = torch.empty(self.L, self.K, dtype=torch.uint8, device=dev)
             self.tac_scratch = (torch.empty(self.L, self.K, dtype=self.dtype, device=dev)
@@ -87,7 +87,7 @@ class SgatLinear:
         into the layer's own code buffers (Xq, s_a, Xe), without the GEMM:
         for a grouped launch of several layers' GEMMs."""
         self.buffers()
-        abi.sgat_quantize_act(X, mask, self.a_m, self.a_u, self.hb, self.d_sh, self.d_m, self.d_u, self.Xq,
+        abi.sgat_quantize_act(X, mask, self.a_m, self.a_u, self.hb, self.d_sh, self.d_m, self.d_u, None,
                               self.s_a, Xe=self.Xe, stream=stream, tac_M=self.tac_M, tac_d=self.tac_d,
                               tac_g=self.tac_g, tac_Mp=self.tac_Mp, tac_scratch=self.tac_scratch)
 
@@ -140,7 +140,7 @@ class AttentionProjections:
                 lin.buffers()
             abi.tac_apply(self.Z, o.tac_M, o.tac_d, o.tac_g, o.tac_scratch, Mp=o.tac_Mp, stream=main)
             io = lambda lin, X: dict(X=X, mask=self.mask, a_m=lin.a_m, a_u=lin.a_u, d_sh=lin.d_sh, d_m=lin.d_m,
-                                     d_u=lin.d_u, Xq=lin.Xq, s_a=lin.s_a, Xe=lin.Xe)
+                                     d_u=lin.d_u, Xq=None, s_a=lin.s_a, Xe=lin.Xe)
             # the QKV rows do not depend on the TAC launch just before them
             abi.sgat_quantize_act_grouped(dict(io(q, self.X), independent=True), io(o, o.tac_scratch), q.hb,
                                           stream=main)

@@ -95,9 +95,9 @@ def gemm_codes(seed, L, N, K, lo=-7, hi=7):
 
 def workspace_views(ws, L, K, with_tac, x_dtype=torch.float32):
     """Views of the intermediates sgat_linear leaves in its workspace
-    (packed codes, per-token scales, E4M3 codes, the TAC output in the input's
-    type x_dtype), following the layout documented for sgat_linear in
-    include/starq.h."""
+    (the packed-code region, which it leaves unwritten, per-token scales,
+    E4M3 codes, the TAC output in the input's type x_dtype), following the
+    layout documented for sgat_linear in include/starq.h."""
     a256 = lambda x: (x + 255) // 256 * 256
     o1 = a256(L * K // 2)
     o2 = o1 + a256(4 * L)
@@ -108,6 +108,18 @@ def workspace_views(ws, L, K, with_tac, x_dtype=torch.float32):
     esz = torch.empty(0, dtype=x_dtype).element_size()
     zt = ws[o3: o3 + esz * L * K].view(x_dtype).view(L, K) if with_tac else None
     return Xq, s_a, Xe, zt
+
+
+def codes_from_e4m3(b):
+    """Integer codes in [-8, 8] back from their E4M3 bytes (the inverse of
+    e4m3_bytes on its range); any other byte fails the check."""
+    b = np.asarray(b.cpu().numpy() if hasattr(b, "cpu") else b, dtype=np.uint8)
+    lut = np.full(256, 127, dtype=np.int32)
+    q = np.arange(-8, 9)
+    lut[e4m3_bytes(q)] = q
+    out = lut[b]
+    assert np.all(out != 127), "bytes that are not the E4M3 of a code in [-8, 8]"
+    return out
 
 
 def e4m3_bytes(q):

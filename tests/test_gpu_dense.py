@@ -113,8 +113,9 @@ def test_sgat_linear_dense(abi, L, K, N, dtype):
                           xf.d_u, Wq, s_w, Y, ws, bias=H.dev(case.bias), We=We)
     abi.check_status()
     a256 = lambda x: (x + 255) // 256 * 256
-    o = 2 * a256(2 * L * K)
-    codes = H.unpack(ws[o: o + L * K // 2].view(L, K // 2))
+    o = 2 * a256(2 * L * K)                       # then [packed-code region, unwritten][s_a][Xe]
+    o_e = o + a256(L * K // 2) + a256(4 * L)
+    codes = H.codes_from_e4m3(ws[o_e: o_e + L * K].view(L, K))
     s_a = ws[o + a256(L * K // 2): o + a256(L * K // 2) + 4 * L].view(torch.float32).cpu().numpy()
     qw, sw = H.unpack(Wq), s_w.cpu().numpy()
     ref = osg.dequant(osg.int_gemm(codes, qw), s_a, sw, case.bias)
@@ -160,8 +161,9 @@ def test_sgat_linear_dense_calibrated_basis(abi):
                               Wq, s_w, Y, ws, We=We)
         abi.check_status()
         a256 = lambda x: (x + 255) // 256 * 256
-        o = 2 * a256(2 * L * K)
-        codes = H.unpack(ws[o: o + L * K // 2].view(L, K // 2))
+        o = 2 * a256(2 * L * K)                   # then [packed-code region, unwritten][s_a][Xe]
+        o_e = o + a256(L * K // 2) + a256(4 * L)
+        codes = H.codes_from_e4m3(ws[o_e: o_e + L * K].view(L, K))
         s_a = ws[o + a256(L * K // 2): o + a256(L * K // 2) + 4 * L].view(torch.float32).cpu().numpy()
         v_gpu = ws[a256(2 * L * K): a256(2 * L * K) + 2 * L * K].view(torch.float16).view(L, K).float().cpu().numpy()
         q, s = osg.quantize_rows_sym(gated(v_gpu, mask, d_sh, d_m, d_u), 4)

@@ -36,7 +36,7 @@ def _check_linear(lin, X_rows, mask_rows, rows, Y_rows, L, what, swiglu=False, b
     xf = lin.xf
     Xq, s_a, Xe, _ = H.workspace_views(lin.workspace, L, lin.K, False)
     codes, s = osg.sgat_quantize_act(X_rows, mask_rows, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, 4)
-    assert np.array_equal(H.unpack(Xq)[rows], codes), f"{what}: activation codes"
+    assert np.array_equal(H.codes_from_e4m3(Xe)[rows], codes), f"{what}: activation codes"
     assert np.array_equal(s_a.cpu().numpy()[rows], s), f"{what}: activation scales"
     assert np.array_equal(Xe.cpu().numpy()[rows], H.e4m3_bytes(codes)), f"{what}: E4M3 codes"
     ref = osg.dequant(osg.int_gemm(codes, H.unpack(lin.Wq)), s, lin.s_w.cpu().numpy(), bias)

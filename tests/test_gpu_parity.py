@@ -73,6 +73,27 @@ def test_quantize_act_bitexact(abi, L, K, hb, dtype, gates):
     assert np.array_equal(s_a.cpu().numpy(), s), "scales differ"
 
 
+@pytest.mark.parametrize("L,K,hb,dtype,bits", [(129, 4096, 4096, "f16", 4), (33, 3584, 512, "bf16", 4),
+                                                (9, 256, 16, "f16", 4), (40, 2048, 2048, "f32", 8)])
+def test_quantize_act_without_packed_codes(abi, L, K, hb, dtype, bits):
+    """Xq = NULL with Xe given (the form sgat_linear and the grouped step
+    use): the operand bytes and scales equal those of a call that also
+    writes the packed codes (row kernel, warp-per-chunk kernel, 8-bit)."""
+    case = inputs.random_linear(L + K + hb + bits, L, K, 128, dtype=dtype, gates_on=True, hb=hb)
+    xf = case.xf
+    X, m = H.dev(case.X, H.torch_dtype(dtype)), H.dev(case.mask)
+    a_m, a_u = H.dev(xf.a_m), H.dev(xf.a_u)
+    qb = K // 2 if bits == 4 else K
+    eb = K if bits == 4 else 2 * K
+    Xq = torch.empty(L, qb, dtype=torch.uint8, device="cuda")
+    s1, s2 = (torch.empty(L, dtype=torch.float32, device="cuda") for _ in range(2))
+    Xe1, Xe2 = (torch.empty(L, eb, dtype=torch.uint8, device="cuda") for _ in range(2))
+    abi.sgat_quantize_act(X, m, a_m, a_u, hb, xf.d_sh, xf.d_m, xf.d_u, Xq, s1, bits=bits, Xe=Xe1)
+    abi.sgat_quantize_act(X, m, a_m, a_u, hb, xf.d_sh, xf.d_m, xf.d_u, None, s2, bits=bits, Xe=Xe2)
+    abi.check_status()
+    assert torch.equal(Xe1, Xe2) and torch.equal(s1, s2)
+
+
 @pytest.mark.parametrize("L,K,hb,dtype", [(300, 4096, 4096, "f16"), (77, 1024, 512, "bf16"), (5, 2048, 2048, "f32"),
                                            (1, 3584, 512, "bf16"), (9, 12288, 4096, "f16"), (4, 256, 16, "f16")])
 def test_quantize_act_grouped(abi, L, K, hb, dtype):
@@ -430,7 +451,7 @@ def run_linear_case(abi, case, out_dtype=None, check_rows=None, weights="e4m3"):
         X_in = z_gpu                      # teacher forcing on the GPU's TAC output
     Y_ref, codes, s_a, acc = osg.sgat_linear(X_in[rows], case.mask[rows], xf.a_m, xf.a_u, xf.hb, xf.d_sh,
                                              xf.d_m, xf.d_u, qw, sw, case.bias, 4)
-    assert np.array_equal(H.unpack(Xq_g)[rows], codes), "activation codes differ"
+    assert np.array_equal(H.codes_from_e4m3(Xe_g)[rows], codes), "activation codes differ"
     assert np.array_equal(Xe_g.cpu().numpy()[rows], H.e4m3_bytes(codes)), "E4M3 codes differ"
     assert np.array_equal(s_a_g.cpu().numpy()[rows], s_a), "activation scales differ"
     H.assert_output_close(H.host(Y)[rows], Y_ref, out_dtype)

@@ -87,7 +87,7 @@ def test_denoise_stack(abi):
         mask = state["mask"][rows]
         Xr = X.float().cpu().numpy()[rows]
         codes, s = osg.sgat_quantize_act(Xr, mask, xf.a_m, xf.a_u, xf.hb, xf.d_sh, xf.d_m, xf.d_u, 4)
-        g_codes = H.unpack(Xq)[rows]
+        g_codes = H.codes_from_e4m3(Xe)[rows]
         assert np.array_equal(g_codes, codes), f"step {step} layer {li} {name}: codes"
         assert np.array_equal(s_a.cpu().numpy()[rows], s), f"step {step} layer {li} {name}: scales"
         assert np.array_equal(Xe.cpu().numpy()[rows], H.e4m3_bytes(codes)), f"step {step} layer {li} {name}: E4M3"

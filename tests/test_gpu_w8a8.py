@@ -152,8 +152,11 @@ def test_sgat_linear_8bit(abi, L, K, N, hb, dtype, tac_g):
                     ws, bias=H.dev(case.bias), tac_M=tac_M, tac_d=tac_d, tac_g=tac_g or 0, bits=8, We=We)
     abi.check_status()
     a256 = lambda x: (x + 255) // 256 * 256
-    Xq = ws[: L * K].view(torch.int8).view(L, K).cpu().numpy().astype(np.int64)
+    # [code region, left unwritten][s_a][Xe: the E4M3 split h | l of each code, c = 16 h + l]
     s_a = ws[a256(L * K): a256(L * K) + 4 * L].view(torch.float32).cpu().numpy()
+    o_e = a256(L * K) + a256(4 * L)
+    Xe = ws[o_e: o_e + 2 * L * K].view(L, 2 * K)
+    Xq = 16 * H.codes_from_e4m3(Xe[:, :K]).astype(np.int64) + H.codes_from_e4m3(Xe[:, K:])
     if tac_g:
         o = a256(L * K) + a256(4 * L) + a256(2 * L * K)
         esz = torch.empty(0, dtype=dt).element_size()
