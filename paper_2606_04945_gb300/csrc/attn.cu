@@ -57,14 +57,14 @@
 // six 32 KB tiles streams each item's Q tile, pass-1 K chunks, pass-2 K and
 // V chunks, M's two halves and then the slot of its output boxes, in the
 // order they are used, running on into the next item.
-// TMEM (512 columns): two S / P buffers (pass 1 also uses the P V^T
-// accumulator's columns as a third), the P V^T accumulator and Q; the TAC
-// accumulator and Z_hat reuse the S buffers. The tensor pipe keeps almost
-// no queue of issued MMAs, so it runs dry whenever the issuing thread
-// waits, and a barrier query costs ~160-380 cycles even on a completed
-// phase: the MMA warp therefore waits once per pass-2 chunk, on all of the
-// chunk's barriers at once, and then issues its P V^T and the Q K^T two
-// chunks ahead back to back. Every wait is bounded.
+// TMEM (512 columns): two S / P buffers, the P V^T accumulator (then the
+// TAC accumulator), Q, and Z_hat's halves (see the column map below). The
+// tensor pipe keeps almost no queue of issued MMAs, so it runs dry
+// whenever the issuing thread is busy elsewhere (its waits and bookkeeping,
+// slowed by the softmax warps that share its scheduler): the MMA warp
+// therefore waits once per pass-2 chunk, on all of the chunk's barriers at
+// once, and then issues its P V^T and the Q K^T two chunks ahead back to
+// back. Every wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
