@@ -176,10 +176,8 @@ int starq_probe_mma(int kind, int iters, unsigned long long* cycles, int* errors
  *   s_a     [L] float32 per-token scales out (0 for an all-zero row).
  *   Xe      the GEMM operand out, 16-byte aligned, or NULL. bits 4: [L][K]
  *           the codes as E4M3 bytes (the form w4a4_gemm streams by TMA).
- *           bits 8: [L][2K], each code c split as c = 16 h + l with
- *           l = ((c + 8) mod 16) - 8 in [-8, 7] and h in [-8, 8]: the E4M3
- *           bytes of h in columns 0..K-1 and of l in columns K..2K-1 (the
- *           operand of w8a8_gemm).
+ *           bits 8: [L][K] the codes as fp16 numbers (exact for |c| <=
+ *           127; the operand of w8a8_gemm).
  *   v_dbg   [L][K] float32 transformed activations out (before rounding),
  *           16-byte aligned, or NULL.
  *   tac     NULL, or TAC on the input first (the attention output before
@@ -259,15 +257,14 @@ int sgat_prepare_weight(const void* W, int w_dtype, int N, int K, const float* i
 int w4_unpack_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
 
 /*
- * w8_split_e4m3 -- 8-bit weight codes in the form w8a8_gemm reads: each code
- * c of Wq [N][K] (int8) split as c = 16 h + l (l = ((c + 8) mod 16) - 8),
- * We [N][2K] = E4M3 bytes of h in columns 0..K-1 and of l in K..2K-1 (both
- * exact E4M3 numbers). Run once per weight after sgat_prepare_weight with
+ * w8_codes_f16 -- 8-bit weight codes in the form w8a8_gemm reads: each code
+ * c of Wq [N][K] (int8) as the fp16 number c (exact for |c| <= 127),
+ * We [N][K] fp16. Run once per weight after sgat_prepare_weight with
  * bits = 8.
  *   Wq, We 16-byte aligned; We caller-owned (2 N K bytes).
  * Shapes: N >= 0, K >= 128 with K % 128 == 0.
  */
-int w8_split_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
+int w8_codes_f16(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
 
 /*
  * w8a8_gemm -- the integer projection and its dequantisation at 8 bits (the
@@ -277,12 +274,13 @@ int w8_split_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream);
  *   Y[i][n]   = (float)acc * s_a[i] * s_w[n] (+ bias[n]) rounded to y_dtype
  *               (float32 products in that order, then one rounding).
  *
- *   Xe [L][2K] activation code halves (sgat_quantize_act, bits 8), We [N][2K]
- *      weight code halves (w8_split_e4m3), 16-byte aligned.
- *   acc = 256 (H_a H_w^T) + 16 (H_a L_w^T + L_a H_w^T) + L_a L_w^T: four FP8
- *   tensor-core products (tcgen05 kind::f8f6f4) into three float32
- *   accumulators, each an integer below 2^24 and so exact, combined in
- *   int32 by the epilogue.
+ *   Xe [L][K] activation codes as fp16 (sgat_quantize_act, bits 8), We [N][K]
+ *      weight codes as fp16 (w8_codes_f16), 16-byte aligned (2 K bytes a
+ *      row each).
+ *   One 16-bit tensor-core product (tcgen05 kind::f16, CTA pairs) on the
+ *   codes, accumulated in float32 in runs of 512 K (each run an integer of
+ *   magnitude at most 512 * 127^2 < 2^23, so exact); the epilogue adds the
+ *   runs in int32.
  *   s_a [L], s_w [N] float32; bias [N] float32 or NULL.
  *   Y  [L][N] out, y_dtype F16, BF16 or F32, 16-byte aligned.
  *   acc_dbg [L][N] int32 out (the exact accumulators) or NULL.
@@ -632,11 +630,11 @@ int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, 
  *   it holds the intermediates, laid out as [a region of L*K/2 bytes (bits
  *   4) or L*K (bits 8), padded to 256, left unwritten: the GEMM reads the
  *   codes in their operand form only][s_a: 4*L bytes, padded to 256][GEMM
- *   operand Xe, the codes: L*K E4M3 bytes (bits 4) or 2*L*K (bits 8),
+ *   operand Xe, the codes: L*K E4M3 bytes (bits 4) or L*K fp16 (bits 8),
  *   padded to 256][TAC output: L*K values of x_dtype (room for float32),
  *   only with TAC]. The TAC output is rounded to x_dtype once, as the
  *   unquantised model stores attention outputs, and the quantiser reads it.
- *   bits 8 (the W8A8 setting): Wq may be NULL; We is the w8_split_e4m3
+ *   bits 8 (the W8A8 setting): Wq may be NULL; We is the w8_codes_f16
  *   output and the GEMM is w8a8_gemm's; N % 128 == 0.
  *
  *   Programmatic launch: the kernels of sgat_linear may start while the

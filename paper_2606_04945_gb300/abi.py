@@ -22,7 +22,7 @@ EXPORTED = (
     "sgat_linear_workspace_size", "sgat_linear", "starq_last_gemm_tile",
     "tac_calibrate_workspace_size", "tac_calibrate", "sgat_linear_swiglu",
     "attention_pv_tac_workspace_size", "attention_pv_tac",
-    "w8_split_e4m3", "w8a8_gemm", "sgat_linear_workspace_size_bits",
+    "w8_codes_f16", "w8a8_gemm", "sgat_linear_workspace_size_bits",
     "sgat_quantize_act_asym", "w4_zero_point_columns", "sgat_linear_asym_workspace_size", "sgat_linear_asym",
     "sgat_dense_workspace_size", "sgat_quantize_act_dense", "sgat_prepare_weight_dense",
     "sgat_linear_dense_workspace_size", "sgat_linear_dense", "sgat_linear_noalloc",
@@ -82,7 +82,7 @@ def _load():
     lib.sgat_prepare_weight.argtypes = [vp, i, i, i, f_p, i, i, u8p, f_p, vp]
     lib.w4_unpack_e4m3.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm.argtypes = [u8p, u8p, f_p, u8p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp, vp]
-    lib.w8_split_e4m3.argtypes = [u8p, i, i, u8p, vp]
+    lib.w8_codes_f16.argtypes = [u8p, i, i, u8p, vp]
     lib.w4a4_gemm_mma_sync.argtypes = [u8p, f_p, u8p, f_p, f_p, i, i, i, vp, i, vp, vp]
     lib.sgat_quantize_act_grouped.argtypes = [vp, vp, i, i, i, i, i, vp]
     lib.w4a4_gemm_grouped.argtypes = [u8p, f_p, u8p, f_p, f_p, i, vp, u8p, f_p, u8p, f_p, f_p, i, vp, i, i, i, vp,
@@ -310,19 +310,21 @@ def sgat_linear_dense(X, mask, a_m, a_u, Pt, d_sh, d_m, d_u, Wq, s_w, Y, workspa
                                  workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
-def w8_split_e4m3(Wq, We, stream=None):
-    """8-bit weight codes [N][K] (int8) -> their E4M3 halves [N][2K] (once per weight)."""
+def w8_codes_f16(Wq, We, stream=None):
+    """8-bit weight codes [N][K] (int8) -> the same codes as fp16 [N][K]
+    (We: 2K bytes a row, any dtype; once per weight)."""
     _contig(Wq, We)
     N, K = Wq.shape
-    _check(lib.w8_split_e4m3(_p(Wq), N, K, _p(We), _stream(stream)))
+    _check(lib.w8_codes_f16(_p(Wq), N, K, _p(We), _stream(stream)))
 
 
 def w8a8_gemm(Xe, s_a, We, s_w, Y, bias=None, acc_dbg=None, stream=None):
-    """Xe: activation code halves [L][2K] (sgat_quantize_act with bits=8);
-    We: weight code halves [N][2K] (w8_split_e4m3); Y [L][N]."""
+    """Xe: activation codes as fp16 [L][K] (sgat_quantize_act with bits=8),
+    We: weight codes as fp16 [N][K] (w8_codes_f16), each held as 2K bytes a
+    row; Y [L][N]."""
     _contig(Xe, s_a, We, s_w, Y, bias, acc_dbg)
     L, N = Y.shape
-    K = We.shape[1] // 2
+    K = We.shape[1] * We.element_size() // 2
     _check(lib.w8a8_gemm(_p(Xe), _p(s_a), _p(We), _p(s_w), _p(bias), L, N, K, _p(Y), dtype_code(Y), _p(acc_dbg),
                          _stream(stream)))
 

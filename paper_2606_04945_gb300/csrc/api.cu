@@ -646,13 +646,13 @@ int sgat_linear_dense(const void* X, int x_dtype, int L, int K, const uint8_t* m
     return STARQ_OK;
 }
 
-int w8_split_e4m3(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream) {
-    if (N > 0 && (!Wq || !We)) return fail(STARQ_ERR_ARG, "w8_split_e4m3: NULL Wq or We");
-    if (N < 0 || K < 128 || K % 128 != 0) return fail(STARQ_ERR_SHAPE, "w8_split_e4m3: N=%d K=%d (K %% 128 == 0)", N, K);
+int w8_codes_f16(const uint8_t* Wq, int N, int K, uint8_t* We, void* stream) {
+    if (N > 0 && (!Wq || !We)) return fail(STARQ_ERR_ARG, "w8_codes_f16: NULL Wq or We");
+    if (N < 0 || K < 128 || K % 128 != 0) return fail(STARQ_ERR_SHAPE, "w8_codes_f16: N=%d K=%d (K %% 128 == 0)", N, K);
     if (N == 0) return STARQ_OK;
-    if (!aligned(Wq, 16) || !aligned(We, 16)) return fail(STARQ_ERR_ALIGN, "w8_split_e4m3: Wq, We alignment");
-    cudaError_t e = launch_w8_split(Wq, We, (size_t)N, K, static_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return cuda_fail(e, "w8_split_e4m3 launch");
+    if (!aligned(Wq, 16) || !aligned(We, 16)) return fail(STARQ_ERR_ALIGN, "w8_codes_f16: Wq, We alignment");
+    cudaError_t e = launch_w8_codes_f16(Wq, We, (size_t)N, K, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "w8_codes_f16 launch");
     return STARQ_OK;
 }
 
@@ -797,7 +797,7 @@ int tac_calibrate(const void* Z_fp, const void* Z_q, int z_dtype, int N, int C, 
 size_t sgat_linear_workspace_size_bits(int L, int K, int with_tac, int bits) {
     if (L < 0 || K < 0 || (bits != 4 && bits != 8)) return 0;
     // codes (packed nibbles or bytes), s_a, the GEMM operand (E4M3 codes or
-    // the E4M3 halves of 8-bit codes), TAC output
+    // 8-bit codes as fp16), TAC output
     const size_t q = bits == 8 ? (size_t)L * K : (size_t)L * K / 2;
     const size_t e = bits == 8 ? (size_t)L * K * 2 : (size_t)L * K;
     size_t n = align256(q) + align256((size_t)L * 4) + align256(e);
@@ -866,6 +866,7 @@ int sgat_linear_impl(const void* X, int x_dtype, int L, int K, const uint8_t* ma
     if ((e = launch_sgat_quant(q, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: quant launch");
     if (bits == 8) {
         GemmArgs g8{nullptr, s_a, nullptr, s_w, bias, L, N, K, Y, y_dtype, nullptr, st, Xe, We};
+        g8.weights_ready = 1;    // the predecessor is the quantiser, which does not write the weights
         if ((e = launch_w8a8_gemm(g8, s)) != cudaSuccess) return cuda_fail(e, "sgat_linear: w8a8 gemm launch");
         return STARQ_OK;
     }

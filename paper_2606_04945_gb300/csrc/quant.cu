@@ -18,10 +18,8 @@
 // Storage by code width. qmax <= 7 (4-bit): Xq packs two codes per byte and
 // Xe holds each code as an E4M3 byte [rows][K]. qmax = 127 (8-bit, the W8A8
 // setting of Tab. 5): Xq holds one code per byte (two's complement) and Xe
-// [rows][2K] holds the nibble split c = 16 h + l, l = ((c + 8) mod 16) - 8 in
-// [-8, 7], h = (c - l) / 16 in [-8, 8]: E4M3 bytes of h in columns 0..K-1
-// and of l in columns K..2K-1 (both exact in E4M3), the operands of the
-// 8-bit GEMM.
+// [rows][K] each code as an fp16 number (exact: |c| <= 127), the operand of
+// the 8-bit GEMM.
 //
 // Asymmetric mode (a.asym, Eq. 2-4, activations): per row X_max = max(max v,
 // 0) and -X_min = max(max -v, 0); s = fl(fl(X_max - X_min) / qmax), r =
@@ -163,8 +161,8 @@ __device__ __forceinline__ void chunk_fwht(float (&v)[E], int hb, int lane, floa
 }
 
 // Eight 8-bit codes -> their bytes (two's complement, code k in byte k) and
-// the E4M3 bytes of their split c = 16 h + l (see the file comment).
-__device__ __forceinline__ void split_codes8(const int* q, uint2& bytes, uint2& eh, uint2& el) {
+// the same codes as fp16 numbers (exact), code k in half k.
+__device__ __forceinline__ void codes8(const int* q, uint2& bytes, uint4& f16) {
     uint32_t b0 = 0, b1 = 0;
     #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -172,16 +170,13 @@ __device__ __forceinline__ void split_codes8(const int* q, uint2& bytes, uint2& 
         b1 |= (uint32_t)(q[k + 4] & 0xFF) << (8 * k);
     }
     bytes = make_uint2(b0, b1);
-    uint16_t hh[4], ll[4];
+    uint32_t h[4];
     #pragma unroll
-    for (int k = 0; k < 4; ++k) {        // upper byte from the first operand
-        const int l0 = ((q[2 * k] + 8) & 15) - 8, l1 = ((q[2 * k + 1] + 8) & 15) - 8;
-        const int h0 = (q[2 * k] - l0) >> 4, h1 = (q[2 * k + 1] - l1) >> 4;
-        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(hh[k]) : "f"((float)h1), "f"((float)h0));
-        asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(ll[k]) : "f"((float)l1), "f"((float)l0));
+    for (int k = 0; k < 4; ++k) {
+        const __half2 p = __floats2half2_rn((float)q[2 * k], (float)q[2 * k + 1]);
+        h[k] = *reinterpret_cast<const uint32_t*>(&p);
     }
-    eh = make_uint2((uint32_t)hh[0] | ((uint32_t)hh[1] << 16), (uint32_t)hh[2] | ((uint32_t)hh[3] << 16));
-    el = make_uint2((uint32_t)ll[0] | ((uint32_t)ll[1] << 16), (uint32_t)ll[2] | ((uint32_t)ll[3] << 16));
+    f16 = make_uint4(h[0], h[1], h[2], h[3]);
 }
 
 // Eight codes in [0, 15] -> E4M3 bytes (byte k = code k).
@@ -361,19 +356,17 @@ sgat_quant_kernel(QuantArgs a, int warps_per_row, int rows_per_cta) {
             }
             continue;
         }
-        if (a.qmax > 15) {               // 8-bit codes: bytes and their E4M3 split
+        if (a.qmax > 15) {               // 8-bit codes: bytes and fp16
             #pragma unroll
             for (int u = 0; u < E / 8; ++u) {
                 int q[8];
                 #pragma unroll
                 for (int k = 0; k < 8; ++k) q[k] = __float2int_rn(__fmul_rn(v[j][8 * u + k], r));
-                uint2 bytes, eh, el;
-                split_codes8(q, bytes, eh, el);
+                uint2 bytes;
+                uint4 f16;
+                codes8(q, bytes, f16);
                 if (a.Xq != nullptr) *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + lo + 8 * u) = bytes;
-                if (a.Xe != nullptr) {
-                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + lo + 8 * u) = eh;
-                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + lo + 8 * u) = el;
-                }
+                if (a.Xe != nullptr) *reinterpret_cast<uint4*>(a.Xe + ((size_t)row * K + lo + 8 * u) * 2) = f16;
             }
             continue;
         }
@@ -769,14 +762,12 @@ sgat_quant_rows_kernel(QuantArgs a0, QuantArgs b) {
                 if (a.Xe != nullptr) *reinterpret_cast<uint2*>(a.Xe + (size_t)row * (K + 128) + e0) = e4m3_of8(q);
                 continue;
             }
-            if (a.qmax > 15) {           // 8-bit codes: bytes and their E4M3 split
-                uint2 bytes, eh, el;
-                split_codes8(qi, bytes, eh, el);
+            if (a.qmax > 15) {           // 8-bit codes: bytes and fp16
+                uint2 bytes;
+                uint4 f16;
+                codes8(qi, bytes, f16);
                 if (a.Xq != nullptr) *reinterpret_cast<uint2*>(a.Xq + (size_t)row * K + e0) = bytes;
-                if (a.Xe != nullptr) {
-                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + e0) = eh;
-                    *reinterpret_cast<uint2*>(a.Xe + (size_t)row * 2 * K + K + e0) = el;
-                }
+                if (a.Xe != nullptr) *reinterpret_cast<uint4*>(a.Xe + ((size_t)row * K + e0) * 2) = f16;
                 continue;
             }
             if (a.Xq != nullptr)

@@ -25,6 +25,7 @@
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
+#include "w8a8.cuh"
 
 namespace starq {
 namespace {
@@ -827,8 +828,10 @@ struct Cfg {
 }  // namespace tmak
 
 // OPK: operand kind -- 0 = E4M3 codes (dequantising epilogue), 1 = fp16,
-// 2 = bf16 (plain float32 accumulator cast to the output type). Every kind
-// reads 128-byte K rows and advances 32 bytes of K per MMA.
+// 2 = bf16 (plain float32 accumulator cast to the output type), 3 = 8-bit
+// codes held as fp16 (exact: |c| <= 127), accumulated in runs of 512 K that
+// the epilogue sums in int32 before dequantising. Every kind reads 128-byte
+// K rows and advances 32 bytes of K per MMA.
 // Tile of the calling thread's last TMA pair GEMM launch: BN * 10 + 2 (CTAs
 // per cluster).
 thread_local int g_last_tile = 0;
@@ -875,7 +878,13 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     static_assert(2 * EPI_CHUNKS * 32 >= BN, "two epilogue warps per row quarter cover the tile");
     constexpr uint32_t IDESC = Tile::IDESC | (OPK == 2 ? ((1u << 7) | (1u << 10)) : 0u);
     constexpr int BKE = OPK == 0 ? BK : BK / 2;          // K elements per stage row
-    constexpr bool DEQUANT = OPK == 0;
+    constexpr bool DEQUANT = OPK == 0 || OPK == 3;
+    // OPK 3: each accumulator takes a run of KRUN K blocks (512 K) and the
+    // epilogue adds the runs in int32, so that no float32 partial sum
+    // reaches 512 * 127^2 < 2^23 (exact); 0: one run per tile.
+    constexpr int KRUN = OPK == 3 ? 512 / BKE : 0;
+    static_assert(OPK != 3 || (BN > (EPI_CHUNKS - 1) * 32 && BN + 32 <= ACC_STRIDE && BN <= 2 * EPI_CHUNKS * 32 - 32),
+                  "kind 3: the fourth box of the first column half keeps its sum in the 32 TMEM columns after BN");
     constexpr uint16_t PAIR = 3u;                        // both CTAs of the cluster (one pair)
     using Smem = tmak::Smem<STAGES>;
 
@@ -977,14 +986,18 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
-            int it = 0;
-            for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters, ++it) {
-                const int acc = it & 1;
-                const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
-                if (!mbar_wait_bounded_warp(smem_addr(&sh->tmem_empty[acc]), acc_phase ^ 1u, abort)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * ACC_STRIDE);
+            int it = 0;          // accumulator runs issued (a tile each, or a K run of a tile: see KRUN)
+            for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters) {
+                uint32_t d_tmem = 0;
                 for (int kc = 0; kc < num_k; ++kc) {
+                    const int kk = KRUN > 0 ? kc % KRUN : kc;    // K block within the run
+                    if (kk == 0) {
+                        const int acc = it & 1;
+                        const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+                        if (!mbar_wait_bounded_warp(smem_addr(&sh->tmem_empty[acc]), acc_phase ^ 1u, abort)) { ok = false; break; }
+                        tc_fence_after();
+                        d_tmem = tmem_base + (uint32_t)(acc * ACC_STRIDE);
+                    }
                     if (!mbar_wait_bounded_warp(smem_addr(&sh->full[stage]), phase, abort)) { ok = false; break; }
                     tc_fence_after();
                     // stage offsets stay below 2^18 bytes, so adding them to
@@ -995,23 +1008,181 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                         #pragma unroll
                         for (int ks = 0; ks < BK / UMMA_K; ++ks) {
                             const uint64_t adk = ad + (uint64_t)(ks * UMMA_K / 16), bdk = bd + (uint64_t)(ks * UMMA_K / 16);
-                            if (OPK == 0) mma_f8f6f4_pair(d_tmem, adk, bdk, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
-                            else mma_f16_pair(d_tmem, adk, bdk, IDESC, (kc > 0 || ks > 0) ? 1u : 0u);
+                            if (OPK == 0) mma_f8f6f4_pair(d_tmem, adk, bdk, IDESC, (kk > 0 || ks > 0) ? 1u : 0u);
+                            else mma_f16_pair(d_tmem, adk, bdk, IDESC, (kk > 0 || ks > 0) ? 1u : 0u);
                         }
                         tc_commit_pair_multicast(smem_addr(&sh->empty[stage]), PAIR);
                     }
                     __syncwarp();
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                    if (kc + 1 == num_k || (KRUN > 0 && kk + 1 == KRUN)) {   // the run is complete
+                        if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->tmem_full[it & 1]), PAIR);
+                        __syncwarp();
+                        ++it;
+                    }
                 }
-                if (!ok) break;
-                if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->tmem_full[acc]), PAIR);
-                __syncwarp();
             }
             if (elect_one()) tc_commit_pair_multicast(smem_addr(&sh->drain), PAIR);
             __syncwarp();
             if (!ok && lane == 0) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
         }
         __syncwarp();
+    } else if (OPK == 3) {
+        // epilogue of the 8-bit kind: the same lanes, columns and boxes as
+        // below; every K run of the tile is read from TMEM, converted
+        // (exact integers) and added in int32 registers, and its accumulator
+        // handed back at once; after the last run the int32 sums are
+        // dequantised, fl(fl(fl32(acc) s_a) s_w) (+ bias), and stored.
+        constexpr int BOX_BYTES = 32 * 32 * (int)sizeof(TOut);
+        constexpr int NBUF = EPI_BOX_WARP_BYTES / BOX_BYTES;
+        const uint32_t leader_tmem_empty0 = mapa_shared(smem_addr(&sh->tmem_empty[0]), leader);
+        const uint32_t ybox0 = base + STAGES * STAGE_BYTES + warp * EPI_BOX_WARP_BYTES;
+        float* epi_sw = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(sh) + sizeof(Smem) +
+                                                 (16 - sizeof(Smem) % 16) % 16) + warp * 2 * (EPI_CHUNKS * 32);
+        float* epi_b = epi_sw + EPI_CHUNKS * 32;
+        const int quarter = warp & 3, chalf = warp >> 2;
+        const int runs = KRUN > 0 ? (num_k + KRUN - 1) / KRUN : 1;
+        bool ok = true;
+        int it = 0;
+        int nbox = 0;
+        for (int tile = cluster; tile < num_tiles && ok; tile += num_clusters) {
+            const bool p1 = G2 && tile >= num_tiles0;
+            const int lt = p1 ? tile - num_tiles0 : tile;
+            const GemmArgs& P = p1 ? b : a;
+            const void* my = p1 ? (const void*)&tmap_y2 : (const void*)&tmap_y;
+            const int N = P.N;
+            const int m0 = (lt % num_m) * 2 * BM + (int)half * BM;
+            const int n0 = (lt / num_m) * BN;
+            const int row = m0 + quarter * 32 + lane;
+            const bool valid = row < L;
+            const float sa = valid ? __ldg(P.s_a + row) : 0.f;
+            {
+                const int ncol = n0 + chalf * (EPI_CHUNKS * 32) + 4 * lane;
+                float4 w = make_float4(0.f, 0.f, 0.f, 0.f), bb = w;
+                if (ncol < N) {
+                    w = __ldg(reinterpret_cast<const float4*>(P.s_w + ncol));
+                    if (P.bias != nullptr) bb = __ldg(reinterpret_cast<const float4*>(P.bias + ncol));
+                }
+                __syncwarp();
+                reinterpret_cast<float4*>(epi_sw)[lane] = w;
+                reinterpret_cast<float4*>(epi_b)[lane] = bb;
+                __syncwarp();
+            }
+            // boxes 0-2 of the warp: int32 sums in registers; box 3 (the
+            // warps of the first column half): in the free TMEM columns
+            // BN .. BN + 31 beside accumulator 0, on the warp's own lanes
+            int sum[EPI_CHUNKS - 1][32];
+            const uint32_t t_sum = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)BN;
+            for (int run = 0; run < runs; ++run, ++it) {
+                const int acc = it & 1;
+                const uint32_t acc_phase = (uint32_t)(it >> 1) & 1u;
+                if (!mbar_wait_bounded_sleepy(smem_addr(&sh->tmem_full[acc]), acc_phase, abort, 64)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t t_row = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * ACC_STRIDE);
+                #pragma unroll
+                for (int cc = 0; cc < EPI_CHUNKS; ++cc) {
+                    const int c = chalf * EPI_CHUNKS + cc;
+                    if (c * 32 < BN && n0 + c * 32 < N) {          // warp-uniform
+                        #pragma unroll
+                        for (int h = 0; h < 4; ++h) {              // 8 columns at a time: registers
+                            uint32_t r[8];
+                            tmem_ld_32x32b_x8(t_row + c * 32 + 8 * h, r);
+                            if (cc < EPI_CHUNKS - 1) {
+                                tmem_ld_wait();
+                                #pragma unroll
+                                for (int t = 0; t < 8; ++t) {
+                                    const int v = __float2int_rn(__uint_as_float(r[t]));
+                                    int& sv = sum[cc < EPI_CHUNKS - 1 ? cc : 0][8 * h + t];
+                                    sv = run == 0 ? v : sv + v;
+                                }
+                            } else {
+                                uint32_t s8[8];
+                                if (run > 0) tmem_ld_32x32b_x8(t_sum + 8 * h, s8);
+                                tmem_ld_wait();
+                                #pragma unroll
+                                for (int t = 0; t < 8; ++t)
+                                    s8[t] = (uint32_t)(__float2int_rn(__uint_as_float(r[t])) + (run > 0 ? (int)s8[t] : 0));
+                                tmem_st_32x32b_x8(t_sum + 8 * h, s8);
+                                tmem_st_wait();
+                            }
+                        }
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + acc * 8);
+            }
+            if (!ok) break;
+            // dequantise one box of sums and store it
+            auto emit = [&](const int (&q)[32], int cc, int nc) {
+                if (P.acc_dbg != nullptr && valid) {
+                    int4* d4 = reinterpret_cast<int4*>(P.acc_dbg + (size_t)row * N + nc);
+                    #pragma unroll
+                    for (int u = 0; u < 8; ++u) d4[u] = make_int4(q[4 * u], q[4 * u + 1], q[4 * u + 2], q[4 * u + 3]);
+                }
+                float y[32];
+                const float4* sw4 = reinterpret_cast<const float4*>(epi_sw + cc * 32);
+                const float4* b4 = reinterpret_cast<const float4*>(epi_b + cc * 32);
+                #pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const float4 sw = sw4[u];
+                    y[4 * u] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u]), sa), sw.x);
+                    y[4 * u + 1] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u + 1]), sa), sw.y);
+                    y[4 * u + 2] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u + 2]), sa), sw.z);
+                    y[4 * u + 3] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u + 3]), sa), sw.w);
+                }
+                if (P.bias != nullptr) {
+                    #pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const float4 bq = b4[u];
+                        y[4 * u] = __fadd_rn(y[4 * u], bq.x);
+                        y[4 * u + 1] = __fadd_rn(y[4 * u + 1], bq.y);
+                        y[4 * u + 2] = __fadd_rn(y[4 * u + 2], bq.z);
+                        y[4 * u + 3] = __fadd_rn(y[4 * u + 3], bq.w);
+                    }
+                }
+                // the buffer's previous store has read it
+                const uint32_t box = ybox0 + (uint32_t)((nbox % NBUF) * BOX_BYTES);
+                if (nbox >= NBUF) {
+                    if (lane == 0) {
+                        if (NBUF == 2) bulk_wait_read1(); else bulk_wait_read0();
+                    }
+                    __syncwarp();
+                }
+                Out<TOut>::stage32(box, lane, y);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(my, nc, m0 + quarter * 32, box);
+                    bulk_commit();
+                }
+                ++nbox;
+            };
+            #pragma unroll
+            for (int cc = 0; cc < EPI_CHUNKS - 1; ++cc) {
+                const int c = chalf * EPI_CHUNKS + cc;
+                if (c * 32 < BN && n0 + c * 32 < N) emit(sum[cc], cc, n0 + c * 32);
+            }
+            {
+                constexpr int cc = EPI_CHUNKS - 1;
+                const int c = chalf * EPI_CHUNKS + cc;
+                if (c * 32 < BN && n0 + c * 32 < N) {
+                    int q[32];
+                    #pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        uint32_t s8[8];
+                        tmem_ld_32x32b_x8(t_sum + 8 * h, s8);
+                        tmem_ld_wait();
+                        #pragma unroll
+                        for (int t = 0; t < 8; ++t) q[8 * h + t] = (int)s8[t];
+                    }
+                    emit(q, cc, n0 + c * 32);
+                }
+            }
+        }
+        if (lane == 0) bulk_wait0();     // this warp's stores are complete
+        __syncwarp();
+        if (!ok) { sh->abort = 1; atomicOr(a.status, STATUS_TIMEOUT_GEMM); }
     } else {
         // epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31, columns
         // (w / 4) * 128 .. + 127 below BN, in 32 x 32 boxes; scales and biases are
@@ -1242,22 +1413,31 @@ cudaError_t launch_tma_cl(const GemmArgs& a, cudaStream_t stream, int clusters, 
 // the LLaDA projections better); the cheaper estimate wins, ties keep 256.
 template <typename TOut, int OPK, bool SW>
 cudaError_t launch_tma_shape(const GemmArgs& a, cudaStream_t stream) {
-    int c256 = 0, c224 = 0;
-    cudaError_t e = tma_max_clusters<TOut, OPK, 256, SW>(&c256);
-    if (e != cudaSuccess) return e;
-    if ((e = tma_max_clusters<TOut, OPK, 224, SW>(&c224)) != cudaSuccess) return e;
-    if (g_pair_limit > 0) {
-        if (c256 > g_pair_limit) c256 = g_pair_limit;
-        if (c224 > g_pair_limit) c224 = g_pair_limit;
-    }
-    const long long t256 = tma_round_cost(a.L, a.N, 256, c256);
-    const long long t224 = tma_round_cost(a.L, a.N, 224, c224);
-    if (t224 < t256) {
+    if constexpr (OPK == 3) {            // 224-wide tiles only: their free TMEM columns hold a box of sums
+        int c224 = 0;
+        const cudaError_t e = tma_max_clusters<TOut, OPK, 224, SW>(&c224);
+        if (e != cudaSuccess) return e;
+        if (g_pair_limit > 0 && c224 > g_pair_limit) c224 = g_pair_limit;
         g_last_tile = 224 * 10 + 2;
         return launch_tma_cl<TOut, OPK, 224, SW>(a, stream, c224);
+    } else {
+        int c256 = 0, c224 = 0;
+        cudaError_t e = tma_max_clusters<TOut, OPK, 256, SW>(&c256);
+        if (e != cudaSuccess) return e;
+        if ((e = tma_max_clusters<TOut, OPK, 224, SW>(&c224)) != cudaSuccess) return e;
+        if (g_pair_limit > 0) {
+            if (c256 > g_pair_limit) c256 = g_pair_limit;
+            if (c224 > g_pair_limit) c224 = g_pair_limit;
+        }
+        const long long t256 = tma_round_cost(a.L, a.N, 256, c256);
+        const long long t224 = tma_round_cost(a.L, a.N, 224, c224);
+        if (t224 < t256) {
+            g_last_tile = 224 * 10 + 2;
+            return launch_tma_cl<TOut, OPK, 224, SW>(a, stream, c224);
+        }
+        g_last_tile = 256 * 10 + 2;
+        return launch_tma_cl<TOut, OPK, 256, SW>(a, stream, c256);
     }
-    g_last_tile = 256 * 10 + 2;
-    return launch_tma_cl<TOut, OPK, 256, SW>(a, stream, c256);
 }
 
 // Two independent problems (same L, K and output type, E4M3 operands, no
@@ -1390,6 +1570,17 @@ cudaError_t launch_fp16_gemm(const GemmArgs& a, cudaStream_t stream) {
     switch (a.y_dtype) {
         case STARQ_F16: return launch_tma_typed<__half, 1>(a, stream);
         case STARQ_BF16: return launch_tma_typed<__nv_bfloat16, 2>(a, stream);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_w8a8_gemm(const GemmArgs& a, cudaStream_t stream) {
+    if (a.L == 0) return cudaSuccess;
+    if (a.Xe == nullptr || a.We == nullptr || a.swiglu) return cudaErrorInvalidValue;
+    switch (a.y_dtype) {
+        case STARQ_F16: return launch_tma_typed<__half, 3>(a, stream);
+        case STARQ_BF16: return launch_tma_typed<__nv_bfloat16, 3>(a, stream);
+        case STARQ_F32: return launch_tma_typed<float, 3>(a, stream);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -77,15 +77,15 @@ def test_w8a8_gemm_validation(lib, L, N, K, code):
     assert lib.lib.starq_last_error()
 
 
-def test_w8_split_validation(lib):
-    assert lib.lib.w8_split_e4m3(P, 4, 200, P, None) == -2          # K % 128
-    assert lib.lib.w8_split_e4m3(ctypes.c_void_p(4100), 4, 256, P, None) == -3
-    assert lib.lib.w8_split_e4m3(P, 0, 256, P, None) == 0           # nothing to do
+def test_w8_codes_validation(lib):
+    assert lib.lib.w8_codes_f16(P, 4, 200, P, None) == -2           # K % 128
+    assert lib.lib.w8_codes_f16(ctypes.c_void_p(4100), 4, 256, P, None) == -3
+    assert lib.lib.w8_codes_f16(P, 0, 256, P, None) == 0            # nothing to do
 
 
 def test_linear_workspace_by_bits(lib):
-    """8-bit codes take a byte each and their E4M3 halves two; 4-bit codes
-    half a byte and one."""
+    """8-bit codes take a byte each and their fp16 operand form two; 4-bit
+    codes half a byte and one."""
     L, K = 1000, 4096
     a256 = lambda x: (x + 255) // 256 * 256
     assert lib.lib.sgat_linear_workspace_size_bits(L, K, 0, 4) == lib.lib.sgat_linear_workspace_size(L, K, 0)

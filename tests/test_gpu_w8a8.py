@@ -2,14 +2,16 @@
 
 The quantiser and the weight preparation take qmax = 127. Their codes and
 scales must be bit-exact with the oracle (`oracle/sgat.py`, generic in the
-bit width and pinned at 8 bits by brute force). The GEMM operand splits
-each code as c = 16 h + l, with l = ((c + 8) mod 16) - 8, and stores the
-E4M3 bytes of h and l. That split is checked against its definition.
-w8a8_gemm's integer sums are compared bit for bit with the oracle's exact
-integer product, and its outputs within the dequantisation tolerance.
-This includes codes at ±127 everywhere, where |acc| = 127² K exceeds the
-float32 integer range and only the int32 combination of the three partial
-sums is exact.
+bit width and pinned at 8 bits by brute force). The GEMM operand holds each
+code as an fp16 number, checked against numpy's own float16 conversion of
+the oracle's codes. w8a8_gemm's integer sums are compared bit for bit with
+the oracle's exact integer product, and its outputs within the
+dequantisation tolerance. This includes codes at ±127 everywhere, where
+|acc| = 127² K exceeds the float32 integer range: only the int32 sum of the
+kernel's 512-K runs (each below 2^23, exact in float32) reaches the full
+value; K that is not a multiple of 512 (a short last run) and CTA pairs
+that take several tiles (the run count carrying the accumulator parity
+across tiles).
 """
 
 import numpy as np
@@ -23,13 +25,11 @@ from tests import helpers as H
 pytestmark = pytest.mark.gpu
 
 
-def split_bytes(codes):
-    """E4M3 bytes [rows][2K] of the halves of 8-bit codes (h first, then l)."""
+def f16_bytes(codes):
+    """Bytes [rows][2K] of 8-bit codes held as fp16 (little-endian halves)."""
     c = np.asarray(codes, dtype=np.int64)
-    lo = ((c + 8) & 15) - 8
-    hi = (c - lo) // 16
-    assert np.array_equal(16 * hi + lo, c)
-    return np.concatenate([H.e4m3_bytes(hi), H.e4m3_bytes(lo)], axis=1)
+    assert np.abs(c).max() <= 127
+    return np.ascontiguousarray(c.astype(np.float16)).view(np.uint8)
 
 
 def quant8(abi, case, with_xe=True):
@@ -52,7 +52,7 @@ def prepare8(abi, case):
     abi.sgat_prepare_weight(H.dev(case.W, H.torch_dtype(case.dtype)), H.dev(case.xf.inv_a_w), case.xf.hb, Wq, s_w,
                             bits=8)
     We = torch.empty(N, 2 * K, dtype=torch.uint8, device="cuda")
-    abi.w8_split_e4m3(Wq, We)
+    abi.w8_codes_f16(Wq, We)
     abi.check_status()
     return Wq, s_w, We
 
@@ -67,7 +67,7 @@ def test_quantize_act_8bit_bitexact(abi, L, K, hb, dtype):
     assert np.abs(codes).max() == 127                      # the row maxima reach qmax
     assert np.array_equal(Xq.cpu().numpy().astype(np.int64), codes), "8-bit codes differ"
     assert np.array_equal(s_a.cpu().numpy(), s), "scales differ"
-    assert np.array_equal(Xe.cpu().numpy(), split_bytes(codes)), "E4M3 halves differ"
+    assert np.array_equal(Xe.cpu().numpy(), f16_bytes(codes)), "fp16 operand differs"
 
 
 @pytest.mark.parametrize("N,K,hb,dtype", [(256, 4096, 4096, "bf16"), (128, 512, 512, "f16"), (384, 1024, 64, "f32")])
@@ -77,17 +77,17 @@ def test_prepare_weight_8bit_bitexact(abi, N, K, hb, dtype):
     q, s = osg.prepare_weight(case.W, case.xf.inv_a_w, hb, 8)
     assert np.array_equal(Wq.cpu().numpy().astype(np.int64), q), "8-bit weight codes differ"
     assert np.array_equal(s_w.cpu().numpy(), s)
-    assert np.array_equal(We.cpu().numpy(), split_bytes(q)), "E4M3 halves differ"
+    assert np.array_equal(We.cpu().numpy(), f16_bytes(q)), "fp16 operand differs"
 
 
 def run_gemm(abi, qa, s_a, qw, s_w, y_dtype, bias=None):
     L, K = qa.shape
     N = qw.shape[0]
-    Xe = torch.from_numpy(split_bytes(qa)).cuda()
+    Xe = torch.from_numpy(f16_bytes(qa)).cuda()
     Wq = torch.from_numpy(qw.astype(np.int8)).cuda()
     We = torch.empty(N, 2 * K, dtype=torch.uint8, device="cuda")
-    abi.w8_split_e4m3(Wq, We)
-    assert np.array_equal(We.cpu().numpy(), split_bytes(qw))
+    abi.w8_codes_f16(Wq, We)
+    assert np.array_equal(We.cpu().numpy(), f16_bytes(qw))
     Y = torch.empty(L, N, dtype=H.torch_dtype(y_dtype), device="cuda")
     acc = torch.empty(L, N, dtype=torch.int32, device="cuda")
     abi.w8a8_gemm(Xe, H.dev(s_a), We, H.dev(s_w), Y, bias=None if bias is None else H.dev(bias), acc_dbg=acc)
@@ -96,9 +96,11 @@ def run_gemm(abi, qa, s_a, qw, s_w, y_dtype, bias=None):
 
 
 @pytest.mark.parametrize("L,N,K,y_dtype", [(128, 128, 128, "f32"), (200, 256, 4096, "f16"), (77, 384, 1024, "bf16"),
-                                            (1, 128, 256, "f16")])
+                                            (1, 128, 256, "f16"), (300, 640, 1152, "f16"), (513, 896, 2560, "bf16")])
 def test_w8a8_gemm_matches_oracle(abi, L, N, K, y_dtype):
-    """Random 8-bit codes over several tiles and a ragged last row tile."""
+    """Random 8-bit codes over several tiles, a ragged last row tile and a
+    ragged last column tile; K from one short run (128) to five runs with a
+    short last one (2560 = 5 x 512; 1152 = 2 x 512 + 128)."""
     rng = np.random.default_rng(L * N + K)
     qa = rng.integers(-127, 128, (L, K))
     qw = rng.integers(-127, 128, (N, K))
@@ -113,10 +115,32 @@ def test_w8a8_gemm_matches_oracle(abi, L, N, K, y_dtype):
     H.assert_output_close(Y, osg.dequant(ref_acc, s_a, s_w, bias), y_dtype)
 
 
+@pytest.mark.parametrize("pairs", [1, 2])
+def test_w8a8_gemm_several_tiles_per_pair(abi, pairs):
+    """Fewer CTA pairs than tiles (the pair limit): each pair runs several
+    tiles, with three runs per tile (K = 1152), so that consecutive tiles
+    start on alternate accumulators."""
+    L, N, K = 300, 640, 1152                       # 2 x 3 tiles of 256 x 224
+    rng = np.random.default_rng(pairs)
+    qa = rng.integers(-127, 128, (L, K))
+    qw = rng.integers(-127, 128, (N, K))
+    s_a = rng.uniform(0.001, 0.05, L).astype(np.float32)
+    s_w = rng.uniform(0.001, 0.05, N).astype(np.float32)
+    bias = rng.normal(0, 0.1, N).astype(np.float32)
+    prev = abi.set_gemm_pair_limit(pairs)
+    try:
+        Y, acc = run_gemm(abi, qa, s_a, qw, s_w, "f16", bias)
+    finally:
+        abi.set_gemm_pair_limit(prev)
+    ref_acc = osg.int_gemm(qa, qw)
+    assert np.array_equal(acc, ref_acc), "integer sums differ"
+    H.assert_output_close(Y, osg.dequant(ref_acc, s_a, s_w, bias), "f16")
+
+
 def test_w8a8_gemm_extreme_codes(abi):
     """Every code ±127 with aligned signs: |acc| = 127² K = 66 M at K = 4096,
-    above 2^24. Each partial sum stays exact in float32 and only their int32
-    combination reaches the full value."""
+    above 2^24. Each 512-K run's sum (127² 512 < 2^23) stays exact in
+    float32 and only their int32 sum reaches the full value."""
     L, N, K = 128, 256, 4096
     rng = np.random.default_rng(1)
     sa = np.where(rng.random((L, 1)) < 0.5, -1, 1)
@@ -152,11 +176,12 @@ def test_sgat_linear_8bit(abi, L, K, N, hb, dtype, tac_g):
                     ws, bias=H.dev(case.bias), tac_M=tac_M, tac_d=tac_d, tac_g=tac_g or 0, bits=8, We=We)
     abi.check_status()
     a256 = lambda x: (x + 255) // 256 * 256
-    # [code region, left unwritten][s_a][Xe: the E4M3 split h | l of each code, c = 16 h + l]
+    # [code region, left unwritten][s_a][Xe: each code as fp16]
     s_a = ws[a256(L * K): a256(L * K) + 4 * L].view(torch.float32).cpu().numpy()
     o_e = a256(L * K) + a256(4 * L)
-    Xe = ws[o_e: o_e + 2 * L * K].view(L, 2 * K)
-    Xq = 16 * H.codes_from_e4m3(Xe[:, :K]).astype(np.int64) + H.codes_from_e4m3(Xe[:, K:])
+    Xe = ws[o_e: o_e + 2 * L * K].cpu().numpy()
+    Xq = Xe.view(np.float16).reshape(L, K).astype(np.int64)
+    assert np.array_equal(f16_bytes(Xq), Xe.reshape(L, 2 * K)), "operand bytes are not fp16 integers"
     if tac_g:
         o = a256(L * K) + a256(4 * L) + a256(2 * L * K)
         esz = torch.empty(0, dtype=dt).element_size()
