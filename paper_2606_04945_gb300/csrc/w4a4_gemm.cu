@@ -829,7 +829,7 @@ struct Cfg {
 
 // OPK: operand kind -- 0 = E4M3 codes (dequantising epilogue), 1 = fp16,
 // 2 = bf16 (plain float32 accumulator cast to the output type), 3 = 8-bit
-// codes held as fp16 (exact: |c| <= 127), accumulated in runs of 512 K that
+// codes held as fp16 (exact: |c| <= 127), accumulated in runs of 256 K that
 // the epilogue sums in int32 before dequantising. Every kind reads 128-byte
 // K rows and advances 32 bytes of K per MMA.
 // Tile of the calling thread's last TMA pair GEMM launch: BN * 10 + 2 (CTAs
@@ -879,10 +879,17 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
     constexpr uint32_t IDESC = Tile::IDESC | (OPK == 2 ? ((1u << 7) | (1u << 10)) : 0u);
     constexpr int BKE = OPK == 0 ? BK : BK / 2;          // K elements per stage row
     constexpr bool DEQUANT = OPK == 0 || OPK == 3;
-    // OPK 3: each accumulator takes a run of KRUN K blocks (512 K) and the
-    // epilogue adds the runs in int32, so that no float32 partial sum
-    // reaches 512 * 127^2 < 2^23 (exact); 0: one run per tile.
-    constexpr int KRUN = OPK == 3 ? 512 / BKE : 0;
+    // OPK 3: each accumulator takes a run of RUN_K K (KRUN K blocks) and
+    // the epilogue adds the runs in int32. A run's sum is an integer of
+    // magnitude at most RUN_K * 127^2 < 2^22 at RUN_K = 256: exact in float32,
+    // and fl(v + 1.5 * 2^23) = 2^23 + 2^22 + v exactly, whose bits are
+    // 0x4B400000 + v (MAGIC: the conversion is one add). The offsets are
+    // summed in wrapping 32-bit arithmetic and removed once per tile.
+    // OPK 0-2: one run per tile (KRUN 0).
+    constexpr int RUN_K = 512;
+    constexpr bool MAGIC = (long long)RUN_K * 127 * 127 < (1LL << 22);
+    static_assert(OPK != 3 || (long long)RUN_K * 127 * 127 < (1LL << 24), "a run's float32 sum is exact");
+    constexpr int KRUN = OPK == 3 ? RUN_K / BKE : 0;
     static_assert(OPK != 3 || (BN > (EPI_CHUNKS - 1) * 32 && BN + 32 <= ACC_STRIDE && BN <= 2 * EPI_CHUNKS * 32 - 32),
                   "kind 3: the fourth box of the first column half keeps its sum in the 32 TMEM columns after BN");
     constexpr uint16_t PAIR = 3u;                        // both CTAs of the cluster (one pair)
@@ -1071,7 +1078,12 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
             // boxes 0-2 of the warp: int32 sums in registers; box 3 (the
             // warps of the first column half): in the free TMEM columns
             // BN .. BN + 31 beside accumulator 0, on the warp's own lanes
-            int sum[EPI_CHUNKS - 1][32];
+            uint32_t sum[EPI_CHUNKS - 1][32];
+            const uint32_t corr = MAGIC ? (uint32_t)runs * 0x4B400000u : 0u;   // the runs' offsets
+            auto run_bits = [](uint32_t x) -> uint32_t {   // a run's exact integer (plus the offset)
+                return MAGIC ? __float_as_uint(__fadd_rn(__uint_as_float(x), 12582912.f))
+                             : (uint32_t)__float2int_rn(__uint_as_float(x));
+            };
             const uint32_t t_sum = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)BN;
             for (int run = 0; run < runs; ++run, ++it) {
                 const int acc = it & 1;
@@ -1083,42 +1095,47 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 for (int cc = 0; cc < EPI_CHUNKS; ++cc) {
                     const int c = chalf * EPI_CHUNKS + cc;
                     if (c * 32 < BN && n0 + c * 32 < N) {          // warp-uniform
-                        #pragma unroll
-                        for (int h = 0; h < 4; ++h) {              // 8 columns at a time: registers
-                            uint32_t r[8];
-                            tmem_ld_32x32b_x8(t_row + c * 32 + 8 * h, r);
-                            if (cc < EPI_CHUNKS - 1) {
-                                tmem_ld_wait();
-                                #pragma unroll
-                                for (int t = 0; t < 8; ++t) {
-                                    const int v = __float2int_rn(__uint_as_float(r[t]));
-                                    int& sv = sum[cc < EPI_CHUNKS - 1 ? cc : 0][8 * h + t];
-                                    sv = run == 0 ? v : sv + v;
-                                }
-                            } else {
-                                uint32_t s8[8];
+                        if (cc < EPI_CHUNKS - 1) {                 // a register box: one load
+                            uint32_t r[32];
+                            tmem_ld_32x32b_x32(t_row + c * 32, r);
+                            tmem_ld_wait();
+                            #pragma unroll
+                            for (int t = 0; t < 32; ++t) {
+                                const uint32_t v = run_bits(r[t]);
+                                uint32_t& sv = sum[cc < EPI_CHUNKS - 1 ? cc : 0][t];
+                                sv = run == 0 ? v : sv + v;
+                            }
+                        } else {                                   // the TMEM box: 8 columns at a time
+                            #pragma unroll
+                            for (int h = 0; h < 4; ++h) {
+                                uint32_t r[8], s8[8];
+                                tmem_ld_32x32b_x8(t_row + c * 32 + 8 * h, r);
                                 if (run > 0) tmem_ld_32x32b_x8(t_sum + 8 * h, s8);
                                 tmem_ld_wait();
                                 #pragma unroll
                                 for (int t = 0; t < 8; ++t)
-                                    s8[t] = (uint32_t)(__float2int_rn(__uint_as_float(r[t])) + (run > 0 ? (int)s8[t] : 0));
+                                    s8[t] = run_bits(r[t]) + (run > 0 ? s8[t] : 0u);
                                 tmem_st_32x32b_x8(t_sum + 8 * h, s8);
-                                tmem_st_wait();
                             }
+                            tmem_st_wait();                        // before the next run reads them back
                         }
                     }
                 }
+                // the run's TMEM reads are complete (tcgen05.wait::ld) and ordered
+                // by the fence: a relaxed arrive hands the accumulator back
+                // without a memory barrier
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + acc * 8);
+                if (lane == 0) mbar_arrive_cluster_relaxed(leader_tmem_empty0 + acc * 8);
             }
             if (!ok) break;
             // dequantise one box of sums and store it
-            auto emit = [&](const int (&q)[32], int cc, int nc) {
+            auto emit = [&](const uint32_t (&qs)[32], int cc, int nc) {
+                auto q = [&](int t) { return (int)(qs[t] - corr); };
                 if (P.acc_dbg != nullptr && valid) {
                     int4* d4 = reinterpret_cast<int4*>(P.acc_dbg + (size_t)row * N + nc);
                     #pragma unroll
-                    for (int u = 0; u < 8; ++u) d4[u] = make_int4(q[4 * u], q[4 * u + 1], q[4 * u + 2], q[4 * u + 3]);
+                    for (int u = 0; u < 8; ++u) d4[u] = make_int4(q(4 * u), q(4 * u + 1), q(4 * u + 2), q(4 * u + 3));
                 }
                 float y[32];
                 const float4* sw4 = reinterpret_cast<const float4*>(epi_sw + cc * 32);
@@ -1126,10 +1143,10 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
                     const float4 sw = sw4[u];
-                    y[4 * u] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u]), sa), sw.x);
-                    y[4 * u + 1] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u + 1]), sa), sw.y);
-                    y[4 * u + 2] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u + 2]), sa), sw.z);
-                    y[4 * u + 3] = __fmul_rn(__fmul_rn(__int2float_rn(q[4 * u + 3]), sa), sw.w);
+                    y[4 * u] = __fmul_rn(__fmul_rn(__int2float_rn(q(4 * u)), sa), sw.x);
+                    y[4 * u + 1] = __fmul_rn(__fmul_rn(__int2float_rn(q(4 * u + 1)), sa), sw.y);
+                    y[4 * u + 2] = __fmul_rn(__fmul_rn(__int2float_rn(q(4 * u + 2)), sa), sw.z);
+                    y[4 * u + 3] = __fmul_rn(__fmul_rn(__int2float_rn(q(4 * u + 3)), sa), sw.w);
                 }
                 if (P.bias != nullptr) {
                     #pragma unroll
@@ -1167,14 +1184,14 @@ w4a4_gemm_tma_pair_kernel(GemmArgs a, const __grid_constant__ CUtensorMap tmap_a
                 constexpr int cc = EPI_CHUNKS - 1;
                 const int c = chalf * EPI_CHUNKS + cc;
                 if (c * 32 < BN && n0 + c * 32 < N) {
-                    int q[32];
+                    uint32_t q[32];
                     #pragma unroll
                     for (int h = 0; h < 4; ++h) {
                         uint32_t s8[8];
                         tmem_ld_32x32b_x8(t_sum + 8 * h, s8);
                         tmem_ld_wait();
                         #pragma unroll
-                        for (int t = 0; t < 8; ++t) q[8 * h + t] = (int)s8[t];
+                        for (int t = 0; t < 8; ++t) q[8 * h + t] = s8[t];
                     }
                     emit(q, cc, n0 + c * 32);
                 }
