@@ -100,6 +100,15 @@ def config_dict(graph, grouped=True):
             "streams": forms[grouped]}
 
 
+STEP_FORMS = {"grouped": True, "grouped-gemm": "gemm", "forked": False}
+
+
+def arm_config(args):
+    """The workload config of a bench line from its command-line arguments:
+    the same for our arm and the reference arm of one command."""
+    return config_dict(not getattr(args, "no_graph", False), STEP_FORMS[getattr(args, "step_form", "grouped")])
+
+
 # ---------------------------------------------------------------------------
 # Clocks during the timed region
 # ---------------------------------------------------------------------------
@@ -624,7 +633,7 @@ def run_ours(args):
     from paper_2606_04945_gb300.pipeline import AttentionProjections
 
     qkv_case, o_case = inputs.llada_attention(seed=rank_seed(rank))
-    grouped = {"grouped": True, "grouped-gemm": "gemm", "forked": False}[args.step_form]
+    grouped = STEP_FORMS[args.step_form]
     step = AttentionProjections(qkv_case, o_case, grouped=grouped)
     L, K = step.L, step.qkv.K
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
@@ -841,7 +850,7 @@ def run_ours(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "int4 (W4A4 codes, exact integer accumulation; fp32 transform and dequant; fp16 I/O)",
         "data": "synthetic (seeded; LLaDA-8B-shaped activations and random-init weights)",
-        "config": config_dict(graph, grouped),
+        "config": arm_config(args),
         "tokens_per_s": round(tokens_s, 1),
         "roofline": {
             "bound": "tensor",
@@ -1030,7 +1039,7 @@ def run_reference(args):
         "metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(sec * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int4 codes, int64-exact GEMM, fp32 transform, fp64 dequant",
-        "data": "synthetic (seeded; LLaDA-8B-shaped)", "config": config_dict(False), "impl": "reference",
+        "data": "synthetic (seeded; LLaDA-8B-shaped)", "config": arm_config(args), "impl": "reference",
         "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "kind": "oracle", "cores": cpu_cores(),
                          "sample": f"each step: {S} random tokens of the 1024-token workload"},
         "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

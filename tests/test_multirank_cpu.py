@@ -90,3 +90,24 @@ def test_job_throughput_is_weak_scaling():
     assert bench.job_tops(ops, 0.1, 4) == pytest.approx(4 * one)
     assert bench.job_tops(ops, 0.2, 2) == pytest.approx(one)
     assert len({bench.rank_seed(r) for r in range(8)}) == 8
+
+
+def test_reference_line_matches_our_arm():
+    """The reference arm's line (rank 0, the oracle on a small sample) has
+    our arm's metric, unit, direction and config for the same arguments,
+    and the keys the contract asks of it."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    class Args(_Args):
+        no_graph = False
+        step_form = "grouped"
+
+    line = bench.run_reference(Args())
+    assert line["impl"] == "reference"
+    assert line["metric"] == bench.METRIC and line["unit"] == bench.UNIT and line["higher_is_better"] is True
+    assert line["config"] == bench.arm_config(Args()) == bench.config_dict(True, True)
+    assert line["value"] > 0 and line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
