@@ -196,3 +196,23 @@ def test_sgat_linear_8bit(abi, L, K, N, hb, dtype, tac_g):
     ref_acc = osg.int_gemm(codes[rows], qw)
     ref = osg.dequant(ref_acc, s[rows], sw_ref, case.bias)
     H.assert_output_close(H.host(Y)[rows], ref, dtype)
+
+
+def test_w8a8_empty_batch(abi):
+    """L = 0 (N = 0 for the weight form) is a valid no-op of every 8-bit
+    entry point."""
+    K, N = 512, 256
+    X = torch.empty(0, K, dtype=torch.float16, device="cuda")
+    Xq = torch.empty(0, K, dtype=torch.int8, device="cuda")
+    s = torch.empty(0, dtype=torch.float32, device="cuda")
+    Xe = torch.empty(0, 2 * K, dtype=torch.uint8, device="cuda")
+    abi.sgat_quantize_act(X, None, None, None, 512, K, 0, 0, Xq, s, bits=8, Xe=Xe)
+    We = torch.zeros(N, 2 * K, dtype=torch.uint8, device="cuda")
+    sw = torch.ones(N, dtype=torch.float32, device="cuda")
+    Y = torch.empty(0, N, dtype=torch.float16, device="cuda")
+    abi.w8a8_gemm(Xe, s, We, sw, Y)
+    abi.w8_codes_f16(torch.empty(0, K, dtype=torch.int8, device="cuda"),
+                     torch.empty(0, 2 * K, dtype=torch.uint8, device="cuda"))
+    ws = torch.empty(256, dtype=torch.uint8, device="cuda")
+    abi.sgat_linear(X, None, None, None, 512, K, 0, 0, None, sw, Y, ws, bits=8, We=We)
+    abi.check_status()
