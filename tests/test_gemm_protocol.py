@@ -127,7 +127,7 @@ def test_gemm_barrier_protocol(num_k, krun, tiles):
 def test_model_catches_a_missing_wait(wait):
     """Without the MMA warp's wait for a drained accumulator, or the TMA
     warp's wait for a consumed stage, a schedule that runs the producer
-    ahead trips a check (or a parity wait two phases on)."""
+    ahead trips the matching hazard check."""
     prefer = ("mma", "tma") if wait == "tmem_empty" else ("tma", "mma")
     what = "accumulator overwritten" if wait == "tmem_empty" else "stage refilled"
     with pytest.raises(AssertionError, match=what):
